@@ -1,0 +1,500 @@
+#!/usr/bin/env python
+"""Benchmark of the Comba chunk-parallel training step (forward + backward) on GB300.
+
+Default workload: the 1.3B-scale layer shape, B=4, H=16, T=4096, dk=dv=128,
+chunk 64, bf16 q/k/v/dO with fp32 gates, fp32 initial state h0 and final
+state gradient dhT.  One step = comba_chunk_fwd (o, hT) + comba_chunk_bwd
+(dq, dk, dv, dalpha, dbeta, db, dd, dh0).  Inputs are seeded synthetic data
+(paper_2506_02475_gb300.inputs); L2 is flushed (256 MiB write) between timed
+steps, outside the timed events.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload lm1p3b|lm340m|varlen64k|decode]
+
+Prints one JSON line (rank 0).  Under torchrun each rank runs an independent
+replica of the workload (the op shards over sequences and heads with no
+data-path collective); value = tokens of all ranks / max-over-ranks time.
+``--impl reference`` times the fp64 CPU oracle on bounded samples instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "Comba fwd+bwd tokens/s and TFLOP/s (% BF16 peak) at H=16,d=128,T=4096"
+DECODE_METRIC = "Comba recurrent decode tokens/s at Bd=256,H=16,d=128 (fp32 state)"
+FLUSH_BYTES = 256 << 20
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {k: float(p[k]) for k in FALLBACK_PEAKS}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def fwd_flops_per_token_head(C=64, dk=128, dv=128):
+    """Five C^2 d GEMMs (K K^T, M K, M V, Q~K^T, P E) and three C d^2 (W H, Q~ H, Kbar^T E)."""
+    return 2 * C * (3 * dk + 2 * dv) + 6 * dk * dv
+
+
+# --------------------------------------------------------------- kernel model
+# Algorithmic FLOPs and HBM bytes per launch of each kernel of the step, per
+# (chunk, head) pair (bf16 storage, C = 64): the products the kernel must form
+# and the tensors it must read/write once.
+
+def stage_model(dk, dv, slots, H, N):
+    C, es = 64, 2
+    pairs = slots * H
+    tile = dv // 64
+    m = {}
+    m["prep"] = dict(flops=pairs * 2 * C * C * (2 * dk + dv),
+                     bytes=pairs * (C * (dk + dv) * es + 2 * C * 4 + C * (dk + dv) * es + C * 4))
+    m["scan_fwd"] = dict(flops=pairs * 4 * C * dk * dv,
+                         bytes=pairs * (C * dk * es * 2 + C * dv * es + dk * dv * es + C * dv * es + C * 4 * tile))
+    m["output"] = dict(flops=pairs * (2 * C * C * dk + 2 * C * dk * dv + 2 * C * C * dv),
+                       bytes=pairs * (2 * C * dk * es + dk * dv * es + C * dv * es + C * dv * es + C * 4))
+    m["scan_bwd"] = dict(flops=pairs * (2 * C * C * dk * tile + 2 * C * dk * dv + 2 * C * C * dv + 4 * C * dk * dv),
+                         bytes=pairs * (3 * C * dk * es + C * dv * es + 2 * dk * dv * es // 2 + C * dv * es + C * 4))
+    m["bwd_local"] = dict(flops=pairs * (2 * C * dk * dv * 3 + 2 * C * C * dv * 2 + 2 * C * C * dv
+                                         + 2 * C * C * dk * 3 + 2 * C * C * C * 2 + 2 * C * C * dk * 5),
+                          bytes=pairs * (C * (2 * dk + 2 * dv) * es + 2 * C * dv * es + 2 * dk * dv * es
+                                         + C * C * 4 + 3 * C * 4 + C * (2 * dk + dv) * es + 2 * C * 4))
+    m["chunk_map"] = dict(flops=0, bytes=slots * 16 + (N + 1) * 8)
+    m["reduce"] = dict(flops=0, bytes=pairs * 8 + 8 * H)
+    return m
+
+
+FWD_STAGES = ["chunk_map", "prep", "scan_fwd", "output"]
+BWD_STAGES = ["chunk_map", "prep", "scan_fwd", "scan_bwd", "bwd_local", "reduce"]
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, device_id):
+        self.proc = None
+        self.device_id = device_id
+
+    def start(self):
+        try:
+            cmd = ["nvidia-smi", "--query-gpu=" + ",".join(self.FIELDS), "--format=csv,noheader,nounits",
+                   "-lms", "200"]
+            if self.device_id is not None:
+                cmd += ["-i", str(self.device_id)]
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < len(self.FIELDS):
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def nvsmi_device_id():
+    import torch
+    try:
+        uuid = str(torch.cuda.get_device_properties(torch.cuda.current_device()).uuid)
+        return uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        return vis.split(",")[torch.cuda.current_device()] if vis else torch.cuda.current_device()
+
+
+# ------------------------------------------------------------- distributed
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def dist_init(world, local, backend):
+    import torch
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return dist if world > 1 else None
+
+
+# -------------------------------------------------------- CPU oracle timing
+
+def oracle_sample(w, rows, heads, tokens):
+    """Bounded slice of a dense workload: batch rows `rows`, heads, first `tokens` tokens."""
+    sl = (slice(rows[0], rows[1]), slice(0, tokens), slice(heads[0], heads[1]))
+
+    def st(x):
+        return None if x is None else np.ascontiguousarray(x[rows[0]:rows[1], heads[0]:heads[1]])
+
+    return dict(q=np.ascontiguousarray(w.q[sl]), k=np.ascontiguousarray(w.k[sl]), v=np.ascontiguousarray(w.v[sl]),
+                alpha=np.ascontiguousarray(w.alpha[sl]), beta=np.ascontiguousarray(w.beta[sl]),
+                b=None if w.b is None else w.b[heads[0]:heads[1]], d=w.d[heads[0]:heads[1]], h0=st(w.h0),
+                dO=np.ascontiguousarray(w.dO[sl]), dhT=st(w.dhT))
+
+
+def time_oracle_step(s):
+    import oracle
+    t0 = time.perf_counter()
+    oracle.fwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], h0=s["h0"])
+    oracle.bwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], s["dO"], h0=s["h0"], dhT=s["dhT"])
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(w, target_s=12.0):
+    """The oracle as it stands on this host's cores: fwd+bwd over batch row 0, all heads,
+    growing the token prefix until about `target_s` seconds of wall time."""
+    import oracle
+    H = w.q.shape[2]
+    T = w.q.shape[1]
+    tokens = min(T, 256)
+    while True:
+        s = oracle_sample(w, (0, 1), (0, H), tokens)
+        dt = time_oracle_step(s)
+        if dt >= target_s or tokens >= T:
+            break
+        tokens = min(T, int(tokens * max(2.0, min(8.0, target_s / max(dt, 1e-3)))) // 64 * 64 or 64)
+    return {"value": tokens / dt, "unit": "tokens/s", "cores": oracle.default_threads(), "kind": "oracle",
+            "sample": f"fwd+bwd, batch row 0, all {H} heads, first {tokens} of {T} tokens (fp64 token recurrence,"
+                      f" exact BPTT); {dt:.2f} s"}
+
+
+# --------------------------------------------------------------- our path
+
+def run_ours(args, world, rank, local):
+    import torch
+    dist = dist_init(world, local, "nccl")
+    torch.cuda.set_device(local)
+    from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, inputs
+    from paper_2506_02475_gb300 import binding
+
+    peaks, peak_src = load_peaks()
+    w = inputs.make(args.workload)
+    dev = torch.device("cuda", local)
+    tdt = torch.bfloat16
+
+    def host(x, dt):
+        return None if x is None else torch.from_numpy(np.ascontiguousarray(x)).to(dt).pin_memory()
+
+    hin = dict(q=host(w.q, tdt), k=host(w.k, tdt), v=host(w.v, tdt), alpha=host(w.alpha, torch.float32),
+               beta=host(w.beta, torch.float32), d=host(w.d, torch.float32), b=host(w.b, torch.float32),
+               h0=host(w.h0, torch.float32), dO=host(w.dO, tdt), dhT=host(w.dhT, torch.float32))
+    cu = None if w.cu_seqlens is None else torch.from_numpy(w.cu_seqlens.astype(np.int32)).to(dev)
+    din = {k: (None if v is None else v.to(dev)) for k, v in hin.items()}
+    q = din["q"]
+    ws_bytes = binding.comba_workspace_size(q, din["v"], cu, backward=True)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    N = w.num_seqs
+    H, dk, dv = w.H, w.dk, w.dv
+    o = torch.empty_like(din["v"])
+    hT = torch.empty((N, H, dk, dv), dtype=torch.float32, device=dev)
+    grads = {"dq": torch.empty_like(q), "dk": torch.empty_like(din["k"]), "dv": torch.empty_like(din["v"]),
+             "dalpha": torch.empty_like(din["alpha"]), "dbeta": torch.empty_like(din["beta"]),
+             "dd": torch.empty_like(din["d"]), "db": torch.empty((H,), dtype=torch.float32, device=dev),
+             "dh0": torch.empty((N, H, dk, dv), dtype=torch.float32, device=dev)}
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    ev_f = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+    for e in ev_f + ev_b:
+        e.record()
+    torch.cuda.synchronize()
+    hf = [e.cuda_event for e in ev_f]
+    hb = [e.cuda_event for e in ev_b]
+
+    def step(t, events=True):
+        comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"], cu_seqlens=cu,
+                        o=o, hT=hT, workspace=ws, stage_events=hf if events else None)
+        comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
+                        dhT=t["dhT"], cu_seqlens=cu, out=grads, workspace=ws, stage_events=hb if events else None)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step(din)
+    torch.cuda.synchronize()
+
+    # ---- timed region: device-resident inputs
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    stage_ms = {("fwd", s): 0.0 for s in FWD_STAGES}
+    stage_ms.update({("bwd", s): 0.0 for s in BWD_STAGES})
+    clocks = ClockSampler(nvsmi_device_id())
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    total_ms = 0.0
+    t_wall = time.perf_counter()
+    for _ in range(args.steps):
+        flush.zero_()
+        start.record()
+        step(din)
+        end.record()
+        end.synchronize()
+        total_ms += start.elapsed_time(end)
+        for i, s in enumerate(FWD_STAGES):
+            stage_ms[("fwd", s)] += ev_f[i].elapsed_time(ev_f[i + 1])
+        for i, s in enumerate(BWD_STAGES):
+            stage_ms[("bwd", s)] += ev_b[i].elapsed_time(ev_b[i + 1])
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t_wall
+    clk = clocks.stop()
+    if dist:
+        dist.barrier()
+    ms = total_ms / args.steps
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    tokens = w.tokens
+    value = tokens * world / (ms / 1e3)
+    flops_step = 3.5 * fwd_flops_per_token_head(64, dk, dv) * tokens * H
+    tflops = flops_step * world / (ms / 1e3) / 1e12
+
+    # ---- dominant kernel and its roofline
+    slots = (tokens // 64 + N) if w.cu_seqlens is not None else w.q.shape[0] * ((w.q.shape[1] + 63) // 64)
+    model = stage_model(dk, dv, slots, H, N)
+    per_kind = {}
+    for (phase, s), v in stage_ms.items():
+        per_kind.setdefault(s, [0.0, 0])
+        per_kind[s][0] += v
+        per_kind[s][1] += args.steps
+    dom = max(per_kind, key=lambda s: per_kind[s][0])
+    launch_ms = per_kind[dom][0] / per_kind[dom][1]
+    mdl = model[dom]
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    ai = mdl["flops"] / max(mdl["bytes"], 1)
+    if ai >= ridge:
+        ach = mdl["flops"] / (launch_ms / 1e3) / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
+    else:
+        ach = mdl["bytes"] / (launch_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof.update({"kernel": dom, "launch_ms": launch_ms, "algorithmic_flops": mdl["flops"],
+                 "algorithmic_bytes": mdl["bytes"], "traffic": None, "peak_source": peak_src + " (burst)"})
+
+    # ---- end to end through the public API with host buffers
+    hout = {"o": torch.empty(o.shape, dtype=o.dtype).pin_memory(),
+            "hT": torch.empty(hT.shape, dtype=hT.dtype).pin_memory()}
+    for k_, v_ in grads.items():
+        hout[k_] = torch.empty(v_.shape, dtype=v_.dtype).pin_memory()
+    dbuf = {k: (None if v is None else torch.empty_like(v)) for k, v in din.items()}
+    bi = sum(v.numel() * v.element_size() for v in hin.values() if v is not None)
+    bo = sum(v.numel() * v.element_size() for v in hout.values())
+    dev_out = {"o": o, "hT": hT, **grads}
+
+    def e2e_step():
+        for k_, v_ in hin.items():
+            if v_ is not None:
+                dbuf[k_].copy_(v_, non_blocking=True)
+        step(dbuf, events=False)
+        for k_, v_ in dev_out.items():
+            hout[k_].copy_(v_, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    e_ms = 0.0
+    for _ in range(args.steps):
+        flush.zero_()
+        start.record()
+        e2e_step()
+        end.record()
+        end.synchronize()
+        e_ms += start.elapsed_time(end)
+    e_ms /= args.steps
+    if dist:
+        t = torch.tensor([e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e_ms = float(t.item())
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; paper's layer shape and gate ranges)",
+            "config": {"workload": f"{args.workload}: " + workload_desc(w), "global_batch": w.num_seqs * world,
+                       "seq_len": int(w.q.shape[1]) if w.cu_seqlens is None else int(w.tokens),
+                       "parallelism": f"replicas x{world} (no data-path collective)",
+                       "l2": "flushed between timed steps (256 MiB write, outside the events)"},
+            "tflops": tflops, "pct_bf16_peak": tflops / peaks["bf16_tflops"] * 100,
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": {"value": tokens * world / (e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": bi,
+                    "d2h_bytes_per_step": bo, "ms_per_step": e_ms},
+            "clocks": clk,
+            "gpu_launches": 10 * args.steps,
+            "stages_ms_per_step": {f"{p}.{s}": v / args.steps for (p, s), v in stage_ms.items()},
+            "wall_s_timed": wall,
+        }
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def workload_desc(w):
+    if w.cu_seqlens is not None:
+        lens = np.diff(w.cu_seqlens).tolist()
+        shape = f"packed {len(lens)} seqs (lengths {lens}), {w.tokens} tokens"
+    else:
+        shape = f"B={w.q.shape[0]} T={w.q.shape[1]}"
+    return (f"{shape} H={w.H} dk={w.dk} dv={w.dv} chunk=64; {w.dtype} q/k/v/dO, fp32 gates/state; "
+            f"h0={'yes' if w.h0 is not None else 'no'}, dhT=yes; step = chunk_fwd(o,hT) + chunk_bwd(all grads)")
+
+
+# ------------------------------------------------------------------ decode
+
+def run_decode(args, world, rank, local):
+    import torch
+    dist = dist_init(world, local, "nccl")
+    torch.cuda.set_device(local)
+    from paper_2506_02475_gb300 import comba_recurrent_step, inputs
+    peaks, peak_src = load_peaks()
+    Bd, H, dk, dv = 256, 16, 128, 128
+    dev = torch.device("cuda", local)
+    state = torch.from_numpy(inputs.decode_state(Bd, H, dk, dv)).to(dev)
+    toks = []
+    for s in range(8):  # cycle over 8 distinct token sets
+        q, k, v, a, be, d = inputs.decode_tokens(s, Bd, H, dk, dv, "bf16")
+        toks.append([torch.from_numpy(x).to(dev).to(torch.bfloat16) for x in (q, k, v)] +
+                    [torch.from_numpy(x).to(dev) for x in (a, be)])
+    d = torch.from_numpy(d).to(dev)
+    o = torch.empty((Bd, H, dv), dtype=torch.bfloat16, device=dev)
+    steps = 1024
+    for i in range(args.warmup):
+        t = toks[i % 8]
+        comba_recurrent_step(t[0], t[1], t[2], t[3], t[4], d, state, o=o)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(nvsmi_device_id())
+    torch.cuda.synchronize()
+    clocks.start()
+    total = 0.0
+    for _ in range(args.steps):
+        start.record()
+        for i in range(steps):
+            t = toks[i % 8]
+            comba_recurrent_step(t[0], t[1], t[2], t[3], t[4], d, state, o=o)
+        end.record()
+        end.synchronize()
+        total += start.elapsed_time(end)
+    clk = clocks.stop()
+    ms = total / args.steps
+    per = ms / steps
+    bytes_step = Bd * H * (2 * dk * dv * 4 + (2 * dk + 2 * dv) * 2 + 8)
+    gbs = bytes_step / (per / 1e3) / 1e9
+    if rank == 0:
+        print(json.dumps({
+            "metric": DECODE_METRIC, "value": Bd * steps * world / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "fp32-state/bf16-tokens", "data": "synthetic",
+            "config": {"workload": f"decode: Bd={Bd} H={H} dk={dk} dv={dv}, {steps} sequential steps per timed step",
+                       "l2": "state (268 MB) larger than L2"},
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": gbs / peaks["hbm_gbs"], "kernel": "k_step", "launch_ms": per, "traffic": None,
+                         "peak_source": peak_src},
+            "clocks": clk, "gpu_launches": steps * args.steps}), flush=True)
+
+
+# --------------------------------------------------------------- reference
+
+def run_reference(args, world, rank, local):
+    """The fp64 CPU oracle as it stands, on bounded samples of the same workload."""
+    if rank != 0:
+        return
+    import oracle
+    from paper_2506_02475_gb300 import inputs
+    w = inputs.make(args.workload)
+    H = w.H
+    tokens = min(int(w.q.shape[1]), args.reference_tokens)
+    s = oracle_sample(w, (0, 1), (0, H), tokens)
+    for _ in range(args.warmup):
+        time_oracle_step(s)
+    dts = [time_oracle_step(s) for _ in range(args.steps)]
+    dt = sum(dts) / len(dts)
+    value = tokens / dt
+    flops = 3.5 * fwd_flops_per_token_head(64, w.dk, w.dv) * tokens * H
+    print(json.dumps({
+        "metric": METRIC, "impl": "reference", "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{args.workload}: " + workload_desc(w),
+                   "sample": f"batch row 0, all {H} heads, first {tokens} tokens per step"},
+        "tflops": flops / dt / 1e12,
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.default_threads(), "kind": "oracle",
+                         "sample": f"fwd+bwd, batch row 0, all {H} heads, first {tokens} tokens"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="lm1p3b", choices=["lm1p3b", "lm340m", "varlen64k", "decode"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--reference-tokens", type=int, default=512)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        return run_reference(args, world, rank, local)
+    if args.workload == "decode":
+        return run_decode(args, world, rank, local)
+    return run_ours(args, world, rank, local)
+
+
+if __name__ == "__main__":
+    main()

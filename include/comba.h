@@ -1,0 +1,167 @@
+/*
+ * comba.h -- C ABI of the GB300 (sm_103a) Comba chunk-parallel library.
+ *
+ * Comba ("Improving Bilinear RNNs with Closed-loop Control", arXiv 2506.02475)
+ * is a bilinear RNN whose state S_t (dv x dk) follows, per sequence and head,
+ *
+ *     S_t = S_{t-1} (alpha_t I - btilde_t k_t k_t^T) + beta_t v_t k_t^T      (section 3, Eq. comba-S)
+ *     o_t = S_t (q_t - d k_t)                                                (output correction, same Eq.)
+ *     btilde_t = b * beta_t                                                  (section 3.1)
+ *
+ * This library stores the state transposed, H = S^T (dk x dv, row-major), as
+ * the paper's recurrent listing does (appendix B.1).  Equivalently
+ *     e_t = beta_t v_t - btilde_t H_{t-1}^T k_t,  H_t = alpha_t H_{t-1} + k_t e_t^T,
+ *     o_t = H_t^T (q_t - d k_t).
+ * There is no query scale.  Training uses the chunk-wise form of section 3.3
+ * (WY representation with a single UT inverse per chunk, Eq. "prepare WY_M",
+ * then the inter-chunk state and output equations); inference uses the
+ * one-token recurrence.
+ *
+ * Conventions shared by every entry point
+ *   - Every tensor argument is a DEVICE pointer owned by the caller.  The
+ *     library allocates and frees nothing; scratch comes from the caller's
+ *     workspace (size from comba_workspace_size).
+ *   - Token tensors are row-major [B, T, H, D] (D contiguous).  For packed
+ *     variable-length input pass B = 1, T = total tokens, num_seqs = N and
+ *     cu_seqlens = device int32 [N+1] offsets (cu[0] = 0, non-decreasing,
+ *     cu[N] = T); the state restarts at every sequence start and chunks never
+ *     straddle a boundary.  With cu_seqlens == NULL, num_seqs must equal B.
+ *   - q, k, v, o, dO, dq, dk, dv use the storage type `dtype` (fp32 or bf16).
+ *     Gates alpha, beta and their gradients are fp32 [B, T, H]; the per-head
+ *     scalars b, d and their gradients are fp32 [H].  States h0, hT, dhT, dh0
+ *     are fp32 [num_seqs, H, dk, dv].  All arithmetic accumulates in fp32.
+ *   - alpha must lie in (0, 1]: the chunk form takes logarithms of alpha.
+ *   - All pointers must be 16-byte aligned.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream).  Outputs are overwritten, never accumulated into.
+ *   - Validation is host-side only; invalid arguments return an error before
+ *     anything is launched.  A failed launch returns COMBA_ERR_CUDA.
+ *   - No global mutable state: calls on different streams may overlap as long
+ *     as their workspaces and outputs are distinct.
+ *   - Results are bitwise reproducible from run to run (fixed reduction order,
+ *     no floating-point atomics).
+ */
+#ifndef COMBA_H
+#define COMBA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    COMBA_OK = 0,
+    COMBA_ERR_INVALID_ARG = 1,  /* NULL required pointer, bad shape, misalignment   */
+    COMBA_ERR_UNSUPPORTED = 2,  /* valid but not implemented (head dim, chunk size) */
+    COMBA_ERR_WORKSPACE = 3,    /* workspace NULL or smaller than required         */
+    COMBA_ERR_CUDA = 4,         /* a CUDA launch or query failed                    */
+    COMBA_ERR_TIMEOUT = 5       /* reserved: a bounded device-side wait gave up     */
+} comba_status_t;
+
+typedef enum { COMBA_F32 = 0, COMBA_BF16 = 1 } comba_dtype_t;
+
+typedef struct {
+    int B;                      /* batch; 1 when cu_seqlens != NULL               */
+    int T;                      /* tokens per sequence, or total packed tokens    */
+    int H;                      /* heads                                          */
+    int dk;                     /* key/query head dim: 64 or 128                  */
+    int dv;                     /* value head dim: 64 or 128                      */
+    int num_seqs;               /* N: == B when cu_seqlens == NULL                */
+    const int32_t *cu_seqlens;  /* device int32 [N+1] or NULL                     */
+    comba_dtype_t dtype;        /* storage type of q, k, v, o and their grads     */
+    int chunk;                  /* chunk length; must be 64                       */
+    /* Optional instrumentation (NULL / 0 = off).  Caller-created cudaEvent_t
+     * handles recorded on `stream` at kernel boundaries: comba_chunk_fwd
+     * records COMBA_FWD_EVENTS of them (before chunk map, prep, state scan,
+     * output, and after output); comba_chunk_bwd records COMBA_BWD_EVENTS
+     * (before chunk map, prep, forward state scan, reverse state scan, local
+     * gradients, head reduction, and after it).  Fewer handles than needed
+     * is COMBA_ERR_INVALID_ARG. */
+    void **stage_events;
+    int num_stage_events;
+} comba_shape_t;
+
+#define COMBA_FWD_EVENTS 5
+#define COMBA_BWD_EVENTS 7
+
+/*
+ * Bytes of device workspace needed by comba_chunk_fwd (backward = 0) or
+ * comba_chunk_bwd (backward = 1) for this shape.  Returns 0 for an invalid
+ * shape.  The bound covers any cu_seqlens with the given T and num_seqs.
+ */
+size_t comba_workspace_size(const comba_shape_t *shape, int backward);
+
+/*
+ * Chunk-parallel forward (section 3.3).  Per chunk of 64 tokens: the
+ * decay-masked, btilde-scaled Gram matrix, its unit-lower-triangular inverse
+ * M = (I + strict_lower(Diag(btilde)(A^{(i-1)/j} * K K^T)))^{-1}, the WY/UT
+ * factors W = M Diag(btilde*gamma_{r-1}) K and U = M Diag(beta) V
+ * (Eq. "prepare WY_M"); then a sequential scan of the chunk states
+ * H_{n+1} = gamma_C H_n + Kbar^T (U - W H_n); then the chunk outputs
+ * O = Diag(gamma) Q~ H_n + Tril(Q~ K^T * A^{i/j}) (U - W H_n), Q~ = Q - d K.
+ *
+ *   q, k [B,T,H,dk]; v [B,T,H,dv]; alpha, beta fp32 [B,T,H];
+ *   b fp32 [H] or NULL (b = 1); d fp32 [H];
+ *   h0 fp32 [N,H,dk,dv] or NULL (zero state);
+ *   o [B,T,H,dv] (written); hT fp32 [N,H,dk,dv] or NULL (final state, written).
+ */
+comba_status_t comba_chunk_fwd(const comba_shape_t *shape,
+                               const void *q, const void *k, const void *v,
+                               const float *alpha, const float *beta,
+                               const float *b, const float *d, const float *h0,
+                               void *o, float *hT,
+                               void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * Chunk-parallel backward: exact gradients of
+ *     L = <o, dO> + <hT, dhT>
+ * through the forward above (the paper prints no backward; these are the
+ * chain-rule derivatives of the chunk form).  The forward chunk factors and
+ * chunk states are recomputed inside the call.
+ *
+ *   inputs as comba_chunk_fwd, plus dO [B,T,H,dv] and dhT fp32 [N,H,dk,dv] or
+ *   NULL (zero);
+ *   dq, dk [B,T,H,dk], dv [B,T,H,dv] (storage type), dalpha, dbeta fp32
+ *   [B,T,H], dd fp32 [H] (all written); db fp32 [H] or NULL (written when
+ *   non-NULL; the gradient w.r.t. b, also when b == NULL meant b = 1);
+ *   dh0 fp32 [N,H,dk,dv] or NULL (written when non-NULL).
+ *   dalpha is d L / d alpha (not d L / d log alpha).
+ *
+ * The fp32 storage type supports dk, dv <= 64 in the backward.
+ */
+comba_status_t comba_chunk_bwd(const comba_shape_t *shape,
+                               const void *q, const void *k, const void *v,
+                               const float *alpha, const float *beta,
+                               const float *b, const float *d, const float *h0,
+                               const void *dO, const float *dhT,
+                               void *dq, void *dk, void *dv,
+                               float *dalpha, float *dbeta, float *db, float *dd, float *dh0,
+                               void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * One decode token (appendix B.1, recurrent form) for Bd independent rows:
+ *     x = H^T k, y = H^T (q - d k), e = beta v - b beta x,
+ *     o = alpha y + e (k . (q - d k)),   H <- alpha H + k e^T
+ * (o equals the new state applied to q - d k).  The state is read once and
+ * written once, in place.
+ *
+ *   q, k [Bd,H,dk], v [Bd,H,dv], o [Bd,H,dv] (storage type `dtype`);
+ *   alpha, beta fp32 [Bd,H]; b fp32 [H] or NULL; d fp32 [H];
+ *   state fp32 [Bd,H,dk,dv], updated in place.
+ */
+comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t dtype,
+                                    const void *q, const void *k, const void *v,
+                                    const float *alpha, const float *beta,
+                                    const float *b, const float *d,
+                                    float *state, void *o, void *stream);
+
+/* Static, human-readable name of a status code. */
+const char *comba_status_string(comba_status_t status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* COMBA_H */

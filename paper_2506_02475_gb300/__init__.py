@@ -1,0 +1,16 @@
+"""GB300-native (sm_103a) Comba chunk-parallel library.
+
+Comba (arXiv 2506.02475) is a bilinear RNN with a scalar-plus-low-rank state
+transition, state feedback and output feedback.  This package is the hot path
+of its training and inference: ``libcomba.so`` (C ABI in ``include/comba.h``,
+CUDA kernels under ``csrc/``) and a thin ctypes binding with the same names.
+"""
+from .binding import (  # noqa: F401
+    CombaError,
+    comba_chunk_bwd,
+    comba_chunk_fwd,
+    comba_recurrent_step,
+    comba_workspace_size,
+    lib,
+    library_path,
+)

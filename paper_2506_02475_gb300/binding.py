@@ -1,0 +1,239 @@
+"""Thin ctypes binding of ``libcomba.so`` (the C ABI in ``include/comba.h``).
+
+Argument marshalling only: tensors are checked, outputs and the workspace are
+allocated with torch (device memory plumbing), raw device pointers and the
+current CUDA stream are passed to the C entry points, and a non-OK status is
+raised as an exception.  Every arithmetic step runs inside the library's
+CUDA kernels; there is no fallback path.  If the compiled library is missing
+the import of any entry point fails loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+_lib = None
+_lock = threading.Lock()
+
+COMBA_F32, COMBA_BF16 = 0, 1
+_STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "workspace missing or too small",
+           4: "CUDA error", 5: "device-side wait timed out"}
+
+
+class CombaError(RuntimeError):
+    def __init__(self, fn, status):
+        super().__init__(f"{fn} failed: {_STATUS.get(status, status)} (status {status})")
+        self.status = status
+
+
+class _Shape(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int), ("dk", ctypes.c_int),
+                ("dv", ctypes.c_int), ("num_seqs", ctypes.c_int), ("cu_seqlens", ctypes.c_void_p),
+                ("dtype", ctypes.c_int), ("chunk", ctypes.c_int), ("stage_events", ctypes.c_void_p),
+                ("num_stage_events", ctypes.c_int)]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """Load libcomba.so (building it first if this checkout has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if not os.path.exists(path) or not _build.up_to_date():
+            _build.build()
+        L = ctypes.CDLL(path)
+        P, I, Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+        SP = ctypes.POINTER(_Shape)
+        L.comba_workspace_size.argtypes = [SP, I]
+        L.comba_workspace_size.restype = Z
+        L.comba_chunk_fwd.argtypes = [SP] + [P] * 10 + [P, Z, P]
+        L.comba_chunk_fwd.restype = I
+        L.comba_chunk_bwd.argtypes = [SP] + [P] * 10 + [P] * 8 + [P, Z, P]
+        L.comba_chunk_bwd.restype = I
+        L.comba_recurrent_step.argtypes = [I, I, I, I, I] + [P] * 9 + [P]
+        L.comba_recurrent_step.restype = I
+        L.comba_status_string.argtypes = [I]
+        L.comba_status_string.restype = ctypes.c_char_p
+        _lib = L
+        return L
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype_code(t):
+    if t.dtype == torch.bfloat16:
+        return COMBA_BF16
+    if t.dtype == torch.float32:
+        return COMBA_F32
+    raise TypeError(f"q/k/v must be float32 or bfloat16, got {t.dtype}")
+
+
+def _check(name, t, dtype=None, shape=None, device=None):
+    if t is None:
+        return
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+
+
+def make_shape(q, v, cu_seqlens=None, stage_events=None):
+    """Build the C shape struct from q [B,T,H,dk] (or packed [Ttot,H,dk]) and v.
+
+    ``stage_events`` (optional): sequence of raw cudaEvent_t handles (ints) recorded at
+    kernel boundaries (instrumentation; see include/comba.h)."""
+    if q.dim() == 3:
+        q = q.unsqueeze(0)
+        v = v.unsqueeze(0)
+    B, T, H, dk = q.shape
+    dv = v.shape[-1]
+    s = _Shape()
+    s.B, s.T, s.H, s.dk, s.dv = B, T, H, dk, dv
+    if cu_seqlens is not None:
+        s.num_seqs = cu_seqlens.numel() - 1
+        s.cu_seqlens = cu_seqlens.data_ptr()
+    else:
+        s.num_seqs = B
+        s.cu_seqlens = None
+    s.dtype = _dtype_code(q)
+    s.chunk = 64
+    if stage_events is not None:
+        arr = (ctypes.c_void_p * len(stage_events))(*stage_events)
+        s._events_keepalive = arr
+        s.stage_events = ctypes.cast(arr, ctypes.c_void_p)
+        s.num_stage_events = len(stage_events)
+    return s
+
+
+def comba_workspace_size(q, v, cu_seqlens=None, backward=False) -> int:
+    return int(lib().comba_workspace_size(ctypes.byref(make_shape(q, v, cu_seqlens)), int(bool(backward))))
+
+
+def _workspace(nbytes, device, workspace):
+    if workspace is not None:
+        if workspace.numel() * workspace.element_size() < nbytes:
+            raise ValueError(f"workspace has {workspace.numel() * workspace.element_size()} bytes, need {nbytes}")
+        return workspace
+    return torch.empty(max(nbytes, 16), dtype=torch.uint8, device=device)
+
+
+def _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens):
+    dev = q.device
+    packed = q.dim() == 3
+    lead = tuple(q.shape[:-1])
+    H, dk, dv = q.shape[-2], q.shape[-1], v.shape[-1]
+    _check("q", q, device=dev)
+    _check("k", k, dtype=q.dtype, shape=q.shape, device=dev)
+    _check("v", v, dtype=q.dtype, shape=lead + (dv,), device=dev)
+    _check("alpha", alpha, torch.float32, lead, dev)
+    _check("beta", beta, torch.float32, lead, dev)
+    _check("b", b, torch.float32, (H,), dev)
+    _check("d", d, torch.float32, (H,), dev)
+    if cu_seqlens is not None:
+        _check("cu_seqlens", cu_seqlens, torch.int32, None, dev)
+        N = cu_seqlens.numel() - 1
+        if not packed and q.shape[0] != 1:
+            raise ValueError("cu_seqlens requires B == 1 (or packed [Ttot,H,D] inputs)")
+    else:
+        N = 1 if packed else q.shape[0]
+    _check("h0", h0, torch.float32, (N, H, dk, dv), dev)
+    return N, H, dk, dv
+
+
+def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, output_final_state=False,
+                    o=None, hT=None, workspace=None, stream=None, stage_events=None):
+    """Chunk-parallel forward.  Returns ``(o, hT)`` (``hT`` is None unless requested)."""
+    N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
+    shape = make_shape(q, v, cu_seqlens, stage_events)
+    L = lib()
+    nbytes = L.comba_workspace_size(ctypes.byref(shape), 0)
+    if nbytes == 0:
+        raise CombaError("comba_workspace_size", 1)
+    ws = _workspace(nbytes, q.device, workspace)
+    if o is None:
+        o = torch.empty_like(v)
+    if hT is None and output_final_state:
+        hT = torch.empty((N, H, dk, dv), dtype=torch.float32, device=q.device)
+    st = L.comba_chunk_fwd(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b),
+                           _ptr(d), _ptr(h0), _ptr(o), _ptr(hT), _ptr(ws), ws.numel() * ws.element_size(),
+                           _stream(stream))
+    if st != 0:
+        raise CombaError("comba_chunk_fwd", st)
+    return o, hT
+
+
+def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_seqlens=None, want_dh0=True,
+                    want_db=True, out=None, workspace=None, stream=None, stage_events=None):
+    """Chunk-parallel backward.  Returns a dict with dq, dk, dv, dalpha, dbeta, dd, db, dh0."""
+    N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
+    _check("dO", dO, q.dtype, v.shape, q.device)
+    _check("dhT", dhT, torch.float32, (N, H, dk, dv), q.device)
+    shape = make_shape(q, v, cu_seqlens, stage_events)
+    L = lib()
+    nbytes = L.comba_workspace_size(ctypes.byref(shape), 1)
+    if nbytes == 0:
+        raise CombaError("comba_workspace_size", 1)
+    ws = _workspace(nbytes, q.device, workspace)
+    g = out if out is not None else {}
+    g.setdefault("dq", torch.empty_like(q))
+    g.setdefault("dk", torch.empty_like(k))
+    g.setdefault("dv", torch.empty_like(v))
+    g.setdefault("dalpha", torch.empty_like(alpha))
+    g.setdefault("dbeta", torch.empty_like(beta))
+    g.setdefault("dd", torch.empty_like(d))
+    if want_db:
+        g.setdefault("db", torch.empty((H,), dtype=torch.float32, device=q.device))
+    if want_dh0:
+        g.setdefault("dh0", torch.empty((N, H, dk, dv), dtype=torch.float32, device=q.device))
+    st = L.comba_chunk_bwd(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b),
+                           _ptr(d), _ptr(h0), _ptr(dO), _ptr(dhT), _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]),
+                           _ptr(g["dalpha"]), _ptr(g["dbeta"]), _ptr(g.get("db")), _ptr(g["dd"]),
+                           _ptr(g.get("dh0")), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream))
+    if st != 0:
+        raise CombaError("comba_chunk_bwd", st)
+    return g
+
+
+def comba_recurrent_step(q, k, v, alpha, beta, d, state, b=None, o=None, stream=None):
+    """One decode token; ``state`` [Bd,H,dk,dv] fp32 is updated in place.  Returns ``o``."""
+    Bd, H, dk = q.shape
+    dv = v.shape[-1]
+    dev = q.device
+    _check("q", q, device=dev)
+    _check("k", k, q.dtype, q.shape, dev)
+    _check("v", v, q.dtype, (Bd, H, dv), dev)
+    _check("alpha", alpha, torch.float32, (Bd, H), dev)
+    _check("beta", beta, torch.float32, (Bd, H), dev)
+    _check("b", b, torch.float32, (H,), dev)
+    _check("d", d, torch.float32, (H,), dev)
+    _check("state", state, torch.float32, (Bd, H, dk, dv), dev)
+    if o is None:
+        o = torch.empty_like(v)
+    st = lib().comba_recurrent_step(Bd, H, dk, dv, _dtype_code(q), _ptr(q), _ptr(k), _ptr(v), _ptr(alpha),
+                                    _ptr(beta), _ptr(b), _ptr(d), _ptr(state), _ptr(o), _stream(stream))
+    if st != 0:
+        raise CombaError("comba_recurrent_step", st)
+    return o

@@ -1,0 +1,208 @@
+// C ABI of the Comba library: argument validation, workspace carve-up and
+// kernel sequencing.  Declarations and the contract live in include/comba.h.
+#include <cuda_runtime.h>
+
+#include "../../include/comba.h"
+#include "params.cuh"
+
+using comba::ChunkParams;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct Layout {
+    size_t slot_info, seq_first, W, U, G, M, Hs, E, dH, dE, part, total;
+    int slots;
+};
+
+// Validates the shape (not the pointers) and computes the workspace layout.
+comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
+    if (!s) return COMBA_ERR_INVALID_ARG;
+    if (s->B < 1 || s->T < 0 || s->H < 1 || s->num_seqs < 1) return COMBA_ERR_INVALID_ARG;
+    if (s->dtype != COMBA_F32 && s->dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
+    if (s->chunk != comba::kChunk) return COMBA_ERR_UNSUPPORTED;
+    if ((s->dk != 64 && s->dk != 128) || (s->dv != 64 && s->dv != 128)) return COMBA_ERR_UNSUPPORTED;
+    if (s->H > 65535) return COMBA_ERR_UNSUPPORTED;
+    if (s->cu_seqlens) {
+        if (s->B != 1) return COMBA_ERR_INVALID_ARG;
+        if (!aligned16(s->cu_seqlens)) return COMBA_ERR_INVALID_ARG;
+    } else if (s->num_seqs != s->B) {
+        return COMBA_ERR_INVALID_ARG;
+    }
+    const long long ttot = (long long)s->B * s->T;
+    if (ttot >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
+    if (backward && s->dtype == COMBA_F32 && (s->dk != 64 || s->dv != 64)) return COMBA_ERR_UNSUPPORTED;
+    const long long slots = s->cu_seqlens ? ttot / comba::kChunk + s->num_seqs
+                                          : (long long)s->B * ((s->T + comba::kChunk - 1) / comba::kChunk);
+    if (slots >= (1LL << 31) / 2) return COMBA_ERR_UNSUPPORTED;
+    const size_t es = s->dtype == COMBA_BF16 ? 2 : 4;
+    const size_t pairs = (size_t)slots * s->H;
+    Layout L{};
+    size_t o = 0;
+    auto take = [&](size_t bytes) { size_t at = o; o = align_up(o + bytes); return at; };
+    L.slot_info = take(sizeof(comba::SlotInfo) * (size_t)slots);
+    L.seq_first = take(sizeof(int) * (size_t)(s->num_seqs + 1));
+    L.W = take(pairs * 64 * s->dk * es);
+    L.U = take(pairs * 64 * s->dv * es);
+    L.G = take(pairs * 64 * sizeof(float));
+    L.Hs = take(pairs * (size_t)s->dk * s->dv * es);
+    L.E = take(pairs * 64 * s->dv * es);
+    if (backward) {
+        L.M = take(pairs * 64 * 64 * sizeof(float));
+        L.dH = take(pairs * (size_t)s->dk * s->dv * es);
+        L.dE = take(pairs * 64 * s->dv * es);
+        L.part = take(pairs * 2 * sizeof(float));
+    }
+    L.total = o;
+    L.slots = (int)slots;
+    *out = L;
+    return COMBA_OK;
+}
+
+comba_status_t check_smem(const comba_shape_t* s, int backward) {
+    int dev = 0, optin = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+        return COMBA_ERR_CUDA;
+    const bool bf = s->dtype == COMBA_BF16;
+    for (int kern = 0; kern < 3; ++kern)
+        if (comba::fwd_smem_bytes(kern, bf, s->dk, s->dv) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
+    if (backward)
+        for (int kern = 0; kern < 2; ++kern)
+            if (comba::bwd_smem_bytes(kern, bf, s->dk, s->dv) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
+    return COMBA_OK;
+}
+
+void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* ws) {
+    char* w = static_cast<char*>(ws);
+    p.B = s->B; p.T = s->T; p.H = s->H; p.dk = s->dk; p.dv = s->dv; p.N = s->num_seqs;
+    p.Ttot = (long long)s->B * s->T;
+    p.cu = s->cu_seqlens;
+    p.slots = L.slots;
+    p.ev = reinterpret_cast<cudaEvent_t*>(s->stage_events);
+    p.nev = s->stage_events ? s->num_stage_events : 0;
+    p.slot_info = reinterpret_cast<comba::SlotInfo*>(w + L.slot_info);
+    p.seq_first = reinterpret_cast<int*>(w + L.seq_first);
+    p.Wb = w + L.W;
+    p.Ub = w + L.U;
+    p.Gb = reinterpret_cast<float*>(w + L.G);
+    p.Hb = w + L.Hs;
+    p.Eb = w + L.E;
+}
+
+#define COMBA_REQUIRE(ptr)                                   \
+    do {                                                     \
+        if (!(ptr) || !aligned16(ptr)) return COMBA_ERR_INVALID_ARG; \
+    } while (0)
+#define COMBA_OPTIONAL(ptr)                                  \
+    do {                                                     \
+        if ((ptr) && !aligned16(ptr)) return COMBA_ERR_INVALID_ARG; \
+    } while (0)
+
+}  // namespace
+
+extern "C" {
+
+const char* comba_status_string(comba_status_t status) {
+    switch (status) {
+        case COMBA_OK: return "ok";
+        case COMBA_ERR_INVALID_ARG: return "invalid argument";
+        case COMBA_ERR_UNSUPPORTED: return "unsupported configuration";
+        case COMBA_ERR_WORKSPACE: return "workspace missing or too small";
+        case COMBA_ERR_CUDA: return "CUDA error";
+        case COMBA_ERR_TIMEOUT: return "device-side wait timed out";
+    }
+    return "unknown status";
+}
+
+size_t comba_workspace_size(const comba_shape_t* shape, int backward) {
+    Layout L;
+    if (plan(shape, backward, &L) != COMBA_OK) return 0;
+    return L.total;
+}
+
+comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const void* k, const void* v,
+                               const float* alpha, const float* beta, const float* b, const float* d,
+                               const float* h0, void* o, float* hT, void* workspace, size_t workspace_bytes,
+                               void* stream) {
+    Layout L;
+    comba_status_t st = plan(shape, 0, &L);
+    if (st != COMBA_OK) return st;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
+    COMBA_REQUIRE(d); COMBA_REQUIRE(o);
+    COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
+    if (shape->stage_events && shape->num_stage_events < COMBA_FWD_EVENTS) return COMBA_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
+    if ((st = check_smem(shape, 0)) != COMBA_OK) return st;
+
+    ChunkParams p{};
+    fill_common(p, shape, L, workspace);
+    p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
+    p.o = o; p.hT = hT;
+    p.Mb = nullptr;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    comba::mark(p, 0, s);
+    if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (comba::launch_fwd(p, shape->dtype == COMBA_BF16, false, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+    return COMBA_OK;
+}
+
+comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const void* k, const void* v,
+                               const float* alpha, const float* beta, const float* b, const float* d,
+                               const float* h0, const void* dO, const float* dhT, void* dq, void* dk, void* dv,
+                               float* dalpha, float* dbeta, float* db, float* dd, float* dh0, void* workspace,
+                               size_t workspace_bytes, void* stream) {
+    Layout L;
+    comba_status_t st = plan(shape, 1, &L);
+    if (st != COMBA_OK) return st;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
+    COMBA_REQUIRE(d); COMBA_REQUIRE(dO);
+    COMBA_REQUIRE(dq); COMBA_REQUIRE(dk); COMBA_REQUIRE(dv); COMBA_REQUIRE(dalpha); COMBA_REQUIRE(dbeta);
+    COMBA_REQUIRE(dd);
+    COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(dhT); COMBA_OPTIONAL(db); COMBA_OPTIONAL(dh0);
+    if (shape->stage_events && shape->num_stage_events < COMBA_BWD_EVENTS) return COMBA_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
+    if ((st = check_smem(shape, 1)) != COMBA_OK) return st;
+
+    char* w = static_cast<char*>(workspace);
+    ChunkParams p{};
+    fill_common(p, shape, L, workspace);
+    p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
+    p.o = nullptr; p.hT = nullptr;
+    p.dO = dO; p.dhT = dhT; p.dq = dq; p.dkk = dk; p.dvv = dv;
+    p.dalpha = dalpha; p.dbeta = dbeta; p.db = db; p.dd = dd; p.dh0 = dh0;
+    p.Mb = reinterpret_cast<float*>(w + L.M);
+    p.dHb = w + L.dH;
+    p.dEb = w + L.dE;
+    p.part = reinterpret_cast<float*>(w + L.part);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bool bf = shape->dtype == COMBA_BF16;
+    comba::mark(p, 0, s);
+    if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (comba::launch_fwd(p, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (comba::launch_bwd(p, bf, s, 3) != cudaSuccess) return COMBA_ERR_CUDA;
+    return COMBA_OK;
+}
+
+comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t dtype, const void* q,
+                                    const void* k, const void* v, const float* alpha, const float* beta,
+                                    const float* b, const float* d, float* state, void* o, void* stream) {
+    if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
+    if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
+    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128)) return COMBA_ERR_UNSUPPORTED;
+    if ((long long)Bd * H * (dv / 32) >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
+    COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
+    COMBA_OPTIONAL(b);
+    if (comba::launch_recurrent_step(Bd, H, dk, dv, dtype == COMBA_BF16, q, k, v, alpha, beta, b, d, state, o,
+                                     static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return COMBA_ERR_CUDA;
+    return COMBA_OK;
+}
+
+}  // extern "C"

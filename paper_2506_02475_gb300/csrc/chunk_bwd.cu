@@ -1,0 +1,654 @@
+// Chunk-parallel Comba backward.  The paper prints no backward pass; these
+// kernels evaluate the exact chain-rule derivatives of the chunk form of
+// section 3.3 (Eq. "prepare WY_M", the inter-chunk state equation and the
+// output equation), with chunk-local log-decays g_r = sum_{j<=r} log alpha_j:
+//
+//   k_scan_bwd  : per (sequence, head, 64-column dv tile), chunks in reverse:
+//                 dE = P^T dO + Kbar dH',   dH = gamma_C dH' + Qhat^T dO - W^T dE
+//                 (dH' = dL/dH at the chunk end, P = Tril(Q~K^T * Gamma),
+//                 Qhat = Diag(gamma) Q~, Kbar = Diag(gamma_C/gamma_r) K)
+//   k_bwd_local : per chunk, every local gradient given H, dH', E, dE:
+//                 dQ~ = dPhat K + Diag(gamma) dO H^T;  dV = Diag(beta) M^T dE;
+//                 dW = -dE H^T;  dM = dE (Diag(beta)V)^T + dW Ktilde^T;
+//                 dA = strict_lower(-M^T dM M^T);  dK from P, Kbar, W and A;
+//                 dbeta, dbtilde, and d log alpha via a reverse cumsum of the
+//                 per-position log-decay gradient inside the chunk
+//   k_reduce_heads : deterministic sums of the per-chunk db, dd partials.
+#include "params.cuh"
+
+namespace comba {
+
+template <typename T, int NT>
+__device__ __forceinline__ void frag_store_g(T* g, long long ld, int m0, int n0, const float (&acc)[NT][4], int valid) {
+#pragma unroll
+    for (int t = 0; t < NT; ++t)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int r = m0 + frag_row(2 * hh);
+            if (r >= valid) continue;
+            T* dst = g + (long long)r * ld + n0 + frag_col(t, 0);
+            dst[0] = from_f<T>(acc[t][2 * hh]);
+            dst[1] = from_f<T>(acc[t][2 * hh + 1]);
+        }
+}
+
+__device__ __forceinline__ void seq_range_b(const ChunkParams& p, int n, long long& start, long long& len) {
+    long long a = p.cu ? p.cu[n] : (long long)n * p.T;
+    long long e = p.cu ? p.cu[n + 1] : (long long)(n + 1) * p.T;
+    a = a < 0 ? 0 : (a > p.Ttot ? p.Ttot : a);
+    e = e < a ? a : (e > p.Ttot ? p.Ttot : e);
+    start = a;
+    len = e - a;
+}
+
+// ------------------------------------------------------- reverse state scan
+
+template <typename T, int DK>
+struct ScanBwdSmem {
+    static constexpr int PK = pitch<T>(DK), PT = pitch<T>(64);
+    static constexpr size_t bytes() {
+        size_t o = 0;
+        o = carve_bytes(o, sizeof(T) * 64 * PK);  // Q~
+        o = carve_bytes(o, sizeof(T) * 64 * PK);  // K
+        o = carve_bytes(o, sizeof(T) * 64 * PK);  // W
+        o = carve_bytes(o, sizeof(T) * 64 * PT);  // P
+        o = carve_bytes(o, sizeof(T) * 64 * PT);  // dO tile
+        o = carve_bytes(o, sizeof(T) * 64 * PT);  // Diag(gamma) dO tile
+        o = carve_bytes(o, sizeof(T) * DK * PT);  // dH' tile
+        o = carve_bytes(o, sizeof(T) * 64 * PT);  // -dE tile
+        o = carve_bytes(o, sizeof(float) * 64);   // G
+        return o;
+    }
+};
+
+template <typename T, int DK, int DV>
+__global__ void __launch_bounds__(128) k_scan_bwd(ChunkParams p) {
+    using S = ScanBwdSmem<T, DK>;
+    constexpr int MT = DK / 64;
+    const int jt = blockIdx.x % (DV / 64), n = blockIdx.x / (DV / 64), h = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int c0 = jt * 64;
+
+    extern __shared__ __align__(128) char smem[];
+    SmemCarver sc(smem);
+    T* sQ = sc.take<T>(64 * S::PK);
+    T* sK = sc.take<T>(64 * S::PK);
+    T* sW = sc.take<T>(64 * S::PK);
+    T* sP = sc.take<T>(64 * S::PT);
+    T* sdO = sc.take<T>(64 * S::PT);
+    T* sdOs = sc.take<T>(64 * S::PT);
+    T* sdH = sc.take<T>(DK * S::PT);
+    T* sdE = sc.take<T>(64 * S::PT);
+    float* sG = sc.take<float>(64);
+
+    float dh[MT][8][4];
+    const float* dhT = p.dhT ? p.dhT + ((long long)n * p.H + h) * DK * DV : nullptr;
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int t = 0; t < 8; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = (warp * MT + mt) * 16 + frag_row(i), c = c0 + frag_col(t, i);
+                dh[mt][t][i] = dhT ? dhT[(long long)r * DV + c] : 0.f;
+            }
+
+    long long start, len;
+    seq_range_b(p, n, start, len);
+    const int nch = (int)((len + kChunk - 1) / kChunk);
+    const int s0 = p.seq_first[n];
+    const float dd = p.d[h];
+
+    for (int c = nch - 1; c >= 0; --c) {
+        const int slot = s0 + c;
+        if (slot >= p.slots) continue;
+        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+        const long long t0 = start + (long long)c * kChunk;
+        const long long idx = (long long)slot * p.H + h;
+
+        load_tile<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+        load_tile<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+        load_tile<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
+        load_tile<T>(sdO, S::PT, (const T*)p.dO + (t0 * p.H + h) * DV + c0, (long long)p.H * DV, 64, 64, L, tid,
+                     128);
+        if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+            const int m0 = (warp * MT + mt) * 16;
+            frag_store<T, 8>(sdH, S::PT, m0, 0, dh[mt]);
+            frag_store_g<T, 8>((T*)p.dHb + idx * DK * DV + c0, DV, m0, 0, dh[mt], DK);
+        }
+        __syncthreads();
+        for (int e = tid; e < 64 * DK; e += 128) {
+            const int r = e / DK, cc = e % DK;
+            sQ[r * S::PK + cc] = from_f<T>(to_f(sQ[r * S::PK + cc]) - dd * to_f(sK[r * S::PK + cc]));
+        }
+        for (int e = tid; e < 64 * 64; e += 128) {
+            const int r = e >> 6, cc = e & 63;
+            sdOs[r * S::PT + cc] = from_f<T>(to_f(sdO[r * S::PT + cc]) * expf(sG[r]));
+        }
+        __syncthreads();
+
+        const float gL = sG[L - 1];
+        {
+            float s[8][4];
+            zero(s);
+            warp_gemm<true, true, 8>(s, sQ, S::PK, sK, S::PK, 16 * warp, 0, DK);
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = 16 * warp + frag_row(i), cc = frag_col(t, i);
+                    const float v = (cc <= r && r < L) ? s[t][i] * expf(sG[r] - sG[cc]) : 0.f;
+                    sP[r * S::PT + cc] = from_f<T>(v);
+                }
+        }
+        __syncthreads();
+        {
+            float de[8][4];
+            zero(de);
+            warp_gemm<true, false, 8>(de, sK, S::PK, sdH, S::PT, 16 * warp, 0, DK);
+            const int r0 = 16 * warp + frag_row(0), r1 = 16 * warp + frag_row(2);
+            const float e0 = r0 < L ? expf(gL - sG[r0]) : 0.f;
+            const float e1 = r1 < L ? expf(gL - sG[r1]) : 0.f;
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                de[t][0] *= e0; de[t][1] *= e0;
+                de[t][2] *= e1; de[t][3] *= e1;
+            }
+            warp_gemm<false, false, 8>(de, sP, S::PT, sdO, S::PT, 16 * warp, 0, 64);
+            frag_store_g<T, 8>((T*)p.dEb + idx * 64 * DV + c0, DV, 16 * warp, 0, de, 64);
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) de[t][i] = -de[t][i];
+            frag_store<T, 8>(sdE, S::PT, 16 * warp, 0, de);
+        }
+        __syncthreads();
+        const float dec = expf(gL);
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+            const int m0 = (warp * MT + mt) * 16;
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dh[mt][t][i] *= dec;
+            warp_gemm<false, false, 8>(dh[mt], sQ, S::PK, sdOs, S::PT, m0, 0, 64);
+            warp_gemm<false, false, 8>(dh[mt], sW, S::PK, sdE, S::PT, m0, 0, 64);
+        }
+        __syncthreads();
+    }
+
+    if (p.dh0) {
+        float* out = p.dh0 + ((long long)n * p.H + h) * DK * DV;
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = (warp * MT + mt) * 16 + frag_row(i), cc = c0 + frag_col(t, i);
+                    out[(long long)r * DV + cc] = dh[mt][t][i];
+                }
+    }
+}
+
+// ------------------------------------------------------ local chunk grads
+
+template <typename T, int DK, int DV>
+struct LocalSmem {
+    static constexpr int PK = pitch<T>(DK), PV = pitch<T>(DV), PL = pitch<T>(64);
+    static constexpr int NROW = 8;  // kinds of per-row partials
+    static constexpr size_t bytes() {
+        size_t o = 0;
+        o = carve_bytes(o, sizeof(T) * 64 * PK);   // K
+        o = carve_bytes(o, sizeof(T) * 64 * PK);   // Q~
+        o = carve_bytes(o, sizeof(T) * 64 * PK);   // dW
+        o = carve_bytes(o, sizeof(T) * 64 * PV);   // V
+        o = carve_bytes(o, sizeof(T) * 64 * PV);   // dO   (phase B: dPhat, dM)
+        o = carve_bytes(o, sizeof(T) * 64 * PV);   // E    (phase B: Y, dG)
+        o = carve_bytes(o, sizeof(T) * 64 * PV);   // dE
+        o = carve_bytes(o, sizeof(T) * DK * PV);   // H
+        o = carve_bytes(o, sizeof(T) * DK * PV);   // dH'
+        o = carve_bytes(o, sizeof(T) * 64 * PL);   // M
+        o = carve_bytes(o, sizeof(float) * 64 * 6);          // G, Gm1, beta, btilde, alpha, dg
+        o = carve_bytes(o, sizeof(float) * NROW * 2 * 64);   // row partials [kind][half][row]
+        o = carve_bytes(o, sizeof(float) * 2 * 4 * 64);      // column partials [kind][rowblock][col]
+        o = carve_bytes(o, sizeof(float) * 8);               // block reduction scratch
+        return o;
+    }
+};
+
+// Row partials of a fragment block, reduced over the quad: lane q == 0 holds the
+// sums for rows g and g + 8.
+template <int NT>
+__device__ __forceinline__ void frag_rowdot(const float (&acc)[NT][4], float& s0, float& s1) {
+    s0 = 0.f; s1 = 0.f;
+#pragma unroll
+    for (int t = 0; t < NT; ++t) { s0 += acc[t][0] + acc[t][1]; s1 += acc[t][2] + acc[t][3]; }
+    s0 = quad_sum(s0);
+    s1 = quad_sum(s1);
+}
+
+template <typename T, int DK, int DV>
+__global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
+    using S = LocalSmem<T, DK, DV>;
+    constexpr int NK = DK / 16, NV = DV / 16;   // n-tiles per warp (half the columns)
+    constexpr int PK = S::PK, PV = S::PV, PL = S::PL;
+    const int slot = blockIdx.x, h = blockIdx.y;
+    const long long idx = (long long)slot * p.H + h;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wr = warp & 3, wc = warp >> 2;
+    const int m0 = 16 * wr;
+    const SlotInfo si = p.slot_info[slot];
+    if (si.len <= 0) {
+        if (tid == 0) { p.part[idx * 2] = 0.f; p.part[idx * 2 + 1] = 0.f; }
+        return;
+    }
+    const int L = si.len;
+    const long long t0 = si.start;
+
+    extern __shared__ __align__(128) char smem[];
+    SmemCarver sc(smem);
+    T* sK = sc.take<T>(64 * PK);
+    T* sQ = sc.take<T>(64 * PK);
+    T* sdW = sc.take<T>(64 * PK);
+    T* sV = sc.take<T>(64 * PV);
+    T* sdO = sc.take<T>(64 * PV);
+    T* sE = sc.take<T>(64 * PV);
+    T* sdE = sc.take<T>(64 * PV);
+    T* sH = sc.take<T>(DK * PV);
+    T* sdH = sc.take<T>(DK * PV);
+    T* sM = sc.take<T>(64 * PL);
+    float* sG = sc.take<float>(64 * 6);
+    float* sGm1 = sG + 64;
+    float* sBe = sG + 128;
+    float* sBt = sG + 192;
+    float* sAl = sG + 256;
+    float* sDg = sG + 320;
+    float* rowp = sc.take<float>(S::NROW * 2 * 64);
+    float* colp = sc.take<float>(2 * 4 * 64);
+    float* red = sc.take<float>(8);
+    // phase-B aliases: dO, E, dE and H are dead after phase A (64 x 64 fits in 64 x dv and dk x dv)
+    T* sdPh = sdO;
+    T* sdM = sE;
+    T* sY = sdE;
+    T* sdG = sH;
+
+    const float bh = p.b ? p.b[h] : 1.f;
+    const float dh = p.d[h];
+    load_tile<T>(sK, PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
+    load_tile<T>(sQ, PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
+    load_tile<T>(sV, PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
+    load_tile<T>(sdO, PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
+    load_tile<T>(sE, PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
+    load_tile<T>(sdE, PV, (const T*)p.dEb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
+    load_tile<T>(sH, PV, (const T*)p.Hb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
+    load_tile<T>(sdH, PV, (const T*)p.dHb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
+    for (int e = tid; e < 64 * 64; e += 256) sM[(e >> 6) * PL + (e & 63)] = from_f<T>(p.Mb[idx * 4096 + e]);
+    if (tid < 64) {
+        sG[tid] = p.Gb[idx * 64 + tid];
+        sGm1[tid] = tid > 0 ? p.Gb[idx * 64 + tid - 1] : 0.f;
+        const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
+        sBe[tid] = be;
+        sBt[tid] = bh * be;
+        sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
+    }
+    __syncthreads();
+    for (int e = tid; e < 64 * DK; e += 256) {
+        const int r = e / DK, c = e % DK;
+        sQ[r * PK + c] = from_f<T>(to_f(sQ[r * PK + c]) - dh * to_f(sK[r * PK + c]));
+    }
+    // <H, dH'> (block reduction in a fixed order)
+    {
+        float s = 0.f;
+        for (int e = tid; e < DK * DV; e += 256) {
+            const int r = e / DV, c = e % DV;
+            s += to_f(sH[r * PV + c]) * to_f(sdH[r * PV + c]);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) red[warp] = s;
+    }
+    __syncthreads();
+
+    const float gL = sG[L - 1];
+    const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows
+    const float eGa = expf(sG[ra]), eGb = expf(sG[rb]);
+    const float sKa = ra < L ? expf(gL - sG[ra]) : 0.f, sKb = rb < L ? expf(gL - sG[rb]) : 0.f;
+    auto rowpart = [&](int kind) { return rowp + (kind * 2 + wc) * 64; };
+    auto put_rows = [&](int kind, float s0, float s1) {
+        if ((lane & 3) == 0) { rowpart(kind)[ra] = s0; rowpart(kind)[rb] = s1; }
+    };
+
+    // ---------------- phase A: contractions over dv
+    float acc_dq[NK][4], acc_dk[NK][4];
+    const int nk0 = wc * (DK / 2);
+    {
+        // dQ~ part: Diag(gamma) dO H^T; its row dot with Q~ is the log-decay gradient of the Q~H term.
+        zero(acc_dq);
+        warp_gemm<true, true, NK>(acc_dq, sdO, PV, sH, PV, m0, nk0, DV);
+        float t0r[NK][4];
+#pragma unroll
+        for (int t = 0; t < NK; ++t) {
+            acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb;
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                t0r[t][i] = acc_dq[t][i] * to_f(sQ[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
+        }
+        float s0, s1;
+        frag_rowdot(t0r, s0, s1);
+        put_rows(0, s0, s1);
+    }
+    {
+        // dK from Kbar: Diag(gamma_C/gamma_r) E dH'^T
+        zero(acc_dk);
+        warp_gemm<true, true, NK>(acc_dk, sE, PV, sdH, PV, m0, nk0, DV);
+        float t0r[NK][4];
+#pragma unroll
+        for (int t = 0; t < NK; ++t) {
+            acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb;
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                t0r[t][i] = acc_dk[t][i] * to_f(sK[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
+        }
+        float s0, s1;
+        frag_rowdot(t0r, s0, s1);
+        put_rows(1, s0, s1);
+    }
+    {
+        // dW = -dE H^T
+        float tmp[NK][4];
+        zero(tmp);
+        warp_gemm<true, true, NK>(tmp, sdE, PV, sH, PV, m0, nk0, DV);
+#pragma unroll
+        for (int t = 0; t < NK; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) tmp[t][i] = -tmp[t][i];
+        frag_store<T, NK>(sdW, PK, m0, nk0, tmp);
+    }
+    float dP[4][4], dMa[4][4];
+    const int nl0 = 32 * wc;
+    zero(dP);
+    warp_gemm<true, true, 4>(dP, sdO, PV, sE, PV, m0, nl0, DV);
+    zero(dMa);
+    warp_gemm<true, true, 4>(dMa, sdE, PV, sV, PV, m0, nl0, DV);
+#pragma unroll
+    for (int t = 0; t < 4; ++t)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) dMa[t][i] *= sBe[nl0 + frag_col(t, i)];
+    {
+        // dV = Diag(beta) M^T dE ; direct dbeta = v . (M^T dE)
+        const int nv0 = wc * (DV / 2);
+        float tv[NV][4];
+        zero(tv);
+        warp_gemm<false, false, NV>(tv, sM, PL, sdE, PV, m0, nv0, 64);
+        float t0r[NV][4];
+#pragma unroll
+        for (int t = 0; t < NV; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                t0r[t][i] = tv[t][i] * to_f(sV[(m0 + frag_row(i)) * PV + nv0 + frag_col(t, i)]);
+        float s0, s1;
+        frag_rowdot(t0r, s0, s1);
+        put_rows(2, s0, s1);
+        const float ba = sBe[ra], bb = sBe[rb];
+#pragma unroll
+        for (int t = 0; t < NV; ++t) { tv[t][0] *= ba; tv[t][1] *= ba; tv[t][2] *= bb; tv[t][3] *= bb; }
+        frag_store_g<T, NV>((T*)p.dvv + (t0 * p.H + h) * DV, (long long)p.H * DV, m0, nv0, tv, L);
+    }
+    __syncthreads();   // dO, E, dE, H, dH' no longer needed; dW complete
+
+    // ---------------- phase B: contractions over dk and the 64 x 64 algebra
+    float gr[4][4], sq[4][4];
+    zero(gr);
+    warp_gemm<true, true, 4>(gr, sK, PK, sK, PK, m0, nl0, DK);   // Gram K K^T
+    zero(sq);
+    warp_gemm<true, true, 4>(sq, sQ, PK, sK, PK, m0, nl0, DK);   // Q~ K^T
+    float mb[4][4];
+    zero(mb);
+    warp_gemm<true, true, 4>(mb, sdW, PK, sK, PK, m0, nl0, DK);  // dW K^T
+    {
+        float rs0 = 0.f, rs1 = 0.f;
+        float cs[4][2];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            cs[t][0] = cs[t][1] = 0.f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
+                const bool incl = c <= r && r < L;
+                const float gam = incl ? expf(sG[r] - sG[c]) : 0.f;
+                const float w = dP[t][i] * sq[t][i] * gam;   // dP * P
+                if (i < 2) rs0 += w; else rs1 += w;
+                cs[t][i & 1] += w;
+                sdPh[r * PL + c] = from_f<T>(dP[t][i] * gam);
+                const float dm = dMa[t][i] + mb[t][i] * sBt[c] * expf(sGm1[c]);
+                sdM[r * PL + c] = from_f<T>(dm);
+            }
+        }
+        rs0 = quad_sum(rs0);
+        rs1 = quad_sum(rs1);
+        put_rows(3, rs0, rs1);
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const float v = col_sum8(cs[t][e]);
+                if ((lane >> 2) == 0) colp[(0 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
+            }
+    }
+    __syncthreads();
+    {
+        float y[4][4];
+        zero(y);
+        warp_gemm<false, false, 4>(y, sM, PL, sdM, PL, m0, nl0, 64);   // Y = M^T dM
+        frag_store<T, 4>(sY, PL, m0, nl0, y);
+    }
+    __syncthreads();
+    {
+        float da[4][4];
+        zero(da);
+        warp_gemm<true, true, 4>(da, sY, PL, sM, PL, m0, nl0, 64);     // Y M^T
+        float rb0 = 0.f, rb1 = 0.f, ra0 = 0.f, ra1 = 0.f;
+        float cs[4][2];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            cs[t][0] = cs[t][1] = 0.f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
+                const bool strict = c < r && r < L;
+                const float gm = strict ? expf(sGm1[r] - sG[c]) : 0.f;
+                const float a = -da[t][i];   // dA (masked below via gm)
+                const float u = a * gm * gr[t][i];           // contributes to dbtilde_r
+                const float w = u * sBt[r];                  // dA * Aval
+                if (i < 2) { rb0 += u; ra0 += w; } else { rb1 += u; ra1 += w; }
+                cs[t][i & 1] += w;
+                sdG[r * PL + c] = from_f<T>(a * sBt[r] * gm);
+            }
+        }
+        rb0 = quad_sum(rb0); rb1 = quad_sum(rb1);
+        ra0 = quad_sum(ra0); ra1 = quad_sum(ra1);
+        put_rows(4, rb0, rb1);
+        put_rows(5, ra0, ra1);
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const float v = col_sum8(cs[t][e]);
+                if ((lane >> 2) == 0) colp[(1 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
+            }
+    }
+    __syncthreads();
+    {
+        // dQ~ = dPhat K + Diag(gamma) dO H^T ; dq = dQ~ ; dd partial = -k . dQ~
+        warp_gemm<true, false, NK>(acc_dq, sdPh, PL, sK, PK, m0, nk0, 64);
+        frag_store_g<T, NK>((T*)p.dq + (t0 * p.H + h) * DK, (long long)p.H * DK, m0, nk0, acc_dq, L);
+        float t0r[NK][4];
+#pragma unroll
+        for (int t = 0; t < NK; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                t0r[t][i] = acc_dq[t][i] * to_f(sK[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
+                acc_dk[t][i] -= dh * acc_dq[t][i];
+            }
+        float s0, s1;
+        frag_rowdot(t0r, s0, s1);
+        put_rows(6, s0, s1);
+    }
+    warp_gemm<false, false, NK>(acc_dk, sdPh, PL, sQ, PK, m0, nk0, 64);   // dPhat^T Q~
+    warp_gemm<true, false, NK>(acc_dk, sdG, PL, sK, PK, m0, nk0, 64);     // dG K
+    warp_gemm<false, false, NK>(acc_dk, sdG, PL, sK, PK, m0, nk0, 64);    // dG^T K
+    {
+        // W path: M^T dW scaled by btilde gamma_{r-1}; its row dot with k feeds dbtilde and d g_{r-1}
+        float tmp[NK][4];
+        zero(tmp);
+        warp_gemm<false, false, NK>(tmp, sM, PL, sdW, PK, m0, nk0, 64);
+        const float wa = sBt[ra] * expf(sGm1[ra]), wb = sBt[rb] * expf(sGm1[rb]);
+        float t0r[NK][4];
+#pragma unroll
+        for (int t = 0; t < NK; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                t0r[t][i] = tmp[t][i] * to_f(sK[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
+                acc_dk[t][i] += (i < 2 ? wa : wb) * tmp[t][i];
+            }
+        float s0, s1;
+        frag_rowdot(t0r, s0, s1);
+        put_rows(7, s0, s1);
+        frag_store_g<T, NK>((T*)p.dkk + (t0 * p.H + h) * DK, (long long)p.H * DK, m0, nk0, acc_dk, L);
+    }
+    __syncthreads();
+
+    // ---------------- per-position scalars (rows 0..63, one thread each)
+    auto rsum = [&](int kind, int r) { return rowp[(kind * 2) * 64 + r] + rowp[(kind * 2 + 1) * 64 + r]; };
+    auto csum = [&](int kind, int c) {
+        return colp[(kind * 4 + 0) * 64 + c] + colp[(kind * 4 + 1) * 64 + c] + colp[(kind * 4 + 2) * 64 + c] +
+               colp[(kind * 4 + 3) * 64 + c];
+    };
+    if (tid < 64) {
+        const int r = tid;
+        float g = 0.f;
+        if (r < L) {
+            g = rsum(0, r) - rsum(1, r) + rsum(3, r) - csum(0, r) - csum(1, r);
+            if (r + 1 < L) {
+                g += rsum(5, r + 1);
+                g += sBt[r + 1] * expf(sGm1[r + 1]) * rsum(7, r + 1);
+            }
+        }
+        sDg[r] = g;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        // terms that land on the last position: gamma_C <H, dH'> and the Kbar total
+        float tk = 0.f;
+        for (int r = 0; r < L; ++r) tk += rsum(1, r);
+        float hd = 0.f;
+        for (int w = 0; w < 8; ++w) hd += red[w];
+        sDg[L - 1] += tk + expf(gL) * hd;
+        // d log alpha_j = sum_{r >= j} dg_r (reverse cumsum inside the chunk)
+        float acc = 0.f;
+        for (int r = L - 1; r >= 0; --r) {
+            acc += sDg[r];
+            sDg[r] = acc;
+        }
+    }
+    __syncthreads();
+    if (tid < 64) {
+        const int r = tid;
+        float dbt = 0.f, db_c = 0.f, dd_c = 0.f;
+        if (r < L) {
+            dbt = rsum(4, r) + expf(sGm1[r]) * rsum(7, r);
+            p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r];
+            p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * dbt;
+            db_c = sBe[r] * dbt;
+            dd_c = -rsum(6, r);
+        }
+        // fixed-order reduction of the two per-chunk partials over 64 rows
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            db_c += __shfl_xor_sync(0xffffffffu, db_c, o);
+            dd_c += __shfl_xor_sync(0xffffffffu, dd_c, o);
+        }
+        if (lane == 0) { red[warp * 2] = db_c; red[warp * 2 + 1] = dd_c; }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        p.part[idx * 2] = red[0] + red[2];
+        p.part[idx * 2 + 1] = red[1] + red[3];
+    }
+}
+
+// One block per head: db[h] = sum over chunk slots of the per-chunk partials,
+// in a fixed order (strided per-thread sums, then a fixed tree).
+__global__ void __launch_bounds__(256) k_reduce_heads(ChunkParams p) {
+    __shared__ float s_db[256], s_dd[256];
+    const int h = blockIdx.x, tid = threadIdx.x;
+    float a = 0.f, c = 0.f;
+    for (int s = tid; s < p.slots; s += 256) {
+        a += p.part[((long long)s * p.H + h) * 2];
+        c += p.part[((long long)s * p.H + h) * 2 + 1];
+    }
+    s_db[tid] = a;
+    s_dd[tid] = c;
+    __syncthreads();
+    for (int o = 128; o > 0; o >>= 1) {
+        if (tid < o) { s_db[tid] += s_db[tid + o]; s_dd[tid] += s_dd[tid + o]; }
+        __syncthreads();
+    }
+    if (tid == 0) {
+        if (p.db) p.db[h] = s_db[0];
+        p.dd[h] = s_dd[0];
+    }
+}
+
+// -------------------------------------------------------------- launchers
+
+template <typename T, int DK, int DV>
+static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
+    const size_t sm_scan = ScanBwdSmem<T, DK>::bytes();
+    const size_t sm_loc = LocalSmem<T, DK, DV>::bytes();
+    cudaError_t e;
+    if ((e = cudaFuncSetAttribute(k_scan_bwd<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_scan)))
+        return e;
+    if ((e = cudaFuncSetAttribute(k_bwd_local<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_loc)))
+        return e;
+    mark(p, ev0, s);
+    k_scan_bwd<T, DK, DV><<<dim3((DV / 64) * p.N, p.H), 128, sm_scan, s>>>(p);
+    if ((e = cudaGetLastError())) return e;
+    mark(p, ev0 + 1, s);
+    if (p.slots > 0) k_bwd_local<T, DK, DV><<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
+    if ((e = cudaGetLastError())) return e;
+    mark(p, ev0 + 2, s);
+    k_reduce_heads<<<p.H, 256, 0, s>>>(p);
+    if ((e = cudaGetLastError())) return e;
+    mark(p, ev0 + 3, s);
+    return cudaSuccess;
+}
+
+cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int ev0) {
+    if (is_bf16) {
+        if (p.dk == 128 && p.dv == 128) return run_bwd<bf16, 128, 128>(p, s, ev0);
+        if (p.dk == 128 && p.dv == 64) return run_bwd<bf16, 128, 64>(p, s, ev0);
+        if (p.dk == 64 && p.dv == 128) return run_bwd<bf16, 64, 128>(p, s, ev0);
+        if (p.dk == 64 && p.dv == 64) return run_bwd<bf16, 64, 64>(p, s, ev0);
+    } else {
+        if (p.dk == 64 && p.dv == 64) return run_bwd<float, 64, 64>(p, s, ev0);
+    }
+    return cudaErrorInvalidValue;
+}
+
+size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
+#define COMBA_SM(T, DK, DV) \
+    if (dk == DK && dv == DV) return kernel == 0 ? ScanBwdSmem<T, DK>::bytes() : LocalSmem<T, DK, DV>::bytes();
+    if (is_bf16) {
+        COMBA_SM(bf16, 128, 128) COMBA_SM(bf16, 128, 64) COMBA_SM(bf16, 64, 128) COMBA_SM(bf16, 64, 64)
+    } else {
+        COMBA_SM(float, 64, 64)
+    }
+#undef COMBA_SM
+    return 0;
+}
+
+}  // namespace comba

@@ -1,0 +1,227 @@
+// Shared device helpers for the Comba chunk kernels (sm_103a).
+//
+// Tiles live in shared memory in the storage type T of the call (bf16 or
+// fp32), row-major with a 16-byte pad per row.  Products of tiles are formed
+// warp by warp on 16 x (8*NT) output blocks held in registers in the
+// accumulator-fragment layout of the m16n8k16 tensor-core MMA:
+//   lane = 4*g + q;  element i of n-tile t sits at
+//   row  m0 + g + 8*(i >> 1),  column  n0 + 8*t + 2*q + (i & 1).
+// For bf16 tiles the product runs on the tensor cores (ldmatrix + mma.sync,
+// fp32 accumulation).  For fp32 tiles the same fragment positions are
+// accumulated with fp32 FMAs, so every kernel has one body for both types.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace comba {
+
+typedef __nv_bfloat16 bf16;
+
+constexpr int kChunk = 64;  // chunk length C
+
+// ------------------------------------------------------------------ scalars
+
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+
+template <typename T> __device__ __forceinline__ T from_f(float x);
+template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float x) { return __float2bfloat16_rn(x); }
+
+// Row pitch (elements) of a shared tile with `cols` columns: 16 bytes of pad
+// keep ldmatrix row addresses and FMA-path row reads on distinct banks.
+template <typename T> __host__ __device__ constexpr int pitch(int cols) { return cols + 16 / (int)sizeof(T); }
+
+// ------------------------------------------------------------ copy helpers
+
+// Copy `rows` x `cols` elements of a strided global matrix into a shared tile,
+// zero-filling rows >= valid_rows.  16-byte vectors; cols * sizeof(T) % 16 == 0.
+template <typename T>
+__device__ __forceinline__ void load_tile(T* s, int sp, const T* g, long long gstride, int rows, int cols,
+                                          int valid_rows, int tid, int nthreads) {
+    constexpr int V = 16 / sizeof(T);
+    const int vpr = cols / V;
+    for (int idx = tid; idx < rows * vpr; idx += nthreads) {
+        const int r = idx / vpr, c = (idx % vpr) * V;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (r < valid_rows) val = *reinterpret_cast<const uint4*>(g + (long long)r * gstride + c);
+        *reinterpret_cast<uint4*>(s + r * sp + c) = val;
+    }
+}
+
+// Store a shared tile to a strided global matrix (rows < valid_rows only).
+template <typename T>
+__device__ __forceinline__ void store_tile(T* g, long long gstride, const T* s, int sp, int rows, int cols,
+                                           int valid_rows, int tid, int nthreads) {
+    constexpr int V = 16 / sizeof(T);
+    const int vpr = cols / V;
+    for (int idx = tid; idx < rows * vpr; idx += nthreads) {
+        const int r = idx / vpr, c = (idx % vpr) * V;
+        if (r < valid_rows)
+            *reinterpret_cast<uint4*>(g + (long long)r * gstride + c) = *reinterpret_cast<const uint4*>(s + r * sp + c);
+    }
+}
+
+// ---------------------------------------------------- tensor-core fragments
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(smem_u32(p)));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(smem_u32(p)));
+}
+
+__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// acc[NT][4] += A(m0.., 0..K) * B(0..K, n0..)
+//   AK: A is stored [m][k] (k contiguous); otherwise stored transposed [k][m].
+//   BK: B is stored [n][k] (k contiguous); otherwise stored [k][n].
+//   lda/ldb are row pitches in elements.  K % 16 == 0, NT even.
+template <bool AK, bool BK, int NT>
+__device__ __forceinline__ void warp_gemm(float (&acc)[NT][4], const bf16* sA, int lda, const bf16* sB, int ldb,
+                                          int m0, int n0, int K) {
+    static_assert(NT % 2 == 0, "NT must be even");
+    const int lane = threadIdx.x & 31;
+    const int j = lane >> 3, r = lane & 7;
+#pragma unroll 2
+    for (int k0 = 0; k0 < K; k0 += 16) {
+        uint32_t a[4];
+        if (AK) {
+            ldsm_x4(a, sA + (m0 + (lane & 15)) * lda + k0 + ((lane >> 4) << 3));
+        } else {
+            ldsm_x4_t(a, sA + (k0 + r + ((j >> 1) << 3)) * lda + m0 + ((j & 1) << 3));
+        }
+#pragma unroll
+        for (int t = 0; t < NT; t += 2) {
+            uint32_t b[4];
+            if (BK) {
+                ldsm_x4(b, sB + (n0 + 8 * t + r + ((j >> 1) << 3)) * ldb + k0 + ((j & 1) << 3));
+            } else {
+                ldsm_x4_t(b, sB + (k0 + r + ((j & 1) << 3)) * ldb + n0 + 8 * t + ((j >> 1) << 3));
+            }
+            mma_bf16(acc[t], a, b[0], b[1]);
+            mma_bf16(acc[t + 1], a, b[2], b[3]);
+        }
+    }
+}
+
+// fp32 tiles: same fragment positions, fp32 FMAs.
+template <bool AK, bool BK, int NT>
+__device__ __forceinline__ void warp_gemm(float (&acc)[NT][4], const float* sA, int lda, const float* sB, int ldb,
+                                          int m0, int n0, int K) {
+    const int lane = threadIdx.x & 31;
+    const int g = lane >> 2, q = lane & 3;
+    const int r0 = m0 + g, r1 = r0 + 8;
+#pragma unroll 4
+    for (int k = 0; k < K; ++k) {
+        const float a0 = AK ? sA[r0 * lda + k] : sA[k * lda + r0];
+        const float a1 = AK ? sA[r1 * lda + k] : sA[k * lda + r1];
+#pragma unroll
+        for (int t = 0; t < NT; ++t) {
+            const int c = n0 + 8 * t + 2 * q;
+            const float b0 = BK ? sB[c * ldb + k] : sB[k * ldb + c];
+            const float b1 = BK ? sB[(c + 1) * ldb + k] : sB[k * ldb + c + 1];
+            acc[t][0] = fmaf(a0, b0, acc[t][0]);
+            acc[t][1] = fmaf(a0, b1, acc[t][1]);
+            acc[t][2] = fmaf(a1, b0, acc[t][2]);
+            acc[t][3] = fmaf(a1, b1, acc[t][3]);
+        }
+    }
+}
+
+template <int NT>
+__device__ __forceinline__ void zero(float (&acc)[NT][4]) {
+#pragma unroll
+    for (int t = 0; t < NT; ++t) acc[t][0] = acc[t][1] = acc[t][2] = acc[t][3] = 0.f;
+}
+
+// Fragment coordinates (relative to the block origin).
+__device__ __forceinline__ int frag_row(int i) { return ((threadIdx.x & 31) >> 2) + ((i >> 1) << 3); }
+__device__ __forceinline__ int frag_col(int t, int i) { return 8 * t + 2 * (threadIdx.x & 3) + (i & 1); }
+
+// Write a fragment block into a shared tile of type T.
+template <typename T, int NT>
+__device__ __forceinline__ void frag_store(T* s, int sp, int m0, int n0, const float (&acc)[NT][4]) {
+#pragma unroll
+    for (int t = 0; t < NT; ++t)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) s[(m0 + frag_row(i)) * sp + n0 + frag_col(t, i)] = from_f<T>(acc[t][i]);
+}
+
+// Sum over the 4 lanes of a quad (lanes sharing fragment rows).
+__device__ __forceinline__ float quad_sum(float x) {
+    x += __shfl_xor_sync(0xffffffffu, x, 1);
+    x += __shfl_xor_sync(0xffffffffu, x, 2);
+    return x;
+}
+// Sum over the 8 lanes sharing a quad position (lanes sharing fragment columns).
+__device__ __forceinline__ float col_sum8(float x) {
+    x += __shfl_xor_sync(0xffffffffu, x, 4);
+    x += __shfl_xor_sync(0xffffffffu, x, 8);
+    x += __shfl_xor_sync(0xffffffffu, x, 16);
+    return x;
+}
+
+// ----------------------------------------------------------------- chunks
+
+// Per chunk slot: first token, length (0 = unused slot), sequence, chunk index.
+struct SlotInfo {
+    int start;
+    int len;
+    int seq;
+    int idx;
+};
+
+// Shared-memory carve-up: bump allocator with 128-byte alignment.
+struct SmemCarver {
+    char* base;
+    size_t off;
+    __device__ explicit SmemCarver(void* b) : base(static_cast<char*>(b)), off(0) {}
+    template <typename T>
+    __device__ T* take(size_t n) {
+        off = (off + 127) & ~size_t(127);
+        T* p = reinterpret_cast<T*>(base + off);
+        off += n * sizeof(T);
+        return p;
+    }
+};
+__host__ __device__ constexpr size_t carve_bytes(size_t off, size_t bytes) { return ((off + 127) & ~size_t(127)) + bytes; }
+
+// Inclusive prefix sum of log(alpha) over a chunk (warp-wide; lane handles
+// positions lane and lane + 32).  Positions >= L contribute 0, so G stays
+// finite there.  Writes G[p] and Gm1[p] = G[p-1] (Gm1[0] = 0).
+__device__ __forceinline__ void chunk_log_cumsum(const float* alpha, long long stride, int L, float* G, float* Gm1) {
+    const int lane = threadIdx.x & 31;
+    float x0 = lane < L ? logf(alpha[(long long)lane * stride]) : 0.f;
+    float x1 = lane + 32 < L ? logf(alpha[(long long)(lane + 32) * stride]) : 0.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float y0 = __shfl_up_sync(0xffffffffu, x0, o);
+        const float y1 = __shfl_up_sync(0xffffffffu, x1, o);
+        if (lane >= o) { x0 += y0; x1 += y1; }
+    }
+    const float tot0 = __shfl_sync(0xffffffffu, x0, 31);
+    x1 += tot0;
+    G[lane] = x0;
+    G[lane + 32] = x1;
+    const float p0 = __shfl_up_sync(0xffffffffu, x0, 1);
+    const float p1 = __shfl_up_sync(0xffffffffu, x1, 1);
+    Gm1[lane] = lane == 0 ? 0.f : p0;
+    Gm1[lane + 32] = lane == 0 ? tot0 : p1;
+}
+
+}  // namespace comba

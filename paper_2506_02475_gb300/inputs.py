@@ -204,3 +204,21 @@ def make_decode(Bd=256, H=16, dk=128, dv=128, steps=1, dtype="bf16", seed_offset
     d = rng.uniform(0.0, 1.0, size=H).astype(np.float32)
     b = rng.uniform(0.0, 1.0, size=H).astype(np.float32) if with_b else None
     return DecodeWorkload(dtype=dtype, state=state, q=q, k=k, v=v, alpha=alpha, beta=beta, d=d, b=b)
+
+
+def decode_state(Bd=256, H=16, dk=128, dv=128, seed_offset=0, state_std=0.05) -> np.ndarray:
+    """fp32 decode state [Bd,H,dk,dv] ~ N(0, state_std^2)."""
+    rng = np.random.Generator(np.random.PCG64(SEED + 6000 + seed_offset))
+    return (state_std * rng.standard_normal((Bd, H, dk, dv), dtype=np.float32)).astype(np.float32)
+
+
+def decode_tokens(step, Bd=256, H=16, dk=128, dv=128, dtype="bf16", seed_offset=0):
+    """Token inputs of one decode step (its own seed, so long decode runs never materialise all steps).
+
+    Returns q, k [Bd,H,dk], v [Bd,H,dv], alpha, beta [Bd,H] and d [H] (d is the same for every step)."""
+    rng = np.random.Generator(np.random.PCG64([SEED + 7000 + seed_offset, step]))
+    q, k, v = _tokens(rng, (Bd,), H, dk, dv, dtype)
+    alpha, beta = _gates(rng, (Bd, H))
+    drng = np.random.Generator(np.random.PCG64(SEED + 8000 + seed_offset))
+    d = drng.uniform(0.0, 1.0, size=H).astype(np.float32)
+    return q, k, v, alpha, beta, d

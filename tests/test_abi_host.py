@@ -1,0 +1,136 @@
+"""Host-side checks of the C ABI that need no GPU.
+
+The library loads and exports every entry point declared in include/comba.h;
+workspace sizing and argument validation answer on the host.  Every call here
+returns an error before anything would be launched (validation runs before
+the first CUDA call), so fake but well-aligned addresses are safe to pass.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2506_02475_gb300 import binding
+from paper_2506_02475_gb300 import build as cbuild
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "comba.h")
+OK, INVALID, UNSUPPORTED, WORKSPACE = 0, 1, 2, 3
+FAKE = 0x100000  # aligned, never dereferenced
+
+
+@pytest.fixture(scope="module")
+def L():
+    return binding.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(comba_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol(L):
+    names = declared_functions()
+    assert set(names) >= {"comba_chunk_fwd", "comba_chunk_bwd", "comba_recurrent_step", "comba_workspace_size",
+                          "comba_status_string"}
+    for name in names:
+        assert hasattr(L, name), name
+
+
+def test_library_is_built_for_sm103a():
+    assert any("compute_103a" in a for a in cbuild.ARCH)
+    assert os.path.exists(binding.library_path())
+
+
+def test_status_strings(L):
+    for code, text in [(0, b"ok"), (1, b"invalid argument"), (3, b"workspace missing or too small")]:
+        assert L.comba_status_string(code) == text
+    assert L.comba_status_string(99) == b"unknown status"
+
+
+def shape(B=2, T=300, H=4, dk=128, dv=128, N=None, cu=None, dtype=1, chunk=64):
+    s = binding._Shape()
+    s.B, s.T, s.H, s.dk, s.dv = B, T, H, dk, dv
+    s.num_seqs = B if N is None else N
+    s.cu_seqlens = cu
+    s.dtype, s.chunk = dtype, chunk
+    return s
+
+
+def ws(L, s, backward=0):
+    return L.comba_workspace_size(ctypes.byref(s), backward)
+
+
+def test_workspace_size_counts_chunks_and_heads(L):
+    a = ws(L, shape(T=256))
+    b = ws(L, shape(T=257))      # one more (ragged) chunk per sequence
+    c = ws(L, shape(T=256, H=8))
+    assert 0 < a < b and c > a
+    assert ws(L, shape(), 1) > ws(L, shape(), 0)
+    # bf16 needs less than fp32 storage
+    assert ws(L, shape(dtype=1)) < ws(L, shape(dtype=0))
+    # packed varlen: bound covers T/64 + N chunk slots
+    assert ws(L, shape(B=1, T=65536, N=12, cu=FAKE)) > ws(L, shape(B=1, T=65536, N=1))
+
+
+@pytest.mark.parametrize("kw", [dict(dk=96), dict(dv=256), dict(chunk=32), dict(H=0), dict(B=0), dict(dtype=7),
+                                dict(B=2, N=3), dict(B=2, cu=FAKE, N=2), dict(T=-1), dict(cu=FAKE + 4, B=1, N=1)])
+def test_invalid_shapes_have_no_workspace(L, kw):
+    assert ws(L, shape(**kw)) == 0
+
+
+def test_fp32_backward_is_limited_to_head_dim_64(L):
+    assert ws(L, shape(dtype=0, dk=64, dv=64), 1) > 0
+    assert ws(L, shape(dtype=0, dk=128, dv=128), 1) == 0
+    assert ws(L, shape(dtype=0, dk=128, dv=128), 0) > 0
+
+
+def fwd(L, s, q=FAKE, k=FAKE, v=FAKE, alpha=FAKE, beta=FAKE, b=None, d=FAKE, h0=None, o=FAKE, hT=None,
+        work=None, nbytes=0):
+    return L.comba_chunk_fwd(ctypes.byref(s), q, k, v, alpha, beta, b, d, h0, o, hT, work, nbytes, None)
+
+
+def test_forward_argument_validation(L):
+    s = shape()
+    assert fwd(L, s, q=None) == INVALID
+    assert fwd(L, s, d=None) == INVALID
+    assert fwd(L, s, o=None) == INVALID
+    assert fwd(L, s, k=FAKE + 8) == INVALID          # misaligned
+    assert fwd(L, s, b=FAKE + 4) == INVALID          # optional but misaligned
+    assert fwd(L, s, work=None, nbytes=1 << 40) == WORKSPACE
+    need = ws(L, s)
+    assert fwd(L, s, work=FAKE, nbytes=need - 1) == WORKSPACE
+    assert fwd(L, shape(dk=80)) == UNSUPPORTED
+
+
+def test_backward_argument_validation(L):
+    s = shape()
+    args = [FAKE] * 10 + [FAKE] * 8
+    base = dict(zip(["q", "k", "v", "alpha", "beta", "b", "d", "h0", "dO", "dhT", "dq", "dk", "dv", "dalpha",
+                     "dbeta", "db", "dd", "dh0"], args))
+
+    def call(nbytes=0, work=None, **over):
+        a = dict(base, **over)
+        return L.comba_chunk_bwd(ctypes.byref(s), *[a[n] for n in base], work, nbytes, None)
+
+    assert call(dO=None) == INVALID
+    assert call(dalpha=None) == INVALID
+    assert call(dd=None) == INVALID
+    assert call() == WORKSPACE                       # db, dh0, dhT, h0, b may be NULL; workspace may not
+    assert call(db=None, dh0=None, dhT=None, h0=None, b=None) == WORKSPACE
+    assert call(work=FAKE, nbytes=ws(L, s, 1) - 256) == WORKSPACE
+
+
+def test_recurrent_step_validation(L):
+    def call(Bd=4, H=2, dk=128, dv=128, dtype=1, **over):
+        a = dict(q=FAKE, k=FAKE, v=FAKE, alpha=FAKE, beta=FAKE, b=None, d=FAKE, state=FAKE, o=FAKE)
+        a.update(over)
+        return L.comba_recurrent_step(Bd, H, dk, dv, dtype, a["q"], a["k"], a["v"], a["alpha"], a["beta"], a["b"],
+                                      a["d"], a["state"], a["o"], None)
+
+    assert call(Bd=0) == INVALID
+    assert call(dk=32) == UNSUPPORTED
+    assert call(dtype=3) == INVALID
+    assert call(state=None) == INVALID
+    assert call(q=FAKE + 2) == INVALID

@@ -1,0 +1,171 @@
+"""GPU parity of the chunk-parallel forward and backward against the fp64 oracle.
+
+Every comparison runs the CUDA library through its C ABI (ctypes binding) on
+seeded synthetic inputs and the oracle on the very same values.  Small cases
+span several 64-token chunks with ragged tails; the full-size workloads run
+the whole problem on the GPU exactly as the benchmark does, and are compared
+on every (sequence) unit of sampled heads, which the oracle can afford.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_helpers import np64, rel, to_dev, tol
+from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, inputs
+
+pytestmark = pytest.mark.gpu
+
+GRADS = ("dq", "dk", "dv", "dalpha", "dbeta", "dh0")
+
+
+def gpu_fwd(t):
+    o, hT = comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"],
+                            cu_seqlens=t["cu_seqlens"], output_final_state=True)
+    torch.cuda.synchronize()
+    return np64(o), np64(hT)
+
+
+def gpu_bwd(t):
+    g = comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
+                        dhT=t["dhT"], cu_seqlens=t["cu_seqlens"])
+    torch.cuda.synchronize()
+    return {key: np64(val) for key, val in g.items()}
+
+
+def check_fwd(w, t=None, report=None):
+    t = t or to_dev(w)
+    o, hT = gpu_fwd(t)
+    ro, rhT = oracle.fwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0, cu_seqlens=w.cu_seqlens)
+    errs = {"o": rel(o, ro), "hT": rel(hT, rhT)}
+    if report is not None:
+        report.update(errs)
+    for key, e in errs.items():
+        assert e <= tol(w.dtype), (key, e)
+
+
+def check_bwd(w, t=None):
+    t = t or to_dev(w)
+    g = gpu_bwd(t)
+    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens)
+    errs = {key: rel(g[key], r[key]) for key in GRADS}
+    errs["dd"] = rel(g["dd"], r["dd"])
+    errs["db"] = rel(g["db"], r["db"])
+    bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
+    assert not bad, (bad, errs)
+    return errs
+
+
+def test_tiny_fp32_forward_workload():
+    """B=1, H=2, T=256, d=64, fp32, d=0.5, zero state: forward only, 1e-4."""
+    w = inputs.make("tiny_fp32")
+    check_fwd(w)
+
+
+SMALL = [
+    # dtype, dk, dv, B, T, with_b, with_h0
+    ("f32", 64, 64, 2, 200, True, True),
+    ("f32", 128, 128, 1, 130, False, True),
+    ("f32", 64, 128, 1, 65, True, False),
+    ("f32", 128, 64, 2, 1, True, True),
+    ("bf16", 128, 128, 2, 300, True, True),
+    ("bf16", 64, 64, 3, 64, False, False),
+    ("bf16", 128, 64, 2, 1, True, True),
+    ("bf16", 64, 128, 1, 127, True, True),
+]
+
+
+@pytest.mark.parametrize("dtype,dk,dv,B,T,with_b,with_h0", SMALL)
+def test_forward_small(dtype, dk, dv, B, T, with_b, with_h0):
+    w = inputs.make("custom", B=B, T=T, H=3, dk=dk, dv=dv, dtype=dtype, with_b=with_b, with_h0=with_h0,
+                    seed_offset=T + dk)
+    check_fwd(w)
+
+
+BWD_SMALL = [
+    ("f32", 64, 64, 2, 200, True, True),
+    ("f32", 64, 64, 1, 64, False, False),
+    ("bf16", 128, 128, 2, 300, True, True),
+    ("bf16", 64, 64, 1, 130, False, True),
+    ("bf16", 128, 64, 2, 70, True, False),
+    ("bf16", 64, 128, 1, 1, True, True),
+]
+
+
+@pytest.mark.parametrize("dtype,dk,dv,B,T,with_b,with_h0", BWD_SMALL)
+def test_backward_small(dtype, dk, dv, B, T, with_b, with_h0):
+    w = inputs.make("custom", B=B, T=T, H=2, dk=dk, dv=dv, dtype=dtype, with_b=with_b, with_h0=with_h0,
+                    with_grads=True, seed_offset=3 * T + dv)
+    check_bwd(w)
+
+
+@pytest.mark.parametrize("dtype,d", [("bf16", 128), ("f32", 64)])
+def test_varlen_small_with_empty_and_ragged_sequences(dtype, d):
+    """Packed sequences of length 1, 63, 64, 65, 0, 200, 7: state resets at every start,
+    an empty sequence passes h0 through to hT (and dhT to dh0)."""
+    lens = [1, 63, 64, 65, 0, 200, 7]
+    w = inputs.make("custom", H=2, dk=d, dv=d, dtype=dtype, with_b=True, with_h0=True, with_grads=True,
+                    lengths=lens, seed_offset=17)
+    t = to_dev(w)
+    check_fwd(w, t)
+    check_bwd(w, t)
+
+
+def test_backward_is_bitwise_deterministic():
+    w = inputs.make("custom", B=2, T=260, H=2, dk=128, dv=128, dtype="bf16", with_b=True, with_h0=True,
+                    with_grads=True, seed_offset=5)
+    t = to_dev(w)
+    a = gpu_bwd(t)
+    b = gpu_bwd(t)
+    for key in a:
+        assert np.array_equal(a[key], b[key]), key
+    o1, h1 = gpu_fwd(t)
+    o2, h2 = gpu_fwd(t)
+    assert np.array_equal(o1, o2) and np.array_equal(h1, h2)
+
+
+def _head_slice(w, h):
+    """The workload restricted to head h (every sequence), for the oracle."""
+    def tok(x):
+        return None if x is None else np.ascontiguousarray(x[..., h:h + 1, :])
+
+    def gate(x):
+        return np.ascontiguousarray(x[..., h:h + 1])
+
+    def st(x):
+        return None if x is None else np.ascontiguousarray(x[:, h:h + 1])
+
+    return dict(q=tok(w.q), k=tok(w.k), v=tok(w.v), alpha=gate(w.alpha), beta=gate(w.beta),
+                b=None if w.b is None else w.b[h:h + 1], d=w.d[h:h + 1], h0=st(w.h0), dO=tok(w.dO), dhT=st(w.dhT),
+                cu_seqlens=w.cu_seqlens)
+
+
+@pytest.mark.parametrize("name,heads", [("lm340m", [0, 7]), ("lm1p3b", [0, 15]), ("varlen64k", [5])])
+def test_full_size_workload_sampled_heads(name, heads):
+    """The full workload (launch configuration of the benchmark) on the GPU; every
+    sequence of the sampled heads against the oracle, forward and backward."""
+    w = inputs.make(name)
+    t = to_dev(w)
+    o, hT = comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"],
+                            cu_seqlens=t["cu_seqlens"], output_final_state=True)
+    g = comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
+                        dhT=t["dhT"], cu_seqlens=t["cu_seqlens"])
+    torch.cuda.synchronize()
+    for h in heads:
+        s = _head_slice(w, h)
+        ro, rhT = oracle.fwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], h0=s["h0"],
+                             cu_seqlens=s["cu_seqlens"])
+        assert rel(np64(o[..., h:h + 1, :]), ro) <= tol(w.dtype)
+        assert rel(np64(hT[:, h:h + 1]), rhT) <= tol(w.dtype)
+        r = oracle.bwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], s["dO"], h0=s["h0"],
+                       dhT=s["dhT"], cu_seqlens=s["cu_seqlens"])
+        errs = {}
+        for key in ("dq", "dk", "dv"):
+            errs[key] = rel(np64(g[key][..., h:h + 1, :]), r[key])
+        for key in ("dalpha", "dbeta"):
+            errs[key] = rel(np64(g[key][..., h:h + 1]), r[key])
+        errs["dh0"] = rel(np64(g["dh0"][:, h:h + 1]), r["dh0"])
+        errs["dd"] = rel(np64(g["dd"][h:h + 1]), r["dd"])
+        errs["db"] = rel(np64(g["db"][h:h + 1]), r["db"])
+        bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
+        assert not bad, (name, h, bad, errs)
