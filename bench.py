@@ -188,21 +188,25 @@ def time_oracle_step(s):
 
 
 def cpu_baseline(w, target_s=12.0):
-    """The oracle as it stands on this host's cores: fwd+bwd over batch row 0, all heads,
-    growing the token prefix until about `target_s` seconds of wall time."""
+    """The oracle as it stands on this host's cores: fwd+bwd over all heads of a growing
+    sample (token prefix of batch row 0, then whole batch rows) until about `target_s`
+    seconds of wall time or the whole workload."""
     import oracle
-    H = w.q.shape[2]
-    T = w.q.shape[1]
-    tokens = min(T, 256)
+    B, T, H = w.q.shape[0], w.q.shape[1], w.q.shape[2]
+    rows, tokens = 1, min(T, 256)
     while True:
-        s = oracle_sample(w, (0, 1), (0, H), tokens)
+        s = oracle_sample(w, (0, rows), (0, H), tokens)
         dt = time_oracle_step(s)
-        if dt >= target_s or tokens >= T:
+        if dt >= target_s or (tokens >= T and rows >= B):
             break
-        tokens = min(T, int(tokens * max(2.0, min(8.0, target_s / max(dt, 1e-3)))) // 64 * 64 or 64)
-    return {"value": tokens / dt, "unit": "tokens/s", "cores": oracle.default_threads(), "kind": "oracle",
-            "sample": f"fwd+bwd, batch row 0, all {H} heads, first {tokens} of {T} tokens (fp64 token recurrence,"
-                      f" exact BPTT); {dt:.2f} s"}
+        grow = max(2.0, min(8.0, target_s / max(dt, 1e-3)))
+        if tokens < T:
+            tokens = min(T, max(64, int(tokens * grow) // 64 * 64))
+        else:
+            rows = min(B, max(rows + 1, int(rows * grow)))
+    what = "the whole workload" if (rows == B and tokens == T) else f"batch rows 0..{rows - 1}, first {tokens} tokens"
+    return {"value": rows * tokens / dt, "unit": "tokens/s", "cores": oracle.default_threads(), "kind": "oracle",
+            "sample": f"fwd+bwd over {what} (all {H} heads; fp64 token recurrence, exact BPTT): {dt:.2f} s"}
 
 
 # --------------------------------------------------------------- our path
