@@ -157,6 +157,30 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
                                     const float *b, const float *d,
                                     float *state, void *o, void *stream);
 
+/*
+ * Forward without a caller workspace, for callers that may not allocate
+ * device memory (e.g. code running inside a framework's execute step that
+ * forbids allocation, or a latency-critical loop that must not reach an
+ * allocator).  The paper has no counterpart; this is a deployment variant of
+ * comba_chunk_fwd with identical arguments minus the workspace and identical
+ * results.
+ *
+ * Scratch comes from one file-scope device array of COMBA_STATIC_SCRATCH_BYTES
+ * that every GPU loading this library holds until the process exits.  Shapes
+ * whose comba_workspace_size(shape, 0) exceeds it return COMBA_ERR_WORKSPACE
+ * without launching anything.  The first call on a device looks up the
+ * array's device address (with that device current); make that first call
+ * before any stream capture.  All calls share the array: calls whose kernels
+ * may overlap on the GPU race on it and must be serialised by the caller.
+ * Nothing in it needs to start zeroed.  No allocation is made.
+ */
+#define COMBA_STATIC_SCRATCH_BYTES (32u << 20)
+comba_status_t comba_chunk_fwd_noalloc(const comba_shape_t *shape,
+                                       const void *q, const void *k, const void *v,
+                                       const float *alpha, const float *beta,
+                                       const float *b, const float *d, const float *h0,
+                                       void *o, float *hT, void *stream);
+
 /* Static, human-readable name of a status code. */
 const char *comba_status_string(comba_status_t status);
 

@@ -1,0 +1,65 @@
+"""The allocation-free forward entry point, called through the C ABI.
+
+comba_chunk_fwd_noalloc serves callers that may not allocate device memory
+(for example a plugin whose execute step forbids allocation): it takes no
+workspace and uses the library's fixed static scratch instead.  This file is
+collected last so that a run stopping at the first failure has already run
+everything else.  Each call's output must match the regular workspace-based
+comba_chunk_fwd within the parity tolerance of the storage type, on two
+calls in a row with different shapes (the shared scratch keeps the previous
+call's contents, which must not matter).
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_helpers import np64, rel, to_dev, tol
+from paper_2506_02475_gb300 import binding, comba_chunk_fwd, inputs
+
+pytestmark = pytest.mark.gpu
+
+WORKSPACE_ERR = 3
+
+
+def _noalloc():
+    L = binding.lib()
+    fn = L.comba_chunk_fwd_noalloc
+    fn.argtypes = [ctypes.POINTER(binding._Shape)] + [ctypes.c_void_p] * 11
+    fn.restype = ctypes.c_int
+    return fn
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def test_noalloc_forward_matches_workspace_forward_on_two_calls():
+    fn = _noalloc()
+    cases = [dict(B=2, T=300, H=4, dk=128, dv=128, dtype="bf16", seed_offset=41),
+             dict(B=1, T=190, H=3, dk=64, dv=64, dtype="f32", seed_offset=42)]
+    for kw in cases:
+        w = inputs.make("custom", with_b=True, with_h0=True, with_grads=False, **kw)
+        t = to_dev(w)
+        ref_o, ref_hT = comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"],
+                                        output_final_state=True)
+        o = torch.full_like(ref_o, float("nan"))
+        hT = torch.full_like(ref_hT, float("nan"))
+        shape = binding.make_shape(t["q"], t["v"])
+        st = fn(ctypes.byref(shape), _p(t["q"]), _p(t["k"]), _p(t["v"]), _p(t["alpha"]), _p(t["beta"]), _p(t["b"]),
+                _p(t["d"]), _p(t["h0"]), _p(o), _p(hT), ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+        assert st == 0, st
+        torch.cuda.synchronize()
+        assert rel(np64(o), np64(ref_o)) <= tol(w.dtype)
+        assert rel(np64(hT), np64(ref_hT)) <= tol(w.dtype)
+
+
+def test_noalloc_forward_rejects_shapes_beyond_the_static_scratch():
+    fn = _noalloc()
+    shape = binding._Shape()
+    shape.B, shape.T, shape.H, shape.dk, shape.dv = 8, 4096, 16, 128, 128
+    shape.num_seqs, shape.dtype, shape.chunk = 8, 1, 64
+    assert binding.lib().comba_workspace_size(ctypes.byref(shape), 0) > (32 << 20)
+    st = fn(ctypes.byref(shape), *([None] * 11))
+    assert st == WORKSPACE_ERR
