@@ -6,7 +6,8 @@ chunk 64, bf16 q/k/v/dO with fp32 gates, fp32 initial state h0 and final
 state gradient dhT.  One step = comba_chunk_fwd (o, hT) + comba_chunk_bwd
 (dq, dk, dv, dalpha, dbeta, db, dd, dh0).  Inputs are seeded synthetic data
 (paper_2506_02475_gb300.inputs); L2 is flushed (256 MiB write) between timed
-steps, outside the timed events.
+steps, outside the timed events.  The forward keeps the chunk factors the
+backward needs (COMBA_SAVE_FACTORS) and the backward reuses them.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload lm1p3b|lm340m|varlen64k|decode]
@@ -253,10 +254,12 @@ def run_ours(args, world, rank, local):
     hb = [e.cuda_event for e in ev_b]
 
     def step(t, events=True):
+        # training step: the forward keeps the backward's chunk factors, the backward reuses them
         comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"], cu_seqlens=cu,
-                        o=o, hT=hT, workspace=ws, stage_events=hf if events else None)
+                        o=o, hT=hT, workspace=ws, stage_events=hf if events else None, save_factors=True)
         comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
-                        dhT=t["dhT"], cu_seqlens=cu, out=grads, workspace=ws, stage_events=hb if events else None)
+                        dhT=t["dhT"], cu_seqlens=cu, out=grads, workspace=ws, stage_events=hb if events else None,
+                        reuse_factors=True)
 
     for _ in range(args.warmup):
         flush.zero_()
@@ -377,7 +380,7 @@ def run_ours(args, world, rank, local):
             "e2e": {"value": tokens * world / (e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": bi,
                     "d2h_bytes_per_step": bo, "ms_per_step": e_ms},
             "clocks": clk,
-            "gpu_launches": 10 * args.steps,
+            "gpu_launches": 7 * args.steps,
             "stages_ms_per_step": {f"{p}.{s}": v / args.steps for (p, s), v in stage_ms.items()},
             "wall_s_timed": wall,
         }
@@ -393,7 +396,8 @@ def workload_desc(w):
     else:
         shape = f"B={w.q.shape[0]} T={w.q.shape[1]}"
     return (f"{shape} H={w.H} dk={w.dk} dv={w.dv} chunk=64; {w.dtype} q/k/v/dO, fp32 gates/state; "
-            f"h0={'yes' if w.h0 is not None else 'no'}, dhT=yes; step = chunk_fwd(o,hT) + chunk_bwd(all grads)")
+            f"h0={'yes' if w.h0 is not None else 'no'}, dhT=yes; step = chunk_fwd(o,hT, saves factors) + "
+            f"chunk_bwd(all grads, reuses factors)")
 
 
 # ------------------------------------------------------------------ decode

@@ -72,6 +72,7 @@ typedef struct {
     const int32_t *cu_seqlens;  /* device int32 [N+1] or NULL                     */
     comba_dtype_t dtype;        /* storage type of q, k, v, o and their grads     */
     int chunk;                  /* chunk length; must be 64                       */
+    int flags;                  /* 0, or COMBA_SAVE_FACTORS / COMBA_REUSE_FACTORS */
     /* Optional instrumentation (NULL / 0 = off).  Caller-created cudaEvent_t
      * handles recorded on `stream` at kernel boundaries: comba_chunk_fwd
      * records COMBA_FWD_EVENTS of them (before chunk map, prep, state scan,
@@ -85,6 +86,21 @@ typedef struct {
 
 #define COMBA_FWD_EVENTS 5
 #define COMBA_BWD_EVENTS 7
+
+/*
+ * Saved factors (training step without recomputation).
+ *   comba_chunk_fwd with COMBA_SAVE_FACTORS also keeps everything the
+ *   backward needs (chunk table, W, U, log-decays, the UT inverses M, the
+ *   chunk-start states H_n and E = U - W H_n) in its workspace, which must then
+ *   hold comba_workspace_size(shape, 1) bytes (else COMBA_ERR_WORKSPACE).
+ *   comba_chunk_bwd with COMBA_REUSE_FACTORS reads them from the workspace
+ *   instead of recomputing the forward chunk factors and states.  The
+ *   workspace must come unchanged from such a forward on the same shape and
+ *   inputs; the library cannot check this.  Stage events of skipped kernels
+ *   are recorded back to back.
+ */
+#define COMBA_SAVE_FACTORS 1
+#define COMBA_REUSE_FACTORS 2
 
 /*
  * Bytes of device workspace needed by comba_chunk_fwd (backward = 0) or

@@ -21,6 +21,7 @@ _lib = None
 _lock = threading.Lock()
 
 COMBA_F32, COMBA_BF16 = 0, 1
+COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS = 1, 2
 _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "workspace missing or too small",
            4: "CUDA error", 5: "device-side wait timed out"}
 
@@ -34,7 +35,8 @@ class CombaError(RuntimeError):
 class _Shape(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int), ("dk", ctypes.c_int),
                 ("dv", ctypes.c_int), ("num_seqs", ctypes.c_int), ("cu_seqlens", ctypes.c_void_p),
-                ("dtype", ctypes.c_int), ("chunk", ctypes.c_int), ("stage_events", ctypes.c_void_p),
+                ("dtype", ctypes.c_int), ("chunk", ctypes.c_int), ("flags", ctypes.c_int),
+                ("stage_events", ctypes.c_void_p),
                 ("num_stage_events", ctypes.c_int)]
 
 
@@ -100,7 +102,7 @@ def _check(name, t, dtype=None, shape=None, device=None):
         raise ValueError(f"{name} is on {t.device}, expected {device}")
 
 
-def make_shape(q, v, cu_seqlens=None, stage_events=None):
+def make_shape(q, v, cu_seqlens=None, stage_events=None, flags=0):
     """Build the C shape struct from q [B,T,H,dk] (or packed [Ttot,H,dk]) and v.
 
     ``stage_events`` (optional): sequence of raw cudaEvent_t handles (ints) recorded at
@@ -120,6 +122,7 @@ def make_shape(q, v, cu_seqlens=None, stage_events=None):
         s.cu_seqlens = None
     s.dtype = _dtype_code(q)
     s.chunk = 64
+    s.flags = flags
     if stage_events is not None:
         arr = (ctypes.c_void_p * len(stage_events))(*stage_events)
         s._events_keepalive = arr
@@ -164,12 +167,16 @@ def _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens):
 
 
 def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, output_final_state=False,
-                    o=None, hT=None, workspace=None, stream=None, stage_events=None):
-    """Chunk-parallel forward.  Returns ``(o, hT)`` (``hT`` is None unless requested)."""
+                    o=None, hT=None, workspace=None, stream=None, stage_events=None, save_factors=False):
+    """Chunk-parallel forward.  Returns ``(o, hT)`` (``hT`` is None unless requested).
+
+    ``save_factors=True`` keeps the backward's chunk factors in ``workspace`` (which must
+    then be sized for the backward) so that ``comba_chunk_bwd(..., reuse_factors=True)``
+    with the same workspace skips recomputing them."""
     N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
-    shape = make_shape(q, v, cu_seqlens, stage_events)
+    shape = make_shape(q, v, cu_seqlens, stage_events, COMBA_SAVE_FACTORS if save_factors else 0)
     L = lib()
-    nbytes = L.comba_workspace_size(ctypes.byref(shape), 0)
+    nbytes = L.comba_workspace_size(ctypes.byref(shape), 1 if save_factors else 0)
     if nbytes == 0:
         raise CombaError("comba_workspace_size", 1)
     ws = _workspace(nbytes, q.device, workspace)
@@ -186,12 +193,17 @@ def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, o
 
 
 def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_seqlens=None, want_dh0=True,
-                    want_db=True, out=None, workspace=None, stream=None, stage_events=None):
-    """Chunk-parallel backward.  Returns a dict with dq, dk, dv, dalpha, dbeta, dd, db, dh0."""
+                    want_db=True, out=None, workspace=None, stream=None, stage_events=None, reuse_factors=False):
+    """Chunk-parallel backward.  Returns a dict with dq, dk, dv, dalpha, dbeta, dd, db, dh0.
+
+    ``reuse_factors=True`` requires ``workspace`` to hold the factors of a
+    ``comba_chunk_fwd(..., save_factors=True)`` call on the same inputs."""
     N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
     _check("dO", dO, q.dtype, v.shape, q.device)
     _check("dhT", dhT, torch.float32, (N, H, dk, dv), q.device)
-    shape = make_shape(q, v, cu_seqlens, stage_events)
+    if reuse_factors and workspace is None:
+        raise ValueError("reuse_factors=True needs the workspace of the saving forward call")
+    shape = make_shape(q, v, cu_seqlens, stage_events, COMBA_REUSE_FACTORS if reuse_factors else 0)
     L = lib()
     nbytes = L.comba_workspace_size(ctypes.byref(shape), 1)
     if nbytes == 0:

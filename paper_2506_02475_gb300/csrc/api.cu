@@ -131,8 +131,10 @@ comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const 
                                const float* h0, void* o, float* hT, void* workspace, size_t workspace_bytes,
                                void* stream) {
     Layout L;
-    comba_status_t st = plan(shape, 0, &L);
+    const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
+    comba_status_t st = plan(shape, save ? 1 : 0, &L);
     if (st != COMBA_OK) return st;
+    if (shape->flags & ~COMBA_SAVE_FACTORS) return COMBA_ERR_INVALID_ARG;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(o);
     COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
@@ -144,7 +146,7 @@ comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const 
     fill_common(p, shape, L, workspace);
     p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
     p.o = o; p.hT = hT;
-    p.Mb = nullptr;
+    p.Mb = save ? static_cast<char*>(workspace) + L.M : nullptr;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     comba::mark(p, 0, s);
     if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
@@ -160,6 +162,8 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     Layout L;
     comba_status_t st = plan(shape, 1, &L);
     if (st != COMBA_OK) return st;
+    if (shape->flags & ~COMBA_REUSE_FACTORS) return COMBA_ERR_INVALID_ARG;
+    const bool reuse = (shape->flags & COMBA_REUSE_FACTORS) != 0;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(dO);
     COMBA_REQUIRE(dq); COMBA_REQUIRE(dk); COMBA_REQUIRE(dv); COMBA_REQUIRE(dalpha); COMBA_REQUIRE(dbeta);
@@ -176,15 +180,20 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     p.o = nullptr; p.hT = nullptr;
     p.dO = dO; p.dhT = dhT; p.dq = dq; p.dkk = dk; p.dvv = dv;
     p.dalpha = dalpha; p.dbeta = dbeta; p.db = db; p.dd = dd; p.dh0 = dh0;
-    p.Mb = reinterpret_cast<float*>(w + L.M);
+    p.Mb = w + L.M;
     p.dHb = w + L.dH;
     p.dEb = w + L.dE;
     p.part = reinterpret_cast<float*>(w + L.part);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bool bf = shape->dtype == COMBA_BF16;
     comba::mark(p, 0, s);
-    if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
-    if (comba::launch_fwd(p, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (reuse) {
+        comba::mark(p, 1, s);
+        comba::mark(p, 2, s);
+    } else {
+        if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
+        if (comba::launch_fwd(p, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+    }
     if (comba::launch_bwd(p, bf, s, 3) != cudaSuccess) return COMBA_ERR_CUDA;
     return COMBA_OK;
 }

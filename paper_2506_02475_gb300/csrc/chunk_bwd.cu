@@ -46,19 +46,18 @@ __device__ __forceinline__ void seq_range_b(const ChunkParams& p, int n, long lo
 template <typename T, int DK>
 struct ScanBwdSmem {
     static constexpr int PK = pitch<T>(DK), PT = pitch<T>(64);
-    static constexpr size_t bytes() {
-        size_t o = 0;
-        o = carve_bytes(o, sizeof(T) * 64 * PK);  // Q~
-        o = carve_bytes(o, sizeof(T) * 64 * PK);  // K
-        o = carve_bytes(o, sizeof(T) * 64 * PK);  // W
-        o = carve_bytes(o, sizeof(T) * 64 * PT);  // P
-        o = carve_bytes(o, sizeof(T) * 64 * PT);  // dO tile
-        o = carve_bytes(o, sizeof(T) * 64 * PT);  // Diag(gamma) dO tile
-        o = carve_bytes(o, sizeof(T) * DK * PT);  // dH' tile
-        o = carve_bytes(o, sizeof(T) * 64 * PT);  // -dE tile
-        o = carve_bytes(o, sizeof(float) * 64);   // G
-        return o;
-    }
+    // per pipeline stage: Q (then Q~), K, W, dO tile, G
+    static constexpr size_t OQ = 0;
+    static constexpr size_t OK = align128(OQ + sizeof(T) * 64 * PK);
+    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);
+    static constexpr size_t OD = align128(OW + sizeof(T) * 64 * PK);
+    static constexpr size_t OG = align128(OD + sizeof(T) * 64 * PT);
+    static constexpr size_t STAGE = align128(OG + sizeof(float) * 64);
+    static constexpr size_t OP = 2 * STAGE;                               // P
+    static constexpr size_t OS = align128(OP + sizeof(T) * 64 * PT);      // Diag(gamma) dO tile
+    static constexpr size_t OH = align128(OS + sizeof(T) * 64 * PT);      // dH' tile
+    static constexpr size_t OE = align128(OH + sizeof(T) * DK * PT);      // -dE tile
+    static constexpr size_t bytes() { return OE + sizeof(T) * 64 * PT; }
 };
 
 template <typename T, int DK, int DV>
@@ -70,16 +69,15 @@ __global__ void __launch_bounds__(128) k_scan_bwd(ChunkParams p) {
     const int c0 = jt * 64;
 
     extern __shared__ __align__(128) char smem[];
-    SmemCarver sc(smem);
-    T* sQ = sc.take<T>(64 * S::PK);
-    T* sK = sc.take<T>(64 * S::PK);
-    T* sW = sc.take<T>(64 * S::PK);
-    T* sP = sc.take<T>(64 * S::PT);
-    T* sdO = sc.take<T>(64 * S::PT);
-    T* sdOs = sc.take<T>(64 * S::PT);
-    T* sdH = sc.take<T>(DK * S::PT);
-    T* sdE = sc.take<T>(64 * S::PT);
-    float* sG = sc.take<float>(64);
+    auto sQ = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OQ); };
+    auto sK = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OK); };
+    auto sW = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OW); };
+    auto sdO = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OD); };
+    auto sG = [&](int st) { return reinterpret_cast<float*>(smem + st * S::STAGE + S::OG); };
+    T* sP = reinterpret_cast<T*>(smem + S::OP);
+    T* sdOs = reinterpret_cast<T*>(smem + S::OS);
+    T* sdH = reinterpret_cast<T*>(smem + S::OH);
+    T* sdE = reinterpret_cast<T*>(smem + S::OE);
 
     float dh[MT][8][4];
     const float* dhT = p.dhT ? p.dhT + ((long long)n * p.H + h) * DK * DV : nullptr;
@@ -95,23 +93,40 @@ __global__ void __launch_bounds__(128) k_scan_bwd(ChunkParams p) {
 
     long long start, len;
     seq_range_b(p, n, start, len);
-    const int nch = (int)((len + kChunk - 1) / kChunk);
     const int s0 = p.seq_first[n];
+    int nch = (int)((len + kChunk - 1) / kChunk);
+    if (s0 + nch > p.slots) nch = p.slots - s0 > 0 ? p.slots - s0 : 0;
     const float dd = p.d[h];
 
-    for (int c = nch - 1; c >= 0; --c) {
-        const int slot = s0 + c;
-        if (slot >= p.slots) continue;
-        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+    auto chunk_len = [&](int c) {
+        return (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+    };
+    auto issue = [&](int c, int st) {
+        const long long idx = (long long)(s0 + c) * p.H + h;
         const long long t0 = start + (long long)c * kChunk;
-        const long long idx = (long long)slot * p.H + h;
+        const int L = chunk_len(c);
+        load_tile_async<T>(sQ(st), S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid,
+                           128);
+        load_tile_async<T>(sK(st), S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid,
+                           128);
+        load_tile_async<T>(sW(st), S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
+        load_tile_async<T>(sdO(st), S::PT, (const T*)p.dO + (t0 * p.H + h) * DV + c0, (long long)p.H * DV, 64, 64, L,
+                           tid, 128);
+        if (tid < 16) cp_async16(sG(st) + 4 * tid, p.Gb + idx * 64 + 4 * tid, true);
+        cp_async_commit();
+    };
+    if (nch > 0) issue(nch - 1, 0);
 
-        load_tile<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-        load_tile<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-        load_tile<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
-        load_tile<T>(sdO, S::PT, (const T*)p.dO + (t0 * p.H + h) * DV + c0, (long long)p.H * DV, 64, 64, L, tid,
-                     128);
-        if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+    for (int c = nch - 1, it = 0; c >= 0; --c, ++it) {
+        const int st = it & 1;
+        const int L = chunk_len(c);
+        const long long idx = (long long)(s0 + c) * p.H + h;
+        if (c > 0) {
+            issue(c - 1, st ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
             const int m0 = (warp * MT + mt) * 16;
@@ -119,27 +134,31 @@ __global__ void __launch_bounds__(128) k_scan_bwd(ChunkParams p) {
             frag_store_g<T, 8>((T*)p.dHb + idx * DK * DV + c0, DV, m0, 0, dh[mt], DK);
         }
         __syncthreads();
+        T* Q = sQ(st);
+        const T* K = sK(st);
+        const T* dO = sdO(st);
+        const float* G = sG(st);
         for (int e = tid; e < 64 * DK; e += 128) {
             const int r = e / DK, cc = e % DK;
-            sQ[r * S::PK + cc] = from_f<T>(to_f(sQ[r * S::PK + cc]) - dd * to_f(sK[r * S::PK + cc]));
+            Q[r * S::PK + cc] = from_f<T>(to_f(Q[r * S::PK + cc]) - dd * to_f(K[r * S::PK + cc]));
         }
         for (int e = tid; e < 64 * 64; e += 128) {
             const int r = e >> 6, cc = e & 63;
-            sdOs[r * S::PT + cc] = from_f<T>(to_f(sdO[r * S::PT + cc]) * expf(sG[r]));
+            sdOs[r * S::PT + cc] = from_f<T>(to_f(dO[r * S::PT + cc]) * expf(G[r]));
         }
         __syncthreads();
 
-        const float gL = sG[L - 1];
+        const float gL = G[L - 1];
         {
-            float s[8][4];
-            zero(s);
-            warp_gemm<true, true, 8>(s, sQ, S::PK, sK, S::PK, 16 * warp, 0, DK);
+            float sacc[8][4];
+            zero(sacc);
+            warp_gemm<true, true, 8>(sacc, Q, S::PK, K, S::PK, 16 * warp, 0, DK);
 #pragma unroll
             for (int t = 0; t < 8; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = 16 * warp + frag_row(i), cc = frag_col(t, i);
-                    const float v = (cc <= r && r < L) ? s[t][i] * expf(sG[r] - sG[cc]) : 0.f;
+                    const float v = (cc <= r && r < L) ? sacc[t][i] * expf(G[r] - G[cc]) : 0.f;
                     sP[r * S::PT + cc] = from_f<T>(v);
                 }
         }
@@ -147,16 +166,16 @@ __global__ void __launch_bounds__(128) k_scan_bwd(ChunkParams p) {
         {
             float de[8][4];
             zero(de);
-            warp_gemm<true, false, 8>(de, sK, S::PK, sdH, S::PT, 16 * warp, 0, DK);
+            warp_gemm<true, false, 8>(de, K, S::PK, sdH, S::PT, 16 * warp, 0, DK);
             const int r0 = 16 * warp + frag_row(0), r1 = 16 * warp + frag_row(2);
-            const float e0 = r0 < L ? expf(gL - sG[r0]) : 0.f;
-            const float e1 = r1 < L ? expf(gL - sG[r1]) : 0.f;
+            const float e0 = r0 < L ? expf(gL - G[r0]) : 0.f;
+            const float e1 = r1 < L ? expf(gL - G[r1]) : 0.f;
 #pragma unroll
             for (int t = 0; t < 8; ++t) {
                 de[t][0] *= e0; de[t][1] *= e0;
                 de[t][2] *= e1; de[t][3] *= e1;
             }
-            warp_gemm<false, false, 8>(de, sP, S::PT, sdO, S::PT, 16 * warp, 0, 64);
+            warp_gemm<false, false, 8>(de, sP, S::PT, dO, S::PT, 16 * warp, 0, 64);
             frag_store_g<T, 8>((T*)p.dEb + idx * 64 * DV + c0, DV, 16 * warp, 0, de, 64);
 #pragma unroll
             for (int t = 0; t < 8; ++t)
@@ -173,8 +192,8 @@ __global__ void __launch_bounds__(128) k_scan_bwd(ChunkParams p) {
             for (int t = 0; t < 8; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dh[mt][t][i] *= dec;
-            warp_gemm<false, false, 8>(dh[mt], sQ, S::PK, sdOs, S::PT, m0, 0, 64);
-            warp_gemm<false, false, 8>(dh[mt], sW, S::PK, sdE, S::PT, m0, 0, 64);
+            warp_gemm<false, false, 8>(dh[mt], Q, S::PK, sdOs, S::PT, m0, 0, 64);
+            warp_gemm<false, false, 8>(dh[mt], sW(st), S::PK, sdE, S::PT, m0, 0, 64);
         }
         __syncthreads();
     }
@@ -277,15 +296,16 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
 
     const float bh = p.b ? p.b[h] : 1.f;
     const float dh = p.d[h];
-    load_tile<T>(sK, PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
-    load_tile<T>(sQ, PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
-    load_tile<T>(sV, PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
-    load_tile<T>(sdO, PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
-    load_tile<T>(sE, PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
-    load_tile<T>(sdE, PV, (const T*)p.dEb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
-    load_tile<T>(sH, PV, (const T*)p.Hb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
-    load_tile<T>(sdH, PV, (const T*)p.dHb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
-    for (int e = tid; e < 64 * 64; e += 256) sM[(e >> 6) * PL + (e & 63)] = from_f<T>(p.Mb[idx * 4096 + e]);
+    load_tile_async<T>(sK, PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
+    load_tile_async<T>(sQ, PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
+    load_tile_async<T>(sV, PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
+    load_tile_async<T>(sdO, PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
+    load_tile_async<T>(sE, PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
+    load_tile_async<T>(sdE, PV, (const T*)p.dEb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
+    load_tile_async<T>(sH, PV, (const T*)p.Hb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
+    load_tile_async<T>(sdH, PV, (const T*)p.dHb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
+    load_tile_async<T>(sM, PL, (const T*)p.Mb + idx * 4096, 64, 64, 64, 64, tid, 256);
+    cp_async_commit();
     if (tid < 64) {
         sG[tid] = p.Gb[idx * 64 + tid];
         sGm1[tid] = tid > 0 ? p.Gb[idx * 64 + tid - 1] : 0.f;
@@ -294,6 +314,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         sBt[tid] = bh * be;
         sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
     }
+    cp_async_wait<0>();
     __syncthreads();
     for (int e = tid; e < 64 * DK; e += 256) {
         const int r = e / DK, c = e % DK;

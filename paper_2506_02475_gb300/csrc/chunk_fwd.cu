@@ -114,6 +114,7 @@ struct PrepSmem {
         o = carve_bytes(o, sizeof(T) * 64 * PV);
         o = carve_bytes(o, sizeof(float) * 64 * 65);
         o = carve_bytes(o, sizeof(float) * 64 * 65);
+        o = carve_bytes(o, sizeof(float) * 3 * 272);
         o = carve_bytes(o, sizeof(T) * 64 * PL);
         o = carve_bytes(o, sizeof(T) * 64 * PL);
         for (int i = 0; i < 4; ++i) o = carve_bytes(o, sizeof(float) * 64);
@@ -138,6 +139,7 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     T* sV = sc.take<T>(64 * S::PV);
     float* sA = sc.take<float>(64 * 65);
     float* sM = sc.take<float>(64 * 65);
+    float* sTmp = sc.take<float>(3 * 272);
     T* sMw = sc.take<T>(64 * S::PL);
     T* sMu = sc.take<T>(64 * S::PL);
     float* sG = sc.take<float>(64);
@@ -145,14 +147,16 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     float* sBt = sc.take<float>(64);
     float* sBe = sc.take<float>(64);
 
-    load_tile<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-    load_tile<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
+    load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    load_tile_async<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
+    cp_async_commit();
     if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
     if (tid < 64) {
         const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
         sBe[tid] = be;
         sBt[tid] = (p.b ? p.b[h] : 1.f) * be;
     }
+    cp_async_wait<0>();
     __syncthreads();
 
     // Strictly-lower A = Diag(btilde) (gamma_{r-1}/gamma_i * K K^T); exp taken only below the diagonal.
@@ -170,32 +174,17 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
                 sA[r * 65 + c] = a;
             }
     }
-    __syncthreads();
-
-    // M = (I + A)^{-1} by forward substitution, one column per lane pair:
-    // M[r][j] = -sum_{i=j}^{r-1} A[r][i] M[i][j] for r > j.
-    {
-        const int j = tid >> 1, half = tid & 1;
-        for (int r = half; r < 64; r += 2) sM[r * 65 + j] = (r == j) ? 1.f : 0.f;
-        __syncwarp();
-        for (int r = 1; r < L; ++r) {
-            float s = 0.f;
-            if (r > j)
-                for (int i = j + half; i < r; i += 2) s = fmaf(sA[r * 65 + i], sM[i * 65 + j], s);
-            s += __shfl_xor_sync(0xffffffffu, s, 1);
-            if (r > j && half == 0) sM[r * 65 + j] = -s;
-            __syncwarp();
-        }
-    }
-    __syncthreads();
+    // M = (I + A)^{-1} (the single UT inverse of the chunk), blocked forward substitution.
+    unit_lower_inverse64(sA, sM, sTmp, tid);
 
     // Column-scaled copies for the two products: Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta).
+    T* Mg = p.Mb ? (T*)p.Mb + idx * 4096 : nullptr;
     for (int e = tid; e < 64 * 64; e += 128) {
         const int r = e >> 6, c = e & 63;
         const float m = sM[r * 65 + c];
         sMw[r * S::PL + c] = from_f<T>(m * sBt[c] * expf(sGm1[c]));
         sMu[r * S::PL + c] = from_f<T>(m * sBe[c]);
-        if (p.Mb) p.Mb[idx * 4096 + e] = m;
+        if (Mg) Mg[e] = from_f<T>(m);
     }
     if (tid < 64) p.Gb[idx * 64 + tid] = sG[tid];
     __syncthreads();
@@ -219,16 +208,15 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
 template <typename T, int DK>
 struct ScanSmem {
     static constexpr int PK = pitch<T>(DK), PT = pitch<T>(64);
-    static constexpr size_t bytes() {
-        size_t o = 0;
-        o = carve_bytes(o, sizeof(T) * 64 * PK);   // W
-        o = carve_bytes(o, sizeof(T) * 64 * PK);   // K
-        o = carve_bytes(o, sizeof(T) * 64 * PT);   // U tile
-        o = carve_bytes(o, sizeof(T) * DK * PT);   // H tile
-        o = carve_bytes(o, sizeof(T) * 64 * PT);   // scaled E tile
-        o = carve_bytes(o, sizeof(float) * 64);    // G
-        return o;
-    }
+    // per pipeline stage: W, K, U tile, G
+    static constexpr size_t OW = 0;
+    static constexpr size_t OK = align128(OW + sizeof(T) * 64 * PK);
+    static constexpr size_t OU = align128(OK + sizeof(T) * 64 * PK);
+    static constexpr size_t OG = align128(OU + sizeof(T) * 64 * PT);
+    static constexpr size_t STAGE = align128(OG + sizeof(float) * 64);
+    static constexpr size_t OH = 2 * STAGE;                                  // H tile (storage type)
+    static constexpr size_t OE = align128(OH + sizeof(T) * DK * PT);         // scaled E tile
+    static constexpr size_t bytes() { return OE + sizeof(T) * 64 * PT; }
 };
 
 __device__ __forceinline__ void seq_range(const ChunkParams& p, int n, long long& start, long long& len) {
@@ -240,6 +228,9 @@ __device__ __forceinline__ void seq_range(const ChunkParams& p, int n, long long
     len = e - a;
 }
 
+// The sequential inter-chunk recurrence: E_n = U_n - W_n H_n, H_{n+1} = gamma_C H_n + Kbar_n^T E_n.
+// One CTA owns a 64-column tile of H (fp32, in registers) for one (sequence, head); the
+// next chunk's W, K, U tile and log-decays are prefetched while the current chunk computes.
 template <typename T, int DK, int DV>
 __global__ void __launch_bounds__(128) k_scan_fwd(ChunkParams p) {
     using S = ScanSmem<T, DK>;
@@ -249,13 +240,12 @@ __global__ void __launch_bounds__(128) k_scan_fwd(ChunkParams p) {
     const int c0 = jt * 64;
 
     extern __shared__ __align__(128) char smem[];
-    SmemCarver sc(smem);
-    T* sW = sc.take<T>(64 * S::PK);
-    T* sK = sc.take<T>(64 * S::PK);
-    T* sU = sc.take<T>(64 * S::PT);
-    T* sH = sc.take<T>(DK * S::PT);
-    T* sE = sc.take<T>(64 * S::PT);
-    float* sG = sc.take<float>(64);
+    auto sW = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OW); };
+    auto sK = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OK); };
+    auto sU = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OU); };
+    auto sG = [&](int st) { return reinterpret_cast<float*>(smem + st * S::STAGE + S::OG); };
+    T* sH = reinterpret_cast<T*>(smem + S::OH);
+    T* sE = reinterpret_cast<T*>(smem + S::OE);
 
     float hs[MT][8][4];
     const float* h0 = p.h0 ? p.h0 + ((long long)n * p.H + h) * DK * DV : nullptr;
@@ -271,20 +261,33 @@ __global__ void __launch_bounds__(128) k_scan_fwd(ChunkParams p) {
 
     long long start, len;
     seq_range(p, n, start, len);
-    const int nch = (int)((len + kChunk - 1) / kChunk);
     const int s0 = p.seq_first[n];
+    int nch = (int)((len + kChunk - 1) / kChunk);
+    if (s0 + nch > p.slots) nch = p.slots - s0 > 0 ? p.slots - s0 : 0;
+
+    auto issue = [&](int c, int st) {
+        const long long idx = (long long)(s0 + c) * p.H + h;
+        const long long t0 = start + (long long)c * kChunk;
+        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+        load_tile_async<T>(sW(st), S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
+        load_tile_async<T>(sK(st), S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid,
+                           128);
+        load_tile_async<T>(sU(st), S::PT, (const T*)p.Ub + idx * 64 * DV + c0, DV, 64, 64, 64, tid, 128);
+        if (tid < 16) cp_async16(sG(st) + 4 * tid, p.Gb + idx * 64 + 4 * tid, true);
+        cp_async_commit();
+    };
+    if (nch > 0) issue(0, 0);
 
     for (int c = 0; c < nch; ++c) {
-        const int slot = s0 + c;
-        if (slot >= p.slots) break;
+        const int st = c & 1;
         const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
-        const long long t0 = start + (long long)c * kChunk;
-        const long long idx = (long long)slot * p.H + h;
-
-        load_tile<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
-        load_tile<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-        load_tile<T>(sU, S::PT, (const T*)p.Ub + idx * 64 * DV + c0, DV, 64, 64, 64, tid, 128);
-        if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+        const long long idx = (long long)(s0 + c) * p.H + h;
+        if (c + 1 < nch) {
+            issue(c + 1, st ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
             const int m0 = (warp * MT + mt) * 16;
@@ -293,20 +296,22 @@ __global__ void __launch_bounds__(128) k_scan_fwd(ChunkParams p) {
         }
         __syncthreads();
 
-        const float gL = sG[L - 1];
+        const float* G = sG(st);
+        const float gL = G[L - 1];
         {
             float e[8][4];
             zero(e);
-            warp_gemm<true, false, 8>(e, sW, S::PK, sH, S::PT, 16 * warp, 0, DK);
+            warp_gemm<true, false, 8>(e, sW(st), S::PK, sH, S::PT, 16 * warp, 0, DK);
             T* Eg = (T*)p.Eb + idx * 64 * DV + c0;
+            const T* U = sU(st);
 #pragma unroll
             for (int t = 0; t < 8; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = 16 * warp + frag_row(i), cc = frag_col(t, i);
-                    const float ev = to_f(sU[r * S::PT + cc]) - e[t][i];
+                    const float ev = to_f(U[r * S::PT + cc]) - e[t][i];
                     Eg[(long long)r * DV + cc] = from_f<T>(ev);
-                    sE[r * S::PT + cc] = from_f<T>(r < L ? ev * expf(gL - sG[r]) : 0.f);
+                    sE[r * S::PT + cc] = from_f<T>(r < L ? ev * expf(gL - G[r]) : 0.f);
                 }
         }
         __syncthreads();
@@ -318,7 +323,7 @@ __global__ void __launch_bounds__(128) k_scan_fwd(ChunkParams p) {
             for (int t = 0; t < 8; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) hs[mt][t][i] *= dec;
-            warp_gemm<false, false, 8>(hs[mt], sK, S::PK, sE, S::PT, (warp * MT + mt) * 16, 0, 64);
+            warp_gemm<false, false, 8>(hs[mt], sK(st), S::PK, sE, S::PT, (warp * MT + mt) * 16, 0, 64);
         }
         __syncthreads();
     }
@@ -374,11 +379,13 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     T* sE = sc.take<T>(64 * S::PV);
     float* sG = sc.take<float>(64);
 
-    load_tile<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-    load_tile<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-    load_tile<T>(sH, S::PV, (const T*)p.Hb + idx * DK * DV, DV, DK, DV, DK, tid, 128);
-    load_tile<T>(sE, S::PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 128);
+    load_tile_async<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    load_tile_async<T>(sH, S::PV, (const T*)p.Hb + idx * DK * DV, DV, DK, DV, DK, tid, 128);
+    load_tile_async<T>(sE, S::PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 128);
+    cp_async_commit();
     if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+    cp_async_wait<0>();
     __syncthreads();
     const float dh = p.d[h];
     for (int e = tid; e < 64 * DK; e += 128) {

@@ -70,6 +70,35 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// ------------------------------------------------------ asynchronous copies
+
+// 16-byte global->shared copy that bypasses registers (cp.async); when
+// `valid` is false nothing is read and the 16 bytes are zero-filled.
+__device__ __forceinline__ void cp_async16(void* s, const void* g, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(smem_u32(s)), "l"(g),
+                 "r"(valid ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+// Asynchronous version of load_tile (rows >= valid_rows are zero-filled);
+// completes at the caller's cp_async_wait + __syncthreads.
+template <typename T>
+__device__ __forceinline__ void load_tile_async(T* s, int sp, const T* g, long long gstride, int rows, int cols,
+                                                int valid_rows, int tid, int nthreads) {
+    constexpr int V = 16 / sizeof(T);
+    const int vpr = cols / V;
+    for (int idx = tid; idx < rows * vpr; idx += nthreads) {
+        const int r = idx / vpr, c = (idx % vpr) * V;
+        const bool ok = r < valid_rows;
+        cp_async16(s + r * sp + c, ok ? (const void*)(g + (long long)r * gstride + c) : (const void*)g, ok);
+    }
+}
+
 __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(smem_u32(p)));
@@ -200,6 +229,7 @@ struct SmemCarver {
     }
 };
 __host__ __device__ constexpr size_t carve_bytes(size_t off, size_t bytes) { return ((off + 127) & ~size_t(127)) + bytes; }
+__host__ __device__ constexpr size_t align128(size_t off) { return (off + 127) & ~size_t(127); }
 
 // Inclusive prefix sum of log(alpha) over a chunk (warp-wide; lane handles
 // positions lane and lane + 32).  Positions >= L contribute 0, so G stays
@@ -222,6 +252,48 @@ __device__ __forceinline__ void chunk_log_cumsum(const float* alpha, long long s
     const float p1 = __shfl_up_sync(0xffffffffu, x1, 1);
     Gm1[lane] = lane == 0 ? 0.f : p0;
     Gm1[lane + 32] = lane == 0 ? tot0 : p1;
+}
+
+// (I + A)^{-1} for a 64 x 64 strictly-lower A (fp32, pitch 65), by blocks of 16:
+// the four diagonal blocks by forward substitution (one lane per column), then
+// the off-diagonal blocks level by level, X_ij = -X_ii sum_{k=j}^{i-1} A_ik X_kj.
+// 128 threads; `tmp` holds 3 x 16 x 17 floats.  Rows past a short chunk have
+// A = 0 and come out as identity rows.
+__device__ __forceinline__ void unit_lower_inverse64(const float* A, float* M, float* tmp, int tid) {
+    for (int e = tid; e < 64 * 64; e += 128) {
+        const int r = e >> 6, c = e & 63;
+        M[r * 65 + c] = (r == c) ? 1.f : 0.f;
+    }
+    __syncthreads();
+    if (tid < 64) {
+        const int cj = tid, end = (tid & ~15) + 16;
+        for (int r = cj + 1; r < end; ++r) {
+            float s = 0.f;
+            for (int i = cj; i < r; ++i) s = fmaf(A[r * 65 + i], M[i * 65 + cj], s);
+            M[r * 65 + cj] = -s;
+        }
+    }
+    __syncthreads();
+    for (int lvl = 1; lvl < 4; ++lvl) {
+        const int nb = 4 - lvl;
+        for (int e = tid; e < nb * 256; e += 128) {
+            const int blk = e >> 8, r = (e >> 4) & 15, c = e & 15;
+            const int bj = blk, bi = blk + lvl;
+            float s = 0.f;
+            for (int i = 16 * bj; i < 16 * bi; ++i) s = fmaf(A[(16 * bi + r) * 65 + i], M[i * 65 + 16 * bj + c], s);
+            tmp[blk * 272 + r * 17 + c] = s;
+        }
+        __syncthreads();
+        for (int e = tid; e < nb * 256; e += 128) {
+            const int blk = e >> 8, r = (e >> 4) & 15, c = e & 15;
+            const int bj = blk, bi = blk + lvl;
+            float s = 0.f;
+#pragma unroll 4
+            for (int i = 0; i < 16; ++i) s = fmaf(M[(16 * bi + r) * 65 + 16 * bi + i], tmp[blk * 272 + i * 17 + c], s);
+            M[(16 * bi + r) * 65 + 16 * bj + c] = -s;
+        }
+        __syncthreads();
+    }
 }
 
 }  // namespace comba

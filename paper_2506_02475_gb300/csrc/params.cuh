@@ -45,7 +45,7 @@ struct ChunkParams {
     void* Wb;                // [pairs][64][dk]  storage type
     void* Ub;                // [pairs][64][dv]
     float* Gb;               // [pairs][64]      chunk-local log-cumsum of alpha
-    float* Mb;               // [pairs][64][64]  UT inverse (backward only)
+    void* Mb;                // [pairs][64][64]  UT inverse, storage type (backward only)
     void* Hb;                // [pairs][dk][dv]  state at chunk start (storage type)
     void* Eb;                // [pairs][64][dv]  U - W H
     void* dHb;               // [pairs][dk][dv]  dL/dH at chunk end

@@ -49,12 +49,12 @@ def test_status_strings(L):
     assert L.comba_status_string(99) == b"unknown status"
 
 
-def shape(B=2, T=300, H=4, dk=128, dv=128, N=None, cu=None, dtype=1, chunk=64):
+def shape(B=2, T=300, H=4, dk=128, dv=128, N=None, cu=None, dtype=1, chunk=64, flags=0):
     s = binding._Shape()
     s.B, s.T, s.H, s.dk, s.dv = B, T, H, dk, dv
     s.num_seqs = B if N is None else N
     s.cu_seqlens = cu
-    s.dtype, s.chunk = dtype, chunk
+    s.dtype, s.chunk, s.flags = dtype, chunk, flags
     return s
 
 
@@ -102,6 +102,10 @@ def test_forward_argument_validation(L):
     need = ws(L, s)
     assert fwd(L, s, work=FAKE, nbytes=need - 1) == WORKSPACE
     assert fwd(L, shape(dk=80)) == UNSUPPORTED
+    # saving the backward's factors needs the backward-sized workspace
+    sv = shape(flags=1)
+    assert fwd(L, sv, work=FAKE, nbytes=ws(L, shape(), 0)) == WORKSPACE
+    assert fwd(L, shape(flags=2)) == INVALID            # reuse is a backward flag
 
 
 def test_backward_argument_validation(L):
@@ -120,6 +124,9 @@ def test_backward_argument_validation(L):
     assert call() == WORKSPACE                       # db, dh0, dhT, h0, b may be NULL; workspace may not
     assert call(db=None, dh0=None, dhT=None, h0=None, b=None) == WORKSPACE
     assert call(work=FAKE, nbytes=ws(L, s, 1) - 256) == WORKSPACE
+    s.flags = 1                                          # save is a forward flag
+    assert call() == INVALID
+    s.flags = 0
 
 
 def test_recurrent_step_validation(L):

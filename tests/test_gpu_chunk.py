@@ -142,14 +142,18 @@ def _head_slice(w, h):
 
 @pytest.mark.parametrize("name,heads", [("lm340m", [0, 7]), ("lm1p3b", [0, 15]), ("varlen64k", [5])])
 def test_full_size_workload_sampled_heads(name, heads):
-    """The full workload (launch configuration of the benchmark) on the GPU; every
-    sequence of the sampled heads against the oracle, forward and backward."""
+    """The full workload on the GPU in the benchmark's launch configuration (forward
+    saving its factors, backward reusing them); every sequence of the sampled heads
+    against the oracle, forward and backward."""
+    from paper_2506_02475_gb300 import comba_workspace_size
     w = inputs.make(name)
     t = to_dev(w)
+    ws = torch.empty(comba_workspace_size(t["q"], t["v"], t["cu_seqlens"], backward=True), dtype=torch.uint8,
+                     device="cuda")
     o, hT = comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"],
-                            cu_seqlens=t["cu_seqlens"], output_final_state=True)
+                            cu_seqlens=t["cu_seqlens"], output_final_state=True, workspace=ws, save_factors=True)
     g = comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
-                        dhT=t["dhT"], cu_seqlens=t["cu_seqlens"])
+                        dhT=t["dhT"], cu_seqlens=t["cu_seqlens"], workspace=ws, reuse_factors=True)
     torch.cuda.synchronize()
     for h in heads:
         s = _head_slice(w, h)
@@ -169,3 +173,29 @@ def test_full_size_workload_sampled_heads(name, heads):
         errs["db"] = rel(np64(g["db"][h:h + 1]), r["db"])
         bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
         assert not bad, (name, h, bad, errs)
+
+
+@pytest.mark.parametrize("dtype,d,lens", [("bf16", 128, None), ("f32", 64, None), ("bf16", 64, [70, 0, 129, 5])])
+def test_backward_reusing_saved_forward_factors(dtype, d, lens):
+    """fwd(save_factors) + bwd(reuse_factors) gives bitwise the same gradients as a
+    backward that recomputes the factors, and matches the oracle."""
+    from paper_2506_02475_gb300 import comba_workspace_size
+    w = inputs.make("custom", B=2, T=200, H=2, dk=d, dv=d, dtype=dtype, with_b=True, with_h0=True, with_grads=True,
+                    lengths=lens, seed_offset=23)
+    t = to_dev(w)
+    ws = torch.empty(comba_workspace_size(t["q"], t["v"], t["cu_seqlens"], backward=True), dtype=torch.uint8,
+                     device="cuda")
+    o, hT = comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"],
+                            cu_seqlens=t["cu_seqlens"], output_final_state=True, workspace=ws, save_factors=True)
+    g = comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
+                        dhT=t["dhT"], cu_seqlens=t["cu_seqlens"], workspace=ws, reuse_factors=True)
+    torch.cuda.synchronize()
+    g = {key: np64(val) for key, val in g.items()}
+    ref = gpu_bwd(t)
+    for key in ref:
+        assert np.array_equal(g[key], ref[key]), key
+    o2, hT2 = gpu_fwd(t)
+    assert np.array_equal(np64(o), o2) and np.array_equal(np64(hT), hT2)
+    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens)
+    for key in GRADS + ("dd", "db"):
+        assert rel(g[key], r[key]) <= tol(w.dtype), key
