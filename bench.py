@@ -54,34 +54,36 @@ def fwd_flops_per_token_head(C=64, dk=128, dv=128):
 
 
 # --------------------------------------------------------------- kernel model
-# Algorithmic FLOPs and HBM bytes per launch of each kernel of the step, per
-# (chunk, head) pair (bf16 storage, C = 64): the products the kernel must form
-# and the tensors it must read/write once.
+# Algorithmic FLOPs and HBM bytes per launch of each kernel of the training step
+# (bf16 storage, C = 64), summed over the (chunk, head) pairs one launch covers:
+# the tile products the kernel must form and the tensors it must read or write
+# once.  Forward saves the backward's factors (M, Atilde^T, E).
 
-def stage_model(dk, dv, slots, H, N):
-    C, es = 64, 2
-    pairs = slots * H
-    tile = dv // 64
+def stage_model(dk, dv, slots, H, N, save=True):
+    C, es, f4 = 64, 2, 4
+    P = slots * H
     m = {}
-    m["prep"] = dict(flops=pairs * 2 * C * C * (2 * dk + dv),
-                     bytes=pairs * (C * (dk + dv) * es + 2 * C * 4 + C * (dk + dv) * es + C * 4))
-    m["scan_fwd"] = dict(flops=pairs * 4 * C * dk * dv,
-                         bytes=pairs * (C * dk * es * 2 + C * dv * es + dk * dv * es + C * dv * es + C * 4 * tile))
-    m["output"] = dict(flops=pairs * (2 * C * C * dk + 2 * C * dk * dv + 2 * C * C * dv),
-                       bytes=pairs * (2 * C * dk * es + dk * dv * es + C * dv * es + C * dv * es + C * 4))
-    m["scan_bwd"] = dict(flops=pairs * (2 * C * C * dk * tile + 2 * C * dk * dv + 2 * C * C * dv + 4 * C * dk * dv),
-                         bytes=pairs * (3 * C * dk * es + C * dv * es + 2 * dk * dv * es // 2 + C * dv * es + C * 4))
-    m["bwd_local"] = dict(flops=pairs * (2 * C * dk * dv * 3 + 2 * C * C * dv * 2 + 2 * C * C * dv
-                                         + 2 * C * C * dk * 3 + 2 * C * C * C * 2 + 2 * C * C * dk * 5),
-                          bytes=pairs * (C * (2 * dk + 2 * dv) * es + 2 * C * dv * es + 2 * dk * dv * es
-                                         + C * C * 4 + 3 * C * 4 + C * (2 * dk + dv) * es + 2 * C * 4))
+    m["prep"] = dict(flops=P * (2 * C * C * (2 * dk + dv) + 2 * dk * C * dk * (2 if save else 1) + 2 * dv * C * dk),
+                     bytes=P * (C * (dk + dv) * es + 2 * C * f4 + C * (dk + dv) * es + C * f4 + dk * dk * es
+                                + dv * dk * es + ((C * C + dk * dk) * es if save else 0)))
+    m["scan_fwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
+    m["output"] = dict(flops=P * (4 * C * dk * dv + 2 * C * C * (dk + dv)),
+                       bytes=P * (3 * C * dk * es + C * dv * es + dv * dk * es + C * dv * es * (2 if save else 1)
+                                  + C * f4))
+    m["bwd_prep"] = dict(flops=P * (4 * C * C * dk + 2 * dv * C * dk),
+                         bytes=P * (3 * C * dk * es + C * dv * es + dv * dk * es + C * f4))
+    m["scan_bwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
+    m["bwd_local"] = dict(flops=P * (2 * C * C * dk * 9 + 2 * C * dk * dv * 4 + 2 * C * C * dv * 4 + 4 * C ** 3),
+                          bytes=P * (C * (2 * dk + 2 * dv) * es + C * dv * es + 2 * dv * dk * es + C * C * es
+                                     + 3 * C * f4 + C * (2 * dk + dv) * es + 2 * C * f4))
     m["chunk_map"] = dict(flops=0, bytes=slots * 16 + (N + 1) * 8)
-    m["reduce"] = dict(flops=0, bytes=pairs * 8 + 8 * H)
+    m["output_E"] = dict(flops=0, bytes=0)
+    m["reduce"] = dict(flops=0, bytes=P * 8 + 8 * H)
     return m
 
 
 FWD_STAGES = ["chunk_map", "prep", "scan_fwd", "output"]
-BWD_STAGES = ["chunk_map", "prep", "scan_fwd", "scan_bwd", "bwd_local", "reduce"]
+BWD_STAGES = ["chunk_map", "prep", "scan_fwd", "output_E", "bwd_prep", "scan_bwd", "bwd_local", "reduce"]
 
 
 # ------------------------------------------------------------------ clocks
@@ -245,8 +247,8 @@ def run_ours(args, world, rank, local):
              "dh0": torch.empty((N, H, dk, dv), dtype=torch.float32, device=dev)}
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
 
-    ev_f = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
-    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+    ev_f = [torch.cuda.Event(enable_timing=True) for _ in range(len(FWD_STAGES) + 1)]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(len(BWD_STAGES) + 1)]
     for e in ev_f + ev_b:
         e.record()
     torch.cuda.synchronize()
@@ -380,7 +382,7 @@ def run_ours(args, world, rank, local):
             "e2e": {"value": tokens * world / (e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": bi,
                     "d2h_bytes_per_step": bo, "ms_per_step": e_ms},
             "clocks": clk,
-            "gpu_launches": 7 * args.steps,
+            "gpu_launches": 8 * args.steps,
             "stages_ms_per_step": {f"{p}.{s}": v / args.steps for (p, s), v in stage_ms.items()},
             "wall_s_timed": wall,
         }

@@ -77,15 +77,15 @@ typedef struct {
      * handles recorded on `stream` at kernel boundaries: comba_chunk_fwd
      * records COMBA_FWD_EVENTS of them (before chunk map, prep, state scan,
      * output, and after output); comba_chunk_bwd records COMBA_BWD_EVENTS
-     * (before chunk map, prep, forward state scan, reverse state scan, local
-     * gradients, head reduction, and after it).  Fewer handles than needed
-     * is COMBA_ERR_INVALID_ARG. */
+     * (before chunk map, prep, forward state scan, forward E, reverse-scan
+     * term C, reverse state scan, local gradients, head reduction, and after
+     * it).  Fewer handles than needed is COMBA_ERR_INVALID_ARG. */
     void **stage_events;
     int num_stage_events;
 } comba_shape_t;
 
 #define COMBA_FWD_EVENTS 5
-#define COMBA_BWD_EVENTS 7
+#define COMBA_BWD_EVENTS 9
 
 /*
  * Saved factors (training step without recomputation).

@@ -16,18 +16,21 @@ size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct Layout {
-    size_t slot_info, seq_first, W, U, G, M, Hs, E, dH, dE, part, total;
+    size_t err, slot_info, seq_first, W, U, G, A, B, Hs, E, M, AT, C, dH, part, total;
     int slots;
 };
 
 // Validates the shape (not the pointers) and computes the workspace layout.
+// The forward needs W, U, G, Atilde, B^T and the chunk states; saving for the
+// backward (and the backward itself) adds E, M, Atilde^T, C^T, dH'^T and the
+// per-chunk partial sums.
 comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (!s) return COMBA_ERR_INVALID_ARG;
     if (s->B < 1 || s->T < 0 || s->H < 1 || s->num_seqs < 1) return COMBA_ERR_INVALID_ARG;
     if (s->dtype != COMBA_F32 && s->dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
     if (s->chunk != comba::kChunk) return COMBA_ERR_UNSUPPORTED;
     if ((s->dk != 64 && s->dk != 128) || (s->dv != 64 && s->dv != 128)) return COMBA_ERR_UNSUPPORTED;
-    if (s->H > 65535) return COMBA_ERR_UNSUPPORTED;
+    if (s->H > 65535 || s->num_seqs > 2147483647 / 4) return COMBA_ERR_UNSUPPORTED;
     if (s->cu_seqlens) {
         if (s->B != 1) return COMBA_ERR_INVALID_ARG;
         if (!aligned16(s->cu_seqlens)) return COMBA_ERR_INVALID_ARG;
@@ -39,23 +42,30 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (backward && s->dtype == COMBA_F32 && (s->dk != 64 || s->dv != 64)) return COMBA_ERR_UNSUPPORTED;
     const long long slots = s->cu_seqlens ? ttot / comba::kChunk + s->num_seqs
                                           : (long long)s->B * ((s->T + comba::kChunk - 1) / comba::kChunk);
-    if (slots >= (1LL << 31) / 2) return COMBA_ERR_UNSUPPORTED;
+    const long long pairs_ll = slots * s->H;
+    // the scan addresses chunk-state rows with 32-bit TMA coordinates
+    if (slots >= (1LL << 30) || pairs_ll * 128 >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
     const size_t es = s->dtype == COMBA_BF16 ? 2 : 4;
-    const size_t pairs = (size_t)slots * s->H;
+    const size_t pairs = (size_t)pairs_ll;
+    const size_t dk = s->dk, dv = s->dv;
     Layout L{};
     size_t o = 0;
     auto take = [&](size_t bytes) { size_t at = o; o = align_up(o + bytes); return at; };
+    L.err = take(sizeof(int));
     L.slot_info = take(sizeof(comba::SlotInfo) * (size_t)slots);
     L.seq_first = take(sizeof(int) * (size_t)(s->num_seqs + 1));
-    L.W = take(pairs * 64 * s->dk * es);
-    L.U = take(pairs * 64 * s->dv * es);
+    L.W = take(pairs * 64 * dk * es);
+    L.U = take(pairs * 64 * dv * es);
     L.G = take(pairs * 64 * sizeof(float));
-    L.Hs = take(pairs * (size_t)s->dk * s->dv * es);
-    L.E = take(pairs * 64 * s->dv * es);
+    L.A = take(pairs * dk * dk * es);
+    L.B = take(pairs * dv * dk * es);
+    L.Hs = take(pairs * dv * dk * es);
     if (backward) {
-        L.M = take(pairs * 64 * 64 * sizeof(float));
-        L.dH = take(pairs * (size_t)s->dk * s->dv * es);
-        L.dE = take(pairs * 64 * s->dv * es);
+        L.E = take(pairs * 64 * dv * es);
+        L.M = take(pairs * 64 * 64 * es);
+        L.AT = take(pairs * dk * dk * es);
+        L.C = take(pairs * dv * dk * es);
+        L.dH = take(pairs * dv * dk * es);
         L.part = take(pairs * 2 * sizeof(float));
     }
     L.total = o;
@@ -78,7 +88,7 @@ comba_status_t check_smem(const comba_shape_t* s, int backward) {
     return COMBA_OK;
 }
 
-void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* ws) {
+void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* ws, bool backward_layout) {
     char* w = static_cast<char*>(ws);
     p.B = s->B; p.T = s->T; p.H = s->H; p.dk = s->dk; p.dv = s->dv; p.N = s->num_seqs;
     p.Ttot = (long long)s->B * s->T;
@@ -86,13 +96,23 @@ void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* 
     p.slots = L.slots;
     p.ev = reinterpret_cast<cudaEvent_t*>(s->stage_events);
     p.nev = s->stage_events ? s->num_stage_events : 0;
+    p.err = reinterpret_cast<int*>(w + L.err);
     p.slot_info = reinterpret_cast<comba::SlotInfo*>(w + L.slot_info);
     p.seq_first = reinterpret_cast<int*>(w + L.seq_first);
     p.Wb = w + L.W;
     p.Ub = w + L.U;
     p.Gb = reinterpret_cast<float*>(w + L.G);
+    p.Ab = w + L.A;
+    p.Bb = w + L.B;
     p.Hb = w + L.Hs;
-    p.Eb = w + L.E;
+    if (backward_layout) {
+        p.Eb = w + L.E;
+        p.Mb = w + L.M;
+        p.ATb = w + L.AT;
+        p.Cb = w + L.C;
+        p.dHb = w + L.dH;
+        p.part = reinterpret_cast<float*>(w + L.part);
+    }
 }
 
 #define COMBA_REQUIRE(ptr)                                   \
@@ -143,14 +163,13 @@ comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const 
     if ((st = check_smem(shape, 0)) != COMBA_OK) return st;
 
     ChunkParams p{};
-    fill_common(p, shape, L, workspace);
+    fill_common(p, shape, L, workspace, save);
     p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
     p.o = o; p.hT = hT;
-    p.Mb = save ? static_cast<char*>(workspace) + L.M : nullptr;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     comba::mark(p, 0, s);
     if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
-    if (comba::launch_fwd(p, shape->dtype == COMBA_BF16, false, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (comba::launch_fwd(p, shape->dtype == COMBA_BF16, save, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
     return COMBA_OK;
 }
 
@@ -173,28 +192,25 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
     if ((st = check_smem(shape, 1)) != COMBA_OK) return st;
 
-    char* w = static_cast<char*>(workspace);
     ChunkParams p{};
-    fill_common(p, shape, L, workspace);
+    fill_common(p, shape, L, workspace, true);
     p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
-    p.o = nullptr; p.hT = nullptr;
     p.dO = dO; p.dhT = dhT; p.dq = dq; p.dkk = dk; p.dvv = dv;
     p.dalpha = dalpha; p.dbeta = dbeta; p.db = db; p.dd = dd; p.dh0 = dh0;
-    p.Mb = w + L.M;
-    p.dHb = w + L.dH;
-    p.dEb = w + L.dE;
-    p.part = reinterpret_cast<float*>(w + L.part);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bool bf = shape->dtype == COMBA_BF16;
     comba::mark(p, 0, s);
     if (reuse) {
-        comba::mark(p, 1, s);
-        comba::mark(p, 2, s);
+        for (int e = 1; e <= 4; ++e) comba::mark(p, e, s);
     } else {
-        if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
-        if (comba::launch_fwd(p, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+        // recompute the forward factors and chunk states (no output, no final state)
+        ChunkParams f = p;
+        f.o = nullptr;
+        f.hT = nullptr;
+        if (comba::launch_chunk_map(f, s) != cudaSuccess) return COMBA_ERR_CUDA;
+        if (comba::launch_fwd(f, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
     }
-    if (comba::launch_bwd(p, bf, s, 3) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (comba::launch_bwd(p, bf, s, 4) != cudaSuccess) return COMBA_ERR_CUDA;
     return COMBA_OK;
 }
 

@@ -1,14 +1,15 @@
 // Chunk-parallel Comba backward.  The paper prints no backward pass; these
 // kernels evaluate the exact chain-rule derivatives of the chunk form of
 // section 3.3 (Eq. "prepare WY_M", the inter-chunk state equation and the
-// output equation), with chunk-local log-decays g_r = sum_{j<=r} log alpha_j:
-//
-//   k_scan_bwd  : per (sequence, head, 64-column dv tile), chunks in reverse:
-//                 dE = P^T dO + Kbar dH',   dH = gamma_C dH' + Qhat^T dO - W^T dE
-//                 (dH' = dL/dH at the chunk end, P = Tril(Q~K^T * Gamma),
-//                 Qhat = Diag(gamma) Q~, Kbar = Diag(gamma_C/gamma_r) K)
-//   k_bwd_local : per chunk, every local gradient given H, dH', E, dE:
-//                 dQ~ = dPhat K + Diag(gamma) dO H^T;  dV = Diag(beta) M^T dE;
+// output equation), with chunk-local log-decays g_r = sum_{j<=r} log alpha_j.
+// With dH' = dL/dH at a chunk's end, P = Tril(Q~K^T * Gamma), Qhat =
+// Diag(gamma) Q~ and Kbar = Diag(gamma_C/gamma_r) K:
+//   dE = P^T dO + Kbar dH',   dH = gamma_C dH' + Qhat^T dO - W^T dE
+//      = gamma_C dH' + Atilde^T dH' + C,   C = (Qhat - P W)^T dO.
+//   k_bwd_prep  : per chunk, C^T (the additive term of the reverse scan)
+//   (scan.cu)   : the reverse scan dH_n = gamma dH_{n+1} + Atilde^T dH_{n+1} + C_n
+//   k_bwd_local : per chunk, every local gradient given H_n, dH', E:
+//                 dE; dQ~ = dPhat K + Diag(gamma) dO H^T;  dV = Diag(beta) M^T dE;
 //                 dW = -dE H^T;  dM = dE (Diag(beta)V)^T + dW Ktilde^T;
 //                 dA = strict_lower(-M^T dM M^T);  dK from P, Kbar, W and A;
 //                 dbeta, dbtilde, and d log alpha via a reverse cumsum of the
@@ -41,174 +42,106 @@ __device__ __forceinline__ void seq_range_b(const ChunkParams& p, int n, long lo
     len = e - a;
 }
 
-// ------------------------------------------------------- reverse state scan
-
-template <typename T, int DK>
-struct ScanBwdSmem {
-    static constexpr int PK = pitch<T>(DK), PT = pitch<T>(64);
-    // per pipeline stage: Q (then Q~), K, W, dO tile, G
-    static constexpr size_t OQ = 0;
-    static constexpr size_t OK = align128(OQ + sizeof(T) * 64 * PK);
-    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);
-    static constexpr size_t OD = align128(OW + sizeof(T) * 64 * PK);
-    static constexpr size_t OG = align128(OD + sizeof(T) * 64 * PT);
-    static constexpr size_t STAGE = align128(OG + sizeof(float) * 64);
-    static constexpr size_t OP = 2 * STAGE;                               // P
-    static constexpr size_t OS = align128(OP + sizeof(T) * 64 * PT);      // Diag(gamma) dO tile
-    static constexpr size_t OH = align128(OS + sizeof(T) * 64 * PT);      // dH' tile
-    static constexpr size_t OE = align128(OH + sizeof(T) * DK * PT);      // -dE tile
-    static constexpr size_t bytes() { return OE + sizeof(T) * 64 * PT; }
-};
+// ------------------------------------------------- reverse-scan additive term
 
 template <typename T, int DK, int DV>
-__global__ void __launch_bounds__(128) k_scan_bwd(ChunkParams p) {
-    using S = ScanBwdSmem<T, DK>;
-    constexpr int MT = DK / 64;
-    const int jt = blockIdx.x % (DV / 64), n = blockIdx.x / (DV / 64), h = blockIdx.y;
+struct BPrepSmem {
+    static constexpr int PK = pitch<T>(DK), PV = pitch<T>(DV), PL = pitch<T>(64);
+    static constexpr size_t OQ = 0;                                      // Q~
+    static constexpr size_t OK = align128(OQ + sizeof(T) * 64 * PK);     // K, later Z = Qhat - P W
+    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);     // W
+    static constexpr size_t OD = align128(OW + sizeof(T) * 64 * PK);     // dO
+    static constexpr size_t OP = align128(OD + sizeof(T) * 64 * PV);     // P
+    static constexpr size_t OG = align128(OP + sizeof(T) * 64 * PL);
+    static constexpr size_t bytes() { return OG + sizeof(float) * 64; }
+};
+
+// C^T = dO^T (Qhat - P W)  [dv][dk], per (chunk, head).
+template <typename T, int DK, int DV>
+__global__ void __launch_bounds__(128) k_bwd_prep(ChunkParams p) {
+    using S = BPrepSmem<T, DK, DV>;
+    const int slot = blockIdx.x, h = blockIdx.y;
+    const SlotInfo si = p.slot_info[slot];
+    if (si.len <= 0) return;
+    const int L = si.len;
+    const long long t0 = si.start;
+    const long long idx = (long long)slot * p.H + h;
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int c0 = jt * 64;
 
     extern __shared__ __align__(128) char smem[];
-    auto sQ = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OQ); };
-    auto sK = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OK); };
-    auto sW = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OW); };
-    auto sdO = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OD); };
-    auto sG = [&](int st) { return reinterpret_cast<float*>(smem + st * S::STAGE + S::OG); };
+    T* sQ = reinterpret_cast<T*>(smem + S::OQ);
+    T* sK = reinterpret_cast<T*>(smem + S::OK);
+    T* sZ = sK;
+    T* sW = reinterpret_cast<T*>(smem + S::OW);
+    T* sdO = reinterpret_cast<T*>(smem + S::OD);
     T* sP = reinterpret_cast<T*>(smem + S::OP);
-    T* sdOs = reinterpret_cast<T*>(smem + S::OS);
-    T* sdH = reinterpret_cast<T*>(smem + S::OH);
-    T* sdE = reinterpret_cast<T*>(smem + S::OE);
+    float* sG = reinterpret_cast<float*>(smem + S::OG);
 
-    float dh[MT][8][4];
-    const float* dhT = p.dhT ? p.dhT + ((long long)n * p.H + h) * DK * DV : nullptr;
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
+    load_tile_async<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
+    load_tile_async<T>(sdO, S::PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
+    cp_async_commit();
+    if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+    cp_async_wait<0>();
+    __syncthreads();
+    const float dd = p.d[h];
+    for (int e = tid; e < 64 * DK; e += 128) {
+        const int r = e / DK, c = e % DK;
+        sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dd * to_f(sK[r * S::PK + c]));
+    }
+    __syncthreads();
+    {
+        float sc[8][4];
+        zero(sc);
+        warp_gemm<true, true, 8>(sc, sQ, S::PK, sK, S::PK, 16 * warp, 0, DK);
 #pragma unroll
         for (int t = 0; t < 8; ++t)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                const int r = (warp * MT + mt) * 16 + frag_row(i), c = c0 + frag_col(t, i);
-                dh[mt][t][i] = dhT ? dhT[(long long)r * DV + c] : 0.f;
+                const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
+                const float v = (c <= r && r < L) ? sc[t][i] * expf(sG[r] - sG[c]) : 0.f;
+                sP[r * S::PL + c] = from_f<T>(v);
             }
-
-    long long start, len;
-    seq_range_b(p, n, start, len);
-    const int s0 = p.seq_first[n];
-    int nch = (int)((len + kChunk - 1) / kChunk);
-    if (s0 + nch > p.slots) nch = p.slots - s0 > 0 ? p.slots - s0 : 0;
-    const float dd = p.d[h];
-
-    auto chunk_len = [&](int c) {
-        return (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
-    };
-    auto issue = [&](int c, int st) {
-        const long long idx = (long long)(s0 + c) * p.H + h;
-        const long long t0 = start + (long long)c * kChunk;
-        const int L = chunk_len(c);
-        load_tile_async<T>(sQ(st), S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid,
-                           128);
-        load_tile_async<T>(sK(st), S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid,
-                           128);
-        load_tile_async<T>(sW(st), S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
-        load_tile_async<T>(sdO(st), S::PT, (const T*)p.dO + (t0 * p.H + h) * DV + c0, (long long)p.H * DV, 64, 64, L,
-                           tid, 128);
-        if (tid < 16) cp_async16(sG(st) + 4 * tid, p.Gb + idx * 64 + 4 * tid, true);
-        cp_async_commit();
-    };
-    if (nch > 0) issue(nch - 1, 0);
-
-    for (int c = nch - 1, it = 0; c >= 0; --c, ++it) {
-        const int st = it & 1;
-        const int L = chunk_len(c);
-        const long long idx = (long long)(s0 + c) * p.H + h;
-        if (c > 0) {
-            issue(c - 1, st ^ 1);
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            const int m0 = (warp * MT + mt) * 16;
-            frag_store<T, 8>(sdH, S::PT, m0, 0, dh[mt]);
-            frag_store_g<T, 8>((T*)p.dHb + idx * DK * DV + c0, DV, m0, 0, dh[mt], DK);
-        }
-        __syncthreads();
-        T* Q = sQ(st);
-        const T* K = sK(st);
-        const T* dO = sdO(st);
-        const float* G = sG(st);
-        for (int e = tid; e < 64 * DK; e += 128) {
-            const int r = e / DK, cc = e % DK;
-            Q[r * S::PK + cc] = from_f<T>(to_f(Q[r * S::PK + cc]) - dd * to_f(K[r * S::PK + cc]));
-        }
-        for (int e = tid; e < 64 * 64; e += 128) {
-            const int r = e >> 6, cc = e & 63;
-            sdOs[r * S::PT + cc] = from_f<T>(to_f(dO[r * S::PT + cc]) * expf(G[r]));
-        }
-        __syncthreads();
-
-        const float gL = G[L - 1];
-        {
-            float sacc[8][4];
-            zero(sacc);
-            warp_gemm<true, true, 8>(sacc, Q, S::PK, K, S::PK, 16 * warp, 0, DK);
-#pragma unroll
-            for (int t = 0; t < 8; ++t)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int r = 16 * warp + frag_row(i), cc = frag_col(t, i);
-                    const float v = (cc <= r && r < L) ? sacc[t][i] * expf(G[r] - G[cc]) : 0.f;
-                    sP[r * S::PT + cc] = from_f<T>(v);
-                }
-        }
-        __syncthreads();
-        {
-            float de[8][4];
-            zero(de);
-            warp_gemm<true, false, 8>(de, K, S::PK, sdH, S::PT, 16 * warp, 0, DK);
-            const int r0 = 16 * warp + frag_row(0), r1 = 16 * warp + frag_row(2);
-            const float e0 = r0 < L ? expf(gL - G[r0]) : 0.f;
-            const float e1 = r1 < L ? expf(gL - G[r1]) : 0.f;
-#pragma unroll
-            for (int t = 0; t < 8; ++t) {
-                de[t][0] *= e0; de[t][1] *= e0;
-                de[t][2] *= e1; de[t][3] *= e1;
-            }
-            warp_gemm<false, false, 8>(de, sP, S::PT, dO, S::PT, 16 * warp, 0, 64);
-            frag_store_g<T, 8>((T*)p.dEb + idx * 64 * DV + c0, DV, 16 * warp, 0, de, 64);
-#pragma unroll
-            for (int t = 0; t < 8; ++t)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) de[t][i] = -de[t][i];
-            frag_store<T, 8>(sdE, S::PT, 16 * warp, 0, de);
-        }
-        __syncthreads();
-        const float dec = expf(gL);
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            const int m0 = (warp * MT + mt) * 16;
-#pragma unroll
-            for (int t = 0; t < 8; ++t)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) dh[mt][t][i] *= dec;
-            warp_gemm<false, false, 8>(dh[mt], Q, S::PK, sdOs, S::PT, m0, 0, 64);
-            warp_gemm<false, false, 8>(dh[mt], sW(st), S::PK, sdE, S::PT, m0, 0, 64);
-        }
-        __syncthreads();
     }
-
-    if (p.dh0) {
-        float* out = p.dh0 + ((long long)n * p.H + h) * DK * DV;
+    __syncthreads();
+    {
+        // Z = Diag(gamma) Q~ - P W  (replaces K)
+        float z[DK / 8][4];
+        zero(z);
+        warp_gemm<true, false, DK / 8>(z, sP, S::PL, sW, S::PK, 16 * warp, 0, 64);
+        const float ea = expf(sG[16 * warp + frag_row(0)]), eb = expf(sG[16 * warp + frag_row(2)]);
 #pragma unroll
-        for (int mt = 0; mt < MT; ++mt)
+        for (int t = 0; t < DK / 8; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
+                z[t][i] = (i < 2 ? ea : eb) * to_f(sQ[r * S::PK + c]) - z[t][i];
+            }
+        __syncthreads();   // every warp is done reading K (via P) before Z overwrites it
+        frag_store<T, DK / 8>(sZ, S::PK, 16 * warp, 0, z);
+    }
+    __syncthreads();
+    // C^T = dO^T Z
+    constexpr int MT = DV / 64;
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+        const int m0 = (warp * MT + mt) * 16;
+#pragma unroll
+        for (int n0 = 0; n0 < DK; n0 += 64) {
+            float acc[8][4];
+            zero(acc);
+            warp_gemm<false, false, 8>(acc, sdO, S::PV, sZ, S::PK, m0, n0, 64);
+            T* g = (T*)p.Cb + idx * DV * DK;
 #pragma unroll
             for (int t = 0; t < 8; ++t)
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int r = (warp * MT + mt) * 16 + frag_row(i), cc = c0 + frag_col(t, i);
-                    out[(long long)r * DV + cc] = dh[mt][t][i];
+                for (int hh = 0; hh < 2; ++hh) {
+                    T* dst = g + (long long)(m0 + frag_row(2 * hh)) * DK + n0 + frag_col(t, 0);
+                    dst[0] = from_f<T>(acc[t][2 * hh]);
+                    dst[1] = from_f<T>(acc[t][2 * hh + 1]);
                 }
+        }
     }
 }
 
@@ -227,8 +160,8 @@ struct LocalSmem {
         o = carve_bytes(o, sizeof(T) * 64 * PV);   // dO   (phase B: dPhat, dM)
         o = carve_bytes(o, sizeof(T) * 64 * PV);   // E    (phase B: Y, dG)
         o = carve_bytes(o, sizeof(T) * 64 * PV);   // dE
-        o = carve_bytes(o, sizeof(T) * DK * PV);   // H
-        o = carve_bytes(o, sizeof(T) * DK * PV);   // dH'
+        o = carve_bytes(o, sizeof(T) * DV * PK);   // H^T
+        o = carve_bytes(o, sizeof(T) * DV * PK);   // dH'^T
         o = carve_bytes(o, sizeof(T) * 64 * PL);   // M
         o = carve_bytes(o, sizeof(float) * 64 * 6);          // G, Gm1, beta, btilde, alpha, dg
         o = carve_bytes(o, sizeof(float) * NROW * 2 * 64);   // row partials [kind][half][row]
@@ -276,8 +209,8 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     T* sdO = sc.take<T>(64 * PV);
     T* sE = sc.take<T>(64 * PV);
     T* sdE = sc.take<T>(64 * PV);
-    T* sH = sc.take<T>(DK * PV);
-    T* sdH = sc.take<T>(DK * PV);
+    T* sH = sc.take<T>(DV * PK);    // H_n^T  [dv][dk]
+    T* sdH = sc.take<T>(DV * PK);   // dH'^T  [dv][dk]
     T* sM = sc.take<T>(64 * PL);
     float* sG = sc.take<float>(64 * 6);
     float* sGm1 = sG + 64;
@@ -288,7 +221,8 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     float* rowp = sc.take<float>(S::NROW * 2 * 64);
     float* colp = sc.take<float>(2 * 4 * 64);
     float* red = sc.take<float>(8);
-    // phase-B aliases: dO, E, dE and H are dead after phase A (64 x 64 fits in 64 x dv and dk x dv)
+    // P (for dE) lives where dW will go; phase-B aliases: dO, E, dE and H are dead after phase A
+    T* sP = sdW;
     T* sdPh = sdO;
     T* sdM = sE;
     T* sY = sdE;
@@ -301,9 +235,8 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     load_tile_async<T>(sV, PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
     load_tile_async<T>(sdO, PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
     load_tile_async<T>(sE, PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
-    load_tile_async<T>(sdE, PV, (const T*)p.dEb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
-    load_tile_async<T>(sH, PV, (const T*)p.Hb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
-    load_tile_async<T>(sdH, PV, (const T*)p.dHb + idx * DK * DV, DV, DK, DV, DK, tid, 256);
+    load_tile_async<T>(sH, PK, (const T*)p.Hb + idx * DV * DK, DK, DV, DK, DV, tid, 256);
+    load_tile_async<T>(sdH, PK, (const T*)p.dHb + idx * DV * DK, DK, DV, DK, DV, tid, 256);
     load_tile_async<T>(sM, PL, (const T*)p.Mb + idx * 4096, 64, 64, 64, 64, tid, 256);
     cp_async_commit();
     if (tid < 64) {
@@ -324,8 +257,8 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     {
         float s = 0.f;
         for (int e = tid; e < DK * DV; e += 256) {
-            const int r = e / DV, c = e % DV;
-            s += to_f(sH[r * PV + c]) * to_f(sdH[r * PV + c]);
+            const int r = e / DK, c = e % DK;
+            s += to_f(sH[r * PK + c]) * to_f(sdH[r * PK + c]);
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
@@ -342,13 +275,40 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         if ((lane & 3) == 0) { rowpart(kind)[ra] = s0; rowpart(kind)[rb] = s1; }
     };
 
+    // ---------------- dE = P^T dO + Kbar dH'  (P = Tril(Q~ K^T * Gamma))
+    {
+        float sc[4][4];
+        zero(sc);
+        warp_gemm<true, true, 4>(sc, sQ, PK, sK, PK, m0, 32 * wc, DK);
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = m0 + frag_row(i), c = 32 * wc + frag_col(t, i);
+                const float v = (c <= r && r < L) ? sc[t][i] * expf(sG[r] - sG[c]) : 0.f;
+                sP[r * PL + c] = from_f<T>(v);
+            }
+    }
+    __syncthreads();
+    {
+        const int nv0 = wc * (DV / 2);
+        float de[NV][4];
+        zero(de);
+        warp_gemm<true, true, NV>(de, sK, PK, sdH, PK, m0, nv0, DK);
+#pragma unroll
+        for (int t = 0; t < NV; ++t) { de[t][0] *= sKa; de[t][1] *= sKa; de[t][2] *= sKb; de[t][3] *= sKb; }
+        warp_gemm<false, false, NV>(de, sP, PL, sdO, PV, m0, nv0, 64);
+        frag_store<T, NV>(sdE, PV, m0, nv0, de);
+    }
+    __syncthreads();
+
     // ---------------- phase A: contractions over dv
     float acc_dq[NK][4], acc_dk[NK][4];
     const int nk0 = wc * (DK / 2);
     {
         // dQ~ part: Diag(gamma) dO H^T; its row dot with Q~ is the log-decay gradient of the Q~H term.
         zero(acc_dq);
-        warp_gemm<true, true, NK>(acc_dq, sdO, PV, sH, PV, m0, nk0, DV);
+        warp_gemm<true, false, NK>(acc_dq, sdO, PV, sH, PK, m0, nk0, DV);
         float t0r[NK][4];
 #pragma unroll
         for (int t = 0; t < NK; ++t) {
@@ -364,7 +324,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     {
         // dK from Kbar: Diag(gamma_C/gamma_r) E dH'^T
         zero(acc_dk);
-        warp_gemm<true, true, NK>(acc_dk, sE, PV, sdH, PV, m0, nk0, DV);
+        warp_gemm<true, false, NK>(acc_dk, sE, PV, sdH, PK, m0, nk0, DV);
         float t0r[NK][4];
 #pragma unroll
         for (int t = 0; t < NK; ++t) {
@@ -381,7 +341,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         // dW = -dE H^T
         float tmp[NK][4];
         zero(tmp);
-        warp_gemm<true, true, NK>(tmp, sdE, PV, sH, PV, m0, nk0, DV);
+        warp_gemm<true, false, NK>(tmp, sdE, PV, sH, PK, m0, nk0, DV);
 #pragma unroll
         for (int t = 0; t < NK; ++t)
 #pragma unroll
@@ -628,23 +588,28 @@ __global__ void __launch_bounds__(256) k_reduce_heads(ChunkParams p) {
 
 template <typename T, int DK, int DV>
 static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
-    const size_t sm_scan = ScanBwdSmem<T, DK>::bytes();
+    const size_t sm_prep = BPrepSmem<T, DK, DV>::bytes();
     const size_t sm_loc = LocalSmem<T, DK, DV>::bytes();
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(k_scan_bwd<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_scan)))
+    if ((e = cudaFuncSetAttribute(k_bwd_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
         return e;
     if ((e = cudaFuncSetAttribute(k_bwd_local<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_loc)))
         return e;
     mark(p, ev0, s);
-    k_scan_bwd<T, DK, DV><<<dim3((DV / 64) * p.N, p.H), 128, sm_scan, s>>>(p);
+    if (p.slots > 0) k_bwd_prep<T, DK, DV><<<dim3(p.slots, p.H), 128, sm_prep, s>>>(p);
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 1, s);
+    ScanArgs a;
+    a.H = p.H; a.N = p.N; a.T = p.T; a.slots = p.slots; a.Ttot = p.Ttot; a.cu = p.cu; a.seq_first = p.seq_first;
+    a.Gb = p.Gb; a.init = p.dhT; a.fin = p.dh0; a.Sout = p.dHb; a.X = p.ATb; a.Y = p.Cb; a.reverse = 1; a.err = p.err;
+    if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)p.slots * p.H, s))) return e;
+    mark(p, ev0 + 2, s);
     if (p.slots > 0) k_bwd_local<T, DK, DV><<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
     if ((e = cudaGetLastError())) return e;
-    mark(p, ev0 + 2, s);
+    mark(p, ev0 + 3, s);
     k_reduce_heads<<<p.H, 256, 0, s>>>(p);
     if ((e = cudaGetLastError())) return e;
-    mark(p, ev0 + 3, s);
+    mark(p, ev0 + 4, s);
     return cudaSuccess;
 }
 
@@ -662,7 +627,7 @@ cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int e
 
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
 #define COMBA_SM(T, DK, DV) \
-    if (dk == DK && dv == DV) return kernel == 0 ? ScanBwdSmem<T, DK>::bytes() : LocalSmem<T, DK, DV>::bytes();
+    if (dk == DK && dv == DV) return kernel == 0 ? BPrepSmem<T, DK, DV>::bytes() : LocalSmem<T, DK, DV>::bytes();
     if (is_bf16) {
         COMBA_SM(bf16, 128, 128) COMBA_SM(bf16, 128, 64) COMBA_SM(bf16, 64, 128) COMBA_SM(bf16, 64, 64)
     } else {

@@ -1,13 +1,14 @@
 // Chunk-parallel Comba forward (section 3.3 of the paper):
 //   k_chunk_map : chunk slots of (packed) sequences
-//   k_prep      : per chunk, Gram matrix, UT inverse M by forward substitution,
-//                 WY factors W = M Diag(btilde gamma_{r-1}) K, U = M Diag(beta) V
-//                 (Eq. "prepare WY_M")
-//   k_scan_fwd  : per (sequence, head, 64-column tile of dv), sequential over
-//                 chunks: E = U - W H, H <- gamma_C H + Kbar^T E (inter-chunk
-//                 state equation)
-//   k_output    : per chunk, O = Diag(gamma) Q~ H + Tril(Q~ K^T * Gamma) E
-//                 (output equation with Q~ = Q - d K)
+//   k_prep      : per chunk, the decay-masked btilde-scaled Gram matrix, its
+//                 UT inverse M, the WY factors W = M Diag(btilde gamma_{r-1}) K
+//                 and U = M Diag(beta) V (Eq. "prepare WY_M"), and the chunk's
+//                 affine state map H -> gamma_C H + Atilde H + B with
+//                 Atilde = -Kbar^T W, B = Kbar^T U (the inter-chunk state
+//                 equation with Kbar = Diag(gamma_C / gamma_r) K)
+//   (scan.cu)   : the sequential scan of those maps
+//   k_output    : per chunk, E = U - W H_n and the output equation
+//                 O = Diag(gamma) Q~ H_n + Tril(Q~ K^T * Gamma) E, Q~ = Q - d K
 #include "params.cuh"
 
 namespace comba {
@@ -21,7 +22,10 @@ __global__ void __launch_bounds__(1024) k_chunk_map(ChunkParams p) {
     __shared__ int carry;
     __shared__ int wsum[32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    if (tid == 0) carry = 0;
+    if (tid == 0) {
+        carry = 0;
+        if (p.err) *p.err = 0;
+    }
     __syncthreads();
     for (int base = 0; base < p.N; base += 1024) {
         const int n = base + tid;
@@ -108,19 +112,38 @@ __device__ __forceinline__ void frag_store_global(T* g, long long ld, int m0, in
 template <typename T, int DK, int DV>
 struct PrepSmem {
     static constexpr int PK = pitch<T>(DK), PV = pitch<T>(DV), PL = pitch<T>(64);
-    static constexpr size_t bytes() {
-        size_t o = 0;
-        o = carve_bytes(o, sizeof(T) * 64 * PK);
-        o = carve_bytes(o, sizeof(T) * 64 * PV);
-        o = carve_bytes(o, sizeof(float) * 64 * 65);
-        o = carve_bytes(o, sizeof(float) * 64 * 65);
-        o = carve_bytes(o, sizeof(float) * 3 * 272);
-        o = carve_bytes(o, sizeof(T) * 64 * PL);
-        o = carve_bytes(o, sizeof(T) * 64 * PL);
-        for (int i = 0; i < 4; ++i) o = carve_bytes(o, sizeof(float) * 64);
-        return o;
-    }
+    static constexpr size_t RA = sizeof(float) * 64 * 65 > sizeof(T) * 64 * PK ? sizeof(float) * 64 * 65
+                                                                                 : sizeof(T) * 64 * PK;
+    static constexpr size_t RM = sizeof(float) * 64 * 65 > sizeof(T) * 64 * PV ? sizeof(float) * 64 * 65
+                                                                                 : sizeof(T) * 64 * PV;
+    static constexpr size_t OK = 0;
+    static constexpr size_t OV = align128(OK + sizeof(T) * 64 * PK);
+    static constexpr size_t OA = align128(OV + sizeof(T) * 64 * PV);   // A (fp32), later Diag(s) W
+    static constexpr size_t OM = align128(OA + RA);                    // M (fp32), later Diag(s) U
+    static constexpr size_t OT = align128(OM + RM);                    // inverse scratch
+    static constexpr size_t OMW = align128(OT + sizeof(float) * 3 * 272);
+    static constexpr size_t OMU = align128(OMW + sizeof(T) * 64 * PL);
+    static constexpr size_t OF = align128(OMU + sizeof(T) * 64 * PL);  // G, Gm1, btilde, beta, s
+    static constexpr size_t bytes() { return OF + sizeof(float) * 64 * 5; }
 };
+
+// Store a [rows x cols] product computed in 16-row m-tiles and 64-column passes.
+template <typename T, bool AK, bool BK, int ROWS, int COLS>
+__device__ __forceinline__ void gemm_to_global(T* g, const T* sA, int lda, const T* sB, int ldb, int K, float sign,
+                                               int warp) {
+    constexpr int MT = ROWS / 64;  // m-tiles per warp (4 warps)
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+        const int m0 = (warp * MT + mt) * 16;
+#pragma unroll
+        for (int n0 = 0; n0 < COLS; n0 += 64) {
+            float acc[8][4];
+            zero(acc);
+            warp_gemm<AK, BK, 8>(acc, sA, lda, sB, ldb, m0, n0, K);
+            frag_store_global<T, 8>(g, COLS, m0, n0, acc, ROWS, sign);
+        }
+    }
+}
 
 template <typename T, int DK, int DV>
 __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
@@ -134,18 +157,20 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     const int tid = threadIdx.x, warp = tid >> 5;
 
     extern __shared__ __align__(128) char smem[];
-    SmemCarver sc(smem);
-    T* sK = sc.take<T>(64 * S::PK);
-    T* sV = sc.take<T>(64 * S::PV);
-    float* sA = sc.take<float>(64 * 65);
-    float* sM = sc.take<float>(64 * 65);
-    float* sTmp = sc.take<float>(3 * 272);
-    T* sMw = sc.take<T>(64 * S::PL);
-    T* sMu = sc.take<T>(64 * S::PL);
-    float* sG = sc.take<float>(64);
-    float* sGm1 = sc.take<float>(64);
-    float* sBt = sc.take<float>(64);
-    float* sBe = sc.take<float>(64);
+    T* sK = reinterpret_cast<T*>(smem + S::OK);
+    T* sV = reinterpret_cast<T*>(smem + S::OV);
+    float* sA = reinterpret_cast<float*>(smem + S::OA);
+    float* sM = reinterpret_cast<float*>(smem + S::OM);
+    T* sWs = reinterpret_cast<T*>(smem + S::OA);
+    T* sUs = reinterpret_cast<T*>(smem + S::OM);
+    float* sTmp = reinterpret_cast<float*>(smem + S::OT);
+    T* sMw = reinterpret_cast<T*>(smem + S::OMW);
+    T* sMu = reinterpret_cast<T*>(smem + S::OMU);
+    float* sG = reinterpret_cast<float*>(smem + S::OF);
+    float* sGm1 = sG + 64;
+    float* sBt = sG + 128;
+    float* sBe = sG + 192;
+    float* sS = sG + 256;
 
     load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
     load_tile_async<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
@@ -158,6 +183,7 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     }
     cp_async_wait<0>();
     __syncthreads();
+    if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;   // Kbar row scale gamma_C / gamma_r
 
     // Strictly-lower A = Diag(btilde) (gamma_{r-1}/gamma_i * K K^T); exp taken only below the diagonal.
     {
@@ -189,157 +215,33 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     if (tid < 64) p.Gb[idx * 64 + tid] = sG[tid];
     __syncthreads();
 
+    // W, U (stored) and their Kbar-row-scaled copies for the chunk's state map.
+    const float sa = sS[16 * warp + frag_row(0)], sb = sS[16 * warp + frag_row(2)];
     {
         float acc[DK / 8][4];
         zero(acc);
         warp_gemm<true, false, DK / 8>(acc, sMw, S::PL, sK, S::PK, 16 * warp, 0, 64);
         frag_store_global<T, DK / 8>((T*)p.Wb + idx * 64 * DK, DK, 16 * warp, 0, acc, 64);
+#pragma unroll
+        for (int t = 0; t < DK / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
+        frag_store<T, DK / 8>(sWs, S::PK, 16 * warp, 0, acc);
     }
     {
         float acc[DV / 8][4];
         zero(acc);
         warp_gemm<true, false, DV / 8>(acc, sMu, S::PL, sV, S::PV, 16 * warp, 0, 64);
         frag_store_global<T, DV / 8>((T*)p.Ub + idx * 64 * DV, DV, 16 * warp, 0, acc, 64);
+#pragma unroll
+        for (int t = 0; t < DV / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
+        frag_store<T, DV / 8>(sUs, S::PV, 16 * warp, 0, acc);
     }
-}
+    __syncthreads();
 
-// ------------------------------------------------------------- state scan
-
-template <typename T, int DK>
-struct ScanSmem {
-    static constexpr int PK = pitch<T>(DK), PT = pitch<T>(64);
-    // per pipeline stage: W, K, U tile, G
-    static constexpr size_t OW = 0;
-    static constexpr size_t OK = align128(OW + sizeof(T) * 64 * PK);
-    static constexpr size_t OU = align128(OK + sizeof(T) * 64 * PK);
-    static constexpr size_t OG = align128(OU + sizeof(T) * 64 * PT);
-    static constexpr size_t STAGE = align128(OG + sizeof(float) * 64);
-    static constexpr size_t OH = 2 * STAGE;                                  // H tile (storage type)
-    static constexpr size_t OE = align128(OH + sizeof(T) * DK * PT);         // scaled E tile
-    static constexpr size_t bytes() { return OE + sizeof(T) * 64 * PT; }
-};
-
-__device__ __forceinline__ void seq_range(const ChunkParams& p, int n, long long& start, long long& len) {
-    long long a = p.cu ? p.cu[n] : (long long)n * p.T;
-    long long e = p.cu ? p.cu[n + 1] : (long long)(n + 1) * p.T;
-    a = a < 0 ? 0 : (a > p.Ttot ? p.Ttot : a);
-    e = e < a ? a : (e > p.Ttot ? p.Ttot : e);
-    start = a;
-    len = e - a;
-}
-
-// The sequential inter-chunk recurrence: E_n = U_n - W_n H_n, H_{n+1} = gamma_C H_n + Kbar_n^T E_n.
-// One CTA owns a 64-column tile of H (fp32, in registers) for one (sequence, head); the
-// next chunk's W, K, U tile and log-decays are prefetched while the current chunk computes.
-template <typename T, int DK, int DV>
-__global__ void __launch_bounds__(128) k_scan_fwd(ChunkParams p) {
-    using S = ScanSmem<T, DK>;
-    constexpr int MT = DK / 64;  // 16-row m-tiles per warp
-    const int jt = blockIdx.x % (DV / 64), n = blockIdx.x / (DV / 64), h = blockIdx.y;
-    const int tid = threadIdx.x, warp = tid >> 5;
-    const int c0 = jt * 64;
-
-    extern __shared__ __align__(128) char smem[];
-    auto sW = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OW); };
-    auto sK = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OK); };
-    auto sU = [&](int st) { return reinterpret_cast<T*>(smem + st * S::STAGE + S::OU); };
-    auto sG = [&](int st) { return reinterpret_cast<float*>(smem + st * S::STAGE + S::OG); };
-    T* sH = reinterpret_cast<T*>(smem + S::OH);
-    T* sE = reinterpret_cast<T*>(smem + S::OE);
-
-    float hs[MT][8][4];
-    const float* h0 = p.h0 ? p.h0 + ((long long)n * p.H + h) * DK * DV : nullptr;
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-        for (int t = 0; t < 8; ++t)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = (warp * MT + mt) * 16 + frag_row(i), c = c0 + frag_col(t, i);
-                hs[mt][t][i] = h0 ? h0[(long long)r * DV + c] : 0.f;
-            }
-
-    long long start, len;
-    seq_range(p, n, start, len);
-    const int s0 = p.seq_first[n];
-    int nch = (int)((len + kChunk - 1) / kChunk);
-    if (s0 + nch > p.slots) nch = p.slots - s0 > 0 ? p.slots - s0 : 0;
-
-    auto issue = [&](int c, int st) {
-        const long long idx = (long long)(s0 + c) * p.H + h;
-        const long long t0 = start + (long long)c * kChunk;
-        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
-        load_tile_async<T>(sW(st), S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
-        load_tile_async<T>(sK(st), S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid,
-                           128);
-        load_tile_async<T>(sU(st), S::PT, (const T*)p.Ub + idx * 64 * DV + c0, DV, 64, 64, 64, tid, 128);
-        if (tid < 16) cp_async16(sG(st) + 4 * tid, p.Gb + idx * 64 + 4 * tid, true);
-        cp_async_commit();
-    };
-    if (nch > 0) issue(0, 0);
-
-    for (int c = 0; c < nch; ++c) {
-        const int st = c & 1;
-        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
-        const long long idx = (long long)(s0 + c) * p.H + h;
-        if (c + 1 < nch) {
-            issue(c + 1, st ^ 1);
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            const int m0 = (warp * MT + mt) * 16;
-            frag_store<T, 8>(sH, S::PT, m0, 0, hs[mt]);
-            frag_store_global<T, 8>((T*)p.Hb + idx * DK * DV + c0, DV, m0, 0, hs[mt], DK);
-        }
-        __syncthreads();
-
-        const float* G = sG(st);
-        const float gL = G[L - 1];
-        {
-            float e[8][4];
-            zero(e);
-            warp_gemm<true, false, 8>(e, sW(st), S::PK, sH, S::PT, 16 * warp, 0, DK);
-            T* Eg = (T*)p.Eb + idx * 64 * DV + c0;
-            const T* U = sU(st);
-#pragma unroll
-            for (int t = 0; t < 8; ++t)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int r = 16 * warp + frag_row(i), cc = frag_col(t, i);
-                    const float ev = to_f(U[r * S::PT + cc]) - e[t][i];
-                    Eg[(long long)r * DV + cc] = from_f<T>(ev);
-                    sE[r * S::PT + cc] = from_f<T>(r < L ? ev * expf(gL - G[r]) : 0.f);
-                }
-        }
-        __syncthreads();
-
-        const float dec = expf(gL);
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-#pragma unroll
-            for (int t = 0; t < 8; ++t)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) hs[mt][t][i] *= dec;
-            warp_gemm<false, false, 8>(hs[mt], sK(st), S::PK, sE, S::PT, (warp * MT + mt) * 16, 0, 64);
-        }
-        __syncthreads();
-    }
-
-    if (p.hT) {
-        float* hT = p.hT + ((long long)n * p.H + h) * DK * DV;
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-            for (int t = 0; t < 8; ++t)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int r = (warp * MT + mt) * 16 + frag_row(i), cc = c0 + frag_col(t, i);
-                    hT[(long long)r * DV + cc] = hs[mt][t][i];
-                }
-    }
+    // Atilde = -K^T Diag(s) W  [dk][dk];  B^T = (Diag(s) U)^T K  [dv][dk];  Atilde^T = -(Diag(s) W)^T K.
+    gemm_to_global<T, false, false, DK, DK>((T*)p.Ab + idx * DK * DK, sK, S::PK, sWs, S::PK, 64, -1.f, warp);
+    gemm_to_global<T, false, false, DV, DK>((T*)p.Bb + idx * DV * DK, sUs, S::PV, sK, S::PK, 64, 1.f, warp);
+    if (p.ATb)
+        gemm_to_global<T, false, false, DK, DK>((T*)p.ATb + idx * DK * DK, sWs, S::PK, sK, S::PK, 64, -1.f, warp);
 }
 
 // ---------------------------------------------------------------- output
@@ -347,16 +249,13 @@ __global__ void __launch_bounds__(128) k_scan_fwd(ChunkParams p) {
 template <typename T, int DK, int DV>
 struct OutSmem {
     static constexpr int PK = pitch<T>(DK), PV = pitch<T>(DV), PL = pitch<T>(64);
-    static constexpr size_t bytes() {
-        size_t o = 0;
-        o = carve_bytes(o, sizeof(T) * 64 * PK);   // Q~
-        o = carve_bytes(o, sizeof(T) * 64 * PK);   // K
-        o = carve_bytes(o, sizeof(T) * 64 * PL);   // P
-        o = carve_bytes(o, sizeof(T) * DK * PV);   // H
-        o = carve_bytes(o, sizeof(T) * 64 * PV);   // E
-        o = carve_bytes(o, sizeof(float) * 64);    // G
-        return o;
-    }
+    static constexpr size_t OQ = 0;                                          // Q~
+    static constexpr size_t OK = align128(OQ + sizeof(T) * 64 * PK);         // K
+    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);         // W, later P
+    static constexpr size_t OU = align128(OW + sizeof(T) * 64 * PK);         // U, later E
+    static constexpr size_t OH = align128(OU + sizeof(T) * 64 * PV);         // H^T [dv][dk]
+    static constexpr size_t OG = align128(OH + sizeof(T) * DV * PK);
+    static constexpr size_t bytes() { return OG + sizeof(float) * 64; }
 };
 
 template <typename T, int DK, int DV>
@@ -371,39 +270,58 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     const int tid = threadIdx.x, warp = tid >> 5;
 
     extern __shared__ __align__(128) char smem[];
-    SmemCarver sc(smem);
-    T* sQ = sc.take<T>(64 * S::PK);
-    T* sK = sc.take<T>(64 * S::PK);
-    T* sP = sc.take<T>(64 * S::PL);
-    T* sH = sc.take<T>(DK * S::PV);
-    T* sE = sc.take<T>(64 * S::PV);
-    float* sG = sc.take<float>(64);
+    T* sQ = reinterpret_cast<T*>(smem + S::OQ);
+    T* sK = reinterpret_cast<T*>(smem + S::OK);
+    T* sW = reinterpret_cast<T*>(smem + S::OW);
+    T* sP = sW;
+    T* sU = reinterpret_cast<T*>(smem + S::OU);
+    T* sE = sU;
+    T* sH = reinterpret_cast<T*>(smem + S::OH);
+    float* sG = reinterpret_cast<float*>(smem + S::OG);
 
     load_tile_async<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
     load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-    load_tile_async<T>(sH, S::PV, (const T*)p.Hb + idx * DK * DV, DV, DK, DV, DK, tid, 128);
-    load_tile_async<T>(sE, S::PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 128);
+    load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
+    load_tile_async<T>(sU, S::PV, (const T*)p.Ub + idx * 64 * DV, DV, 64, DV, 64, tid, 128);
+    load_tile_async<T>(sH, S::PK, (const T*)p.Hb + idx * DV * DK, DK, DV, DK, DV, tid, 128);
     cp_async_commit();
     if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
     cp_async_wait<0>();
     __syncthreads();
+
+    // E = U - W H  (B operand H[c][j] read from H^T[j][c]); E replaces U in shared memory.
+    {
+        float e[DV / 8][4];
+        zero(e);
+        warp_gemm<true, true, DV / 8>(e, sW, S::PK, sH, S::PK, 16 * warp, 0, DK);
+#pragma unroll
+        for (int t = 0; t < DV / 8; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
+                e[t][i] = to_f(sU[r * S::PV + c]) - e[t][i];
+            }
+        if (p.Eb) frag_store_global<T, DV / 8>((T*)p.Eb + idx * 64 * DV, DV, 16 * warp, 0, e, 64);
+        frag_store<T, DV / 8>(sE, S::PV, 16 * warp, 0, e);
+    }
     const float dh = p.d[h];
     for (int e = tid; e < 64 * DK; e += 128) {
         const int r = e / DK, c = e % DK;
         sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dh * to_f(sK[r * S::PK + c]));
     }
     __syncthreads();
+    if (!p.o) return;
 
     {
-        float s[8][4];
-        zero(s);
-        warp_gemm<true, true, 8>(s, sQ, S::PK, sK, S::PK, 16 * warp, 0, DK);
+        float sc[8][4];
+        zero(sc);
+        warp_gemm<true, true, 8>(sc, sQ, S::PK, sK, S::PK, 16 * warp, 0, DK);
 #pragma unroll
         for (int t = 0; t < 8; ++t)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
-                const float v = (c <= r && r < L) ? s[t][i] * expf(sG[r] - sG[c]) : 0.f;
+                const float v = (c <= r && r < L) ? sc[t][i] * expf(sG[r] - sG[c]) : 0.f;
                 sP[r * S::PL + c] = from_f<T>(v);
             }
     }
@@ -411,7 +329,7 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
 
     float o[DV / 8][4];
     zero(o);
-    warp_gemm<true, false, DV / 8>(o, sQ, S::PK, sH, S::PV, 16 * warp, 0, DK);
+    warp_gemm<true, true, DV / 8>(o, sQ, S::PK, sH, S::PK, 16 * warp, 0, DK);
     {
         const float e0 = expf(sG[16 * warp + frag_row(0)]);
         const float e1 = expf(sG[16 * warp + frag_row(2)]);
@@ -428,29 +346,28 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
 // -------------------------------------------------------------- launchers
 
 template <typename T, int DK, int DV>
-static cudaError_t run_fwd(const ChunkParams& p, bool for_backward, cudaStream_t s, int ev0) {
+static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int ev0) {
     const size_t sm_prep = PrepSmem<T, DK, DV>::bytes();
-    const size_t sm_scan = ScanSmem<T, DK>::bytes();
     const size_t sm_out = OutSmem<T, DK, DV>::bytes();
     cudaError_t e;
     if ((e = cudaFuncSetAttribute(k_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
         return e;
-    if ((e = cudaFuncSetAttribute(k_scan_fwd<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_scan)))
-        return e;
     if ((e = cudaFuncSetAttribute(k_output<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out)))
         return e;
-    mark(p, ev0, s);
-    if (p.slots > 0) k_prep<T, DK, DV><<<dim3(p.slots, p.H), 128, sm_prep, s>>>(p);
+    ChunkParams q = p;
+    if (!save) { q.Mb = nullptr; q.ATb = nullptr; q.Eb = nullptr; }
+    mark(q, ev0, s);
+    if (q.slots > 0) k_prep<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_prep, s>>>(q);
     if ((e = cudaGetLastError())) return e;
-    mark(p, ev0 + 1, s);
-    k_scan_fwd<T, DK, DV><<<dim3((DV / 64) * p.N, p.H), 128, sm_scan, s>>>(p);
+    mark(q, ev0 + 1, s);
+    ScanArgs a;
+    a.H = q.H; a.N = q.N; a.T = q.T; a.slots = q.slots; a.Ttot = q.Ttot; a.cu = q.cu; a.seq_first = q.seq_first;
+    a.Gb = q.Gb; a.init = q.h0; a.fin = q.hT; a.Sout = q.Hb; a.X = q.Ab; a.Y = q.Bb; a.reverse = 0; a.err = q.err;
+    if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)q.slots * q.H, s))) return e;
+    mark(q, ev0 + 2, s);
+    if (q.slots > 0 && (q.o || q.Eb)) k_output<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_out, s>>>(q);
     if ((e = cudaGetLastError())) return e;
-    if (!for_backward) {
-        mark(p, ev0 + 2, s);
-        if (p.slots > 0) k_output<T, DK, DV><<<dim3(p.slots, p.H), 128, sm_out, s>>>(p);
-        if ((e = cudaGetLastError())) return e;
-        mark(p, ev0 + 3, s);
-    }
+    mark(q, ev0 + 3, s);
     return cudaSuccess;
 }
 
@@ -459,26 +376,22 @@ cudaError_t launch_chunk_map(const ChunkParams& p, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool for_backward, cudaStream_t s, int ev0) {
+cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream_t s, int ev0) {
+#define COMBA_FWD(T, DK, DV) \
+    if (p.dk == DK && p.dv == DV) return run_fwd<T, DK, DV>(p, save, s, ev0);
     if (is_bf16) {
-        if (p.dk == 128 && p.dv == 128) return run_fwd<bf16, 128, 128>(p, for_backward, s, ev0);
-        if (p.dk == 128 && p.dv == 64) return run_fwd<bf16, 128, 64>(p, for_backward, s, ev0);
-        if (p.dk == 64 && p.dv == 128) return run_fwd<bf16, 64, 128>(p, for_backward, s, ev0);
-        if (p.dk == 64 && p.dv == 64) return run_fwd<bf16, 64, 64>(p, for_backward, s, ev0);
+        COMBA_FWD(bf16, 128, 128) COMBA_FWD(bf16, 128, 64) COMBA_FWD(bf16, 64, 128) COMBA_FWD(bf16, 64, 64)
     } else {
-        if (p.dk == 128 && p.dv == 128) return run_fwd<float, 128, 128>(p, for_backward, s, ev0);
-        if (p.dk == 128 && p.dv == 64) return run_fwd<float, 128, 64>(p, for_backward, s, ev0);
-        if (p.dk == 64 && p.dv == 128) return run_fwd<float, 64, 128>(p, for_backward, s, ev0);
-        if (p.dk == 64 && p.dv == 64) return run_fwd<float, 64, 64>(p, for_backward, s, ev0);
+        COMBA_FWD(float, 128, 128) COMBA_FWD(float, 128, 64) COMBA_FWD(float, 64, 128) COMBA_FWD(float, 64, 64)
     }
+#undef COMBA_FWD
     return cudaErrorInvalidValue;
 }
 
 size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
-#define COMBA_SM(T, DK, DV)                                                                          \
-    if (dk == DK && dv == DV)                                                                        \
-        return kernel == 0 ? PrepSmem<T, DK, DV>::bytes()                                            \
-                           : (kernel == 1 ? ScanSmem<T, DK>::bytes() : OutSmem<T, DK, DV>::bytes());
+    if (kernel == 1) return scan_smem_bytes(is_bf16, dk, dv);
+#define COMBA_SM(T, DK, DV) \
+    if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes() : OutSmem<T, DK, DV>::bytes();
     if (is_bf16) {
         COMBA_SM(bf16, 128, 128) COMBA_SM(bf16, 128, 64) COMBA_SM(bf16, 64, 128) COMBA_SM(bf16, 64, 64)
     } else {

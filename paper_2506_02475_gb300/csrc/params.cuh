@@ -42,15 +42,19 @@ struct ChunkParams {
     // workspace views (per (slot, head) pair idx = slot*H + h)
     SlotInfo* slot_info;     // [slots]
     int* seq_first;          // [N+1] first slot of each sequence
-    void* Wb;                // [pairs][64][dk]  storage type
-    void* Ub;                // [pairs][64][dv]
+    void* Wb;                // [pairs][64][dk]  WY factor W (storage type)
+    void* Ub;                // [pairs][64][dv]  WY factor U
     float* Gb;               // [pairs][64]      chunk-local log-cumsum of alpha
-    void* Mb;                // [pairs][64][64]  UT inverse, storage type (backward only)
-    void* Hb;                // [pairs][dk][dv]  state at chunk start (storage type)
-    void* Eb;                // [pairs][64][dv]  U - W H
-    void* dHb;               // [pairs][dk][dv]  dL/dH at chunk end
-    void* dEb;               // [pairs][64][dv]
+    void* Ab;                // [pairs][dk][dk]  Atilde = -Kbar^T W (forward scan operand)
+    void* Bb;                // [pairs][dv][dk]  (Kbar^T U)^T (forward scan additive term)
+    void* Hb;                // [pairs][dv][dk]  chunk-start state, transposed
+    void* Eb;                // [pairs][64][dv]  E = U - W H (saved for the backward)
+    void* Mb;                // [pairs][64][64]  UT inverse M (saved for the backward)
+    void* ATb;               // [pairs][dk][dk]  Atilde^T (backward scan operand)
+    void* Cb;                // [pairs][dv][dk]  ((Qhat - P W)^T dO)^T (backward scan additive term)
+    void* dHb;               // [pairs][dv][dk]  dL/dH at chunk end, transposed
     float* part;             // [pairs][2]       per-chunk db, dd partial sums
+    int* err;                // device status word (nonzero: a bounded wait gave up)
 
     // optional stage-boundary events (instrumentation)
     cudaEvent_t* ev;
@@ -62,12 +66,33 @@ inline void mark(const ChunkParams& p, int i, cudaStream_t s) {
     if (p.ev && i < p.nev) cudaEventRecord(p.ev[i], s);
 }
 
+// Arguments of the sequential scan S^T <- gamma S^T + S^T X^T + Y (see scan.cu).
+struct ScanArgs {
+    int H, N, T, slots;
+    long long Ttot;
+    const int32_t* cu;
+    const int* seq_first;
+    const float* Gb;         // chunk log-decays: gamma_n = exp(G[L-1])
+    const float* init;       // [N,H,dk,dv] initial state (h0 or dhT) or null
+    float* fin;              // [N,H,dk,dv] final state (hT or dh0) or null
+    void* Sout;              // [pairs][dv][dk] state each chunk starts from (storage type)
+    const void* X;           // [pairs][dk][dk] row-major
+    const void* Y;           // [pairs][dv][dk]
+    int reverse;
+    int* err;
+};
+cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s);
+size_t scan_smem_bytes(bool is_bf16, int dk, int dv);
+
 // Kernel launchers (one translation unit each); return cudaGetLastError().
 cudaError_t launch_chunk_map(const ChunkParams& p, cudaStream_t s);
-// Stage events: launch_fwd marks ev0 before prep, ev0+1 before the scan, ev0+2 before the
-// output (forward only) and ev0+3 after the last kernel; launch_bwd marks ev0 before the
-// reverse scan, ev0+1 before the local gradients, ev0+2 before the head reduction, ev0+3 after.
-cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool for_backward, cudaStream_t s, int ev0);
+// Forward kernels: prep (W, U, G, Atilde, B^T; M and Atilde^T when `save`), the scan,
+// and the output kernel (O when p.o is set; E when `save`).  Stage events: ev0 before
+// prep, ev0+1 before the scan, ev0+2 before the output, ev0+3 after it.
+cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream_t s, int ev0);
+// Backward kernels given the saved factors: C^T, the reverse scan, local gradients and
+// the head reduction.  Stage events: ev0 before C^T, ev0+1 before the scan, ev0+2 before
+// the local gradients, ev0+3 before the reduction, ev0+4 after it.
 cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int ev0);
 size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);

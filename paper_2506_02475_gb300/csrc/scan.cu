@@ -1,0 +1,340 @@
+// Sequential inter-chunk scan, shared by the forward and the backward.
+//
+// Folding each chunk of section 3.3's state equation into one affine map,
+//     H_{n+1} = gamma_n H_n + Atilde_n H_n + B_n,
+//     Atilde_n = -Kbar_n^T W_n,  B_n = Kbar_n^T U_n,  gamma_n = gamma_C of chunk n,
+// leaves a single dense product on the sequential path.  The backward's
+// reverse recurrence has the same form,
+//     dH_n = gamma_n dH_{n+1} + Atilde_n^T dH_{n+1} + C_n,  C_n = (Qhat_n - P_n W_n)^T dO_n.
+// Both are evaluated transposed, one state row (a dv index) per thread:
+//     S^T <- gamma S^T + S^T X^T + Y,
+// with X = Atilde (forward) or Atilde^T (backward) stored [dk][dk] row-major,
+// and Y = B^T or C^T stored [dv][dk].  Each chunk stores the state it started
+// from (H_n^T, or dH_{n+1}^T in the backward) for the parallel kernels.
+//
+// bf16 storage: one CTA per (sequence, head), 128 threads; the fp32 state row
+// stays in registers; S^T (bf16) is written into a 128-byte-swizzled K-major
+// shared tile; X and Y stream in by TMA through a multi-stage mbarrier
+// pipeline; one thread issues the tcgen05 MMAs (M = 128, N = dk, K = dk)
+// into a TMEM accumulator that all threads read back with tcgen05.ld.
+// fp32 storage: the same recurrence with FMA tile products (tolerance 1e-4).
+#include <cuda.h>
+
+#include "params.cuh"
+
+namespace comba {
+
+__device__ __forceinline__ void scan_seq_range(const ScanArgs& a, int n, long long& start, long long& len) {
+    long long s = a.cu ? a.cu[n] : (long long)n * a.T;
+    long long e = a.cu ? a.cu[n + 1] : (long long)(n + 1) * a.T;
+    s = s < 0 ? 0 : (s > a.Ttot ? a.Ttot : s);
+    e = e < s ? s : (e > a.Ttot ? a.Ttot : e);
+    start = s;
+    len = e - s;
+}
+
+// ------------------------------------------------------------ tcgen05 path
+
+template <int DK, int DV>
+struct ScanTcSmem {
+    static constexpr int STAGES = DK == 128 ? 3 : 4;
+    static constexpr uint32_t A_BYTES = 128 * DK * 2;   // S^T tile, M = 128 rows (rows >= DV are zero)
+    static constexpr uint32_t X_BYTES = DK * DK * 2;
+    static constexpr uint32_t Y_BYTES = DV * DK * 2;
+    static constexpr uint32_t STAGE = X_BYTES + Y_BYTES;
+    static constexpr size_t bytes() { return 1024 + A_BYTES + STAGES * (size_t)STAGE; }
+};
+
+template <int DK, int DV>
+__global__ void __launch_bounds__(128, 1)
+    k_scan_tc(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY) {
+    using S = ScanTcSmem<DK, DV>;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t full_bar[S::STAGES];
+    __shared__ uint64_t mma_bar;
+    __shared__ uint32_t tmem_base;
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int n = blockIdx.x, h = blockIdx.y;
+    const int j = tid;  // state row (dv index)
+    const bool live = j < DV;
+    uint8_t* sA = smem;
+    const uint32_t sA_u = smem_u32(sA);
+
+    float st[DK];
+    const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
+#pragma unroll
+    for (int m = 0; m < DK; ++m) st[m] = (init && live) ? init[(long long)m * DV + j] : 0.f;
+
+    long long start, len;
+    scan_seq_range(a, n, start, len);
+    const int s0 = a.seq_first[n];
+    int nch = (int)((len + kChunk - 1) / kChunk);
+    if (s0 + nch > a.slots) nch = a.slots - s0 > 0 ? a.slots - s0 : 0;
+
+    if (tid == 0) {
+        for (int s = 0; s < S::STAGES; ++s) mbar_init(smem_u32(&full_bar[s]), 1);
+        mbar_init(smem_u32(&mma_bar), 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&tmem_base), DK);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    auto chunk_of = [&](int it) { return a.reverse ? nch - 1 - it : it; };
+    auto stage_x = [&](int s) { return sA_u + S::A_BYTES + s * S::STAGE; };
+    auto stage_y = [&](int s) { return sA_u + S::A_BYTES + s * S::STAGE + S::X_BYTES; };
+    auto issue = [&](int it) {
+        const int s = it % S::STAGES;
+        const long long idx = (long long)(s0 + chunk_of(it)) * a.H + h;
+        const uint32_t fb = smem_u32(&full_bar[s]);
+        mbar_expect_tx(fb, S::STAGE);
+#pragma unroll
+        for (int half = 0; half < DK / 64; ++half) {
+            tma_load_2d(stage_x(s) + half * DK * 128, &tmX, half * 64, (int)(idx * DK), fb);
+            tma_load_2d(stage_y(s) + half * DV * 128, &tmY, half * 64, (int)(idx * DV), fb);
+        }
+    };
+    if (tid == 0)
+        for (int it = 0; it < S::STAGES - 1 && it < nch; ++it) issue(it);
+
+    constexpr uint32_t idesc = idesc_bf16_f32(128, DK);
+    for (int it = 0; it < nch; ++it) {
+        const int c = chunk_of(it), s = it % S::STAGES;
+        const long long idx = (long long)(s0 + c) * a.H + h;
+        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+        const float gam = expf(a.Gb[idx * 64 + L - 1]);
+
+        // The state this chunk starts from: A operand (bf16, swizzled) and per-chunk output.
+        bf16* out = reinterpret_cast<bf16*>(a.Sout) + (idx * DV + j) * DK;
+#pragma unroll
+        for (int q = 0; q < DK / 8; ++q) {
+            __nv_bfloat162 v0 = __floats2bfloat162_rn(st[8 * q + 0], st[8 * q + 1]);
+            __nv_bfloat162 v1 = __floats2bfloat162_rn(st[8 * q + 2], st[8 * q + 3]);
+            __nv_bfloat162 v2 = __floats2bfloat162_rn(st[8 * q + 4], st[8 * q + 5]);
+            __nv_bfloat162 v3 = __floats2bfloat162_rn(st[8 * q + 6], st[8 * q + 7]);
+            uint4 pk;
+            pk.x = *reinterpret_cast<uint32_t*>(&v0);
+            pk.y = *reinterpret_cast<uint32_t*>(&v1);
+            pk.z = *reinterpret_cast<uint32_t*>(&v2);
+            pk.w = *reinterpret_cast<uint32_t*>(&v3);
+            *reinterpret_cast<uint4*>(sA + sw128_offset(j, 8 * q, 128)) = pk;
+            if (live) *reinterpret_cast<uint4*>(out + 8 * q) = pk;
+        }
+        fence_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+
+        int bad = 0;
+        if (tid == 0) {
+            // Refill the stage that chunk it-1 used (everyone is past its epilogue now).
+            if (it + S::STAGES - 1 < nch) issue(it + S::STAGES - 1);
+            if (mbar_wait(smem_u32(&full_bar[s]), (it / S::STAGES) & 1)) {
+#pragma unroll
+                for (int ks = 0; ks < DK / 16; ++ks) {
+                    const int half = ks >> 2, sub = ks & 3;
+                    const uint64_t ad = smem_desc_sw128(sA_u + half * 128 * 128 + sub * 32);
+                    const uint64_t bd = smem_desc_sw128(stage_x(s) + half * DK * 128 + sub * 32);
+                    tc_mma_bf16(tmem, ad, bd, idesc, ks > 0 ? 1u : 0u);
+                }
+            } else {
+                bad = 1;
+            }
+            tc_commit(smem_u32(&mma_bar));
+        }
+        if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
+        if (!mbar_wait(smem_u32(&full_bar[s]), (it / S::STAGES) & 1)) bad = 1;
+        if (__syncthreads_or(bad)) {
+            if (tid == 0 && a.err) atomicExch(a.err, 1);
+            break;
+        }
+        tc_fence_after();
+
+        // S^T <- gamma S^T + (S^T X^T) + Y
+        const uint8_t* sY = smem + S::A_BYTES + s * S::STAGE + S::X_BYTES;
+#pragma unroll
+        for (int g = 0; g < DK / 32; ++g) {
+            float d[32];
+            tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + g * 32, d);
+            if (live) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 yv = *reinterpret_cast<const uint4*>(sY + sw128_offset(j, 32 * g + 8 * q, DV));
+                    const __nv_bfloat162* y2 = reinterpret_cast<const __nv_bfloat162*>(&yv);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 yf = __bfloat1622float2(y2[e]);
+                        const int m = 32 * g + 8 * q + 2 * e;
+                        st[m] = fmaf(gam, st[m], d[8 * q + 2 * e] + yf.x);
+                        st[m + 1] = fmaf(gam, st[m + 1], d[8 * q + 2 * e + 1] + yf.y);
+                    }
+                }
+            }
+        }
+        tc_fence_before();
+    }
+
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, DK);
+    if (a.fin && live) {
+        float* fin = a.fin + ((long long)n * a.H + h) * DK * DV;
+#pragma unroll
+        for (int m = 0; m < DK; ++m) fin[(long long)m * DV + j] = st[m];
+    }
+}
+
+// ------------------------------------------------------------- fp32 path
+
+template <int DK>
+struct ScanSimtSmem {
+    static constexpr int PK = pitch<float>(DK);
+    static constexpr size_t OS = 0;                                       // state tile [64][DK]
+    static constexpr size_t OX = align128(OS + sizeof(float) * 64 * PK);  // X [DK][DK]
+    static constexpr size_t OY = align128(OX + sizeof(float) * DK * PK);  // Y tile [64][DK]
+    static constexpr size_t bytes() { return OY + sizeof(float) * 64 * PK; }
+};
+
+// One CTA per (sequence x 64-row dv tile, head); warp w owns state rows 16w..16w+15.
+template <int DK, int DV>
+__global__ void __launch_bounds__(128) k_scan_simt(ScanArgs a) {
+    using S = ScanSimtSmem<DK>;
+    constexpr int NT = DK / 8;
+    const int jt = blockIdx.x % (DV / 64), n = blockIdx.x / (DV / 64), h = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int j0 = jt * 64;
+    extern __shared__ __align__(128) char smem[];
+    float* sS = reinterpret_cast<float*>(smem + S::OS);
+    float* sX = reinterpret_cast<float*>(smem + S::OX);
+    float* sY = reinterpret_cast<float*>(smem + S::OY);
+
+    float acc[NT][4];
+    const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
+#pragma unroll
+    for (int t = 0; t < NT; ++t)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int r = j0 + 16 * warp + frag_row(i), m = frag_col(t, i);
+            acc[t][i] = init ? init[(long long)m * DV + r] : 0.f;
+        }
+
+    long long start, len;
+    scan_seq_range(a, n, start, len);
+    const int s0 = a.seq_first[n];
+    int nch = (int)((len + kChunk - 1) / kChunk);
+    if (s0 + nch > a.slots) nch = a.slots - s0 > 0 ? a.slots - s0 : 0;
+
+    for (int it = 0; it < nch; ++it) {
+        const int c = a.reverse ? nch - 1 - it : it;
+        const long long idx = (long long)(s0 + c) * a.H + h;
+        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+        const float gam = expf(a.Gb[idx * 64 + L - 1]);
+        load_tile_async<float>(sX, S::PK, reinterpret_cast<const float*>(a.X) + idx * DK * DK, DK, DK, DK, DK, tid,
+                               128);
+        load_tile_async<float>(sY, S::PK, reinterpret_cast<const float*>(a.Y) + (idx * DV + j0) * DK, DK, 64, DK, 64,
+                               tid, 128);
+        cp_async_commit();
+        frag_store<float, NT>(sS, S::PK, 16 * warp, 0, acc);
+        float* out = reinterpret_cast<float*>(a.Sout) + (idx * DV + j0) * DK;
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                out[(long long)(16 * warp + frag_row(i)) * DK + frag_col(t, i)] = acc[t][i];
+        cp_async_wait<0>();
+        __syncthreads();
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                acc[t][i] = fmaf(gam, acc[t][i], sY[(16 * warp + frag_row(i)) * S::PK + frag_col(t, i)]);
+        warp_gemm<true, true, NT>(acc, sS, S::PK, sX, S::PK, 16 * warp, 0, DK);
+        __syncthreads();
+    }
+    if (a.fin) {
+        float* fin = a.fin + ((long long)n * a.H + h) * DK * DV;
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = j0 + 16 * warp + frag_row(i), m = frag_col(t, i);
+                fin[(long long)m * DV + r] = acc[t][i];
+            }
+    }
+}
+
+// ---------------------------------------------------------------- launcher
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// 2D bf16 view [rows][cols] with 128-byte swizzle and a [box_rows][64] box.
+static bool make_map(CUtensorMap* m, const void* base, long long rows, int cols, int box_rows) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t gdim[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t gstride[1] = {(cuuint64_t)cols * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int DK, int DV>
+static cudaError_t run_scan_tc(const ScanArgs& a, long long pairs, cudaStream_t s) {
+    using S = ScanTcSmem<DK, DV>;
+    CUtensorMap tx, ty;
+    if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, DV))
+        return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k_scan_tc<DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)S::bytes());
+    if (e) return e;
+    k_scan_tc<DK, DV><<<dim3(a.N, a.H), 128, S::bytes(), s>>>(a, tx, ty);
+    return cudaGetLastError();
+}
+
+template <int DK, int DV>
+static cudaError_t run_scan_simt(const ScanArgs& a, cudaStream_t s) {
+    using S = ScanSimtSmem<DK>;
+    cudaError_t e = cudaFuncSetAttribute(k_scan_simt<DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)S::bytes());
+    if (e) return e;
+    k_scan_simt<DK, DV><<<dim3((DV / 64) * a.N, a.H), 128, S::bytes(), s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s) {
+#define COMBA_SCAN(DK, DV)                                                                    \
+    if (dk == DK && dv == DV) return is_bf16 ? run_scan_tc<DK, DV>(a, pairs, s) : run_scan_simt<DK, DV>(a, s);
+    COMBA_SCAN(128, 128) COMBA_SCAN(128, 64) COMBA_SCAN(64, 128) COMBA_SCAN(64, 64)
+#undef COMBA_SCAN
+    return cudaErrorInvalidValue;
+}
+
+size_t scan_smem_bytes(bool is_bf16, int dk, int dv) {
+    if (is_bf16) {
+        if (dk == 128) return dv == 128 ? ScanTcSmem<128, 128>::bytes() : ScanTcSmem<128, 64>::bytes();
+        return dv == 128 ? ScanTcSmem<64, 128>::bytes() : ScanTcSmem<64, 64>::bytes();
+    }
+    return dk == 128 ? ScanSimtSmem<128>::bytes() : ScanSimtSmem<64>::bytes();
+}
+
+}  // namespace comba
