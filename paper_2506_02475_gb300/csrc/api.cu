@@ -63,7 +63,8 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (backward) {
         L.E = take(pairs * 64 * dv * es);
         L.M = take(pairs * 64 * 64 * es);
-        L.AT = take(pairs * dk * dk * es);
+        // Atilde^T is only materialised off the tcgen05 path (that reverse scan reads Atilde directly)
+        if (!comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv)) L.AT = take(pairs * dk * dk * es);
         L.C = take(pairs * dv * dk * es);
         L.dH = take(pairs * dv * dk * es);
         L.part = take(pairs * 2 * sizeof(float));
@@ -108,7 +109,7 @@ void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* 
     if (backward_layout) {
         p.Eb = w + L.E;
         p.Mb = w + L.M;
-        p.ATb = w + L.AT;
+        p.ATb = comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv) ? nullptr : w + L.AT;
         p.Cb = w + L.C;
         p.dHb = w + L.dH;
         p.part = reinterpret_cast<float*>(w + L.part);

@@ -595,13 +595,20 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
         return e;
     if ((e = cudaFuncSetAttribute(k_bwd_local<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_loc)))
         return e;
+    const bool tcp = use_tc_path(sizeof(T) == 2, DK, DV);
     mark(p, ev0, s);
-    if (p.slots > 0) k_bwd_prep<T, DK, DV><<<dim3(p.slots, p.H), 128, sm_prep, s>>>(p);
+    if (tcp) {
+        if ((e = launch_bwd_prep_tc(p, s))) return e;
+    } else if (p.slots > 0) {
+        k_bwd_prep<T, DK, DV><<<dim3(p.slots, p.H), 128, sm_prep, s>>>(p);
+    }
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 1, s);
     ScanArgs a;
     a.H = p.H; a.N = p.N; a.T = p.T; a.slots = p.slots; a.Ttot = p.Ttot; a.cu = p.cu; a.seq_first = p.seq_first;
-    a.Gb = p.Gb; a.init = p.dhT; a.fin = p.dh0; a.Sout = p.dHb; a.X = p.ATb; a.Y = p.Cb; a.reverse = 1; a.err = p.err;
+    a.Gb = p.Gb; a.init = p.dhT; a.fin = p.dh0; a.Sout = p.dHb; a.Y = p.Cb; a.reverse = 1; a.err = p.err;
+    a.X = tcp ? p.Ab : p.ATb;   // tcgen05 path: Atilde read as an MN-major operand
+    a.x_mn = tcp ? 1 : 0;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)p.slots * p.H, s))) return e;
     mark(p, ev0 + 2, s);
     if (p.slots > 0) k_bwd_local<T, DK, DV><<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
@@ -626,6 +633,7 @@ cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int e
 }
 
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
+    if (kernel == 0 && use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(2);
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? BPrepSmem<T, DK, DV>::bytes() : LocalSmem<T, DK, DV>::bytes();
     if (is_bf16) {

@@ -354,18 +354,31 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
         return e;
     if ((e = cudaFuncSetAttribute(k_output<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out)))
         return e;
+    const bool tcp = use_tc_path(sizeof(T) == 2, DK, DV);
     ChunkParams q = p;
     if (!save) { q.Mb = nullptr; q.ATb = nullptr; q.Eb = nullptr; }
+    if (tcp) q.ATb = nullptr;   // the tcgen05 reverse scan reads Atilde directly
     mark(q, ev0, s);
-    if (q.slots > 0) k_prep<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_prep, s>>>(q);
+    if (tcp) {
+        if ((e = launch_prep_tc(q, s))) return e;
+    } else if (q.slots > 0) {
+        k_prep<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_prep, s>>>(q);
+    }
     if ((e = cudaGetLastError())) return e;
     mark(q, ev0 + 1, s);
     ScanArgs a;
     a.H = q.H; a.N = q.N; a.T = q.T; a.slots = q.slots; a.Ttot = q.Ttot; a.cu = q.cu; a.seq_first = q.seq_first;
-    a.Gb = q.Gb; a.init = q.h0; a.fin = q.hT; a.Sout = q.Hb; a.X = q.Ab; a.Y = q.Bb; a.reverse = 0; a.err = q.err;
+    a.Gb = q.Gb; a.init = q.h0; a.fin = q.hT; a.Sout = q.Hb; a.X = q.Ab; a.Y = q.Bb; a.reverse = 0; a.x_mn = 0;
+    a.err = q.err;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)q.slots * q.H, s))) return e;
     mark(q, ev0 + 2, s);
-    if (q.slots > 0 && (q.o || q.Eb)) k_output<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_out, s>>>(q);
+    if (q.o || q.Eb) {
+        if (tcp) {
+            if ((e = launch_output_tc(q, s))) return e;
+        } else if (q.slots > 0) {
+            k_output<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_out, s>>>(q);
+        }
+    }
     if ((e = cudaGetLastError())) return e;
     mark(q, ev0 + 3, s);
     return cudaSuccess;
@@ -390,6 +403,7 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
 
 size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
     if (kernel == 1) return scan_smem_bytes(is_bf16, dk, dv);
+    if (use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(kernel == 0 ? 0 : 1);
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes() : OutSmem<T, DK, DV>::bytes();
     if (is_bf16) {

@@ -1,0 +1,600 @@
+// tcgen05 (5th-generation tensor core) kernels for the bf16, dk = dv = 128 path.
+//
+// Every tile product is issued by one thread as tcgen05.mma (M = 128, fp32
+// accumulator in TMEM) on 128-byte-swizzled shared-memory tiles; the other
+// threads stage tiles with asynchronous copies and run the epilogues on the
+// rows they read back from TMEM (one row per thread).  Products are formed
+// transposed where that puts a 128-wide head dimension on M (W^T, U^T, E^T,
+// O^T, C^T); 64 x 64 chunk products pad M to 128 with zero rows.
+//
+//   k_prep_tc      Gram K K^T -> decay/btilde mask -> UT inverse M (fp32, blocked
+//                  forward substitution) -> W^T = K^T Mw^T, U^T = V^T Mu^T ->
+//                  Atilde = -K^T Diag(s) W, B^T = (Diag(s) U)^T K  (s = gamma_C/gamma_r)
+//   k_output_tc    P = Tril(Q~ K^T * Gamma), E^T = U^T - H^T W^T,
+//                  O^T = H^T Qhat^T + E^T P^T  (Qhat = Diag(gamma) Q~)
+//   k_bwd_prep_tc  C^T = dO^T (Qhat - P W)
+//
+// Workspace tensors of this path: W^T, U^T [pairs][128][64]; Atilde, B^T,
+// H^T, C^T, dH^T [pairs][128][128]; E [pairs][64][128] row-major; M [pairs][64][64].
+#include "params.cuh"
+
+namespace comba {
+namespace tc {
+
+constexpr int D = 128;  // head dim of this path
+
+// cp.async a row-major bf16 matrix (rows r < valid; `cols` in {64, 128}) into a
+// 128B-swizzled tile with `alloc` rows; rows valid..alloc-1 are zero-filled.
+__device__ __forceinline__ void load_sw(uint8_t* tile, int alloc, int cols, const bf16* g, long long gstride,
+                                        int valid, int tid) {
+    const int cpr = cols / 8;
+    for (int idx = tid; idx < alloc * cpr; idx += 128) {
+        const int r = idx / cpr, ch = idx - r * cpr;
+        const bool ok = r < valid;
+        cp_async16(tile + sw128_offset(r, ch * 8, alloc),
+                   ok ? (const void*)(g + (long long)r * gstride + ch * 8) : (const void*)g, ok);
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float* v) {
+    uint4 r;
+    __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
+    __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
+    __nv_bfloat162 c = __floats2bfloat162_rn(v[4], v[5]);
+    __nv_bfloat162 d = __floats2bfloat162_rn(v[6], v[7]);
+    r.x = *reinterpret_cast<uint32_t*>(&a);
+    r.y = *reinterpret_cast<uint32_t*>(&b);
+    r.z = *reinterpret_cast<uint32_t*>(&c);
+    r.w = *reinterpret_cast<uint32_t*>(&d);
+    return r;
+}
+__device__ __forceinline__ void unpack8(uint4 u, float* v) {
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(h[i]);
+        v[2 * i] = f.x;
+        v[2 * i + 1] = f.y;
+    }
+}
+
+// One-barrier MMA completion tracker (all threads keep the same phase).
+struct MmaSync {
+    uint32_t bar;
+    uint32_t phase;
+    // Thread 0 has issued MMAs; commit, wait everywhere, and report failure uniformly.
+    __device__ __forceinline__ bool finish(int tid) {
+        if (tid == 0) tc_commit(bar);
+        const bool ok = mbar_wait(bar, phase);
+        phase ^= 1;
+        const bool any_bad = __syncthreads_or(!ok);
+        tc_fence_after();
+        return !any_bad;
+    }
+};
+
+__device__ __forceinline__ void flag_error(const ChunkParams& p) {
+    if (p.err) atomicExch(p.err, 1);
+}
+
+// Make generic-proxy shared-memory writes visible to the tensor core and order
+// prior TMEM reads before the next MMA.
+__device__ __forceinline__ void publish_smem() {
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+}
+
+// ------------------------------------------------------------------ prep
+
+struct PrepTcSmem {
+    static constexpr uint32_t OK = 0;                    // K  [128 alloc rows][128]   32 KB
+    static constexpr uint32_t OV = OK + 32768;           // V  [64][128]               16 KB
+    static constexpr uint32_t OMW = OV + 16384;          // Mw [64][64] K-major         8 KB
+    static constexpr uint32_t OMU = OMW + 8192;          // Mu [64][64]                 8 KB
+    static constexpr uint32_t OR = OMU + 8192;           // A, M fp32 then sW^T, sU^T [128][64]
+    static constexpr uint32_t R_BYTES = 2 * 64 * 65 * 4 > 2 * 16384 ? 2 * 64 * 65 * 4 : 2 * 16384;
+    static constexpr uint32_t OT = OR + ((R_BYTES + 1023) & ~1023u);
+    static constexpr uint32_t OF = OT + 3 * 272 * 4;
+    static constexpr size_t bytes() { return 1024 + OF + 64 * 6 * 4; }
+};
+
+__global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
+    using S = PrepTcSmem;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t bar;
+    __shared__ uint32_t tbase;
+    const int slot = blockIdx.x, h = blockIdx.y;
+    const SlotInfo si = p.slot_info[slot];
+    if (si.len <= 0) return;
+    const int L = si.len;
+    const long long t0 = si.start;
+    const long long idx = (long long)slot * p.H + h;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sK = sm + S::OK;
+    uint8_t* sV = sm + S::OV;
+    uint8_t* sMw = sm + S::OMW;
+    uint8_t* sMu = sm + S::OMU;
+    float* sA = reinterpret_cast<float*>(sm + S::OR);
+    float* sM = sA + 64 * 65;
+    uint8_t* sWt = sm + S::OR;            // aliases A after the inverse
+    uint8_t* sUt = sm + S::OR + 16384;    // aliases M after Mw/Mu are built
+    float* sTmp = reinterpret_cast<float*>(sm + S::OT);
+    float* sG = reinterpret_cast<float*>(sm + S::OF);
+    float* sGm1 = sG + 64;
+    float* sBt = sG + 128;
+    float* sBe = sG + 192;
+    float* sS = sG + 256;
+
+    load_sw(sK, 128, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    cp_async_commit();
+    if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
+    if (tid < 64) {
+        const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
+        sBe[tid] = be;
+        sBt[tid] = (p.b ? p.b[h] : 1.f) * be;
+    }
+    if (tid == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
+    cp_async_wait<0>();
+    publish_smem();
+    const uint32_t tmem = tbase;
+    MmaSync ms{smem_u32(&bar), 0};
+    const int row = tid;  // TMEM lane / accumulator row of this thread
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    bool ok = true;
+
+    // Gram K K^T (rows >= 64 of the A tile are zero).
+    if (tid == 0) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sK), 128, 64, D, false);
+    if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;
+    ok = ms.finish(tid);
+    if (ok) {
+        // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T); exp only below the diagonal.
+        float d[32];
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+            tmem_ld32(trow + g * 32, d);
+            if (row < 64) {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    const int i = 32 * g + c;
+                    sA[row * 65 + i] = (i < row && row < L) ? sBt[row] * expf(sGm1[row] - sG[i]) * d[c] : 0.f;
+                }
+            }
+        }
+    }
+    __syncthreads();
+    if (ok) {
+        unit_lower_inverse64(sA, sM, sTmp, tid);
+        // Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta) as K-major [p][p'] tiles; M saved for the backward.
+        bf16* Mg = p.Mb ? (bf16*)p.Mb + idx * 4096 : nullptr;
+        for (int e = tid; e < 64 * 8; e += 128) {
+            const int r = e >> 3, ch = e & 7;
+            float mw[8], mu[8], mm[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int c = 8 * ch + q;
+                mm[q] = sM[r * 65 + c];
+                mw[q] = mm[q] * sBt[c] * expf(sGm1[c]);
+                mu[q] = mm[q] * sBe[c];
+            }
+            *reinterpret_cast<uint4*>(sMw + sw128_offset(r, 8 * ch, 64)) = pack8(mw);
+            *reinterpret_cast<uint4*>(sMu + sw128_offset(r, 8 * ch, 64)) = pack8(mu);
+            if (Mg) *reinterpret_cast<uint4*>(Mg + r * 64 + 8 * ch) = pack8(mm);
+        }
+        if (tid < 64) p.Gb[idx * 64 + tid] = sG[tid];
+    }
+    publish_smem();
+
+    // W^T = K^T Mw^T (A = K as MN-major), U^T = V^T Mu^T.
+    if (ok && tid == 0) {
+        tc_gemm<true, false>(tmem + 64, smem_u32(sK), 128, smem_u32(sMw), 64, 64, 64, false);
+        tc_gemm<true, false>(tmem + 128, smem_u32(sV), 64, smem_u32(sMu), 64, 64, 64, false);
+    }
+    ok = ok && ms.finish(tid);
+    if (ok) {
+        float d[32], v[8], w[8];
+        bf16* Wt = (bf16*)p.Wb + (idx * D + row) * 64;
+        bf16* Ut = (bf16*)p.Ub + (idx * D + row) * 64;
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+            tmem_ld32(trow + 64 + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    v[e] = d[8 * q + e];
+                    w[e] = v[e] * sS[32 * g + 8 * q + e];
+                }
+                *reinterpret_cast<uint4*>(Wt + 32 * g + 8 * q) = pack8(v);
+                *reinterpret_cast<uint4*>(sWt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+            tmem_ld32(trow + 128 + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    v[e] = d[8 * q + e];
+                    w[e] = v[e] * sS[32 * g + 8 * q + e];
+                }
+                *reinterpret_cast<uint4*>(Ut + 32 * g + 8 * q) = pack8(v);
+                *reinterpret_cast<uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
+            }
+        }
+    }
+    publish_smem();
+
+    // Atilde = -K^T (Diag(s) W) -> cols [0,128);  B^T = (Diag(s) U)^T K -> cols [128,256).
+    if (ok && tid == 0) {
+        tc_gemm<true, false>(tmem, smem_u32(sK), 128, smem_u32(sWt), 128, 128, 64, false);
+        tc_gemm<false, true>(tmem + 128, smem_u32(sUt), 128, smem_u32(sK), 128, 128, 64, false);
+    }
+    ok = ok && ms.finish(tid);
+    if (ok) {
+        float d[32], v[8];
+        bf16* At = (bf16*)p.Ab + (idx * D + row) * D;
+        bf16* Bt = (bf16*)p.Bb + (idx * D + row) * D;
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            tmem_ld32(trow + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v[e] = -d[8 * q + e];
+                *reinterpret_cast<uint4*>(At + 32 * g + 8 * q) = pack8(v);
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            tmem_ld32(trow + 128 + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) *reinterpret_cast<uint4*>(Bt + 32 * g + 8 * q) = pack8(d + 8 * q);
+        }
+    }
+    if (!ok && tid == 0) flag_error(p);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, 256);
+}
+
+// ---------------------------------------------------------------- output
+
+struct OutTcSmem {
+    static constexpr uint32_t OQ = 0;              // Q -> Q~ -> Qhat   [128 alloc rows][128]  32 KB
+    static constexpr uint32_t OK = 32768;          // K [64][128], later P [64][64]            16 KB
+    static constexpr uint32_t OW = OK + 16384;     // W^T [128][64] (MN-major B), later E^T    16 KB
+    static constexpr uint32_t OU = OW + 16384;     // U^T [128][64]                            16 KB
+    static constexpr uint32_t OH = OU + 16384;     // H^T [128][128] K-major, later O staging  32 KB
+    static constexpr uint32_t OG = OH + 32768;
+    static constexpr size_t bytes() { return 1024 + OG + 64 * 4; }
+};
+
+__global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
+    using S = OutTcSmem;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t bar;
+    __shared__ uint32_t tbase;
+    const int slot = blockIdx.x, h = blockIdx.y;
+    const SlotInfo si = p.slot_info[slot];
+    if (si.len <= 0) return;
+    const int L = si.len;
+    const long long t0 = si.start;
+    const long long idx = (long long)slot * p.H + h;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sQ = sm + S::OQ;
+    uint8_t* sK = sm + S::OK;
+    uint8_t* sP = sK;
+    uint8_t* sWt = sm + S::OW;
+    uint8_t* sEt = sWt;
+    uint8_t* sUt = sm + S::OU;
+    uint8_t* sHt = sm + S::OH;
+    bf16* sO = reinterpret_cast<bf16*>(sHt);   // [64][136] staging of O
+    float* sG = reinterpret_cast<float*>(sm + S::OG);
+
+    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid);
+    load_sw(sUt, 128, 64, (const bf16*)p.Ub + idx * D * 64, 64, 128, tid);
+    load_sw(sHt, 128, D, (const bf16*)p.Hb + idx * D * D, D, 128, tid);
+    cp_async_commit();
+    if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+    if (tid == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
+    cp_async_wait<0>();
+    __syncthreads();
+    // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
+    const float dh = p.d[h];
+    for (int e = tid; e < 64 * 16; e += 128) {
+        const int r = e >> 4, ch = e & 15;
+        uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
+        const uint4 ka = *reinterpret_cast<const uint4*>(sK + sw128_offset(r, 8 * ch, 64));
+        float qv[8], kv[8];
+        unpack8(*qa, qv);
+        unpack8(ka, kv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
+        *qa = pack8(qv);
+    }
+    publish_smem();
+    const uint32_t tmem = tbase;
+    MmaSync ms{smem_u32(&bar), 0};
+    const int row = tid;
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+    // S = Q~ K^T -> cols [0,64);  E^T' = H^T W^T -> cols [64,128)
+    if (tid == 0) {
+        tc_gemm<false, false>(tmem, smem_u32(sQ), 128, smem_u32(sK), 64, 64, D, false);
+        tc_gemm<false, true>(tmem + 64, smem_u32(sHt), 128, smem_u32(sWt), 128, 64, D, false);
+    }
+    bool ok = ms.finish(tid);
+    if (ok) {
+        float d[32], v[8];
+        // P = Tril(S * Gamma) into a K-major [64][64] tile (B operand of E^T P^T)
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+            tmem_ld32(trow + g * 32, d);
+            if (row < 64) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const int i = 32 * g + 8 * q + e;
+                        v[e] = (i <= row && row < L) ? d[8 * q + e] * expf(sG[row] - sG[i]) : 0.f;
+                    }
+                    *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 64)) = pack8(v);
+                }
+            }
+        }
+        // E^T = U^T - H^T W^T  (row j of E^T per thread; saved as E [64][128] for the backward)
+        bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+            tmem_ld32(trow + 64 + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float u[8];
+                unpack8(*reinterpret_cast<const uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)), u);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v[e] = u[e] - d[8 * q + e];
+                // sEt aliases sWt: every thread reads only its own row, and W^T is no longer needed
+                *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
+                if (Eg) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) Eg[(32 * g + 8 * q + e) * D + row] = __float2bfloat16_rn(v[e]);
+                }
+            }
+        }
+        // Qhat = Diag(gamma) Q~ in place
+        for (int e = tid; e < 64 * 16; e += 128) {
+            const int r = e >> 4, ch = e & 15;
+            uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
+            float qv[8];
+            unpack8(*qa, qv);
+            const float gr = expf(sG[r]);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) qv[i] *= gr;
+            *qa = pack8(qv);
+        }
+    }
+    publish_smem();
+    if (!p.o) ok = false;   // E only (backward recompute): nothing more to do
+
+    // O^T = H^T Qhat^T + E^T P^T -> cols [128,192)
+    if (ok && tid == 0) {
+        tc_gemm<false, false>(tmem + 128, smem_u32(sHt), 128, smem_u32(sQ), 128, 64, D, false);
+        tc_gemm<false, false>(tmem + 128, smem_u32(sEt), 128, smem_u32(sP), 64, 64, 64, true);
+    }
+    if (p.o) {
+        ok = ok && ms.finish(tid);
+        if (ok) {
+            float d[32];
+#pragma unroll
+            for (int g = 0; g < 2; ++g) {
+                tmem_ld32(trow + 128 + g * 32, d);
+#pragma unroll
+                for (int c = 0; c < 32; ++c) sO[(32 * g + c) * 136 + row] = __float2bfloat16_rn(d[c]);
+            }
+        }
+        __syncthreads();
+        if (ok) {
+            bf16* Og = (bf16*)p.o + (t0 * p.H + h) * D;
+            for (int e = tid; e < L * 16; e += 128) {
+                const int r = e >> 4, ch = e & 15;
+                *reinterpret_cast<uint4*>(Og + (long long)r * p.H * D + 8 * ch) =
+                    *reinterpret_cast<const uint4*>(sO + r * 136 + 8 * ch);
+            }
+        } else if (tid == 0) {
+            flag_error(p);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, 256);
+}
+
+// ------------------------------------------------- reverse-scan additive term
+
+struct BPrepTcSmem {
+    static constexpr uint32_t OQ = 0;              // Q -> Q~ -> Qhat [128 alloc rows][128]   32 KB
+    static constexpr uint32_t OK = 32768;          // K [64][128], later P [128 alloc][64]    16 KB
+    static constexpr uint32_t OW = OK + 16384;     // W^T [128][64] (K-major B), later Z      16 KB
+    static constexpr uint32_t OD = OW + 16384;     // dO [64][128] (MN-major A)               16 KB
+    static constexpr uint32_t OG = OD + 16384;
+    static constexpr size_t bytes() { return 1024 + OG + 64 * 4; }
+};
+
+__global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
+    using S = BPrepTcSmem;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t bar;
+    __shared__ uint32_t tbase;
+    const int slot = blockIdx.x, h = blockIdx.y;
+    const SlotInfo si = p.slot_info[slot];
+    if (si.len <= 0) return;
+    const int L = si.len;
+    const long long t0 = si.start;
+    const long long idx = (long long)slot * p.H + h;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sQ = sm + S::OQ;
+    uint8_t* sK = sm + S::OK;
+    uint8_t* sP = sK;
+    uint8_t* sWt = sm + S::OW;
+    uint8_t* sZ = sWt;
+    uint8_t* sdO = sm + S::OD;
+    float* sG = reinterpret_cast<float*>(sm + S::OG);
+
+    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid);
+    load_sw(sdO, 64, D, (const bf16*)p.dO + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    cp_async_commit();
+    if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+    if (tid == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
+    cp_async_wait<0>();
+    __syncthreads();
+    const float dh = p.d[h];
+    for (int e = tid; e < 64 * 16; e += 128) {
+        const int r = e >> 4, ch = e & 15;
+        uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
+        const uint4 ka = *reinterpret_cast<const uint4*>(sK + sw128_offset(r, 8 * ch, 64));
+        float qv[8], kv[8];
+        unpack8(*qa, qv);
+        unpack8(ka, kv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
+        *qa = pack8(qv);
+    }
+    publish_smem();
+    const uint32_t tmem = tbase;
+    MmaSync ms{smem_u32(&bar), 0};
+    const int row = tid;
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+
+    if (tid == 0) tc_gemm<false, false>(tmem, smem_u32(sQ), 128, smem_u32(sK), 64, 64, D, false);   // Q~ K^T
+    bool ok = ms.finish(tid);
+    if (ok) {
+        // P [128 alloc rows][64] K-major A operand (rows >= 64 zero); Qhat = Diag(gamma) Q~ in place.
+        float d[32], v[8];
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+            tmem_ld32(trow + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const int i = 32 * g + 8 * q + e;
+                    v[e] = (row < 64 && i <= row && row < L) ? d[8 * q + e] * expf(sG[row] - sG[i]) : 0.f;
+                }
+                *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
+            }
+        }
+        for (int e = tid; e < 64 * 16; e += 128) {
+            const int r = e >> 4, ch = e & 15;
+            uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
+            float qv[8];
+            unpack8(*qa, qv);
+            const float gr = expf(sG[r]);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) qv[i] *= gr;
+            *qa = pack8(qv);
+        }
+    }
+    publish_smem();
+    // P W -> cols [64,192)  (B = W via W^T [c][i], K-major)
+    if (ok && tid == 0) tc_gemm<false, false>(tmem + 64, smem_u32(sP), 128, smem_u32(sWt), 128, 128, 64, false);
+    ok = ok && ms.finish(tid);
+    if (ok && row < 64) {
+        // Z = Qhat - P W, written as an MN-major [64 k-rows][128] tile (B operand of dO^T Z)
+        float d[32], v[8];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            tmem_ld32(trow + 64 + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float qh[8];
+                unpack8(*reinterpret_cast<const uint4*>(sQ + sw128_offset(row, 32 * g + 8 * q, 128)), qh);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v[e] = qh[e] - d[8 * q + e];
+                *reinterpret_cast<uint4*>(sZ + mn128_offset(32 * g + 8 * q, row, 64)) = pack8(v);
+            }
+        }
+    } else if (ok) {
+        float d[32];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) tmem_ld32(trow + 64 + g * 32, d);   // keep the warp-collective loads aligned
+    }
+    publish_smem();
+    // C^T = dO^T Z -> cols [0,128)
+    if (ok && tid == 0) tc_gemm<true, true>(tmem, smem_u32(sdO), 64, smem_u32(sZ), 64, 128, 64, false);
+    ok = ok && ms.finish(tid);
+    if (ok) {
+        float d[32];
+        bf16* Cg = (bf16*)p.Cb + (idx * D + row) * D;
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            tmem_ld32(trow + g * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) *reinterpret_cast<uint4*>(Cg + 32 * g + 8 * q) = pack8(d + 8 * q);
+        }
+    } else if (tid == 0) {
+        flag_error(p);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, 256);
+}
+
+}  // namespace tc
+
+// -------------------------------------------------------------- launchers
+
+cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s) {
+    const size_t sm = tc::PrepTcSmem::bytes();
+    cudaError_t e = cudaFuncSetAttribute(tc::k_prep_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e) return e;
+    if (p.slots > 0) tc::k_prep_tc<<<dim3(p.slots, p.H), 128, sm, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s) {
+    const size_t sm = tc::OutTcSmem::bytes();
+    cudaError_t e = cudaFuncSetAttribute(tc::k_output_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e) return e;
+    if (p.slots > 0) tc::k_output_tc<<<dim3(p.slots, p.H), 128, sm, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_bwd_prep_tc(const ChunkParams& p, cudaStream_t s) {
+    const size_t sm = tc::BPrepTcSmem::bytes();
+    cudaError_t e = cudaFuncSetAttribute(tc::k_bwd_prep_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e) return e;
+    if (p.slots > 0) tc::k_bwd_prep_tc<<<dim3(p.slots, p.H), 128, sm, s>>>(p);
+    return cudaGetLastError();
+}
+
+size_t tc_smem_bytes(int kernel) {
+    return kernel == 0 ? tc::PrepTcSmem::bytes() : (kernel == 1 ? tc::OutTcSmem::bytes() : tc::BPrepTcSmem::bytes());
+}
+
+}  // namespace comba

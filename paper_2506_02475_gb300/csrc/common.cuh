@@ -349,6 +349,46 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// Descriptors of the 16-deep K step `ks` of a bf16 operand tile in the 128-byte
+// swizzle layout.  K-major tile: K split in 64-element halves, each a
+// [rows][128 B] block (rows = the tile's allocated M or N extent).  MN-major
+// tile: M/N split in 64-element halves, each a [krows][128 B] block (krows =
+// the tile's allocated K extent); consecutive K rows are 128 B apart.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFF);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+__device__ __forceinline__ uint64_t desc_kmajor(uint32_t base, int rows, int ks) {
+    return smem_desc(base + (ks >> 2) * rows * 128 + (ks & 3) * 32, 16, 1024);
+}
+__device__ __forceinline__ uint64_t desc_mnmajor(uint32_t base, int krows, int ks) {
+    return smem_desc(base + ks * 2048, krows * 128, 1024);
+}
+
+// D[tmem, 128 x N fp32] (+)= A[128 x K] * B[K x N] on bf16 smem tiles, issued by one
+// thread.  AMN/BMN select MN-major operand tiles; a_ext/b_ext are the tiles'
+// allocated row counts (see above).  K % 16 == 0.
+template <bool AMN, bool BMN>
+__device__ __forceinline__ void tc_gemm(uint32_t tmem, uint32_t a, int a_ext, uint32_t b, int b_ext, int N, int K,
+                                        bool accumulate) {
+    const uint32_t idesc = idesc_bf16_f32(128, N) | (AMN ? 1u << 15 : 0u) | (BMN ? 1u << 16 : 0u);
+    for (int ks = 0; ks < K / 16; ++ks) {
+        const uint64_t ad = AMN ? desc_mnmajor(a, a_ext, ks) : desc_kmajor(a, a_ext, ks);
+        const uint64_t bd = BMN ? desc_mnmajor(b, b_ext, ks) : desc_kmajor(b, b_ext, ks);
+        tc_mma_bf16(tmem, ad, bd, idesc, (accumulate || ks > 0) ? 1u : 0u);
+    }
+}
+
+// Byte offset of element (mn, k) of an MN-major bf16 tile (allocated K extent krows).
+__host__ __device__ constexpr uint32_t mn128_offset(int mn, int k, int krows) {
+    return (uint32_t)((mn >> 6) * krows * 128 + k * 128 + ((((mn & 63) >> 3) ^ (k & 7)) << 4) + (mn & 7) * 2);
+}
+
 // Byte offset of element (row, k) of a K-major bf16 tile in the 128-byte swizzle
 // layout: K is split in halves of 64 elements, each a [rows][128 B] block.
 __host__ __device__ constexpr uint32_t sw128_offset(int row, int k, int rows) {

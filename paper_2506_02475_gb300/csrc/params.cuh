@@ -79,6 +79,7 @@ struct ScanArgs {
     const void* X;           // [pairs][dk][dk] row-major
     const void* Y;           // [pairs][dv][dk]
     int reverse;
+    int x_mn;                // X is read as an MN-major operand ([k][m] row-major, no transpose)
     int* err;
 };
 cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s);
@@ -95,6 +96,12 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
 // the local gradients, ev0+3 before the reduction, ev0+4 after it.
 cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int ev0);
 size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);
+// tcgen05 kernels of the bf16 dk = dv = 128 path (chunk_tc.cu)
+cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s);
+cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s);
+cudaError_t launch_bwd_prep_tc(const ChunkParams& p, cudaStream_t s);
+size_t tc_smem_bytes(int kernel);
+inline bool use_tc_path(bool is_bf16, int dk, int dv) { return is_bf16 && dk == 128 && dv == 128; }
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);
 cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, const void* q, const void* k,
                                   const void* v, const float* alpha, const float* beta, const float* b,

@@ -45,7 +45,7 @@ struct ScanTcSmem {
     static constexpr size_t bytes() { return 1024 + A_BYTES + STAGES * (size_t)STAGE; }
 };
 
-template <int DK, int DV>
+template <int DK, int DV, bool XMN>
 __global__ void __launch_bounds__(128, 1)
     k_scan_tc(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY) {
     using S = ScanTcSmem<DK, DV>;
@@ -100,7 +100,7 @@ __global__ void __launch_bounds__(128, 1)
     if (tid == 0)
         for (int it = 0; it < S::STAGES - 1 && it < nch; ++it) issue(it);
 
-    constexpr uint32_t idesc = idesc_bf16_f32(128, DK);
+    constexpr uint32_t idesc = idesc_bf16_f32(128, DK) | (XMN ? 1u << 16 : 0u);
     for (int it = 0; it < nch; ++it) {
         const int c = chunk_of(it), s = it % S::STAGES;
         const long long idx = (long long)(s0 + c) * a.H + h;
@@ -137,7 +137,8 @@ __global__ void __launch_bounds__(128, 1)
                 for (int ks = 0; ks < DK / 16; ++ks) {
                     const int half = ks >> 2, sub = ks & 3;
                     const uint64_t ad = smem_desc_sw128(sA_u + half * 128 * 128 + sub * 32);
-                    const uint64_t bd = smem_desc_sw128(stage_x(s) + half * DK * 128 + sub * 32);
+                    const uint64_t bd = XMN ? desc_mnmajor(stage_x(s), DK, ks)
+                                            : smem_desc_sw128(stage_x(s) + half * DK * 128 + sub * 32);
                     tc_mma_bf16(tmem, ad, bd, idesc, ks > 0 ? 1u : 0u);
                 }
             } else {
@@ -298,16 +299,16 @@ static bool make_map(CUtensorMap* m, const void* base, long long rows, int cols,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int DK, int DV>
+template <int DK, int DV, bool XMN>
 static cudaError_t run_scan_tc(const ScanArgs& a, long long pairs, cudaStream_t s) {
     using S = ScanTcSmem<DK, DV>;
     CUtensorMap tx, ty;
     if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, DV))
         return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(k_scan_tc<DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_scan_tc<DK, DV, XMN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)S::bytes());
     if (e) return e;
-    k_scan_tc<DK, DV><<<dim3(a.N, a.H), 128, S::bytes(), s>>>(a, tx, ty);
+    k_scan_tc<DK, DV, XMN><<<dim3(a.N, a.H), 128, S::bytes(), s>>>(a, tx, ty);
     return cudaGetLastError();
 }
 
@@ -322,8 +323,10 @@ static cudaError_t run_scan_simt(const ScanArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s) {
-#define COMBA_SCAN(DK, DV)                                                                    \
-    if (dk == DK && dv == DV) return is_bf16 ? run_scan_tc<DK, DV>(a, pairs, s) : run_scan_simt<DK, DV>(a, s);
+#define COMBA_SCAN(DK, DV)                                                                          \
+    if (dk == DK && dv == DV)                                                                        \
+        return !is_bf16 ? run_scan_simt<DK, DV>(a, s)                                                \
+                        : (a.x_mn ? run_scan_tc<DK, DV, true>(a, pairs, s) : run_scan_tc<DK, DV, false>(a, pairs, s));
     COMBA_SCAN(128, 128) COMBA_SCAN(128, 64) COMBA_SCAN(64, 128) COMBA_SCAN(64, 64)
 #undef COMBA_SCAN
     return cudaErrorInvalidValue;
