@@ -8,12 +8,13 @@
 //     dH_n = gamma_n dH_{n+1} + Atilde_n^T dH_{n+1} + C_n,  C_n = (Qhat_n - P_n W_n)^T dO_n.
 // Both are evaluated transposed, one state row (a dv index) per thread:
 //     S^T <- gamma S^T + S^T X^T + Y,
-// with X = Atilde (forward) or Atilde^T (backward) stored [dk][dk] row-major,
-// and Y = B^T or C^T stored [dv][dk].  Each chunk stores the state it started
+// with X = Atilde (forward; row-major [dk][dk], read K-major) or, in the
+// backward, Atilde read as an MN-major operand (bf16 path) or Atilde^T
+// (fp32 path); Y = B^T or C^T stored [dv][dk].  Each chunk stores the state it started
 // from (H_n^T, or dH_{n+1}^T in the backward) for the parallel kernels.
 //
-// bf16 storage: one CTA per (sequence, head), 128 threads; the fp32 state row
-// stays in registers; S^T (bf16) is written into a 128-byte-swizzled K-major
+// bf16 storage: one CTA per (sequence, head), 256 threads (two per state row,
+// each holding half of the row's dk columns); the fp32 state stays in registers; S^T (bf16) is written into a 128-byte-swizzled K-major
 // shared tile; X and Y stream in by TMA through a multi-stage mbarrier
 // pipeline; one thread issues the tcgen05 MMAs (M = 128, N = dk, K = dk)
 // into a TMEM accumulator that all threads read back with tcgen05.ld.
@@ -46,9 +47,10 @@ struct ScanTcSmem {
 };
 
 template <int DK, int DV, bool XMN>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(256, 1)
     k_scan_tc(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY) {
     using S = ScanTcSmem<DK, DV>;
+    constexpr int HC = DK / 2;  // state columns per thread: two threads per state row
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t full_bar[S::STAGES];
     __shared__ uint64_t mma_bar;
@@ -56,15 +58,16 @@ __global__ void __launch_bounds__(128, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5;
     const int n = blockIdx.x, h = blockIdx.y;
-    const int j = tid;  // state row (dv index)
+    const int j = tid & 127;           // state row (dv index); warps w and w+4 share TMEM lanes
+    const int c0 = (tid >> 7) * HC;    // first state column of this thread
     const bool live = j < DV;
     uint8_t* sA = smem;
     const uint32_t sA_u = smem_u32(sA);
 
-    float st[DK];
+    float st[HC];
     const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
 #pragma unroll
-    for (int m = 0; m < DK; ++m) st[m] = (init && live) ? init[(long long)m * DV + j] : 0.f;
+    for (int m = 0; m < HC; ++m) st[m] = (init && live) ? init[(long long)(c0 + m) * DV + j] : 0.f;
 
     long long start, len;
     scan_seq_range(a, n, start, len);
@@ -82,6 +85,7 @@ __global__ void __launch_bounds__(128, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base;
+    const uint32_t tlane = tmem + ((uint32_t)((warp & 3) * 32) << 16);
 
     auto chunk_of = [&](int it) { return a.reverse ? nch - 1 - it : it; };
     auto stage_x = [&](int s) { return sA_u + S::A_BYTES + s * S::STAGE; };
@@ -101,16 +105,24 @@ __global__ void __launch_bounds__(128, 1)
         for (int it = 0; it < S::STAGES - 1 && it < nch; ++it) issue(it);
 
     constexpr uint32_t idesc = idesc_bf16_f32(128, DK) | (XMN ? 1u << 16 : 0u);
+    // log gamma_C of the chunk processed at step `it` (loaded one step ahead so the load latency hides)
+    auto log_decay = [&](int it) {
+        const int c = chunk_of(it);
+        const long long idx = (long long)(s0 + c) * a.H + h;
+        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+        return __ldg(a.Gb + idx * 64 + L - 1);
+    };
+    float g_next = nch > 0 ? log_decay(0) : 0.f;
     for (int it = 0; it < nch; ++it) {
         const int c = chunk_of(it), s = it % S::STAGES;
         const long long idx = (long long)(s0 + c) * a.H + h;
-        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
-        const float gam = expf(a.Gb[idx * 64 + L - 1]);
+        const float gam = expf(g_next);
+        if (it + 1 < nch) g_next = log_decay(it + 1);
 
         // The state this chunk starts from: A operand (bf16, swizzled) and per-chunk output.
-        bf16* out = reinterpret_cast<bf16*>(a.Sout) + (idx * DV + j) * DK;
+        bf16* out = reinterpret_cast<bf16*>(a.Sout) + (idx * DV + j) * DK + c0;
 #pragma unroll
-        for (int q = 0; q < DK / 8; ++q) {
+        for (int q = 0; q < HC / 8; ++q) {
             __nv_bfloat162 v0 = __floats2bfloat162_rn(st[8 * q + 0], st[8 * q + 1]);
             __nv_bfloat162 v1 = __floats2bfloat162_rn(st[8 * q + 2], st[8 * q + 3]);
             __nv_bfloat162 v2 = __floats2bfloat162_rn(st[8 * q + 4], st[8 * q + 5]);
@@ -120,7 +132,7 @@ __global__ void __launch_bounds__(128, 1)
             pk.y = *reinterpret_cast<uint32_t*>(&v1);
             pk.z = *reinterpret_cast<uint32_t*>(&v2);
             pk.w = *reinterpret_cast<uint32_t*>(&v3);
-            *reinterpret_cast<uint4*>(sA + sw128_offset(j, 8 * q, 128)) = pk;
+            *reinterpret_cast<uint4*>(sA + sw128_offset(j, c0 + 8 * q, 128)) = pk;
             if (live) *reinterpret_cast<uint4*>(out + 8 * q) = pk;
         }
         fence_async_smem();
@@ -154,21 +166,21 @@ __global__ void __launch_bounds__(128, 1)
         }
         tc_fence_after();
 
-        // S^T <- gamma S^T + (S^T X^T) + Y
+        // S^T <- gamma S^T + (S^T X^T) + Y   (this thread's HC columns)
         const uint8_t* sY = smem + S::A_BYTES + s * S::STAGE + S::X_BYTES;
 #pragma unroll
-        for (int g = 0; g < DK / 32; ++g) {
-            float d[32];
-            tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + g * 32, d);
+        for (int g = 0; g < HC / 16; ++g) {
+            float d[16];
+            tmem_ld16(tlane + c0 + g * 16, d);
             if (live) {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint4 yv = *reinterpret_cast<const uint4*>(sY + sw128_offset(j, 32 * g + 8 * q, DV));
+                for (int q = 0; q < 2; ++q) {
+                    const uint4 yv = *reinterpret_cast<const uint4*>(sY + sw128_offset(j, c0 + 16 * g + 8 * q, DV));
                     const __nv_bfloat162* y2 = reinterpret_cast<const __nv_bfloat162*>(&yv);
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
                         const float2 yf = __bfloat1622float2(y2[e]);
-                        const int m = 32 * g + 8 * q + 2 * e;
+                        const int m = 16 * g + 8 * q + 2 * e;
                         st[m] = fmaf(gam, st[m], d[8 * q + 2 * e] + yf.x);
                         st[m + 1] = fmaf(gam, st[m + 1], d[8 * q + 2 * e + 1] + yf.y);
                     }
@@ -184,7 +196,7 @@ __global__ void __launch_bounds__(128, 1)
     if (a.fin && live) {
         float* fin = a.fin + ((long long)n * a.H + h) * DK * DV;
 #pragma unroll
-        for (int m = 0; m < DK; ++m) fin[(long long)m * DV + j] = st[m];
+        for (int m = 0; m < HC; ++m) fin[(long long)(c0 + m) * DV + j] = st[m];
     }
 }
 
@@ -232,7 +244,7 @@ __global__ void __launch_bounds__(128) k_scan_simt(ScanArgs a) {
         const int c = a.reverse ? nch - 1 - it : it;
         const long long idx = (long long)(s0 + c) * a.H + h;
         const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
-        const float gam = expf(a.Gb[idx * 64 + L - 1]);
+        const float gam = expf(__ldg(a.Gb + idx * 64 + L - 1));
         load_tile_async<float>(sX, S::PK, reinterpret_cast<const float*>(a.X) + idx * DK * DK, DK, DK, DK, DK, tid,
                                128);
         load_tile_async<float>(sY, S::PK, reinterpret_cast<const float*>(a.Y) + (idx * DV + j0) * DK, DK, 64, DK, 64,
@@ -308,7 +320,7 @@ static cudaError_t run_scan_tc(const ScanArgs& a, long long pairs, cudaStream_t 
     cudaError_t e = cudaFuncSetAttribute(k_scan_tc<DK, DV, XMN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)S::bytes());
     if (e) return e;
-    k_scan_tc<DK, DV, XMN><<<dim3(a.N, a.H), 128, S::bytes(), s>>>(a, tx, ty);
+    k_scan_tc<DK, DV, XMN><<<dim3(a.N, a.H), 256, S::bytes(), s>>>(a, tx, ty);
     return cudaGetLastError();
 }
 
