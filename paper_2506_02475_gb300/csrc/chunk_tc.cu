@@ -565,6 +565,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
+
 }  // namespace tc
 
 // -------------------------------------------------------------- launchers

@@ -384,6 +384,19 @@ __device__ __forceinline__ void tc_gemm(uint32_t tmem, uint32_t a, int a_ext, ui
     }
 }
 
+// Same with M = 64: D row m lives in TMEM lane 32*(m/16) + m%16 (lanes 0-15 of
+// each warp's quadrant), column n in column n.
+template <bool AMN, bool BMN>
+__device__ __forceinline__ void tc_gemm_m64(uint32_t tmem, uint32_t a, int a_ext, uint32_t b, int b_ext, int N, int K,
+                                            bool accumulate) {
+    const uint32_t idesc = idesc_bf16_f32(64, N) | (AMN ? 1u << 15 : 0u) | (BMN ? 1u << 16 : 0u);
+    for (int ks = 0; ks < K / 16; ++ks) {
+        const uint64_t ad = AMN ? desc_mnmajor(a, a_ext, ks) : desc_kmajor(a, a_ext, ks);
+        const uint64_t bd = BMN ? desc_mnmajor(b, b_ext, ks) : desc_kmajor(b, b_ext, ks);
+        tc_mma_bf16(tmem, ad, bd, idesc, (accumulate || ks > 0) ? 1u : 0u);
+    }
+}
+
 // Byte offset of element (mn, k) of an MN-major bf16 tile (allocated K extent krows).
 __host__ __device__ constexpr uint32_t mn128_offset(int mn, int k, int krows) {
     return (uint32_t)((mn >> 6) * krows * 128 + k * 128 + ((((mn & 63) >> 3) ^ (k & 7)) << 4) + (mn & 7) * 2);
@@ -401,6 +414,16 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
+
+// Issue a 16-column TMEM load without waiting; complete with tmem_wait_ld().
+__device__ __forceinline__ void tmem_ld16_async(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
 
 // Byte offset of element (row, k) of a K-major bf16 tile in the 128-byte swizzle
 // layout: K is split in halves of 64 elements, each a [rows][128 B] block.

@@ -119,21 +119,19 @@ __global__ void __launch_bounds__(256, 1)
         const float gam = expf(g_next);
         if (it + 1 < nch) g_next = log_decay(it + 1);
 
-        // The state this chunk starts from: A operand (bf16, swizzled) and per-chunk output.
-        bf16* out = reinterpret_cast<bf16*>(a.Sout) + (idx * DV + j) * DK + c0;
+        // The state this chunk starts from: the MMA's A operand (bf16, swizzled) ...
+        uint4 pk[HC / 8];
 #pragma unroll
         for (int q = 0; q < HC / 8; ++q) {
             __nv_bfloat162 v0 = __floats2bfloat162_rn(st[8 * q + 0], st[8 * q + 1]);
             __nv_bfloat162 v1 = __floats2bfloat162_rn(st[8 * q + 2], st[8 * q + 3]);
             __nv_bfloat162 v2 = __floats2bfloat162_rn(st[8 * q + 4], st[8 * q + 5]);
             __nv_bfloat162 v3 = __floats2bfloat162_rn(st[8 * q + 6], st[8 * q + 7]);
-            uint4 pk;
-            pk.x = *reinterpret_cast<uint32_t*>(&v0);
-            pk.y = *reinterpret_cast<uint32_t*>(&v1);
-            pk.z = *reinterpret_cast<uint32_t*>(&v2);
-            pk.w = *reinterpret_cast<uint32_t*>(&v3);
-            *reinterpret_cast<uint4*>(sA + sw128_offset(j, c0 + 8 * q, 128)) = pk;
-            if (live) *reinterpret_cast<uint4*>(out + 8 * q) = pk;
+            pk[q].x = *reinterpret_cast<uint32_t*>(&v0);
+            pk[q].y = *reinterpret_cast<uint32_t*>(&v1);
+            pk[q].z = *reinterpret_cast<uint32_t*>(&v2);
+            pk[q].w = *reinterpret_cast<uint32_t*>(&v3);
+            *reinterpret_cast<uint4*>(sA + sw128_offset(j, c0 + 8 * q, 128)) = pk[q];
         }
         fence_async_smem();
         tc_fence_before();
@@ -142,8 +140,6 @@ __global__ void __launch_bounds__(256, 1)
 
         int bad = 0;
         if (tid == 0) {
-            // Refill the stage that chunk it-1 used (everyone is past its epilogue now).
-            if (it + S::STAGES - 1 < nch) issue(it + S::STAGES - 1);
             if (mbar_wait(smem_u32(&full_bar[s]), (it / S::STAGES) & 1)) {
 #pragma unroll
                 for (int ks = 0; ks < DK / 16; ++ks) {
@@ -157,6 +153,14 @@ __global__ void __launch_bounds__(256, 1)
                 bad = 1;
             }
             tc_commit(smem_u32(&mma_bar));
+            // Refill the stage that chunk it-1 used (everyone is past its epilogue now).
+            if (it + S::STAGES - 1 < nch) issue(it + S::STAGES - 1);
+        }
+        // ... and the per-chunk state output, written while the MMA runs.
+        if (live) {
+            bf16* out = reinterpret_cast<bf16*>(a.Sout) + (idx * DV + j) * DK + c0;
+#pragma unroll
+            for (int q = 0; q < HC / 8; ++q) *reinterpret_cast<uint4*>(out + 8 * q) = pk[q];
         }
         if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
         if (!mbar_wait(smem_u32(&full_bar[s]), (it / S::STAGES) & 1)) bad = 1;
@@ -166,25 +170,25 @@ __global__ void __launch_bounds__(256, 1)
         }
         tc_fence_after();
 
-        // S^T <- gamma S^T + (S^T X^T) + Y   (this thread's HC columns)
+        // S^T <- gamma S^T + (S^T X^T) + Y   (this thread's HC columns; all TMEM loads in flight at once)
         const uint8_t* sY = smem + S::A_BYTES + s * S::STAGE + S::X_BYTES;
+        uint32_t d[HC / 16][16];
 #pragma unroll
-        for (int g = 0; g < HC / 16; ++g) {
-            float d[16];
-            tmem_ld16(tlane + c0 + g * 16, d);
-            if (live) {
+        for (int g = 0; g < HC / 16; ++g) tmem_ld16_async(tlane + c0 + g * 16, d[g]);
+        uint4 yv[HC / 8];
 #pragma unroll
-                for (int q = 0; q < 2; ++q) {
-                    const uint4 yv = *reinterpret_cast<const uint4*>(sY + sw128_offset(j, c0 + 16 * g + 8 * q, DV));
-                    const __nv_bfloat162* y2 = reinterpret_cast<const __nv_bfloat162*>(&yv);
+        for (int q = 0; q < HC / 8; ++q)
+            yv[q] = live ? *reinterpret_cast<const uint4*>(sY + sw128_offset(j, c0 + 8 * q, DV)) : make_uint4(0, 0, 0, 0);
+        tmem_wait_ld();
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float2 yf = __bfloat1622float2(y2[e]);
-                        const int m = 16 * g + 8 * q + 2 * e;
-                        st[m] = fmaf(gam, st[m], d[8 * q + 2 * e] + yf.x);
-                        st[m + 1] = fmaf(gam, st[m + 1], d[8 * q + 2 * e + 1] + yf.y);
-                    }
-                }
+        for (int q = 0; q < HC / 8; ++q) {
+            const __nv_bfloat162* y2 = reinterpret_cast<const __nv_bfloat162*>(&yv[q]);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float2 yf = __bfloat1622float2(y2[e]);
+                const int m = 8 * q + 2 * e;
+                st[m] = fmaf(gam, st[m], __uint_as_float(d[m >> 4][m & 15]) + yf.x);
+                st[m + 1] = fmaf(gam, st[m + 1], __uint_as_float(d[(m + 1) >> 4][(m + 1) & 15]) + yf.y);
             }
         }
         tc_fence_before();
