@@ -45,22 +45,40 @@ def build(force: bool = False) -> str:
     return _LIB_PATH
 
 
+def _bind(lib):
+    P = ctypes.c_void_p
+    I = ctypes.c_int
+    lib.comba_oracle_fwd.argtypes = [I, P, I, I, I] + [P] * 10 + [I]
+    lib.comba_oracle_fwd.restype = I
+    lib.comba_oracle_bwd.argtypes = [I, P, I, I, I] + [P] * 8 + [P, P] + [P] * 8 + [I]
+    lib.comba_oracle_bwd.restype = I
+    lib.comba_oracle_step.argtypes = [I, I, I, I] + [P] * 9 + [I]
+    lib.comba_oracle_step.restype = I
+    return lib
+
+
 def _load():
     global _lib
     with _lock:
-        if _lib is not None:
-            return _lib
-        lib = ctypes.CDLL(build())
-        P = ctypes.c_void_p
-        I = ctypes.c_int
-        lib.comba_oracle_fwd.argtypes = [I, P, I, I, I] + [P] * 10 + [I]
-        lib.comba_oracle_fwd.restype = I
-        lib.comba_oracle_bwd.argtypes = [I, P, I, I, I] + [P] * 8 + [P, P] + [P] * 8 + [I]
-        lib.comba_oracle_bwd.restype = I
-        lib.comba_oracle_step.argtypes = [I, I, I, I] + [P] * 9 + [I]
-        lib.comba_oracle_step.restype = I
-        _lib = lib
-        return lib
+        if _lib is None:
+            _lib = _bind(ctypes.CDLL(build()))
+        return _lib
+
+
+def build_variant(source_text: str, out_dir: str) -> str:
+    """Compile an edited copy of the oracle source (used by tests that plant mistakes)."""
+    os.makedirs(out_dir, exist_ok=True)
+    src = os.path.join(out_dir, "variant.c")
+    lib = os.path.join(out_dir, "libvariant.so")
+    with open(src, "w") as f:
+        f.write(source_text)
+    subprocess.run(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-pthread", "-o", lib, src], check=True)
+    return lib
+
+
+def source_text() -> str:
+    with open(_SRC) as f:
+        return f.read()
 
 
 def default_threads() -> int:
@@ -94,7 +112,7 @@ def _packed(q, k, v, alpha, beta, cu_seqlens):
     return q, k, v, alpha, beta, cu, shape
 
 
-def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None):
+def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=None):
     """Token recurrence forward.  Returns ``(o, hT)`` in float64."""
     q, k, v, alpha, beta, b, d, h0 = map(_f64, (q, k, v, alpha, beta, b, d, h0))
     q, k, v, alpha, beta, cu, shape = _packed(q, k, v, alpha, beta, cu_seqlens)
@@ -104,7 +122,7 @@ def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None):
     q, k, v, alpha, beta = map(np.ascontiguousarray, (q, k, v, alpha, beta))
     o = np.zeros((Ttot, H, dv), np.float64)
     hT = np.zeros((N, H, dk, dv), np.float64)
-    rc = _load().comba_oracle_fwd(N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta),
+    rc = (lib or _load()).comba_oracle_fwd(N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta),
                                   _ptr(b), _ptr(d), _ptr(h0), _ptr(o), _ptr(hT), threads or default_threads())
     if rc:
         raise MemoryError("oracle forward failed to allocate")
@@ -113,7 +131,7 @@ def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None):
     return o, hT
 
 
-def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, threads=None):
+def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, threads=None, lib=None):
     """Exact BPTT.  Returns a dict with dq, dk, dv, dalpha, dbeta, db, dd, dh0."""
     q, k, v, alpha, beta, b, d, h0, dO, dhT = map(_f64, (q, k, v, alpha, beta, b, d, h0, dO, dhT))
     batched = q.ndim == 4
@@ -129,7 +147,7 @@ def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, thre
         "dalpha": np.zeros((Ttot, H)), "dbeta": np.zeros((Ttot, H)),
         "db": np.zeros(H), "dd": np.zeros(H), "dh0": np.zeros((N, H, dk, dv)),
     }
-    rc = _load().comba_oracle_bwd(
+    rc = (lib or _load()).comba_oracle_bwd(
         N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b), _ptr(d), _ptr(h0),
         _ptr(dO), _ptr(dhT), _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]), _ptr(out["dalpha"]),
         _ptr(out["dbeta"]), _ptr(out["db"]), _ptr(out["dd"]), _ptr(out["dh0"]), threads or default_threads())
@@ -144,15 +162,20 @@ def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, thre
     return out
 
 
-def step(q, k, v, alpha, beta, b, d, state, threads=None):
+def step(q, k, v, alpha, beta, b, d, state, threads=None, lib=None):
     """One decode token.  ``state`` [Bd,H,dk,dv] is copied, updated and returned with ``o``."""
     q, k, v, alpha, beta, b, d = map(_f64, (q, k, v, alpha, beta, b, d))
     st = np.array(state, dtype=np.float64, copy=True, order="C")
     Bd, H, dk = q.shape
     dv = v.shape[-1]
     o = np.zeros((Bd, H, dv), np.float64)
-    rc = _load().comba_oracle_step(Bd, H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b),
+    rc = (lib or _load()).comba_oracle_step(Bd, H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b),
                                    _ptr(d), _ptr(st), _ptr(o), threads or default_threads())
     if rc:
         raise MemoryError("oracle step failed to allocate")
     return o, st
+
+
+def load_variant(path):
+    """ctypes handle of a compiled oracle variant, for the ``lib=`` argument of fwd/bwd/step."""
+    return _bind(ctypes.CDLL(path))
