@@ -218,11 +218,12 @@ def run_ours(args, world, rank, local):
     import torch
     dist = dist_init(world, local, "nccl")
     torch.cuda.set_device(local)
-    from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, inputs
+    from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, inputs, shard
     from paper_2506_02475_gb300 import binding
 
     peaks, peak_src = load_peaks()
-    w = inputs.make(args.workload)
+    # weak scaling: each rank owns its own batch of sequences (same parameters, own data)
+    w = inputs.make(args.workload, seed_offset=shard.rank_seed_offset(rank))
     dev = torch.device("cuda", local)
     tdt = torch.bfloat16
 
@@ -295,11 +296,7 @@ def run_ours(args, world, rank, local):
     clk = clocks.stop()
     if dist:
         dist.barrier()
-    ms = total_ms / args.steps
-    if dist:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = shard.max_over_ranks(total_ms / args.steps, dist, dev)
 
     tokens = w.tokens
     value = tokens * world / (ms / 1e3)
@@ -357,11 +354,7 @@ def run_ours(args, world, rank, local):
         end.record()
         end.synchronize()
         e_ms += start.elapsed_time(end)
-    e_ms /= args.steps
-    if dist:
-        t = torch.tensor([e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e_ms = float(t.item())
+    e_ms = shard.max_over_ranks(e_ms / args.steps, dist, dev)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -374,7 +367,7 @@ def run_ours(args, world, rank, local):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; paper's layer shape and gate ranges)",
             "config": {"workload": f"{args.workload}: " + workload_desc(w), "global_batch": w.num_seqs * world,
                        "seq_len": int(w.q.shape[1]) if w.cu_seqlens is None else int(w.tokens),
-                       "parallelism": f"replicas x{world} (no data-path collective)",
+                       "parallelism": f"data-parallel x{world}: each rank its own sequences, no data-path collective",
                        "l2": "flushed between timed steps (256 MiB write, outside the events)"},
             "tflops": tflops, "pct_bf16_peak": tflops / peaks["bf16_tflops"] * 100,
             "roofline": roof,
@@ -408,14 +401,15 @@ def run_decode(args, world, rank, local):
     import torch
     dist = dist_init(world, local, "nccl")
     torch.cuda.set_device(local)
-    from paper_2506_02475_gb300 import comba_recurrent_step, inputs
+    from paper_2506_02475_gb300 import comba_recurrent_step, inputs, shard
     peaks, peak_src = load_peaks()
     Bd, H, dk, dv = 256, 16, 128, 128
     dev = torch.device("cuda", local)
-    state = torch.from_numpy(inputs.decode_state(Bd, H, dk, dv)).to(dev)
+    off = shard.rank_seed_offset(rank)
+    state = torch.from_numpy(inputs.decode_state(Bd, H, dk, dv, seed_offset=off)).to(dev)
     toks = []
     for s in range(8):  # cycle over 8 distinct token sets
-        q, k, v, a, be, d = inputs.decode_tokens(s, Bd, H, dk, dv, "bf16")
+        q, k, v, a, be, d = inputs.decode_tokens(s, Bd, H, dk, dv, "bf16", seed_offset=off)
         toks.append([torch.from_numpy(x).to(dev).to(torch.bfloat16) for x in (q, k, v)] +
                     [torch.from_numpy(x).to(dev) for x in (a, be)])
     d = torch.from_numpy(d).to(dev)
@@ -426,6 +420,8 @@ def run_decode(args, world, rank, local):
         comba_recurrent_step(t[0], t[1], t[2], t[3], t[4], d, state, o=o)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(nvsmi_device_id())
+    if dist:
+        dist.barrier()
     torch.cuda.synchronize()
     clocks.start()
     total = 0.0
@@ -438,7 +434,9 @@ def run_decode(args, world, rank, local):
         end.synchronize()
         total += start.elapsed_time(end)
     clk = clocks.stop()
-    ms = total / args.steps
+    if dist:
+        dist.barrier()
+    ms = shard.max_over_ranks(total / args.steps, dist, dev)
     per = ms / steps
     bytes_step = Bd * H * (2 * dk * dv * 4 + (2 * dk + 2 * dv) * 2 + 8)
     gbs = bytes_step / (per / 1e3) / 1e9
@@ -453,6 +451,8 @@ def run_decode(args, world, rank, local):
                          "frac": gbs / peaks["hbm_gbs"], "kernel": "k_step", "launch_ms": per, "traffic": None,
                          "peak_source": peak_src},
             "clocks": clk, "gpu_launches": steps * args.steps}), flush=True)
+    if dist:
+        dist.destroy_process_group()
 
 
 # --------------------------------------------------------------- reference

@@ -165,11 +165,14 @@ def make(name: str, *, B=None, T=None, H=None, dk=None, dv=None, dtype=None, see
         N = B
     q, k, v = _tokens(rng, lead, H, dk, dv, dtype)
     alpha, beta = _gates(rng, lead + (H,))
+    # per-head parameters come from their own generator: ranks of a data-parallel
+    # run (different seed_offset) share d and b and differ only in their data
+    prng = np.random.Generator(np.random.PCG64(SEED + 1000 * off + 500))
     if name == "tiny_fp32":
         d = np.full(H, 0.5, np.float32)
     else:
-        d = rng.uniform(0.0, 1.0, size=H).astype(np.float32)
-    b = rng.uniform(0.0, 1.0, size=H).astype(np.float32) if with_b else None
+        d = prng.uniform(0.0, 1.0, size=H).astype(np.float32)
+    b = prng.uniform(0.0, 1.0, size=H).astype(np.float32) if with_b else None
     h0 = (0.1 * rng.standard_normal((N, H, dk, dv))).astype(np.float32) if with_h0 else None
     dO = dhT = None
     if with_grads:
@@ -219,6 +222,6 @@ def decode_tokens(step, Bd=256, H=16, dk=128, dv=128, dtype="bf16", seed_offset=
     rng = np.random.Generator(np.random.PCG64([SEED + 7000 + seed_offset, step]))
     q, k, v = _tokens(rng, (Bd,), H, dk, dv, dtype)
     alpha, beta = _gates(rng, (Bd, H))
-    drng = np.random.Generator(np.random.PCG64(SEED + 8000 + seed_offset))
+    drng = np.random.Generator(np.random.PCG64(SEED + 8000))   # a parameter: shared by every rank
     d = drng.uniform(0.0, 1.0, size=H).astype(np.float32)
     return q, k, v, alpha, beta, d
