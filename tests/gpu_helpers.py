@@ -5,6 +5,17 @@ Error metric (per output tensor): max-norm relative error
     rel = max_i |x_i - r_i| / max_i |r_i|.
 Tolerances: 1e-4 for the fp32 storage path, 2e-2 for bf16 storage with fp32
 state and accumulation.
+
+The per-head parameter gradients db and dd are sums over every token of the
+batch of per-token contributions c_t (dd: -k_t . dq~_t, from the output
+correction q~ = q - d k; db: beta_t dbtilde_t, from btilde = b beta).  Their
+error is measured on the scale of that sum, max_h |x_h - r_h| / sum_t |c_t|:
+the bound a sum meets when each contribution meets the tolerance.  The plain
+relative error of such a sum is ill-conditioned (at the 340M layer shape the
+sum is about 1/4000 of sum_t |c_t|).  The contributions come from the
+oracle's outputs alone: c_t(dd) = -k_t . dq_t, and
+c_t(db) = (beta_t dbeta_t - v_t . dv_t) / b, since dbeta = v . de + b dbtilde
+and dv = beta de.
 """
 import numpy as np
 import torch
@@ -18,6 +29,33 @@ def rel(x, ref):
     ref = np.asarray(ref, np.float64)
     den = np.abs(ref).max()
     return float(np.abs(x - ref).max() / den) if den > 0 else float(np.abs(x).max())
+
+
+def _heads_last(x):
+    """[..., H] -> [tokens, H]."""
+    return x.reshape(-1, x.shape[-1])
+
+
+def param_grad_scales(k, v, beta, b, ref):
+    """Per-head sums of |per-token contribution| to dd and db (see the module docstring)."""
+    k, v, beta = (np.asarray(x, np.float64) for x in (k, v, beta))
+    H = k.shape[-2]
+    cdd = -np.einsum("...hd,...hd->...h", k, ref["dq"])
+    bh = np.ones(H) if b is None else np.asarray(b, np.float64)
+    cdb = (beta * ref["dbeta"] - np.einsum("...hd,...hd->...h", v, ref["dv"])) / bh
+    return {"dd": np.abs(_heads_last(cdd)).sum(0), "db": np.abs(_heads_last(cdb)).sum(0)}
+
+
+def rel_sum(x, ref, scale):
+    """max_h |x_h - r_h| / scale_h for per-head sums over tokens."""
+    x, ref, scale = (np.asarray(a, np.float64).reshape(-1) for a in (x, ref, scale))
+    return float(np.max(np.abs(x - ref) / np.maximum(scale, 1e-300)))
+
+
+def param_grad_errors(g, ref, k, v, beta, b):
+    """dd and db errors on the summation scale."""
+    sc = param_grad_scales(k, v, beta, b, ref)
+    return {key: rel_sum(g[key], ref[key], sc[key]) for key in ("dd", "db")}
 
 
 def tol(dtype):

@@ -11,7 +11,7 @@ import pytest
 import torch
 
 import oracle
-from gpu_helpers import np64, rel, to_dev, tol
+from gpu_helpers import np64, param_grad_errors, rel, to_dev, tol
 from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, inputs
 
 pytestmark = pytest.mark.gpu
@@ -49,8 +49,7 @@ def check_bwd(w, t=None):
     g = gpu_bwd(t)
     r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens)
     errs = {key: rel(g[key], r[key]) for key in GRADS}
-    errs["dd"] = rel(g["dd"], r["dd"])
-    errs["db"] = rel(g["db"], r["db"])
+    errs.update(param_grad_errors(g, r, w.k, w.v, w.beta, w.b))
     bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
     assert not bad, (bad, errs)
     return errs
@@ -169,8 +168,8 @@ def test_full_size_workload_sampled_heads(name, heads):
         for key in ("dalpha", "dbeta"):
             errs[key] = rel(np64(g[key][..., h:h + 1]), r[key])
         errs["dh0"] = rel(np64(g["dh0"][:, h:h + 1]), r["dh0"])
-        errs["dd"] = rel(np64(g["dd"][h:h + 1]), r["dd"])
-        errs["db"] = rel(np64(g["db"][h:h + 1]), r["db"])
+        errs.update(param_grad_errors({"dd": np64(g["dd"][h:h + 1]), "db": np64(g["db"][h:h + 1])}, r,
+                                      s["k"], s["v"], s["beta"], s["b"]))
         bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
         assert not bad, (name, h, bad, errs)
 
@@ -197,5 +196,7 @@ def test_backward_reusing_saved_forward_factors(dtype, d, lens):
     o2, hT2 = gpu_fwd(t)
     assert np.array_equal(np64(o), o2) and np.array_equal(np64(hT), hT2)
     r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens)
-    for key in GRADS + ("dd", "db"):
+    for key in GRADS:
         assert rel(g[key], r[key]) <= tol(w.dtype), key
+    for key, e in param_grad_errors(g, r, w.k, w.v, w.beta, w.b).items():
+        assert e <= tol(w.dtype), key

@@ -317,3 +317,16 @@ def test_thread_count_does_not_change_bits():
     g4 = oracle.bwd(dO=dO, threads=4, **p)
     for key in g1:
         assert np.array_equal(g1[key], g4[key]), key
+
+
+def test_param_gradients_are_sums_of_token_contributions():
+    """dd = -sum_t k_t . dq~_t (q~ = q - d k, section 3) and db = sum_t beta_t dbtilde_t with
+    dbtilde_t = (dbeta_t - v_t . dv_t / beta_t) / b (btilde = b beta, section 3.1; dv = beta de):
+    the per-head sums rebuilt from the oracle's per-token outputs equal its db and dd."""
+    from paper_2506_02475_gb300 import inputs
+    w = inputs.make("custom", B=2, T=100, H=3, dk=8, dv=8, with_b=True, with_h0=True, with_grads=True, dtype="f32")
+    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT)
+    cdd = -np.einsum("bthd,bthd->h", w.k, r["dq"])
+    cdb = ((w.beta * r["dbeta"] - np.einsum("bthd,bthd->bth", w.v, r["dv"])) / w.b).sum((0, 1))
+    np.testing.assert_allclose(cdd, r["dd"], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(cdb, r["db"], rtol=1e-12, atol=1e-12)
