@@ -14,10 +14,15 @@
 // from (H_n^T, or dH_{n+1}^T in the backward) for the parallel kernels.
 //
 // bf16 storage: one CTA per (sequence, head), 256 threads (two per state row,
-// each holding half of the row's dk columns); the fp32 state stays in registers; S^T (bf16) is written into a 128-byte-swizzled K-major
-// shared tile; X and Y stream in by TMA through a multi-stage mbarrier
-// pipeline; one thread issues the tcgen05 MMAs (M = 128, N = dk, K = dk)
-// into a TMEM accumulator that all threads read back with tcgen05.ld.
+// each holding half of the row's dk columns); the fp32 state stays in registers.
+// Each chunk, S^T (bf16) is written into one of two 128-byte-swizzled K-major
+// shared tiles: it is the MMA's A operand and, by a bulk tensor store issued
+// right after the MMAs, the chunk's stored starting state (one SM writes
+// global memory at only a few tens of bytes per cycle, so the store must not
+// sit on the chunk-to-chunk path; it drains while the next chunks compute).
+// X and Y stream in by TMA through mbarrier pipelines (3 and 2 stages); one
+// thread issues the tcgen05 MMAs (M = 128, N = dk, K = dk) into a TMEM
+// accumulator that all threads read back with tcgen05.ld.
 // fp32 storage: the same recurrence with FMA tile products (tolerance 1e-4).
 #include <cuda.h>
 
@@ -38,21 +43,35 @@ __device__ __forceinline__ void scan_seq_range(const ScanArgs& a, int n, long lo
 
 template <int DK, int DV>
 struct ScanTcSmem {
-    static constexpr int STAGES = DK == 128 ? 3 : 4;
-    static constexpr uint32_t A_BYTES = 128 * DK * 2;   // S^T tile, M = 128 rows (rows >= DV are zero)
+    static constexpr int SX = 3;                          // X stages (refilled once the MMA that read them is done)
+    static constexpr int SY = 2;                          // Y stages (refilled once the epilogue that read them is done)
+    static constexpr uint32_t A_BYTES = 128 * DK * 2;     // S^T tile, M = 128 rows (rows >= DV are zero); two buffers
     static constexpr uint32_t X_BYTES = DK * DK * 2;
     static constexpr uint32_t Y_BYTES = DV * DK * 2;
-    static constexpr uint32_t STAGE = X_BYTES + Y_BYTES;
-    static constexpr size_t bytes() { return 1024 + A_BYTES + STAGES * (size_t)STAGE; }
+    static constexpr uint32_t OX = 2 * A_BYTES;
+    static constexpr uint32_t OY = OX + SX * X_BYTES;
+    static constexpr size_t bytes() { return 1024 + OY + (size_t)SY * Y_BYTES; }
 };
+
+__device__ __forceinline__ void tma_store_2d(const void* tmap, int x, int y, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];\n"
+                 ::"l"(tmap), "r"(x), "r"(y), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
+// Wait until at most N bulk groups still read shared memory (resp. are incomplete).
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read %0;\n" ::"n"(N) : "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
 
 template <int DK, int DV, bool XMN>
 __global__ void __launch_bounds__(256, 1)
-    k_scan_tc(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY) {
+    k_scan_tc(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY,
+              const __grid_constant__ CUtensorMap tmS) {
     using S = ScanTcSmem<DK, DV>;
     constexpr int HC = DK / 2;  // state columns per thread: two threads per state row
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t full_bar[S::STAGES];
+    __shared__ uint64_t full_x[S::SX], full_y[S::SY];
     __shared__ uint64_t mma_bar;
     __shared__ uint32_t tmem_base;
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -61,8 +80,7 @@ __global__ void __launch_bounds__(256, 1)
     const int j = tid & 127;           // state row (dv index); warps w and w+4 share TMEM lanes
     const int c0 = (tid >> 7) * HC;    // first state column of this thread
     const bool live = j < DV;
-    uint8_t* sA = smem;
-    const uint32_t sA_u = smem_u32(sA);
+    const uint32_t smem_u = smem_u32(smem);
 
     float st[HC];
     const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
@@ -76,7 +94,8 @@ __global__ void __launch_bounds__(256, 1)
     if (s0 + nch > a.slots) nch = a.slots - s0 > 0 ? a.slots - s0 : 0;
 
     if (tid == 0) {
-        for (int s = 0; s < S::STAGES; ++s) mbar_init(smem_u32(&full_bar[s]), 1);
+        for (int s = 0; s < S::SX; ++s) mbar_init(smem_u32(&full_x[s]), 1);
+        for (int s = 0; s < S::SY; ++s) mbar_init(smem_u32(&full_y[s]), 1);
         mbar_init(smem_u32(&mma_bar), 1);
         mbar_fence_init();
     }
@@ -88,50 +107,57 @@ __global__ void __launch_bounds__(256, 1)
     const uint32_t tlane = tmem + ((uint32_t)((warp & 3) * 32) << 16);
 
     auto chunk_of = [&](int it) { return a.reverse ? nch - 1 - it : it; };
-    auto stage_x = [&](int s) { return sA_u + S::A_BYTES + s * S::STAGE; };
-    auto stage_y = [&](int s) { return sA_u + S::A_BYTES + s * S::STAGE + S::X_BYTES; };
-    auto issue = [&](int it) {
-        const int s = it % S::STAGES;
-        const long long idx = (long long)(s0 + chunk_of(it)) * a.H + h;
-        const uint32_t fb = smem_u32(&full_bar[s]);
-        mbar_expect_tx(fb, S::STAGE);
+    auto unit_of = [&](int it) { return (long long)(s0 + chunk_of(it)) * a.H + h; };
+    auto a_buf = [&](int it) { return smem_u + (uint32_t)(it & 1) * S::A_BYTES; };
+    auto x_buf = [&](int it) { return smem_u + S::OX + (uint32_t)(it % S::SX) * S::X_BYTES; };
+    auto y_off = [&](int it) { return S::OY + (uint32_t)(it % S::SY) * S::Y_BYTES; };
+    auto issue_x = [&](int it) {
+        const uint32_t fb = smem_u32(&full_x[it % S::SX]);
+        mbar_expect_tx(fb, S::X_BYTES);
 #pragma unroll
-        for (int half = 0; half < DK / 64; ++half) {
-            tma_load_2d(stage_x(s) + half * DK * 128, &tmX, half * 64, (int)(idx * DK), fb);
-            tma_load_2d(stage_y(s) + half * DV * 128, &tmY, half * 64, (int)(idx * DV), fb);
-        }
+        for (int half = 0; half < DK / 64; ++half)
+            tma_load_2d(x_buf(it) + half * DK * 128, &tmX, half * 64, (int)(unit_of(it) * DK), fb);
     };
-    if (tid == 0)
-        for (int it = 0; it < S::STAGES - 1 && it < nch; ++it) issue(it);
+    auto issue_y = [&](int it) {
+        const uint32_t fb = smem_u32(&full_y[it % S::SY]);
+        mbar_expect_tx(fb, S::Y_BYTES);
+#pragma unroll
+        for (int half = 0; half < DK / 64; ++half)
+            tma_load_2d(smem_u + y_off(it) + half * DV * 128, &tmY, half * 64, (int)(unit_of(it) * DV), fb);
+    };
+    int nx = 0, ny = 0;   // chunks whose X / Y loads have been issued (thread 0)
+    if (tid == 0) {
+        for (; nx < S::SX - 1 && nx < nch; ++nx) issue_x(nx);
+        for (; ny < S::SY - 1 && ny < nch; ++ny) issue_y(ny);
+    }
 
     constexpr uint32_t idesc = idesc_bf16_f32(128, DK) | (XMN ? 1u << 16 : 0u);
     // log gamma_C of the chunk processed at step `it` (loaded one step ahead so the load latency hides)
     auto log_decay = [&](int it) {
         const int c = chunk_of(it);
-        const long long idx = (long long)(s0 + c) * a.H + h;
         const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
-        return __ldg(a.Gb + idx * 64 + L - 1);
+        return __ldg(a.Gb + unit_of(it) * 64 + L - 1);
     };
     float g_next = nch > 0 ? log_decay(0) : 0.f;
     for (int it = 0; it < nch; ++it) {
-        const int c = chunk_of(it), s = it % S::STAGES;
-        const long long idx = (long long)(s0 + c) * a.H + h;
         const float gam = expf(g_next);
         if (it + 1 < nch) g_next = log_decay(it + 1);
 
-        // The state this chunk starts from: the MMA's A operand (bf16, swizzled) ...
-        uint4 pk[HC / 8];
+        // The state this chunk starts from, as the MMA's A operand (bf16, swizzled, buffer it % 2;
+        // the bulk store that read this buffer two chunks ago has finished reading it).
+        uint8_t* sA = smem + (it & 1) * S::A_BYTES;
 #pragma unroll
         for (int q = 0; q < HC / 8; ++q) {
             __nv_bfloat162 v0 = __floats2bfloat162_rn(st[8 * q + 0], st[8 * q + 1]);
             __nv_bfloat162 v1 = __floats2bfloat162_rn(st[8 * q + 2], st[8 * q + 3]);
             __nv_bfloat162 v2 = __floats2bfloat162_rn(st[8 * q + 4], st[8 * q + 5]);
             __nv_bfloat162 v3 = __floats2bfloat162_rn(st[8 * q + 6], st[8 * q + 7]);
-            pk[q].x = *reinterpret_cast<uint32_t*>(&v0);
-            pk[q].y = *reinterpret_cast<uint32_t*>(&v1);
-            pk[q].z = *reinterpret_cast<uint32_t*>(&v2);
-            pk[q].w = *reinterpret_cast<uint32_t*>(&v3);
-            *reinterpret_cast<uint4*>(sA + sw128_offset(j, c0 + 8 * q, 128)) = pk[q];
+            uint4 pk;
+            pk.x = *reinterpret_cast<uint32_t*>(&v0);
+            pk.y = *reinterpret_cast<uint32_t*>(&v1);
+            pk.z = *reinterpret_cast<uint32_t*>(&v2);
+            pk.w = *reinterpret_cast<uint32_t*>(&v3);
+            *reinterpret_cast<uint4*>(sA + sw128_offset(j, c0 + 8 * q, 128)) = pk;
         }
         fence_async_smem();
         tc_fence_before();
@@ -140,38 +166,47 @@ __global__ void __launch_bounds__(256, 1)
 
         int bad = 0;
         if (tid == 0) {
-            if (mbar_wait(smem_u32(&full_bar[s]), (it / S::STAGES) & 1)) {
+            if (mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
 #pragma unroll
                 for (int ks = 0; ks < DK / 16; ++ks) {
                     const int half = ks >> 2, sub = ks & 3;
-                    const uint64_t ad = smem_desc_sw128(sA_u + half * 128 * 128 + sub * 32);
-                    const uint64_t bd = XMN ? desc_mnmajor(stage_x(s), DK, ks)
-                                            : smem_desc_sw128(stage_x(s) + half * DK * 128 + sub * 32);
+                    const uint64_t ad = smem_desc_sw128(a_buf(it) + half * 128 * 128 + sub * 32);
+                    const uint64_t bd = XMN ? desc_mnmajor(x_buf(it), DK, ks)
+                                            : smem_desc_sw128(x_buf(it) + half * DK * 128 + sub * 32);
                     tc_mma_bf16(tmem, ad, bd, idesc, ks > 0 ? 1u : 0u);
                 }
             } else {
                 bad = 1;
             }
             tc_commit(smem_u32(&mma_bar));
-            // Refill the stage that chunk it-1 used (everyone is past its epilogue now).
-            if (it + S::STAGES - 1 < nch) issue(it + S::STAGES - 1);
-        }
-        // ... and the per-chunk state output, written while the MMA runs.
-        if (live) {
-            bf16* out = reinterpret_cast<bf16*>(a.Sout) + (idx * DV + j) * DK + c0;
+            // The chunk's starting state goes out by one bulk tensor store from the same tile,
+            // asynchronously: rows >= DV of the tile are not part of the box.
 #pragma unroll
-            for (int q = 0; q < HC / 8; ++q) *reinterpret_cast<uint4*>(out + 8 * q) = pk[q];
+            for (int half = 0; half < DK / 64; ++half)
+                tma_store_2d(&tmS, half * 64, (int)(unit_of(it) * DV), a_buf(it) + half * 128 * 128);
+            bulk_commit();
+            // Refill the stages chunk it-1 used: its MMA (X) and its epilogue (Y) are done.
+            if (nx < nch) issue_x(nx++);
+            if (ny < nch) issue_y(ny++);
         }
         if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
-        if (!mbar_wait(smem_u32(&full_bar[s]), (it / S::STAGES) & 1)) bad = 1;
+        if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1)) bad = 1;
+        // Before the next chunk packs into the other A buffer, the store issued one chunk ago
+        // (from that buffer) must have finished reading it.
+        if (tid == 0) bulk_wait_read<1>();
         if (__syncthreads_or(bad)) {
-            if (tid == 0 && a.err) atomicExch(a.err, 1);
+            if (tid == 0) {
+                if (a.err) atomicExch(a.err, 1);
+                // drain the loads still in flight into this CTA's shared memory (bounded waits)
+                for (int c = it; c < nx; ++c) mbar_wait(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
+                for (int c = it; c < ny; ++c) mbar_wait(smem_u32(&full_y[c % S::SY]), (c / S::SY) & 1);
+            }
             break;
         }
         tc_fence_after();
 
         // S^T <- gamma S^T + (S^T X^T) + Y   (this thread's HC columns; all TMEM loads in flight at once)
-        const uint8_t* sY = smem + S::A_BYTES + s * S::STAGE + S::X_BYTES;
+        const uint8_t* sY = smem + y_off(it);
         uint32_t d[HC / 16][16];
 #pragma unroll
         for (int g = 0; g < HC / 16; ++g) tmem_ld16_async(tlane + c0 + g * 16, d[g]);
@@ -194,6 +229,8 @@ __global__ void __launch_bounds__(256, 1)
         tc_fence_before();
     }
 
+    // every bulk store of this CTA completes before its shared memory is released
+    if (tid == 0) bulk_wait_all();
     __syncthreads();
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, DK);
@@ -318,13 +355,14 @@ static bool make_map(CUtensorMap* m, const void* base, long long rows, int cols,
 template <int DK, int DV, bool XMN>
 static cudaError_t run_scan_tc(const ScanArgs& a, long long pairs, cudaStream_t s) {
     using S = ScanTcSmem<DK, DV>;
-    CUtensorMap tx, ty;
-    if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, DV))
+    CUtensorMap tx, ty, ts;
+    if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, DV) ||
+        !make_map(&ts, a.Sout, pairs * DV, DK, DV))
         return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(k_scan_tc<DK, DV, XMN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)S::bytes());
     if (e) return e;
-    k_scan_tc<DK, DV, XMN><<<dim3(a.N, a.H), 256, S::bytes(), s>>>(a, tx, ty);
+    k_scan_tc<DK, DV, XMN><<<dim3(a.N, a.H), 256, S::bytes(), s>>>(a, tx, ty, ts);
     return cudaGetLastError();
 }
 
