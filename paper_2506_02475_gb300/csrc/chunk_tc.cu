@@ -93,10 +93,9 @@ struct PrepTcSmem {
     static constexpr uint32_t OV = OK + 32768;           // V  [64][128]               16 KB
     static constexpr uint32_t OMW = OV + 16384;          // Mw [64][64] K-major         8 KB
     static constexpr uint32_t OMU = OMW + 8192;          // Mu [64][64]                 8 KB
-    static constexpr uint32_t OR = OMU + 8192;           // A, M fp32 then sW^T, sU^T [128][64]
-    static constexpr uint32_t R_BYTES = 2 * 64 * 65 * 4 > 2 * 16384 ? 2 * 64 * 65 * 4 : 2 * 16384;
-    static constexpr uint32_t OT = OR + ((R_BYTES + 1023) & ~1023u);
-    static constexpr uint32_t OF = OT + 3 * 272 * 4;
+    static constexpr uint32_t OR = OMU + 8192;           // A^T (pitch 68), M (pitch 65), T fp32, then sW^T, sU^T [128][64]
+    static constexpr uint32_t R_BYTES = (64 * 68 + 64 * 65 + 32 * 36) * 4;
+    static constexpr uint32_t OF = OR + ((R_BYTES + 1023) & ~1023u);
     static constexpr size_t bytes() { return 1024 + OF + 64 * 6 * 4; }
 };
 
@@ -117,18 +116,29 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     uint8_t* sV = sm + S::OV;
     uint8_t* sMw = sm + S::OMW;
     uint8_t* sMu = sm + S::OMU;
-    float* sA = reinterpret_cast<float*>(sm + S::OR);
-    float* sM = sA + 64 * 65;
+    float* sAt = reinterpret_cast<float*>(sm + S::OR);   // A transposed, pitch 68
+    float* sM = sAt + 64 * 68;
+    float* sTi = sM + 64 * 65;                         // inverse scratch, 32 x 36
     uint8_t* sWt = sm + S::OR;            // aliases A after the inverse
     uint8_t* sUt = sm + S::OR + 16384;    // aliases M after Mw/Mu are built
-    float* sTmp = reinterpret_cast<float*>(sm + S::OT);
     float* sG = reinterpret_cast<float*>(sm + S::OF);
     float* sGm1 = sG + 64;
     float* sBt = sG + 128;
     float* sBe = sG + 192;
     float* sS = sG + 256;
+    float* sWs = sG + 320;   // btilde_c gamma_{c-1}: the column scale of Mw
 
-    load_sw(sK, 128, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    // K into both halves of the 128-row tile: rows 64..127 repeat rows 0..63, so the
+    // padded Gram product puts a copy of each Gram row in TMEM lanes r and r + 64.
+    {
+        const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
+        for (int e = tid; e < 128 * 16; e += 128) {
+            const int r = e >> 4, ch = e & 15, rr = r & 63;
+            const bool okr = rr < L;
+            cp_async16(sK + sw128_offset(r, ch * 8, 128),
+                       okr ? (const void*)(kg + (long long)rr * p.H * D + ch * 8) : (const void*)kg, okr);
+        }
+    }
     load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
     cp_async_commit();
     if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
@@ -137,6 +147,8 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
         sBe[tid] = be;
         sBt[tid] = (p.b ? p.b[h] : 1.f) * be;
     }
+    __syncthreads();   // sG, sGm1, sBt complete
+    if (tid < 64) sWs[tid] = sBt[tid] * expf(sGm1[tid]);
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
         mbar_fence_init();
@@ -155,23 +167,22 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;
     ok = ms.finish(tid);
     if (ok) {
-        // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T); exp only below the diagonal.
+        // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T), stored transposed; exp only
+        // below the diagonal.  Thread t holds Gram row t & 63 and fills columns [32 (t >> 6), +32).
+        const int r = row & 63, i0 = 32 * (row >> 6);
         float d[32];
+        tmem_ld32(trow + i0, d);
+        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
 #pragma unroll
-        for (int g = 0; g < 2; ++g) {
-            tmem_ld32(trow + g * 32, d);
-            if (row < 64) {
-#pragma unroll
-                for (int c = 0; c < 32; ++c) {
-                    const int i = 32 * g + c;
-                    sA[row * 65 + i] = (i < row && row < L) ? sBt[row] * expf(sGm1[row] - sG[i]) * d[c] : 0.f;
-                }
-            }
+        for (int c = 0; c < 32; ++c) {
+            const int i = i0 + c;
+            sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
         }
     }
     __syncthreads();
     if (ok) {
-        unit_lower_inverse64(sA, sM, sTmp, tid);
+        unit_lower_inverse64_blocked(sAt, sM, 65, sTi, tid);
+        __syncthreads();
         // Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta) as K-major [p][p'] tiles; M saved for the backward.
         bf16* Mg = p.Mb ? (bf16*)p.Mb + idx * 4096 : nullptr;
         for (int e = tid; e < 64 * 8; e += 128) {
@@ -181,7 +192,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
             for (int q = 0; q < 8; ++q) {
                 const int c = 8 * ch + q;
                 mm[q] = sM[r * 65 + c];
-                mw[q] = mm[q] * sBt[c] * expf(sGm1[c]);
+                mw[q] = mm[q] * sWs[c];
                 mu[q] = mm[q] * sBe[c];
             }
             *reinterpret_cast<uint4*>(sMw + sw128_offset(r, 8 * ch, 64)) = pack8(mw);

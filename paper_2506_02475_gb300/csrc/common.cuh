@@ -473,4 +473,83 @@ __device__ __forceinline__ void unit_lower_inverse64(const float* A, float* M, f
     }
 }
 
+// Diagonal 32 x 32 block [C0, C0+32) of (I + A)^{-1} for a strictly lower 64 x 64
+// A, by right-looking forward substitution: the calling thread owns column j of
+// the block and keeps the running row sums s_r = sum_{i<r} A_ri x_i of that
+// column in registers; each solved entry x_r updates the sums of the rows below
+// it.  At is A transposed (At[i][r] = A[r][i], pitch 68 floats, zero on and
+// above the diagonal of A), so an update reads one contiguous row of At (the
+// same address across the warp).  Writes rows [C0, C0+32) of column j of M
+// (pitch `pm`), and zeros above them.
+template <int C0>
+__device__ __forceinline__ void unit_lower_inverse_diag32(const float* At, float* M, int pm, int j) {
+    float s[32];
+#pragma unroll
+    for (int r = 0; r < 32; ++r) s[r] = 0.f;
+#pragma unroll
+    for (int r = C0; r < C0 + 32; ++r) {
+        const float x = r == j ? 1.f : (r < j ? 0.f : -s[r - C0]);
+        M[r * pm + j] = x;
+        // rows r2 >= 4 floor((r+1)/4) of the block: At[r][r2] = A[r2][r] is zero for r2 <= r,
+        // and the sums of rows <= r are no longer read, so aligned groups of four are updated whole
+#pragma unroll
+        for (int g = (r + 1) >> 2; g < (C0 + 32) / 4; ++g) {
+            const float4 a = *reinterpret_cast<const float4*>(At + r * 68 + 4 * g);
+            s[4 * g + 0 - C0] = fmaf(a.x, x, s[4 * g + 0 - C0]);
+            s[4 * g + 1 - C0] = fmaf(a.y, x, s[4 * g + 1 - C0]);
+            s[4 * g + 2 - C0] = fmaf(a.z, x, s[4 * g + 2 - C0]);
+            s[4 * g + 3 - C0] = fmaf(a.w, x, s[4 * g + 3 - C0]);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < C0; ++r) M[r * pm + j] = 0.f;
+}
+
+// (I + A)^{-1} for a strictly lower 64 x 64 A (128 threads), by 32 x 32 blocks:
+// M11 = (I + A11)^{-1} and M22 = (I + A22)^{-1} (warps 0 and 1, in registers),
+// then M21 = -M22 (A21 M11) with 4 x 2 register tiles per thread.  At as above;
+// M has pitch `pm`; T is 32 x 36 floats of scratch.  Rows past a short chunk
+// have A = 0 and come out as identity rows.
+__device__ __forceinline__ void unit_lower_inverse64_blocked(const float* At, float* M, int pm, float* T, int tid) {
+    if (tid < 32) unit_lower_inverse_diag32<0>(At, M, pm, tid);
+    else if (tid < 64) unit_lower_inverse_diag32<32>(At, M, pm, tid);
+    __syncthreads();
+    const int r0 = 4 * (tid >> 4), c0 = 2 * (tid & 15);
+    {
+        // T = A21 M11: T[r][c] = sum_k A[32 + r][k] M[k][c]
+        float t[4][2] = {};
+#pragma unroll 8
+        for (int k = 0; k < 32; ++k) {
+            const float4 a = *reinterpret_cast<const float4*>(At + k * 68 + 32 + r0);
+            const float m0 = M[k * pm + c0], m1 = M[k * pm + c0 + 1];
+            t[0][0] = fmaf(a.x, m0, t[0][0]); t[0][1] = fmaf(a.x, m1, t[0][1]);
+            t[1][0] = fmaf(a.y, m0, t[1][0]); t[1][1] = fmaf(a.y, m1, t[1][1]);
+            t[2][0] = fmaf(a.z, m0, t[2][0]); t[2][1] = fmaf(a.z, m1, t[2][1]);
+            t[3][0] = fmaf(a.w, m0, t[3][0]); t[3][1] = fmaf(a.w, m1, t[3][1]);
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) *reinterpret_cast<float2*>(T + (r0 + e) * 36 + c0) = make_float2(t[e][0], t[e][1]);
+    }
+    __syncthreads();
+    {
+        // M21 = -M22 T: M[32 + r][c] = -sum_k M[32 + r][32 + k] T[k][c]
+        float t[4][2] = {};
+#pragma unroll 8
+        for (int k = 0; k < 32; ++k) {
+            const float2 b = *reinterpret_cast<const float2*>(T + k * 36 + c0);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float m = M[(32 + r0 + e) * pm + 32 + k];
+                t[e][0] = fmaf(m, b.x, t[e][0]);
+                t[e][1] = fmaf(m, b.y, t[e][1]);
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            M[(32 + r0 + e) * pm + c0] = -t[e][0];
+            M[(32 + r0 + e) * pm + c0 + 1] = -t[e][1];
+        }
+    }
+}
+
 }  // namespace comba
