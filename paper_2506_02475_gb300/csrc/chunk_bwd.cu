@@ -100,7 +100,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep(ChunkParams p) {
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
-                const float v = (c <= r && r < L) ? sc[t][i] * expf(sG[r] - sG[c]) : 0.f;
+                const float v = (c <= r && r < L) ? sc[t][i] * __expf(sG[r] - sG[c]) : 0.f;
                 sP[r * S::PL + c] = from_f<T>(v);
             }
     }
@@ -163,7 +163,8 @@ struct LocalSmem {
         o = carve_bytes(o, sizeof(T) * DV * PK);   // H^T
         o = carve_bytes(o, sizeof(T) * DV * PK);   // dH'^T
         o = carve_bytes(o, sizeof(T) * 64 * PL);   // M
-        o = carve_bytes(o, sizeof(float) * 64 * 6);          // G, Gm1, beta, btilde, alpha, dg
+        o = carve_bytes(o, sizeof(T) * 64 * PV);   // dV staging (coalesced store at the end)
+        o = carve_bytes(o, sizeof(float) * 64 * 8);          // G, Gm1, beta, btilde, alpha, dg, e^{Gm1}, btilde e^{Gm1}
         o = carve_bytes(o, sizeof(float) * NROW * 2 * 64);   // row partials [kind][half][row]
         o = carve_bytes(o, sizeof(float) * 2 * 4 * 64);      // column partials [kind][rowblock][col]
         o = carve_bytes(o, sizeof(float) * 8);               // block reduction scratch
@@ -212,12 +213,15 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     T* sH = sc.take<T>(DV * PK);    // H_n^T  [dv][dk]
     T* sdH = sc.take<T>(DV * PK);   // dH'^T  [dv][dk]
     T* sM = sc.take<T>(64 * PL);
-    float* sG = sc.take<float>(64 * 6);
+    T* sDV = sc.take<T>(64 * PV);
+    float* sG = sc.take<float>(64 * 8);
     float* sGm1 = sG + 64;
     float* sBe = sG + 128;
     float* sBt = sG + 192;
     float* sAl = sG + 256;
     float* sDg = sG + 320;
+    float* sEm1 = sG + 384;   // gamma_{r-1}
+    float* sWs = sG + 448;    // btilde_r gamma_{r-1}
     float* rowp = sc.take<float>(S::NROW * 2 * 64);
     float* colp = sc.take<float>(2 * 4 * 64);
     float* red = sc.take<float>(8);
@@ -246,19 +250,34 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         sBe[tid] = be;
         sBt[tid] = bh * be;
         sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
+        const float em1 = tid > 0 ? __expf(p.Gb[idx * 64 + tid - 1]) : 1.f;
+        sEm1[tid] = em1;
+        sWs[tid] = bh * be * em1;
     }
     cp_async_wait<0>();
     __syncthreads();
-    for (int e = tid; e < 64 * DK; e += 256) {
-        const int r = e / DK, c = e % DK;
-        sQ[r * PK + c] = from_f<T>(to_f(sQ[r * PK + c]) - dh * to_f(sK[r * PK + c]));
+    constexpr int VE = 16 / (int)sizeof(T);   // elements per 16-byte vector
+    for (int e = tid; e < 64 * DK / VE; e += 256) {
+        const int r = e / (DK / VE), c = (e % (DK / VE)) * VE;
+        uint4 qv = *reinterpret_cast<const uint4*>(sQ + r * PK + c);
+        const uint4 kv = *reinterpret_cast<const uint4*>(sK + r * PK + c);
+        T* qe = reinterpret_cast<T*>(&qv);
+        const T* ke = reinterpret_cast<const T*>(&kv);
+#pragma unroll
+        for (int i = 0; i < VE; ++i) qe[i] = from_f<T>(to_f(qe[i]) - dh * to_f(ke[i]));
+        *reinterpret_cast<uint4*>(sQ + r * PK + c) = qv;
     }
     // <H, dH'> (block reduction in a fixed order)
     {
         float s = 0.f;
-        for (int e = tid; e < DK * DV; e += 256) {
-            const int r = e / DK, c = e % DK;
-            s += to_f(sH[r * PK + c]) * to_f(sdH[r * PK + c]);
+        for (int e = tid; e < DV * DK / VE; e += 256) {
+            const int r = e / (DK / VE), c = (e % (DK / VE)) * VE;
+            const uint4 hv = *reinterpret_cast<const uint4*>(sH + r * PK + c);
+            const uint4 gv = *reinterpret_cast<const uint4*>(sdH + r * PK + c);
+            const T* he = reinterpret_cast<const T*>(&hv);
+            const T* ge = reinterpret_cast<const T*>(&gv);
+#pragma unroll
+            for (int i = 0; i < VE; ++i) s = fmaf(to_f(he[i]), to_f(ge[i]), s);
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
@@ -268,8 +287,8 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
 
     const float gL = sG[L - 1];
     const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows
-    const float eGa = expf(sG[ra]), eGb = expf(sG[rb]);
-    const float sKa = ra < L ? expf(gL - sG[ra]) : 0.f, sKb = rb < L ? expf(gL - sG[rb]) : 0.f;
+    const float eGa = __expf(sG[ra]), eGb = __expf(sG[rb]);
+    const float sKa = ra < L ? __expf(gL - sG[ra]) : 0.f, sKb = rb < L ? __expf(gL - sG[rb]) : 0.f;
     auto rowpart = [&](int kind) { return rowp + (kind * 2 + wc) * 64; };
     auto put_rows = [&](int kind, float s0, float s1) {
         if ((lane & 3) == 0) { rowpart(kind)[ra] = s0; rowpart(kind)[rb] = s1; }
@@ -285,7 +304,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int r = m0 + frag_row(i), c = 32 * wc + frag_col(t, i);
-                const float v = (c <= r && r < L) ? sc[t][i] * expf(sG[r] - sG[c]) : 0.f;
+                const float v = (c <= r && r < L) ? sc[t][i] * __expf(sG[r] - sG[c]) : 0.f;
                 sP[r * PL + c] = from_f<T>(v);
             }
     }
@@ -376,7 +395,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         const float ba = sBe[ra], bb = sBe[rb];
 #pragma unroll
         for (int t = 0; t < NV; ++t) { tv[t][0] *= ba; tv[t][1] *= ba; tv[t][2] *= bb; tv[t][3] *= bb; }
-        frag_store_g<T, NV>((T*)p.dvv + (t0 * p.H + h) * DV, (long long)p.H * DV, m0, nv0, tv, L);
+        frag_store<T, NV>(sDV, PV, m0, nv0, tv);
     }
     __syncthreads();   // dO, E, dE, H, dH' no longer needed; dW complete
 
@@ -399,12 +418,12 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
             for (int i = 0; i < 4; ++i) {
                 const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
                 const bool incl = c <= r && r < L;
-                const float gam = incl ? expf(sG[r] - sG[c]) : 0.f;
+                const float gam = incl ? __expf(sG[r] - sG[c]) : 0.f;
                 const float w = dP[t][i] * sq[t][i] * gam;   // dP * P
                 if (i < 2) rs0 += w; else rs1 += w;
                 cs[t][i & 1] += w;
                 sdPh[r * PL + c] = from_f<T>(dP[t][i] * gam);
-                const float dm = dMa[t][i] + mb[t][i] * sBt[c] * expf(sGm1[c]);
+                const float dm = dMa[t][i] + mb[t][i] * sWs[c];
                 sdM[r * PL + c] = from_f<T>(dm);
             }
         }
@@ -440,7 +459,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
             for (int i = 0; i < 4; ++i) {
                 const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
                 const bool strict = c < r && r < L;
-                const float gm = strict ? expf(sGm1[r] - sG[c]) : 0.f;
+                const float gm = strict ? __expf(sGm1[r] - sG[c]) : 0.f;
                 const float a = -da[t][i];   // dA (masked below via gm)
                 const float u = a * gm * gr[t][i];           // contributes to dbtilde_r
                 const float w = u * sBt[r];                  // dA * Aval
@@ -465,7 +484,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     {
         // dQ~ = dPhat K + Diag(gamma) dO H^T ; dq = dQ~ ; dd partial = -k . dQ~
         warp_gemm<true, false, NK>(acc_dq, sdPh, PL, sK, PK, m0, nk0, 64);
-        frag_store_g<T, NK>((T*)p.dq + (t0 * p.H + h) * DK, (long long)p.H * DK, m0, nk0, acc_dq, L);
+
         float t0r[NK][4];
 #pragma unroll
         for (int t = 0; t < NK; ++t)
@@ -486,7 +505,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         float tmp[NK][4];
         zero(tmp);
         warp_gemm<false, false, NK>(tmp, sM, PL, sdW, PK, m0, nk0, 64);
-        const float wa = sBt[ra] * expf(sGm1[ra]), wb = sBt[rb] * expf(sGm1[rb]);
+        const float wa = sWs[ra], wb = sWs[rb];
         float t0r[NK][4];
 #pragma unroll
         for (int t = 0; t < NK; ++t)
@@ -498,9 +517,29 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         float s0, s1;
         frag_rowdot(t0r, s0, s1);
         put_rows(7, s0, s1);
-        frag_store_g<T, NK>((T*)p.dkk + (t0 * p.H + h) * DK, (long long)p.H * DK, m0, nk0, acc_dk, L);
     }
     __syncthreads();
+    // dq, dk, dv rows of this chunk: staged in the dead Q~ and K tiles (dv has its own),
+    // then coalesced 16-byte copies to global memory
+    frag_store<T, NK>(sQ, PK, m0, nk0, acc_dq);
+    frag_store<T, NK>(sK, PK, m0, nk0, acc_dk);
+    __syncthreads();
+    {
+        constexpr int CK = DK / VE, CV = DV / VE;
+        T* gq = (T*)p.dq + (t0 * p.H + h) * DK;
+        T* gk = (T*)p.dkk + (t0 * p.H + h) * DK;
+        T* gv = (T*)p.dvv + (t0 * p.H + h) * DV;
+        const long long sk = (long long)p.H * DK, sv = (long long)p.H * DV;
+        for (int e = tid; e < L * CK; e += 256) {
+            const int r = e / CK, c = (e % CK) * VE;
+            *reinterpret_cast<uint4*>(gq + r * sk + c) = *reinterpret_cast<const uint4*>(sQ + r * PK + c);
+            *reinterpret_cast<uint4*>(gk + r * sk + c) = *reinterpret_cast<const uint4*>(sK + r * PK + c);
+        }
+        for (int e = tid; e < L * CV; e += 256) {
+            const int r = e / CV, c = (e % CV) * VE;
+            *reinterpret_cast<uint4*>(gv + r * sv + c) = *reinterpret_cast<const uint4*>(sDV + r * PV + c);
+        }
+    }
 
     // ---------------- per-position scalars (rows 0..63, one thread each)
     auto rsum = [&](int kind, int r) { return rowp[(kind * 2) * 64 + r] + rowp[(kind * 2 + 1) * 64 + r]; };
@@ -515,32 +554,42 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
             g = rsum(0, r) - rsum(1, r) + rsum(3, r) - csum(0, r) - csum(1, r);
             if (r + 1 < L) {
                 g += rsum(5, r + 1);
-                g += sBt[r + 1] * expf(sGm1[r + 1]) * rsum(7, r + 1);
+                g += sWs[r + 1] * rsum(7, r + 1);
             }
         }
         sDg[r] = g;
     }
     __syncthreads();
-    if (tid == 0) {
-        // terms that land on the last position: gamma_C <H, dH'> and the Kbar total
-        float tk = 0.f;
-        for (int r = 0; r < L; ++r) tk += rsum(1, r);
-        float hd = 0.f;
-        for (int w = 0; w < 8; ++w) hd += red[w];
-        sDg[L - 1] += tk + expf(gL) * hd;
-        // d log alpha_j = sum_{r >= j} dg_r (reverse cumsum inside the chunk)
-        float acc = 0.f;
-        for (int r = L - 1; r >= 0; --r) {
-            acc += sDg[r];
-            sDg[r] = acc;
+    if (warp == 0) {
+        // terms that land on the last position: gamma_C <H, dH'> and the Kbar total (fixed-order
+        // warp reductions), then d log alpha_j = sum_{r >= j} dg_r, a suffix sum inside the chunk
+        float tk = (lane < L ? rsum(1, lane) : 0.f) + (lane + 32 < L ? rsum(1, lane + 32) : 0.f);
+        float hd = lane < 8 ? red[lane] : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            tk += __shfl_xor_sync(0xffffffffu, tk, o);
+            hd += __shfl_xor_sync(0xffffffffu, hd, o);
         }
+        float x0 = sDg[lane], x1 = sDg[lane + 32];   // zero past L
+        const float last = tk + __expf(gL) * hd;
+        if (L - 1 == lane) x0 += last;
+        if (L - 1 == lane + 32) x1 += last;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const float y0 = __shfl_down_sync(0xffffffffu, x0, o);
+            const float y1 = __shfl_down_sync(0xffffffffu, x1, o);
+            if (lane + o < 32) { x0 += y0; x1 += y1; }
+        }
+        x0 += __shfl_sync(0xffffffffu, x1, 0);
+        sDg[lane] = x0;
+        sDg[lane + 32] = x1;
     }
     __syncthreads();
     if (tid < 64) {
         const int r = tid;
         float dbt = 0.f, db_c = 0.f, dd_c = 0.f;
         if (r < L) {
-            dbt = rsum(4, r) + expf(sGm1[r]) * rsum(7, r);
+            dbt = rsum(4, r) + sEm1[r] * rsum(7, r);
             p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r];
             p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * dbt;
             db_c = sBe[r] * dbt;
