@@ -86,6 +86,22 @@ __device__ __forceinline__ void publish_smem() {
     tc_fence_after();
 }
 
+// Row-per-thread staging of a [128][8 NCH] bf16 tile whose 16-byte chunks are
+// rotated by row (chunk c of row r at slot (c + r) mod NCH), so the 32 lanes of a
+// warp writing one chunk of 32 consecutive rows hit distinct banks; then a
+// coalesced copy of the tile to contiguous global memory by all 128 threads.
+template <int NCH>
+__device__ __forceinline__ void stage_chunk(uint8_t* st, int row, int c, uint4 v) {
+    *reinterpret_cast<uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16) = v;
+}
+template <int NCH>
+__device__ __forceinline__ void copy_staged(bf16* g, const uint8_t* st, int tid) {
+    for (int e = tid; e < 128 * NCH; e += 128) {
+        const int row = e / NCH, c = e % NCH;
+        reinterpret_cast<uint4*>(g)[e] = *reinterpret_cast<const uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16);
+    }
+}
+
 // ------------------------------------------------------------------ prep
 
 struct PrepTcSmem {
@@ -209,10 +225,11 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
         tc_gemm<true, false>(tmem + 128, smem_u32(sV), 64, smem_u32(sMu), 64, 64, 64, false);
     }
     ok = ok && ms.finish(tid);
+    // W^T and U^T for the workspace are staged over the dead V and Mw/Mu tiles.
+    uint8_t* stW = sV;
+    uint8_t* stU = sMw;
     if (ok) {
         float d[32], v[8], w[8];
-        bf16* Wt = (bf16*)p.Wb + (idx * D + row) * 64;
-        bf16* Ut = (bf16*)p.Ub + (idx * D + row) * 64;
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
             tmem_ld32(trow + 64 + g * 32, d);
@@ -223,7 +240,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
                     v[e] = d[8 * q + e];
                     w[e] = v[e] * sS[32 * g + 8 * q + e];
                 }
-                *reinterpret_cast<uint4*>(Wt + 32 * g + 8 * q) = pack8(v);
+                stage_chunk<8>(stW, row, 4 * g + q, pack8(v));
                 *reinterpret_cast<uint4*>(sWt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
             }
         }
@@ -237,7 +254,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
                     v[e] = d[8 * q + e];
                     w[e] = v[e] * sS[32 * g + 8 * q + e];
                 }
-                *reinterpret_cast<uint4*>(Ut + 32 * g + 8 * q) = pack8(v);
+                stage_chunk<8>(stU, row, 4 * g + q, pack8(v));
                 *reinterpret_cast<uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
             }
         }
@@ -249,11 +266,17 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
         tc_gemm<true, false>(tmem, smem_u32(sK), 128, smem_u32(sWt), 128, 128, 64, false);
         tc_gemm<false, true>(tmem + 128, smem_u32(sUt), 128, smem_u32(sK), 128, 128, 64, false);
     }
+    if (ok) {
+        // W^T, U^T out while the tensor core works
+        copy_staged<8>((bf16*)p.Wb + idx * D * 64, stW, tid);
+        copy_staged<8>((bf16*)p.Ub + idx * D * 64, stU, tid);
+    }
     ok = ok && ms.finish(tid);
+    // Atilde over the dead K tile, B^T over the dead V/Mw/Mu tiles (their copies are done)
+    uint8_t* stA = sK;
+    uint8_t* stB = sV;
     if (ok) {
         float d[32], v[8];
-        bf16* At = (bf16*)p.Ab + (idx * D + row) * D;
-        bf16* Bt = (bf16*)p.Bb + (idx * D + row) * D;
 #pragma unroll
         for (int g = 0; g < 4; ++g) {
             tmem_ld32(trow + g * 32, d);
@@ -261,15 +284,20 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
             for (int q = 0; q < 4; ++q) {
 #pragma unroll
                 for (int e = 0; e < 8; ++e) v[e] = -d[8 * q + e];
-                *reinterpret_cast<uint4*>(At + 32 * g + 8 * q) = pack8(v);
+                stage_chunk<16>(stA, row, 4 * g + q, pack8(v));
             }
         }
 #pragma unroll
         for (int g = 0; g < 4; ++g) {
             tmem_ld32(trow + 128 + g * 32, d);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) *reinterpret_cast<uint4*>(Bt + 32 * g + 8 * q) = pack8(d + 8 * q);
+            for (int q = 0; q < 4; ++q) stage_chunk<16>(stB, row, 4 * g + q, pack8(d + 8 * q));
         }
+    }
+    __syncthreads();
+    if (ok) {
+        copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid);
+        copy_staged<16>((bf16*)p.Bb + idx * D * D, stB, tid);
     }
     if (!ok && tid == 0) flag_error(p);
     tc_fence_before();
@@ -281,14 +309,20 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
 // ---------------------------------------------------------------- output
 
 struct OutTcSmem {
-    static constexpr uint32_t OQ = 0;              // Q -> Q~ -> Qhat   [128 alloc rows][128]  32 KB
-    static constexpr uint32_t OK = 32768;          // K [64][128], later P [64][64]            16 KB
-    static constexpr uint32_t OW = OK + 16384;     // W^T [128][64] (MN-major B), later E^T    16 KB
-    static constexpr uint32_t OU = OW + 16384;     // U^T [128][64]                            16 KB
+    static constexpr uint32_t OQK = 0;             // [128 rows][128]: rows 0-63 Q -> Q~ -> Qhat, rows 64-127 K;
+                                                   // P [64][64] later over K's first half     32 KB
+    static constexpr uint32_t OW = 32768;          // W^T [128][64] (MN-major B), later E^T    16 KB
+    static constexpr uint32_t OU = OW + 16384;     // U^T [128][64], later E [64][128]         16 KB
     static constexpr uint32_t OH = OU + 16384;     // H^T [128][128] K-major, later O staging  32 KB
     static constexpr uint32_t OG = OH + 32768;
     static constexpr size_t bytes() { return 1024 + OG + 64 * 4; }
 };
+
+__device__ __forceinline__ void bulk_copy_s2g(void* g, uint32_t s, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n" ::"l"(g), "r"(s), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all_reads() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
 
 __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
     using S = OutTcSmem;
@@ -303,18 +337,27 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
     const long long idx = (long long)slot * p.H + h;
     const int tid = threadIdx.x, warp = tid >> 5;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sQ = sm + S::OQ;
-    uint8_t* sK = sm + S::OK;
-    uint8_t* sP = sK;
+    uint8_t* sQK = sm + S::OQK;
+    uint8_t* sP = sQK + 64 * 128;   // K's rows of the first 64-column half, dead after S = Q~ K^T
     uint8_t* sWt = sm + S::OW;
     uint8_t* sEt = sWt;
     uint8_t* sUt = sm + S::OU;
+    bf16* sE = reinterpret_cast<bf16*>(sUt);   // [64][128] row-major staging of E
     uint8_t* sHt = sm + S::OH;
     bf16* sO = reinterpret_cast<bf16*>(sHt);   // [64][136] staging of O
     float* sG = reinterpret_cast<float*>(sm + S::OG);
 
-    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
-    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    {
+        // Q into rows 0-63 and K into rows 64-127 of one K-major tile (rows past the chunk zero)
+        const bf16* qg = (const bf16*)p.q + (t0 * p.H + h) * D;
+        const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
+        for (int e = tid; e < 128 * 16; e += 128) {
+            const int r = e >> 4, ch = e & 15, rr = r & 63;
+            const bool okr = rr < L;
+            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * p.H * D + ch * 8;
+            cp_async16(sQK + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
+        }
+    }
     load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid);
     load_sw(sUt, 128, 64, (const bf16*)p.Ub + idx * D * 64, 64, 128, tid);
     load_sw(sHt, 128, D, (const bf16*)p.Hb + idx * D * D, D, 128, tid);
@@ -331,8 +374,8 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
     const float dh = p.d[h];
     for (int e = tid; e < 64 * 16; e += 128) {
         const int r = e >> 4, ch = e & 15;
-        uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
-        const uint4 ka = *reinterpret_cast<const uint4*>(sK + sw128_offset(r, 8 * ch, 64));
+        uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
+        const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
         float qv[8], kv[8];
         unpack8(*qa, qv);
         unpack8(ka, kv);
@@ -346,12 +389,14 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
     const int row = tid;
     const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 
-    // S = Q~ K^T -> cols [0,64);  E^T' = H^T W^T -> cols [64,128)
+    // [Q~; K] K^T -> cols [0,64) (lanes 0-63: S = Q~ K^T; lanes 64-127 unused);  E^T' = H^T W^T -> cols [64,128)
     if (tid == 0) {
-        tc_gemm<false, false>(tmem, smem_u32(sQ), 128, smem_u32(sK), 64, 64, D, false);
+        tc_gemm<false, false>(tmem, smem_u32(sQK), 128, smem_u32(sQK) + 64 * 128, 128, 64, D, false);
         tc_gemm<false, true>(tmem + 64, smem_u32(sHt), 128, smem_u32(sWt), 128, 64, D, false);
     }
     bool ok = ms.finish(tid);
+    bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
+    uint32_t ev[32];   // this thread's row j of E^T (64 positions), packed bf16 pairs
     if (ok) {
         float d[32], v[8];
         // P = Tril(S * Gamma) into a K-major [64][64] tile (B operand of E^T P^T)
@@ -359,19 +404,19 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
         for (int g = 0; g < 2; ++g) {
             tmem_ld32(trow + g * 32, d);
             if (row < 64) {
+                const float gr = sG[row];
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
                         const int i = 32 * g + 8 * q + e;
-                        v[e] = (i <= row && row < L) ? d[8 * q + e] * expf(sG[row] - sG[i]) : 0.f;
+                        v[e] = (i <= row && row < L) ? d[8 * q + e] * __expf(gr - sG[i]) : 0.f;
                     }
                     *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 64)) = pack8(v);
                 }
             }
         }
-        // E^T = U^T - H^T W^T  (row j of E^T per thread; saved as E [64][128] for the backward)
-        bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
+        // E^T = U^T - H^T W^T  (row j of E^T per thread)
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
             tmem_ld32(trow + 64 + g * 32, d);
@@ -382,31 +427,43 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
 #pragma unroll
                 for (int e = 0; e < 8; ++e) v[e] = u[e] - d[8 * q + e];
                 // sEt aliases sWt: every thread reads only its own row, and W^T is no longer needed
-                *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
-                if (Eg) {
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) Eg[(32 * g + 8 * q + e) * D + row] = __float2bfloat16_rn(v[e]);
-                }
+                const uint4 pk = pack8(v);
+                *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * g + 8 * q, 128)) = pk;
+                const int b0 = (32 * g + 8 * q) / 2;
+                ev[b0] = pk.x; ev[b0 + 1] = pk.y; ev[b0 + 2] = pk.z; ev[b0 + 3] = pk.w;
             }
         }
         // Qhat = Diag(gamma) Q~ in place
         for (int e = tid; e < 64 * 16; e += 128) {
             const int r = e >> 4, ch = e & 15;
-            uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
+            uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
             float qv[8];
             unpack8(*qa, qv);
-            const float gr = expf(sG[r]);
+            const float gr = __expf(sG[r]);
 #pragma unroll
             for (int i = 0; i < 8; ++i) qv[i] *= gr;
             *qa = pack8(qv);
         }
     }
     publish_smem();
+    if (ok && Eg) {
+        // E [64][128] row-major over the dead U^T tile (every thread is past its U^T reads), then
+        // one 16 KB bulk copy to the workspace
+#pragma unroll
+        for (int pp = 0; pp < 32; ++pp) {
+            const __nv_bfloat162 two = *reinterpret_cast<const __nv_bfloat162*>(&ev[pp]);
+            sE[(2 * pp) * D + row] = two.x;
+            sE[(2 * pp + 1) * D + row] = two.y;
+        }
+        fence_async_smem();
+    }
+    __syncthreads();
+    if (ok && Eg && tid == 0) bulk_copy_s2g(Eg, smem_u32(sE), 64 * D * 2);
     if (!p.o) ok = false;   // E only (backward recompute): nothing more to do
 
     // O^T = H^T Qhat^T + E^T P^T -> cols [128,192)
     if (ok && tid == 0) {
-        tc_gemm<false, false>(tmem + 128, smem_u32(sHt), 128, smem_u32(sQ), 128, 64, D, false);
+        tc_gemm<false, false>(tmem + 128, smem_u32(sHt), 128, smem_u32(sQK), 128, 64, D, false);
         tc_gemm<false, false>(tmem + 128, smem_u32(sEt), 128, smem_u32(sP), 64, 64, 64, true);
     }
     if (p.o) {
@@ -432,6 +489,7 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
             flag_error(p);
         }
     }
+    if (Eg && tid == 0) bulk_wait_all_reads();   // the E copy has read its staging before exit
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -506,17 +564,24 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     if (ok) {
         // P [128 alloc rows][64] K-major A operand (rows >= 64 zero); Qhat = Diag(gamma) Q~ in place.
         float d[32], v[8];
+        const float gr = row < 64 ? sG[row] : 0.f;
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
             tmem_ld32(trow + g * 32, d);
+            if (row < 64) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
+                for (int q = 0; q < 4; ++q) {
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int i = 32 * g + 8 * q + e;
-                    v[e] = (row < 64 && i <= row && row < L) ? d[8 * q + e] * expf(sG[row] - sG[i]) : 0.f;
+                    for (int e = 0; e < 8; ++e) {
+                        const int i = 32 * g + 8 * q + e;
+                        v[e] = (i <= row && row < L) ? d[8 * q + e] * __expf(gr - sG[i]) : 0.f;
+                    }
+                    *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
                 }
-                *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 128)) = make_uint4(0, 0, 0, 0);
             }
         }
         for (int e = tid; e < 64 * 16; e += 128) {
@@ -524,7 +589,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
             uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
             float qv[8];
             unpack8(*qa, qv);
-            const float gr = expf(sG[r]);
+            const float gr = __expf(sG[r]);
 #pragma unroll
             for (int i = 0; i < 8; ++i) qv[i] *= gr;
             *qa = pack8(qv);
@@ -559,14 +624,18 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     if (ok && tid == 0) tc_gemm<true, true>(tmem, smem_u32(sdO), 64, smem_u32(sZ), 64, 128, 64, false);
     ok = ok && ms.finish(tid);
     if (ok) {
+        // C^T staged over the dead Qhat tile, then copied out coalesced
         float d[32];
-        bf16* Cg = (bf16*)p.Cb + (idx * D + row) * D;
 #pragma unroll
         for (int g = 0; g < 4; ++g) {
             tmem_ld32(trow + g * 32, d);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) *reinterpret_cast<uint4*>(Cg + 32 * g + 8 * q) = pack8(d + 8 * q);
+            for (int q = 0; q < 4; ++q) stage_chunk<16>(sQ, row, 4 * g + q, pack8(d + 8 * q));
         }
+    }
+    __syncthreads();
+    if (ok) {
+        copy_staged<16>((bf16*)p.Cb + idx * D * D, sQ, tid);
     } else if (tid == 0) {
         flag_error(p);
     }
