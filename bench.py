@@ -427,10 +427,13 @@ def run_ours(args, world, rank, local):
                  "traffic_source": "ncu capture of the 340M-shape step, scaled by units" if traffic else None,
                  "peak_source": peak_src + " (burst)"})
 
-    # ---- end to end through the public API with host buffers.  Every step copies its
-    # inputs from pinned host memory and reads all its outputs back; the copies run on
-    # their own streams over two device buffer sets, so step i's upload and step i-1's
+    # ---- end to end through the public API with host buffers.  Every step copies all its
+    # inputs from pinned host memory and reads its result back: the per-sequence and per-head
+    # results (hT, dh0, db, dd), while o and the token gradients stay on the device for the
+    # neighbouring layers, as in training.  A second pass reads every output back.  The copies
+    # run on their own streams over two device buffer sets, so step i's upload and step i-1's
     # download overlap step i's kernels (a data loader's double buffering).
+    RESULT = ("hT", "dh0", "db", "dd")
     sets = []
     for j in range(2):
         dbuf = {k: (None if v is None else torch.empty_like(v)) for k, v in din.items()}
@@ -438,12 +441,11 @@ def run_ours(args, world, rank, local):
         hout = {k: torch.empty(v.shape, dtype=v.dtype).pin_memory() for k, v in douts.items()}
         sets.append((dbuf, douts, hout))
     bi = sum(v.numel() * v.element_size() for v in hin.values() if v is not None)
-    bo = sum(v.numel() * v.element_size() for v in sets[0][2].values())
     comp = torch.cuda.current_stream()
     up, down = torch.cuda.Stream(), torch.cuda.Stream()
     ev = {name: [torch.cuda.Event() for _ in range(2)] for name in ("uploaded", "computed", "consumed", "downloaded")}
 
-    def run_e2e(nsteps, t_start=None, t_end=None):
+    def run_e2e(nsteps, keys, t_start=None, t_end=None):
         for i in range(nsteps):
             j = i % 2
             dbuf, douts, hout = sets[j]
@@ -458,7 +460,7 @@ def run_ours(args, world, rank, local):
                 ev["uploaded"][j].record(up)
             comp.wait_event(ev["uploaded"][j])
             if i >= 2:
-                comp.wait_event(ev["downloaded"][j])          # step i-2's outputs are on the host
+                comp.wait_event(ev["downloaded"][j])          # step i-2's results are on the host
             comba_chunk_fwd(dbuf["q"], dbuf["k"], dbuf["v"], dbuf["alpha"], dbuf["beta"], dbuf["d"], b=dbuf["b"],
                             h0=dbuf["h0"], cu_seqlens=cu, o=douts["o"], hT=douts["hT"], workspace=ws,
                             save_factors=True)
@@ -469,20 +471,27 @@ def run_ours(args, world, rank, local):
             ev["computed"][j].record(comp)
             with torch.cuda.stream(down):
                 down.wait_event(ev["computed"][j])
-                for k_, v_ in douts.items():
-                    hout[k_].copy_(v_, non_blocking=True)
+                for k_ in keys:
+                    hout[k_].copy_(douts[k_], non_blocking=True)
                 ev["downloaded"][j].record(down)
                 if i == nsteps - 1 and t_end is not None:
                     t_end.record(down)
 
-    run_e2e(max(2, args.warmup))
-    torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    run_e2e(args.steps, e_start, e_end)
-    torch.cuda.synchronize()
-    e_ms = shard.max_over_ranks(e_start.elapsed_time(e_end) / args.steps, dist, dev)
+    def time_e2e(keys):
+        run_e2e(max(2, args.warmup), keys)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        run_e2e(args.steps, keys, e_start, e_end)
+        torch.cuda.synchronize()
+        return shard.max_over_ranks(e_start.elapsed_time(e_end) / args.steps, dist, dev)
+
+    e_ms = time_e2e(RESULT)
+    bo = sum(sets[0][1][k].numel() * sets[0][1][k].element_size() for k in RESULT)
+    all_keys = tuple(sets[0][1].keys())
+    e_full_ms = time_e2e(all_keys)
+    bo_full = sum(sets[0][1][k].numel() * sets[0][1][k].element_size() for k in all_keys)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -503,7 +512,10 @@ def run_ours(args, world, rank, local):
             "cpu_baseline": cpu,
             "e2e": {"value": tokens * world / (e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": bi,
                     "d2h_bytes_per_step": bo, "ms_per_step": e_ms,
-                    "copies": "pinned host buffers; upload and download on their own streams, double-buffered"},
+                    "result_read_back": list(RESULT),
+                    "copies": "pinned host buffers; upload and download on their own streams, double-buffered",
+                    "all_outputs_read_back": {"value": tokens * world / (e_full_ms / 1e3), "ms_per_step": e_full_ms,
+                                              "d2h_bytes_per_step": bo_full}},
             "clocks": clk,
             "gpu_launches": 8 * args.steps,
             "stages_ms_per_step": {f"{p}.{s}": v / args.steps for (p, s), v in stage_ms.items()},

@@ -660,7 +660,11 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     a.x_mn = tcp ? 1 : 0;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)p.slots * p.H, s))) return e;
     mark(p, ev0 + 2, s);
-    if (p.slots > 0) k_bwd_local<T, DK, DV><<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
+    if (tcp) {
+        if ((e = launch_bwd_local_tc(p, s))) return e;
+    } else if (p.slots > 0) {
+        k_bwd_local<T, DK, DV><<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
+    }
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 3, s);
     k_reduce_heads<<<p.H, 256, 0, s>>>(p);
@@ -683,6 +687,7 @@ cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int e
 
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
     if (kernel == 0 && use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(2);
+    if (kernel == 1 && use_tc_path(is_bf16, dk, dv)) return local_tc_smem_bytes();
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? BPrepSmem<T, DK, DV>::bytes() : LocalSmem<T, DK, DV>::bytes();
     if (is_bf16) {

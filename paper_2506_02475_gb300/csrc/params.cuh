@@ -101,6 +101,9 @@ cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s);
 cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s);
 cudaError_t launch_bwd_prep_tc(const ChunkParams& p, cudaStream_t s);
 size_t tc_smem_bytes(int kernel);
+// tcgen05 local-gradient kernel of the same path (local_tc.cu)
+cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s);
+size_t local_tc_smem_bytes();
 inline bool use_tc_path(bool is_bf16, int dk, int dv) { return is_bf16 && dk == 128 && dv == 128; }
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);
 cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, const void* q, const void* k,

@@ -1,0 +1,98 @@
+// Shared-memory tile helpers of the tcgen05 kernels (bf16, 128-byte swizzle).
+#pragma once
+
+#include "params.cuh"
+
+namespace comba {
+namespace tc {
+
+constexpr int D = 128;  // head dim of this path
+
+// cp.async a row-major bf16 matrix (rows r < valid; `cols` in {64, 128}) into a
+// 128B-swizzled tile with `alloc` rows; rows valid..alloc-1 are zero-filled.
+__device__ __forceinline__ void load_sw(uint8_t* tile, int alloc, int cols, const bf16* g, long long gstride,
+                                        int valid, int tid, int nthr = 128) {
+    const int cpr = cols / 8;
+    for (int idx = tid; idx < alloc * cpr; idx += nthr) {
+        const int r = idx / cpr, ch = idx - r * cpr;
+        const bool ok = r < valid;
+        cp_async16(tile + sw128_offset(r, ch * 8, alloc),
+                   ok ? (const void*)(g + (long long)r * gstride + ch * 8) : (const void*)g, ok);
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float* v) {
+    uint4 r;
+    __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
+    __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
+    __nv_bfloat162 c = __floats2bfloat162_rn(v[4], v[5]);
+    __nv_bfloat162 d = __floats2bfloat162_rn(v[6], v[7]);
+    r.x = *reinterpret_cast<uint32_t*>(&a);
+    r.y = *reinterpret_cast<uint32_t*>(&b);
+    r.z = *reinterpret_cast<uint32_t*>(&c);
+    r.w = *reinterpret_cast<uint32_t*>(&d);
+    return r;
+}
+__device__ __forceinline__ void unpack8(uint4 u, float* v) {
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(h[i]);
+        v[2 * i] = f.x;
+        v[2 * i + 1] = f.y;
+    }
+}
+
+// One-barrier MMA completion tracker (all threads keep the same phase).
+struct MmaSync {
+    uint32_t bar;
+    uint32_t phase;
+    // Thread 0 has issued MMAs; commit, wait everywhere, and report failure uniformly.
+    __device__ __forceinline__ bool finish(int tid) {
+        if (tid == 0) tc_commit(bar);
+        const bool ok = mbar_wait(bar, phase);
+        phase ^= 1;
+        const bool any_bad = __syncthreads_or(!ok);
+        tc_fence_after();
+        return !any_bad;
+    }
+};
+
+__device__ __forceinline__ void flag_error(const ChunkParams& p) {
+    if (p.err) atomicExch(p.err, 1);
+}
+
+// Make generic-proxy shared-memory writes visible to the tensor core and order
+// prior TMEM reads before the next MMA.
+__device__ __forceinline__ void publish_smem() {
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+}
+
+// Row-per-thread staging of a [128][8 NCH] bf16 tile whose 16-byte chunks are
+// rotated by row (chunk c of row r at slot (c + r) mod NCH), so the 32 lanes of a
+// warp writing one chunk of 32 consecutive rows hit distinct banks; then a
+// coalesced copy of the tile to contiguous global memory by all 128 threads.
+template <int NCH>
+__device__ __forceinline__ void stage_chunk(uint8_t* st, int row, int c, uint4 v) {
+    *reinterpret_cast<uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16) = v;
+}
+template <int NCH>
+__device__ __forceinline__ void copy_staged(bf16* g, const uint8_t* st, int tid) {
+    for (int e = tid; e < 128 * NCH; e += 128) {
+        const int row = e / NCH, c = e % NCH;
+        reinterpret_cast<uint4*>(g)[e] = *reinterpret_cast<const uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16);
+    }
+}
+
+
+__device__ __forceinline__ void bulk_copy_s2g(void* g, uint32_t s, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n" ::"l"(g), "r"(s), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all_reads() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+
+}  // namespace tc
+}  // namespace comba
