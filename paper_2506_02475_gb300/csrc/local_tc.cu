@@ -118,22 +118,27 @@ __device__ __forceinline__ void rowdot(const float (&acc)[NT][4], float& s0, flo
     s1 = quad_sum(s1);
 }
 
-__global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p) {
+struct UnitRef {
+    long long idx, t0;   // (slot, head) unit index, first token
+    int L, h;
+};
+__device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
+    const SlotInfo si = p.slot_info[u / p.H];
+    return {u, si.start, si.len, (int)(u % p.H)};
+}
+
+// Persistent: CTA b handles units b, b + G, b + 2G, ... (G = gridDim.x, about one CTA per SM).
+// While unit u computes, the tiles of unit u + G stream into buffers as soon as their last
+// reader in unit u has finished (dH'^T after R1, H^T after R3, E after the dv copy, dO, V,
+// M after R7), so the loads of consecutive units overlap the tensor-core and epilogue work
+// instead of every SM loading at the same moment; only Q and K load at the top of a unit.
+__global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long long units) {
     using S = LocalTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar;
     __shared__ uint32_t tbase;
-    const int slot = blockIdx.x, h = blockIdx.y;
-    const long long idx = (long long)slot * p.H + h;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wr = warp & 3, wc = warp >> 2, m0 = 16 * wr;
-    const SlotInfo si = p.slot_info[slot];
-    if (si.len <= 0) {
-        if (tid == 0) { p.part[idx * 2] = 0.f; p.part[idx * 2 + 1] = 0.f; }
-        return;
-    }
-    const int L = si.len;
-    const long long t0 = si.start;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQK = sm + S::OQK;
     uint8_t* sKt = sQK + 64 * 128;   // K: rows 64-127 of the 128-row tile
@@ -145,11 +150,11 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p) {
     uint8_t* sM = sm + S::OM;
     uint8_t* sP = sm + S::OP;
     uint8_t* sdE = sm + S::ODE;
-    uint8_t* sdW = sdHt;              // after R1
-    uint8_t* sdPh = sHt;              // after R3
-    uint8_t* sdM = sHt + 8192;
-    uint8_t* sY = sHt + 16384;
-    uint8_t* sdG = sHt + 24576;
+    uint8_t* sdW = sdO;               // after R2
+    uint8_t* sdPh = sdE;              // after R3
+    uint8_t* sdM = sdE + 8192;
+    uint8_t* sY = sV;                 // after E3
+    uint8_t* sdG = sV + 8192;
     uint8_t* stV = sE;                // dv staging, after R1
     float* sG = reinterpret_cast<float*>(sm + S::OF);
     float* sGm1 = sG + 64;
@@ -162,86 +167,42 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p) {
     float* rowp = sG + 512;           // [kind][column half][row]
     float* colp = rowp + 8 * 2 * 64;  // [kind][row block][column]
     float* red = colp + 2 * 4 * 64;
-
-    const float bh = p.b ? p.b[h] : 1.f;
-    const float dh = p.d[h];
-    {
-        const bf16* qg = (const bf16*)p.q + (t0 * p.H + h) * D;
-        const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
-        for (int e = tid; e < 128 * 16; e += 256) {
-            const int r = e >> 4, ch = e & 15, rr = r & 63;
-            const bool okr = rr < L;
-            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * p.H * D + ch * 8;
-            cp_async16(sQK + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
-        }
-    }
-    load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, 256);
-    load_sw(sdO, 64, D, (const bf16*)p.dO + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, 256);
-    load_sw(sE, 64, D, (const bf16*)p.Eb + idx * 64 * D, D, 64, tid, 256);
-    load_sw(sHt, 128, D, (const bf16*)p.Hb + idx * D * D, D, 128, tid, 256);
-    load_sw(sdHt, 128, D, (const bf16*)p.dHb + idx * D * D, D, 128, tid, 256);
-    load_sw(sM, 64, 64, (const bf16*)p.Mb + idx * 4096, 64, 64, tid, 256);
-    cp_async_commit();
-    if (tid < 64) {
-        const float g = p.Gb[idx * 64 + tid];
-        const float gm1 = tid > 0 ? p.Gb[idx * 64 + tid - 1] : 0.f;
-        sG[tid] = g;
-        sGm1[tid] = gm1;
-        const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
-        sBe[tid] = be;
-        sBt[tid] = bh * be;
-        sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
-        const float em1 = tid > 0 ? __expf(gm1) : 1.f;
-        sEm1[tid] = em1;
-        sWs[tid] = bh * be * em1;
-    }
-    if (tid == 0) {
-        mbar_init(smem_u32(&bar), 1);
-        mbar_fence_init();
-    }
-    if (warp == 0) tmem_alloc(smem_u32(&tbase), 512);
-    cp_async_wait<0>();
-    __syncthreads();
-    // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
-    for (int e = tid; e < 64 * 16; e += 256) {
-        const int r = e >> 4, ch = e & 15;
-        uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
-        const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
-        float qv[8], kv[8];
-        unpack8(*qa, qv);
-        unpack8(ka, kv);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
-        *qa = pack8(qv);
-    }
-    // <H, dH'>: the two tiles share one layout, so matching 16-byte chunks pair up
-    {
-        float s = 0.f;
-        for (int e = tid; e < 128 * 16; e += 256) {
-            float hv[8], gv[8];
-            unpack8(reinterpret_cast<const uint4*>(sHt)[e], hv);
-            unpack8(reinterpret_cast<const uint4*>(sdHt)[e], gv);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) s = fmaf(hv[i], gv[i], s);
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        if (lane == 0) red[warp] = s;
-    }
-    publish_smem();
-    const uint32_t tmem = tbase;
-    const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16);   // this warp's TMEM lanes
-    MmaSync ms{smem_u32(&bar), 0};
     const uint32_t uQK = smem_u32(sQK), uK = smem_u32(sKt), uV = smem_u32(sV), udO = smem_u32(sdO),
                    uE = smem_u32(sE), uH = smem_u32(sHt), udH = smem_u32(sdHt), uM = smem_u32(sM),
                    uP = smem_u32(sP), udE = smem_u32(sdE), udW = smem_u32(sdW), udPh = smem_u32(sdPh),
                    udM = smem_u32(sdM), uY = smem_u32(sY), udG = smem_u32(sdG);
 
-    const float gL = sG[L - 1];
-    const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows
-    const float eGa = __expf(sG[ra]), eGb = __expf(sG[rb]);
-    const float sKa = ra < L ? __expf(gL - sG[ra]) : 0.f, sKb = rb < L ? __expf(gL - sG[rb]) : 0.f;
+    auto load_qk = [&](const UnitRef& x) {
+        const bf16* qg = (const bf16*)p.q + (x.t0 * p.H + x.h) * D;
+        const bf16* kg = (const bf16*)p.k + (x.t0 * p.H + x.h) * D;
+        for (int e = tid; e < 128 * 16; e += 256) {
+            const int r = e >> 4, ch = e & 15, rr = r & 63;
+            const bool okr = rr < x.L;
+            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * p.H * D + ch * 8;
+            cp_async16(sQK + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
+        }
+    };
+    auto load_tok = [&](uint8_t* dst, const void* base, const UnitRef& x) {
+        load_sw(dst, 64, D, (const bf16*)base + (x.t0 * p.H + x.h) * D, (long long)p.H * D, x.L, tid, 256);
+    };
+    auto load_dH = [&](const UnitRef& x) { load_sw(sdHt, 128, D, (const bf16*)p.dHb + x.idx * D * D, D, 128, tid, 256); };
+    auto load_H = [&](const UnitRef& x) { load_sw(sHt, 128, D, (const bf16*)p.Hb + x.idx * D * D, D, 128, tid, 256); };
+    auto load_E = [&](const UnitRef& x) { load_sw(sE, 64, D, (const bf16*)p.Eb + x.idx * 64 * D, D, 64, tid, 256); };
+    auto load_M = [&](const UnitRef& x) { load_sw(sM, 64, 64, (const bf16*)p.Mb + x.idx * 4096, 64, 64, tid, 256); };
+
+    if (tid == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&tbase), 512);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tbase;
+    const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16);   // this warp's TMEM lanes
+    MmaSync ms{smem_u32(&bar), 0};
     const int nl0 = 32 * wc, nk0 = 64 * wc;   // this warp's columns of 64- and 128-wide results
+    const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows
     auto put_rows = [&](int kind, float s0, float s1) {
         if ((lane & 3) == 0) { rowp[(kind * 2 + wc) * 64 + ra] = s0; rowp[(kind * 2 + wc) * 64 + rb] = s1; }
     };
@@ -259,316 +220,404 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p) {
         rowdot(prod, s0, s1);
     };
 
-    // ---------------- R1
-    if (tid == 0) {
-        tc_gemm_m64<false, false>(tmem + 0, uQK, 128, uK, 128, 64, D, false);      // S = Q~ K^T
-        tc_gemm_m64<false, false>(tmem + 64, udO, 64, uE, 64, 64, D, false);       // dP = dO E^T
-        tc_gemm_m64<false, true>(tmem + 128, udO, 64, uH, 128, 128, D, false);     // dO H^T
-        tc_gemm_m64<false, true>(tmem + 256, uE, 64, udH, 128, 128, D, false);     // E dH'^T
-        tc_gemm_m64<false, false>(tmem + 384, uK, 128, udH, 128, 128, D, false);   // K dH'
-    }
-    bool ok = ms.finish(tid);
-    float sc[4][4], dP[4][4], acc_dq[8][4], acc_dk[8][4], de[8][4];
-    if (ok) {
-        // P = Tril(S * Gamma)
-        tmem_frag4(tq + 0 + nl0, sc);
-#pragma unroll
-        for (int t = 0; t < 4; ++t)
-#pragma unroll
-            for (int hh = 0; hh < 2; ++hh) {
-                const int r = m0 + frag_row(2 * hh), c = nl0 + frag_col(t, 0);
-                const float gr = sG[r];
-                const float v0 = (c <= r && r < L) ? sc[t][2 * hh] * __expf(gr - sG[c]) : 0.f;
-                const float v1 = (c + 1 <= r && r < L) ? sc[t][2 * hh + 1] * __expf(gr - sG[c + 1]) : 0.f;
-                st_pair(sP, 64, r, c, v0, v1);
-            }
-        tmem_frag4(tq + 64 + nl0, dP);
-        // dQ~ part Diag(gamma) dO H^T; its row dot with Q~ is the log-decay gradient of the Q~ H term
-        tmem_frag8(tq + 128 + nk0, acc_dq);
-#pragma unroll
-        for (int t = 0; t < 8; ++t) { acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb; }
-        float s0, s1;
-        tile_rowdot(acc_dq, sQK, 128, 0, s0, s1);
-        put_rows(0, s0, s1);
-        // dK from Kbar: Diag(gamma_C / gamma_r) E dH'^T
-        tmem_frag8(tq + 256 + nk0, acc_dk);
-#pragma unroll
-        for (int t = 0; t < 8; ++t) { acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb; }
-        tile_rowdot(acc_dk, sQK, 128, 64, s0, s1);
-        put_rows(1, s0, s1);
-        // Kbar dH' part of dE
-        tmem_frag8(tq + 384 + nk0, de);
-#pragma unroll
-        for (int t = 0; t < 8; ++t) { de[t][0] *= sKa; de[t][1] *= sKa; de[t][2] *= sKb; de[t][3] *= sKb; }
-    }
-    publish_smem();
+    bool ok = true;
+    bool pre = false;   // this unit's dH'^T, H^T, E, dO, V, M were requested by the previous unit
+    for (long long u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const UnitRef cur = unit_ref(p, u);
+        if (cur.L <= 0) {
+            if (tid == 0) { p.part[u * 2] = 0.f; p.part[u * 2 + 1] = 0.f; }
+            pre = false;
+            continue;
+        }
+        const long long un = u + gridDim.x;
+        UnitRef nxt{0, 0, 0, 0};
+        if (un < units) nxt = unit_ref(p, un);
+        const bool has_next = nxt.L > 0;
+        const int L = cur.L, h = cur.h;
+        const long long t0 = cur.t0, idx = cur.idx;
 
-    // ---------------- R2: dE = Kbar dH' + P^T dO
-    if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
-    ok = ok && ms.finish(tid);
-    if (ok) {
-        float t2[8][4];
-        tmem_frag8(tq + 0 + nk0, t2);
+        load_qk(cur);
+        if (!pre) {
+            load_tok(sdO, p.dO, cur);
+            load_E(cur);
+            load_H(cur);
+            load_dH(cur);
+            load_tok(sV, p.v, cur);
+            load_M(cur);
+        }
+        cp_async_commit();
+        const float bh = p.b ? p.b[h] : 1.f;
+        const float dh = p.d[h];
+        if (tid < 64) {
+            const float g = p.Gb[idx * 64 + tid];
+            const float gm1 = tid > 0 ? p.Gb[idx * 64 + tid - 1] : 0.f;
+            sG[tid] = g;
+            sGm1[tid] = gm1;
+            const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
+            sBe[tid] = be;
+            sBt[tid] = bh * be;
+            sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
+            const float em1 = tid > 0 ? __expf(gm1) : 1.f;
+            sEm1[tid] = em1;
+            sWs[tid] = bh * be * em1;
+        }
+        cp_async_wait<0>();
+        __syncthreads();
+        // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
+        for (int e = tid; e < 64 * 16; e += 256) {
+            const int r = e >> 4, ch = e & 15;
+            uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
+            const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
+            float qv[8], kv[8];
+            unpack8(*qa, qv);
+            unpack8(ka, kv);
 #pragma unroll
-        for (int t = 0; t < 8; ++t)
+            for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
+            *qa = pack8(qv);
+        }
+        // <H, dH'>: the two tiles share one layout, so matching 16-byte chunks pair up
+        {
+            float sacc = 0.f;
+            for (int e = tid; e < 128 * 16; e += 256) {
+                float hv[8], gv[8];
+                unpack8(reinterpret_cast<const uint4*>(sHt)[e], hv);
+                unpack8(reinterpret_cast<const uint4*>(sdHt)[e], gv);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) de[t][i] += t2[t][i];
-        frag_store_sw<8>(sdE, 64, m0, nk0, de);
-    }
-    publish_smem();
-
-    // ---------------- R3
-    if (ok && tid == 0) {
-        tc_gemm_m64<false, true>(tmem + 0, udE, 64, uH, 128, 128, D, false);        // dE H^T
-        tc_gemm_m64<false, false>(tmem + 128, udE, 64, uV, 64, 64, D, false);       // dE V^T
-        tc_gemm_m64<true, true>(tmem + 192, uM, 64, udE, 64, 128, 64, false);       // M^T dE
-        tc_gemm_m64<false, false>(tmem + 320, uK, 128, uK, 128, 64, D, false);      // K K^T
-    }
-    ok = ok && ms.finish(tid);
-    float dMa[4][4], gr[4][4];
-    if (ok) {
-        float t3[8][4];
-        // dW = -dE H^T (over the dead dH'^T tile)
-        tmem_frag8(tq + 0 + nk0, t3);
-#pragma unroll
-        for (int t = 0; t < 8; ++t)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) t3[t][i] = -t3[t][i];
-        frag_store_sw<8>(sdW, 64, m0, nk0, t3);
-        tmem_frag4(tq + 128 + nl0, dMa);
-#pragma unroll
-        for (int t = 0; t < 4; ++t)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) dMa[t][i] *= sBe[nl0 + frag_col(t, i)];
-        // dV = Diag(beta) M^T dE ; direct dbeta = v . (M^T dE)
-        tmem_frag8(tq + 192 + nk0, t3);
-        float s0, s1;
-        tile_rowdot(t3, sV, 64, 0, s0, s1);
-        put_rows(2, s0, s1);
-        const float ba = sBe[ra], bb = sBe[rb];
-#pragma unroll
-        for (int t = 0; t < 8; ++t) { t3[t][0] *= ba; t3[t][1] *= ba; t3[t][2] *= bb; t3[t][3] *= bb; }
-        frag_stage<8>(stV, m0, nk0, t3);
-        tmem_frag4(tq + 320 + nl0, gr);
-    }
-    publish_smem();
-
-    // ---------------- R4: dM = dE V^T Diag(beta) + dW K^T Diag(btilde gamma_{-1})
-    if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 0, udW, 64, uK, 128, 64, D, false);
-    ok = ok && ms.finish(tid);
-    if (ok) {
-        float mb[4][4];
-        tmem_frag4(tq + 0 + nl0, mb);
-        float rs0 = 0.f, rs1 = 0.f;
-        float cs[4][2];
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-            cs[t][0] = cs[t][1] = 0.f;
-            float ph[4], dm[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
-                const bool incl = c <= r && r < L;
-                const float gam = incl ? __expf(sG[r] - sG[c]) : 0.f;
-                const float w = dP[t][i] * sc[t][i] * gam;   // dP * P
-                if (i < 2) rs0 += w; else rs1 += w;
-                cs[t][i & 1] += w;
-                ph[i] = dP[t][i] * gam;
-                dm[i] = dMa[t][i] + mb[t][i] * sWs[c];
+                for (int i = 0; i < 8; ++i) sacc = fmaf(hv[i], gv[i], sacc);
             }
-            const int c0 = nl0 + frag_col(t, 0);
-            st_pair(sdPh, 64, m0 + frag_row(0), c0, ph[0], ph[1]);
-            st_pair(sdPh, 64, m0 + frag_row(2), c0, ph[2], ph[3]);
-            st_pair(sdM, 64, m0 + frag_row(0), c0, dm[0], dm[1]);
-            st_pair(sdM, 64, m0 + frag_row(2), c0, dm[2], dm[3]);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, o);
+            if (lane == 0) red[warp] = sacc;
         }
-        rs0 = quad_sum(rs0);
-        rs1 = quad_sum(rs1);
-        put_rows(3, rs0, rs1);
-#pragma unroll
-        for (int t = 0; t < 4; ++t)
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const float v = col_sum8(cs[t][e]);
-                if ((lane >> 2) == 0) colp[(0 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
-            }
-    }
-    publish_smem();
+        publish_smem();
 
-    // ---------------- R5: Y = M^T dM
-    if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 64, uM, 64, udM, 64, 64, 64, false);
-    ok = ok && ms.finish(tid);
-    if (ok) {
-        float y[4][4];
-        tmem_frag4(tq + 64 + nl0, y);
-        frag_store_sw<4>(sY, 64, m0, nl0, y);
-    }
-    publish_smem();
+        const float gL = sG[L - 1];
+        const float eGa = __expf(sG[ra]), eGb = __expf(sG[rb]);
+        const float sKa = ra < L ? __expf(gL - sG[ra]) : 0.f, sKb = rb < L ? __expf(gL - sG[rb]) : 0.f;
 
-    // ---------------- R6: dA = -(Y M^T) on the strict lower triangle -> dG
-    if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 128, uY, 64, uM, 64, 64, 64, false);
-    ok = ok && ms.finish(tid);
-    if (ok) {
-        float da[4][4];
-        tmem_frag4(tq + 128 + nl0, da);
-        float rb0 = 0.f, rb1 = 0.f, ra0 = 0.f, ra1 = 0.f;
-        float cs[4][2];
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-            cs[t][0] = cs[t][1] = 0.f;
-            float g4[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
-                const bool strict = c < r && r < L;
-                const float gm = strict ? __expf(sGm1[r] - sG[c]) : 0.f;
-                const float a = -da[t][i];
-                const float u = a * gm * gr[t][i];   // contributes to dbtilde_r
-                const float w = u * sBt[r];          // dA * Aval
-                if (i < 2) { rb0 += u; ra0 += w; } else { rb1 += u; ra1 += w; }
-                cs[t][i & 1] += w;
-                g4[i] = a * sBt[r] * gm;
-            }
-            const int c0 = nl0 + frag_col(t, 0);
-            st_pair(sdG, 64, m0 + frag_row(0), c0, g4[0], g4[1]);
-            st_pair(sdG, 64, m0 + frag_row(2), c0, g4[2], g4[3]);
+        // ---------------- R1
+        if (tid == 0) {
+            tc_gemm_m64<false, false>(tmem + 0, uQK, 128, uK, 128, 64, D, false);      // S = Q~ K^T
+            tc_gemm_m64<false, false>(tmem + 64, udO, 64, uE, 64, 64, D, false);       // dP = dO E^T
+            tc_gemm_m64<false, true>(tmem + 128, udO, 64, uH, 128, 128, D, false);     // dO H^T
+            tc_gemm_m64<false, true>(tmem + 256, uE, 64, udH, 128, 128, D, false);     // E dH'^T
+            tc_gemm_m64<false, false>(tmem + 384, uK, 128, udH, 128, 128, D, false);   // K dH'
         }
-        rb0 = quad_sum(rb0); rb1 = quad_sum(rb1);
-        ra0 = quad_sum(ra0); ra1 = quad_sum(ra1);
-        put_rows(4, rb0, rb1);
-        put_rows(5, ra0, ra1);
-#pragma unroll
-        for (int t = 0; t < 4; ++t)
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const float v = col_sum8(cs[t][e]);
-                if ((lane >> 2) == 0) colp[(1 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
-            }
-    }
-    publish_smem();
-
-    // ---------------- R7: dQ~ += dPhat K ; dK += dPhat^T Q~ + dG K + dG^T K ; M^T dW
-    if (ok && tid == 0) {
-        tc_gemm_m64<false, true>(tmem + 0, udPh, 64, uK, 128, 128, 64, false);
-        tc_gemm_m64<true, true>(tmem + 128, udPh, 64, uQK, 128, 128, 64, false);
-        tc_gemm_m64<false, true>(tmem + 128, udG, 64, uK, 128, 128, 64, true);
-        tc_gemm_m64<true, true>(tmem + 128, udG, 64, uK, 128, 128, 64, true);
-        tc_gemm_m64<true, true>(tmem + 256, uM, 64, udW, 64, 128, 64, false);
-    }
-    ok = ok && ms.finish(tid);
-    if (ok) {
-        float t7[8][4], s0, s1;
-        // dq = dQ~ ; dd partial = -k . dQ~ ; dk -= d dQ~
-        tmem_frag8(tq + 0 + nk0, t7);
-#pragma unroll
-        for (int t = 0; t < 8; ++t)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                acc_dq[t][i] += t7[t][i];
-                acc_dk[t][i] -= dh * acc_dq[t][i];
-            }
-        tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
-        put_rows(6, s0, s1);
-        tmem_frag8(tq + 128 + nk0, t7);
-#pragma unroll
-        for (int t = 0; t < 8; ++t)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) acc_dk[t][i] += t7[t][i];
-        // W path: M^T dW scaled by btilde gamma_{r-1}; its row dot with k feeds dbtilde and d g_{r-1}
-        tmem_frag8(tq + 256 + nk0, t7);
-        tile_rowdot(t7, sQK, 128, 64, s0, s1);
-        put_rows(7, s0, s1);
-        const float wa = sWs[ra], wb = sWs[rb];
-#pragma unroll
-        for (int t = 0; t < 8; ++t) {
-            acc_dk[t][0] += wa * t7[t][0]; acc_dk[t][1] += wa * t7[t][1];
-            acc_dk[t][2] += wb * t7[t][2]; acc_dk[t][3] += wb * t7[t][3];
-        }
-    }
-    __syncthreads();   // every row dot has read the Q~/K tile
-    if (ok) {
-        frag_stage<8>(sQK, m0, nk0, acc_dq);
-        frag_stage<8>(sQK + 16384, m0, nk0, acc_dk);
-    }
-    __syncthreads();
-    if (ok) {
-        const long long ld = (long long)p.H * D;
-        copy_stage_rows((bf16*)p.dq + (t0 * p.H + h) * D, ld, sQK, L, tid);
-        copy_stage_rows((bf16*)p.dkk + (t0 * p.H + h) * D, ld, sQK + 16384, L, tid);
-        copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, ld, stV, L, tid);
-    }
-
-    // ---------------- per-position scalars (rows 0..63, one thread each)
-    auto rsum = [&](int kind, int r) { return rowp[(kind * 2) * 64 + r] + rowp[(kind * 2 + 1) * 64 + r]; };
-    auto csum = [&](int kind, int c) {
-        return colp[(kind * 4 + 0) * 64 + c] + colp[(kind * 4 + 1) * 64 + c] + colp[(kind * 4 + 2) * 64 + c] +
-               colp[(kind * 4 + 3) * 64 + c];
-    };
-    if (ok && tid < 64) {
-        const int r = tid;
-        float g = 0.f;
-        if (r < L) {
-            g = rsum(0, r) - rsum(1, r) + rsum(3, r) - csum(0, r) - csum(1, r);
-            if (r + 1 < L) {
-                g += rsum(5, r + 1);
-                g += sWs[r + 1] * rsum(7, r + 1);
-            }
-        }
-        sDg[r] = g;
-    }
-    __syncthreads();
-    if (ok && warp == 0) {
-        // terms on the last position: gamma_C <H, dH'> and the Kbar total (fixed-order warp
-        // reductions), then d log alpha_j = sum_{r >= j} dg_r, a suffix sum inside the chunk
-        float tk = (lane < L ? rsum(1, lane) : 0.f) + (lane + 32 < L ? rsum(1, lane + 32) : 0.f);
-        float hd = lane < 8 ? red[lane] : 0.f;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            tk += __shfl_xor_sync(0xffffffffu, tk, o);
-            hd += __shfl_xor_sync(0xffffffffu, hd, o);
-        }
-        float x0 = sDg[lane], x1 = sDg[lane + 32];   // zero past L
-        const float last = tk + __expf(gL) * hd;
-        if (L - 1 == lane) x0 += last;
-        if (L - 1 == lane + 32) x1 += last;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const float y0 = __shfl_down_sync(0xffffffffu, x0, o);
-            const float y1 = __shfl_down_sync(0xffffffffu, x1, o);
-            if (lane + o < 32) { x0 += y0; x1 += y1; }
-        }
-        x0 += __shfl_sync(0xffffffffu, x1, 0);
-        sDg[lane] = x0;
-        sDg[lane + 32] = x1;
-    }
-    __syncthreads();
-    if (ok && tid < 64) {
-        const int r = tid;
-        float dbt = 0.f, db_c = 0.f, dd_c = 0.f;
-        if (r < L) {
-            dbt = rsum(4, r) + sEm1[r] * rsum(7, r);
-            p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r];
-            p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * dbt;
-            db_c = sBe[r] * dbt;
-            dd_c = -rsum(6, r);
-        }
-        // fixed-order reduction of the two per-chunk partials over 64 rows
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            db_c += __shfl_xor_sync(0xffffffffu, db_c, o);
-            dd_c += __shfl_xor_sync(0xffffffffu, dd_c, o);
-        }
-        if (lane == 0) { red[warp * 2] = db_c; red[warp * 2 + 1] = dd_c; }
-    }
-    __syncthreads();
-    if (tid == 0) {
+        ok = ms.finish(tid);
+        if (ok && has_next) { load_dH(nxt); cp_async_commit(); }
+        float sc[4][4], dP[4][4], acc_dq[8][4], acc_dk[8][4], de[8][4];
         if (ok) {
-            p.part[idx * 2] = red[0] + red[2];
-            p.part[idx * 2 + 1] = red[1] + red[3];
-        } else {
-            flag_error(p);
+            // P = Tril(S * Gamma)
+            tmem_frag4(tq + 0 + nl0, sc);
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int r = m0 + frag_row(2 * hh), c = nl0 + frag_col(t, 0);
+                    const float gr = sG[r];
+                    const float v0 = (c <= r && r < L) ? sc[t][2 * hh] * __expf(gr - sG[c]) : 0.f;
+                    const float v1 = (c + 1 <= r && r < L) ? sc[t][2 * hh + 1] * __expf(gr - sG[c + 1]) : 0.f;
+                    st_pair(sP, 64, r, c, v0, v1);
+                }
+            tmem_frag4(tq + 64 + nl0, dP);
+            // dQ~ part Diag(gamma) dO H^T; its row dot with Q~ is the log-decay gradient of the Q~ H term
+            tmem_frag8(tq + 128 + nk0, acc_dq);
+#pragma unroll
+            for (int t = 0; t < 8; ++t) { acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb; }
+            float s0, s1;
+            tile_rowdot(acc_dq, sQK, 128, 0, s0, s1);
+            put_rows(0, s0, s1);
+            // dK from Kbar: Diag(gamma_C / gamma_r) E dH'^T
+            tmem_frag8(tq + 256 + nk0, acc_dk);
+#pragma unroll
+            for (int t = 0; t < 8; ++t) { acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb; }
+            tile_rowdot(acc_dk, sQK, 128, 64, s0, s1);
+            put_rows(1, s0, s1);
+            // Kbar dH' part of dE
+            tmem_frag8(tq + 384 + nk0, de);
+#pragma unroll
+            for (int t = 0; t < 8; ++t) { de[t][0] *= sKa; de[t][1] *= sKa; de[t][2] *= sKb; de[t][3] *= sKb; }
         }
+        publish_smem();
+
+        // ---------------- R2: dE = Kbar dH' + P^T dO
+        if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
+        ok = ok && ms.finish(tid);
+        if (ok) {
+            float t2[8][4];
+            tmem_frag8(tq + 0 + nk0, t2);
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) de[t][i] += t2[t][i];
+            frag_store_sw<8>(sdE, 64, m0, nk0, de);
+        }
+        publish_smem();
+
+        // ---------------- R3
+        if (ok && tid == 0) {
+            tc_gemm_m64<false, true>(tmem + 0, udE, 64, uH, 128, 128, D, false);        // dE H^T
+            tc_gemm_m64<false, false>(tmem + 128, udE, 64, uV, 64, 64, D, false);       // dE V^T
+            tc_gemm_m64<true, true>(tmem + 192, uM, 64, udE, 64, 128, 64, false);       // M^T dE
+            tc_gemm_m64<false, false>(tmem + 320, uK, 128, uK, 128, 64, D, false);      // K K^T
+        }
+        ok = ok && ms.finish(tid);
+        if (ok && has_next) { load_H(nxt); cp_async_commit(); }
+        float dMa[4][4], gr[4][4];
+        if (ok) {
+            float t3[8][4];
+            // dW = -dE H^T (over the dead dO tile)
+            tmem_frag8(tq + 0 + nk0, t3);
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) t3[t][i] = -t3[t][i];
+            frag_store_sw<8>(sdW, 64, m0, nk0, t3);
+            tmem_frag4(tq + 128 + nl0, dMa);
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dMa[t][i] *= sBe[nl0 + frag_col(t, i)];
+            // dV = Diag(beta) M^T dE ; direct dbeta = v . (M^T dE)
+            tmem_frag8(tq + 192 + nk0, t3);
+            float s0, s1;
+            tile_rowdot(t3, sV, 64, 0, s0, s1);
+            put_rows(2, s0, s1);
+            const float ba = sBe[ra], bb = sBe[rb];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) { t3[t][0] *= ba; t3[t][1] *= ba; t3[t][2] *= bb; t3[t][3] *= bb; }
+            frag_stage<8>(stV, m0, nk0, t3);
+            tmem_frag4(tq + 320 + nl0, gr);
+        }
+        publish_smem();
+
+        // ---------------- R4: dM = dE V^T Diag(beta) + dW K^T Diag(btilde gamma_{-1}); dv leaves meanwhile
+        if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 0, udW, 64, uK, 128, 64, D, false);
+        if (ok) copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, (long long)p.H * D, stV, L, tid);
+        ok = ok && ms.finish(tid);
+        if (ok && has_next) { load_E(nxt); cp_async_commit(); }
+        if (ok) {
+            float mb[4][4];
+            tmem_frag4(tq + 0 + nl0, mb);
+            float rs0 = 0.f, rs1 = 0.f;
+            float cs[4][2];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                cs[t][0] = cs[t][1] = 0.f;
+                float ph[4], dm[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
+                    const bool incl = c <= r && r < L;
+                    const float gam = incl ? __expf(sG[r] - sG[c]) : 0.f;
+                    const float w = dP[t][i] * sc[t][i] * gam;   // dP * P
+                    if (i < 2) rs0 += w; else rs1 += w;
+                    cs[t][i & 1] += w;
+                    ph[i] = dP[t][i] * gam;
+                    dm[i] = dMa[t][i] + mb[t][i] * sWs[c];
+                }
+                const int c0 = nl0 + frag_col(t, 0);
+                st_pair(sdPh, 64, m0 + frag_row(0), c0, ph[0], ph[1]);
+                st_pair(sdPh, 64, m0 + frag_row(2), c0, ph[2], ph[3]);
+                st_pair(sdM, 64, m0 + frag_row(0), c0, dm[0], dm[1]);
+                st_pair(sdM, 64, m0 + frag_row(2), c0, dm[2], dm[3]);
+            }
+            rs0 = quad_sum(rs0);
+            rs1 = quad_sum(rs1);
+            put_rows(3, rs0, rs1);
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const float v = col_sum8(cs[t][e]);
+                    if ((lane >> 2) == 0) colp[(0 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
+                }
+        }
+        publish_smem();
+
+        // ---------------- R5: Y = M^T dM
+        if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 64, uM, 64, udM, 64, 64, 64, false);
+        ok = ok && ms.finish(tid);
+        if (ok) {
+            float y[4][4];
+            tmem_frag4(tq + 64 + nl0, y);
+            frag_store_sw<4>(sY, 64, m0, nl0, y);
+        }
+        publish_smem();
+
+        // ---------------- R6: dA = -(Y M^T) on the strict lower triangle -> dG
+        if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 128, uY, 64, uM, 64, 64, 64, false);
+        ok = ok && ms.finish(tid);
+        if (ok) {
+            float da[4][4];
+            tmem_frag4(tq + 128 + nl0, da);
+            float rb0 = 0.f, rb1 = 0.f, ra0 = 0.f, ra1 = 0.f;
+            float cs[4][2];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                cs[t][0] = cs[t][1] = 0.f;
+                float g4[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
+                    const bool strict = c < r && r < L;
+                    const float gm = strict ? __expf(sGm1[r] - sG[c]) : 0.f;
+                    const float a = -da[t][i];
+                    const float uu = a * gm * gr[t][i];   // contributes to dbtilde_r
+                    const float w = uu * sBt[r];          // dA * Aval
+                    if (i < 2) { rb0 += uu; ra0 += w; } else { rb1 += uu; ra1 += w; }
+                    cs[t][i & 1] += w;
+                    g4[i] = a * sBt[r] * gm;
+                }
+                const int c0 = nl0 + frag_col(t, 0);
+                st_pair(sdG, 64, m0 + frag_row(0), c0, g4[0], g4[1]);
+                st_pair(sdG, 64, m0 + frag_row(2), c0, g4[2], g4[3]);
+            }
+            rb0 = quad_sum(rb0); rb1 = quad_sum(rb1);
+            ra0 = quad_sum(ra0); ra1 = quad_sum(ra1);
+            put_rows(4, rb0, rb1);
+            put_rows(5, ra0, ra1);
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const float v = col_sum8(cs[t][e]);
+                    if ((lane >> 2) == 0) colp[(1 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
+                }
+        }
+        publish_smem();
+
+        // ---------------- R7: dQ~ += dPhat K ; dK += dPhat^T Q~ + dG K + dG^T K ; M^T dW
+        if (ok && tid == 0) {
+            tc_gemm_m64<false, true>(tmem + 0, udPh, 64, uK, 128, 128, 64, false);
+            tc_gemm_m64<true, true>(tmem + 128, udPh, 64, uQK, 128, 128, 64, false);
+            tc_gemm_m64<false, true>(tmem + 128, udG, 64, uK, 128, 128, 64, true);
+            tc_gemm_m64<true, true>(tmem + 128, udG, 64, uK, 128, 128, 64, true);
+            tc_gemm_m64<true, true>(tmem + 256, uM, 64, udW, 64, 128, 64, false);
+        }
+        ok = ok && ms.finish(tid);
+        if (ok && has_next) {
+            load_tok(sdO, p.dO, nxt);
+            load_tok(sV, p.v, nxt);
+            load_M(nxt);
+            cp_async_commit();
+        }
+        if (ok) {
+            float t7[8][4], s0, s1;
+            // dq = dQ~ ; dd partial = -k . dQ~ ; dk -= d dQ~
+            tmem_frag8(tq + 0 + nk0, t7);
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    acc_dq[t][i] += t7[t][i];
+                    acc_dk[t][i] -= dh * acc_dq[t][i];
+                }
+            tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
+            put_rows(6, s0, s1);
+            tmem_frag8(tq + 128 + nk0, t7);
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc_dk[t][i] += t7[t][i];
+            // W path: M^T dW scaled by btilde gamma_{r-1}; its row dot with k feeds dbtilde and d g_{r-1}
+            tmem_frag8(tq + 256 + nk0, t7);
+            tile_rowdot(t7, sQK, 128, 64, s0, s1);
+            put_rows(7, s0, s1);
+            const float wa = sWs[ra], wb = sWs[rb];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                acc_dk[t][0] += wa * t7[t][0]; acc_dk[t][1] += wa * t7[t][1];
+                acc_dk[t][2] += wb * t7[t][2]; acc_dk[t][3] += wb * t7[t][3];
+            }
+        }
+        __syncthreads();   // every row dot has read the Q~/K tile
+        if (ok) {
+            frag_stage<8>(sQK, m0, nk0, acc_dq);
+            frag_stage<8>(sQK + 16384, m0, nk0, acc_dk);
+        }
+        __syncthreads();
+        if (ok) {
+            const long long ld = (long long)p.H * D;
+            copy_stage_rows((bf16*)p.dq + (t0 * p.H + h) * D, ld, sQK, L, tid);
+            copy_stage_rows((bf16*)p.dkk + (t0 * p.H + h) * D, ld, sQK + 16384, L, tid);
+        }
+
+        // ---------------- per-position scalars (rows 0..63, one thread each)
+        auto rsum = [&](int kind, int r) { return rowp[(kind * 2) * 64 + r] + rowp[(kind * 2 + 1) * 64 + r]; };
+        auto csum = [&](int kind, int c) {
+            return colp[(kind * 4 + 0) * 64 + c] + colp[(kind * 4 + 1) * 64 + c] + colp[(kind * 4 + 2) * 64 + c] +
+                   colp[(kind * 4 + 3) * 64 + c];
+        };
+        if (ok && tid < 64) {
+            const int r = tid;
+            float g = 0.f;
+            if (r < L) {
+                g = rsum(0, r) - rsum(1, r) + rsum(3, r) - csum(0, r) - csum(1, r);
+                if (r + 1 < L) {
+                    g += rsum(5, r + 1);
+                    g += sWs[r + 1] * rsum(7, r + 1);
+                }
+            }
+            sDg[r] = g;
+        }
+        __syncthreads();
+        if (ok && warp == 0) {
+            // terms on the last position: gamma_C <H, dH'> and the Kbar total (fixed-order warp
+            // reductions), then d log alpha_j = sum_{r >= j} dg_r, a suffix sum inside the chunk
+            float tk = (lane < L ? rsum(1, lane) : 0.f) + (lane + 32 < L ? rsum(1, lane + 32) : 0.f);
+            float hd = lane < 8 ? red[lane] : 0.f;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                tk += __shfl_xor_sync(0xffffffffu, tk, o);
+                hd += __shfl_xor_sync(0xffffffffu, hd, o);
+            }
+            float x0 = sDg[lane], x1 = sDg[lane + 32];   // zero past L
+            const float last = tk + __expf(gL) * hd;
+            if (L - 1 == lane) x0 += last;
+            if (L - 1 == lane + 32) x1 += last;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const float y0 = __shfl_down_sync(0xffffffffu, x0, o);
+                const float y1 = __shfl_down_sync(0xffffffffu, x1, o);
+                if (lane + o < 32) { x0 += y0; x1 += y1; }
+            }
+            x0 += __shfl_sync(0xffffffffu, x1, 0);
+            sDg[lane] = x0;
+            sDg[lane + 32] = x1;
+        }
+        __syncthreads();
+        if (ok && tid < 64) {
+            const int r = tid;
+            float dbt = 0.f, db_c = 0.f, dd_c = 0.f;
+            if (r < L) {
+                dbt = rsum(4, r) + sEm1[r] * rsum(7, r);
+                p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r];
+                p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * dbt;
+                db_c = sBe[r] * dbt;
+                dd_c = -rsum(6, r);
+            }
+            // fixed-order reduction of the two per-chunk partials over 64 rows
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                db_c += __shfl_xor_sync(0xffffffffu, db_c, o);
+                dd_c += __shfl_xor_sync(0xffffffffu, dd_c, o);
+            }
+            if (lane == 0) { red[warp * 2] = db_c; red[warp * 2 + 1] = dd_c; }
+        }
+        __syncthreads();
+        if (tid == 0) {
+            if (ok) {
+                p.part[idx * 2] = red[0] + red[2];
+                p.part[idx * 2 + 1] = red[1] + red[3];
+            } else {
+                flag_error(p);
+            }
+        }
+        __syncthreads();   // the next unit's Q/K copies overwrite the staging tile read above
+        pre = has_next;
     }
+    cp_async_wait<0>();   // no copy is still writing shared memory at exit
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -581,7 +630,11 @@ cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s) {
     const size_t sm = tc::LocalTcSmem::bytes();
     cudaError_t e = cudaFuncSetAttribute(tc::k_bwd_local_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
-    if (p.slots > 0) tc::k_bwd_local_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p);
+    int dev = 0, nsm = 0;
+    if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
+    const long long units = (long long)p.slots * p.H;
+    const int grid = (int)(units < nsm ? units : nsm);   // one resident CTA per SM
+    if (grid > 0) tc::k_bwd_local_tc<<<grid, 256, sm, s>>>(p, units);
     return cudaGetLastError();
 }
 

@@ -241,6 +241,203 @@ __global__ void __launch_bounds__(256, 1)
     }
 }
 
+// Row-split variant (dk = dv = 128): two CTAs per (sequence, head), each owning 64 of
+// the state's dv rows (rows are independent under S^T <- gamma S^T + S^T X^T + Y).
+// The MMA is M = 64 (this CTA's rows) x N = dk x K = dk against the full X; read
+// back with tcgen05.ld.16x256b, the accumulator arrives in the m16n8 fragment
+// layout, so each thread keeps 32 state values (rows 16 (w & 3) + g, + 8; columns
+// 64 (w >> 2) + 8 t + 2 q, + 1).  Per chunk each SM loads X plus half of Y and
+// stores half of the chunk state, and the epilogue is half as long.
+template <int DK, int DV>
+struct ScanSplitSmem {
+    static constexpr int SX = 3, SY = 2;
+    static constexpr uint32_t A_BYTES = 64 * DK * 2;    // this CTA's 64 rows of S^T; two buffers
+    static constexpr uint32_t X_BYTES = DK * DK * 2;
+    static constexpr uint32_t Y_BYTES = 64 * DK * 2;
+    static constexpr uint32_t OX = 2 * A_BYTES;
+    static constexpr uint32_t OY = OX + SX * X_BYTES;
+    static constexpr size_t bytes() { return 1024 + OY + (size_t)SY * Y_BYTES; }
+};
+
+template <int DK, int DV, bool XMN>
+__global__ void __launch_bounds__(256, 1)
+    k_scan_tc_split(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY,
+                    const __grid_constant__ CUtensorMap tmS) {
+    static_assert(DK == 128 && DV == 128, "row split is laid out for dk = dv = 128");
+    using S = ScanSplitSmem<DK, DV>;
+    constexpr int NT = DK / 16;   // 8-column tiles per thread (half of the columns)
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t full_x[S::SX], full_y[S::SY];
+    __shared__ uint64_t mma_bar;
+    __shared__ uint32_t tmem_base;
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int n = blockIdx.x >> 1, rhalf = blockIdx.x & 1, h = blockIdx.y;
+    const int wr = warp & 3, wc = warp >> 2;
+    const int r0 = 16 * wr + (lane >> 2);          // local rows r0, r0 + 8
+    const int cq = 64 * wc + 2 * (lane & 3);       // columns cq + 8 t, + 1
+    const uint32_t smem_u = smem_u32(smem);
+
+    float st[NT][4];
+    {
+        const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int j = 64 * rhalf + r0 + 8 * (i >> 1), m = cq + 8 * t + (i & 1);
+                st[t][i] = init ? init[(long long)m * DV + j] : 0.f;
+            }
+    }
+
+    long long start, len;
+    scan_seq_range(a, n, start, len);
+    const int s0 = a.seq_first[n];
+    int nch = (int)((len + kChunk - 1) / kChunk);
+    if (s0 + nch > a.slots) nch = a.slots - s0 > 0 ? a.slots - s0 : 0;
+
+    if (tid == 0) {
+        for (int s = 0; s < S::SX; ++s) mbar_init(smem_u32(&full_x[s]), 1);
+        for (int s = 0; s < S::SY; ++s) mbar_init(smem_u32(&full_y[s]), 1);
+        mbar_init(smem_u32(&mma_bar), 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&tmem_base), DK);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+    const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16) + 64 * wc;
+
+    auto chunk_of = [&](int it) { return a.reverse ? nch - 1 - it : it; };
+    auto unit_of = [&](int it) { return (long long)(s0 + chunk_of(it)) * a.H + h; };
+    auto a_buf = [&](int it) { return smem_u + (uint32_t)(it & 1) * S::A_BYTES; };
+    auto x_buf = [&](int it) { return smem_u + S::OX + (uint32_t)(it % S::SX) * S::X_BYTES; };
+    auto y_off = [&](int it) { return S::OY + (uint32_t)(it % S::SY) * S::Y_BYTES; };
+    auto issue_x = [&](int it) {
+        const uint32_t fb = smem_u32(&full_x[it % S::SX]);
+        mbar_expect_tx(fb, S::X_BYTES);
+#pragma unroll
+        for (int half = 0; half < DK / 64; ++half)
+            tma_load_2d(x_buf(it) + half * DK * 128, &tmX, half * 64, (int)(unit_of(it) * DK), fb);
+    };
+    auto issue_y = [&](int it) {
+        const uint32_t fb = smem_u32(&full_y[it % S::SY]);
+        mbar_expect_tx(fb, S::Y_BYTES);
+#pragma unroll
+        for (int half = 0; half < DK / 64; ++half)
+            tma_load_2d(smem_u + y_off(it) + half * 64 * 128, &tmY, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), fb);
+    };
+    int nx = 0, ny = 0;
+    if (tid == 0) {
+        for (; nx < S::SX - 1 && nx < nch; ++nx) issue_x(nx);
+        for (; ny < S::SY - 1 && ny < nch; ++ny) issue_y(ny);
+    }
+
+    constexpr uint32_t idesc = idesc_bf16_f32(64, DK) | (XMN ? 1u << 16 : 0u);
+    auto log_decay = [&](int it) {
+        const int c = chunk_of(it);
+        const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
+        return __ldg(a.Gb + unit_of(it) * 64 + L - 1);
+    };
+    float g_next = nch > 0 ? log_decay(0) : 0.f;
+    for (int it = 0; it < nch; ++it) {
+        const float gam = expf(g_next);
+        if (it + 1 < nch) g_next = log_decay(it + 1);
+
+        // this CTA's rows of the chunk's starting state: bf16 A operand in buffer it % 2
+        uint8_t* sA = smem + (it & 1) * S::A_BYTES;
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh)
+                *reinterpret_cast<__nv_bfloat162*>(sA + sw128_offset(r0 + 8 * hh, cq + 8 * t, 64)) =
+                    __floats2bfloat162_rn(st[t][2 * hh], st[t][2 * hh + 1]);
+        fence_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+
+        int bad = 0;
+        if (tid == 0) {
+            if (mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
+#pragma unroll
+                for (int ks = 0; ks < DK / 16; ++ks) {
+                    const int half = ks >> 2, sub = ks & 3;
+                    const uint64_t ad = smem_desc_sw128(a_buf(it) + half * 64 * 128 + sub * 32);
+                    const uint64_t bd = XMN ? desc_mnmajor(x_buf(it), DK, ks)
+                                            : smem_desc_sw128(x_buf(it) + half * DK * 128 + sub * 32);
+                    tc_mma_bf16(tmem, ad, bd, idesc, ks > 0 ? 1u : 0u);
+                }
+            } else {
+                bad = 1;
+            }
+            tc_commit(smem_u32(&mma_bar));
+#pragma unroll
+            for (int half = 0; half < DK / 64; ++half)
+                tma_store_2d(&tmS, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), a_buf(it) + half * 64 * 128);
+            bulk_commit();
+            if (nx < nch) issue_x(nx++);
+            if (ny < nch) issue_y(ny++);
+        }
+        if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
+        if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1)) bad = 1;
+        if (tid == 0) bulk_wait_read<1>();
+        if (__syncthreads_or(bad)) {
+            if (tid == 0) {
+                if (a.err) atomicExch(a.err, 1);
+                for (int c = it; c < nx; ++c) mbar_wait(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
+                for (int c = it; c < ny; ++c) mbar_wait(smem_u32(&full_y[c % S::SY]), (c / S::SY) & 1);
+            }
+            break;
+        }
+        tc_fence_after();
+
+        // S^T <- gamma S^T + (S^T X^T) + Y  on this thread's 32 values
+        uint32_t d[32];
+        asm volatile(
+            "tcgen05.ld.sync.aligned.16x256b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+            "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+            : "=r"(d[0]), "=r"(d[1]), "=r"(d[2]), "=r"(d[3]), "=r"(d[4]), "=r"(d[5]), "=r"(d[6]), "=r"(d[7]),
+              "=r"(d[8]), "=r"(d[9]), "=r"(d[10]), "=r"(d[11]), "=r"(d[12]), "=r"(d[13]), "=r"(d[14]), "=r"(d[15]),
+              "=r"(d[16]), "=r"(d[17]), "=r"(d[18]), "=r"(d[19]), "=r"(d[20]), "=r"(d[21]), "=r"(d[22]), "=r"(d[23]),
+              "=r"(d[24]), "=r"(d[25]), "=r"(d[26]), "=r"(d[27]), "=r"(d[28]), "=r"(d[29]), "=r"(d[30]), "=r"(d[31])
+            : "r"(tq));
+        const uint8_t* sY = smem + y_off(it);
+        __nv_bfloat162 yv[NT][2];
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh)
+                yv[t][hh] = *reinterpret_cast<const __nv_bfloat162*>(sY + sw128_offset(r0 + 8 * hh, cq + 8 * t, 64));
+        tmem_wait_ld();
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+                const float2 yf = __bfloat1622float2(yv[t][hh]);
+                st[t][2 * hh] = fmaf(gam, st[t][2 * hh], __uint_as_float(d[4 * t + 2 * hh]) + yf.x);
+                st[t][2 * hh + 1] = fmaf(gam, st[t][2 * hh + 1], __uint_as_float(d[4 * t + 2 * hh + 1]) + yf.y);
+            }
+        tc_fence_before();
+    }
+
+    if (tid == 0) bulk_wait_all();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, DK);
+    if (a.fin) {
+        float* fin = a.fin + ((long long)n * a.H + h) * DK * DV;
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int j = 64 * rhalf + r0 + 8 * (i >> 1), m = cq + 8 * t + (i & 1);
+                fin[(long long)m * DV + j] = st[t][i];
+            }
+    }
+}
+
 // ------------------------------------------------------------- fp32 path
 
 template <int DK>
@@ -353,7 +550,22 @@ static bool make_map(CUtensorMap* m, const void* base, long long rows, int cols,
 }
 
 template <int DK, int DV, bool XMN>
+static cudaError_t run_scan_tc_split(const ScanArgs& a, long long pairs, cudaStream_t s) {
+    using S = ScanSplitSmem<DK, DV>;
+    CUtensorMap tx, ty, ts;
+    if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, 64) ||
+        !make_map(&ts, a.Sout, pairs * DV, DK, 64))
+        return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k_scan_tc_split<DK, DV, XMN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)S::bytes());
+    if (e) return e;
+    k_scan_tc_split<DK, DV, XMN><<<dim3(2 * a.N, a.H), 256, S::bytes(), s>>>(a, tx, ty, ts);
+    return cudaGetLastError();
+}
+
+template <int DK, int DV, bool XMN>
 static cudaError_t run_scan_tc(const ScanArgs& a, long long pairs, cudaStream_t s) {
+    if constexpr (DK == 128 && DV == 128) return run_scan_tc_split<DK, DV, XMN>(a, pairs, s);
     using S = ScanTcSmem<DK, DV>;
     CUtensorMap tx, ty, ts;
     if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, DV) ||
@@ -388,7 +600,7 @@ cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long lo
 
 size_t scan_smem_bytes(bool is_bf16, int dk, int dv) {
     if (is_bf16) {
-        if (dk == 128) return dv == 128 ? ScanTcSmem<128, 128>::bytes() : ScanTcSmem<128, 64>::bytes();
+        if (dk == 128) return dv == 128 ? ScanSplitSmem<128, 128>::bytes() : ScanTcSmem<128, 64>::bytes();
         return dv == 128 ? ScanTcSmem<64, 128>::bytes() : ScanTcSmem<64, 64>::bytes();
     }
     return dk == 128 ? ScanSimtSmem<128>::bytes() : ScanSimtSmem<64>::bytes();
