@@ -48,11 +48,11 @@ def build(force: bool = False) -> str:
 def _bind(lib):
     P = ctypes.c_void_p
     I = ctypes.c_int
-    lib.comba_oracle_fwd.argtypes = [I, P, I, I, I] + [P] * 10 + [I]
+    lib.comba_oracle_fwd.argtypes = [I, P, I, I, I] + [P] * 10 + [I, I]
     lib.comba_oracle_fwd.restype = I
-    lib.comba_oracle_bwd.argtypes = [I, P, I, I, I] + [P] * 8 + [P, P] + [P] * 8 + [I]
+    lib.comba_oracle_bwd.argtypes = [I, P, I, I, I] + [P] * 8 + [P, P] + [P] * 8 + [I, I]
     lib.comba_oracle_bwd.restype = I
-    lib.comba_oracle_step.argtypes = [I, I, I, I] + [P] * 9 + [I]
+    lib.comba_oracle_step.argtypes = [I, I, I, I] + [P] * 9 + [I, I]
     lib.comba_oracle_step.restype = I
     return lib
 
@@ -112,8 +112,13 @@ def _packed(q, k, v, alpha, beta, cu_seqlens):
     return q, k, v, alpha, beta, cu, shape
 
 
-def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=None):
-    """Token recurrence forward.  Returns ``(o, hT)`` in float64."""
+VARIANTS = {"splr": 0, "iplr": 1}
+
+
+def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=None, variant="splr"):
+    """Token recurrence forward.  Returns ``(o, hT)`` in float64.
+
+    ``variant="iplr"``: the Comba-iplr transition alpha (I - 2 btilde k k^T)."""
     q, k, v, alpha, beta, b, d, h0 = map(_f64, (q, k, v, alpha, beta, b, d, h0))
     q, k, v, alpha, beta, cu, shape = _packed(q, k, v, alpha, beta, cu_seqlens)
     Ttot, H, dk = q.shape
@@ -123,7 +128,8 @@ def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=
     o = np.zeros((Ttot, H, dv), np.float64)
     hT = np.zeros((N, H, dk, dv), np.float64)
     rc = (lib or _load()).comba_oracle_fwd(N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta),
-                                  _ptr(b), _ptr(d), _ptr(h0), _ptr(o), _ptr(hT), threads or default_threads())
+                                  _ptr(b), _ptr(d), _ptr(h0), _ptr(o), _ptr(hT), threads or default_threads(),
+                                  VARIANTS[variant])
     if rc:
         raise MemoryError("oracle forward failed to allocate")
     if shape is not None:
@@ -131,7 +137,8 @@ def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=
     return o, hT
 
 
-def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, threads=None, lib=None):
+def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, threads=None, lib=None,
+        variant="splr"):
     """Exact BPTT.  Returns a dict with dq, dk, dv, dalpha, dbeta, db, dd, dh0."""
     q, k, v, alpha, beta, b, d, h0, dO, dhT = map(_f64, (q, k, v, alpha, beta, b, d, h0, dO, dhT))
     batched = q.ndim == 4
@@ -150,7 +157,8 @@ def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, thre
     rc = (lib or _load()).comba_oracle_bwd(
         N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b), _ptr(d), _ptr(h0),
         _ptr(dO), _ptr(dhT), _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]), _ptr(out["dalpha"]),
-        _ptr(out["dbeta"]), _ptr(out["db"]), _ptr(out["dd"]), _ptr(out["dh0"]), threads or default_threads())
+        _ptr(out["dbeta"]), _ptr(out["db"]), _ptr(out["dd"]), _ptr(out["dh0"]), threads or default_threads(),
+        VARIANTS[variant])
     if rc:
         raise MemoryError("oracle backward failed to allocate")
     if shape is not None:
@@ -162,7 +170,7 @@ def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, thre
     return out
 
 
-def step(q, k, v, alpha, beta, b, d, state, threads=None, lib=None):
+def step(q, k, v, alpha, beta, b, d, state, threads=None, lib=None, variant="splr"):
     """One decode token.  ``state`` [Bd,H,dk,dv] is copied, updated and returned with ``o``."""
     q, k, v, alpha, beta, b, d = map(_f64, (q, k, v, alpha, beta, b, d))
     st = np.array(state, dtype=np.float64, copy=True, order="C")
@@ -170,7 +178,7 @@ def step(q, k, v, alpha, beta, b, d, state, threads=None, lib=None):
     dv = v.shape[-1]
     o = np.zeros((Bd, H, dv), np.float64)
     rc = (lib or _load()).comba_oracle_step(Bd, H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b),
-                                   _ptr(d), _ptr(st), _ptr(o), threads or default_threads())
+                                   _ptr(d), _ptr(st), _ptr(o), threads or default_threads(), VARIANTS[variant])
     if rc:
         raise MemoryError("oracle step failed to allocate")
     return o, st

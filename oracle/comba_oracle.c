@@ -18,6 +18,10 @@
  *
  * H_0 = h0 (zero if absent); hT = H_T.  No query scale (the paper has none).
  *
+ * Variant 1 is Comba-iplr (table of state transitions for the Comba variants):
+ * the transition alpha_t (I - 2 btilde_t k_t k_t^T), i.e. the same recurrence
+ * with the feedback strength btilde_t replaced by 2 alpha_t b_h beta_t.
+ *
  * The backward pass is exact back-propagation through time of that
  * recurrence (the paper prints no backward; these are the chain-rule
  * derivatives of the four lines above).  States are checkpointed every
@@ -49,7 +53,11 @@ typedef struct {
     double *db_part, *dd_part; /* [N*H] */
     int nthreads, tid;
     int status;
+    int variant; /* 0: SPLR (alpha - btilde k k^T); 1: iplr alpha (I - 2 btilde k k^T) */
 } job_t;
+
+/* Feedback strength of token t relative to b_h beta_t: 1, or 2 alpha_t for iplr. */
+static double fb_scale(const job_t *J, double a) { return J->variant == 1 ? 2.0 * a : 1.0; }
 
 /* ---------------------------------------------------------------- forward */
 
@@ -70,7 +78,7 @@ static void fwd_unit(const job_t *J, int n, int h, double *Hs, double *x, double
         const double *vt = J->v + ((size_t)t * Hh + h) * dv;
         const double a = J->alpha[(size_t)t * Hh + h];
         const double be = J->beta[(size_t)t * Hh + h];
-        const double bt = bh * be;
+        const double bt = bh * be * fb_scale(J, a);
         /* x = H^T k, read from the state before this token's update */
         for (int j = 0; j < dv; ++j) x[j] = 0.0;
         for (int i = 0; i < dk; ++i) {
@@ -159,7 +167,7 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
             for (int j = 0; j < dv; ++j) x[j] = 0.0;
             for (int i = 0; i < dk; ++i)
                 for (int j = 0; j < dv; ++j) x[j] += Hn[(size_t)i * dv + j] * kt[i];
-            for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bh * be * x[j];
+            for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bh * be * fb_scale(J, a) * x[j];
             for (int i = 0; i < dk; ++i)
                 for (int j = 0; j < dv; ++j) Hn[(size_t)i * dv + j] = a * Hn[(size_t)i * dv + j] + kt[i] * e[j];
         }
@@ -186,7 +194,7 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
             for (int j = 0; j < dv; ++j) x[j] = 0.0;
             for (int i = 0; i < dk; ++i)
                 for (int j = 0; j < dv; ++j) x[j] += P[(size_t)i * dv + j] * kt[i];
-            for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bh * be * x[j];
+            for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bh * be * fb_scale(J, a) * x[j];
             for (int i = 0; i < dk; ++i)
                 for (int j = 0; j < dv; ++j) Q[(size_t)i * dv + j] = a * P[(size_t)i * dv + j] + kt[i] * e[j];
         }
@@ -196,7 +204,8 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
             const double *kt = J->k + tk, *qt = J->q + tk, *vt = J->v + tv, *dOt = J->dO + tv;
             const double a = J->alpha[(size_t)t * Hh + h];
             const double be = J->beta[(size_t)t * Hh + h];
-            const double bt = bh * be;
+            const double f = fb_scale(J, a);
+            const double bt = bh * be * f;
             const double *P = seg + (size_t)r * ssz;       /* H_{t-1} */
             const double *Hc = seg + (size_t)(r + 1) * ssz; /* H_t     */
             /* recompute x_t, e_t */
@@ -243,8 +252,10 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
                 vde += vt[j] * de[j];
                 xde += x[j] * de[j];
             }
-            J->dbeta[(size_t)t * Hh + h] = vde - bh * xde;
-            db_acc -= be * xde;
+            /* dbtilde = -x.de, through btilde = b beta f (f = 1, or 2 alpha for iplr) */
+            J->dbeta[(size_t)t * Hh + h] = vde - bh * f * xde;
+            db_acc -= be * f * xde;
+            if (J->variant == 1) J->dalpha[(size_t)t * Hh + h] -= 2.0 * bh * be * xde;
             dd_acc -= kdq;
             /* carry to H_{t-1} */
             for (int i = 0; i < dk; ++i)
@@ -321,10 +332,11 @@ static int run_pool(job_t *proto, void *(*fn)(void *))
 int comba_oracle_fwd(int N, const int64_t *cu, int H, int dk, int dv,
                      const double *q, const double *k, const double *v,
                      const double *alpha, const double *beta, const double *b, const double *d,
-                     const double *h0, double *o, double *hT, int nthreads)
+                     const double *h0, double *o, double *hT, int nthreads, int variant)
 {
     job_t J;
     memset(&J, 0, sizeof(J));
+    J.variant = variant;
     J.N = N; J.H = H; J.dk = dk; J.dv = dv; J.cu = cu;
     J.q = q; J.k = k; J.v = v; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d; J.h0 = h0;
     J.o = o; J.hT = hT; J.nthreads = nthreads;
@@ -336,10 +348,11 @@ int comba_oracle_bwd(int N, const int64_t *cu, int H, int dk, int dv,
                      const double *alpha, const double *beta, const double *b, const double *d,
                      const double *h0, const double *dO, const double *dhT,
                      double *dq, double *dk_, double *dv_, double *dalpha, double *dbeta,
-                     double *db, double *dd, double *dh0, int nthreads)
+                     double *db, double *dd, double *dh0, int nthreads, int variant)
 {
     job_t J;
     memset(&J, 0, sizeof(J));
+    J.variant = variant;
     J.N = N; J.H = H; J.dk = dk; J.dv = dv; J.cu = cu;
     J.q = q; J.k = k; J.v = v; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d; J.h0 = h0;
     J.dO = dO; J.dhT = dhT;
@@ -380,7 +393,7 @@ static void *step_worker(void *arg)
             const double *kt = J->k + (size_t)u * dk, *qt = J->q + (size_t)u * dk, *vt = J->v + (size_t)u * dv;
             double *Hs = J->hT + (size_t)u * dk * dv;
             const double a = J->alpha[u], be = J->beta[u];
-            const double bt = (J->b ? J->b[h] : 1.0) * be;
+            const double bt = (J->b ? J->b[h] : 1.0) * be * fb_scale(J, a);
             for (int j = 0; j < dv; ++j) x[j] = 0.0;
             for (int r = 0; r < dk; ++r)
                 for (int j = 0; j < dv; ++j) x[j] += Hs[(size_t)r * dv + j] * kt[r];
@@ -401,10 +414,11 @@ static void *step_worker(void *arg)
 int comba_oracle_step(int Bd, int H, int dk, int dv,
                       const double *q, const double *k, const double *v,
                       const double *alpha, const double *beta, const double *b, const double *d,
-                      double *state, double *o, int nthreads)
+                      double *state, double *o, int nthreads, int variant)
 {
     job_t J;
     memset(&J, 0, sizeof(J));
+    J.variant = variant;
     J.N = Bd; J.H = H; J.dk = dk; J.dv = dv;
     J.q = q; J.k = k; J.v = v; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d;
     J.hT = state; J.o = o; J.nthreads = nthreads;

@@ -16,7 +16,7 @@ MUTATIONS = {
     "feedback_reads_decayed_state": ("x[j] += row[j] * ki;", "x[j] += a * row[j] * ki;"),
     "no_output_correction": ("qn[i] = qt[i] - dh * kt[i];", "qn[i] = qt[i];"),
     "feedback_sign_flipped": ("e[j] = be * vt[j] - bt * x[j];", "e[j] = be * vt[j] + bt * x[j];"),
-    "btilde_ignores_b": ("const double bt = bh * be;", "const double bt = be;"),
+    "btilde_ignores_b": ("const double bt = bh * be * fb_scale(J, a);", "const double bt = be * fb_scale(J, a);"),
     "bwd_drops_feedback_term_in_dk": ("dkt[i] = ge - bt * pde - dh * dqn[i];", "dkt[i] = ge - dh * dqn[i];"),
     "bwd_dalpha_uses_new_state": ("da += G[(size_t)i * dv + j] * P[(size_t)i * dv + j];",
                                   "da += G[(size_t)i * dv + j] * Hc[(size_t)i * dv + j];"),
