@@ -320,6 +320,7 @@ def run_ours(args, world, rank, local):
     from paper_2506_02475_gb300 import binding
 
     peaks, peak_src = load_peaks()
+    iplr = args.variant == "iplr"
     # weak scaling: each rank owns its own batch of sequences (same parameters, own data)
     w = inputs.make(args.workload, seed_offset=shard.rank_seed_offset(rank))
     dev = torch.device("cuda", local)
@@ -357,10 +358,10 @@ def run_ours(args, world, rank, local):
     def step(t, events=True):
         # training step: the forward keeps the backward's chunk factors, the backward reuses them
         comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"], cu_seqlens=cu,
-                        o=o, hT=hT, workspace=ws, stage_events=hf if events else None, save_factors=True)
+                        o=o, hT=hT, workspace=ws, stage_events=hf if events else None, save_factors=True, iplr=iplr)
         comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
                         dhT=t["dhT"], cu_seqlens=cu, out=grads, workspace=ws, stage_events=hb if events else None,
-                        reuse_factors=True)
+                        reuse_factors=True, iplr=iplr)
 
     for _ in range(args.warmup):
         flush.zero_()
@@ -463,10 +464,10 @@ def run_ours(args, world, rank, local):
                 comp.wait_event(ev["downloaded"][j])          # step i-2's results are on the host
             comba_chunk_fwd(dbuf["q"], dbuf["k"], dbuf["v"], dbuf["alpha"], dbuf["beta"], dbuf["d"], b=dbuf["b"],
                             h0=dbuf["h0"], cu_seqlens=cu, o=douts["o"], hT=douts["hT"], workspace=ws,
-                            save_factors=True)
+                            save_factors=True, iplr=iplr)
             comba_chunk_bwd(dbuf["q"], dbuf["k"], dbuf["v"], dbuf["alpha"], dbuf["beta"], dbuf["d"], dbuf["dO"],
                             b=dbuf["b"], h0=dbuf["h0"], dhT=dbuf["dhT"], cu_seqlens=cu,
-                            out={k: douts[k] for k in grads}, workspace=ws, reuse_factors=True)
+                            out={k: douts[k] for k in grads}, workspace=ws, reuse_factors=True, iplr=iplr)
             ev["consumed"][j].record(comp)
             ev["computed"][j].record(comp)
             with torch.cuda.stream(down):
@@ -502,7 +503,8 @@ def run_ours(args, world, rank, local):
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; paper's layer shape and gate ranges)",
-            "config": {"workload": f"{args.workload}: " + workload_desc(w), "global_batch": w.num_seqs * world,
+            "config": {"workload": f"{args.workload}: " + workload_desc(w), "variant": args.variant,
+                       "global_batch": w.num_seqs * world,
                        "seq_len": int(w.q.shape[1]) if w.cu_seqlens is None else int(w.tokens),
                        "parallelism": f"data-parallel x{world}: each rank its own sequences, no data-path collective",
                        "l2": "device-timed steps: flushed between steps (256 MiB write, outside the events); "
@@ -637,6 +639,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="lm1p3b", choices=["lm1p3b", "lm340m", "varlen64k", "decode"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--variant", default="splr", choices=["splr", "iplr"],
+                    help="state transition: Comba (alpha - btilde k k^T) or Comba-iplr alpha (I - 2 btilde k k^T)")
     ap.add_argument("--reference-tokens", type=int, default=512)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":

@@ -72,7 +72,7 @@ typedef struct {
     const int32_t *cu_seqlens;  /* device int32 [N+1] or NULL                     */
     comba_dtype_t dtype;        /* storage type of q, k, v, o and their grads     */
     int chunk;                  /* chunk length; must be 64                       */
-    int flags;                  /* 0, or COMBA_SAVE_FACTORS / COMBA_REUSE_FACTORS */
+    int flags;                  /* COMBA_SAVE_FACTORS / COMBA_REUSE_FACTORS, | COMBA_IPLR */
     /* Optional instrumentation (NULL / 0 = off).  Caller-created cudaEvent_t
      * handles recorded on `stream` at kernel boundaries: comba_chunk_fwd
      * records COMBA_FWD_EVENTS of them (before chunk map, prep, state scan,
@@ -101,6 +101,17 @@ typedef struct {
  */
 #define COMBA_SAVE_FACTORS 1
 #define COMBA_REUSE_FACTORS 2
+
+/*
+ * Comba-iplr variant (table of state transitions for the Comba variants):
+ * the transition alpha_t (I - 2 btilde_t k_t k_t^T) instead of
+ * (alpha_t I - btilde_t k_t k_t^T), i.e. every formula above with the
+ * feedback strength b beta_t replaced by 2 alpha_t b beta_t (gradients
+ * included: dalpha gains the term through that factor).  A flag bit of
+ * comba_chunk_fwd, comba_chunk_bwd (a backward that reuses saved factors must
+ * use the variant of the forward that saved them) and comba_recurrent_step.
+ */
+#define COMBA_IPLR 4
 
 /*
  * Bytes of device workspace needed by comba_chunk_fwd (backward = 0) or
@@ -166,12 +177,14 @@ comba_status_t comba_chunk_bwd(const comba_shape_t *shape,
  *   q, k [Bd,H,dk], v [Bd,H,dv], o [Bd,H,dv] (storage type `dtype`);
  *   alpha, beta fp32 [Bd,H]; b fp32 [H] or NULL; d fp32 [H];
  *   state fp32 [Bd,H,dk,dv], updated in place.
+ *   flags: 0 or COMBA_IPLR (b beta replaced by 2 alpha b beta); other bits are
+ *   COMBA_ERR_INVALID_ARG.
  */
 comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t dtype,
                                     const void *q, const void *k, const void *v,
                                     const float *alpha, const float *beta,
                                     const float *b, const float *d,
-                                    float *state, void *o, void *stream);
+                                    float *state, void *o, int flags, void *stream);
 
 /*
  * Forward without a caller workspace, for callers that may not allocate

@@ -21,7 +21,7 @@ _lib = None
 _lock = threading.Lock()
 
 COMBA_F32, COMBA_BF16 = 0, 1
-COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS = 1, 2
+COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS, COMBA_IPLR = 1, 2, 4
 _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "workspace missing or too small",
            4: "CUDA error", 5: "device-side wait timed out"}
 
@@ -62,7 +62,7 @@ def lib():
         L.comba_chunk_fwd.restype = I
         L.comba_chunk_bwd.argtypes = [SP] + [P] * 10 + [P] * 8 + [P, Z, P]
         L.comba_chunk_bwd.restype = I
-        L.comba_recurrent_step.argtypes = [I, I, I, I, I] + [P] * 9 + [P]
+        L.comba_recurrent_step.argtypes = [I, I, I, I, I] + [P] * 9 + [I, P]
         L.comba_recurrent_step.restype = I
         L.comba_status_string.argtypes = [I]
         L.comba_status_string.restype = ctypes.c_char_p
@@ -167,14 +167,17 @@ def _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens):
 
 
 def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, output_final_state=False,
-                    o=None, hT=None, workspace=None, stream=None, stage_events=None, save_factors=False):
+                    o=None, hT=None, workspace=None, stream=None, stage_events=None, save_factors=False,
+                    iplr=False):
     """Chunk-parallel forward.  Returns ``(o, hT)`` (``hT`` is None unless requested).
 
     ``save_factors=True`` keeps the backward's chunk factors in ``workspace`` (which must
     then be sized for the backward) so that ``comba_chunk_bwd(..., reuse_factors=True)``
-    with the same workspace skips recomputing them."""
+    with the same workspace skips recomputing them.  ``iplr=True``: the Comba-iplr
+    transition alpha (I - 2 btilde k k^T)."""
     N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
-    shape = make_shape(q, v, cu_seqlens, stage_events, COMBA_SAVE_FACTORS if save_factors else 0)
+    shape = make_shape(q, v, cu_seqlens, stage_events,
+                       (COMBA_SAVE_FACTORS if save_factors else 0) | (COMBA_IPLR if iplr else 0))
     L = lib()
     nbytes = L.comba_workspace_size(ctypes.byref(shape), 1 if save_factors else 0)
     if nbytes == 0:
@@ -193,7 +196,8 @@ def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, o
 
 
 def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_seqlens=None, want_dh0=True,
-                    want_db=True, out=None, workspace=None, stream=None, stage_events=None, reuse_factors=False):
+                    want_db=True, out=None, workspace=None, stream=None, stage_events=None, reuse_factors=False,
+                    iplr=False):
     """Chunk-parallel backward.  Returns a dict with dq, dk, dv, dalpha, dbeta, dd, db, dh0.
 
     ``reuse_factors=True`` requires ``workspace`` to hold the factors of a
@@ -203,7 +207,8 @@ def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_s
     _check("dhT", dhT, torch.float32, (N, H, dk, dv), q.device)
     if reuse_factors and workspace is None:
         raise ValueError("reuse_factors=True needs the workspace of the saving forward call")
-    shape = make_shape(q, v, cu_seqlens, stage_events, COMBA_REUSE_FACTORS if reuse_factors else 0)
+    shape = make_shape(q, v, cu_seqlens, stage_events,
+                       (COMBA_REUSE_FACTORS if reuse_factors else 0) | (COMBA_IPLR if iplr else 0))
     L = lib()
     nbytes = L.comba_workspace_size(ctypes.byref(shape), 1)
     if nbytes == 0:
@@ -229,7 +234,7 @@ def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_s
     return g
 
 
-def comba_recurrent_step(q, k, v, alpha, beta, d, state, b=None, o=None, stream=None):
+def comba_recurrent_step(q, k, v, alpha, beta, d, state, b=None, o=None, stream=None, iplr=False):
     """One decode token; ``state`` [Bd,H,dk,dv] fp32 is updated in place.  Returns ``o``."""
     Bd, H, dk = q.shape
     dv = v.shape[-1]
@@ -245,7 +250,8 @@ def comba_recurrent_step(q, k, v, alpha, beta, d, state, b=None, o=None, stream=
     if o is None:
         o = torch.empty_like(v)
     st = lib().comba_recurrent_step(Bd, H, dk, dv, _dtype_code(q), _ptr(q), _ptr(k), _ptr(v), _ptr(alpha),
-                                    _ptr(beta), _ptr(b), _ptr(d), _ptr(state), _ptr(o), _stream(stream))
+                                    _ptr(beta), _ptr(b), _ptr(d), _ptr(state), _ptr(o), COMBA_IPLR if iplr else 0,
+                                    _stream(stream))
     if st != 0:
         raise CombaError("comba_recurrent_step", st)
     return o

@@ -95,6 +95,7 @@ void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* 
     p.Ttot = (long long)s->B * s->T;
     p.cu = s->cu_seqlens;
     p.slots = L.slots;
+    p.iplr = (s->flags & COMBA_IPLR) != 0;
     p.ev = reinterpret_cast<cudaEvent_t*>(s->stage_events);
     p.nev = s->stage_events ? s->num_stage_events : 0;
     p.err = reinterpret_cast<int*>(w + L.err);
@@ -155,7 +156,7 @@ comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const 
     const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
     comba_status_t st = plan(shape, save ? 1 : 0, &L);
     if (st != COMBA_OK) return st;
-    if (shape->flags & ~COMBA_SAVE_FACTORS) return COMBA_ERR_INVALID_ARG;
+    if (shape->flags & ~(COMBA_SAVE_FACTORS | COMBA_IPLR)) return COMBA_ERR_INVALID_ARG;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(o);
     COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
@@ -182,7 +183,7 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     Layout L;
     comba_status_t st = plan(shape, 1, &L);
     if (st != COMBA_OK) return st;
-    if (shape->flags & ~COMBA_REUSE_FACTORS) return COMBA_ERR_INVALID_ARG;
+    if (shape->flags & ~(COMBA_REUSE_FACTORS | COMBA_IPLR)) return COMBA_ERR_INVALID_ARG;
     const bool reuse = (shape->flags & COMBA_REUSE_FACTORS) != 0;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(dO);
@@ -217,8 +218,10 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
 
 comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t dtype, const void* q,
                                     const void* k, const void* v, const float* alpha, const float* beta,
-                                    const float* b, const float* d, float* state, void* o, void* stream) {
+                                    const float* b, const float* d, float* state, void* o, int flags,
+                                    void* stream) {
     if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
+    if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
     if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
     if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128)) return COMBA_ERR_UNSUPPORTED;
     if ((long long)Bd * H * (dv / 32) >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
@@ -226,7 +229,7 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
     COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
     COMBA_OPTIONAL(b);
     if (comba::launch_recurrent_step(Bd, H, dk, dv, dtype == COMBA_BF16, q, k, v, alpha, beta, b, d, state, o,
-                                     static_cast<cudaStream_t>(stream)) != cudaSuccess)
+                                     (flags & COMBA_IPLR) != 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
         return COMBA_ERR_CUDA;
     return COMBA_OK;
 }

@@ -179,7 +179,8 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     if (tid < 64) {
         const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
         sBe[tid] = be;
-        sBt[tid] = (p.b ? p.b[h] : 1.f) * be;
+        const float al = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
+        sBt[tid] = (p.b ? p.b[h] : 1.f) * be * feedback_scale(p.iplr, al);
     }
     cp_async_wait<0>();
     __syncthreads();

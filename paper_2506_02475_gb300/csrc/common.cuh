@@ -21,6 +21,10 @@ typedef __nv_bfloat16 bf16;
 
 constexpr int kChunk = 64;  // chunk length C
 
+// Feedback strength btilde_t relative to b beta_t: 1 (SPLR), or 2 alpha_t for the
+// Comba-iplr transition alpha_t (I - 2 btilde_t k_t k_t^T).
+__host__ __device__ __forceinline__ float feedback_scale(int iplr, float alpha) { return iplr ? 2.f * alpha : 1.f; }
+
 // ------------------------------------------------------------------ scalars
 
 __device__ __forceinline__ float to_f(float x) { return x; }

@@ -15,7 +15,7 @@ __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, co
                                               const T* __restrict__ v, const float* __restrict__ alpha,
                                               const float* __restrict__ beta, const float* __restrict__ b,
                                               const float* __restrict__ d, float* __restrict__ state,
-                                              T* __restrict__ o) {
+                                              T* __restrict__ o, int iplr) {
     constexpr int NT = DV / 32;   // column tiles per (row, head)
     constexpr int RPT = DK / 16;  // state rows per thread
     const int tile = blockIdx.x % NT;
@@ -73,7 +73,7 @@ __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, co
     if (tid < 32) {
         const float xs = rx[0][tid] + rx[1][tid] + rx[2][tid] + rx[3][tid];
         const float ys = ry[0][tid] + ry[1][tid] + ry[2][tid] + ry[3][tid];
-        const float e = be * to_f(v[u * DV + col0 + tid]) - (b ? b[h] : 1.f) * be * xs;
+        const float e = be * to_f(v[u * DV + col0 + tid]) - (b ? b[h] : 1.f) * be * feedback_scale(iplr, a) * xs;
         se[tid] = e;
         o[u * DV + col0 + tid] = from_f<T>(a * ys + e * skq);
     }
@@ -94,18 +94,18 @@ __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, co
 template <typename T, int DK, int DV>
 static cudaError_t run_step(int Bd, int H, const void* q, const void* k, const void* v, const float* alpha,
                             const float* beta, const float* b, const float* d, float* state, void* o,
-                            cudaStream_t s) {
+                            bool iplr, cudaStream_t s) {
     const long long blocks = (long long)Bd * H * (DV / 32);
     k_step<T, DK, DV><<<(unsigned)blocks, 128, 0, s>>>(H, (const T*)q, (const T*)k, (const T*)v, alpha, beta, b, d,
-                                                       state, (T*)o);
+                                                       state, (T*)o, iplr ? 1 : 0);
     return cudaGetLastError();
 }
 
 cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, const void* q, const void* k,
                                   const void* v, const float* alpha, const float* beta, const float* b,
-                                  const float* d, float* state, void* o, cudaStream_t s) {
+                                  const float* d, float* state, void* o, bool iplr, cudaStream_t s) {
 #define COMBA_STEP(T, DK, DV) \
-    if (dk == DK && dv == DV) return run_step<T, DK, DV>(Bd, H, q, k, v, alpha, beta, b, d, state, o, s);
+    if (dk == DK && dv == DV) return run_step<T, DK, DV>(Bd, H, q, k, v, alpha, beta, b, d, state, o, iplr, s);
     if (is_bf16) {
         COMBA_STEP(bf16, 128, 128) COMBA_STEP(bf16, 128, 64) COMBA_STEP(bf16, 64, 128) COMBA_STEP(bf16, 64, 64)
     } else {

@@ -255,11 +255,12 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             sGm1[tid] = gm1;
             const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
             sBe[tid] = be;
-            sBt[tid] = bh * be;
+            const float fsc = feedback_scale(p.iplr, tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f);
+            sBt[tid] = bh * be * fsc;
             sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
             const float em1 = tid > 0 ? __expf(gm1) : 1.f;
             sEm1[tid] = em1;
-            sWs[tid] = bh * be * em1;
+            sWs[tid] = bh * be * fsc * em1;
         }
         cp_async_wait<0>();
         __syncthreads();
@@ -592,9 +593,11 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             float dbt = 0.f, db_c = 0.f, dd_c = 0.f;
             if (r < L) {
                 dbt = rsum(4, r) + sEm1[r] * rsum(7, r);
-                p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r];
-                p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * dbt;
-                db_c = sBe[r] * dbt;
+                // dbt is the gradient of btilde_r = b beta_r f_r (f_r = 1, or 2 alpha_r for iplr)
+                const float fr = feedback_scale(p.iplr, sAl[r]);
+                p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r] + (p.iplr ? 2.f * bh * sBe[r] * dbt : 0.f);
+                p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * fr * dbt;
+                db_c = sBe[r] * fr * dbt;
                 dd_c = -rsum(6, r);
             }
             // fixed-order reduction of the two per-chunk partials over 64 rows

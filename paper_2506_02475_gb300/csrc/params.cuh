@@ -22,6 +22,7 @@ struct ChunkParams {
     const float* alpha;
     const float* beta;
     const float* b;          // [H] or null (b = 1)
+    int iplr;                // Comba-iplr: feedback strength 2 alpha b beta instead of b beta
     const float* d;          // [H]
     const float* h0;         // [N,H,dk,dv] or null
     void* o;
@@ -108,6 +109,6 @@ inline bool use_tc_path(bool is_bf16, int dk, int dv) { return is_bf16 && dk == 
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);
 cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, const void* q, const void* k,
                                   const void* v, const float* alpha, const float* beta, const float* b,
-                                  const float* d, float* state, void* o, cudaStream_t s);
+                                  const float* d, float* state, void* o, bool iplr, cudaStream_t s);
 
 }  // namespace comba

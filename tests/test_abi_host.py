@@ -106,6 +106,8 @@ def test_forward_argument_validation(L):
     sv = shape(flags=1)
     assert fwd(L, sv, work=FAKE, nbytes=ws(L, shape(), 0)) == WORKSPACE
     assert fwd(L, shape(flags=2)) == INVALID            # reuse is a backward flag
+    assert fwd(L, shape(flags=8)) == INVALID            # unknown bit
+    assert fwd(L, shape(flags=4), q=None) == INVALID    # iplr is a valid forward flag; q still required
 
 
 def test_backward_argument_validation(L):
@@ -126,15 +128,20 @@ def test_backward_argument_validation(L):
     assert call(work=FAKE, nbytes=ws(L, s, 1) - 256) == WORKSPACE
     s.flags = 1                                          # save is a forward flag
     assert call() == INVALID
+    s.flags = 4 | 2                                      # iplr + reuse: valid flags, workspace still missing
+    assert call() == WORKSPACE
     s.flags = 0
 
 
 def test_recurrent_step_validation(L):
-    def call(Bd=4, H=2, dk=128, dv=128, dtype=1, **over):
+    def call(Bd=4, H=2, dk=128, dv=128, dtype=1, flags=0, **over):
         a = dict(q=FAKE, k=FAKE, v=FAKE, alpha=FAKE, beta=FAKE, b=None, d=FAKE, state=FAKE, o=FAKE)
         a.update(over)
         return L.comba_recurrent_step(Bd, H, dk, dv, dtype, a["q"], a["k"], a["v"], a["alpha"], a["beta"], a["b"],
-                                      a["d"], a["state"], a["o"], None)
+                                      a["d"], a["state"], a["o"], flags, None)
+
+    assert call(flags=8) == INVALID                  # only COMBA_IPLR is a step flag
+    assert call(flags=1) == INVALID
 
     assert call(Bd=0) == INVALID
     assert call(dk=32) == UNSUPPORTED

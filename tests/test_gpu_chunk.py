@@ -200,3 +200,39 @@ def test_backward_reusing_saved_forward_factors(dtype, d, lens):
         assert rel(g[key], r[key]) <= tol(w.dtype), key
     for key, e in param_grad_errors(g, r, w.k, w.v, w.beta, w.b).items():
         assert e <= tol(w.dtype), key
+
+
+@pytest.mark.parametrize("dtype,d,lens", [("bf16", 128, [130, 0, 257, 64]), ("bf16", 64, None), ("f32", 64, [70, 5, 133])])
+def test_iplr_variant_forward_backward(dtype, d, lens):
+    """Comba-iplr (transition alpha (I - 2 btilde k k^T)) through the same kernels, forward and backward,
+    including the saved-factor step, against the oracle's iplr variant."""
+    from paper_2506_02475_gb300 import comba_workspace_size
+    w = inputs.make("custom", B=2, T=200, H=3, dk=d, dv=d, dtype=dtype, with_b=True, with_h0=True, with_grads=True,
+                    lengths=lens, seed_offset=61)
+    t = to_dev(w)
+    ws = torch.empty(comba_workspace_size(t["q"], t["v"], t["cu_seqlens"], backward=True), dtype=torch.uint8,
+                     device="cuda")
+    o, hT = comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"],
+                            cu_seqlens=t["cu_seqlens"], output_final_state=True, workspace=ws, save_factors=True,
+                            iplr=True)
+    g = comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
+                        dhT=t["dhT"], cu_seqlens=t["cu_seqlens"], workspace=ws, reuse_factors=True, iplr=True)
+    g2 = comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
+                         dhT=t["dhT"], cu_seqlens=t["cu_seqlens"], iplr=True)
+    torch.cuda.synchronize()
+    ro, rhT = oracle.fwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0, cu_seqlens=w.cu_seqlens, variant="iplr")
+    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens,
+                   variant="iplr")
+    assert rel(np64(o), ro) <= tol(dtype)
+    assert rel(np64(hT), rhT) <= tol(dtype)
+    gn = {key: np64(val) for key, val in g.items()}
+    for key in GRADS:
+        assert np.array_equal(gn[key], np64(g2[key])), key          # reuse == recompute, bitwise
+        assert rel(gn[key], r[key]) <= tol(dtype), (key, rel(gn[key], r[key]))
+    # db, dd on their summation scale: with btilde' = 2 alpha b beta, (beta dbeta - v.dv) / b is still
+    # the per-token contribution beta dbtilde' (2 alpha)
+    for key, e in param_grad_errors(gn, r, w.k, w.v, w.beta, w.b).items():
+        assert e <= tol(dtype), (key, e)
+    # and it is not the SPLR result
+    ro_s, _ = oracle.fwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0, cu_seqlens=w.cu_seqlens)
+    assert rel(np64(o), ro_s) > 2 * tol(dtype)

@@ -57,3 +57,22 @@ def test_decode_workload_1024_steps_sampled_rows():
     torch.cuda.synchronize()
     assert worst_o <= TOL_BF16
     assert rel(np64(st_gpu[rows]), st_ref) <= TOL_BF16
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_decode_steps_iplr(dtype):
+    """Comba-iplr decode (feedback strength 2 alpha b beta) against the oracle's iplr step."""
+    Bd, H, dk, dv, steps = 6, 2, 128, 128, 5
+    state = inputs.decode_state(Bd, H, dk, dv, seed_offset=7)
+    b = np.random.default_rng(2).uniform(0, 1, H).astype(np.float32)
+    st_gpu = _f32(state)
+    st_ref = state.astype(np.float64)
+    for s in range(steps):
+        q, k, v, a, be, d = inputs.decode_tokens(s, Bd, H, dk, dv, dtype)
+        o = comba_recurrent_step(_tok(q, dtype), _tok(k, dtype), _tok(v, dtype), _f32(a), _f32(be), _f32(d), st_gpu,
+                                 b=_f32(b), iplr=True)
+        ro, st_ref = oracle.step(q, k, v, a, be, b, d, st_ref, variant="iplr")
+        torch.cuda.synchronize()
+        tl = TOL_BF16 if dtype == "bf16" else TOL_F32
+        assert rel(np64(o), ro) <= tl
+        assert rel(np64(st_gpu), st_ref) <= tl
