@@ -91,14 +91,14 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 113_184, ("chunk_tc.cu", "common.cuh", "params.cuh"), "d1fe44378000f358"),
-    "scan_fwd": ("k_scan_tc<128,128,0>", 83_099, ("scan.cu", "common.cuh", "params.cuh"), "e883c9cfa97a4cb6"),
-    "output": ("k_output_tc", 120_889, ("chunk_tc.cu", "common.cuh", "params.cuh"), "d1fe44378000f358"),
-    "bwd_prep": ("k_bwd_prep_tc", 81_431, ("chunk_tc.cu", "common.cuh", "params.cuh"), "d1fe44378000f358"),
-    "scan_bwd": ("k_scan_tc<128,128,1>", 84_557, ("scan.cu", "common.cuh", "params.cuh"), "e883c9cfa97a4cb6"),
-    "bwd_local": ("k_bwd_local", 195_907, ("chunk_bwd.cu", "common.cuh", "params.cuh"), "240d6db52b9f6c5a"),
+    "prep": ("k_prep_tc", 110_757, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "8037a0f379eeca70"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_659, ('scan.cu', 'common.cuh', 'params.cuh'), "078fa92632262989"),
+    "output": ("k_output_tc", 118_728, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "8037a0f379eeca70"),
+    "bwd_prep": ("k_bwd_prep_tc", 82_599, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "8037a0f379eeca70"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_522, ('scan.cu', 'common.cuh', 'params.cuh'), "078fa92632262989"),
+    "bwd_local": ("k_bwd_local_tc", 194_416, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "7bdbfc4ffe1922cb"),
 }
-DECODE_TRAFFIC = (481_764_352, ("decode.cu",), "00e53ed850cc9c96")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (482_097_920, ('decode.cu', 'common.cuh', 'params.cuh'), "0daad7feb5fb12b6")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
