@@ -27,8 +27,9 @@ namespace comba {
 namespace tc {
 
 struct LocalTcSmem {
-    static constexpr uint32_t OQK = 0;             // [128][128]: rows 0-63 Q -> Q~, rows 64-127 K; later dq, dk staging
-    static constexpr uint32_t OV = OQK + 32768;    // V [64][128]
+    static constexpr uint32_t OQK = 0;             // two [128][128] tiles (consecutive units alternate): rows 0-63
+                                                   // Q -> Q~, rows 64-127 K; later dq, dk staging
+    static constexpr uint32_t OV = OQK + 2 * 32768;  // V [64][128]
     static constexpr uint32_t ODO = OV + 16384;    // dO [64][128]
     static constexpr uint32_t OE = ODO + 16384;    // E [64][128]; later dv staging
     static constexpr uint32_t OH = OE + 16384;     // H^T [128][128]; later dPhat, dM, Y, dG [64][64]
@@ -130,8 +131,9 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 // Persistent: CTA b handles units b, b + G, b + 2G, ... (G = gridDim.x, about one CTA per SM).
 // While unit u computes, the tiles of unit u + G stream into buffers as soon as their last
 // reader in unit u has finished (dH'^T after R1, H^T after R3, E after the dv copy, dO, V,
-// M after R7), so the loads of consecutive units overlap the tensor-core and epilogue work
-// instead of every SM loading at the same moment; only Q and K load at the top of a unit.
+// M after R7; Q and K into the second of two alternating tiles at the start of the unit; the
+// per-row scalars into registers), so the loads of consecutive units overlap the tensor-core
+// and epilogue work instead of every SM loading at the same moment.
 __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long long units) {
     using S = LocalTcSmem;
     extern __shared__ uint8_t smem_raw[];
@@ -140,8 +142,6 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wr = warp & 3, wc = warp >> 2, m0 = 16 * wr;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sQK = sm + S::OQK;
-    uint8_t* sKt = sQK + 64 * 128;   // K: rows 64-127 of the 128-row tile
     uint8_t* sV = sm + S::OV;
     uint8_t* sdO = sm + S::ODO;
     uint8_t* sE = sm + S::OE;
@@ -167,20 +167,32 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
     float* rowp = sG + 512;           // [kind][column half][row]
     float* colp = rowp + 8 * 2 * 64;  // [kind][row block][column]
     float* red = colp + 2 * 4 * 64;
-    const uint32_t uQK = smem_u32(sQK), uK = smem_u32(sKt), uV = smem_u32(sV), udO = smem_u32(sdO),
+    const uint32_t uV = smem_u32(sV), udO = smem_u32(sdO),
                    uE = smem_u32(sE), uH = smem_u32(sHt), udH = smem_u32(sdHt), uM = smem_u32(sM),
                    uP = smem_u32(sP), udE = smem_u32(sdE), udW = smem_u32(sdW), udPh = smem_u32(sdPh),
                    udM = smem_u32(sdM), uY = smem_u32(sY), udG = smem_u32(sdG);
 
-    auto load_qk = [&](const UnitRef& x) {
+    auto load_qk = [&](uint8_t* dst, const UnitRef& x) {
         const bf16* qg = (const bf16*)p.q + (x.t0 * p.H + x.h) * D;
         const bf16* kg = (const bf16*)p.k + (x.t0 * p.H + x.h) * D;
         for (int e = tid; e < 128 * 16; e += 256) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < x.L;
             const bf16* src = (r < 64 ? qg : kg) + (long long)rr * p.H * D + ch * 8;
-            cp_async16(sQK + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
+            cp_async16(dst + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
         }
+    };
+    // per-row scalars of a unit (rows tid < 64): log-decay G_r, G_{r-1}, beta, alpha
+    struct RowIn { float g, gm1, be, al; };
+    auto load_rows = [&](const UnitRef& x) {
+        RowIn r{0.f, 0.f, 0.f, 1.f};
+        if (tid < 64) {
+            r.g = p.Gb[x.idx * 64 + tid];
+            r.gm1 = tid > 0 ? p.Gb[x.idx * 64 + tid - 1] : 0.f;
+            r.be = tid < x.L ? p.beta[(x.t0 + tid) * p.H + x.h] : 0.f;
+            r.al = tid < x.L ? p.alpha[(x.t0 + tid) * p.H + x.h] : 1.f;
+        }
+        return r;
     };
     auto load_tok = [&](uint8_t* dst, const void* base, const UnitRef& x) {
         load_sw(dst, 64, D, (const bf16*)base + (x.t0 * p.H + x.h) * D, (long long)p.H * D, x.L, tid, 256);
@@ -221,49 +233,61 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
     };
 
     bool ok = true;
-    bool pre = false;   // this unit's dH'^T, H^T, E, dO, V, M were requested by the previous unit
-    for (long long u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        const UnitRef cur = unit_ref(p, u);
+    bool pre = false;   // this unit's tiles and row scalars were requested by the previous unit
+    long long u = blockIdx.x;
+    UnitRef cur = u < units ? unit_ref(p, u) : UnitRef{0, 0, 0, 0};
+    RowIn rin{0.f, 0.f, 0.f, 1.f};
+    for (int it = 0; u < units && ok; ++it) {
+        const long long un = u + gridDim.x;
+        UnitRef nxt{0, 0, 0, 0};
+        if (un < units) nxt = unit_ref(p, un);   // used from the first prefetch point on
+        uint8_t* sQK = sm + S::OQK + (it & 1) * 32768;
+        uint8_t* sQKn = sm + S::OQK + ((it + 1) & 1) * 32768;   // the next unit's Q/K tile
         if (cur.L <= 0) {
             if (tid == 0) { p.part[u * 2] = 0.f; p.part[u * 2 + 1] = 0.f; }
             pre = false;
+            u = un;
+            cur = nxt;
             continue;
         }
-        const long long un = u + gridDim.x;
-        UnitRef nxt{0, 0, 0, 0};
-        if (un < units) nxt = unit_ref(p, un);
+        uint8_t* sKt = sQK + 64 * 128;   // K: rows 64-127 of the 128-row tile
+        const uint32_t uQK = smem_u32(sQK), uK = smem_u32(sKt);
         const bool has_next = nxt.L > 0;
         const int L = cur.L, h = cur.h;
         const long long t0 = cur.t0, idx = cur.idx;
 
-        load_qk(cur);
         if (!pre) {
+            load_qk(sQK, cur);
             load_tok(sdO, p.dO, cur);
             load_E(cur);
             load_H(cur);
             load_dH(cur);
             load_tok(sV, p.v, cur);
             load_M(cur);
+            cp_async_commit();
+            rin = load_rows(cur);
         }
-        cp_async_commit();
         const float bh = p.b ? p.b[h] : 1.f;
         const float dh = p.d[h];
         if (tid < 64) {
-            const float g = p.Gb[idx * 64 + tid];
-            const float gm1 = tid > 0 ? p.Gb[idx * 64 + tid - 1] : 0.f;
-            sG[tid] = g;
-            sGm1[tid] = gm1;
-            const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
-            sBe[tid] = be;
-            const float fsc = feedback_scale(p.iplr, tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f);
-            sBt[tid] = bh * be * fsc;
-            sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
-            const float em1 = tid > 0 ? __expf(gm1) : 1.f;
+            sG[tid] = rin.g;
+            sGm1[tid] = rin.gm1;
+            sBe[tid] = rin.be;
+            const float fsc = feedback_scale(p.iplr, rin.al);
+            sBt[tid] = bh * rin.be * fsc;
+            sAl[tid] = rin.al;
+            const float em1 = tid > 0 ? __expf(rin.gm1) : 1.f;
             sEm1[tid] = em1;
-            sWs[tid] = bh * be * fsc * em1;
+            sWs[tid] = bh * rin.be * fsc * em1;
         }
         cp_async_wait<0>();
         __syncthreads();
+        // the next unit's Q/K tile streams in during this unit (its buffer was last read by the
+        // previous unit's staging copies, finished before this unit began)
+        if (has_next) {
+            load_qk(sQKn, nxt);
+            cp_async_commit();
+        }
         // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
         for (int e = tid; e < 64 * 16; e += 256) {
             const int r = e >> 4, ch = e & 15;
@@ -502,6 +526,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             load_tok(sV, p.v, nxt);
             load_M(nxt);
             cp_async_commit();
+            rin = load_rows(nxt);
         }
         if (ok) {
             float t7[8][4], s0, s1;
@@ -617,8 +642,10 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                 flag_error(p);
             }
         }
-        __syncthreads();   // the next unit's Q/K copies overwrite the staging tile read above
+        __syncthreads();   // the staging tile read above takes the Q/K copies of the unit after next
         pre = has_next;
+        u = un;
+        cur = nxt;
     }
     cp_async_wait<0>();   // no copy is still writing shared memory at exit
     tc_fence_before();
