@@ -345,6 +345,13 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                     st_pair(sP, 64, r, c, v0, v1);
                 }
             tmem_frag4(tq + 64 + nl0, dP);
+        }
+        publish_smem();
+
+        // ---------------- R2: dE = Kbar dH' + P^T dO, into the columns of S and dP (already read);
+        // the rest of the R1 epilogue runs while it computes
+        if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
+        if (ok) {
             // dQ~ part Diag(gamma) dO H^T; its row dot with Q~ is the log-decay gradient of the Q~ H term
             tmem_frag8(tq + 128 + nk0, acc_dq);
 #pragma unroll
@@ -363,10 +370,6 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
 #pragma unroll
             for (int t = 0; t < 8; ++t) { de[t][0] *= sKa; de[t][1] *= sKa; de[t][2] *= sKb; de[t][3] *= sKb; }
         }
-        publish_smem();
-
-        // ---------------- R2: dE = Kbar dH' + P^T dO
-        if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
         ok = ok && ms.finish(tid);
         if (ok) {
             float t2[8][4];
@@ -389,8 +392,8 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         ok = ok && ms.finish(tid);
         if (ok && has_next) { load_H(nxt); cp_async_commit(); }
         float dMa[4][4], gr[4][4];
+        float t3[8][4];
         if (ok) {
-            float t3[8][4];
             // dW = -dE H^T (over the dead dO tile)
             tmem_frag8(tq + 0 + nk0, t3);
 #pragma unroll
@@ -398,6 +401,13 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
 #pragma unroll
                 for (int i = 0; i < 4; ++i) t3[t][i] = -t3[t][i];
             frag_store_sw<8>(sdW, 64, m0, nk0, t3);
+        }
+        publish_smem();
+
+        // ---------------- R4: dM = dE V^T Diag(beta) + dW K^T Diag(btilde gamma_{-1}), into the dW
+        // columns (already read); the rest of the R3 epilogue and the dv store run meanwhile
+        if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 0, udW, 64, uK, 128, 64, D, false);
+        if (ok) {
             tmem_frag4(tq + 128 + nl0, dMa);
 #pragma unroll
             for (int t = 0; t < 4; ++t)
@@ -414,10 +424,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             frag_stage<8>(stV, m0, nk0, t3);
             tmem_frag4(tq + 320 + nl0, gr);
         }
-        publish_smem();
-
-        // ---------------- R4: dM = dE V^T Diag(beta) + dW K^T Diag(btilde gamma_{-1}); dv leaves meanwhile
-        if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 0, udW, 64, uK, 128, 64, D, false);
+        __syncthreads();
         if (ok) copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, (long long)p.H * D, stV, L, tid);
         ok = ok && ms.finish(tid);
         if (ok && has_next) { load_E(nxt); cp_async_commit(); }
