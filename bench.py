@@ -539,6 +539,89 @@ def workload_desc(w):
             f"chunk_bwd(all grads, reuses factors)")
 
 
+# ------------------------------------------------------------ gated step
+
+def run_gated(args, world, rank, local):
+    """The training step with the gate and normalisation prologue (raw q, k, gate pre-activations):
+    comba_chunk_fwd_gated (saving factors) + comba_chunk_bwd_gated (reusing them), device-resident."""
+    import torch
+    dist = dist_init(world, local, "nccl")
+    torch.cuda.set_device(local)
+    from paper_2506_02475_gb300 import binding, comba_chunk_bwd_gated, comba_chunk_fwd_gated, inputs, shard
+    base = inputs.make(args.workload, with_grads=False)
+    lens = None if base.cu_seqlens is None else np.diff(base.cu_seqlens)
+    B = base.q.shape[0] if base.cu_seqlens is None else 1
+    T = base.q.shape[1] if base.cu_seqlens is None else int(base.tokens)
+    w = inputs.make_gated(B=B, T=T, H=base.H, dk=base.dk, dv=base.dv, dtype="bf16",
+                          seed_offset=shard.rank_seed_offset(rank), lengths=lens)
+    dev = torch.device("cuda", local)
+    tok = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev).to(torch.bfloat16)
+    f32 = lambda x: None if x is None else torch.from_numpy(np.ascontiguousarray(x, np.float32)).to(dev)
+    t = dict(q=tok(w.q), k=tok(w.k), v=tok(w.v), dO=tok(w.dO))
+    for key in ("g_alpha", "g_beta", "a", "c", "b_raw", "d", "h0", "dhT"):
+        t[key] = f32(getattr(w, key))
+    cu = None if w.cu_seqlens is None else torch.from_numpy(w.cu_seqlens.astype(np.int32)).to(dev)
+    iplr = args.variant == "iplr"
+    shape = binding.make_shape(t["q"], t["v"], cu, None, binding.COMBA_GATED)
+    ws = torch.empty(binding.lib().comba_workspace_size(binding.ctypes.byref(shape), 1), dtype=torch.uint8,
+                     device=dev)
+    o = torch.empty_like(t["v"])
+    N, H, dk, dv = base.num_seqs, base.H, base.dk, base.dv
+    hT = torch.empty((N, H, dk, dv), dtype=torch.float32, device=dev)
+    grads = {}
+    ev_f = [torch.cuda.Event(enable_timing=True) for _ in range(len(FWD_STAGES) + 1)]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(len(BWD_STAGES) + 1)]
+    for e in ev_f + ev_b:
+        e.record()
+    torch.cuda.synchronize()
+    hf, hb = [e.cuda_event for e in ev_f], [e.cuda_event for e in ev_b]
+    args_ = (t["q"], t["k"], t["v"], t["g_alpha"], t["g_beta"], t["a"], t["c"], t["b_raw"], t["d"])
+
+    def step():
+        comba_chunk_fwd_gated(*args_, h0=t["h0"], cu_seqlens=cu, o=o, hT=hT, workspace=ws, stage_events=hf,
+                              save_factors=True, iplr=iplr)
+        comba_chunk_bwd_gated(*args_, t["dO"], h0=t["h0"], dhT=t["dhT"], cu_seqlens=cu, out=grads, workspace=ws,
+                              stage_events=hb, reuse_factors=True, iplr=iplr)
+
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    for _ in range(max(3, args.warmup)):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = NvmlClockSampler(nvsmi_device_id())
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    total, kern = 0.0, 0.0
+    for _ in range(args.steps):
+        flush.zero_()
+        start.record()
+        step()
+        end.record()
+        end.synchronize()
+        total += start.elapsed_time(end)
+        kern += sum(ev_f[i].elapsed_time(ev_f[i + 1]) for i in range(len(FWD_STAGES)))
+        kern += sum(ev_b[i].elapsed_time(ev_b[i + 1]) for i in range(len(BWD_STAGES)))
+    clk = clocks.stop()
+    ms = shard.max_over_ranks(total / args.steps, dist, dev)
+    tokens = base.tokens
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC + ", with the gate and L2-norm prologue", "value": tokens * world / (ms / 1e3),
+            "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
+            "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (raw q, k with per-row scale in [0.5, 2]; gate pre-activations N(0,1))",
+            "config": {"workload": f"{args.workload} gated: " + workload_desc(base), "variant": args.variant,
+                       "l2": "flushed between timed steps (256 MiB write, outside the events)"},
+            "chunk_kernels_ms_per_step": kern / args.steps,
+            "prologue_epilogue_ms_per_step": ms - kern / args.steps,
+            "clocks": clk}), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
 # ------------------------------------------------------------------ decode
 
 def run_decode(args, world, rank, local):
@@ -639,6 +722,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="lm1p3b", choices=["lm1p3b", "lm340m", "varlen64k", "decode"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--gated", action="store_true",
+                    help="raw q, k and gate pre-activations through the gate and normalisation prologue")
     ap.add_argument("--variant", default="splr", choices=["splr", "iplr"],
                     help="state transition: Comba (alpha - btilde k k^T) or Comba-iplr alpha (I - 2 btilde k k^T)")
     ap.add_argument("--reference-tokens", type=int, default=512)
@@ -650,6 +735,8 @@ def main():
         return run_reference(args, world, rank, local)
     if args.workload == "decode":
         return run_decode(args, world, rank, local)
+    if args.gated:
+        return run_gated(args, world, rank, local)
     return run_ours(args, world, rank, local)
 
 

@@ -114,6 +114,50 @@ typedef struct {
 #define COMBA_IPLR 4
 
 /*
+ * Gate and normalisation prologue (section 3.1 gates; L2-normalised q and k of
+ * the neural-architecture section), for comba_chunk_fwd_gated and
+ * comba_chunk_bwd_gated, which take raw q, k and gate pre-activations:
+ *     q_hat = q / sqrt(|q|^2 + 1e-6)   (per token and head; likewise k)
+ *     alpha = exp(-a_h softplus(g_alpha + c_h)),  beta = sigmoid(g_beta),
+ *     b_h = sigmoid(b_raw_h)            (btilde = b beta)
+ * and run the recurrence above on (q_hat, k_hat, v, alpha, beta, b, d).  The
+ * shape passed to these calls and to comba_workspace_size must carry
+ * COMBA_GATED (the workspace then also holds the prologue's outputs).
+ */
+#define COMBA_GATED 8
+
+/*
+ * The gated forward: as comba_chunk_fwd, with raw q, k [B,T,H,dk] (storage type),
+ * gate pre-activations g_alpha, g_beta fp32 [B,T,H] and per-head fp32 a, c,
+ * b_raw, d [H] (all required) instead of alpha, beta, b.  shape->flags must
+ * contain COMBA_GATED and may add COMBA_SAVE_FACTORS (then the saved factors
+ * include the prologue's outputs) and COMBA_IPLR.
+ */
+comba_status_t comba_chunk_fwd_gated(const comba_shape_t *shape,
+                                     const void *q, const void *k, const void *v,
+                                     const float *g_alpha, const float *g_beta,
+                                     const float *a, const float *c, const float *b_raw, const float *d,
+                                     const float *h0, void *o, float *hT,
+                                     void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * The gated backward: gradients of L = <o,dO> + <hT,dhT> w.r.t. the raw inputs:
+ * dq, dk (storage type), dv, dg_alpha, dg_beta fp32 [B,T,H], da, dc, dd fp32
+ * [H], db_raw fp32 [H] or NULL, dh0 or NULL.  da, dc, db_raw and dd are sums over
+ * all tokens in a fixed order.  shape->flags must contain COMBA_GATED and may
+ * add COMBA_REUSE_FACTORS (after a gated forward with COMBA_SAVE_FACTORS on the
+ * same workspace) and COMBA_IPLR.
+ */
+comba_status_t comba_chunk_bwd_gated(const comba_shape_t *shape,
+                                     const void *q, const void *k, const void *v,
+                                     const float *g_alpha, const float *g_beta,
+                                     const float *a, const float *c, const float *b_raw, const float *d,
+                                     const float *h0, const void *dO, const float *dhT,
+                                     void *dq, void *dk, void *dv, float *dg_alpha, float *dg_beta,
+                                     float *da, float *dc, float *db_raw, float *dd, float *dh0,
+                                     void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * Bytes of device workspace needed by comba_chunk_fwd (backward = 0) or
  * comba_chunk_bwd (backward = 1) for this shape.  Returns 0 for an invalid
  * shape.  The bound covers any cu_seqlens with the given T and num_seqs.

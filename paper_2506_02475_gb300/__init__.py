@@ -8,7 +8,9 @@ CUDA kernels under ``csrc/``) and a thin ctypes binding with the same names.
 from .binding import (  # noqa: F401
     CombaError,
     comba_chunk_bwd,
+    comba_chunk_bwd_gated,
     comba_chunk_fwd,
+    comba_chunk_fwd_gated,
     comba_recurrent_step,
     comba_workspace_size,
     lib,

@@ -21,7 +21,7 @@ _lib = None
 _lock = threading.Lock()
 
 COMBA_F32, COMBA_BF16 = 0, 1
-COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS, COMBA_IPLR = 1, 2, 4
+COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS, COMBA_IPLR, COMBA_GATED = 1, 2, 4, 8
 _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "workspace missing or too small",
            4: "CUDA error", 5: "device-side wait timed out"}
 
@@ -64,6 +64,10 @@ def lib():
         L.comba_chunk_bwd.restype = I
         L.comba_recurrent_step.argtypes = [I, I, I, I, I] + [P] * 9 + [I, P]
         L.comba_recurrent_step.restype = I
+        L.comba_chunk_fwd_gated.argtypes = [SP] + [P] * 12 + [P, Z, P]
+        L.comba_chunk_fwd_gated.restype = I
+        L.comba_chunk_bwd_gated.argtypes = [SP] + [P] * 12 + [P] * 10 + [P, Z, P]
+        L.comba_chunk_bwd_gated.restype = I
         L.comba_status_string.argtypes = [I]
         L.comba_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -255,3 +259,73 @@ def comba_recurrent_step(q, k, v, alpha, beta, d, state, b=None, o=None, stream=
     if st != 0:
         raise CombaError("comba_recurrent_step", st)
     return o
+
+
+def _check_gated(q, k, v, g_alpha, g_beta, a, c, b_raw, d, h0, cu_seqlens):
+    N, H, dk, dv = _check_inputs(q, k, v, g_alpha, g_beta, None, d, h0, cu_seqlens)
+    for name, t in (("a", a), ("c", c), ("b_raw", b_raw)):
+        if t is None:
+            raise ValueError(f"{name} is required")
+        _check(name, t, torch.float32, (H,), q.device)
+    return N, H, dk, dv
+
+
+def comba_chunk_fwd_gated(q, k, v, g_alpha, g_beta, a, c, b_raw, d, h0=None, cu_seqlens=None,
+                          output_final_state=False, o=None, hT=None, workspace=None, stream=None, stage_events=None,
+                          save_factors=False, iplr=False):
+    """Forward with the gate and normalisation prologue: raw q, k; alpha = exp(-a softplus(g_alpha + c)),
+    beta = sigmoid(g_beta), b = sigmoid(b_raw); q, k L2-normalised in the kernels.  Returns ``(o, hT)``."""
+    N, H, dk, dv = _check_gated(q, k, v, g_alpha, g_beta, a, c, b_raw, d, h0, cu_seqlens)
+    flags = COMBA_GATED | (COMBA_SAVE_FACTORS if save_factors else 0) | (COMBA_IPLR if iplr else 0)
+    shape = make_shape(q, v, cu_seqlens, stage_events, flags)
+    L = lib()
+    nbytes = L.comba_workspace_size(ctypes.byref(shape), 1 if save_factors else 0)
+    if nbytes == 0:
+        raise CombaError("comba_workspace_size", 1)
+    ws = _workspace(nbytes, q.device, workspace)
+    if o is None:
+        o = torch.empty_like(v)
+    if hT is None and output_final_state:
+        hT = torch.empty((N, H, dk, dv), dtype=torch.float32, device=q.device)
+    st = L.comba_chunk_fwd_gated(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(g_alpha), _ptr(g_beta),
+                                 _ptr(a), _ptr(c), _ptr(b_raw), _ptr(d), _ptr(h0), _ptr(o), _ptr(hT), _ptr(ws),
+                                 ws.numel() * ws.element_size(), _stream(stream))
+    if st != 0:
+        raise CombaError("comba_chunk_fwd_gated", st)
+    return o, hT
+
+
+def comba_chunk_bwd_gated(q, k, v, g_alpha, g_beta, a, c, b_raw, d, dO, h0=None, dhT=None, cu_seqlens=None,
+                          want_dh0=True, out=None, workspace=None, stream=None, stage_events=None,
+                          reuse_factors=False, iplr=False):
+    """Gradients w.r.t. the raw inputs: dq, dk, dv, dg_alpha, dg_beta, da, dc, db_raw, dd, dh0."""
+    N, H, dk, dv = _check_gated(q, k, v, g_alpha, g_beta, a, c, b_raw, d, h0, cu_seqlens)
+    _check("dO", dO, q.dtype, v.shape, q.device)
+    _check("dhT", dhT, torch.float32, (N, H, dk, dv), q.device)
+    if reuse_factors and workspace is None:
+        raise ValueError("reuse_factors=True needs the workspace of the saving forward call")
+    flags = COMBA_GATED | (COMBA_REUSE_FACTORS if reuse_factors else 0) | (COMBA_IPLR if iplr else 0)
+    shape = make_shape(q, v, cu_seqlens, stage_events, flags)
+    L = lib()
+    nbytes = L.comba_workspace_size(ctypes.byref(shape), 1)
+    if nbytes == 0:
+        raise CombaError("comba_workspace_size", 1)
+    ws = _workspace(nbytes, q.device, workspace)
+    g = out if out is not None else {}
+    g.setdefault("dq", torch.empty_like(q))
+    g.setdefault("dk", torch.empty_like(k))
+    g.setdefault("dv", torch.empty_like(v))
+    g.setdefault("dg_alpha", torch.empty_like(g_alpha))
+    g.setdefault("dg_beta", torch.empty_like(g_beta))
+    for key in ("da", "dc", "db_raw", "dd"):
+        g.setdefault(key, torch.empty((H,), dtype=torch.float32, device=q.device))
+    if want_dh0:
+        g.setdefault("dh0", torch.empty((N, H, dk, dv), dtype=torch.float32, device=q.device))
+    st = L.comba_chunk_bwd_gated(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(g_alpha), _ptr(g_beta),
+                                 _ptr(a), _ptr(c), _ptr(b_raw), _ptr(d), _ptr(h0), _ptr(dO), _ptr(dhT),
+                                 _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]), _ptr(g["dg_alpha"]),
+                                 _ptr(g["dg_beta"]), _ptr(g["da"]), _ptr(g["dc"]), _ptr(g["db_raw"]), _ptr(g["dd"]),
+                                 _ptr(g.get("dh0")), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream))
+    if st != 0:
+        raise CombaError("comba_chunk_bwd_gated", st)
+    return g

@@ -16,7 +16,11 @@ size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct Layout {
-    size_t err, slot_info, seq_first, W, U, G, A, B, Hs, E, M, AT, C, dH, part, total;
+    size_t err, slot_info, seq_first, W, U, G, A, B, Hs, E, M, AT, C, dH, part;
+    // gate and normalisation prologue (COMBA_GATED): its outputs, and the backward's gradients
+    // w.r.t. them with the per-row contributions to da, dc
+    size_t qh, kh, ga, gb, bg, dqh, dkh, dal, dbe, dbi, dar, dcr, dpa, dpc;
+    size_t total;
     int slots;
 };
 
@@ -68,6 +72,26 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
         L.C = take(pairs * dv * dk * es);
         L.dH = take(pairs * dv * dk * es);
         L.part = take(pairs * 2 * sizeof(float));
+    }
+    if (s->flags & COMBA_GATED) {
+        const size_t rows = (size_t)ttot * s->H;
+        L.qh = take(rows * dk * es);
+        L.kh = take(rows * dk * es);
+        L.ga = take(rows * sizeof(float));
+        L.gb = take(rows * sizeof(float));
+        L.bg = take((size_t)s->H * sizeof(float));
+        if (backward) {
+            L.dqh = take(rows * dk * es);
+            L.dkh = take(rows * dk * es);
+            L.dal = take(rows * sizeof(float));
+            L.dbe = take(rows * sizeof(float));
+            L.dbi = take((size_t)s->H * sizeof(float));
+            L.dar = take(rows * sizeof(float));
+            L.dcr = take(rows * sizeof(float));
+            const size_t parts = (size_t)((ttot + 63) / 64) * s->H;   // token blocks of the per-head sums
+            L.dpa = take(parts * sizeof(float));
+            L.dpc = take(parts * sizeof(float));
+        }
     }
     L.total = o;
     L.slots = (int)slots;
@@ -148,6 +172,74 @@ size_t comba_workspace_size(const comba_shape_t* shape, int backward) {
     return L.total;
 }
 
+}  // extern "C"
+
+namespace {
+
+// Launch the forward on validated arguments (L from plan(); shape checks done).
+comba_status_t forward_run(const comba_shape_t* shape, const Layout& L, void* workspace, const void* q, const void* k,
+                           const void* v, const float* alpha, const float* beta, const float* b, const float* d,
+                           const float* h0, void* o, float* hT, bool save, cudaStream_t s) {
+    comba_status_t st;
+    if ((st = check_smem(shape, 0)) != COMBA_OK) return st;
+    ChunkParams p{};
+    fill_common(p, shape, L, workspace, save);
+    p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
+    p.o = o; p.hT = hT;
+    comba::mark(p, 0, s);
+    if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (comba::launch_fwd(p, shape->dtype == COMBA_BF16, save, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+    return COMBA_OK;
+}
+
+comba_status_t backward_run(const comba_shape_t* shape, const Layout& L, void* workspace, const void* q,
+                            const void* k, const void* v, const float* alpha, const float* beta, const float* b,
+                            const float* d, const float* h0, const void* dO, const float* dhT, void* dq, void* dk,
+                            void* dv, float* dalpha, float* dbeta, float* db, float* dd, float* dh0, bool reuse,
+                            cudaStream_t s) {
+    comba_status_t st;
+    if ((st = check_smem(shape, 1)) != COMBA_OK) return st;
+    ChunkParams p{};
+    fill_common(p, shape, L, workspace, true);
+    p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
+    p.dO = dO; p.dhT = dhT; p.dq = dq; p.dkk = dk; p.dvv = dv;
+    p.dalpha = dalpha; p.dbeta = dbeta; p.db = db; p.dd = dd; p.dh0 = dh0;
+    const bool bf = shape->dtype == COMBA_BF16;
+    comba::mark(p, 0, s);
+    if (reuse) {
+        for (int e = 1; e <= 4; ++e) comba::mark(p, e, s);
+    } else {
+        // recompute the forward factors and chunk states (no output, no final state)
+        ChunkParams f = p;
+        f.o = nullptr;
+        f.hT = nullptr;
+        if (comba::launch_chunk_map(f, s) != cudaSuccess) return COMBA_ERR_CUDA;
+        if (comba::launch_fwd(f, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
+    }
+    if (comba::launch_bwd(p, bf, s, 4) != cudaSuccess) return COMBA_ERR_CUDA;
+    return COMBA_OK;
+}
+
+comba::GateParams gate_params(const comba_shape_t* shape, const Layout& L, void* workspace, const void* q,
+                              const void* k, const float* g_alpha, const float* g_beta, const float* a,
+                              const float* c, const float* b_raw) {
+    char* w = static_cast<char*>(workspace);
+    comba::GateParams g{};
+    g.rows = (long long)shape->B * shape->T * shape->H;
+    g.H = shape->H;
+    g.eps = 1e-6f;
+    g.q = q; g.k = k; g.g_alpha = g_alpha; g.g_beta = g_beta; g.a = a; g.c = c; g.b_raw = b_raw;
+    g.qh = w + L.qh; g.kh = w + L.kh;
+    g.alpha = reinterpret_cast<float*>(w + L.ga);
+    g.beta = reinterpret_cast<float*>(w + L.gb);
+    g.bgate = reinterpret_cast<float*>(w + L.bg);
+    return g;
+}
+
+}  // namespace
+
+extern "C" {
+
 comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const void* k, const void* v,
                                const float* alpha, const float* beta, const float* b, const float* d,
                                const float* h0, void* o, float* hT, void* workspace, size_t workspace_bytes,
@@ -162,17 +254,8 @@ comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const 
     COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
     if (shape->stage_events && shape->num_stage_events < COMBA_FWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
-    if ((st = check_smem(shape, 0)) != COMBA_OK) return st;
-
-    ChunkParams p{};
-    fill_common(p, shape, L, workspace, save);
-    p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
-    p.o = o; p.hT = hT;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    comba::mark(p, 0, s);
-    if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
-    if (comba::launch_fwd(p, shape->dtype == COMBA_BF16, save, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
-    return COMBA_OK;
+    return forward_run(shape, L, workspace, q, k, v, alpha, beta, b, d, h0, o, hT, save,
+                       static_cast<cudaStream_t>(stream));
 }
 
 comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const void* k, const void* v,
@@ -184,7 +267,6 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     comba_status_t st = plan(shape, 1, &L);
     if (st != COMBA_OK) return st;
     if (shape->flags & ~(COMBA_REUSE_FACTORS | COMBA_IPLR)) return COMBA_ERR_INVALID_ARG;
-    const bool reuse = (shape->flags & COMBA_REUSE_FACTORS) != 0;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(dO);
     COMBA_REQUIRE(dq); COMBA_REQUIRE(dk); COMBA_REQUIRE(dv); COMBA_REQUIRE(dalpha); COMBA_REQUIRE(dbeta);
@@ -192,27 +274,70 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(dhT); COMBA_OPTIONAL(db); COMBA_OPTIONAL(dh0);
     if (shape->stage_events && shape->num_stage_events < COMBA_BWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
-    if ((st = check_smem(shape, 1)) != COMBA_OK) return st;
+    return backward_run(shape, L, workspace, q, k, v, alpha, beta, b, d, h0, dO, dhT, dq, dk, dv, dalpha, dbeta, db,
+                        dd, dh0, (shape->flags & COMBA_REUSE_FACTORS) != 0, static_cast<cudaStream_t>(stream));
+}
 
-    ChunkParams p{};
-    fill_common(p, shape, L, workspace, true);
-    p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
-    p.dO = dO; p.dhT = dhT; p.dq = dq; p.dkk = dk; p.dvv = dv;
-    p.dalpha = dalpha; p.dbeta = dbeta; p.db = db; p.dd = dd; p.dh0 = dh0;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+comba_status_t comba_chunk_fwd_gated(const comba_shape_t* shape, const void* q, const void* k, const void* v,
+                                     const float* g_alpha, const float* g_beta, const float* a, const float* c,
+                                     const float* b_raw, const float* d, const float* h0, void* o, float* hT,
+                                     void* workspace, size_t workspace_bytes, void* stream) {
+    Layout L;
+    const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
+    comba_status_t st = plan(shape, save ? 1 : 0, &L);
+    if (st != COMBA_OK) return st;
+    if (!(shape->flags & COMBA_GATED) || (shape->flags & ~(COMBA_GATED | COMBA_SAVE_FACTORS | COMBA_IPLR)))
+        return COMBA_ERR_INVALID_ARG;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(g_alpha); COMBA_REQUIRE(g_beta);
+    COMBA_REQUIRE(a); COMBA_REQUIRE(c); COMBA_REQUIRE(b_raw); COMBA_REQUIRE(d); COMBA_REQUIRE(o);
+    COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
+    if (shape->stage_events && shape->num_stage_events < COMBA_FWD_EVENTS) return COMBA_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const comba::GateParams g = gate_params(shape, L, workspace, q, k, g_alpha, g_beta, a, c, b_raw);
+    if (comba::launch_gate_prologue(g, shape->dtype == COMBA_BF16, shape->dk, s) != cudaSuccess) return COMBA_ERR_CUDA;
+    return forward_run(shape, L, workspace, g.qh, g.kh, v, g.alpha, g.beta, g.bgate, d, h0, o, hT, save, s);
+}
+
+comba_status_t comba_chunk_bwd_gated(const comba_shape_t* shape, const void* q, const void* k, const void* v,
+                                     const float* g_alpha, const float* g_beta, const float* a, const float* c,
+                                     const float* b_raw, const float* d, const float* h0, const void* dO,
+                                     const float* dhT, void* dq, void* dk, void* dv, float* dg_alpha, float* dg_beta,
+                                     float* da, float* dc, float* db_raw, float* dd, float* dh0, void* workspace,
+                                     size_t workspace_bytes, void* stream) {
+    Layout L;
+    comba_status_t st = plan(shape, 1, &L);
+    if (st != COMBA_OK) return st;
+    if (!(shape->flags & COMBA_GATED) || (shape->flags & ~(COMBA_GATED | COMBA_REUSE_FACTORS | COMBA_IPLR)))
+        return COMBA_ERR_INVALID_ARG;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(g_alpha); COMBA_REQUIRE(g_beta);
+    COMBA_REQUIRE(a); COMBA_REQUIRE(c); COMBA_REQUIRE(b_raw); COMBA_REQUIRE(d); COMBA_REQUIRE(dO);
+    COMBA_REQUIRE(dq); COMBA_REQUIRE(dk); COMBA_REQUIRE(dv); COMBA_REQUIRE(dg_alpha); COMBA_REQUIRE(dg_beta);
+    COMBA_REQUIRE(da); COMBA_REQUIRE(dc); COMBA_REQUIRE(dd);
+    COMBA_OPTIONAL(h0); COMBA_OPTIONAL(dhT); COMBA_OPTIONAL(db_raw); COMBA_OPTIONAL(dh0);
+    if (shape->stage_events && shape->num_stage_events < COMBA_BWD_EVENTS) return COMBA_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bool reuse = (shape->flags & COMBA_REUSE_FACTORS) != 0;
     const bool bf = shape->dtype == COMBA_BF16;
-    comba::mark(p, 0, s);
-    if (reuse) {
-        for (int e = 1; e <= 4; ++e) comba::mark(p, e, s);
-    } else {
-        // recompute the forward factors and chunk states (no output, no final state)
-        ChunkParams f = p;
-        f.o = nullptr;
-        f.hT = nullptr;
-        if (comba::launch_chunk_map(f, s) != cudaSuccess) return COMBA_ERR_CUDA;
-        if (comba::launch_fwd(f, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
-    }
-    if (comba::launch_bwd(p, bf, s, 4) != cudaSuccess) return COMBA_ERR_CUDA;
+    comba::GateParams g = gate_params(shape, L, workspace, q, k, g_alpha, g_beta, a, c, b_raw);
+    // with reused factors the saving forward left the prologue's outputs in the workspace
+    if (!reuse && comba::launch_gate_prologue(g, bf, shape->dk, s) != cudaSuccess) return COMBA_ERR_CUDA;
+    char* w = static_cast<char*>(workspace);
+    g.dqh = w + L.dqh; g.dkh = w + L.dkh;
+    g.dalpha = reinterpret_cast<float*>(w + L.dal);
+    g.dbeta = reinterpret_cast<float*>(w + L.dbe);
+    g.db = reinterpret_cast<float*>(w + L.dbi);
+    g.dq = dq; g.dk = dk; g.dg_alpha = dg_alpha; g.dg_beta = dg_beta; g.da = da; g.dc = dc; g.db_raw = db_raw;
+    g.da_rows = reinterpret_cast<float*>(w + L.dar);
+    g.dc_rows = reinterpret_cast<float*>(w + L.dcr);
+    g.da_part = reinterpret_cast<float*>(w + L.dpa);
+    g.dc_part = reinterpret_cast<float*>(w + L.dpc);
+    st = backward_run(shape, L, workspace, g.qh, g.kh, v, g.alpha, g.beta, g.bgate, d, h0, dO, dhT,
+                      const_cast<void*>(g.dqh), const_cast<void*>(g.dkh), dv, const_cast<float*>(g.dalpha),
+                      const_cast<float*>(g.dbeta), const_cast<float*>(g.db), dd, dh0, reuse, s);
+    if (st != COMBA_OK) return st;
+    if (comba::launch_gate_epilogue(g, bf, shape->dk, s) != cudaSuccess) return COMBA_ERR_CUDA;
     return COMBA_OK;
 }
 

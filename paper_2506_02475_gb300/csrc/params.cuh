@@ -62,6 +62,44 @@ struct ChunkParams {
     int nev;
 };
 
+// Gate and normalisation prologue / epilogue (gates.cu): raw inputs, the prologue's outputs
+// in the workspace, and (backward) the chunk backward's gradients mapped to the raw inputs.
+struct GateParams {
+    long long rows;          // tokens * H
+    int H;
+    float eps;
+    const void* q;           // raw q, k [tokens, H, dk]
+    const void* k;
+    const float* g_alpha;    // [tokens, H] gate pre-activations
+    const float* g_beta;
+    const float* a;          // [H] per-head scalars
+    const float* c;
+    const float* b_raw;
+    void* qh;                // prologue outputs
+    void* kh;
+    float* alpha;
+    float* beta;
+    float* bgate;            // [H] sigmoid(b_raw)
+    const void* dqh;         // chunk backward outputs (gradients w.r.t. the prologue outputs)
+    const void* dkh;
+    const float* dalpha;
+    const float* dbeta;
+    const float* db;
+    void* dq;                // gradients w.r.t. the raw inputs
+    void* dk;
+    float* dg_alpha;
+    float* dg_beta;
+    float* da;
+    float* dc;
+    float* db_raw;
+    float* da_rows;          // [tokens, H] per-row contributions, summed per head in a fixed order
+    float* dc_rows;
+    float* da_part;          // [H, ceil(tokens / 64)] token-block sums of da_rows, dc_rows
+    float* dc_part;
+};
+cudaError_t launch_gate_prologue(const GateParams& g, bool is_bf16, int dk, cudaStream_t s);
+cudaError_t launch_gate_epilogue(const GateParams& g, bool is_bf16, int dk, cudaStream_t s);
+
 // Record stage-boundary event i on stream s when instrumentation is on.
 inline void mark(const ChunkParams& p, int i, cudaStream_t s) {
     if (p.ev && i < p.nev) cudaEventRecord(p.ev[i], s);

@@ -225,3 +225,54 @@ def decode_tokens(step, Bd=256, H=16, dk=128, dv=128, dtype="bf16", seed_offset=
     drng = np.random.Generator(np.random.PCG64(SEED + 8000))   # a parameter: shared by every rank
     d = drng.uniform(0.0, 1.0, size=H).astype(np.float32)
     return q, k, v, alpha, beta, d
+
+
+@dataclass
+class GatedWorkload:
+    """Raw inputs of the gate and normalisation prologue (q, k not normalised; gate pre-activations)."""
+    dtype: str
+    q: np.ndarray            # [B,T,H,dk] or packed [Ttot,H,dk]
+    k: np.ndarray
+    v: np.ndarray
+    g_alpha: np.ndarray      # [B,T,H] or [Ttot,H]
+    g_beta: np.ndarray
+    a: np.ndarray            # [H]
+    c: np.ndarray
+    b_raw: np.ndarray
+    d: np.ndarray
+    h0: Optional[np.ndarray]
+    dO: np.ndarray
+    dhT: np.ndarray
+    cu_seqlens: Optional[np.ndarray] = None
+
+
+def make_gated(B=2, T=200, H=3, dk=128, dv=128, dtype="bf16", seed_offset=0, lengths=None, with_h0=True):
+    """Seeded raw inputs: q, k ~ N(0, s^2) with a per-row scale s in [0.5, 2] (so the in-kernel L2
+    norm has work to do), v ~ N(0,1), gate pre-activations ~ N(0,1), a ~ U(0.05, 0.3) (alpha near 1
+    as the forgetting section asks), c, b_raw ~ U(-1, 1), d ~ U(0, 1); bf16 rounding on the host."""
+    rng = np.random.Generator(np.random.PCG64(SEED + 9000 + seed_offset))
+    cu = None
+    if lengths is not None:
+        lengths = np.asarray(lengths, dtype=np.int64)
+        cu = np.concatenate([[0], np.cumsum(lengths)]).astype(np.int64)
+        lead, N = (int(cu[-1]),), len(lengths)
+    else:
+        lead, N = (B, T), B
+    q = rng.standard_normal(lead + (H, dk)) * rng.uniform(0.5, 2.0, lead + (H, 1))
+    k = rng.standard_normal(lead + (H, dk)) * rng.uniform(0.5, 2.0, lead + (H, 1))
+    v = rng.standard_normal(lead + (H, dv))
+    dO = rng.standard_normal(lead + (H, dv))
+    q, k, v, dO = (x.astype(np.float32) for x in (q, k, v, dO))
+    if dtype == "bf16":
+        q, k, v, dO = (round_bf16(x) for x in (q, k, v, dO))
+    g_alpha = rng.standard_normal(lead + (H,)).astype(np.float32)
+    g_beta = rng.standard_normal(lead + (H,)).astype(np.float32)
+    prng = np.random.Generator(np.random.PCG64(SEED + 9500))
+    a = prng.uniform(0.05, 0.3, H).astype(np.float32)
+    c = prng.uniform(-1.0, 1.0, H).astype(np.float32)
+    b_raw = prng.uniform(-1.0, 1.0, H).astype(np.float32)
+    d = prng.uniform(0.0, 1.0, H).astype(np.float32)
+    h0 = (0.1 * rng.standard_normal((N, H, dk, dv))).astype(np.float32) if with_h0 else None
+    dhT = (0.1 * rng.standard_normal((N, H, dk, dv))).astype(np.float32)
+    return GatedWorkload(dtype=dtype, q=q, k=k, v=v, g_alpha=g_alpha, g_beta=g_beta, a=a, c=c, b_raw=b_raw, d=d,
+                         h0=h0, dO=dO, dhT=dhT, cu_seqlens=cu)

@@ -148,3 +148,19 @@ def test_recurrent_step_validation(L):
     assert call(dtype=3) == INVALID
     assert call(state=None) == INVALID
     assert call(q=FAKE + 2) == INVALID
+
+
+def test_gated_flag_rules(L):
+    """COMBA_GATED selects the gated entry points; the plain ones reject it, and the gated
+    workspace is larger (it holds the prologue's outputs)."""
+    plain, gated_ws = ws(L, shape(), 1), ws(L, shape(flags=8), 1)
+    assert gated_ws > plain
+    assert fwd(L, shape(flags=8)) == INVALID
+    s = shape(flags=0)
+    args = [FAKE] * 12
+    # the gated forward without COMBA_GATED in the shape is invalid
+    assert L.comba_chunk_fwd_gated(ctypes.byref(s), *args, FAKE, 1 << 40, None) == INVALID
+    s.flags = 8
+    assert L.comba_chunk_fwd_gated(ctypes.byref(s), *args, None, 0, None) == WORKSPACE
+    args[5] = None   # a is required
+    assert L.comba_chunk_fwd_gated(ctypes.byref(s), *args, None, 0, None) == INVALID
