@@ -91,14 +91,14 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 110_757, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "8037a0f379eeca70"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_659, ('scan.cu', 'common.cuh', 'params.cuh'), "078fa92632262989"),
-    "output": ("k_output_tc", 118_728, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "8037a0f379eeca70"),
-    "bwd_prep": ("k_bwd_prep_tc", 82_599, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "8037a0f379eeca70"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_522, ('scan.cu', 'common.cuh', 'params.cuh'), "078fa92632262989"),
-    "bwd_local": ("k_bwd_local_tc", 194_416, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "7bdbfc4ffe1922cb"),
+    "prep": ("k_prep_tc", 110_865, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "f839f342596f289d"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_531, ('scan.cu', 'common.cuh', 'params.cuh'), "de0526678a01fe09"),
+    "output": ("k_output_tc", 118_692, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "f839f342596f289d"),
+    "bwd_prep": ("k_bwd_prep_tc", 82_581, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "f839f342596f289d"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_381, ('scan.cu', 'common.cuh', 'params.cuh'), "de0526678a01fe09"),
+    "bwd_local": ("k_bwd_local_tc", 194_263, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "69eee2248b1e4386"),
 }
-DECODE_TRAFFIC = (482_097_920, ('decode.cu', 'common.cuh', 'params.cuh'), "0daad7feb5fb12b6")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (482_260_224, ('decode.cu', 'common.cuh', 'params.cuh'), "8adc5b26525edb4b")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
@@ -268,23 +268,35 @@ def dist_init(world, local, backend):
 # -------------------------------------------------------- CPU oracle timing
 
 def oracle_sample(w, rows, heads, tokens):
-    """Bounded slice of a dense workload: batch rows `rows`, heads, first `tokens` tokens."""
-    sl = (slice(rows[0], rows[1]), slice(0, tokens), slice(heads[0], heads[1]))
+    """Bounded slice of a workload: batch rows `rows`, heads, first `tokens` tokens (a packed
+    workload: the first `tokens` tokens of the packed stream, its sequences cut there)."""
+    if w.cu_seqlens is not None:
+        sl = (slice(0, tokens), slice(heads[0], heads[1]))
+        cu = np.asarray(w.cu_seqlens, np.int64)
+        cu = np.concatenate([cu[cu < tokens], [tokens]])
+        n = len(cu) - 1
 
-    def st(x):
-        return None if x is None else np.ascontiguousarray(x[rows[0]:rows[1], heads[0]:heads[1]])
+        def st(x):
+            return None if x is None else np.ascontiguousarray(x[:n, heads[0]:heads[1]])
+    else:
+        sl = (slice(rows[0], rows[1]), slice(0, tokens), slice(heads[0], heads[1]))
+        cu = None
+
+        def st(x):
+            return None if x is None else np.ascontiguousarray(x[rows[0]:rows[1], heads[0]:heads[1]])
 
     return dict(q=np.ascontiguousarray(w.q[sl]), k=np.ascontiguousarray(w.k[sl]), v=np.ascontiguousarray(w.v[sl]),
                 alpha=np.ascontiguousarray(w.alpha[sl]), beta=np.ascontiguousarray(w.beta[sl]),
                 b=None if w.b is None else w.b[heads[0]:heads[1]], d=w.d[heads[0]:heads[1]], h0=st(w.h0),
-                dO=np.ascontiguousarray(w.dO[sl]), dhT=st(w.dhT))
+                dO=np.ascontiguousarray(w.dO[sl]), dhT=st(w.dhT), cu_seqlens=cu)
 
 
 def time_oracle_step(s):
     import oracle
     t0 = time.perf_counter()
-    oracle.fwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], h0=s["h0"])
-    oracle.bwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], s["dO"], h0=s["h0"], dhT=s["dhT"])
+    oracle.fwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], h0=s["h0"], cu_seqlens=s["cu_seqlens"])
+    oracle.bwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], s["dO"], h0=s["h0"], dhT=s["dhT"],
+               cu_seqlens=s["cu_seqlens"])
     return time.perf_counter() - t0
 
 
@@ -293,7 +305,10 @@ def cpu_baseline(w, target_s=12.0):
     sample (token prefix of batch row 0, then whole batch rows) until about `target_s`
     seconds of wall time or the whole workload."""
     import oracle
-    B, T, H = w.q.shape[0], w.q.shape[1], w.q.shape[2]
+    if w.cu_seqlens is not None:
+        B, T, H = 1, w.q.shape[0], w.q.shape[1]
+    else:
+        B, T, H = w.q.shape[0], w.q.shape[1], w.q.shape[2]
     rows, tokens = 1, min(T, 256)
     while True:
         s = oracle_sample(w, (0, rows), (0, H), tokens)
@@ -624,6 +639,46 @@ def run_gated(args, world, rank, local):
 
 # ------------------------------------------------------------------ decode
 
+def decode_oracle_sample(Bd, H, dk, dv, rows):
+    """The first `rows` decode rows (all heads) of the decode workload: fp32 state and the
+    8 token sets the GPU leg cycles through."""
+    from paper_2506_02475_gb300 import inputs
+    state = inputs.decode_state(Bd, H, dk, dv)[:rows]
+    toks = []
+    for s_ in range(8):
+        q, k, v, a, be, d = inputs.decode_tokens(s_, Bd, H, dk, dv, "bf16")
+        toks.append((q[:rows], k[:rows], v[:rows], a[:rows], be[:rows]))
+    return state, toks, d
+
+
+def time_oracle_decode(state, toks, d, nsteps):
+    """`nsteps` sequential oracle decode steps from `state`; wall seconds."""
+    import oracle
+    t0 = time.perf_counter()
+    st = state
+    for i in range(nsteps):
+        q, k, v, a, be = toks[i % 8]
+        _, st = oracle.step(q, k, v, a, be, None, d, st)
+    return time.perf_counter() - t0
+
+
+def decode_cpu_baseline(Bd, H, dk, dv, rows=32, target_s=10.0):
+    """The oracle's decode step on the host cores: the first `rows` decode rows, all heads,
+    sequential token steps until about `target_s` seconds."""
+    import oracle
+    state, toks, d = decode_oracle_sample(Bd, H, dk, dv, rows)
+    n, dt = 2, 0.0
+    while True:
+        dt = time_oracle_decode(state, toks, d, n)
+        if dt >= target_s or n >= 4096:
+            break
+        n = int(n * max(2.0, min(8.0, target_s / max(dt, 1e-3))))
+    return {"value": rows * n / dt, "unit": "tokens/s", "cores": oracle.default_threads(), "kind": "oracle",
+            "sample": f"decode rows 0..{rows - 1} of {Bd}, all {H} heads, {n} sequential token steps "
+                      f"(fp64 recurrence, fp32 state widened): {dt:.2f} s"}
+
+
+
 def run_decode(args, world, rank, local):
     import torch
     dist = dist_init(world, local, "nccl")
@@ -667,6 +722,55 @@ def run_decode(args, world, rank, local):
     per = ms / steps
     bytes_step = Bd * H * (2 * dk * dv * 4 + (2 * dk + 2 * dv) * 2 + 8)
     gbs = bytes_step / (per / 1e3) / 1e9
+
+    # ---- end to end through the public API: every token step uploads its q, k, v, alpha,
+    # beta from pinned host memory and reads its o back; the recurrent state is the model's
+    # memory and stays resident on the device.  Upload and download run on their own streams
+    # over two device buffer sets, so step i's upload and step i-1's download overlap step i.
+    htoks = [[x.cpu().pin_memory() for x in t] for t in toks]
+    sets = [([torch.empty_like(x) for x in toks[0]], torch.empty_like(o), torch.empty(o.shape, dtype=o.dtype).pin_memory())
+            for _ in range(2)]
+    comp, up, down = torch.cuda.current_stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    ev = {n_: [torch.cuda.Event() for _ in range(2)] for n_ in ("uploaded", "computed", "downloaded")}
+
+    def run_e2e(nsteps, t_start=None, t_end=None):
+        for i in range(nsteps):
+            j = i % 2
+            dbuf, dout, hout = sets[j]
+            with torch.cuda.stream(up):
+                if i == 0 and t_start is not None:
+                    t_start.record(up)
+                if i >= 2:
+                    up.wait_event(ev["computed"][j])          # step i-2 finished reading this buffer set
+                for dst, src in zip(dbuf, htoks[i % 8]):
+                    dst.copy_(src, non_blocking=True)
+                ev["uploaded"][j].record(up)
+            comp.wait_event(ev["uploaded"][j])
+            if i >= 2:
+                comp.wait_event(ev["downloaded"][j])          # step i-2's o is on the host
+            comba_recurrent_step(dbuf[0], dbuf[1], dbuf[2], dbuf[3], dbuf[4], d, state, o=dout)
+            ev["computed"][j].record(comp)
+            with torch.cuda.stream(down):
+                down.wait_event(ev["computed"][j])
+                hout.copy_(dout, non_blocking=True)
+                ev["downloaded"][j].record(down)
+                if i == nsteps - 1 and t_end is not None:
+                    t_end.record(down)
+
+    run_e2e(max(2, args.warmup))
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    run_e2e(steps, e_start, e_end)
+    torch.cuda.synchronize()
+    e_ms = shard.max_over_ranks(e_start.elapsed_time(e_end), dist, dev)
+    bi = sum(x.numel() * x.element_size() for x in htoks[0])
+    bo = o.numel() * o.element_size()
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = decode_cpu_baseline(Bd, H, dk, dv)
     if rank == 0:
         print(json.dumps({
             "metric": DECODE_METRIC, "value": Bd * steps * world / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
@@ -678,6 +782,11 @@ def run_decode(args, world, rank, local):
                          "frac": gbs / peaks["hbm_gbs"], "kernel": "k_step", "launch_ms": per,
                          "traffic": DECODE_TRAFFIC[0] if sources_hash(DECODE_TRAFFIC[1]) == DECODE_TRAFFIC[2] else None,
                          "peak_source": peak_src},
+            "cpu_baseline": cpu,
+            "e2e": {"value": Bd * steps * world / (e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": bi,
+                    "d2h_bytes_per_step": bo, "ms_per_token_step": e_ms / steps,
+                    "copies": "q, k, v, alpha, beta uploaded from pinned host memory and o read back every token "
+                              "step (own streams, double-buffered); the state stays on the device"},
             "clocks": clk, "gpu_launches": steps * args.steps}), flush=True)
     if dist:
         dist.destroy_process_group()
@@ -691,9 +800,28 @@ def run_reference(args, world, rank, local):
         return
     import oracle
     from paper_2506_02475_gb300 import inputs
+    if args.workload == "decode":
+        Bd, H, dk, dv, rows, per_step = 256, 16, 128, 128, 32, 8
+        state, toks, d = decode_oracle_sample(Bd, H, dk, dv, rows)
+        for _ in range(args.warmup):
+            time_oracle_decode(state, toks, d, per_step)
+        dt = sum(time_oracle_decode(state, toks, d, per_step) for _ in range(args.steps)) / args.steps
+        value = rows * per_step / dt
+        sample = f"decode rows 0..{rows - 1} of {Bd}, all {H} heads, {per_step} sequential token steps per step"
+        print(json.dumps({
+            "metric": DECODE_METRIC, "impl": "reference", "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"decode: Bd={Bd} H={H} dk={dk} dv={dv}", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.default_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }), flush=True)
+        return
     w = inputs.make(args.workload)
     H = w.H
-    tokens = min(int(w.q.shape[1]), args.reference_tokens)
+    total = int(w.q.shape[0] if w.cu_seqlens is not None else w.q.shape[1])   # tokens of batch row 0 / the pack
+    tokens = min(total, args.reference_tokens)
     s = oracle_sample(w, (0, 1), (0, H), tokens)
     for _ in range(args.warmup):
         time_oracle_step(s)
