@@ -48,11 +48,11 @@ def build(force: bool = False) -> str:
 def _bind(lib):
     P = ctypes.c_void_p
     I = ctypes.c_int
-    lib.comba_oracle_fwd.argtypes = [I, P, I, I, I] + [P] * 10 + [I, I]
+    lib.comba_oracle_fwd.argtypes = [I, P, I, I, I] + [P] * 11 + [I, I]
     lib.comba_oracle_fwd.restype = I
-    lib.comba_oracle_bwd.argtypes = [I, P, I, I, I] + [P] * 8 + [P, P] + [P] * 8 + [I, I]
+    lib.comba_oracle_bwd.argtypes = [I, P, I, I, I] + [P] * 9 + [P, P] + [P] * 9 + [I, I]
     lib.comba_oracle_bwd.restype = I
-    lib.comba_oracle_step.argtypes = [I, I, I, I] + [P] * 9 + [I, I]
+    lib.comba_oracle_step.argtypes = [I, I, I, I] + [P] * 10 + [I, I]
     lib.comba_oracle_step.restype = I
     return lib
 
@@ -93,7 +93,7 @@ def _ptr(x):
     return None if x is None else x.ctypes.data_as(ctypes.c_void_p)
 
 
-def _packed(q, k, v, alpha, beta, cu_seqlens):
+def _packed(q, k, v, alpha, beta, cu_seqlens, p=None):
     """Return packed [Ttot,H,D] views plus int64 cu, and the original batch shape."""
     if q.ndim == 4:
         if cu_seqlens is not None:
@@ -102,6 +102,7 @@ def _packed(q, k, v, alpha, beta, cu_seqlens):
         cu = np.arange(B + 1, dtype=np.int64) * T
         shape = (B, T)
         q, k, v = (x.reshape(B * T, H, x.shape[-1]) for x in (q, k, v))
+        p = None if p is None else p.reshape(B * T, H, p.shape[-1])
         alpha, beta = alpha.reshape(B * T, H), beta.reshape(B * T, H)
     else:
         if cu_seqlens is None:
@@ -109,27 +110,30 @@ def _packed(q, k, v, alpha, beta, cu_seqlens):
         else:
             cu = np.ascontiguousarray(cu_seqlens, dtype=np.int64)
         shape = None
-    return q, k, v, alpha, beta, cu, shape
+    return q, k, v, alpha, beta, cu, shape, p
 
 
 VARIANTS = {"splr": 0, "iplr": 1}
 
 
-def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=None, variant="splr"):
+def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=None, variant="splr", p=None):
     """Token recurrence forward.  Returns ``(o, hT)`` in float64.
 
-    ``variant="iplr"``: the Comba-iplr transition alpha (I - 2 btilde k k^T)."""
-    q, k, v, alpha, beta, b, d, h0 = map(_f64, (q, k, v, alpha, beta, b, d, h0))
-    q, k, v, alpha, beta, cu, shape = _packed(q, k, v, alpha, beta, cu_seqlens)
+    ``variant="iplr"``: the Comba-iplr transition alpha (I - 2 btilde k k^T).
+    ``p`` (shaped like k): the Comba-pk feedback vectors of appendix B.3, read
+    back from the state and used in the output correction in place of k."""
+    q, k, v, alpha, beta, b, d, h0, p = map(_f64, (q, k, v, alpha, beta, b, d, h0, p))
+    q, k, v, alpha, beta, cu, shape, p = _packed(q, k, v, alpha, beta, cu_seqlens, p)
     Ttot, H, dk = q.shape
     dv = v.shape[-1]
     N = cu.shape[0] - 1
     q, k, v, alpha, beta = map(np.ascontiguousarray, (q, k, v, alpha, beta))
+    p = None if p is None else np.ascontiguousarray(p)
     o = np.zeros((Ttot, H, dv), np.float64)
     hT = np.zeros((N, H, dk, dv), np.float64)
-    rc = (lib or _load()).comba_oracle_fwd(N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta),
-                                  _ptr(b), _ptr(d), _ptr(h0), _ptr(o), _ptr(hT), threads or default_threads(),
-                                  VARIANTS[variant])
+    rc = (lib or _load()).comba_oracle_fwd(N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(p), _ptr(alpha),
+                                  _ptr(beta), _ptr(b), _ptr(d), _ptr(h0), _ptr(o), _ptr(hT),
+                                  threads or default_threads(), VARIANTS[variant])
     if rc:
         raise MemoryError("oracle forward failed to allocate")
     if shape is not None:
@@ -138,47 +142,54 @@ def fwd(q, k, v, alpha, beta, b, d, h0=None, cu_seqlens=None, threads=None, lib=
 
 
 def bwd(q, k, v, alpha, beta, b, d, dO, h0=None, dhT=None, cu_seqlens=None, threads=None, lib=None,
-        variant="splr"):
-    """Exact BPTT.  Returns a dict with dq, dk, dv, dalpha, dbeta, db, dd, dh0."""
-    q, k, v, alpha, beta, b, d, h0, dO, dhT = map(_f64, (q, k, v, alpha, beta, b, d, h0, dO, dhT))
+        variant="splr", p=None):
+    """Exact BPTT.  Returns a dict with dq, dk, dv, dalpha, dbeta, db, dd, dh0 (and dp when
+    the Comba-pk feedback vectors ``p`` are given)."""
+    q, k, v, alpha, beta, b, d, h0, dO, dhT, p = map(_f64, (q, k, v, alpha, beta, b, d, h0, dO, dhT, p))
     batched = q.ndim == 4
-    q, k, v, alpha, beta, cu, shape = _packed(q, k, v, alpha, beta, cu_seqlens)
+    q, k, v, alpha, beta, cu, shape, p = _packed(q, k, v, alpha, beta, cu_seqlens, p)
     if batched:
         dO = dO.reshape(-1, dO.shape[-2], dO.shape[-1])
     Ttot, H, dk = q.shape
     dv = v.shape[-1]
     N = cu.shape[0] - 1
     q, k, v, alpha, beta, dO = map(np.ascontiguousarray, (q, k, v, alpha, beta, dO))
+    p = None if p is None else np.ascontiguousarray(p)
     out = {
         "dq": np.zeros((Ttot, H, dk)), "dk": np.zeros((Ttot, H, dk)), "dv": np.zeros((Ttot, H, dv)),
         "dalpha": np.zeros((Ttot, H)), "dbeta": np.zeros((Ttot, H)),
         "db": np.zeros(H), "dd": np.zeros(H), "dh0": np.zeros((N, H, dk, dv)),
     }
+    if p is not None:
+        out["dp"] = np.zeros((Ttot, H, dk))
     rc = (lib or _load()).comba_oracle_bwd(
-        N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b), _ptr(d), _ptr(h0),
-        _ptr(dO), _ptr(dhT), _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]), _ptr(out["dalpha"]),
-        _ptr(out["dbeta"]), _ptr(out["db"]), _ptr(out["dd"]), _ptr(out["dh0"]), threads or default_threads(),
-        VARIANTS[variant])
+        N, _ptr(cu), H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(p), _ptr(alpha), _ptr(beta), _ptr(b), _ptr(d),
+        _ptr(h0), _ptr(dO), _ptr(dhT), _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]), _ptr(out.get("dp")),
+        _ptr(out["dalpha"]), _ptr(out["dbeta"]), _ptr(out["db"]), _ptr(out["dd"]), _ptr(out["dh0"]),
+        threads or default_threads(), VARIANTS[variant])
     if rc:
         raise MemoryError("oracle backward failed to allocate")
     if shape is not None:
         B, T = shape
-        for key in ("dq", "dk", "dv"):
-            out[key] = out[key].reshape(B, T, H, -1)
+        for key in ("dq", "dk", "dv", "dp"):
+            if key in out:
+                out[key] = out[key].reshape(B, T, H, -1)
         for key in ("dalpha", "dbeta"):
             out[key] = out[key].reshape(B, T, H)
     return out
 
 
-def step(q, k, v, alpha, beta, b, d, state, threads=None, lib=None, variant="splr"):
-    """One decode token.  ``state`` [Bd,H,dk,dv] is copied, updated and returned with ``o``."""
-    q, k, v, alpha, beta, b, d = map(_f64, (q, k, v, alpha, beta, b, d))
+def step(q, k, v, alpha, beta, b, d, state, threads=None, lib=None, variant="splr", p=None):
+    """One decode token.  ``state`` [Bd,H,dk,dv] is copied, updated and returned with ``o``.
+    ``p`` [Bd,H,dk]: Comba-pk feedback vectors (default: k)."""
+    q, k, v, alpha, beta, b, d, p = map(_f64, (q, k, v, alpha, beta, b, d, p))
     st = np.array(state, dtype=np.float64, copy=True, order="C")
     Bd, H, dk = q.shape
     dv = v.shape[-1]
     o = np.zeros((Bd, H, dv), np.float64)
-    rc = (lib or _load()).comba_oracle_step(Bd, H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(alpha), _ptr(beta), _ptr(b),
-                                   _ptr(d), _ptr(st), _ptr(o), threads or default_threads(), VARIANTS[variant])
+    rc = (lib or _load()).comba_oracle_step(Bd, H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(p), _ptr(alpha),
+                                   _ptr(beta), _ptr(b), _ptr(d), _ptr(st), _ptr(o), threads or default_threads(),
+                                   VARIANTS[variant])
     if rc:
         raise MemoryError("oracle step failed to allocate")
     return o, st

@@ -22,13 +22,23 @@
  * the transition alpha_t (I - 2 btilde_t k_t k_t^T), i.e. the same recurrence
  * with the feedback strength btilde_t replaced by 2 alpha_t b_h beta_t.
  *
+ * Comba-pk (appendix B.3, the "p" form of the recurrence): a per-token feedback
+ * vector p_t replaces k_t where the state is read back and in the output
+ * correction, while k_t still writes the state:
+ *
+ *   x_t = H_{t-1}^T p_t,   e_t = beta_t v_t - btilde_t x_t,
+ *   H_t = alpha_t H_{t-1} + k_t e_t^T,   o_t = H_t^T (q_t - d_h p_t)
+ *
+ * (transition alpha_t I - btilde_t p_t k_t^T on S).  p = NULL means p_t = k_t,
+ * which is the form above; p = b k with b = 1 in the pk form is the same model.
+ *
  * The backward pass is exact back-propagation through time of that
  * recurrence (the paper prints no backward; these are the chain-rule
  * derivatives of the four lines above).  States are checkpointed every
  * SEG tokens and each segment is recomputed before it is differentiated.
  *
  * Layouts (all row-major, doubles, host memory):
- *   q, k      [Ttot, H, dk]      v, o, dO  [Ttot, H, dv]
+ *   q, k, p   [Ttot, H, dk]      v, o, dO  [Ttot, H, dv]
  *   alpha,beta[Ttot, H]          b, d      [H]  (b may be NULL: b = 1)
  *   h0, hT    [N, H, dk, dv]     cu        int64 [N+1], token offsets
  * A dense batch [B, T, H, D] is the packed layout with cu = {0, T, 2T, ...}.
@@ -47,9 +57,10 @@ typedef struct {
     int N, H, dk, dv;
     const int64_t *cu;
     const double *q, *k, *v, *alpha, *beta, *b, *d, *h0;
+    const double *p; /* [Ttot, H, dk] feedback vectors (Comba-pk), or NULL: p_t = k_t */
     double *o, *hT;
     const double *dO, *dhT;
-    double *dq, *dk_, *dv_, *dalpha, *dbeta, *dh0;
+    double *dq, *dk_, *dv_, *dp, *dalpha, *dbeta, *dh0;
     double *db_part, *dd_part; /* [N*H] */
     int nthreads, tid;
     int status;
@@ -58,6 +69,9 @@ typedef struct {
 
 /* Feedback strength of token t relative to b_h beta_t: 1, or 2 alpha_t for iplr. */
 static double fb_scale(const job_t *J, double a) { return J->variant == 1 ? 2.0 * a : 1.0; }
+
+/* The feedback vector of token t (row offset tk = (t * H + h) * dk): p_t, or k_t. */
+static const double *fb_vec(const job_t *J, size_t tk) { return J->p ? J->p + tk : J->k + tk; }
 
 /* ---------------------------------------------------------------- forward */
 
@@ -74,17 +88,18 @@ static void fwd_unit(const job_t *J, int n, int h, double *Hs, double *x, double
 
     for (int64_t t = J->cu[n]; t < J->cu[n + 1]; ++t) {
         const double *kt = J->k + ((size_t)t * Hh + h) * dk;
+        const double *ft = fb_vec(J, ((size_t)t * Hh + h) * dk);
         const double *qt = J->q + ((size_t)t * Hh + h) * dk;
         const double *vt = J->v + ((size_t)t * Hh + h) * dv;
         const double a = J->alpha[(size_t)t * Hh + h];
         const double be = J->beta[(size_t)t * Hh + h];
         const double bt = bh * be * fb_scale(J, a);
-        /* x = H^T k, read from the state before this token's update */
+        /* x = H^T p (p = k unless given), read from the state before this token's update */
         for (int j = 0; j < dv; ++j) x[j] = 0.0;
         for (int i = 0; i < dk; ++i) {
-            const double ki = kt[i];
+            const double fi = ft[i];
             const double *row = Hs + (size_t)i * dv;
-            for (int j = 0; j < dv; ++j) x[j] += row[j] * ki;
+            for (int j = 0; j < dv; ++j) x[j] += row[j] * fi;
         }
         for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bt * x[j];
         for (int i = 0; i < dk; ++i) {
@@ -92,7 +107,7 @@ static void fwd_unit(const job_t *J, int n, int h, double *Hs, double *x, double
             double *row = Hs + (size_t)i * dv;
             for (int j = 0; j < dv; ++j) row[j] = a * row[j] + ki * e[j];
         }
-        for (int i = 0; i < dk; ++i) qn[i] = qt[i] - dh * kt[i];
+        for (int i = 0; i < dk; ++i) qn[i] = qt[i] - dh * ft[i];
         double *ot = J->o + ((size_t)t * Hh + h) * dv;
         for (int j = 0; j < dv; ++j) ot[j] = 0.0;
         for (int i = 0; i < dk; ++i) {
@@ -125,17 +140,19 @@ static void *fwd_worker(void *arg)
 
 /*
  * One unit.  G holds dL/dH_t while walking t downwards.  For token t, with
- * P = H_{t-1}, the local derivatives are
+ * P = H_{t-1} and f_t the feedback vector (p_t, or k_t), the local derivatives are
  *   G      += qn_t dO_t^T                 (o_t = H_t^T qn_t)
  *   dqn_t   = H_t dO_t
  *   dalpha_t= <G, P>
  *   de_t    = G^T k_t
- *   dk_t    = G e_t - btilde_t P de_t - d_h dqn_t
+ *   dk_t    = G e_t                       (k writes the state)
+ *   df_t    = -btilde_t P de_t - d_h dqn_t (f is read back and corrects q)
  *   dv_t    = beta_t de_t
  *   dbeta_t = v_t.de_t - b_h x_t.de_t     (direct + through btilde)
  *   db     -= beta_t x_t.de_t
- *   dd     -= k_t.dqn_t
- *   G       = alpha_t G - btilde_t k_t de_t^T
+ *   dd     -= f_t.dqn_t
+ *   G       = alpha_t G - btilde_t f_t de_t^T
+ * With f = k (no p) dk_t collects both lines.
  */
 static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *G,
                      double *x, double *e, double *qn, double *de, double *dqn)
@@ -161,12 +178,13 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
         const int64_t ta = t0 + s * SEG, tb = (ta + SEG < t1) ? ta + SEG : t1;
         for (int64_t t = ta; t < tb; ++t) {
             const double *kt = J->k + ((size_t)t * Hh + h) * dk;
+            const double *ft = fb_vec(J, ((size_t)t * Hh + h) * dk);
             const double *vt = J->v + ((size_t)t * Hh + h) * dv;
             const double a = J->alpha[(size_t)t * Hh + h];
             const double be = J->beta[(size_t)t * Hh + h];
             for (int j = 0; j < dv; ++j) x[j] = 0.0;
             for (int i = 0; i < dk; ++i)
-                for (int j = 0; j < dv; ++j) x[j] += Hn[(size_t)i * dv + j] * kt[i];
+                for (int j = 0; j < dv; ++j) x[j] += Hn[(size_t)i * dv + j] * ft[i];
             for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bh * be * fb_scale(J, a) * x[j];
             for (int i = 0; i < dk; ++i)
                 for (int j = 0; j < dv; ++j) Hn[(size_t)i * dv + j] = a * Hn[(size_t)i * dv + j] + kt[i] * e[j];
@@ -186,6 +204,7 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
         for (int r = 0; r < m; ++r) {
             const int64_t t = ta + r;
             const double *kt = J->k + ((size_t)t * Hh + h) * dk;
+            const double *ft = fb_vec(J, ((size_t)t * Hh + h) * dk);
             const double *vt = J->v + ((size_t)t * Hh + h) * dv;
             const double a = J->alpha[(size_t)t * Hh + h];
             const double be = J->beta[(size_t)t * Hh + h];
@@ -193,7 +212,7 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
             double *Q = seg + (size_t)(r + 1) * ssz;
             for (int j = 0; j < dv; ++j) x[j] = 0.0;
             for (int i = 0; i < dk; ++i)
-                for (int j = 0; j < dv; ++j) x[j] += P[(size_t)i * dv + j] * kt[i];
+                for (int j = 0; j < dv; ++j) x[j] += P[(size_t)i * dv + j] * ft[i];
             for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bh * be * fb_scale(J, a) * x[j];
             for (int i = 0; i < dk; ++i)
                 for (int j = 0; j < dv; ++j) Q[(size_t)i * dv + j] = a * P[(size_t)i * dv + j] + kt[i] * e[j];
@@ -202,6 +221,7 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
             const int64_t t = ta + r;
             const size_t tk = ((size_t)t * Hh + h) * dk, tv = ((size_t)t * Hh + h) * dv;
             const double *kt = J->k + tk, *qt = J->q + tk, *vt = J->v + tv, *dOt = J->dO + tv;
+            const double *ft = fb_vec(J, tk);
             const double a = J->alpha[(size_t)t * Hh + h];
             const double be = J->beta[(size_t)t * Hh + h];
             const double f = fb_scale(J, a);
@@ -211,9 +231,9 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
             /* recompute x_t, e_t */
             for (int j = 0; j < dv; ++j) x[j] = 0.0;
             for (int i = 0; i < dk; ++i)
-                for (int j = 0; j < dv; ++j) x[j] += P[(size_t)i * dv + j] * kt[i];
+                for (int j = 0; j < dv; ++j) x[j] += P[(size_t)i * dv + j] * ft[i];
             for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bt * x[j];
-            for (int i = 0; i < dk; ++i) qn[i] = qt[i] - dh * kt[i];
+            for (int i = 0; i < dk; ++i) qn[i] = qt[i] - dh * ft[i];
 
             /* output: G += qn dO^T ; dqn = H_t dO */
             for (int i = 0; i < dk; ++i) {
@@ -233,18 +253,24 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
                     de[j] += G[(size_t)i * dv + j] * kt[i];
                 }
             J->dalpha[(size_t)t * Hh + h] = da;
-            /* dk = G e - btilde P de - d dqn ; dq = dqn */
+            /* dk = G e ; df = -btilde P de - d dqn (into dk when f = k) ; dq = dqn */
             double *dkt = J->dk_ + tk, *dqt = J->dq + tk, *dvt = J->dv_ + tv;
-            double kdq = 0.0;
+            double fdq = 0.0;
             for (int i = 0; i < dk; ++i) {
                 double ge = 0.0, pde = 0.0;
                 for (int j = 0; j < dv; ++j) {
                     ge += G[(size_t)i * dv + j] * e[j];
                     pde += P[(size_t)i * dv + j] * de[j];
                 }
-                dkt[i] = ge - bt * pde - dh * dqn[i];
+                const double df = -bt * pde - dh * dqn[i];
+                if (J->p) {
+                    dkt[i] = ge;
+                    J->dp[tk + i] = df;
+                } else {
+                    dkt[i] = ge + df;
+                }
                 dqt[i] = dqn[i];
-                kdq += kt[i] * dqn[i];
+                fdq += ft[i] * dqn[i];
             }
             double vde = 0.0, xde = 0.0;
             for (int j = 0; j < dv; ++j) {
@@ -256,11 +282,11 @@ static void bwd_unit(job_t *J, int n, int h, double *ckpt, double *seg, double *
             J->dbeta[(size_t)t * Hh + h] = vde - bh * f * xde;
             db_acc -= be * f * xde;
             if (J->variant == 1) J->dalpha[(size_t)t * Hh + h] -= 2.0 * bh * be * xde;
-            dd_acc -= kdq;
+            dd_acc -= fdq;
             /* carry to H_{t-1} */
             for (int i = 0; i < dk; ++i)
                 for (int j = 0; j < dv; ++j)
-                    G[(size_t)i * dv + j] = a * G[(size_t)i * dv + j] - bt * kt[i] * de[j];
+                    G[(size_t)i * dv + j] = a * G[(size_t)i * dv + j] - bt * ft[i] * de[j];
         }
     }
     if (J->dh0) memcpy(J->dh0 + ((size_t)n * Hh + h) * ssz, G, ssz * sizeof(double));
@@ -330,7 +356,7 @@ static int run_pool(job_t *proto, void *(*fn)(void *))
 /* --------------------------------------------------------------- exports */
 
 int comba_oracle_fwd(int N, const int64_t *cu, int H, int dk, int dv,
-                     const double *q, const double *k, const double *v,
+                     const double *q, const double *k, const double *v, const double *p,
                      const double *alpha, const double *beta, const double *b, const double *d,
                      const double *h0, double *o, double *hT, int nthreads, int variant)
 {
@@ -338,25 +364,26 @@ int comba_oracle_fwd(int N, const int64_t *cu, int H, int dk, int dv,
     memset(&J, 0, sizeof(J));
     J.variant = variant;
     J.N = N; J.H = H; J.dk = dk; J.dv = dv; J.cu = cu;
-    J.q = q; J.k = k; J.v = v; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d; J.h0 = h0;
+    J.q = q; J.k = k; J.v = v; J.p = p; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d; J.h0 = h0;
     J.o = o; J.hT = hT; J.nthreads = nthreads;
     return run_pool(&J, fwd_worker);
 }
 
 int comba_oracle_bwd(int N, const int64_t *cu, int H, int dk, int dv,
-                     const double *q, const double *k, const double *v,
+                     const double *q, const double *k, const double *v, const double *p,
                      const double *alpha, const double *beta, const double *b, const double *d,
                      const double *h0, const double *dO, const double *dhT,
-                     double *dq, double *dk_, double *dv_, double *dalpha, double *dbeta,
+                     double *dq, double *dk_, double *dv_, double *dp, double *dalpha, double *dbeta,
                      double *db, double *dd, double *dh0, int nthreads, int variant)
 {
     job_t J;
     memset(&J, 0, sizeof(J));
     J.variant = variant;
     J.N = N; J.H = H; J.dk = dk; J.dv = dv; J.cu = cu;
-    J.q = q; J.k = k; J.v = v; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d; J.h0 = h0;
+    J.q = q; J.k = k; J.v = v; J.p = p; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d; J.h0 = h0;
     J.dO = dO; J.dhT = dhT;
-    J.dq = dq; J.dk_ = dk_; J.dv_ = dv_; J.dalpha = dalpha; J.dbeta = dbeta; J.dh0 = dh0;
+    J.dq = dq; J.dk_ = dk_; J.dv_ = dv_; J.dp = dp; J.dalpha = dalpha; J.dbeta = dbeta; J.dh0 = dh0;
+    if (p && !dp) return 1;
     J.nthreads = nthreads;
     J.db_part = (double *)calloc((size_t)N * H, sizeof(double));
     J.dd_part = (double *)calloc((size_t)N * H, sizeof(double));
@@ -374,7 +401,7 @@ int comba_oracle_bwd(int N, const int64_t *cu, int H, int dk, int dv,
 
 /*
  * One decode token for Bd independent (row, head) states, updated in place:
- * the same four lines as the forward, applied once.  q,k [Bd,H,dk], v,o
+ * the same four lines as the forward, applied once.  q,k,p [Bd,H,dk], v,o
  * [Bd,H,dv], alpha,beta [Bd,H], state [Bd,H,dk,dv].  Rows are the N of the
  * thread pool; the state is indexed by (row, head) like h0.
  */
@@ -391,16 +418,17 @@ static void *step_worker(void *arg)
         for (int u = J->tid; u < J->N * Hh; u += J->nthreads) {
             const int h = u % Hh;
             const double *kt = J->k + (size_t)u * dk, *qt = J->q + (size_t)u * dk, *vt = J->v + (size_t)u * dv;
+            const double *ft = fb_vec(J, (size_t)u * dk);
             double *Hs = J->hT + (size_t)u * dk * dv;
             const double a = J->alpha[u], be = J->beta[u];
             const double bt = (J->b ? J->b[h] : 1.0) * be * fb_scale(J, a);
             for (int j = 0; j < dv; ++j) x[j] = 0.0;
             for (int r = 0; r < dk; ++r)
-                for (int j = 0; j < dv; ++j) x[j] += Hs[(size_t)r * dv + j] * kt[r];
+                for (int j = 0; j < dv; ++j) x[j] += Hs[(size_t)r * dv + j] * ft[r];
             for (int j = 0; j < dv; ++j) e[j] = be * vt[j] - bt * x[j];
             for (int r = 0; r < dk; ++r)
                 for (int j = 0; j < dv; ++j) Hs[(size_t)r * dv + j] = a * Hs[(size_t)r * dv + j] + kt[r] * e[j];
-            for (int r = 0; r < dk; ++r) qn[r] = qt[r] - J->d[h] * kt[r];
+            for (int r = 0; r < dk; ++r) qn[r] = qt[r] - J->d[h] * ft[r];
             double *ot = J->o + (size_t)u * dv;
             for (int j = 0; j < dv; ++j) ot[j] = 0.0;
             for (int r = 0; r < dk; ++r)
@@ -412,7 +440,7 @@ static void *step_worker(void *arg)
 }
 
 int comba_oracle_step(int Bd, int H, int dk, int dv,
-                      const double *q, const double *k, const double *v,
+                      const double *q, const double *k, const double *v, const double *p,
                       const double *alpha, const double *beta, const double *b, const double *d,
                       double *state, double *o, int nthreads, int variant)
 {
@@ -420,7 +448,7 @@ int comba_oracle_step(int Bd, int H, int dk, int dv,
     memset(&J, 0, sizeof(J));
     J.variant = variant;
     J.N = Bd; J.H = H; J.dk = dk; J.dv = dv;
-    J.q = q; J.k = k; J.v = v; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d;
+    J.q = q; J.k = k; J.v = v; J.p = p; J.alpha = alpha; J.beta = beta; J.b = b; J.d = d;
     J.hT = state; J.o = o; J.nthreads = nthreads;
     return run_pool(&J, step_worker);
 }
