@@ -59,9 +59,10 @@ def fwd_flops_per_token_head(C=64, dk=128, dv=128):
 # the tile products the kernel must form and the tensors it must read or write
 # once.  Forward saves the backward's factors (M, Atilde^T, E).
 
-def stage_model(dk, dv, slots, H, N, save=True, tc=True):
+def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False):
     """`tc`: the tcgen05 path (bf16, d=128), whose reverse scan reads Atilde itself, so
-    the forward saves M but no Atilde^T."""
+    the forward saves M but no Atilde^T.  `pk`: Comba-pk feedback vectors P, read by prep and
+    by the local gradients, which also write dP."""
     C, es, f4 = 64, 2, 4
     P = slots * H
     at = save and not tc
@@ -79,6 +80,9 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True):
     m["bwd_local"] = dict(flops=P * (2 * C * C * dk * 9 + 2 * C * dk * dv * 4 + 2 * C * C * dv * 4 + 4 * C ** 3),
                           bytes=P * (C * (2 * dk + 2 * dv) * es + C * dv * es + 2 * dv * dk * es + C * C * es
                                      + 3 * C * f4 + C * (2 * dk + dv) * es + 2 * C * f4))
+    if pk:
+        m["prep"]["bytes"] += P * C * dk * es
+        m["bwd_local"]["bytes"] += P * 2 * C * dk * es
     m["chunk_map"] = dict(flops=0, bytes=slots * 16 + (N + 1) * 8)
     m["output_E"] = dict(flops=0, bytes=0)
     m["reduce"] = dict(flops=0, bytes=P * 8 + 8 * H)
@@ -110,9 +114,9 @@ def sources_hash(files):
     return m.hexdigest()[:16]
 
 
-def captured_traffic(stage, units, dk, dv, dtype="bf16"):
+def captured_traffic(stage, units, dk, dv, dtype="bf16", tc=True):
     entry = CAPTURED_TRAFFIC.get(stage)
-    if entry is None or dk != 128 or dv != 128 or dtype != "bf16":
+    if entry is None or not tc or dk != 128 or dv != 128 or dtype != "bf16":
         return None, None
     kernel, per_unit, files, digest = entry
     if sources_hash(files) != digest:
@@ -267,9 +271,10 @@ def dist_init(world, local, backend):
 
 # -------------------------------------------------------- CPU oracle timing
 
-def oracle_sample(w, rows, heads, tokens):
+def oracle_sample(w, rows, heads, tokens, p=None, variant="splr"):
     """Bounded slice of a workload: batch rows `rows`, heads, first `tokens` tokens (a packed
-    workload: the first `tokens` tokens of the packed stream, its sequences cut there)."""
+    workload: the first `tokens` tokens of the packed stream, its sequences cut there), with the
+    Comba-pk feedback vectors `p` (shaped like k) when given."""
     if w.cu_seqlens is not None:
         sl = (slice(0, tokens), slice(heads[0], heads[1]))
         cu = np.asarray(w.cu_seqlens, np.int64)
@@ -288,19 +293,20 @@ def oracle_sample(w, rows, heads, tokens):
     return dict(q=np.ascontiguousarray(w.q[sl]), k=np.ascontiguousarray(w.k[sl]), v=np.ascontiguousarray(w.v[sl]),
                 alpha=np.ascontiguousarray(w.alpha[sl]), beta=np.ascontiguousarray(w.beta[sl]),
                 b=None if w.b is None else w.b[heads[0]:heads[1]], d=w.d[heads[0]:heads[1]], h0=st(w.h0),
-                dO=np.ascontiguousarray(w.dO[sl]), dhT=st(w.dhT), cu_seqlens=cu)
+                dO=np.ascontiguousarray(w.dO[sl]), dhT=st(w.dhT), cu_seqlens=cu,
+                p=None if p is None else np.ascontiguousarray(p[sl]), variant=variant)
 
 
 def time_oracle_step(s):
     import oracle
     t0 = time.perf_counter()
-    oracle.fwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], h0=s["h0"], cu_seqlens=s["cu_seqlens"])
-    oracle.bwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], s["dO"], h0=s["h0"], dhT=s["dhT"],
-               cu_seqlens=s["cu_seqlens"])
+    kw = dict(cu_seqlens=s["cu_seqlens"], p=s["p"], variant=s["variant"])
+    oracle.fwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], h0=s["h0"], **kw)
+    oracle.bwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], s["dO"], h0=s["h0"], dhT=s["dhT"], **kw)
     return time.perf_counter() - t0
 
 
-def cpu_baseline(w, target_s=12.0):
+def cpu_baseline(w, target_s=12.0, p=None, variant="splr"):
     """The oracle as it stands on this host's cores: fwd+bwd over all heads of a growing
     sample (token prefix of batch row 0, then whole batch rows) until about `target_s`
     seconds of wall time or the whole workload."""
@@ -311,7 +317,7 @@ def cpu_baseline(w, target_s=12.0):
         B, T, H = w.q.shape[0], w.q.shape[1], w.q.shape[2]
     rows, tokens = 1, min(T, 256)
     while True:
-        s = oracle_sample(w, (0, rows), (0, H), tokens)
+        s = oracle_sample(w, (0, rows), (0, H), tokens, p=p, variant=variant)
         dt = time_oracle_step(s)
         if dt >= target_s or (tokens >= T and rows >= B):
             break
@@ -331,11 +337,13 @@ def run_ours(args, world, rank, local):
     import torch
     dist = dist_init(world, local, "nccl")
     torch.cuda.set_device(local)
-    from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, inputs, shard
+    from paper_2506_02475_gb300 import (comba_chunk_bwd, comba_chunk_bwd_pk, comba_chunk_fwd, comba_chunk_fwd_pk,
+                                        inputs, shard)
     from paper_2506_02475_gb300 import binding
 
     peaks, peak_src = load_peaks()
     iplr = args.variant == "iplr"
+    pk = args.variant == "pk"   # Comba-pk feedback vectors (runs the mma.sync kernels)
     # weak scaling: each rank owns its own batch of sequences (same parameters, own data)
     w = inputs.make(args.workload, seed_offset=shard.rank_seed_offset(rank))
     dev = torch.device("cuda", local)
@@ -347,10 +355,13 @@ def run_ours(args, world, rank, local):
     hin = dict(q=host(w.q, tdt), k=host(w.k, tdt), v=host(w.v, tdt), alpha=host(w.alpha, torch.float32),
                beta=host(w.beta, torch.float32), d=host(w.d, torch.float32), b=host(w.b, torch.float32),
                h0=host(w.h0, torch.float32), dO=host(w.dO, tdt), dhT=host(w.dhT, torch.float32))
+    p_np = inputs.feedback_vectors(w.k, w.dtype, seed_offset=shard.rank_seed_offset(rank)) if pk else None
+    if pk:
+        hin["p"] = host(p_np, tdt)
     cu = None if w.cu_seqlens is None else torch.from_numpy(w.cu_seqlens.astype(np.int32)).to(dev)
     din = {k: (None if v is None else v.to(dev)) for k, v in hin.items()}
     q = din["q"]
-    ws_bytes = binding.comba_workspace_size(q, din["v"], cu, backward=True)
+    ws_bytes = binding.comba_workspace_size(q, din["v"], cu, backward=True, flags=binding.COMBA_PK if pk else 0)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
     N = w.num_seqs
     H, dk, dv = w.H, w.dk, w.dv
@@ -360,6 +371,8 @@ def run_ours(args, world, rank, local):
              "dalpha": torch.empty_like(din["alpha"]), "dbeta": torch.empty_like(din["beta"]),
              "dd": torch.empty_like(din["d"]), "db": torch.empty((H,), dtype=torch.float32, device=dev),
              "dh0": torch.empty((N, H, dk, dv), dtype=torch.float32, device=dev)}
+    if pk:
+        grads["dp"] = torch.empty_like(q)
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
 
     ev_f = [torch.cuda.Event(enable_timing=True) for _ in range(len(FWD_STAGES) + 1)]
@@ -370,13 +383,26 @@ def run_ours(args, world, rank, local):
     hf = [e.cuda_event for e in ev_f]
     hb = [e.cuda_event for e in ev_b]
 
+    def fwd_call(t, o_, hT_, events=None):
+        kw = dict(b=t["b"], h0=t["h0"], cu_seqlens=cu, o=o_, hT=hT_, workspace=ws, stage_events=events,
+                  save_factors=True, iplr=iplr)
+        if pk:
+            comba_chunk_fwd_pk(t["q"], t["k"], t["v"], t["p"], t["alpha"], t["beta"], t["d"], **kw)
+        else:
+            comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], **kw)
+
+    def bwd_call(t, out_, events=None):
+        kw = dict(b=t["b"], h0=t["h0"], dhT=t["dhT"], cu_seqlens=cu, out=out_, workspace=ws, stage_events=events,
+                  reuse_factors=True, iplr=iplr)
+        if pk:
+            comba_chunk_bwd_pk(t["q"], t["k"], t["v"], t["p"], t["alpha"], t["beta"], t["d"], t["dO"], **kw)
+        else:
+            comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], **kw)
+
     def step(t, events=True):
         # training step: the forward keeps the backward's chunk factors, the backward reuses them
-        comba_chunk_fwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], b=t["b"], h0=t["h0"], cu_seqlens=cu,
-                        o=o, hT=hT, workspace=ws, stage_events=hf if events else None, save_factors=True, iplr=iplr)
-        comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
-                        dhT=t["dhT"], cu_seqlens=cu, out=grads, workspace=ws, stage_events=hb if events else None,
-                        reuse_factors=True, iplr=iplr)
+        fwd_call(t, o, hT, hf if events else None)
+        bwd_call(t, grads, hb if events else None)
 
     for _ in range(args.warmup):
         flush.zero_()
@@ -419,14 +445,12 @@ def run_ours(args, world, rank, local):
 
     # ---- dominant kernel and its roofline
     slots = (tokens // 64 + N) if w.cu_seqlens is not None else w.q.shape[0] * ((w.q.shape[1] + 63) // 64)
-    model = stage_model(dk, dv, slots, H, N, tc=(w.dtype == "bf16" and dk == 128 and dv == 128))
-    per_kind = {}
-    for (phase, s), v in stage_ms.items():
-        per_kind.setdefault(s, [0.0, 0])
-        per_kind[s][0] += v
-        per_kind[s][1] += args.steps
-    dom = max(per_kind, key=lambda s: per_kind[s][0])
-    launch_ms = per_kind[dom][0] / per_kind[dom][1]
+    tc = w.dtype == "bf16" and dk == 128 and dv == 128
+    model = stage_model(dk, dv, slots, H, N, tc=tc, pk=pk)
+    # the dominant launch: the (phase, stage) with the most time (a stage the backward skips
+    # because it reuses the forward's factors is not averaged with its empty slot)
+    dom_phase, dom = max(stage_ms, key=lambda ps: stage_ms[ps])
+    launch_ms = stage_ms[(dom_phase, dom)] / args.steps
     mdl = model[dom]
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
     ai = mdl["flops"] / max(mdl["bytes"], 1)
@@ -437,7 +461,8 @@ def run_ours(args, world, rank, local):
         ach = mdl["bytes"] / (launch_ms / 1e3) / 1e9
         roof = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    traffic, kname = captured_traffic(dom, slots * H, dk, dv, w.dtype)
+    # captured figures are for the kernels without Comba-pk feedback vectors
+    traffic, kname = captured_traffic(dom, slots * H, dk, dv, w.dtype, tc=tc and not pk)
     roof.update({"kernel": kname or dom, "stage": dom, "launch_ms": launch_ms, "algorithmic_flops": mdl["flops"],
                  "algorithmic_bytes": mdl["bytes"], "traffic": traffic,
                  "traffic_source": "ncu capture of the 340M-shape step, scaled by units" if traffic else None,
@@ -477,12 +502,8 @@ def run_ours(args, world, rank, local):
             comp.wait_event(ev["uploaded"][j])
             if i >= 2:
                 comp.wait_event(ev["downloaded"][j])          # step i-2's results are on the host
-            comba_chunk_fwd(dbuf["q"], dbuf["k"], dbuf["v"], dbuf["alpha"], dbuf["beta"], dbuf["d"], b=dbuf["b"],
-                            h0=dbuf["h0"], cu_seqlens=cu, o=douts["o"], hT=douts["hT"], workspace=ws,
-                            save_factors=True, iplr=iplr)
-            comba_chunk_bwd(dbuf["q"], dbuf["k"], dbuf["v"], dbuf["alpha"], dbuf["beta"], dbuf["d"], dbuf["dO"],
-                            b=dbuf["b"], h0=dbuf["h0"], dhT=dbuf["dhT"], cu_seqlens=cu,
-                            out={k: douts[k] for k in grads}, workspace=ws, reuse_factors=True, iplr=iplr)
+            fwd_call(dbuf, douts["o"], douts["hT"])
+            bwd_call(dbuf, {k: douts[k] for k in grads})
             ev["consumed"][j].record(comp)
             ev["computed"][j].record(comp)
             with torch.cuda.stream(down):
@@ -511,7 +532,9 @@ def run_ours(args, world, rank, local):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w)
+        cpu = cpu_baseline(w, p=p_np, variant="splr" if pk else args.variant)
+        if pk:
+            cpu["sample"] = "Comba-pk " + cpu["sample"]
 
     if rank == 0:
         line = {
@@ -822,7 +845,8 @@ def run_reference(args, world, rank, local):
     H = w.H
     total = int(w.q.shape[0] if w.cu_seqlens is not None else w.q.shape[1])   # tokens of batch row 0 / the pack
     tokens = min(total, args.reference_tokens)
-    s = oracle_sample(w, (0, 1), (0, H), tokens)
+    pv = inputs.feedback_vectors(w.k, w.dtype) if args.variant == "pk" else None
+    s = oracle_sample(w, (0, 1), (0, H), tokens, p=pv, variant="splr" if args.variant == "pk" else args.variant)
     for _ in range(args.warmup):
         time_oracle_step(s)
     dts = [time_oracle_step(s) for _ in range(args.steps)]
@@ -833,7 +857,7 @@ def run_reference(args, world, rank, local):
         "metric": METRIC, "impl": "reference", "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": f"{args.workload}: " + workload_desc(w),
+        "config": {"workload": f"{args.workload}: " + workload_desc(w), "variant": args.variant,
                    "sample": f"batch row 0, all {H} heads, first {tokens} tokens per step"},
         "tflops": flops / dt / 1e12,
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.default_threads(), "kind": "oracle",
@@ -852,8 +876,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--gated", action="store_true",
                     help="raw q, k and gate pre-activations through the gate and normalisation prologue")
-    ap.add_argument("--variant", default="splr", choices=["splr", "iplr"],
-                    help="state transition: Comba (alpha - btilde k k^T) or Comba-iplr alpha (I - 2 btilde k k^T)")
+    ap.add_argument("--variant", default="splr", choices=["splr", "iplr", "pk"],
+                    help="state transition: Comba (alpha - btilde k k^T), Comba-iplr alpha (I - 2 btilde k k^T), "
+                         "or Comba-pk (alpha - btilde p k^T with per-token feedback vectors p)")
     ap.add_argument("--reference-tokens", type=int, default=512)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":

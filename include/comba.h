@@ -72,7 +72,7 @@ typedef struct {
     const int32_t *cu_seqlens;  /* device int32 [N+1] or NULL                     */
     comba_dtype_t dtype;        /* storage type of q, k, v, o and their grads     */
     int chunk;                  /* chunk length; must be 64                       */
-    int flags;                  /* COMBA_SAVE_FACTORS / COMBA_REUSE_FACTORS, | COMBA_IPLR */
+    int flags;                  /* COMBA_SAVE_FACTORS / COMBA_REUSE_FACTORS, | COMBA_IPLR, COMBA_GATED, COMBA_PK */
     /* Optional instrumentation (NULL / 0 = off).  Caller-created cudaEvent_t
      * handles recorded on `stream` at kernel boundaries: comba_chunk_fwd
      * records COMBA_FWD_EVENTS of them (before chunk map, prep, state scan,
@@ -158,6 +158,48 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t *shape,
                                      void *workspace, size_t workspace_bytes, void *stream);
 
 /*
+ * Comba-pk (appendix B.3, the "p" form of the recurrence): a per-token feedback
+ * vector p_t, shaped like k_t, is read back from the state and corrects the query,
+ * while k_t still writes the state:
+ *     x_t = H_{t-1}^T p_t,  e_t = beta_t v_t - btilde_t x_t,
+ *     H_t = alpha_t H_{t-1} + k_t e_t^T,  o_t = H_t^T (q_t - d p_t)
+ * (transition alpha_t I - btilde_t p_t k_t^T on S = H^T; p = k is the form above,
+ * p = b k with b = 1 the paper's way of folding b into p).  In the chunk form the
+ * Gram inside the inverse becomes P K^T and W = M Diag(btilde gamma_{r-1}) P.  The
+ * shape passed to the pk calls and to comba_workspace_size must carry COMBA_PK (the
+ * workspace then also holds q - d p).  The local-gradient kernel of these calls is
+ * the mma.sync one for every shape.
+ */
+#define COMBA_PK 16
+
+/*
+ * The pk forward: as comba_chunk_fwd plus p [B,T,H,dk] (storage type, required).
+ * shape->flags must contain COMBA_PK and may add COMBA_SAVE_FACTORS and COMBA_IPLR.
+ */
+comba_status_t comba_chunk_fwd_pk(const comba_shape_t *shape,
+                                  const void *q, const void *k, const void *v, const void *p,
+                                  const float *alpha, const float *beta,
+                                  const float *b, const float *d, const float *h0,
+                                  void *o, float *hT,
+                                  void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * The pk backward: as comba_chunk_bwd plus p and its gradient dp [B,T,H,dk]
+ * (storage type, written).  dk then holds only the gradient through the state
+ * write; dd = -sum_t p_t . dq_t.  shape->flags must contain COMBA_PK and may add
+ * COMBA_REUSE_FACTORS (after a pk forward with COMBA_SAVE_FACTORS on the same
+ * workspace) and COMBA_IPLR.
+ */
+comba_status_t comba_chunk_bwd_pk(const comba_shape_t *shape,
+                                  const void *q, const void *k, const void *v, const void *p,
+                                  const float *alpha, const float *beta,
+                                  const float *b, const float *d, const float *h0,
+                                  const void *dO, const float *dhT,
+                                  void *dq, void *dk, void *dv, void *dp,
+                                  float *dalpha, float *dbeta, float *db, float *dd, float *dh0,
+                                  void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * Bytes of device workspace needed by comba_chunk_fwd (backward = 0) or
  * comba_chunk_bwd (backward = 1) for this shape.  Returns 0 for an invalid
  * shape.  The bound covers any cu_seqlens with the given T and num_seqs.
@@ -229,6 +271,18 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
                                     const float *alpha, const float *beta,
                                     const float *b, const float *d,
                                     float *state, void *o, int flags, void *stream);
+
+/*
+ * One Comba-pk decode token: as comba_recurrent_step with the feedback vector
+ * p [Bd,H,dk] (storage type, required) in place of k where the state is read
+ * back and in the correction: x = H^T p, y = H^T (q - d p),
+ * o = alpha y + e (k . (q - d p)), H <- alpha H + k e^T.
+ */
+comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtype_t dtype,
+                                       const void *q, const void *k, const void *v, const void *p,
+                                       const float *alpha, const float *beta,
+                                       const float *b, const float *d,
+                                       float *state, void *o, int flags, void *stream);
 
 /*
  * Forward without a caller workspace, for callers that may not allocate

@@ -9,9 +9,12 @@ from .binding import (  # noqa: F401
     CombaError,
     comba_chunk_bwd,
     comba_chunk_bwd_gated,
+    comba_chunk_bwd_pk,
     comba_chunk_fwd,
     comba_chunk_fwd_gated,
+    comba_chunk_fwd_pk,
     comba_recurrent_step,
+    comba_recurrent_step_pk,
     comba_workspace_size,
     lib,
     library_path,

@@ -21,7 +21,7 @@ _lib = None
 _lock = threading.Lock()
 
 COMBA_F32, COMBA_BF16 = 0, 1
-COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS, COMBA_IPLR, COMBA_GATED = 1, 2, 4, 8
+COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS, COMBA_IPLR, COMBA_GATED, COMBA_PK = 1, 2, 4, 8, 16
 _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "workspace missing or too small",
            4: "CUDA error", 5: "device-side wait timed out"}
 
@@ -68,6 +68,12 @@ def lib():
         L.comba_chunk_fwd_gated.restype = I
         L.comba_chunk_bwd_gated.argtypes = [SP] + [P] * 12 + [P] * 10 + [P, Z, P]
         L.comba_chunk_bwd_gated.restype = I
+        L.comba_chunk_fwd_pk.argtypes = [SP] + [P] * 11 + [P, Z, P]
+        L.comba_chunk_fwd_pk.restype = I
+        L.comba_chunk_bwd_pk.argtypes = [SP] + [P] * 11 + [P] * 9 + [P, Z, P]
+        L.comba_chunk_bwd_pk.restype = I
+        L.comba_recurrent_step_pk.argtypes = [I, I, I, I, I] + [P] * 10 + [I, P]
+        L.comba_recurrent_step_pk.restype = I
         L.comba_status_string.argtypes = [I]
         L.comba_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -135,8 +141,9 @@ def make_shape(q, v, cu_seqlens=None, stage_events=None, flags=0):
     return s
 
 
-def comba_workspace_size(q, v, cu_seqlens=None, backward=False) -> int:
-    return int(lib().comba_workspace_size(ctypes.byref(make_shape(q, v, cu_seqlens)), int(bool(backward))))
+def comba_workspace_size(q, v, cu_seqlens=None, backward=False, flags=0) -> int:
+    return int(lib().comba_workspace_size(ctypes.byref(make_shape(q, v, cu_seqlens, None, flags)),
+                                          int(bool(backward))))
 
 
 def _workspace(nbytes, device, workspace):
@@ -329,3 +336,92 @@ def comba_chunk_bwd_gated(q, k, v, g_alpha, g_beta, a, c, b_raw, d, dO, h0=None,
     if st != 0:
         raise CombaError("comba_chunk_bwd_gated", st)
     return g
+
+
+def comba_chunk_fwd_pk(q, k, v, p, alpha, beta, d, b=None, h0=None, cu_seqlens=None, output_final_state=False,
+                       o=None, hT=None, workspace=None, stream=None, stage_events=None, save_factors=False,
+                       iplr=False):
+    """Comba-pk forward: feedback vectors ``p`` (shaped like k) read back from the state and used in
+    the correction q - d p, while k writes the state.  Returns ``(o, hT)``."""
+    N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
+    _check("p", p, q.dtype, q.shape, q.device)
+    flags = COMBA_PK | (COMBA_SAVE_FACTORS if save_factors else 0) | (COMBA_IPLR if iplr else 0)
+    shape = make_shape(q, v, cu_seqlens, stage_events, flags)
+    L = lib()
+    nbytes = L.comba_workspace_size(ctypes.byref(shape), 1 if save_factors else 0)
+    if nbytes == 0:
+        raise CombaError("comba_workspace_size", 1)
+    ws = _workspace(nbytes, q.device, workspace)
+    if o is None:
+        o = torch.empty_like(v)
+    if hT is None and output_final_state:
+        hT = torch.empty((N, H, dk, dv), dtype=torch.float32, device=q.device)
+    st = L.comba_chunk_fwd_pk(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(p), _ptr(alpha), _ptr(beta),
+                              _ptr(b), _ptr(d), _ptr(h0), _ptr(o), _ptr(hT), _ptr(ws), ws.numel() * ws.element_size(),
+                              _stream(stream))
+    if st != 0:
+        raise CombaError("comba_chunk_fwd_pk", st)
+    return o, hT
+
+
+def comba_chunk_bwd_pk(q, k, v, p, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_seqlens=None, want_dh0=True,
+                       want_db=True, out=None, workspace=None, stream=None, stage_events=None, reuse_factors=False,
+                       iplr=False):
+    """Comba-pk backward.  Returns a dict with dq, dk, dv, dp, dalpha, dbeta, dd, db, dh0."""
+    N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
+    _check("p", p, q.dtype, q.shape, q.device)
+    _check("dO", dO, q.dtype, v.shape, q.device)
+    _check("dhT", dhT, torch.float32, (N, H, dk, dv), q.device)
+    if reuse_factors and workspace is None:
+        raise ValueError("reuse_factors=True needs the workspace of the saving forward call")
+    flags = COMBA_PK | (COMBA_REUSE_FACTORS if reuse_factors else 0) | (COMBA_IPLR if iplr else 0)
+    shape = make_shape(q, v, cu_seqlens, stage_events, flags)
+    L = lib()
+    nbytes = L.comba_workspace_size(ctypes.byref(shape), 1)
+    if nbytes == 0:
+        raise CombaError("comba_workspace_size", 1)
+    ws = _workspace(nbytes, q.device, workspace)
+    g = out if out is not None else {}
+    g.setdefault("dq", torch.empty_like(q))
+    g.setdefault("dk", torch.empty_like(k))
+    g.setdefault("dv", torch.empty_like(v))
+    g.setdefault("dp", torch.empty_like(p))
+    g.setdefault("dalpha", torch.empty_like(alpha))
+    g.setdefault("dbeta", torch.empty_like(beta))
+    g.setdefault("dd", torch.empty_like(d))
+    if want_db:
+        g.setdefault("db", torch.empty((H,), dtype=torch.float32, device=q.device))
+    if want_dh0:
+        g.setdefault("dh0", torch.empty((N, H, dk, dv), dtype=torch.float32, device=q.device))
+    st = L.comba_chunk_bwd_pk(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(p), _ptr(alpha), _ptr(beta),
+                              _ptr(b), _ptr(d), _ptr(h0), _ptr(dO), _ptr(dhT), _ptr(g["dq"]), _ptr(g["dk"]),
+                              _ptr(g["dv"]), _ptr(g["dp"]), _ptr(g["dalpha"]), _ptr(g["dbeta"]), _ptr(g.get("db")),
+                              _ptr(g["dd"]), _ptr(g.get("dh0")), _ptr(ws), ws.numel() * ws.element_size(),
+                              _stream(stream))
+    if st != 0:
+        raise CombaError("comba_chunk_bwd_pk", st)
+    return g
+
+
+def comba_recurrent_step_pk(q, k, v, p, alpha, beta, d, state, b=None, o=None, stream=None, iplr=False):
+    """One Comba-pk decode token (feedback vector ``p`` [Bd,H,dk]); ``state`` is updated in place."""
+    Bd, H, dk = q.shape
+    dv = v.shape[-1]
+    dev = q.device
+    _check("q", q, device=dev)
+    _check("k", k, q.dtype, q.shape, dev)
+    _check("p", p, q.dtype, q.shape, dev)
+    _check("v", v, q.dtype, (Bd, H, dv), dev)
+    _check("alpha", alpha, torch.float32, (Bd, H), dev)
+    _check("beta", beta, torch.float32, (Bd, H), dev)
+    _check("b", b, torch.float32, (H,), dev)
+    _check("d", d, torch.float32, (H,), dev)
+    _check("state", state, torch.float32, (Bd, H, dk, dv), dev)
+    if o is None:
+        o = torch.empty_like(v)
+    st = lib().comba_recurrent_step_pk(Bd, H, dk, dv, _dtype_code(q), _ptr(q), _ptr(k), _ptr(v), _ptr(p),
+                                       _ptr(alpha), _ptr(beta), _ptr(b), _ptr(d), _ptr(state), _ptr(o),
+                                       COMBA_IPLR if iplr else 0, _stream(stream))
+    if st != 0:
+        raise CombaError("comba_recurrent_step_pk", st)
+    return o

@@ -20,6 +20,8 @@ struct Layout {
     // gate and normalisation prologue (COMBA_GATED): its outputs, and the backward's gradients
     // w.r.t. them with the per-row contributions to da, dc
     size_t qh, kh, ga, gb, bg, dqh, dkh, dal, dbe, dbi, dar, dcr, dpa, dpc;
+    // Comba-pk (COMBA_PK): the corrected queries q - d p and the zero d the chunk kernels then see
+    size_t qt, dz;
     size_t total;
     int slots;
 };
@@ -93,6 +95,10 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
             L.dpc = take(parts * sizeof(float));
         }
     }
+    if (s->flags & COMBA_PK) {
+        L.qt = take((size_t)ttot * s->H * dk * es);
+        L.dz = take((size_t)s->H * sizeof(float));
+    }
     L.total = o;
     L.slots = (int)slots;
     *out = L;
@@ -104,12 +110,12 @@ comba_status_t check_smem(const comba_shape_t* s, int backward) {
     if (cudaGetDevice(&dev) != cudaSuccess) return COMBA_ERR_CUDA;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
         return COMBA_ERR_CUDA;
-    const bool bf = s->dtype == COMBA_BF16;
+    const bool bf = s->dtype == COMBA_BF16, pk = (s->flags & COMBA_PK) != 0;
     for (int kern = 0; kern < 3; ++kern)
-        if (comba::fwd_smem_bytes(kern, bf, s->dk, s->dv) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
+        if (comba::fwd_smem_bytes(kern, bf, s->dk, s->dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
     if (backward)
         for (int kern = 0; kern < 2; ++kern)
-            if (comba::bwd_smem_bytes(kern, bf, s->dk, s->dv) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
+            if (comba::bwd_smem_bytes(kern, bf, s->dk, s->dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
     return COMBA_OK;
 }
 
@@ -176,15 +182,24 @@ size_t comba_workspace_size(const comba_shape_t* shape, int backward) {
 
 namespace {
 
+// Comba-pk arguments of the chunk kernels: feedback vectors, the d of the correction applied
+// to q beforehand, and dL/dp (backward).
+struct PkArgs {
+    const void* p = nullptr;
+    const float* d = nullptr;
+    void* dp = nullptr;
+};
+
 // Launch the forward on validated arguments (L from plan(); shape checks done).
 comba_status_t forward_run(const comba_shape_t* shape, const Layout& L, void* workspace, const void* q, const void* k,
                            const void* v, const float* alpha, const float* beta, const float* b, const float* d,
-                           const float* h0, void* o, float* hT, bool save, cudaStream_t s) {
+                           const float* h0, void* o, float* hT, bool save, cudaStream_t s, PkArgs pk = {}) {
     comba_status_t st;
     if ((st = check_smem(shape, 0)) != COMBA_OK) return st;
     ChunkParams p{};
     fill_common(p, shape, L, workspace, save);
     p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
+    p.p = pk.p; p.d_fb = pk.d;
     p.o = o; p.hT = hT;
     comba::mark(p, 0, s);
     if (comba::launch_chunk_map(p, s) != cudaSuccess) return COMBA_ERR_CUDA;
@@ -196,12 +211,13 @@ comba_status_t backward_run(const comba_shape_t* shape, const Layout& L, void* w
                             const void* k, const void* v, const float* alpha, const float* beta, const float* b,
                             const float* d, const float* h0, const void* dO, const float* dhT, void* dq, void* dk,
                             void* dv, float* dalpha, float* dbeta, float* db, float* dd, float* dh0, bool reuse,
-                            cudaStream_t s) {
+                            cudaStream_t s, PkArgs pk = {}) {
     comba_status_t st;
     if ((st = check_smem(shape, 1)) != COMBA_OK) return st;
     ChunkParams p{};
     fill_common(p, shape, L, workspace, true);
     p.q = q; p.k = k; p.v = v; p.alpha = alpha; p.beta = beta; p.b = b; p.d = d; p.h0 = h0;
+    p.p = pk.p; p.d_fb = pk.d; p.dpp = pk.dp;
     p.dO = dO; p.dhT = dhT; p.dq = dq; p.dkk = dk; p.dvv = dv;
     p.dalpha = dalpha; p.dbeta = dbeta; p.db = db; p.dd = dd; p.dh0 = dh0;
     const bool bf = shape->dtype == COMBA_BF16;
@@ -341,6 +357,88 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t* shape, const void* q, 
     return COMBA_OK;
 }
 
+// Comba-pk: q - d p into the workspace and a zeroed d for the chunk kernels.
+static comba_status_t pk_prologue(const comba_shape_t* shape, const Layout& L, void* workspace, const void* q,
+                                  const void* p, const float* d, cudaStream_t s, void** qt, float** dz) {
+    char* w = static_cast<char*>(workspace);
+    *qt = w + L.qt;
+    *dz = reinterpret_cast<float*>(w + L.dz);
+    if (cudaMemsetAsync(*dz, 0, (size_t)shape->H * sizeof(float), s) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (comba::launch_pk_qtilde(q, p, d, *qt, (long long)shape->B * shape->T * shape->H, shape->H, shape->dk,
+                                shape->dtype == COMBA_BF16, s) != cudaSuccess)
+        return COMBA_ERR_CUDA;
+    return COMBA_OK;
+}
+
+comba_status_t comba_chunk_fwd_pk(const comba_shape_t* shape, const void* q, const void* k, const void* v,
+                                  const void* p, const float* alpha, const float* beta, const float* b,
+                                  const float* d, const float* h0, void* o, float* hT, void* workspace,
+                                  size_t workspace_bytes, void* stream) {
+    Layout L;
+    const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
+    comba_status_t st = plan(shape, save ? 1 : 0, &L);
+    if (st != COMBA_OK) return st;
+    if (!(shape->flags & COMBA_PK) || (shape->flags & ~(COMBA_PK | COMBA_SAVE_FACTORS | COMBA_IPLR)))
+        return COMBA_ERR_INVALID_ARG;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(p); COMBA_REQUIRE(alpha);
+    COMBA_REQUIRE(beta); COMBA_REQUIRE(d); COMBA_REQUIRE(o);
+    COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
+    if (shape->stage_events && shape->num_stage_events < COMBA_FWD_EVENTS) return COMBA_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    void* qt;
+    float* dz;
+    if ((st = pk_prologue(shape, L, workspace, q, p, d, s, &qt, &dz)) != COMBA_OK) return st;
+    PkArgs pk;
+    pk.p = p; pk.d = d;
+    return forward_run(shape, L, workspace, qt, k, v, alpha, beta, b, dz, h0, o, hT, save, s, pk);
+}
+
+comba_status_t comba_chunk_bwd_pk(const comba_shape_t* shape, const void* q, const void* k, const void* v,
+                                  const void* p, const float* alpha, const float* beta, const float* b,
+                                  const float* d, const float* h0, const void* dO, const float* dhT, void* dq,
+                                  void* dk, void* dv, void* dp, float* dalpha, float* dbeta, float* db, float* dd,
+                                  float* dh0, void* workspace, size_t workspace_bytes, void* stream) {
+    Layout L;
+    comba_status_t st = plan(shape, 1, &L);
+    if (st != COMBA_OK) return st;
+    if (!(shape->flags & COMBA_PK) || (shape->flags & ~(COMBA_PK | COMBA_REUSE_FACTORS | COMBA_IPLR)))
+        return COMBA_ERR_INVALID_ARG;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(p); COMBA_REQUIRE(alpha);
+    COMBA_REQUIRE(beta); COMBA_REQUIRE(d); COMBA_REQUIRE(dO);
+    COMBA_REQUIRE(dq); COMBA_REQUIRE(dk); COMBA_REQUIRE(dv); COMBA_REQUIRE(dp); COMBA_REQUIRE(dalpha);
+    COMBA_REQUIRE(dbeta); COMBA_REQUIRE(dd);
+    COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(dhT); COMBA_OPTIONAL(db); COMBA_OPTIONAL(dh0);
+    if (shape->stage_events && shape->num_stage_events < COMBA_BWD_EVENTS) return COMBA_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    void* qt;
+    float* dz;
+    if ((st = pk_prologue(shape, L, workspace, q, p, d, s, &qt, &dz)) != COMBA_OK) return st;
+    PkArgs pk;
+    pk.p = p; pk.d = d; pk.dp = dp;
+    return backward_run(shape, L, workspace, qt, k, v, alpha, beta, b, dz, h0, dO, dhT, dq, dk, dv, dalpha, dbeta, db,
+                        dd, dh0, (shape->flags & COMBA_REUSE_FACTORS) != 0, s, pk);
+}
+
+comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtype_t dtype, const void* q,
+                                       const void* k, const void* v, const void* p, const float* alpha,
+                                       const float* beta, const float* b, const float* d, float* state, void* o,
+                                       int flags, void* stream) {
+    if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
+    if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
+    if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
+    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128)) return COMBA_ERR_UNSUPPORTED;
+    if ((long long)Bd * H * (dv / 32) >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
+    COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(p); COMBA_REQUIRE(alpha);
+    COMBA_REQUIRE(beta); COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
+    COMBA_OPTIONAL(b);
+    if (comba::launch_recurrent_step(Bd, H, dk, dv, dtype == COMBA_BF16, q, k, v, p, alpha, beta, b, d, state, o,
+                                     (flags & COMBA_IPLR) != 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return COMBA_ERR_CUDA;
+    return COMBA_OK;
+}
+
 comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t dtype, const void* q,
                                     const void* k, const void* v, const float* alpha, const float* beta,
                                     const float* b, const float* d, float* state, void* o, int flags,
@@ -353,8 +451,8 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
     COMBA_OPTIONAL(b);
-    if (comba::launch_recurrent_step(Bd, H, dk, dv, dtype == COMBA_BF16, q, k, v, alpha, beta, b, d, state, o,
-                                     (flags & COMBA_IPLR) != 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    if (comba::launch_recurrent_step(Bd, H, dk, dv, dtype == COMBA_BF16, q, k, v, nullptr, alpha, beta, b, d, state,
+                                     o, (flags & COMBA_IPLR) != 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
         return COMBA_ERR_CUDA;
     return COMBA_OK;
 }

@@ -183,7 +183,10 @@ __device__ __forceinline__ void frag_rowdot(const float (&acc)[NT][4], float& s0
     s1 = quad_sum(s1);
 }
 
-template <typename T, int DK, int DV>
+// PKV: Comba-pk feedback vectors P (p.p).  They replace K as the left factor of the Gram
+// (A = strict_lower(Diag(btilde) Gamma- * P K^T)) and in W = M Diag(s) P, so the gradients of
+// those uses go to dp instead of dk, and the correction's share -d dq (d = p.d_fb) too.
+template <typename T, int DK, int DV, bool PKV>
 __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     using S = LocalSmem<T, DK, DV>;
     constexpr int NK = DK / 16, NV = DV / 16;   // n-tiles per warp (half the columns)
@@ -357,6 +360,15 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         frag_rowdot(t0r, s0, s1);
         put_rows(1, s0, s1);
     }
+    // Feedback vectors: K itself, or for Comba-pk P, loaded into the dH' tile (read for the
+    // last time above) under the remaining phase-A products.
+    T* sF = sK;
+    if constexpr (PKV) {
+        __syncthreads();
+        sF = sdH;
+        load_tile_async<T>(sF, PK, (const T*)p.p + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
+        cp_async_commit();
+    }
     {
         // dW = -dE H^T
         float tmp[NK][4];
@@ -398,17 +410,18 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         for (int t = 0; t < NV; ++t) { tv[t][0] *= ba; tv[t][1] *= ba; tv[t][2] *= bb; tv[t][3] *= bb; }
         frag_store<T, NV>(sDV, PV, m0, nv0, tv);
     }
-    __syncthreads();   // dO, E, dE, H, dH' no longer needed; dW complete
+    if constexpr (PKV) cp_async_wait<0>();
+    __syncthreads();   // dO, E, dE, H, dH' no longer needed; dW complete (and P landed)
 
     // ---------------- phase B: contractions over dk and the 64 x 64 algebra
     float gr[4][4], sq[4][4];
     zero(gr);
-    warp_gemm<true, true, 4>(gr, sK, PK, sK, PK, m0, nl0, DK);   // Gram K K^T
+    warp_gemm<true, true, 4>(gr, sF, PK, sK, PK, m0, nl0, DK);   // Gram P K^T (P = K unless pk)
     zero(sq);
     warp_gemm<true, true, 4>(sq, sQ, PK, sK, PK, m0, nl0, DK);   // Q~ K^T
     float mb[4][4];
     zero(mb);
-    warp_gemm<true, true, 4>(mb, sdW, PK, sK, PK, m0, nl0, DK);  // dW K^T
+    warp_gemm<true, true, 4>(mb, sdW, PK, sF, PK, m0, nl0, DK);  // dW P^T
     {
         float rs0 = 0.f, rs1 = 0.f;
         float cs[4][2];
@@ -482,27 +495,38 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
             }
     }
     __syncthreads();
+    // dp accumulator (Comba-pk only)
+    float acc_dp[PKV ? NK : 1][4];
+    if constexpr (PKV) zero(acc_dp);
     {
-        // dQ~ = dPhat K + Diag(gamma) dO H^T ; dq = dQ~ ; dd partial = -k . dQ~
+        // dQ~ = dPhat K + Diag(gamma) dO H^T ; dq = dQ~ ; dd partial = -p . dQ~ (p = k unless pk)
         warp_gemm<true, false, NK>(acc_dq, sdPh, PL, sK, PK, m0, nk0, 64);
 
         float t0r[NK][4];
+        const float dfb = PKV ? p.d_fb[h] : 0.f;
 #pragma unroll
         for (int t = 0; t < NK; ++t)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                t0r[t][i] = acc_dq[t][i] * to_f(sK[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
-                acc_dk[t][i] -= dh * acc_dq[t][i];
+                t0r[t][i] = acc_dq[t][i] * to_f(sF[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
+                if constexpr (PKV) acc_dp[t][i] -= dfb * acc_dq[t][i];
+                else acc_dk[t][i] -= dh * acc_dq[t][i];
             }
         float s0, s1;
         frag_rowdot(t0r, s0, s1);
         put_rows(6, s0, s1);
     }
     warp_gemm<false, false, NK>(acc_dk, sdPh, PL, sQ, PK, m0, nk0, 64);   // dPhat^T Q~
-    warp_gemm<true, false, NK>(acc_dk, sdG, PL, sK, PK, m0, nk0, 64);     // dG K
-    warp_gemm<false, false, NK>(acc_dk, sdG, PL, sK, PK, m0, nk0, 64);    // dG^T K
+    if constexpr (PKV) {
+        warp_gemm<true, false, NK>(acc_dp, sdG, PL, sK, PK, m0, nk0, 64);  // dG K: the Gram's left factor P
+        warp_gemm<false, false, NK>(acc_dk, sdG, PL, sF, PK, m0, nk0, 64); // dG^T P: its right factor K
+    } else {
+        warp_gemm<true, false, NK>(acc_dk, sdG, PL, sK, PK, m0, nk0, 64);  // dG K
+        warp_gemm<false, false, NK>(acc_dk, sdG, PL, sK, PK, m0, nk0, 64); // dG^T K
+    }
     {
-        // W path: M^T dW scaled by btilde gamma_{r-1}; its row dot with k feeds dbtilde and d g_{r-1}
+        // W path (W = M Diag(s) P): M^T dW scaled by btilde gamma_{r-1} goes to dp (dk unless pk); its
+        // row dot with p feeds dbtilde and d g_{r-1}
         float tmp[NK][4];
         zero(tmp);
         warp_gemm<false, false, NK>(tmp, sM, PL, sdW, PK, m0, nk0, 64);
@@ -512,8 +536,9 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         for (int t = 0; t < NK; ++t)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                t0r[t][i] = tmp[t][i] * to_f(sK[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
-                acc_dk[t][i] += (i < 2 ? wa : wb) * tmp[t][i];
+                t0r[t][i] = tmp[t][i] * to_f(sF[(m0 + frag_row(i)) * PK + nk0 + frag_col(t, i)]);
+                if constexpr (PKV) acc_dp[t][i] += (i < 2 ? wa : wb) * tmp[t][i];
+                else acc_dk[t][i] += (i < 2 ? wa : wb) * tmp[t][i];
             }
         float s0, s1;
         frag_rowdot(t0r, s0, s1);
@@ -524,6 +549,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     // then coalesced 16-byte copies to global memory
     frag_store<T, NK>(sQ, PK, m0, nk0, acc_dq);
     frag_store<T, NK>(sK, PK, m0, nk0, acc_dk);
+    if constexpr (PKV) frag_store<T, NK>(sF, PK, m0, nk0, acc_dp);
     __syncthreads();
     {
         constexpr int CK = DK / VE, CV = DV / VE;
@@ -535,6 +561,13 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
             const int r = e / CK, c = (e % CK) * VE;
             *reinterpret_cast<uint4*>(gq + r * sk + c) = *reinterpret_cast<const uint4*>(sQ + r * PK + c);
             *reinterpret_cast<uint4*>(gk + r * sk + c) = *reinterpret_cast<const uint4*>(sK + r * PK + c);
+        }
+        if constexpr (PKV) {
+            T* gp = (T*)p.dpp + (t0 * p.H + h) * DK;
+            for (int e = tid; e < L * CK; e += 256) {
+                const int r = e / CK, c = (e % CK) * VE;
+                *reinterpret_cast<uint4*>(gp + r * sk + c) = *reinterpret_cast<const uint4*>(sF + r * PK + c);
+            }
         }
         for (int e = tid; e < L * CV; e += 256) {
             const int r = e / CV, c = (e % CV) * VE;
@@ -642,10 +675,12 @@ template <typename T, int DK, int DV>
 static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     const size_t sm_prep = BPrepSmem<T, DK, DV>::bytes();
     const size_t sm_loc = LocalSmem<T, DK, DV>::bytes();
+    const bool pk = p.p != nullptr;
+    auto local = pk ? k_bwd_local<T, DK, DV, true> : k_bwd_local<T, DK, DV, false>;
     cudaError_t e;
     if ((e = cudaFuncSetAttribute(k_bwd_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
         return e;
-    if ((e = cudaFuncSetAttribute(k_bwd_local<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_loc)))
+    if ((e = cudaFuncSetAttribute(local, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_loc)))
         return e;
     const bool tcp = use_tc_path(sizeof(T) == 2, DK, DV);
     mark(p, ev0, s);
@@ -663,10 +698,12 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     a.x_mn = tcp ? 1 : 0;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)p.slots * p.H, s))) return e;
     mark(p, ev0 + 2, s);
-    if (tcp) {
+    if (tcp && !pk) {
         if ((e = launch_bwd_local_tc(p, s))) return e;
     } else if (p.slots > 0) {
-        k_bwd_local<T, DK, DV><<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
+        // the mma.sync local kernel also serves Comba-pk on the tcgen05 path: it reads the same
+        // row-major E, M and transposed chunk states
+        local<<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
     }
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 3, s);
@@ -688,9 +725,9 @@ cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int e
     return cudaErrorInvalidValue;
 }
 
-size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
+size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk) {
     if (kernel == 0 && use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(2);
-    if (kernel == 1 && use_tc_path(is_bf16, dk, dv)) return local_tc_smem_bytes();
+    if (kernel == 1 && use_tc_path(is_bf16, dk, dv) && !pk) return local_tc_smem_bytes();
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? BPrepSmem<T, DK, DV>::bytes() : LocalSmem<T, DK, DV>::bytes();
     if (is_bf16) {

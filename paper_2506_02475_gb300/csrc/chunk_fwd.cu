@@ -124,7 +124,8 @@ struct PrepSmem {
     static constexpr size_t OMW = align128(OT + sizeof(float) * 3 * 272);
     static constexpr size_t OMU = align128(OMW + sizeof(T) * 64 * PL);
     static constexpr size_t OF = align128(OMU + sizeof(T) * 64 * PL);  // G, Gm1, btilde, beta, s
-    static constexpr size_t bytes() { return OF + sizeof(float) * 64 * 5; }
+    static constexpr size_t OP = align128(OF + sizeof(float) * 64 * 5);  // Comba-pk feedback vectors P
+    static constexpr size_t bytes(bool pk = false) { return pk ? OP + sizeof(T) * 64 * PK : OF + sizeof(float) * 64 * 5; }
 };
 
 // Store a [rows x cols] product computed in 16-row m-tiles and 64-column passes.
@@ -171,8 +172,12 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     float* sBt = sG + 128;
     float* sBe = sG + 192;
     float* sS = sG + 256;
+    // feedback vectors: P for Comba-pk (Gram P K^T, W = M Diag P), else K itself
+    T* sF = p.p ? reinterpret_cast<T*>(smem + S::OP) : sK;
 
     load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    if (p.p)
+        load_tile_async<T>(sF, S::PK, (const T*)p.p + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
     load_tile_async<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
     cp_async_commit();
     if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
@@ -186,11 +191,12 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     __syncthreads();
     if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;   // Kbar row scale gamma_C / gamma_r
 
-    // Strictly-lower A = Diag(btilde) (gamma_{r-1}/gamma_i * K K^T); exp taken only below the diagonal.
+    // Strictly-lower A = Diag(btilde) (gamma_{r-1}/gamma_i * P K^T) (P = K unless Comba-pk);
+    // exp taken only below the diagonal.
     {
         float acc[8][4];
         zero(acc);
-        warp_gemm<true, true, 8>(acc, sK, S::PK, sK, S::PK, 16 * warp, 0, DK);
+        warp_gemm<true, true, 8>(acc, sF, S::PK, sK, S::PK, 16 * warp, 0, DK);
 #pragma unroll
         for (int t = 0; t < 8; ++t)
 #pragma unroll
@@ -216,12 +222,12 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     if (tid < 64) p.Gb[idx * 64 + tid] = sG[tid];
     __syncthreads();
 
-    // W, U (stored) and their Kbar-row-scaled copies for the chunk's state map.
+    // W = Mw P, U = Mu V (stored) and their Kbar-row-scaled copies for the chunk's state map.
     const float sa = sS[16 * warp + frag_row(0)], sb = sS[16 * warp + frag_row(2)];
     {
         float acc[DK / 8][4];
         zero(acc);
-        warp_gemm<true, false, DK / 8>(acc, sMw, S::PL, sK, S::PK, 16 * warp, 0, 64);
+        warp_gemm<true, false, DK / 8>(acc, sMw, S::PL, sF, S::PK, 16 * warp, 0, 64);
         frag_store_global<T, DK / 8>((T*)p.Wb + idx * 64 * DK, DK, 16 * warp, 0, acc, 64);
 #pragma unroll
         for (int t = 0; t < DK / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
@@ -348,7 +354,7 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
 
 template <typename T, int DK, int DV>
 static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int ev0) {
-    const size_t sm_prep = PrepSmem<T, DK, DV>::bytes();
+    const size_t sm_prep = PrepSmem<T, DK, DV>::bytes(p.p != nullptr);
     const size_t sm_out = OutSmem<T, DK, DV>::bytes();
     cudaError_t e;
     if ((e = cudaFuncSetAttribute(k_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
@@ -402,11 +408,11 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
     return cudaErrorInvalidValue;
 }
 
-size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv) {
+size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk) {
     if (kernel == 1) return scan_smem_bytes(is_bf16, dk, dv);
     if (use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(kernel == 0 ? 0 : 1);
 #define COMBA_SM(T, DK, DV) \
-    if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes() : OutSmem<T, DK, DV>::bytes();
+    if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes(pk) : OutSmem<T, DK, DV>::bytes();
     if (is_bf16) {
         COMBA_SM(bf16, 128, 128) COMBA_SM(bf16, 128, 64) COMBA_SM(bf16, 64, 128) COMBA_SM(bf16, 64, 64)
     } else {

@@ -9,7 +9,8 @@
 //
 //   k_prep_tc      Gram K K^T -> decay/btilde mask -> UT inverse M (fp32, blocked
 //                  forward substitution) -> W^T = K^T Mw^T, U^T = V^T Mu^T ->
-//                  Atilde = -K^T Diag(s) W, B^T = (Diag(s) U)^T K  (s = gamma_C/gamma_r)
+//                  Atilde = -K^T Diag(s) W, B^T = (Diag(s) U)^T K  (s = gamma_C/gamma_r);
+//                  with Comba-pk feedback vectors P: Gram P K^T and W^T = P^T Mw^T
 //   k_output_tc    P = Tril(Q~ K^T * Gamma), E^T = U^T - H^T W^T,
 //                  O^T = H^T Qhat^T + E^T P^T  (Qhat = Diag(gamma) Q~)
 //   k_bwd_prep_tc  C^T = dO^T (Qhat - P W)
@@ -64,16 +65,22 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     float* sWs = sG + 320;   // btilde_c gamma_{c-1}: the column scale of Mw
 
     // K into both halves of the 128-row tile: rows 64..127 repeat rows 0..63, so the
-    // padded Gram product puts a copy of each Gram row in TMEM lanes r and r + 64.
+    // padded Gram product puts a copy of each Gram row in TMEM lanes r and r + 64.  With
+    // Comba-pk feedback vectors the tile is [P; K] instead: the Gram's lanes 0..63 hold
+    // P K^T, and K (rows 64..127) is the operand of every later product that takes K.
+    const bool pk = p.p != nullptr;
     {
         const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
+        const bf16* fg = pk ? (const bf16*)p.p + (t0 * p.H + h) * D : kg;
         for (int e = tid; e < 128 * 16; e += 128) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < L;
+            const bf16* src = r < 64 ? fg : kg;
             cp_async16(sK + sw128_offset(r, ch * 8, 128),
-                       okr ? (const void*)(kg + (long long)rr * p.H * D + ch * 8) : (const void*)kg, okr);
+                       okr ? (const void*)(src + (long long)rr * p.H * D + ch * 8) : (const void*)src, okr);
         }
     }
+    const uint8_t* sKk = pk ? sK + 64 * 128 : sK;   // the 64 key rows (rows 64.. of each K-half for pk)
     load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
     cp_async_commit();
     if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
@@ -98,11 +105,11 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
     bool ok = true;
 
-    // Gram K K^T (rows >= 64 of the A tile are zero).
-    if (tid == 0) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sK), 128, 64, D, false);
+    // Gram K K^T over the 128-row tile (P K^T in lanes 0..63 for Comba-pk).
+    if (tid == 0) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sKk), 128, 64, D, false);
     if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;
     ok = ms.finish(tid);
-    if (ok) {
+    if (ok && !pk) {
         // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T), stored transposed; exp only
         // below the diagonal.  Thread t holds Gram row t & 63 and fills columns [32 (t >> 6), +32).
         const int r = row & 63, i0 = 32 * (row >> 6);
@@ -113,6 +120,20 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
         for (int c = 0; c < 32; ++c) {
             const int i = i0 + c;
             sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+        }
+    } else if (ok && row < 64) {
+        // Comba-pk: P K^T rows are in lanes 0..63 only; warps 0 and 1 take both column halves.
+        const int r = row;
+        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
+        float d[32];
+#pragma unroll
+        for (int i0 = 0; i0 < 64; i0 += 32) {
+            tmem_ld32(trow + i0, d);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                const int i = i0 + c;
+                sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+            }
         }
     }
     __syncthreads();
@@ -139,7 +160,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     }
     publish_smem();
 
-    // W^T = K^T Mw^T (A = K as MN-major), U^T = V^T Mu^T.
+    // W^T = K^T Mw^T (A = K as MN-major; P^T Mw^T for Comba-pk, tile rows 0..63), U^T = V^T Mu^T.
     if (ok && tid == 0) {
         tc_gemm<true, false>(tmem + 64, smem_u32(sK), 128, smem_u32(sMw), 64, 64, 64, false);
         tc_gemm<true, false>(tmem + 128, smem_u32(sV), 64, smem_u32(sMu), 64, 64, 64, false);
@@ -183,8 +204,8 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
 
     // Atilde = -K^T (Diag(s) W) -> cols [0,128);  B^T = (Diag(s) U)^T K -> cols [128,256).
     if (ok && tid == 0) {
-        tc_gemm<true, false>(tmem, smem_u32(sK), 128, smem_u32(sWt), 128, 128, 64, false);
-        tc_gemm<false, true>(tmem + 128, smem_u32(sUt), 128, smem_u32(sK), 128, 128, 64, false);
+        tc_gemm<true, false>(tmem, smem_u32(sKk), 128, smem_u32(sWt), 128, 128, 64, false);
+        tc_gemm<false, true>(tmem + 128, smem_u32(sUt), 128, smem_u32(sKk), 128, 128, 64, false);
     }
     if (ok) {
         // W^T, U^T out while the tensor core works

@@ -1,6 +1,7 @@
 // One-token Comba recurrence (appendix B.1, recurrent form) for a batch of
-// independent decode rows.  Per (row, head) with H = S^T (dk x dv):
-//   x = H^T k, y = H^T q~ (q~ = q - d k), e = beta v - b beta x,
+// independent decode rows.  Per (row, head) with H = S^T (dk x dv) and feedback
+// vector f (f = k; the Comba-pk vector p of appendix B.3 when given):
+//   x = H^T f, y = H^T q~ (q~ = q - d f), e = beta v - b beta x,
 //   o = alpha y + e (k . q~),  H <- alpha H + k e^T.
 // Columns of H are independent, so a block owns one (row, head, 32-column
 // tile): it reads its 32 columns of the state once with 16-byte streaming
@@ -12,7 +13,8 @@ namespace comba {
 
 template <typename T, int DK, int DV>
 __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, const T* __restrict__ k,
-                                              const T* __restrict__ v, const float* __restrict__ alpha,
+                                              const T* __restrict__ v, const T* __restrict__ pf,
+                                              const float* __restrict__ alpha,
                                               const float* __restrict__ beta, const float* __restrict__ b,
                                               const float* __restrict__ d, float* __restrict__ state,
                                               T* __restrict__ o, int iplr) {
@@ -26,7 +28,7 @@ __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, co
     const int rg = tid >> 3;             // row group 0..15
     const int col0 = tile * 32;
 
-    __shared__ float sk[DK], sq[DK];
+    __shared__ float sk[DK], sq[DK], sf[DK];
     __shared__ float rx[4][32], ry[4][32];
     __shared__ float se[32];
     __shared__ float skq;
@@ -39,8 +41,10 @@ __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, co
     const float dh = d[h];
     for (int i = tid; i < DK; i += 128) {
         const float kk = to_f(k[u * DK + i]);
+        const float ff = pf ? to_f(pf[u * DK + i]) : kk;
         sk[i] = kk;
-        sq[i] = to_f(q[u * DK + i]) - dh * kk;
+        sf[i] = ff;
+        sq[i] = to_f(q[u * DK + i]) - dh * ff;
     }
     __syncthreads();
     if (warp == 0) {
@@ -53,7 +57,7 @@ __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, co
     float x[4] = {0.f, 0.f, 0.f, 0.f}, y[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int r = 0; r < RPT; ++r) {
-        const float kr = sk[rg + 16 * r], qr = sq[rg + 16 * r];
+        const float kr = sf[rg + 16 * r], qr = sq[rg + 16 * r];   // feedback read through f
         x[0] += hv[r].x * kr; x[1] += hv[r].y * kr; x[2] += hv[r].z * kr; x[3] += hv[r].w * kr;
         y[0] += hv[r].x * qr; y[1] += hv[r].y * qr; y[2] += hv[r].z * qr; y[3] += hv[r].w * qr;
     }
@@ -92,20 +96,21 @@ __global__ void __launch_bounds__(128) k_step(int H, const T* __restrict__ q, co
 }
 
 template <typename T, int DK, int DV>
-static cudaError_t run_step(int Bd, int H, const void* q, const void* k, const void* v, const float* alpha,
+static cudaError_t run_step(int Bd, int H, const void* q, const void* k, const void* v, const void* pf,
+                            const float* alpha,
                             const float* beta, const float* b, const float* d, float* state, void* o,
                             bool iplr, cudaStream_t s) {
     const long long blocks = (long long)Bd * H * (DV / 32);
-    k_step<T, DK, DV><<<(unsigned)blocks, 128, 0, s>>>(H, (const T*)q, (const T*)k, (const T*)v, alpha, beta, b, d,
-                                                       state, (T*)o, iplr ? 1 : 0);
+    k_step<T, DK, DV><<<(unsigned)blocks, 128, 0, s>>>(H, (const T*)q, (const T*)k, (const T*)v, (const T*)pf, alpha,
+                                                       beta, b, d, state, (T*)o, iplr ? 1 : 0);
     return cudaGetLastError();
 }
 
 cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, const void* q, const void* k,
-                                  const void* v, const float* alpha, const float* beta, const float* b,
-                                  const float* d, float* state, void* o, bool iplr, cudaStream_t s) {
+                                  const void* v, const void* p, const float* alpha, const float* beta,
+                                  const float* b, const float* d, float* state, void* o, bool iplr, cudaStream_t s) {
 #define COMBA_STEP(T, DK, DV) \
-    if (dk == DK && dv == DV) return run_step<T, DK, DV>(Bd, H, q, k, v, alpha, beta, b, d, state, o, iplr, s);
+    if (dk == DK && dv == DV) return run_step<T, DK, DV>(Bd, H, q, k, v, p, alpha, beta, b, d, state, o, iplr, s);
     if (is_bf16) {
         COMBA_STEP(bf16, 128, 128) COMBA_STEP(bf16, 128, 64) COMBA_STEP(bf16, 64, 128) COMBA_STEP(bf16, 64, 64)
     } else {

@@ -24,6 +24,9 @@ struct ChunkParams {
     const float* b;          // [H] or null (b = 1)
     int iplr;                // Comba-iplr: feedback strength 2 alpha b beta instead of b beta
     const float* d;          // [H]
+    const void* p;           // Comba-pk feedback vectors [tokens,H,dk] (storage type), or null (p = k)
+    const float* d_fb;       // Comba-pk: the per-head d of the correction q - d p, applied to q before
+                             // the chunk kernels (which then see d = 0); its share of dp is -d dq
     const float* h0;         // [N,H,dk,dv] or null
     void* o;
     float* hT;
@@ -34,6 +37,7 @@ struct ChunkParams {
     void* dq;
     void* dkk;
     void* dvv;
+    void* dpp;               // Comba-pk: dL/dp [tokens,H,dk]
     float* dalpha;
     float* dbeta;
     float* db;
@@ -134,7 +138,7 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
 // the head reduction.  Stage events: ev0 before C^T, ev0+1 before the scan, ev0+2 before
 // the local gradients, ev0+3 before the reduction, ev0+4 after it.
 cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int ev0);
-size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);
+size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false);
 // tcgen05 kernels of the bf16 dk = dv = 128 path (chunk_tc.cu)
 cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s);
 cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s);
@@ -143,10 +147,17 @@ size_t tc_smem_bytes(int kernel);
 // tcgen05 local-gradient kernel of the same path (local_tc.cu)
 cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s);
 size_t local_tc_smem_bytes();
+// The tcgen05 kernels serve bf16 dk = dv = 128 (with Comba-pk feedback vectors all but the
+// local-gradient kernel, which then is the mma.sync one); every other case runs the mma.sync
+// kernels.
 inline bool use_tc_path(bool is_bf16, int dk, int dv) { return is_bf16 && dk == 128 && dv == 128; }
-size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv);
+size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false);
+// `p`: Comba-pk feedback vectors [Bd,H,dk] or null (p = k).
 cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, const void* q, const void* k,
-                                  const void* v, const float* alpha, const float* beta, const float* b,
-                                  const float* d, float* state, void* o, bool iplr, cudaStream_t s);
+                                  const void* v, const void* p, const float* alpha, const float* beta,
+                                  const float* b, const float* d, float* state, void* o, bool iplr, cudaStream_t s);
+// Comba-pk correction applied before the chunk kernels: qt = q - d_h p over [rows = tokens*H, dk].
+cudaError_t launch_pk_qtilde(const void* q, const void* p, const float* d, void* qt, long long rows, int H, int dk,
+                             bool is_bf16, cudaStream_t s);
 
 }  // namespace comba

@@ -15,7 +15,12 @@ keys/queries L2-normalised as in section 3, "SPLR" paragraph):
   * optional initial state h0 ~ 0.1*N(0,1) fp32; gradients dO ~ N(0,1),
     dhT ~ 0.1*N(0,1);
   * bf16 workloads round q, k, v, dO to bf16 (round to nearest even) on the
-    host; arrays are returned as float32 holding bf16-representable values.
+    host; arrays are returned as float32 holding bf16-representable values;
+  * Comba-pk feedback vectors (``feedback_vectors``): p = s * normalise(k + 0.5 n),
+    n ~ N(0,1), s ~ U(0.5, 1) per (token, head): a perturbed, rescaled copy of
+    the key (the appendix's p = b k plus a learned deviation), so that p . k > 0
+    mostly and the transitions alpha I - btilde p k^T stay contracting over
+    long sequences.
 
 Seeds: numpy PCG64 with seed 42 (the paper's training seed) plus a fixed
 per-workload offset.
@@ -276,3 +281,14 @@ def make_gated(B=2, T=200, H=3, dk=128, dv=128, dtype="bf16", seed_offset=0, len
     dhT = (0.1 * rng.standard_normal((N, H, dk, dv))).astype(np.float32)
     return GatedWorkload(dtype=dtype, q=q, k=k, v=v, g_alpha=g_alpha, g_beta=g_beta, a=a, c=c, b_raw=b_raw, d=d,
                          h0=h0, dO=dO, dhT=dhT, cu_seqlens=cu)
+
+
+def feedback_vectors(k: np.ndarray, dtype: str = "bf16", seed_offset: int = 0) -> np.ndarray:
+    """Comba-pk feedback vectors shaped like ``k``: s * normalise(k + 0.5 n), n ~ N(0,1),
+    s ~ U(0.5, 1) per row; bf16-rounded for bf16 workloads."""
+    rng = np.random.Generator(np.random.PCG64(SEED + 11000 + seed_offset))
+    k = np.asarray(k, np.float32)
+    n = rng.standard_normal(k.shape, dtype=np.float32)
+    s = rng.uniform(0.5, 1.0, k.shape[:-1] + (1,)).astype(np.float32)
+    p = (s * _l2norm(k + 0.5 * n)).astype(np.float32)
+    return round_bf16(p) if dtype == "bf16" else p

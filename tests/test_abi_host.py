@@ -164,3 +164,37 @@ def test_gated_flag_rules(L):
     assert L.comba_chunk_fwd_gated(ctypes.byref(s), *args, None, 0, None) == WORKSPACE
     args[5] = None   # a is required
     assert L.comba_chunk_fwd_gated(ctypes.byref(s), *args, None, 0, None) == INVALID
+
+
+def test_pk_flag_rules(L):
+    """COMBA_PK selects the Comba-pk entry points; the plain and gated ones reject it, its
+    workspace also holds q - d p, and p (and dp) are required."""
+    plain, pk_ws = ws(L, shape(), 1), ws(L, shape(flags=16), 1)
+    assert pk_ws > plain
+    assert fwd(L, shape(flags=16)) == INVALID
+    s = shape(flags=0)
+    args = [FAKE] * 11   # q k v p alpha beta b d h0 o hT
+    assert L.comba_chunk_fwd_pk(ctypes.byref(s), *args, FAKE, 1 << 40, None) == INVALID   # flag missing
+    s.flags = 16 | 8
+    assert L.comba_chunk_fwd_pk(ctypes.byref(s), *args, FAKE, 1 << 40, None) == INVALID   # not with gated
+    s.flags = 16
+    assert L.comba_chunk_fwd_pk(ctypes.byref(s), *args, None, 0, None) == WORKSPACE
+    args[3] = None   # p is required
+    assert L.comba_chunk_fwd_pk(ctypes.byref(s), *args, None, 0, None) == INVALID
+    s.flags = 16 | 2
+    bargs = [FAKE] * 20   # q k v p alpha beta b d h0 dO dhT dq dk dv dp dalpha dbeta db dd dh0
+    assert L.comba_chunk_bwd_pk(ctypes.byref(s), *bargs, None, 0, None) == WORKSPACE
+    bargs[14] = None   # dp is required
+    assert L.comba_chunk_bwd_pk(ctypes.byref(s), *bargs, None, 0, None) == INVALID
+    s.flags = 16 | 1   # the saving flag belongs to the forward
+    assert L.comba_chunk_bwd_pk(ctypes.byref(s), *([FAKE] * 20), None, 0, None) == INVALID
+
+    def step(flags=0, **over):
+        a = dict(q=FAKE, k=FAKE, v=FAKE, p=FAKE, alpha=FAKE, beta=FAKE, b=None, d=FAKE, state=FAKE, o=FAKE)
+        a.update(over)
+        return L.comba_recurrent_step_pk(4, 2, 128, 128, 1, a["q"], a["k"], a["v"], a["p"], a["alpha"], a["beta"],
+                                         a["b"], a["d"], a["state"], a["o"], flags, None)
+
+    assert step(p=None) == INVALID
+    assert step(flags=16) == INVALID
+    assert step(p=FAKE + 4) == INVALID
