@@ -35,7 +35,9 @@ struct PrepTcSmem {
     static constexpr size_t bytes() { return 1024 + OF + 64 * 6 * 4; }
 };
 
-__global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
+// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
+__global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
+    constexpr int NTH = 256;
     using S = PrepTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar;
@@ -72,7 +74,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     {
         const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
         const bf16* fg = pk ? (const bf16*)p.p + (t0 * p.H + h) * D : kg;
-        for (int e = tid; e < 128 * 16; e += 128) {
+        for (int e = tid; e < 128 * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < L;
             const bf16* src = r < 64 ? fg : kg;
@@ -81,7 +83,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
         }
     }
     const uint8_t* sKk = pk ? sK + 64 * 128 : sK;   // the 64 key rows (rows 64.. of each K-half for pk)
-    load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
     cp_async_commit();
     if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
     if (tid < 64) {
@@ -101,8 +103,8 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     publish_smem();
     const uint32_t tmem = tbase;
     MmaSync ms{smem_u32(&bar), 0};
-    const int row = tid;  // TMEM lane / accumulator row of this thread
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const int row = tid & 127, half = tid >> 7;   // TMEM lane / accumulator row, and which column half
+    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     bool ok = true;
 
     // Gram K K^T over the 128-row tile (P K^T in lanes 0..63 for Comba-pk).
@@ -111,38 +113,36 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     ok = ms.finish(tid);
     if (ok && !pk) {
         // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T), stored transposed; exp only
-        // below the diagonal.  Thread t holds Gram row t & 63 and fills columns [32 (t >> 6), +32).
-        const int r = row & 63, i0 = 32 * (row >> 6);
+        // below the diagonal.  Lane l holds Gram row l & 63; its two threads fill columns
+        // [32 (l >> 6) + 16 half, +16).
+        const int r = row & 63, i0 = 32 * (row >> 6) + 16 * half;
+        float d[16];
+        tmem_ld16(trow + i0, d);
+        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+            const int i = i0 + c;
+            sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+        }
+    } else if (ok && row < 64) {
+        // Comba-pk: P K^T rows are in lanes 0..63 only; the two threads of each take one column half.
+        const int r = row, i0 = 32 * half;
+        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
         float d[32];
         tmem_ld32(trow + i0, d);
-        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
 #pragma unroll
         for (int c = 0; c < 32; ++c) {
             const int i = i0 + c;
             sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
         }
-    } else if (ok && row < 64) {
-        // Comba-pk: P K^T rows are in lanes 0..63 only; warps 0 and 1 take both column halves.
-        const int r = row;
-        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
-        float d[32];
-#pragma unroll
-        for (int i0 = 0; i0 < 64; i0 += 32) {
-            tmem_ld32(trow + i0, d);
-#pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                const int i = i0 + c;
-                sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
-            }
-        }
     }
     __syncthreads();
     if (ok) {
-        unit_lower_inverse64_blocked(sAt, sM, 65, sTi, tid);
+        unit_lower_inverse64_blocked<NTH>(sAt, sM, 65, sTi, tid);
         __syncthreads();
         // Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta) as K-major [p][p'] tiles; M saved for the backward.
         bf16* Mg = p.Mb ? (bf16*)p.Mb + idx * 4096 : nullptr;
-        for (int e = tid; e < 64 * 8; e += 128) {
+        for (int e = tid; e < 64 * 8; e += NTH) {
             const int r = e >> 3, ch = e & 7;
             float mw[8], mu[8], mm[8];
 #pragma unroll
@@ -171,8 +171,8 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     uint8_t* stU = sMw;
     if (ok) {
         float d[32], v[8], w[8];
-#pragma unroll
-        for (int g = 0; g < 2; ++g) {
+        {
+            const int g = half;
             tmem_ld32(trow + 64 + g * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -185,8 +185,8 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
                 *reinterpret_cast<uint4*>(sWt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
             }
         }
-#pragma unroll
-        for (int g = 0; g < 2; ++g) {
+        {
+            const int g = half;
             tmem_ld32(trow + 128 + g * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -209,8 +209,8 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     }
     if (ok) {
         // W^T, U^T out while the tensor core works
-        copy_staged<8>((bf16*)p.Wb + idx * D * 64, stW, tid);
-        copy_staged<8>((bf16*)p.Ub + idx * D * 64, stU, tid);
+        copy_staged<8>((bf16*)p.Wb + idx * D * 64, stW, tid, NTH);
+        copy_staged<8>((bf16*)p.Ub + idx * D * 64, stU, tid, NTH);
     }
     ok = ok && ms.finish(tid);
     // Atilde over the dead K tile, B^T over the dead V/Mw/Mu tiles (their copies are done)
@@ -219,7 +219,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     if (ok) {
         float d[32], v[8];
 #pragma unroll
-        for (int g = 0; g < 4; ++g) {
+        for (int g = 2 * half; g < 2 * half + 2; ++g) {
             tmem_ld32(trow + g * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -229,7 +229,7 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
             }
         }
 #pragma unroll
-        for (int g = 0; g < 4; ++g) {
+        for (int g = 2 * half; g < 2 * half + 2; ++g) {
             tmem_ld32(trow + 128 + g * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) stage_chunk<16>(stB, row, 4 * g + q, pack8(d + 8 * q));
@@ -237,8 +237,8 @@ __global__ void __launch_bounds__(128) k_prep_tc(ChunkParams p) {
     }
     __syncthreads();
     if (ok) {
-        copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid);
-        copy_staged<16>((bf16*)p.Bb + idx * D * D, stB, tid);
+        copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
+        copy_staged<16>((bf16*)p.Bb + idx * D * D, stB, tid, NTH);
     }
     if (!ok && tid == 0) flag_error(p);
     tc_fence_before();
@@ -260,7 +260,9 @@ struct OutTcSmem {
 };
 
 
-__global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
+// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
+__global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
+    constexpr int NTH = 256;
     using S = OutTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar;
@@ -287,16 +289,16 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
         // Q into rows 0-63 and K into rows 64-127 of one K-major tile (rows past the chunk zero)
         const bf16* qg = (const bf16*)p.q + (t0 * p.H + h) * D;
         const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
-        for (int e = tid; e < 128 * 16; e += 128) {
+        for (int e = tid; e < 128 * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < L;
             const bf16* src = (r < 64 ? qg : kg) + (long long)rr * p.H * D + ch * 8;
             cp_async16(sQK + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
         }
     }
-    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid);
-    load_sw(sUt, 128, 64, (const bf16*)p.Ub + idx * D * 64, 64, 128, tid);
-    load_sw(sHt, 128, D, (const bf16*)p.Hb + idx * D * D, D, 128, tid);
+    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid, NTH);
+    load_sw(sUt, 128, 64, (const bf16*)p.Ub + idx * D * 64, 64, 128, tid, NTH);
+    load_sw(sHt, 128, D, (const bf16*)p.Hb + idx * D * D, D, 128, tid, NTH);
     cp_async_commit();
     if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
     if (tid == 0) {
@@ -308,7 +310,7 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
     __syncthreads();
     // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
     const float dh = p.d[h];
-    for (int e = tid; e < 64 * 16; e += 128) {
+    for (int e = tid; e < 64 * 16; e += NTH) {
         const int r = e >> 4, ch = e & 15;
         uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
         const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
@@ -322,8 +324,8 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
     publish_smem();
     const uint32_t tmem = tbase;
     MmaSync ms{smem_u32(&bar), 0};
-    const int row = tid;
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const int row = tid & 127, half = tid >> 7;   // TMEM lane, and which 32 of each 64 columns
+    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
 
     // [Q~; K] K^T -> cols [0,64) (lanes 0-63: S = Q~ K^T; lanes 64-127 unused);  E^T' = H^T W^T -> cols [64,128)
     if (tid == 0) {
@@ -332,12 +334,12 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
     }
     bool ok = ms.finish(tid);
     bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
-    uint32_t ev[32];   // this thread's row j of E^T (64 positions), packed bf16 pairs
+    uint32_t ev[16];   // this thread's 32 positions of row j of E^T, packed bf16 pairs
     if (ok) {
         float d[32], v[8];
         // P = Tril(S * Gamma) into a K-major [64][64] tile (B operand of E^T P^T)
-#pragma unroll
-        for (int g = 0; g < 2; ++g) {
+        {
+            const int g = half;
             tmem_ld32(trow + g * 32, d);
             if (row < 64) {
                 const float gr = sG[row];
@@ -352,9 +354,9 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
                 }
             }
         }
-        // E^T = U^T - H^T W^T  (row j of E^T per thread)
-#pragma unroll
-        for (int g = 0; g < 2; ++g) {
+        // E^T = U^T - H^T W^T  (half of row j of E^T per thread)
+        {
+            const int g = half;
             tmem_ld32(trow + 64 + g * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -365,12 +367,12 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
                 // sEt aliases sWt: every thread reads only its own row, and W^T is no longer needed
                 const uint4 pk = pack8(v);
                 *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * g + 8 * q, 128)) = pk;
-                const int b0 = (32 * g + 8 * q) / 2;
+                const int b0 = 4 * q;
                 ev[b0] = pk.x; ev[b0 + 1] = pk.y; ev[b0 + 2] = pk.z; ev[b0 + 3] = pk.w;
             }
         }
         // Qhat = Diag(gamma) Q~ in place
-        for (int e = tid; e < 64 * 16; e += 128) {
+        for (int e = tid; e < 64 * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15;
             uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
             float qv[8];
@@ -386,10 +388,10 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
         // E [64][128] row-major over the dead U^T tile (every thread is past its U^T reads), then
         // one 16 KB bulk copy to the workspace
 #pragma unroll
-        for (int pp = 0; pp < 32; ++pp) {
+        for (int pp = 0; pp < 16; ++pp) {
             const __nv_bfloat162 two = *reinterpret_cast<const __nv_bfloat162*>(&ev[pp]);
-            sE[(2 * pp) * D + row] = two.x;
-            sE[(2 * pp + 1) * D + row] = two.y;
+            sE[(32 * half + 2 * pp) * D + row] = two.x;
+            sE[(32 * half + 2 * pp + 1) * D + row] = two.y;
         }
         fence_async_smem();
     }
@@ -406,17 +408,14 @@ __global__ void __launch_bounds__(128) k_output_tc(ChunkParams p) {
         ok = ok && ms.finish(tid);
         if (ok) {
             float d[32];
+            tmem_ld32(trow + 128 + half * 32, d);
 #pragma unroll
-            for (int g = 0; g < 2; ++g) {
-                tmem_ld32(trow + 128 + g * 32, d);
-#pragma unroll
-                for (int c = 0; c < 32; ++c) sO[(32 * g + c) * 136 + row] = __float2bfloat16_rn(d[c]);
-            }
+            for (int c = 0; c < 32; ++c) sO[(32 * half + c) * 136 + row] = __float2bfloat16_rn(d[c]);
         }
         __syncthreads();
         if (ok) {
             bf16* Og = (bf16*)p.o + (t0 * p.H + h) * D;
-            for (int e = tid; e < L * 16; e += 128) {
+            for (int e = tid; e < L * 16; e += NTH) {
                 const int r = e >> 4, ch = e & 15;
                 *reinterpret_cast<uint4*>(Og + (long long)r * p.H * D + 8 * ch) =
                     *reinterpret_cast<const uint4*>(sO + r * 136 + 8 * ch);
@@ -443,7 +442,9 @@ struct BPrepTcSmem {
     static constexpr size_t bytes() { return 1024 + OG + 64 * 4; }
 };
 
-__global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
+// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
+__global__ void __launch_bounds__(256) k_bwd_prep_tc(ChunkParams p) {
+    constexpr int NTH = 256;
     using S = BPrepTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar;
@@ -464,10 +465,10 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     uint8_t* sdO = sm + S::OD;
     float* sG = reinterpret_cast<float*>(sm + S::OG);
 
-    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
-    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
-    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid);
-    load_sw(sdO, 64, D, (const bf16*)p.dO + (t0 * p.H + h) * D, (long long)p.H * D, L, tid);
+    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
+    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
+    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid, NTH);
+    load_sw(sdO, 64, D, (const bf16*)p.dO + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
     cp_async_commit();
     if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
     if (tid == 0) {
@@ -478,7 +479,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     cp_async_wait<0>();
     __syncthreads();
     const float dh = p.d[h];
-    for (int e = tid; e < 64 * 16; e += 128) {
+    for (int e = tid; e < 64 * 16; e += NTH) {
         const int r = e >> 4, ch = e & 15;
         uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
         const uint4 ka = *reinterpret_cast<const uint4*>(sK + sw128_offset(r, 8 * ch, 64));
@@ -492,8 +493,8 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     publish_smem();
     const uint32_t tmem = tbase;
     MmaSync ms{smem_u32(&bar), 0};
-    const int row = tid;
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const int row = tid & 127, half = tid >> 7;   // TMEM lane, and which half of the columns
+    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
 
     if (tid == 0) tc_gemm<false, false>(tmem, smem_u32(sQ), 128, smem_u32(sK), 64, 64, D, false);   // Q~ K^T
     bool ok = ms.finish(tid);
@@ -501,8 +502,8 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
         // P [128 alloc rows][64] K-major A operand (rows >= 64 zero); Qhat = Diag(gamma) Q~ in place.
         float d[32], v[8];
         const float gr = row < 64 ? sG[row] : 0.f;
-#pragma unroll
-        for (int g = 0; g < 2; ++g) {
+        {
+            const int g = half;
             tmem_ld32(trow + g * 32, d);
             if (row < 64) {
 #pragma unroll
@@ -520,7 +521,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
                     *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 128)) = make_uint4(0, 0, 0, 0);
             }
         }
-        for (int e = tid; e < 64 * 16; e += 128) {
+        for (int e = tid; e < 64 * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15;
             uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
             float qv[8];
@@ -539,7 +540,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
         // Z = Qhat - P W, written as an MN-major [64 k-rows][128] tile (B operand of dO^T Z)
         float d[32], v[8];
 #pragma unroll
-        for (int g = 0; g < 4; ++g) {
+        for (int g = 2 * half; g < 2 * half + 2; ++g) {
             tmem_ld32(trow + 64 + g * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -553,7 +554,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     } else if (ok) {
         float d[32];
 #pragma unroll
-        for (int g = 0; g < 4; ++g) tmem_ld32(trow + 64 + g * 32, d);   // keep the warp-collective loads aligned
+        for (int g = 2 * half; g < 2 * half + 2; ++g) tmem_ld32(trow + 64 + g * 32, d);   // keep the warp-collective loads aligned
     }
     publish_smem();
     // C^T = dO^T Z -> cols [0,128)
@@ -563,7 +564,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
         // C^T staged over the dead Qhat tile, then copied out coalesced
         float d[32];
 #pragma unroll
-        for (int g = 0; g < 4; ++g) {
+        for (int g = 2 * half; g < 2 * half + 2; ++g) {
             tmem_ld32(trow + g * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) stage_chunk<16>(sQ, row, 4 * g + q, pack8(d + 8 * q));
@@ -571,7 +572,7 @@ __global__ void __launch_bounds__(128) k_bwd_prep_tc(ChunkParams p) {
     }
     __syncthreads();
     if (ok) {
-        copy_staged<16>((bf16*)p.Cb + idx * D * D, sQ, tid);
+        copy_staged<16>((bf16*)p.Cb + idx * D * D, sQ, tid, NTH);
     } else if (tid == 0) {
         flag_error(p);
     }
@@ -590,7 +591,7 @@ cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s) {
     const size_t sm = tc::PrepTcSmem::bytes();
     cudaError_t e = cudaFuncSetAttribute(tc::k_prep_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
-    if (p.slots > 0) tc::k_prep_tc<<<dim3(p.slots, p.H), 128, sm, s>>>(p);
+    if (p.slots > 0) tc::k_prep_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p);
     return cudaGetLastError();
 }
 
@@ -598,7 +599,7 @@ cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s) {
     const size_t sm = tc::OutTcSmem::bytes();
     cudaError_t e = cudaFuncSetAttribute(tc::k_output_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
-    if (p.slots > 0) tc::k_output_tc<<<dim3(p.slots, p.H), 128, sm, s>>>(p);
+    if (p.slots > 0) tc::k_output_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p);
     return cudaGetLastError();
 }
 
@@ -606,7 +607,7 @@ cudaError_t launch_bwd_prep_tc(const ChunkParams& p, cudaStream_t s) {
     const size_t sm = tc::BPrepTcSmem::bytes();
     cudaError_t e = cudaFuncSetAttribute(tc::k_bwd_prep_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
-    if (p.slots > 0) tc::k_bwd_prep_tc<<<dim3(p.slots, p.H), 128, sm, s>>>(p);
+    if (p.slots > 0) tc::k_bwd_prep_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p);
     return cudaGetLastError();
 }
 

@@ -514,42 +514,53 @@ __device__ __forceinline__ void unit_lower_inverse_diag32(const float* At, float
 // then M21 = -M22 (A21 M11) with 4 x 2 register tiles per thread.  At as above;
 // M has pitch `pm`; T is 32 x 36 floats of scratch.  Rows past a short chunk
 // have A = 0 and come out as identity rows.
+template <int NTH = 128>
 __device__ __forceinline__ void unit_lower_inverse64_blocked(const float* At, float* M, int pm, float* T, int tid) {
+    static_assert(NTH == 128 || NTH == 256, "one 32 x 32 block product over 128 or 256 threads");
+    constexpr int RPT = 512 / NTH;   // rows of the 32 x 32 products per thread (4 or 2)
     if (tid < 32) unit_lower_inverse_diag32<0>(At, M, pm, tid);
     else if (tid < 64) unit_lower_inverse_diag32<32>(At, M, pm, tid);
     __syncthreads();
-    const int r0 = 4 * (tid >> 4), c0 = 2 * (tid & 15);
+    const int r0 = RPT * (tid >> 4), c0 = 2 * (tid & 15);
     {
         // T = A21 M11: T[r][c] = sum_k A[32 + r][k] M[k][c]
-        float t[4][2] = {};
+        float t[RPT][2] = {};
 #pragma unroll 8
         for (int k = 0; k < 32; ++k) {
-            const float4 a = *reinterpret_cast<const float4*>(At + k * 68 + 32 + r0);
+            float a[RPT];
+            if constexpr (RPT == 4) {
+                const float4 a4 = *reinterpret_cast<const float4*>(At + k * 68 + 32 + r0);
+                a[0] = a4.x; a[1] = a4.y; a[2] = a4.z; a[3] = a4.w;
+            } else {
+                const float2 a2 = *reinterpret_cast<const float2*>(At + k * 68 + 32 + r0);
+                a[0] = a2.x; a[1] = a2.y;
+            }
             const float m0 = M[k * pm + c0], m1 = M[k * pm + c0 + 1];
-            t[0][0] = fmaf(a.x, m0, t[0][0]); t[0][1] = fmaf(a.x, m1, t[0][1]);
-            t[1][0] = fmaf(a.y, m0, t[1][0]); t[1][1] = fmaf(a.y, m1, t[1][1]);
-            t[2][0] = fmaf(a.z, m0, t[2][0]); t[2][1] = fmaf(a.z, m1, t[2][1]);
-            t[3][0] = fmaf(a.w, m0, t[3][0]); t[3][1] = fmaf(a.w, m1, t[3][1]);
+#pragma unroll
+            for (int e = 0; e < RPT; ++e) {
+                t[e][0] = fmaf(a[e], m0, t[e][0]);
+                t[e][1] = fmaf(a[e], m1, t[e][1]);
+            }
         }
 #pragma unroll
-        for (int e = 0; e < 4; ++e) *reinterpret_cast<float2*>(T + (r0 + e) * 36 + c0) = make_float2(t[e][0], t[e][1]);
+        for (int e = 0; e < RPT; ++e) *reinterpret_cast<float2*>(T + (r0 + e) * 36 + c0) = make_float2(t[e][0], t[e][1]);
     }
     __syncthreads();
     {
         // M21 = -M22 T: M[32 + r][c] = -sum_k M[32 + r][32 + k] T[k][c]
-        float t[4][2] = {};
+        float t[RPT][2] = {};
 #pragma unroll 8
         for (int k = 0; k < 32; ++k) {
             const float2 b = *reinterpret_cast<const float2*>(T + k * 36 + c0);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
+            for (int e = 0; e < RPT; ++e) {
                 const float m = M[(32 + r0 + e) * pm + 32 + k];
                 t[e][0] = fmaf(m, b.x, t[e][0]);
                 t[e][1] = fmaf(m, b.y, t[e][1]);
             }
         }
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
+        for (int e = 0; e < RPT; ++e) {
             M[(32 + r0 + e) * pm + c0] = -t[e][0];
             M[(32 + r0 + e) * pm + c0 + 1] = -t[e][1];
         }

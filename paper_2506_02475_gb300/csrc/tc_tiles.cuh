@@ -80,8 +80,8 @@ __device__ __forceinline__ void stage_chunk(uint8_t* st, int row, int c, uint4 v
     *reinterpret_cast<uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16) = v;
 }
 template <int NCH>
-__device__ __forceinline__ void copy_staged(bf16* g, const uint8_t* st, int tid) {
-    for (int e = tid; e < 128 * NCH; e += 128) {
+__device__ __forceinline__ void copy_staged(bf16* g, const uint8_t* st, int tid, int nthr = 128) {
+    for (int e = tid; e < 128 * NCH; e += nthr) {
         const int row = e / NCH, c = e % NCH;
         reinterpret_cast<uint4*>(g)[e] = *reinterpret_cast<const uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16);
     }
