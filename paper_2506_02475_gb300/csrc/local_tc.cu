@@ -442,7 +442,9 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                     const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
                     const bool incl = c <= r && r < L;
                     const float gam = incl ? __expf(sG[r] - sG[c]) : 0.f;
-                    const float w = dP[t][i] * sc[t][i] * gam;   // dP * P
+                    // dP * P into the log-decay gradient; the diagonal's decay factor is exactly 1
+                    // (no g-dependence), so it is left out rather than added and cancelled
+                    const float w = c < r ? dP[t][i] * sc[t][i] * gam : 0.f;
                     if (i < 2) rs0 += w; else rs1 += w;
                     cs[t][i & 1] += w;
                     ph[i] = dP[t][i] * gam;
@@ -496,7 +498,9 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                     const float gm = strict ? __expf(sGm1[r] - sG[c]) : 0.f;
                     const float a = -da[t][i];
                     const float uu = a * gm * gr[t][i];   // contributes to dbtilde_r
-                    const float w = uu * sBt[r];          // dA * Aval
+                    // dA * Aval into the log-decay gradient; on the first sub-diagonal the decay
+                    // factor gamma_{r-1}/gamma_c is exactly 1, so it is left out (it would cancel)
+                    const float w = c + 1 < r ? uu * sBt[r] : 0.f;
                     if (i < 2) { rb0 += uu; ra0 += w; } else { rb1 += uu; ra1 += w; }
                     cs[t][i & 1] += w;
                     g4[i] = a * sBt[r] * gm;
@@ -586,7 +590,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             const int r = tid;
             float g = 0.f;
             if (r < L) {
-                g = rsum(0, r) - rsum(1, r) + rsum(3, r) - csum(0, r) - csum(1, r);
+                g = rsum(0, r) + rsum(3, r) - csum(0, r) - csum(1, r);   // Kbar terms: prefix sum below
                 if (r + 1 < L) {
                     g += rsum(5, r + 1);
                     g += sWs[r + 1] * rsum(7, r + 1);
@@ -596,17 +600,25 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         }
         __syncthreads();
         if (ok && warp == 0) {
-            // terms on the last position: gamma_C <H, dH'> and the Kbar total (fixed-order warp
-            // reductions), then d log alpha_j = sum_{r >= j} dg_r, a suffix sum inside the chunk
-            float tk = (lane < L ? rsum(1, lane) : 0.f) + (lane + 32 < L ? rsum(1, lane + 32) : 0.f);
+            // d log alpha_j = sum_{r >= j} dg_r (a suffix sum inside the chunk) plus gamma_C <H, dH'> at the
+            // last position; the Kbar terms, which reach it as (their total - their suffix), are
+            // added as the exclusive prefix sum_{r < j} instead, so nothing cancels.
+            float k0 = lane < L ? rsum(1, lane) : 0.f, k1 = lane + 32 < L ? rsum(1, lane + 32) : 0.f;
             float hd = lane < 8 ? red[lane] : 0.f;
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                tk += __shfl_xor_sync(0xffffffffu, tk, o);
-                hd += __shfl_xor_sync(0xffffffffu, hd, o);
+            for (int o = 16; o > 0; o >>= 1) hd += __shfl_xor_sync(0xffffffffu, hd, o);
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {   // inclusive prefix sums of the Kbar terms
+                const float y0 = __shfl_up_sync(0xffffffffu, k0, o);
+                const float y1 = __shfl_up_sync(0xffffffffu, k1, o);
+                if (lane >= o) { k0 += y0; k1 += y1; }
             }
+            const float half0 = __shfl_sync(0xffffffffu, k0, 31);
+            k1 += half0;
+            const float e0p = __shfl_up_sync(0xffffffffu, k0, 1), e1p = __shfl_up_sync(0xffffffffu, k1, 1);
+            const float e0 = lane == 0 ? 0.f : e0p, e1 = lane == 0 ? half0 : e1p;   // exclusive prefixes
             float x0 = sDg[lane], x1 = sDg[lane + 32];   // zero past L
-            const float last = tk + __expf(gL) * hd;
+            const float last = __expf(gL) * hd;
             if (L - 1 == lane) x0 += last;
             if (L - 1 == lane + 32) x1 += last;
 #pragma unroll
@@ -616,8 +628,8 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                 if (lane + o < 32) { x0 += y0; x1 += y1; }
             }
             x0 += __shfl_sync(0xffffffffu, x1, 0);
-            sDg[lane] = x0;
-            sDg[lane + 32] = x1;
+            sDg[lane] = x0 + e0;
+            sDg[lane + 32] = x1 + e1;
         }
         __syncthreads();
         if (ok && tid < 64) {
