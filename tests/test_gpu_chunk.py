@@ -236,3 +236,24 @@ def test_iplr_variant_forward_backward(dtype, d, lens):
     # and it is not the SPLR result
     ro_s, _ = oracle.fwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0, cu_seqlens=w.cu_seqlens)
     assert rel(np64(o), ro_s) > 2 * tol(dtype)
+
+
+def test_single_long_sequence():
+    """One sequence of 32768 tokens (512 chunks through each scan), bf16 d=128, two heads:
+    forward and backward against the oracle."""
+    w = inputs.make("custom", B=1, T=32768, H=2, dk=128, dv=128, dtype="bf16", with_b=True, with_h0=True,
+                    with_grads=True, seed_offset=77)
+    t = to_dev(w)
+    check_fwd(w, t)
+    check_bwd(w, t)
+
+
+def test_thousands_of_tiny_sequences():
+    """1200 packed sequences of 0-5 tokens: far more sequences than chunks of work, every chunk
+    ragged, many empty sequences passing h0 through."""
+    lens = np.random.default_rng(11).integers(0, 6, 1200).tolist()
+    w = inputs.make("custom", H=2, dk=128, dv=128, dtype="bf16", with_b=True, with_h0=True, with_grads=True,
+                    lengths=lens, seed_offset=23)
+    t = to_dev(w)
+    check_fwd(w, t)
+    check_bwd(w, t)
