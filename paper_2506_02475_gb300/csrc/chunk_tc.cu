@@ -138,7 +138,7 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
     }
     __syncthreads();
     if (ok) {
-        unit_lower_inverse64_blocked<NTH>(sAt, sM, 65, sTi, tid);
+        unit_lower_inverse64_h16(sAt, sM, 65, sTi, tid);
         __syncthreads();
         // Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta) as K-major [p][p'] tiles; M saved for the backward.
         bf16* Mg = p.Mb ? (bf16*)p.Mb + idx * 4096 : nullptr;

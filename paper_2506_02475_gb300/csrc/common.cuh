@@ -477,90 +477,109 @@ __device__ __forceinline__ void unit_lower_inverse64(const float* A, float* M, f
     }
 }
 
-// Diagonal 32 x 32 block [C0, C0+32) of (I + A)^{-1} for a strictly lower 64 x 64
-// A, by right-looking forward substitution: the calling thread owns column j of
-// the block and keeps the running row sums s_r = sum_{i<r} A_ri x_i of that
-// column in registers; each solved entry x_r updates the sums of the rows below
-// it.  At is A transposed (At[i][r] = A[r][i], pitch 68 floats, zero on and
-// above the diagonal of A), so an update reads one contiguous row of At (the
-// same address across the warp).  Writes rows [C0, C0+32) of column j of M
-// (pitch `pm`), and zeros above them.
-template <int C0>
-__device__ __forceinline__ void unit_lower_inverse_diag32(const float* At, float* M, int pm, int j) {
-    float s[32];
+// Column j (of 16) of (I + A_bb)^{-1} for the 16 x 16 diagonal block starting at B0, by
+// forward substitution in registers: M[r2][j] = delta - sum_{r < r2} A[r2][r] M[r][j].
+// At is A transposed (pitch 68): its row r holds column r of A, zero at and above r.
+template <int B0>
+__device__ __forceinline__ void unit_lower_inverse_diag16(const float* At, float* M, int pm, int j) {
+    float s[16];
 #pragma unroll
-    for (int r = 0; r < 32; ++r) s[r] = 0.f;
+    for (int r = 0; r < 16; ++r) s[r] = 0.f;
 #pragma unroll
-    for (int r = C0; r < C0 + 32; ++r) {
-        const float x = r == j ? 1.f : (r < j ? 0.f : -s[r - C0]);
-        M[r * pm + j] = x;
-        // rows r2 >= 4 floor((r+1)/4) of the block: At[r][r2] = A[r2][r] is zero for r2 <= r,
-        // and the sums of rows <= r are no longer read, so aligned groups of four are updated whole
+    for (int r = 0; r < 16; ++r) {
+        const float x = r == j ? 1.f : (r < j ? 0.f : -s[r]);
+        M[(B0 + r) * pm + B0 + j] = x;
 #pragma unroll
-        for (int g = (r + 1) >> 2; g < (C0 + 32) / 4; ++g) {
-            const float4 a = *reinterpret_cast<const float4*>(At + r * 68 + 4 * g);
-            s[4 * g + 0 - C0] = fmaf(a.x, x, s[4 * g + 0 - C0]);
-            s[4 * g + 1 - C0] = fmaf(a.y, x, s[4 * g + 1 - C0]);
-            s[4 * g + 2 - C0] = fmaf(a.z, x, s[4 * g + 2 - C0]);
-            s[4 * g + 3 - C0] = fmaf(a.w, x, s[4 * g + 3 - C0]);
+        for (int g = (r + 1) >> 2; g < 4; ++g) {
+            const float4 a = *reinterpret_cast<const float4*>(At + (B0 + r) * 68 + B0 + 4 * g);
+            s[4 * g + 0] = fmaf(a.x, x, s[4 * g + 0]);
+            s[4 * g + 1] = fmaf(a.y, x, s[4 * g + 1]);
+            s[4 * g + 2] = fmaf(a.z, x, s[4 * g + 2]);
+            s[4 * g + 3] = fmaf(a.w, x, s[4 * g + 3]);
         }
     }
-#pragma unroll
-    for (int r = 0; r < C0; ++r) M[r * pm + j] = 0.f;
 }
 
-// (I + A)^{-1} for a strictly lower 64 x 64 A (128 threads), by 32 x 32 blocks:
-// M11 = (I + A11)^{-1} and M22 = (I + A22)^{-1} (warps 0 and 1, in registers),
-// then M21 = -M22 (A21 M11) with 4 x 2 register tiles per thread.  At as above;
-// M has pitch `pm`; T is 32 x 36 floats of scratch.  Rows past a short chunk
-// have A = 0 and come out as identity rows.
-template <int NTH = 128>
-__device__ __forceinline__ void unit_lower_inverse64_blocked(const float* At, float* M, int pm, float* T, int tid) {
-    static_assert(NTH == 128 || NTH == 256, "one 32 x 32 block product over 128 or 256 threads");
-    constexpr int RPT = 512 / NTH;   // rows of the 32 x 32 products per thread (4 or 2)
-    if (tid < 32) unit_lower_inverse_diag32<0>(At, M, pm, tid);
-    else if (tid < 64) unit_lower_inverse_diag32<32>(At, M, pm, tid);
-    __syncthreads();
-    const int r0 = RPT * (tid >> 4), c0 = 2 * (tid & 15);
-    {
-        // T = A21 M11: T[r][c] = sum_k A[32 + r][k] M[k][c]
-        float t[RPT][2] = {};
-#pragma unroll 8
-        for (int k = 0; k < 32; ++k) {
-            float a[RPT];
-            if constexpr (RPT == 4) {
-                const float4 a4 = *reinterpret_cast<const float4*>(At + k * 68 + 32 + r0);
-                a[0] = a4.x; a[1] = a4.y; a[2] = a4.z; a[3] = a4.w;
-            } else {
-                const float2 a2 = *reinterpret_cast<const float2*>(At + k * 68 + 32 + r0);
-                a[0] = a2.x; a[1] = a2.y;
-            }
-            const float m0 = M[k * pm + c0], m1 = M[k * pm + c0 + 1];
-#pragma unroll
-            for (int e = 0; e < RPT; ++e) {
-                t[e][0] = fmaf(a[e], m0, t[e][0]);
-                t[e][1] = fmaf(a[e], m1, t[e][1]);
-            }
+// (I + A)^{-1} for a strictly lower 64 x 64 A over 256 threads, in three levels: the four
+// 16 x 16 diagonal blocks (threads 0..63, one column each), then the 32 x 32 blocks
+// M10 = -M11 (A10 M00) of both halves, then the 64 x 64 M21 = -M22 (A21 M11).  At is A
+// transposed with pitch 68; M has pitch `pm` and is written in full (zeros above the
+// diagonal); T holds 32 x 36 floats of scratch.
+__device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float* M, int pm, float* T, int tid) {
+    if (tid < 64) {
+        const int j = tid & 15;
+        switch (tid >> 4) {
+            case 0: unit_lower_inverse_diag16<0>(At, M, pm, j); break;
+            case 1: unit_lower_inverse_diag16<16>(At, M, pm, j); break;
+            case 2: unit_lower_inverse_diag16<32>(At, M, pm, j); break;
+            default: unit_lower_inverse_diag16<48>(At, M, pm, j); break;
         }
+    } else {
+        // zeros above the diagonal blocks: rows 0..47, columns past each row's block
+        for (int e = tid - 64; e < 64 * 64; e += 192) {
+            const int r = e >> 6, c = e & 63;
+            if ((c >> 4) > (r >> 4)) M[r * pm + c] = 0.f;
+        }
+    }
+    __syncthreads();
+    // level 1, both halves h (block rows 2h+1, block columns 2h): thread -> (h, r, c pair)
+    const int h1 = tid >> 7, r1 = (tid >> 3) & 15, c1 = 2 * (tid & 7);
+    const int o1 = 32 * h1;
+    {
+        // T1 = A10 M00: T1[r][c] = sum_k A[o1 + 16 + r][o1 + k] M[o1 + k][o1 + c]
+        float t0 = 0.f, t1 = 0.f;
 #pragma unroll
-        for (int e = 0; e < RPT; ++e) *reinterpret_cast<float2*>(T + (r0 + e) * 36 + c0) = make_float2(t[e][0], t[e][1]);
+        for (int k = 0; k < 16; ++k) {
+            const float a = At[(o1 + k) * 68 + o1 + 16 + r1];
+            t0 = fmaf(a, M[(o1 + k) * pm + o1 + c1], t0);
+            t1 = fmaf(a, M[(o1 + k) * pm + o1 + c1 + 1], t1);
+        }
+        *reinterpret_cast<float2*>(T + h1 * 16 * 18 + r1 * 18 + c1) = make_float2(t0, t1);
     }
     __syncthreads();
     {
-        // M21 = -M22 T: M[32 + r][c] = -sum_k M[32 + r][32 + k] T[k][c]
-        float t[RPT][2] = {};
+        // M10 = -M11 T1: M[o1 + 16 + r][o1 + c] = -sum_k M[o1 + 16 + r][o1 + 16 + k] T1[k][c]
+        float t0 = 0.f, t1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            const float m = M[(o1 + 16 + r1) * pm + o1 + 16 + k];
+            const float2 b = *reinterpret_cast<const float2*>(T + h1 * 16 * 18 + k * 18 + c1);
+            t0 = fmaf(m, b.x, t0);
+            t1 = fmaf(m, b.y, t1);
+        }
+        M[(o1 + 16 + r1) * pm + o1 + c1] = -t0;
+        M[(o1 + 16 + r1) * pm + o1 + c1 + 1] = -t1;
+    }
+    __syncthreads();
+    // level 2: M21 = -M22 (A21 M11) over the 32 x 32 blocks, 2 x 2 outputs per thread
+    const int r0 = 2 * (tid >> 4), c0 = 2 * (tid & 15);
+    {
+        float t[2][2] = {};
+#pragma unroll 8
+        for (int k = 0; k < 32; ++k) {
+            const float2 a2 = *reinterpret_cast<const float2*>(At + k * 68 + 32 + r0);
+            const float m0 = M[k * pm + c0], m1 = M[k * pm + c0 + 1];
+            t[0][0] = fmaf(a2.x, m0, t[0][0]); t[0][1] = fmaf(a2.x, m1, t[0][1]);
+            t[1][0] = fmaf(a2.y, m0, t[1][0]); t[1][1] = fmaf(a2.y, m1, t[1][1]);
+        }
+        *reinterpret_cast<float2*>(T + r0 * 36 + c0) = make_float2(t[0][0], t[0][1]);
+        *reinterpret_cast<float2*>(T + (r0 + 1) * 36 + c0) = make_float2(t[1][0], t[1][1]);
+    }
+    __syncthreads();
+    {
+        float t[2][2] = {};
 #pragma unroll 8
         for (int k = 0; k < 32; ++k) {
             const float2 b = *reinterpret_cast<const float2*>(T + k * 36 + c0);
 #pragma unroll
-            for (int e = 0; e < RPT; ++e) {
+            for (int e = 0; e < 2; ++e) {
                 const float m = M[(32 + r0 + e) * pm + 32 + k];
                 t[e][0] = fmaf(m, b.x, t[e][0]);
                 t[e][1] = fmaf(m, b.y, t[e][1]);
             }
         }
 #pragma unroll
-        for (int e = 0; e < RPT; ++e) {
+        for (int e = 0; e < 2; ++e) {
             M[(32 + r0 + e) * pm + c0] = -t[e][0];
             M[(32 + r0 + e) * pm + c0 + 1] = -t[e][1];
         }
