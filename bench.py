@@ -95,14 +95,14 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 110_865, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "f839f342596f289d"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_531, ('scan.cu', 'common.cuh', 'params.cuh'), "de0526678a01fe09"),
-    "output": ("k_output_tc", 118_692, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "f839f342596f289d"),
-    "bwd_prep": ("k_bwd_prep_tc", 82_581, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "f839f342596f289d"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_381, ('scan.cu', 'common.cuh', 'params.cuh'), "de0526678a01fe09"),
-    "bwd_local": ("k_bwd_local_tc", 194_263, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "69eee2248b1e4386"),
+    "prep": ("k_prep_tc", 110_802, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c38997b1ac5319b7"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_487, ('scan.cu', 'common.cuh', 'params.cuh'), "bd55d18df9523763"),
+    "output": ("k_output_tc", 118_759, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c38997b1ac5319b7"),
+    "bwd_prep": ("k_bwd_prep_tc", 82_468, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c38997b1ac5319b7"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_409, ('scan.cu', 'common.cuh', 'params.cuh'), "bd55d18df9523763"),
+    "bwd_local": ("k_bwd_local_tc", 194_260, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c382ee4e8c042aa7"),
 }
-DECODE_TRAFFIC = (482_260_224, ('decode.cu', 'common.cuh', 'params.cuh'), "8adc5b26525edb4b")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (481_426_688, ('decode.cu', 'common.cuh', 'params.cuh'), "3956f50c494e5178")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
