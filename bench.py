@@ -445,8 +445,12 @@ def run_ours(args, world, rank, local):
 
     # ---- dominant kernel and its roofline
     slots = (tokens // 64 + N) if w.cu_seqlens is not None else w.q.shape[0] * ((w.q.shape[1] + 63) // 64)
-    tc = w.dtype == "bf16" and dk == 128 and dv == 128
-    model = stage_model(dk, dv, slots, H, N, tc=tc, pk=pk)
+    # value-head groups: dv beyond 128 runs as dv / 128 value heads of width 128 per key head, and
+    # every kernel's unit is a (chunk, value head) pair
+    vg = dv // 128 if dv > 128 else 1
+    dv_u, H_u = dv // vg, H * vg
+    tc = w.dtype == "bf16" and dk == 128 and dv_u == 128
+    model = stage_model(dk, dv_u, slots, H_u, N, tc=tc, pk=pk)
     # the dominant launch: the (phase, stage) with the most time (a stage the backward skips
     # because it reuses the forward's factors is not averaged with its empty slot)
     dom_phase, dom = max(stage_ms, key=lambda ps: stage_ms[ps])
@@ -462,7 +466,7 @@ def run_ours(args, world, rank, local):
         roof = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     # captured figures are for the kernels without Comba-pk feedback vectors
-    traffic, kname = captured_traffic(dom, slots * H, dk, dv, w.dtype, tc=tc and not pk)
+    traffic, kname = captured_traffic(dom, slots * H_u, dk, dv_u, w.dtype, tc=tc and not pk)
     roof.update({"kernel": kname or dom, "stage": dom, "launch_ms": launch_ms, "algorithmic_flops": mdl["flops"],
                  "algorithmic_bytes": mdl["bytes"], "traffic": traffic,
                  "traffic_source": "ncu capture of the 340M-shape step, scaled by units" if traffic else None,
@@ -872,7 +876,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="lm1p3b", choices=["lm1p3b", "lm340m", "varlen64k", "decode"])
+    ap.add_argument("--workload", default="lm1p3b", choices=["lm1p3b", "lm340m", "varlen64k", "lm1p3b_v256", "decode"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--gated", action="store_true",
                     help="raw q, k and gate pre-activations through the gate and normalisation prologue")

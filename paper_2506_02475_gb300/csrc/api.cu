@@ -22,9 +22,16 @@ struct Layout {
     size_t qh, kh, ga, gb, bg, dqh, dkh, dal, dbe, dbi, dar, dcr, dpa, dpc;
     // Comba-pk (COMBA_PK): the corrected queries q - d p and the zero d the chunk kernels then see
     size_t qt, dz;
+    // value-head groups (dv = vg * 128, vg > 1): the backward's per-value-head dq, dk, dalpha, dbeta
+    size_t gdq, gdk, gda, gdb;
     size_t total;
     int slots;
+    int vg;      // value heads per key head; the kernels see H * vg heads of width dv / vg
 };
+
+// Value heads per key head: dv beyond 128 (a multiple of 128, dk = 128, bf16, plain or iplr
+// form) runs as dv / 128 value heads of width 128 that share the key head's q, k and gates.
+int value_groups(const comba_shape_t* s) { return s->dv > 128 ? s->dv / 128 : 1; }
 
 // Validates the shape (not the pointers) and computes the workspace layout.
 // The forward needs W, U, G, Atilde, B^T and the chunk states; saving for the
@@ -35,8 +42,15 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (s->B < 1 || s->T < 0 || s->H < 1 || s->num_seqs < 1) return COMBA_ERR_INVALID_ARG;
     if (s->dtype != COMBA_F32 && s->dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
     if (s->chunk != comba::kChunk) return COMBA_ERR_UNSUPPORTED;
-    if ((s->dk != 64 && s->dk != 128) || (s->dv != 64 && s->dv != 128)) return COMBA_ERR_UNSUPPORTED;
-    if (s->H > 65535 || s->num_seqs > 2147483647 / 4) return COMBA_ERR_UNSUPPORTED;
+    const int vg = value_groups(s);
+    if (vg > 1) {
+        // dv = 256, 384 or 512 as groups of 128-wide value heads on the tcgen05 path
+        if (s->dv % 128 != 0 || vg > 4 || s->dk != 128 || s->dtype != COMBA_BF16) return COMBA_ERR_UNSUPPORTED;
+        if (s->flags & (COMBA_GATED | COMBA_PK)) return COMBA_ERR_UNSUPPORTED;
+    } else if ((s->dk != 64 && s->dk != 128) || (s->dv != 64 && s->dv != 128)) {
+        return COMBA_ERR_UNSUPPORTED;
+    }
+    if ((long long)s->H * vg > 65535 || s->num_seqs > 2147483647 / 4) return COMBA_ERR_UNSUPPORTED;
     if (s->cu_seqlens) {
         if (s->B != 1) return COMBA_ERR_INVALID_ARG;
         if (!aligned16(s->cu_seqlens)) return COMBA_ERR_INVALID_ARG;
@@ -48,13 +62,14 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (backward && s->dtype == COMBA_F32 && (s->dk != 64 || s->dv != 64)) return COMBA_ERR_UNSUPPORTED;
     const long long slots = s->cu_seqlens ? ttot / comba::kChunk + s->num_seqs
                                           : (long long)s->B * ((s->T + comba::kChunk - 1) / comba::kChunk);
-    const long long pairs_ll = slots * s->H;
+    const long long pairs_ll = slots * s->H * vg;   // (chunk slot, value head) units
     // the scan addresses chunk-state rows with 32-bit TMA coordinates
     if (slots >= (1LL << 30) || pairs_ll * 128 >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
     const size_t es = s->dtype == COMBA_BF16 ? 2 : 4;
     const size_t pairs = (size_t)pairs_ll;
-    const size_t dk = s->dk, dv = s->dv;
+    const size_t dk = s->dk, dv = s->dv / vg;       // one value head's width
     Layout L{};
+    L.vg = vg;
     size_t o = 0;
     auto take = [&](size_t bytes) { size_t at = o; o = align_up(o + bytes); return at; };
     L.err = take(sizeof(int));
@@ -99,6 +114,13 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
         L.qt = take((size_t)ttot * s->H * dk * es);
         L.dz = take((size_t)s->H * sizeof(float));
     }
+    if (backward && vg > 1) {
+        const size_t vrows = (size_t)ttot * s->H * vg;
+        L.gdq = take(vrows * dk * es);
+        L.gdk = take(vrows * dk * es);
+        L.gda = take(vrows * sizeof(float));
+        L.gdb = take(vrows * sizeof(float));
+    }
     L.total = o;
     L.slots = (int)slots;
     *out = L;
@@ -111,17 +133,21 @@ comba_status_t check_smem(const comba_shape_t* s, int backward) {
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
         return COMBA_ERR_CUDA;
     const bool bf = s->dtype == COMBA_BF16, pk = (s->flags & COMBA_PK) != 0;
+    const int dv = s->dv / value_groups(s);
     for (int kern = 0; kern < 3; ++kern)
-        if (comba::fwd_smem_bytes(kern, bf, s->dk, s->dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
+        if (comba::fwd_smem_bytes(kern, bf, s->dk, dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
     if (backward)
         for (int kern = 0; kern < 2; ++kern)
-            if (comba::bwd_smem_bytes(kern, bf, s->dk, s->dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
+            if (comba::bwd_smem_bytes(kern, bf, s->dk, dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
     return COMBA_OK;
 }
 
 void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* ws, bool backward_layout) {
     char* w = static_cast<char*>(ws);
-    p.B = s->B; p.T = s->T; p.H = s->H; p.dk = s->dk; p.dv = s->dv; p.N = s->num_seqs;
+    p.B = s->B; p.T = s->T; p.N = s->num_seqs;
+    p.vg = L.vg;
+    p.H = s->H * L.vg;                 // value heads
+    p.dk = s->dk; p.dv = s->dv / L.vg;
     p.Ttot = (long long)s->B * s->T;
     p.cu = s->cu_seqlens;
     p.slots = L.slots;
@@ -220,6 +246,13 @@ comba_status_t backward_run(const comba_shape_t* shape, const Layout& L, void* w
     p.p = pk.p; p.d_fb = pk.d; p.dpp = pk.dp;
     p.dO = dO; p.dhT = dhT; p.dq = dq; p.dkk = dk; p.dvv = dv;
     p.dalpha = dalpha; p.dbeta = dbeta; p.db = db; p.dd = dd; p.dh0 = dh0;
+    if (L.vg > 1) {
+        // per-value-head key-side gradients into the workspace, summed per key head below
+        char* w = static_cast<char*>(workspace);
+        p.dq = w + L.gdq; p.dkk = w + L.gdk;
+        p.dalpha = reinterpret_cast<float*>(w + L.gda);
+        p.dbeta = reinterpret_cast<float*>(w + L.gdb);
+    }
     const bool bf = shape->dtype == COMBA_BF16;
     comba::mark(p, 0, s);
     if (reuse) {
@@ -233,6 +266,9 @@ comba_status_t backward_run(const comba_shape_t* shape, const Layout& L, void* w
         if (comba::launch_fwd(f, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
     }
     if (comba::launch_bwd(p, bf, s, 4) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (L.vg > 1 && comba::launch_group_sum(p.dq, p.dkk, p.dalpha, p.dbeta, dq, dk, dalpha, dbeta, p.Ttot, p.H, L.vg,
+                                            p.dk, bf, s) != cudaSuccess)
+        return COMBA_ERR_CUDA;
     return COMBA_OK;
 }
 
@@ -428,7 +464,7 @@ comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtyp
     if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
     if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
     if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
-    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128)) return COMBA_ERR_UNSUPPORTED;
+    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128 && !(dv == 256 && dk == 128))) return COMBA_ERR_UNSUPPORTED;
     if ((long long)Bd * H * (dv / 32) >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(p); COMBA_REQUIRE(alpha);
     COMBA_REQUIRE(beta); COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
@@ -446,7 +482,7 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
     if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
     if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
     if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
-    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128)) return COMBA_ERR_UNSUPPORTED;
+    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128 && !(dv == 256 && dk == 128))) return COMBA_ERR_UNSUPPORTED;
     if ((long long)Bd * H * (dv / 32) >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);

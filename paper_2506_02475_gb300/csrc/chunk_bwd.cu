@@ -658,16 +658,18 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     }
 }
 
-// One block per head: db[h] = sum over chunk slots of the per-chunk partials,
-// in a fixed order (strided per-thread sums, then a fixed tree).
+// One block per key head: db, dd = sums over chunk slots (and over the key head's vg value
+// heads) of the per-chunk partials, in a fixed order (strided per-thread sums, then a fixed tree).
 __global__ void __launch_bounds__(256) k_reduce_heads(ChunkParams p) {
     __shared__ float s_db[256], s_dd[256];
-    const int h = blockIdx.x, tid = threadIdx.x;
+    const int hk = blockIdx.x, tid = threadIdx.x;
     float a = 0.f, c = 0.f;
-    for (int s = tid; s < p.slots; s += 256) {
-        a += p.part[((long long)s * p.H + h) * 2];
-        c += p.part[((long long)s * p.H + h) * 2 + 1];
-    }
+    for (int s = tid; s < p.slots; s += 256)
+        for (int j = 0; j < p.vg; ++j) {
+            const long long u = (long long)s * p.H + hk * p.vg + j;
+            a += p.part[u * 2];
+            c += p.part[u * 2 + 1];
+        }
     s_db[tid] = a;
     s_dd[tid] = c;
     __syncthreads();
@@ -676,9 +678,52 @@ __global__ void __launch_bounds__(256) k_reduce_heads(ChunkParams p) {
         __syncthreads();
     }
     if (tid == 0) {
-        if (p.db) p.db[h] = s_db[0];
-        p.dd[h] = s_dd[0];
+        if (p.db) p.db[hk] = s_db[0];
+        p.dd[hk] = s_dd[0];
     }
+}
+
+// Value-head groups: out[t, hk, :] = sum_{j < vg} in[t, hk * vg + j, :] in order j = 0, 1, ...
+// for dq, dk (D wide, storage type) and dalpha, dbeta (one float), one thread per element.
+template <typename T>
+__global__ void __launch_bounds__(256) k_group_sum(const T* __restrict__ dq_v, const T* __restrict__ dk_v,
+                                                   const float* __restrict__ da_v, const float* __restrict__ db_v,
+                                                   T* __restrict__ dq, T* __restrict__ dk, float* __restrict__ dalpha,
+                                                   float* __restrict__ dbeta, long long rows_k, int vg, int D) {
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < rows_k * D; e += stride) {
+        const long long rk = e / D, c = e - rk * D;   // key row (token * Hk + hk), column
+        float sq = 0.f, sk = 0.f;
+        for (int j = 0; j < vg; ++j) {
+            const long long iv = (rk * vg + j) * D + c;
+            sq += to_f(dq_v[iv]);
+            sk += to_f(dk_v[iv]);
+        }
+        dq[e] = from_f<T>(sq);
+        dk[e] = from_f<T>(sk);
+        if (c == 0) {
+            float sa = 0.f, sb = 0.f;
+            for (int j = 0; j < vg; ++j) { sa += da_v[rk * vg + j]; sb += db_v[rk * vg + j]; }
+            dalpha[rk] = sa;
+            dbeta[rk] = sb;
+        }
+    }
+}
+
+cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da_v, const float* db_v, void* dq,
+                             void* dk, float* dalpha, float* dbeta, long long tokens, int H, int vg, int dk_,
+                             bool is_bf16, cudaStream_t s) {
+    const long long rows_k = tokens * (H / vg);
+    if (rows_k <= 0) return cudaSuccess;
+    long long blocks = (rows_k * dk_ + 255) / 256;
+    if (blocks > 8 * 152) blocks = 8 * 152;
+    if (is_bf16)
+        k_group_sum<bf16><<<(unsigned)blocks, 256, 0, s>>>((const bf16*)dq_v, (const bf16*)dk_v, da_v, db_v, (bf16*)dq,
+                                                          (bf16*)dk, dalpha, dbeta, rows_k, vg, dk_);
+    else
+        k_group_sum<float><<<(unsigned)blocks, 256, 0, s>>>((const float*)dq_v, (const float*)dk_v, da_v, db_v,
+                                                           (float*)dq, (float*)dk, dalpha, dbeta, rows_k, vg, dk_);
+    return cudaGetLastError();
 }
 
 // -------------------------------------------------------------- launchers
@@ -704,7 +749,7 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 1, s);
     ScanArgs a;
-    a.H = p.H; a.N = p.N; a.T = p.T; a.slots = p.slots; a.Ttot = p.Ttot; a.cu = p.cu; a.seq_first = p.seq_first;
+    a.H = p.H; a.vg = p.vg; a.N = p.N; a.T = p.T; a.slots = p.slots; a.Ttot = p.Ttot; a.cu = p.cu; a.seq_first = p.seq_first;
     a.Gb = p.Gb; a.init = p.dhT; a.fin = p.dh0; a.Sout = p.dHb; a.Y = p.Cb; a.reverse = 1; a.err = p.err;
     a.X = tcp ? p.Ab : p.ATb;   // tcgen05 path: Atilde read as an MN-major operand
     a.x_mn = tcp ? 1 : 0;
@@ -719,7 +764,7 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     }
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 3, s);
-    k_reduce_heads<<<p.H, 256, 0, s>>>(p);
+    k_reduce_heads<<<p.H / p.vg, 256, 0, s>>>(p);
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 4, s);
     return cudaSuccess;

@@ -71,26 +71,27 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
     // Comba-pk feedback vectors the tile is [P; K] instead: the Gram's lanes 0..63 hold
     // P K^T, and K (rows 64..127) is the operand of every later product that takes K.
     const bool pk = p.p != nullptr;
+    const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
     {
-        const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
-        const bf16* fg = pk ? (const bf16*)p.p + (t0 * p.H + h) * D : kg;
+        const bf16* kg = (const bf16*)p.k + (t0 * Hk + hk) * D;
+        const bf16* fg = pk ? (const bf16*)p.p + (t0 * Hk + hk) * D : kg;
         for (int e = tid; e < 128 * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < L;
             const bf16* src = r < 64 ? fg : kg;
             cp_async16(sK + sw128_offset(r, ch * 8, 128),
-                       okr ? (const void*)(src + (long long)rr * p.H * D + ch * 8) : (const void*)src, okr);
+                       okr ? (const void*)(src + (long long)rr * Hk * D + ch * 8) : (const void*)src, okr);
         }
     }
     const uint8_t* sKk = pk ? sK + 64 * 128 : sK;   // the 64 key rows (rows 64.. of each K-half for pk)
     load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
     cp_async_commit();
-    if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
+    if (warp == 0) chunk_log_cumsum(p.alpha + t0 * Hk + hk, Hk, L, sG, sGm1);
     if (tid < 64) {
-        const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
+        const float be = tid < L ? p.beta[(t0 + tid) * Hk + hk] : 0.f;
         sBe[tid] = be;
-        const float al = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
-        sBt[tid] = (p.b ? p.b[h] : 1.f) * be * feedback_scale(p.iplr, al);
+        const float al = tid < L ? p.alpha[(t0 + tid) * Hk + hk] : 1.f;
+        sBt[tid] = (p.b ? p.b[hk] : 1.f) * be * feedback_scale(p.iplr, al);
     }
     __syncthreads();   // sG, sGm1, sBt complete
     if (tid < 64) sWs[tid] = sBt[tid] * expf(sGm1[tid]);
@@ -273,6 +274,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     const int L = si.len;
     const long long t0 = si.start;
     const long long idx = (long long)slot * p.H + h;
+    const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
     const int tid = threadIdx.x, warp = tid >> 5;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQK = sm + S::OQK;
@@ -287,12 +289,12 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
 
     {
         // Q into rows 0-63 and K into rows 64-127 of one K-major tile (rows past the chunk zero)
-        const bf16* qg = (const bf16*)p.q + (t0 * p.H + h) * D;
-        const bf16* kg = (const bf16*)p.k + (t0 * p.H + h) * D;
+        const bf16* qg = (const bf16*)p.q + (t0 * Hk + hk) * D;
+        const bf16* kg = (const bf16*)p.k + (t0 * Hk + hk) * D;
         for (int e = tid; e < 128 * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < L;
-            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * p.H * D + ch * 8;
+            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * Hk * D + ch * 8;
             cp_async16(sQK + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
         }
     }
@@ -309,7 +311,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     cp_async_wait<0>();
     __syncthreads();
     // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
-    const float dh = p.d[h];
+    const float dh = p.d[hk];
     for (int e = tid; e < 64 * 16; e += NTH) {
         const int r = e >> 4, ch = e & 15;
         uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
@@ -455,6 +457,7 @@ __global__ void __launch_bounds__(256) k_bwd_prep_tc(ChunkParams p) {
     const int L = si.len;
     const long long t0 = si.start;
     const long long idx = (long long)slot * p.H + h;
+    const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
     const int tid = threadIdx.x, warp = tid >> 5;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQ = sm + S::OQ;
@@ -465,8 +468,8 @@ __global__ void __launch_bounds__(256) k_bwd_prep_tc(ChunkParams p) {
     uint8_t* sdO = sm + S::OD;
     float* sG = reinterpret_cast<float*>(sm + S::OG);
 
-    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
-    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
+    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * Hk + hk) * D, (long long)Hk * D, L, tid, NTH);
+    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * Hk + hk) * D, (long long)Hk * D, L, tid, NTH);
     load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid, NTH);
     load_sw(sdO, 64, D, (const bf16*)p.dO + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
     cp_async_commit();
@@ -478,7 +481,7 @@ __global__ void __launch_bounds__(256) k_bwd_prep_tc(ChunkParams p) {
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
     cp_async_wait<0>();
     __syncthreads();
-    const float dh = p.d[h];
+    const float dh = p.d[hk];
     for (int e = tid; e < 64 * 16; e += NTH) {
         const int r = e >> 4, ch = e & 15;
         uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));

@@ -172,13 +172,14 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                    uP = smem_u32(sP), udE = smem_u32(sdE), udW = smem_u32(sdW), udPh = smem_u32(sdPh),
                    udM = smem_u32(sdM), uY = smem_u32(sY), udG = smem_u32(sdG);
 
+    const int Hk = p.H / p.vg;   // key heads: q, k, alpha, beta, b, d of value head h are key head h / vg's
     auto load_qk = [&](uint8_t* dst, const UnitRef& x) {
-        const bf16* qg = (const bf16*)p.q + (x.t0 * p.H + x.h) * D;
-        const bf16* kg = (const bf16*)p.k + (x.t0 * p.H + x.h) * D;
+        const bf16* qg = (const bf16*)p.q + (x.t0 * Hk + x.h / p.vg) * D;
+        const bf16* kg = (const bf16*)p.k + (x.t0 * Hk + x.h / p.vg) * D;
         for (int e = tid; e < 128 * 16; e += 256) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < x.L;
-            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * p.H * D + ch * 8;
+            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * Hk * D + ch * 8;
             cp_async16(dst + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
         }
     };
@@ -189,8 +190,8 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         if (tid < 64) {
             r.g = p.Gb[x.idx * 64 + tid];
             r.gm1 = tid > 0 ? p.Gb[x.idx * 64 + tid - 1] : 0.f;
-            r.be = tid < x.L ? p.beta[(x.t0 + tid) * p.H + x.h] : 0.f;
-            r.al = tid < x.L ? p.alpha[(x.t0 + tid) * p.H + x.h] : 1.f;
+            r.be = tid < x.L ? p.beta[(x.t0 + tid) * Hk + x.h / p.vg] : 0.f;
+            r.al = tid < x.L ? p.alpha[(x.t0 + tid) * Hk + x.h / p.vg] : 1.f;
         }
         return r;
     };
@@ -267,8 +268,8 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             cp_async_commit();
             rin = load_rows(cur);
         }
-        const float bh = p.b ? p.b[h] : 1.f;
-        const float dh = p.d[h];
+        const float bh = p.b ? p.b[h / p.vg] : 1.f;
+        const float dh = p.d[h / p.vg];
         if (tid < 64) {
             sG[tid] = rin.g;
             sGm1[tid] = rin.gm1;

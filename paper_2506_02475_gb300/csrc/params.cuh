@@ -10,7 +10,9 @@ namespace comba {
 
 struct ChunkParams {
     // problem
-    int B, T, H, dk, dv, N;
+    int B, T, H, dk, dv, N;  // H: value heads; dk, dv: one head's widths
+    int vg;                  // value heads per key head (>= 1): head h takes q, k, p, alpha, beta, b, d
+                             // of key head h / vg; v, o, dO, dv and the chunk states are per value head
     long long Ttot;          // packed tokens (B*T, or T when varlen)
     const int32_t* cu;       // device [N+1] or null (dense: sequence n starts at n*T)
     int slots;               // chunk slots (upper bound on the number of chunks)
@@ -104,6 +106,12 @@ struct GateParams {
 cudaError_t launch_gate_prologue(const GateParams& g, bool is_bf16, int dk, cudaStream_t s);
 cudaError_t launch_gate_epilogue(const GateParams& g, bool is_bf16, int dk, cudaStream_t s);
 
+// Key-side row of (token t, value head h): q, k, p, alpha, beta (and their gradients' scratch
+// indexing stays per value head).
+__host__ __device__ __forceinline__ long long krow(const ChunkParams& p, long long t, int h) {
+    return t * (p.H / p.vg) + h / p.vg;
+}
+
 // Record stage-boundary event i on stream s when instrumentation is on.
 inline void mark(const ChunkParams& p, int i, cudaStream_t s) {
     if (p.ev && i < p.nev) cudaEventRecord(p.ev[i], s);
@@ -123,6 +131,7 @@ struct ScanArgs {
     const void* Y;           // [pairs][dv][dk]
     int reverse;
     int x_mn;                // X is read as an MN-major operand ([k][m] row-major, no transpose)
+    int vg;                  // value heads per key head: init/fin are [N, H / vg, dk, vg * dv]
     int* err;
 };
 cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s);
@@ -156,6 +165,11 @@ size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false)
 cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, const void* q, const void* k,
                                   const void* v, const void* p, const float* alpha, const float* beta,
                                   const float* b, const float* d, float* state, void* o, bool iplr, cudaStream_t s);
+// Value-head groups: sums over the vg value heads of each key head, in a fixed order, of the
+// backward's per-value-head dq, dk [tokens, H, dk] (storage type) and dalpha, dbeta [tokens, H].
+cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da_v, const float* db_v, void* dq,
+                             void* dk, float* dalpha, float* dbeta, long long tokens, int H, int vg, int dk_,
+                             bool is_bf16, cudaStream_t s);
 // Comba-pk correction applied before the chunk kernels: qt = q - d_h p over [rows = tokens*H, dk].
 cudaError_t launch_pk_qtilde(const void* q, const void* p, const float* d, void* qt, long long rows, int H, int dk,
                              bool is_bf16, cudaStream_t s);

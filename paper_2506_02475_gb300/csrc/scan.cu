@@ -30,6 +30,13 @@
 
 namespace comba {
 
+// Offset of the initial / final state of (sequence n, value head h): states are [N, H / vg, dk,
+// vg * dv], so value head h holds the dv-column block h % vg of key head h / vg's rows.
+__device__ __forceinline__ long long state_off(const ScanArgs& a, int n, int h, int DK, int DV) {
+    const int hk = h / a.vg, j = h - hk * a.vg;
+    return ((long long)n * (a.H / a.vg) + hk) * DK * ((long long)a.vg * DV) + (long long)j * DV;
+}
+
 __device__ __forceinline__ void scan_seq_range(const ScanArgs& a, int n, long long& start, long long& len) {
     long long s = a.cu ? a.cu[n] : (long long)n * a.T;
     long long e = a.cu ? a.cu[n + 1] : (long long)(n + 1) * a.T;
@@ -83,9 +90,9 @@ __global__ void __launch_bounds__(256, 1)
     const uint32_t smem_u = smem_u32(smem);
 
     float st[HC];
-    const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
+    const float* init = a.init ? a.init + state_off(a, n, h, DK, DV) : nullptr;
 #pragma unroll
-    for (int m = 0; m < HC; ++m) st[m] = (init && live) ? init[(long long)(c0 + m) * DV + j] : 0.f;
+    for (int m = 0; m < HC; ++m) st[m] = (init && live) ? init[(long long)(c0 + m) * a.vg * DV + j] : 0.f;
 
     long long start, len;
     scan_seq_range(a, n, start, len);
@@ -235,9 +242,9 @@ __global__ void __launch_bounds__(256, 1)
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, DK);
     if (a.fin && live) {
-        float* fin = a.fin + ((long long)n * a.H + h) * DK * DV;
+        float* fin = a.fin + state_off(a, n, h, DK, DV);
 #pragma unroll
-        for (int m = 0; m < HC; ++m) fin[(long long)(c0 + m) * DV + j] = st[m];
+        for (int m = 0; m < HC; ++m) fin[(long long)(c0 + m) * a.vg * DV + j] = st[m];
     }
 }
 
@@ -280,13 +287,13 @@ __global__ void __launch_bounds__(256, 1)
 
     float st[NT][4];
     {
-        const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
+        const float* init = a.init ? a.init + state_off(a, n, h, DK, DV) : nullptr;
 #pragma unroll
         for (int t = 0; t < NT; ++t)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int j = 64 * rhalf + r0 + 8 * (i >> 1), m = cq + 8 * t + (i & 1);
-                st[t][i] = init ? init[(long long)m * DV + j] : 0.f;
+                st[t][i] = init ? init[(long long)m * a.vg * DV + j] : 0.f;
             }
     }
 
@@ -427,13 +434,13 @@ __global__ void __launch_bounds__(256, 1)
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, DK);
     if (a.fin) {
-        float* fin = a.fin + ((long long)n * a.H + h) * DK * DV;
+        float* fin = a.fin + state_off(a, n, h, DK, DV);
 #pragma unroll
         for (int t = 0; t < NT; ++t)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int j = 64 * rhalf + r0 + 8 * (i >> 1), m = cq + 8 * t + (i & 1);
-                fin[(long long)m * DV + j] = st[t][i];
+                fin[(long long)m * a.vg * DV + j] = st[t][i];
             }
     }
 }
@@ -463,13 +470,13 @@ __global__ void __launch_bounds__(128) k_scan_simt(ScanArgs a) {
     float* sY = reinterpret_cast<float*>(smem + S::OY);
 
     float acc[NT][4];
-    const float* init = a.init ? a.init + ((long long)n * a.H + h) * DK * DV : nullptr;
+    const float* init = a.init ? a.init + state_off(a, n, h, DK, DV) : nullptr;
 #pragma unroll
     for (int t = 0; t < NT; ++t)
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int r = j0 + 16 * warp + frag_row(i), m = frag_col(t, i);
-            acc[t][i] = init ? init[(long long)m * DV + r] : 0.f;
+            acc[t][i] = init ? init[(long long)m * a.vg * DV + r] : 0.f;
         }
 
     long long start, len;
@@ -506,13 +513,13 @@ __global__ void __launch_bounds__(128) k_scan_simt(ScanArgs a) {
         __syncthreads();
     }
     if (a.fin) {
-        float* fin = a.fin + ((long long)n * a.H + h) * DK * DV;
+        float* fin = a.fin + state_off(a, n, h, DK, DV);
 #pragma unroll
         for (int t = 0; t < NT; ++t)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int r = j0 + 16 * warp + frag_row(i), m = frag_col(t, i);
-                fin[(long long)m * DV + r] = acc[t][i];
+                fin[(long long)m * a.vg * DV + r] = acc[t][i];
             }
     }
 }

@@ -140,13 +140,15 @@ def make(name: str, *, B=None, T=None, H=None, dk=None, dv=None, dtype=None, see
          with_b=False, with_h0=None, with_grads=None, lengths=None) -> Workload:
     """Build a named workload; keyword arguments shrink or vary it for tests.
 
-    Names: ``tiny_fp32``, ``lm340m``, ``lm1p3b``, ``varlen64k``, ``custom``.
+    Names: ``tiny_fp32``, ``lm340m``, ``lm1p3b``, ``lm1p3b_v256`` (value heads twice as wide as the
+    keys: dk = 128, dv = 256), ``varlen64k``, ``custom``.
     """
     presets = {
         # name: (B, T, H, dk, dv, dtype, h0, grads, offset)
         "tiny_fp32": (1, 256, 2, 64, 64, "f32", False, False, 1),
         "lm340m": (8, 2048, 8, 128, 128, "bf16", False, True, 2),
         "lm1p3b": (4, 4096, 16, 128, 128, "bf16", True, True, 3),
+        "lm1p3b_v256": (4, 4096, 8, 128, 256, "bf16", True, True, 5),
         "varlen64k": (1, 65536, 16, 128, 128, "bf16", False, True, 4),
         "custom": (1, 256, 2, 64, 64, "f32", False, True, 9),
     }

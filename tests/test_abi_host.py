@@ -74,7 +74,8 @@ def test_workspace_size_counts_chunks_and_heads(L):
     assert ws(L, shape(B=1, T=65536, N=12, cu=FAKE)) > ws(L, shape(B=1, T=65536, N=1))
 
 
-@pytest.mark.parametrize("kw", [dict(dk=96), dict(dv=256), dict(chunk=32), dict(H=0), dict(B=0), dict(dtype=7),
+@pytest.mark.parametrize("kw", [dict(dk=96), dict(dv=192), dict(dv=256, dk=64), dict(dv=256, dtype=0), dict(dv=640),
+                                dict(dv=256, flags=8), dict(dv=256, flags=16), dict(chunk=32), dict(H=0), dict(B=0), dict(dtype=7),
                                 dict(B=2, N=3), dict(B=2, cu=FAKE, N=2), dict(T=-1), dict(cu=FAKE + 4, B=1, N=1)])
 def test_invalid_shapes_have_no_workspace(L, kw):
     assert ws(L, shape(**kw)) == 0
@@ -198,3 +199,18 @@ def test_pk_flag_rules(L):
     assert step(p=None) == INVALID
     assert step(flags=16) == INVALID
     assert step(p=FAKE + 4) == INVALID
+
+
+def test_value_head_groups(L):
+    """dv = 256 / 384 / 512 with dk = 128 (bf16) runs as groups of 128-wide value heads: the
+    workspace grows with the value heads (and the backward's per-value-head key-side gradients)."""
+    w128, w256, w512 = (ws(L, shape(dv=d), 1) for d in (128, 256, 512))
+    assert 0 < w128 < w256 < w512
+    assert ws(L, shape(dv=384), 0) > 0
+    assert ws(L, shape(dv=256, H=65535 // 2 + 1)) == 0   # value heads H * 2 beyond the head limit
+
+    def step(dv, dk=128, dtype=1):
+        return L.comba_recurrent_step(4, 2, dk, dv, dtype, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 0,
+                                      None)
+    assert step(256, dk=64) == UNSUPPORTED
+    assert step(384) == UNSUPPORTED
