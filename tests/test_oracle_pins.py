@@ -330,3 +330,34 @@ def test_param_gradients_are_sums_of_token_contributions():
     cdb = ((w.beta * r["dbeta"] - np.einsum("bthd,bthd->bth", w.v, r["dv"])) / w.b).sum((0, 1))
     np.testing.assert_allclose(cdd, r["dd"], rtol=1e-12, atol=1e-12)
     np.testing.assert_allclose(cdb, r["db"], rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("variant", ["splr", "iplr"])
+def test_value_columns_split_into_independent_heads(variant):
+    """The state's dv columns evolve independently given (q, k, gates): a head with dv = 8 equals two
+    heads with dv = 4 that share q, k, alpha, beta, b, d (the value-head-group reading): outputs
+    and dv concatenate, the key-side gradients add, h0/hT/dh0 split by columns."""
+    rng = np.random.default_rng(61)
+    T, H, dk, dv = 70, 2, 5, 8
+    k = rng.standard_normal((1, T, H, dk))
+    k /= np.linalg.norm(k, axis=-1, keepdims=True)
+    p = dict(q=rng.standard_normal((1, T, H, dk)), k=k, v=rng.standard_normal((1, T, H, dv)),
+             alpha=rng.uniform(0.6, 1.0, (1, T, H)), beta=rng.uniform(0.1, 1.0, (1, T, H)), b=rng.uniform(0.2, 0.9, H),
+             d=rng.uniform(-1, 1, H), h0=0.3 * rng.standard_normal((1, H, dk, dv)))
+    dO = rng.standard_normal((1, T, H, dv))
+    dhT = rng.standard_normal((1, H, dk, dv))
+    o, hT = oracle.fwd(**p, variant=variant)
+    g = oracle.bwd(**p, dO=dO, dhT=dhT, variant=variant)
+    halves = [slice(0, 4), slice(4, 8)]
+    parts = []
+    for sl in halves:
+        ph = dict(p, v=p["v"][..., sl], h0=p["h0"][..., sl])
+        oh, hTh = oracle.fwd(**ph, variant=variant)
+        gh = oracle.bwd(**ph, dO=dO[..., sl], dhT=dhT[..., sl], variant=variant)
+        parts.append((oh, hTh, gh))
+    np.testing.assert_allclose(np.concatenate([x[0] for x in parts], -1), o, rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(np.concatenate([x[1] for x in parts], -1), hT, rtol=1e-12, atol=1e-13)
+    for key in ("dv", "dh0"):
+        np.testing.assert_allclose(np.concatenate([x[2][key] for x in parts], -1), g[key], rtol=1e-11, atol=1e-12)
+    for key in ("dq", "dk", "dalpha", "dbeta", "db", "dd"):
+        np.testing.assert_allclose(parts[0][2][key] + parts[1][2][key], g[key], rtol=1e-10, atol=1e-11, err_msg=key)
