@@ -715,8 +715,11 @@ cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da
                              bool is_bf16, cudaStream_t s) {
     const long long rows_k = tokens * (H / vg);
     if (rows_k <= 0) return cudaSuccess;
-    long long blocks = (rows_k * dk_ + 255) / 256;
-    if (blocks > 8 * 152) blocks = 8 * 152;
+    int dev = 0, nsm = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
+    long long blocks = (rows_k * dk_ + 255) / 256;   // grid-stride: at most 8 blocks per SM
+    if (blocks > 8LL * nsm) blocks = 8LL * nsm;
     if (is_bf16)
         k_group_sum<bf16><<<(unsigned)blocks, 256, 0, s>>>((const bf16*)dq_v, (const bf16*)dk_v, da_v, db_v, (bf16*)dq,
                                                           (bf16*)dk, dalpha, dbeta, rows_k, vg, dk_);
@@ -749,7 +752,8 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 1, s);
     ScanArgs a;
-    a.H = p.H; a.vg = p.vg; a.N = p.N; a.T = p.T; a.slots = p.slots; a.Ttot = p.Ttot; a.cu = p.cu; a.seq_first = p.seq_first;
+    a.H = p.H; a.vg = p.vg; a.N = p.N; a.T = p.T; a.slots = p.slots; a.Ttot = p.Ttot; a.cu = p.cu;
+    a.seq_first = p.seq_first;
     a.Gb = p.Gb; a.init = p.dhT; a.fin = p.dh0; a.Sout = p.dHb; a.Y = p.Cb; a.reverse = 1; a.err = p.err;
     a.X = tcp ? p.Ab : p.ATb;   // tcgen05 path: Atilde read as an MN-major operand
     a.x_mn = tcp ? 1 : 0;

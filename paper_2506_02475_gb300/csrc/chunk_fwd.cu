@@ -374,7 +374,8 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     if ((e = cudaGetLastError())) return e;
     mark(q, ev0 + 1, s);
     ScanArgs a;
-    a.H = q.H; a.vg = q.vg; a.N = q.N; a.T = q.T; a.slots = q.slots; a.Ttot = q.Ttot; a.cu = q.cu; a.seq_first = q.seq_first;
+    a.H = q.H; a.vg = q.vg; a.N = q.N; a.T = q.T; a.slots = q.slots; a.Ttot = q.Ttot; a.cu = q.cu;
+    a.seq_first = q.seq_first;
     a.Gb = q.Gb; a.init = q.h0; a.fin = q.hT; a.Sout = q.Hb; a.X = q.Ab; a.Y = q.Bb; a.reverse = 0; a.x_mn = 0;
     a.err = q.err;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)q.slots * q.H, s))) return e;

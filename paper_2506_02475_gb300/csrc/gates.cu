@@ -110,7 +110,8 @@ constexpr int kRingBytes = 200 * 1024;
 // Ring depth: as many stages as fit in kRingBytes, 2..8.
 template <int STAGE_BYTES>
 struct Ring {
-    static constexpr int n = kRingBytes / STAGE_BYTES > 8 ? 8 : (kRingBytes / STAGE_BYTES < 2 ? 2 : kRingBytes / STAGE_BYTES);
+    static constexpr int fit = kRingBytes / STAGE_BYTES;
+    static constexpr int n = fit > 8 ? 8 : (fit < 2 ? 2 : fit);
     static constexpr int bytes = n * STAGE_BYTES;
 };
 

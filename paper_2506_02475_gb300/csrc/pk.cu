@@ -49,7 +49,8 @@ cudaError_t launch_pk_qtilde(const void* q, const void* p, const float* d, void*
     long long grid = (nvec + 256LL * 4 - 1) / (256LL * 4);
     if (grid > 8LL * nsm) grid = 8LL * nsm;
     if (is_bf16)
-        k_pk_qtilde<bf16><<<(unsigned)grid, 256, 0, s>>>((const bf16*)q, (const bf16*)p, d, (bf16*)qt, nvec, vec_per_row, H);
+        k_pk_qtilde<bf16><<<(unsigned)grid, 256, 0, s>>>((const bf16*)q, (const bf16*)p, d, (bf16*)qt, nvec,
+                                                         vec_per_row, H);
     else
         k_pk_qtilde<float><<<(unsigned)grid, 256, 0, s>>>((const float*)q, (const float*)p, d, (float*)qt, nvec,
                                                           vec_per_row, H);
