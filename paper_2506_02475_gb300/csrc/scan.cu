@@ -254,10 +254,12 @@ __global__ void __launch_bounds__(256, 1)
 // back with tcgen05.ld.16x256b, the accumulator arrives in the m16n8 fragment
 // layout, so each thread keeps 32 state values (rows 16 (w & 3) + g, + 8; columns
 // 64 (w >> 2) + 8 t + 2 q, + 1).  Per chunk each SM loads X plus half of Y and
-// stores half of the chunk state, and the epilogue is half as long.
+// stores half of the chunk state, and the epilogue is half as long.  X and Y each
+// stream three chunks deep; one thread issues the MMAs while another issues the TMA
+// stores and loads, so a step's critical path is the MMA, not the issue sequence.
 template <int DK, int DV>
 struct ScanSplitSmem {
-    static constexpr int SX = 3, SY = 2;
+    static constexpr int SX = 3, SY = 3;
     static constexpr uint32_t A_BYTES = 64 * DK * 2;    // this CTA's 64 rows of S^T; two buffers
     static constexpr uint32_t X_BYTES = DK * DK * 2;
     static constexpr uint32_t Y_BYTES = 64 * DK * 2;
@@ -335,8 +337,11 @@ __global__ void __launch_bounds__(256, 1)
         for (int half = 0; half < DK / 64; ++half)
             tma_load_2d(smem_u + y_off(it) + half * 64 * 128, &tmY, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), fb);
     };
+    // Thread 0 issues the MMAs; thread 32 (warp 1) the TMA traffic: the chunk-state stores, the
+    // X / Y loads and the bulk-group waits, so neither waits for the other's issue sequence.
+    constexpr int kTma = 32;
     int nx = 0, ny = 0;
-    if (tid == 0) {
+    if (tid == kTma) {
         for (; nx < S::SX - 1 && nx < nch; ++nx) issue_x(nx);
         for (; ny < S::SY - 1 && ny < nch; ++ny) issue_y(ny);
     }
@@ -380,6 +385,7 @@ __global__ void __launch_bounds__(256, 1)
                 bad = 1;
             }
             tc_commit(smem_u32(&mma_bar));
+        } else if (tid == kTma) {
 #pragma unroll
             for (int half = 0; half < DK / 64; ++half)
                 tma_store_2d(&tmS, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), a_buf(it) + half * 64 * 128);
@@ -389,9 +395,9 @@ __global__ void __launch_bounds__(256, 1)
         }
         if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
         if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1)) bad = 1;
-        if (tid == 0) bulk_wait_read<1>();
+        if (tid == kTma) bulk_wait_read<1>();
         if (__syncthreads_or(bad)) {
-            if (tid == 0) {
+            if (tid == kTma) {
                 if (a.err) atomicExch(a.err, 1);
                 for (int c = it; c < nx; ++c) mbar_wait(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
                 for (int c = it; c < ny; ++c) mbar_wait(smem_u32(&full_y[c % S::SY]), (c / S::SY) & 1);
@@ -429,7 +435,7 @@ __global__ void __launch_bounds__(256, 1)
         tc_fence_before();
     }
 
-    if (tid == 0) bulk_wait_all();
+    if (tid == kTma) bulk_wait_all();
     __syncthreads();
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, DK);
