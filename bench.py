@@ -62,21 +62,32 @@ def fwd_flops_per_token_head(C=64, dk=128, dv=128):
 def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False):
     """`tc`: the tcgen05 path (bf16, d=128), whose reverse scan reads Atilde itself, so
     the forward saves M but no Atilde^T.  `pk`: Comba-pk feedback vectors P, read by prep and
-    by the local gradients, which also write dP."""
+    by the local gradients, which also write dP.  At dk = 256 no chunk map is formed: the
+    scans read W, K and U (forward) or C^T (backward) and form two products per chunk."""
     C, es, f4 = 64, 2, 4
     P = slots * H
-    at = save and not tc
+    wide = dk > 128
+    at = save and not tc and not wide
+    mp = 0 if wide else 1   # the chunk map Atilde, B^T
     m = {}
-    m["prep"] = dict(flops=P * (2 * C * C * (2 * dk + dv) + 2 * dk * C * dk * (2 if at else 1) + 2 * dv * C * dk),
-                     bytes=P * (C * (dk + dv) * es + 2 * C * f4 + C * (dk + dv) * es + C * f4 + dk * dk * es
-                                + dv * dk * es + (C * C * es if save else 0) + (dk * dk * es if at else 0)))
-    m["scan_fwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
+    m["prep"] = dict(flops=P * (2 * C * C * (2 * dk + dv)
+                                + mp * (2 * dk * C * dk * (2 if at else 1) + 2 * dv * C * dk)),
+                     bytes=P * (C * (dk + dv) * es + 2 * C * f4 + C * (dk + dv) * es + C * f4
+                                + mp * (dk * dk * es + dv * dk * es) + (C * C * es if save else 0)
+                                + (dk * dk * es if at else 0)))
+    if wide:
+        m["scan_fwd"] = dict(flops=P * 4 * C * dk * dv, bytes=P * ((2 * C * dk + C * dv + dv * dk) * es + C * f4))
+    else:
+        m["scan_fwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
     m["output"] = dict(flops=P * (4 * C * dk * dv + 2 * C * C * (dk + dv)),
                        bytes=P * (3 * C * dk * es + C * dv * es + dv * dk * es + C * dv * es * (2 if save else 1)
                                   + C * f4))
     m["bwd_prep"] = dict(flops=P * (4 * C * C * dk + 2 * dv * C * dk),
                          bytes=P * (3 * C * dk * es + C * dv * es + dv * dk * es + C * f4))
-    m["scan_bwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
+    if wide:
+        m["scan_bwd"] = dict(flops=P * 4 * C * dk * dv, bytes=P * ((2 * C * dk + 2 * dv * dk) * es + C * f4))
+    else:
+        m["scan_bwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
     m["bwd_local"] = dict(flops=P * (2 * C * C * dk * 9 + 2 * C * dk * dv * 4 + 2 * C * C * dv * 4 + 4 * C ** 3),
                           bytes=P * (C * (2 * dk + 2 * dv) * es + C * dv * es + 2 * dv * dk * es + C * C * es
                                      + 3 * C * f4 + C * (2 * dk + dv) * es + 2 * C * f4))
@@ -445,9 +456,9 @@ def run_ours(args, world, rank, local):
 
     # ---- dominant kernel and its roofline
     slots = (tokens // 64 + N) if w.cu_seqlens is not None else w.q.shape[0] * ((w.q.shape[1] + 63) // 64)
-    # value-head groups: dv beyond 128 runs as dv / 128 value heads of width 128 per key head, and
-    # every kernel's unit is a (chunk, value head) pair
-    vg = dv // 128 if dv > 128 else 1
+    # value-head groups: dv beyond 128 runs as dv / 128 value heads of width 128 per key head (at
+    # dk = 256: value heads 64 wide), and every kernel's unit is a (chunk, value head) pair
+    vg = dv // 64 if dk == 256 else (dv // 128 if dv > 128 else 1)
     dv_u, H_u = dv // vg, H * vg
     tc = w.dtype == "bf16" and dk == 128 and dv_u == 128
     model = stage_model(dk, dv_u, slots, H_u, N, tc=tc, pk=pk)
@@ -876,7 +887,8 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="lm1p3b", choices=["lm1p3b", "lm340m", "varlen64k", "lm1p3b_v256", "decode"])
+    ap.add_argument("--workload", default="lm1p3b",
+                    choices=["lm1p3b", "lm340m", "varlen64k", "lm1p3b_v256", "lm1p3b_d256", "decode"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--gated", action="store_true",
                     help="raw q, k and gate pre-activations through the gate and normalisation prologue")

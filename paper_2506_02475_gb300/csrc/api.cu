@@ -22,7 +22,7 @@ struct Layout {
     size_t qh, kh, ga, gb, bg, dqh, dkh, dal, dbe, dbi, dar, dcr, dpa, dpc;
     // Comba-pk (COMBA_PK): the corrected queries q - d p and the zero d the chunk kernels then see
     size_t qt, dz;
-    // value-head groups (dv = vg * 128, vg > 1): the backward's per-value-head dq, dk, dalpha, dbeta
+    // value-head groups (vg > 1): the backward's per-value-head dq, dk, dalpha, dbeta
     size_t gdq, gdk, gda, gdb;
     size_t total;
     int slots;
@@ -30,8 +30,16 @@ struct Layout {
 };
 
 // Value heads per key head: dv beyond 128 (a multiple of 128, dk = 128, bf16, plain or iplr
-// form) runs as dv / 128 value heads of width 128 that share the key head's q, k and gates.
-int value_groups(const comba_shape_t* s) { return s->dv > 128 ? s->dv / 128 : 1; }
+// form) runs as dv / 128 value heads of width 128 that share the key head's q, k and gates;
+// at head dim dk = 256 the value heads are 64 wide (dv = 64 .. 256).
+int value_groups(const comba_shape_t* s) {
+    if (s->dk == 256) return s->dv >= 64 ? s->dv / 64 : 1;
+    return s->dv > 128 ? s->dv / 128 : 1;
+}
+
+// Key widths with a chunk map Atilde (dk x dk) in the workspace; at dk = 256 the scan forms
+// E = U - W H per chunk instead.
+bool has_chunk_map(int dk) { return dk <= 128; }
 
 // Validates the shape (not the pointers) and computes the workspace layout.
 // The forward needs W, U, G, Atilde, B^T and the chunk states; saving for the
@@ -43,7 +51,11 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (s->dtype != COMBA_F32 && s->dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
     if (s->chunk != comba::kChunk) return COMBA_ERR_UNSUPPORTED;
     const int vg = value_groups(s);
-    if (vg > 1) {
+    if (s->dk == 256) {
+        // head dim 256 (bf16, plain or iplr form): value heads 64 wide, at most four per key head
+        if (s->dtype != COMBA_BF16 || s->dv < 64 || s->dv % 64 != 0 || vg > 4) return COMBA_ERR_UNSUPPORTED;
+        if (s->flags & (COMBA_GATED | COMBA_PK)) return COMBA_ERR_UNSUPPORTED;
+    } else if (vg > 1) {
         // dv = 256, 384 or 512 as groups of 128-wide value heads on the tcgen05 path
         if (s->dv % 128 != 0 || vg > 4 || s->dk != 128 || s->dtype != COMBA_BF16) return COMBA_ERR_UNSUPPORTED;
         if (s->flags & (COMBA_GATED | COMBA_PK)) return COMBA_ERR_UNSUPPORTED;
@@ -78,14 +90,17 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     L.W = take(pairs * 64 * dk * es);
     L.U = take(pairs * 64 * dv * es);
     L.G = take(pairs * 64 * sizeof(float));
-    L.A = take(pairs * dk * dk * es);
-    L.B = take(pairs * dv * dk * es);
+    if (has_chunk_map(s->dk)) {
+        L.A = take(pairs * dk * dk * es);
+        L.B = take(pairs * dv * dk * es);
+    }
     L.Hs = take(pairs * dv * dk * es);
     if (backward) {
         L.E = take(pairs * 64 * dv * es);
         L.M = take(pairs * 64 * 64 * es);
         // Atilde^T is only materialised off the tcgen05 path (that reverse scan reads Atilde directly)
-        if (!comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv)) L.AT = take(pairs * dk * dk * es);
+        if (has_chunk_map(s->dk) && !comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv))
+            L.AT = take(pairs * dk * dk * es);
         L.C = take(pairs * dv * dk * es);
         L.dH = take(pairs * dv * dk * es);
         L.part = take(pairs * 2 * sizeof(float));
@@ -160,13 +175,14 @@ void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* 
     p.Wb = w + L.W;
     p.Ub = w + L.U;
     p.Gb = reinterpret_cast<float*>(w + L.G);
-    p.Ab = w + L.A;
-    p.Bb = w + L.B;
+    // (offset 0 is the status word, so a zero offset marks a region that is not allocated)
+    p.Ab = L.A ? w + L.A : nullptr;
+    p.Bb = L.B ? w + L.B : nullptr;
     p.Hb = w + L.Hs;
     if (backward_layout) {
         p.Eb = w + L.E;
         p.Mb = w + L.M;
-        p.ATb = comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv) ? nullptr : w + L.AT;
+        p.ATb = L.AT ? w + L.AT : nullptr;
         p.Cb = w + L.C;
         p.dHb = w + L.dH;
         p.part = reinterpret_cast<float*>(w + L.part);
@@ -270,6 +286,12 @@ comba_status_t backward_run(const comba_shape_t* shape, const Layout& L, void* w
                                             p.dk, bf, s) != cudaSuccess)
         return COMBA_ERR_CUDA;
     return COMBA_OK;
+}
+
+// Decode head widths: dk in {64, 128, 256}; dv in {64, 128}, or 256 with dk >= 128.
+bool step_dims_ok(int dk, int dv) {
+    if (dk != 64 && dk != 128 && dk != 256) return false;
+    return dv == 64 || dv == 128 || (dv == 256 && dk >= 128);
 }
 
 comba::GateParams gate_params(const comba_shape_t* shape, const Layout& L, void* workspace, const void* q,
@@ -464,7 +486,7 @@ comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtyp
     if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
     if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
     if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
-    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128 && !(dv == 256 && dk == 128))) return COMBA_ERR_UNSUPPORTED;
+    if (!step_dims_ok(dk, dv)) return COMBA_ERR_UNSUPPORTED;
     if ((long long)Bd * H * (dv / 32) >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(p); COMBA_REQUIRE(alpha);
     COMBA_REQUIRE(beta); COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
@@ -482,7 +504,7 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
     if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
     if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
     if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
-    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128 && !(dv == 256 && dk == 128))) return COMBA_ERR_UNSUPPORTED;
+    if (!step_dims_ok(dk, dv)) return COMBA_ERR_UNSUPPORTED;
     if ((long long)Bd * H * (dv / 32) >= (1LL << 31)) return COMBA_ERR_UNSUPPORTED;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);

@@ -77,15 +77,16 @@ __global__ void __launch_bounds__(128) k_bwd_prep(ChunkParams p) {
     T* sP = reinterpret_cast<T*>(smem + S::OP);
     float* sG = reinterpret_cast<float*>(smem + S::OG);
 
-    load_tile_async<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-    load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;   // key-side rows
+    load_tile_async<T>(sQ, S::PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 128);
+    load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
     load_tile_async<T>(sdO, S::PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
     cp_async_commit();
     if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
     cp_async_wait<0>();
     __syncthreads();
-    const float dd = p.d[h];
+    const float dd = p.d[h / p.vg];
     for (int e = tid; e < 64 * DK; e += 128) {
         const int r = e / DK, c = e % DK;
         sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dd * to_f(sK[r * S::PK + c]));
@@ -163,7 +164,6 @@ struct LocalSmem {
         o = carve_bytes(o, sizeof(T) * DV * PK);   // H^T
         o = carve_bytes(o, sizeof(T) * DV * PK);   // dH'^T
         o = carve_bytes(o, sizeof(T) * 64 * PL);   // M
-        o = carve_bytes(o, sizeof(T) * 64 * PV);   // dV staging (coalesced store at the end)
         o = carve_bytes(o, sizeof(float) * 64 * 8);          // G, Gm1, beta, btilde, alpha, dg, e^{Gm1}, btilde e^{Gm1}
         o = carve_bytes(o, sizeof(float) * NROW * 2 * 64);   // row partials [kind][half][row]
         o = carve_bytes(o, sizeof(float) * 2 * 4 * 64);      // column partials [kind][rowblock][col]
@@ -216,7 +216,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     T* sH = sc.take<T>(DV * PK);    // H_n^T  [dv][dk]
     T* sdH = sc.take<T>(DV * PK);   // dH'^T  [dv][dk]
     T* sM = sc.take<T>(64 * PL);
-    T* sDV = sc.take<T>(64 * PV);
+    T* sDV = sV;   // dV is staged in the V tile once phase A has read V
     float* sG = sc.take<float>(64 * 8);
     float* sGm1 = sG + 64;
     float* sBe = sG + 128;
@@ -235,10 +235,12 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     T* sY = sdE;
     T* sdG = sH;
 
-    const float bh = p.b ? p.b[h] : 1.f;
-    const float dh = p.d[h];
-    load_tile_async<T>(sK, PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
-    load_tile_async<T>(sQ, PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
+    const int hk = h / p.vg;   // key head: q, k, p, alpha, beta, b, d
+    const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;
+    const float bh = p.b ? p.b[hk] : 1.f;
+    const float dh = p.d[hk];
+    load_tile_async<T>(sK, PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 256);
+    load_tile_async<T>(sQ, PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 256);
     load_tile_async<T>(sV, PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
     load_tile_async<T>(sdO, PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
     load_tile_async<T>(sE, PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
@@ -249,11 +251,12 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     if (tid < 64) {
         sG[tid] = p.Gb[idx * 64 + tid];
         sGm1[tid] = tid > 0 ? p.Gb[idx * 64 + tid - 1] : 0.f;
-        const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
+        const float be = tid < L ? p.beta[krow(p, t0 + tid, h)] : 0.f;
         sBe[tid] = be;
-        const float fsc = feedback_scale(p.iplr, tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f);
+        const float al = tid < L ? p.alpha[krow(p, t0 + tid, h)] : 1.f;
+        const float fsc = feedback_scale(p.iplr, al);
         sBt[tid] = bh * be * fsc;
-        sAl[tid] = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
+        sAl[tid] = al;
         const float em1 = tid > 0 ? __expf(p.Gb[idx * 64 + tid - 1]) : 1.f;
         sEm1[tid] = em1;
         sWs[tid] = bh * be * fsc * em1;
@@ -366,7 +369,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     if constexpr (PKV) {
         __syncthreads();
         sF = sdH;
-        load_tile_async<T>(sF, PK, (const T*)p.p + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 256);
+        load_tile_async<T>(sF, PK, (const T*)p.p + kr0 * DK, kld, 64, DK, L, tid, 256);
         cp_async_commit();
     }
     {
@@ -408,6 +411,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         const float ba = sBe[ra], bb = sBe[rb];
 #pragma unroll
         for (int t = 0; t < NV; ++t) { tv[t][0] *= ba; tv[t][1] *= ba; tv[t][2] *= bb; tv[t][3] *= bb; }
+        __syncthreads();   // every warp has read V (dM, the row dots) before dV replaces it
         frag_store<T, NV>(sDV, PV, m0, nv0, tv);
     }
     if constexpr (PKV) cp_async_wait<0>();
@@ -507,7 +511,7 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         warp_gemm<true, false, NK>(acc_dq, sdPh, PL, sK, PK, m0, nk0, 64);
 
         float t0r[NK][4];
-        const float dfb = PKV ? p.d_fb[h] : 0.f;
+        const float dfb = PKV ? p.d_fb[hk] : 0.f;
 #pragma unroll
         for (int t = 0; t < NK; ++t)
 #pragma unroll
@@ -757,6 +761,7 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     a.Gb = p.Gb; a.init = p.dhT; a.fin = p.dh0; a.Sout = p.dHb; a.Y = p.Cb; a.reverse = 1; a.err = p.err;
     a.X = tcp ? p.Ab : p.ATb;   // tcgen05 path: Atilde read as an MN-major operand
     a.x_mn = tcp ? 1 : 0;
+    a.W = p.Wb; a.K = p.k;      // dk = 256: dH = gamma dH' + C - W^T Kbar dH' per chunk
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)p.slots * p.H, s))) return e;
     mark(p, ev0 + 2, s);
     if (tcp && !pk) {
@@ -780,6 +785,7 @@ cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int e
         if (p.dk == 128 && p.dv == 64) return run_bwd<bf16, 128, 64>(p, s, ev0);
         if (p.dk == 64 && p.dv == 128) return run_bwd<bf16, 64, 128>(p, s, ev0);
         if (p.dk == 64 && p.dv == 64) return run_bwd<bf16, 64, 64>(p, s, ev0);
+        if (p.dk == 256 && p.dv == 64) return run_bwd<bf16, 256, 64>(p, s, ev0);
     } else {
         if (p.dk == 64 && p.dv == 64) return run_bwd<float, 64, 64>(p, s, ev0);
     }
@@ -793,6 +799,7 @@ size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk) {
     if (dk == DK && dv == DV) return kernel == 0 ? BPrepSmem<T, DK, DV>::bytes() : LocalSmem<T, DK, DV>::bytes();
     if (is_bf16) {
         COMBA_SM(bf16, 128, 128) COMBA_SM(bf16, 128, 64) COMBA_SM(bf16, 64, 128) COMBA_SM(bf16, 64, 64)
+        COMBA_SM(bf16, 256, 64)
     } else {
         COMBA_SM(float, 64, 64)
     }

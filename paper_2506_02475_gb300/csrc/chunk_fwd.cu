@@ -175,17 +175,17 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     // feedback vectors: P for Comba-pk (Gram P K^T, W = M Diag P), else K itself
     T* sF = p.p ? reinterpret_cast<T*>(smem + S::OP) : sK;
 
-    load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-    if (p.p)
-        load_tile_async<T>(sF, S::PK, (const T*)p.p + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;   // key-side rows
+    load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
+    if (p.p) load_tile_async<T>(sF, S::PK, (const T*)p.p + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
     cp_async_commit();
-    if (warp == 0) chunk_log_cumsum(p.alpha + t0 * p.H + h, p.H, L, sG, sGm1);
+    if (warp == 0) chunk_log_cumsum(p.alpha + kr0, p.H / p.vg, L, sG, sGm1);
     if (tid < 64) {
-        const float be = tid < L ? p.beta[(t0 + tid) * p.H + h] : 0.f;
+        const float be = tid < L ? p.beta[krow(p, t0 + tid, h)] : 0.f;
         sBe[tid] = be;
-        const float al = tid < L ? p.alpha[(t0 + tid) * p.H + h] : 1.f;
-        sBt[tid] = (p.b ? p.b[h] : 1.f) * be * feedback_scale(p.iplr, al);
+        const float al = tid < L ? p.alpha[krow(p, t0 + tid, h)] : 1.f;
+        sBt[tid] = (p.b ? p.b[h / p.vg] : 1.f) * be * feedback_scale(p.iplr, al);
     }
     cp_async_wait<0>();
     __syncthreads();
@@ -223,32 +223,39 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     __syncthreads();
 
     // W = Mw P, U = Mu V (stored) and their Kbar-row-scaled copies for the chunk's state map.
+    // At dk = 256 the scan applies E = U - W H itself and no map is formed.
+    constexpr bool kMap = DK <= 128;
     const float sa = sS[16 * warp + frag_row(0)], sb = sS[16 * warp + frag_row(2)];
     {
         float acc[DK / 8][4];
         zero(acc);
         warp_gemm<true, false, DK / 8>(acc, sMw, S::PL, sF, S::PK, 16 * warp, 0, 64);
         frag_store_global<T, DK / 8>((T*)p.Wb + idx * 64 * DK, DK, 16 * warp, 0, acc, 64);
+        if constexpr (kMap) {
 #pragma unroll
-        for (int t = 0; t < DK / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
-        frag_store<T, DK / 8>(sWs, S::PK, 16 * warp, 0, acc);
+            for (int t = 0; t < DK / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
+            frag_store<T, DK / 8>(sWs, S::PK, 16 * warp, 0, acc);
+        }
     }
     {
         float acc[DV / 8][4];
         zero(acc);
         warp_gemm<true, false, DV / 8>(acc, sMu, S::PL, sV, S::PV, 16 * warp, 0, 64);
         frag_store_global<T, DV / 8>((T*)p.Ub + idx * 64 * DV, DV, 16 * warp, 0, acc, 64);
+        if constexpr (kMap) {
 #pragma unroll
-        for (int t = 0; t < DV / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
-        frag_store<T, DV / 8>(sUs, S::PV, 16 * warp, 0, acc);
+            for (int t = 0; t < DV / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
+            frag_store<T, DV / 8>(sUs, S::PV, 16 * warp, 0, acc);
+        }
     }
-    __syncthreads();
-
-    // Atilde = -K^T Diag(s) W  [dk][dk];  B^T = (Diag(s) U)^T K  [dv][dk];  Atilde^T = -(Diag(s) W)^T K.
-    gemm_to_global<T, false, false, DK, DK>((T*)p.Ab + idx * DK * DK, sK, S::PK, sWs, S::PK, 64, -1.f, warp);
-    gemm_to_global<T, false, false, DV, DK>((T*)p.Bb + idx * DV * DK, sUs, S::PV, sK, S::PK, 64, 1.f, warp);
-    if (p.ATb)
-        gemm_to_global<T, false, false, DK, DK>((T*)p.ATb + idx * DK * DK, sWs, S::PK, sK, S::PK, 64, -1.f, warp);
+    if constexpr (kMap) {
+        __syncthreads();
+        // Atilde = -K^T Diag(s) W  [dk][dk];  B^T = (Diag(s) U)^T K  [dv][dk];  Atilde^T = -(Diag(s) W)^T K.
+        gemm_to_global<T, false, false, DK, DK>((T*)p.Ab + idx * DK * DK, sK, S::PK, sWs, S::PK, 64, -1.f, warp);
+        gemm_to_global<T, false, false, DV, DK>((T*)p.Bb + idx * DV * DK, sUs, S::PV, sK, S::PK, 64, 1.f, warp);
+        if (p.ATb)
+            gemm_to_global<T, false, false, DK, DK>((T*)p.ATb + idx * DK * DK, sWs, S::PK, sK, S::PK, 64, -1.f, warp);
+    }
 }
 
 // ---------------------------------------------------------------- output
@@ -286,8 +293,9 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     T* sH = reinterpret_cast<T*>(smem + S::OH);
     float* sG = reinterpret_cast<float*>(smem + S::OG);
 
-    load_tile_async<T>(sQ, S::PK, (const T*)p.q + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
-    load_tile_async<T>(sK, S::PK, (const T*)p.k + (t0 * p.H + h) * DK, (long long)p.H * DK, 64, DK, L, tid, 128);
+    const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;   // key-side rows
+    load_tile_async<T>(sQ, S::PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 128);
+    load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
     load_tile_async<T>(sU, S::PV, (const T*)p.Ub + idx * 64 * DV, DV, 64, DV, 64, tid, 128);
     load_tile_async<T>(sH, S::PK, (const T*)p.Hb + idx * DV * DK, DK, DV, DK, DV, tid, 128);
@@ -311,7 +319,7 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
         if (p.Eb) frag_store_global<T, DV / 8>((T*)p.Eb + idx * 64 * DV, DV, 16 * warp, 0, e, 64);
         frag_store<T, DV / 8>(sE, S::PV, 16 * warp, 0, e);
     }
-    const float dh = p.d[h];
+    const float dh = p.d[h / p.vg];
     for (int e = tid; e < 64 * DK; e += 128) {
         const int r = e / DK, c = e % DK;
         sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dh * to_f(sK[r * S::PK + c]));
@@ -377,6 +385,8 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     a.H = q.H; a.vg = q.vg; a.N = q.N; a.T = q.T; a.slots = q.slots; a.Ttot = q.Ttot; a.cu = q.cu;
     a.seq_first = q.seq_first;
     a.Gb = q.Gb; a.init = q.h0; a.fin = q.hT; a.Sout = q.Hb; a.X = q.Ab; a.Y = q.Bb; a.reverse = 0; a.x_mn = 0;
+    a.W = q.Wb; a.K = q.k;
+    if (DK == 256) a.Y = q.Ub;   // the wide scan forms E = U - W H itself
     a.err = q.err;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)q.slots * q.H, s))) return e;
     mark(q, ev0 + 2, s);
@@ -402,6 +412,7 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
     if (p.dk == DK && p.dv == DV) return run_fwd<T, DK, DV>(p, save, s, ev0);
     if (is_bf16) {
         COMBA_FWD(bf16, 128, 128) COMBA_FWD(bf16, 128, 64) COMBA_FWD(bf16, 64, 128) COMBA_FWD(bf16, 64, 64)
+        COMBA_FWD(bf16, 256, 64)
     } else {
         COMBA_FWD(float, 128, 128) COMBA_FWD(float, 128, 64) COMBA_FWD(float, 64, 128) COMBA_FWD(float, 64, 64)
     }
@@ -416,6 +427,7 @@ size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk) {
     if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes(pk) : OutSmem<T, DK, DV>::bytes();
     if (is_bf16) {
         COMBA_SM(bf16, 128, 128) COMBA_SM(bf16, 128, 64) COMBA_SM(bf16, 64, 128) COMBA_SM(bf16, 64, 64)
+        COMBA_SM(bf16, 256, 64)
     } else {
         COMBA_SM(float, 128, 128) COMBA_SM(float, 128, 64) COMBA_SM(float, 64, 128) COMBA_SM(float, 64, 64)
     }

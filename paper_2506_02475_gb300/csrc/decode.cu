@@ -113,10 +113,10 @@ cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, c
     if (dk == DK && dv == DV) return run_step<T, DK, DV>(Bd, H, q, k, v, p, alpha, beta, b, d, state, o, iplr, s);
     if (is_bf16) {
         COMBA_STEP(bf16, 128, 128) COMBA_STEP(bf16, 128, 64) COMBA_STEP(bf16, 64, 128) COMBA_STEP(bf16, 64, 64)
-        COMBA_STEP(bf16, 128, 256)
+        COMBA_STEP(bf16, 128, 256) COMBA_STEP(bf16, 256, 64) COMBA_STEP(bf16, 256, 128) COMBA_STEP(bf16, 256, 256)
     } else {
         COMBA_STEP(float, 128, 128) COMBA_STEP(float, 128, 64) COMBA_STEP(float, 64, 128) COMBA_STEP(float, 64, 64)
-        COMBA_STEP(float, 128, 256)
+        COMBA_STEP(float, 128, 256) COMBA_STEP(float, 256, 64) COMBA_STEP(float, 256, 128) COMBA_STEP(float, 256, 256)
     }
 #undef COMBA_STEP
     return cudaErrorInvalidValue;

@@ -128,7 +128,9 @@ struct ScanArgs {
     float* fin;              // [N,H,dk,dv] final state (hT or dh0) or null
     void* Sout;              // [pairs][dv][dk] state each chunk starts from (storage type)
     const void* X;           // [pairs][dk][dk] row-major
-    const void* Y;           // [pairs][dv][dk]
+    const void* Y;           // [pairs][dv][dk]; at dk = 256 the forward's is U [pairs][64][dv] instead
+    const void* W;           // dk = 256: the chunks' W [pairs][64][dk] and the keys [tokens, H / vg, dk]
+    const void* K;           //           (the scan applies E = U - W H per chunk instead of Atilde)
     int reverse;
     int x_mn;                // X is read as an MN-major operand ([k][m] row-major, no transpose)
     int vg;                  // value heads per key head: init/fin are [N, H / vg, dk, vg * dv]
@@ -136,6 +138,9 @@ struct ScanArgs {
 };
 cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s);
 size_t scan_smem_bytes(bool is_bf16, int dk, int dv);
+// dk = 256 (bf16, value heads 64 wide): the scan of scan_wide.cu
+cudaError_t launch_scan_wide(const ScanArgs& a, cudaStream_t s);
+size_t scan_wide_smem_bytes();
 
 // Kernel launchers (one translation unit each); return cudaGetLastError().
 cudaError_t launch_chunk_map(const ChunkParams& p, cudaStream_t s);

@@ -602,6 +602,7 @@ static cudaError_t run_scan_simt(const ScanArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s) {
+    if (dk == 256) return is_bf16 && dv == 64 ? launch_scan_wide(a, s) : cudaErrorInvalidValue;
 #define COMBA_SCAN(DK, DV)                                                                          \
     if (dk == DK && dv == DV)                                                                        \
         return !is_bf16 ? run_scan_simt<DK, DV>(a, s)                                                \
@@ -612,6 +613,7 @@ cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long lo
 }
 
 size_t scan_smem_bytes(bool is_bf16, int dk, int dv) {
+    if (dk == 256) return is_bf16 && dv == 64 ? scan_wide_smem_bytes() : 0;
     if (is_bf16) {
         if (dk == 128) return dv == 128 ? ScanSplitSmem<128, 128>::bytes() : ScanTcSmem<128, 64>::bytes();
         return dv == 128 ? ScanTcSmem<64, 128>::bytes() : ScanTcSmem<64, 64>::bytes();

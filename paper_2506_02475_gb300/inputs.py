@@ -141,7 +141,8 @@ def make(name: str, *, B=None, T=None, H=None, dk=None, dv=None, dtype=None, see
     """Build a named workload; keyword arguments shrink or vary it for tests.
 
     Names: ``tiny_fp32``, ``lm340m``, ``lm1p3b``, ``lm1p3b_v256`` (value heads twice as wide as the
-    keys: dk = 128, dv = 256), ``varlen64k``, ``custom``.
+    keys: dk = 128, dv = 256), ``lm1p3b_d256`` (head dim 256: dk = dv = 256, half the heads),
+    ``varlen64k``, ``custom``.
     """
     presets = {
         # name: (B, T, H, dk, dv, dtype, h0, grads, offset)
@@ -149,6 +150,7 @@ def make(name: str, *, B=None, T=None, H=None, dk=None, dv=None, dtype=None, see
         "lm340m": (8, 2048, 8, 128, 128, "bf16", False, True, 2),
         "lm1p3b": (4, 4096, 16, 128, 128, "bf16", True, True, 3),
         "lm1p3b_v256": (4, 4096, 8, 128, 256, "bf16", True, True, 5),
+        "lm1p3b_d256": (4, 4096, 8, 256, 256, "bf16", True, True, 6),
         "varlen64k": (1, 65536, 16, 128, 128, "bf16", False, True, 4),
         "custom": (1, 256, 2, 64, 64, "f32", False, True, 9),
     }

@@ -214,3 +214,19 @@ def test_value_head_groups(L):
                                       None)
     assert step(256, dk=64) == UNSUPPORTED
     assert step(384) == UNSUPPORTED
+
+
+def test_head_dim_256(L):
+    """dk = 256 (bf16, plain or iplr) runs as value heads 64 wide: dv = 64 .. 256 in steps of 64."""
+    w64, w128, w256 = (ws(L, shape(dk=256, dv=d), 1) for d in (64, 128, 256))
+    assert 0 < w64 < w128 < w256
+    assert ws(L, shape(dk=256, dv=192), 0) > 0
+    assert ws(L, shape(dk=256, dv=64, flags=4), 1) > 0
+    for kw in (dict(dv=320), dict(dv=32), dict(dv=96), dict(dtype=0), dict(flags=8), dict(flags=16)):
+        assert ws(L, shape(dk=256, **kw)) == 0, kw
+
+    def step(dv, dk=256):
+        return L.comba_recurrent_step(4, 2, dk, dv, 1, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 0,
+                                      None)
+    assert step(384) == UNSUPPORTED
+    assert step(256, dk=64) == UNSUPPORTED
