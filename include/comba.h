@@ -40,6 +40,15 @@
  *     as their workspaces and outputs are distinct.
  *   - Results are bitwise reproducible from run to run (fixed reduction order,
  *     no floating-point atomics).
+ *
+ * Head widths (chunk entry points; comba_workspace_size returns 0 for the rest)
+ *   - dk, dv in {64, 128}, either storage type (the fp32 backward: dk = dv = 64).
+ *   - dk = 128 with dv = 256, 384 or 512 (bf16, plain or iplr form): each head
+ *     runs as dv / 128 value heads of width 128 that share its q, k and gates
+ *     (a state's columns evolve independently), and the key-side gradients are
+ *     summed over them in a fixed order.
+ *   - dk = 256 (the paper's head dim 256; bf16, plain or iplr form) with dv =
+ *     64, 128, 192 or 256: value heads 64 wide, the same way.
  */
 #ifndef COMBA_H
 #define COMBA_H
@@ -66,8 +75,11 @@ typedef struct {
     int B;                      /* batch; 1 when cu_seqlens != NULL               */
     int T;                      /* tokens per sequence, or total packed tokens    */
     int H;                      /* heads                                          */
-    int dk;                     /* key/query head dim: 64 or 128                  */
-    int dv;                     /* value head dim: 64 or 128                      */
+    int dk;                     /* key/query head dim: 64, 128 or 256             */
+    int dv;                     /* value head dim: 64 or 128; with dk = 128 also  */
+                                /* 256, 384, 512; with dk = 256 64, 128, 192, 256 */
+                                /* (wider dv and dk = 256: bf16, plain or iplr    */
+                                /* form; see "Head widths" below)                 */
     int num_seqs;               /* N: == B when cu_seqlens == NULL                */
     const int32_t *cu_seqlens;  /* device int32 [N+1] or NULL                     */
     comba_dtype_t dtype;        /* storage type of q, k, v, o and their grads     */
@@ -263,6 +275,8 @@ comba_status_t comba_chunk_bwd(const comba_shape_t *shape,
  *   q, k [Bd,H,dk], v [Bd,H,dv], o [Bd,H,dv] (storage type `dtype`);
  *   alpha, beta fp32 [Bd,H]; b fp32 [H] or NULL; d fp32 [H];
  *   state fp32 [Bd,H,dk,dv], updated in place.
+ *   dk in {64, 128, 256}; dv in {64, 128}, or 256 with dk >= 128 (either dtype);
+ *   other widths are COMBA_ERR_UNSUPPORTED.
  *   flags: 0 or COMBA_IPLR (b beta replaced by 2 alpha b beta); other bits are
  *   COMBA_ERR_INVALID_ARG.
  */

@@ -49,23 +49,25 @@ struct BPrepSmem {
     static constexpr int PK = pitch<T>(DK), PV = pitch<T>(DV), PL = pitch<T>(64);
     static constexpr size_t OQ = 0;                                      // Q~
     static constexpr size_t OK = align128(OQ + sizeof(T) * 64 * PK);     // K, later Z = Qhat - P W
-    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);     // W
-    static constexpr size_t OD = align128(OW + sizeof(T) * 64 * PK);     // dO
-    static constexpr size_t OP = align128(OD + sizeof(T) * 64 * PV);     // P
+    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);     // W, later dO
+    static constexpr size_t OD = OW;
+    static constexpr size_t OP = align128(OW + sizeof(T) * 64 * (PK > PV ? PK : PV));   // P
     static constexpr size_t OG = align128(OP + sizeof(T) * 64 * PL);
     static constexpr size_t bytes() { return OG + sizeof(float) * 64; }
 };
 
 // C^T = dO^T (Qhat - P W)  [dv][dk], per (chunk, head).
+// One CTA per (chunk slot, key head): P and Z depend on the key head only (W and G are the
+// same for each of its value heads); C^T is formed per value head from its dO.
 template <typename T, int DK, int DV>
 __global__ void __launch_bounds__(128) k_bwd_prep(ChunkParams p) {
     using S = BPrepSmem<T, DK, DV>;
-    const int slot = blockIdx.x, h = blockIdx.y;
+    const int slot = blockIdx.x, hk = blockIdx.y, Hk = p.H / p.vg;
     const SlotInfo si = p.slot_info[slot];
     if (si.len <= 0) return;
     const int L = si.len;
     const long long t0 = si.start;
-    const long long idx = (long long)slot * p.H + h;
+    const long long idx0 = (long long)slot * p.H + hk * p.vg;   // the key head's first value head
     const int tid = threadIdx.x, warp = tid >> 5;
 
     extern __shared__ __align__(128) char smem[];
@@ -77,16 +79,19 @@ __global__ void __launch_bounds__(128) k_bwd_prep(ChunkParams p) {
     T* sP = reinterpret_cast<T*>(smem + S::OP);
     float* sG = reinterpret_cast<float*>(smem + S::OG);
 
-    const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;   // key-side rows
+    const long long kr0 = t0 * Hk + hk, kld = (long long)Hk * DK;   // key-side rows
+    auto load_do = [&](int j) {
+        load_tile_async<T>(sdO, S::PV, (const T*)p.dO + (t0 * p.H + hk * p.vg + j) * DV, (long long)p.H * DV, 64, DV,
+                           L, tid, 128);
+    };
     load_tile_async<T>(sQ, S::PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
-    load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
-    load_tile_async<T>(sdO, S::PV, (const T*)p.dO + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
+    load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx0 * 64 * DK, DK, 64, DK, 64, tid, 128);
     cp_async_commit();
-    if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+    if (tid < 64) sG[tid] = p.Gb[idx0 * 64 + tid];
     cp_async_wait<0>();
     __syncthreads();
-    const float dd = p.d[h / p.vg];
+    const float dd = p.d[hk];
     for (int e = tid; e < 64 * DK; e += 128) {
         const int r = e / DK, c = e % DK;
         sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dd * to_f(sK[r * S::PK + c]));
@@ -119,29 +124,39 @@ __global__ void __launch_bounds__(128) k_bwd_prep(ChunkParams p) {
                 const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
                 z[t][i] = (i < 2 ? ea : eb) * to_f(sQ[r * S::PK + c]) - z[t][i];
             }
-        __syncthreads();   // every warp is done reading K (via P) before Z overwrites it
+        __syncthreads();   // every warp is done reading K and W (via P) before Z and dO replace them
+        load_do(0);
+        cp_async_commit();
         frag_store<T, DK / 8>(sZ, S::PK, 16 * warp, 0, z);
     }
-    __syncthreads();
-    // C^T = dO^T Z
+    // C^T = dO^T Z per value head
     constexpr int MT = DV / 64;
+    for (int j = 0; j < p.vg; ++j) {
+        if (j > 0) {   // the previous value head's product has read dO
+            __syncthreads();
+            load_do(j);
+            cp_async_commit();
+        }
+        cp_async_wait<0>();
+        __syncthreads();
+        T* g = (T*)p.Cb + (idx0 + j) * DV * DK;
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt) {
-        const int m0 = (warp * MT + mt) * 16;
+        for (int mt = 0; mt < MT; ++mt) {
+            const int m0 = (warp * MT + mt) * 16;
 #pragma unroll
-        for (int n0 = 0; n0 < DK; n0 += 64) {
-            float acc[8][4];
-            zero(acc);
-            warp_gemm<false, false, 8>(acc, sdO, S::PV, sZ, S::PK, m0, n0, 64);
-            T* g = (T*)p.Cb + idx * DV * DK;
+            for (int n0 = 0; n0 < DK; n0 += 64) {
+                float acc[8][4];
+                zero(acc);
+                warp_gemm<false, false, 8>(acc, sdO, S::PV, sZ, S::PK, m0, n0, 64);
 #pragma unroll
-            for (int t = 0; t < 8; ++t)
+                for (int t = 0; t < 8; ++t)
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    T* dst = g + (long long)(m0 + frag_row(2 * hh)) * DK + n0 + frag_col(t, 0);
-                    dst[0] = from_f<T>(acc[t][2 * hh]);
-                    dst[1] = from_f<T>(acc[t][2 * hh + 1]);
-                }
+                    for (int hh = 0; hh < 2; ++hh) {
+                        T* dst = g + (long long)(m0 + frag_row(2 * hh)) * DK + n0 + frag_col(t, 0);
+                        dst[0] = from_f<T>(acc[t][2 * hh]);
+                        dst[1] = from_f<T>(acc[t][2 * hh + 1]);
+                    }
+            }
         }
     }
 }
@@ -751,7 +766,7 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     if (tcp) {
         if ((e = launch_bwd_prep_tc(p, s))) return e;
     } else if (p.slots > 0) {
-        k_bwd_prep<T, DK, DV><<<dim3(p.slots, p.H), 128, sm_prep, s>>>(p);
+        k_bwd_prep<T, DK, DV><<<dim3(p.slots, p.H / p.vg), 128, sm_prep, s>>>(p);   // one CTA per key head
     }
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 1, s);

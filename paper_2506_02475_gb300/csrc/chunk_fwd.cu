@@ -111,11 +111,13 @@ __device__ __forceinline__ void frag_store_global(T* g, long long ld, int m0, in
 
 template <typename T, int DK, int DV>
 struct PrepSmem {
+    // dk <= 128: the chunk map (Atilde, B^T) is formed from Kbar-scaled copies of W and U that
+    // reuse the A and M regions; at dk = 256 there is no map and those regions hold fp32 only.
+    static constexpr bool kMap = DK <= 128;
     static constexpr int PK = pitch<T>(DK), PV = pitch<T>(DV), PL = pitch<T>(64);
-    static constexpr size_t RA = sizeof(float) * 64 * 65 > sizeof(T) * 64 * PK ? sizeof(float) * 64 * 65
-                                                                                 : sizeof(T) * 64 * PK;
-    static constexpr size_t RM = sizeof(float) * 64 * 65 > sizeof(T) * 64 * PV ? sizeof(float) * 64 * 65
-                                                                                 : sizeof(T) * 64 * PV;
+    static constexpr size_t F64 = sizeof(float) * 64 * 65;
+    static constexpr size_t RA = kMap && sizeof(T) * 64 * PK > F64 ? sizeof(T) * 64 * PK : F64;
+    static constexpr size_t RM = kMap && sizeof(T) * 64 * PV > F64 ? sizeof(T) * 64 * PV : F64;
     static constexpr size_t OK = 0;
     static constexpr size_t OV = align128(OK + sizeof(T) * 64 * PK);
     static constexpr size_t OA = align128(OV + sizeof(T) * 64 * PV);   // A (fp32), later Diag(s) W
@@ -146,15 +148,19 @@ __device__ __forceinline__ void gemm_to_global(T* g, const T* sA, int lda, const
     }
 }
 
+// One CTA per (chunk slot, key head).  The Gram, the UT inverse and W depend on the key head
+// only: they are formed once and written to each of its vg value heads (units slot * H + hk *
+// vg + j), which differ in V and so in U = M Diag(beta) V.
 template <typename T, int DK, int DV>
 __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     using S = PrepSmem<T, DK, DV>;
-    const int slot = blockIdx.x, h = blockIdx.y;
+    constexpr bool kMap = S::kMap;
+    const int slot = blockIdx.x, hk = blockIdx.y, Hk = p.H / p.vg;
     const SlotInfo si = p.slot_info[slot];
     if (si.len <= 0) return;
     const int L = si.len;
     const long long t0 = si.start;
-    const long long idx = (long long)slot * p.H + h;
+    auto vidx = [&](int j) { return (long long)slot * p.H + hk * p.vg + j; };   // value-head units
     const int tid = threadIdx.x, warp = tid >> 5;
 
     extern __shared__ __align__(128) char smem[];
@@ -175,17 +181,21 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     // feedback vectors: P for Comba-pk (Gram P K^T, W = M Diag P), else K itself
     T* sF = p.p ? reinterpret_cast<T*>(smem + S::OP) : sK;
 
-    const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;   // key-side rows
+    const long long kr0 = t0 * Hk + hk, kld = (long long)Hk * DK;   // key-side rows
+    auto load_v = [&](int j) {
+        load_tile_async<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + hk * p.vg + j) * DV, (long long)p.H * DV, 64, DV,
+                           L, tid, 128);
+    };
     load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
     if (p.p) load_tile_async<T>(sF, S::PK, (const T*)p.p + kr0 * DK, kld, 64, DK, L, tid, 128);
-    load_tile_async<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 128);
+    load_v(0);
     cp_async_commit();
-    if (warp == 0) chunk_log_cumsum(p.alpha + kr0, p.H / p.vg, L, sG, sGm1);
+    if (warp == 0) chunk_log_cumsum(p.alpha + kr0, Hk, L, sG, sGm1);
     if (tid < 64) {
-        const float be = tid < L ? p.beta[krow(p, t0 + tid, h)] : 0.f;
+        const float be = tid < L ? p.beta[kr0 + (long long)tid * Hk] : 0.f;
         sBe[tid] = be;
-        const float al = tid < L ? p.alpha[krow(p, t0 + tid, h)] : 1.f;
-        sBt[tid] = (p.b ? p.b[h / p.vg] : 1.f) * be * feedback_scale(p.iplr, al);
+        const float al = tid < L ? p.alpha[kr0 + (long long)tid * Hk] : 1.f;
+        sBt[tid] = (p.b ? p.b[hk] : 1.f) * be * feedback_scale(p.iplr, al);
     }
     cp_async_wait<0>();
     __syncthreads();
@@ -211,50 +221,63 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     unit_lower_inverse64(sA, sM, sTmp, tid);
 
     // Column-scaled copies for the two products: Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta).
-    T* Mg = p.Mb ? (T*)p.Mb + idx * 4096 : nullptr;
     for (int e = tid; e < 64 * 64; e += 128) {
         const int r = e >> 6, c = e & 63;
         const float m = sM[r * 65 + c];
         sMw[r * S::PL + c] = from_f<T>(m * sBt[c] * expf(sGm1[c]));
         sMu[r * S::PL + c] = from_f<T>(m * sBe[c]);
-        if (Mg) Mg[e] = from_f<T>(m);
+        if (p.Mb)
+            for (int j = 0; j < p.vg; ++j) ((T*)p.Mb + vidx(j) * 4096)[e] = from_f<T>(m);
     }
-    if (tid < 64) p.Gb[idx * 64 + tid] = sG[tid];
+    if (tid < 64)
+        for (int j = 0; j < p.vg; ++j) p.Gb[vidx(j) * 64 + tid] = sG[tid];
     __syncthreads();
 
-    // W = Mw P, U = Mu V (stored) and their Kbar-row-scaled copies for the chunk's state map.
+    // W = Mw P, U = Mu V (stored) and, for the chunk's state map, their Kbar-row-scaled copies.
     // At dk = 256 the scan applies E = U - W H itself and no map is formed.
-    constexpr bool kMap = DK <= 128;
     const float sa = sS[16 * warp + frag_row(0)], sb = sS[16 * warp + frag_row(2)];
     {
         float acc[DK / 8][4];
         zero(acc);
         warp_gemm<true, false, DK / 8>(acc, sMw, S::PL, sF, S::PK, 16 * warp, 0, 64);
-        frag_store_global<T, DK / 8>((T*)p.Wb + idx * 64 * DK, DK, 16 * warp, 0, acc, 64);
+        for (int j = 0; j < p.vg; ++j)
+            frag_store_global<T, DK / 8>((T*)p.Wb + vidx(j) * 64 * DK, DK, 16 * warp, 0, acc, 64);
         if constexpr (kMap) {
 #pragma unroll
             for (int t = 0; t < DK / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
             frag_store<T, DK / 8>(sWs, S::PK, 16 * warp, 0, acc);
         }
     }
-    {
-        float acc[DV / 8][4];
-        zero(acc);
-        warp_gemm<true, false, DV / 8>(acc, sMu, S::PL, sV, S::PV, 16 * warp, 0, 64);
-        frag_store_global<T, DV / 8>((T*)p.Ub + idx * 64 * DV, DV, 16 * warp, 0, acc, 64);
-        if constexpr (kMap) {
-#pragma unroll
-            for (int t = 0; t < DV / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
-            frag_store<T, DV / 8>(sUs, S::PV, 16 * warp, 0, acc);
+    for (int j = 0; j < p.vg; ++j) {
+        const long long idx = vidx(j);
+        if (j > 0) {   // the previous value head's products have read V
+            __syncthreads();
+            load_v(j);
+            cp_async_commit();
+            cp_async_wait<0>();
+            __syncthreads();
         }
-    }
-    if constexpr (kMap) {
-        __syncthreads();
-        // Atilde = -K^T Diag(s) W  [dk][dk];  B^T = (Diag(s) U)^T K  [dv][dk];  Atilde^T = -(Diag(s) W)^T K.
-        gemm_to_global<T, false, false, DK, DK>((T*)p.Ab + idx * DK * DK, sK, S::PK, sWs, S::PK, 64, -1.f, warp);
-        gemm_to_global<T, false, false, DV, DK>((T*)p.Bb + idx * DV * DK, sUs, S::PV, sK, S::PK, 64, 1.f, warp);
-        if (p.ATb)
-            gemm_to_global<T, false, false, DK, DK>((T*)p.ATb + idx * DK * DK, sWs, S::PK, sK, S::PK, 64, -1.f, warp);
+        {
+            float acc[DV / 8][4];
+            zero(acc);
+            warp_gemm<true, false, DV / 8>(acc, sMu, S::PL, sV, S::PV, 16 * warp, 0, 64);
+            frag_store_global<T, DV / 8>((T*)p.Ub + idx * 64 * DV, DV, 16 * warp, 0, acc, 64);
+            if constexpr (kMap) {
+#pragma unroll
+                for (int t = 0; t < DV / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }
+                frag_store<T, DV / 8>(sUs, S::PV, 16 * warp, 0, acc);
+            }
+        }
+        if constexpr (kMap) {
+            __syncthreads();
+            // Atilde = -K^T Diag(s) W [dk][dk];  B^T = (Diag(s) U)^T K [dv][dk];  Atilde^T = -(Diag(s) W)^T K.
+            gemm_to_global<T, false, false, DK, DK>((T*)p.Ab + idx * DK * DK, sK, S::PK, sWs, S::PK, 64, -1.f, warp);
+            gemm_to_global<T, false, false, DV, DK>((T*)p.Bb + idx * DV * DK, sUs, S::PV, sK, S::PK, 64, 1.f, warp);
+            if (p.ATb)
+                gemm_to_global<T, false, false, DK, DK>((T*)p.ATb + idx * DK * DK, sWs, S::PK, sK, S::PK, 64, -1.f,
+                                                        warp);
+            if (j + 1 < p.vg) __syncthreads();   // the next U's scaled copy replaces this one
+        }
     }
 }
 
@@ -377,7 +400,7 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     if (tcp) {
         if ((e = launch_prep_tc(q, s))) return e;
     } else if (q.slots > 0) {
-        k_prep<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_prep, s>>>(q);
+        k_prep<T, DK, DV><<<dim3(q.slots, q.H / q.vg), 128, sm_prep, s>>>(q);   // one CTA per key head
     }
     if ((e = cudaGetLastError())) return e;
     mark(q, ev0 + 1, s);
