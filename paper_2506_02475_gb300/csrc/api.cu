@@ -150,7 +150,8 @@ comba_status_t check_smem(const comba_shape_t* s, int backward) {
     const bool bf = s->dtype == COMBA_BF16, pk = (s->flags & COMBA_PK) != 0;
     const int dv = s->dv / value_groups(s);
     for (int kern = 0; kern < 3; ++kern)
-        if (comba::fwd_smem_bytes(kern, bf, s->dk, dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;
+        if (comba::fwd_smem_bytes(kern, bf, s->dk, dv, pk, value_groups(s) > 1) > (size_t)optin)
+            return COMBA_ERR_UNSUPPORTED;
     if (backward)
         for (int kern = 0; kern < 2; ++kern)
             if (comba::bwd_smem_bytes(kern, bf, s->dk, dv, pk) > (size_t)optin) return COMBA_ERR_UNSUPPORTED;

@@ -288,69 +288,64 @@ struct OutSmem {
     static constexpr int PK = pitch<T>(DK), PV = pitch<T>(DV), PL = pitch<T>(64);
     static constexpr size_t OQ = 0;                                          // Q~
     static constexpr size_t OK = align128(OQ + sizeof(T) * 64 * PK);         // K
-    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);         // W, later P
-    static constexpr size_t OU = align128(OW + sizeof(T) * 64 * PK);         // U, later E
-    static constexpr size_t OH = align128(OU + sizeof(T) * 64 * PV);         // H^T [dv][dk]
-    static constexpr size_t OG = align128(OH + sizeof(T) * DV * PK);
-    static constexpr size_t bytes() { return OG + sizeof(float) * 64; }
+    static constexpr size_t OW = align128(OK + sizeof(T) * 64 * PK);         // W
+    static constexpr size_t OP = align128(OW + sizeof(T) * 64 * PK);         // P
+    static constexpr size_t OG = align128(OP + sizeof(T) * 64 * PL);         // log-decays
+    static constexpr size_t OB = align128(OG + sizeof(float) * 64);          // value-head buffers: U (later E), H^T
+    static constexpr size_t BU = 0;
+    static constexpr size_t BH = align128(sizeof(T) * 64 * PV);
+    static constexpr size_t BUF = align128(BH + sizeof(T) * DV * PK);
+    // a second buffer when a key head has several value heads (the next one's tiles stream in)
+    static constexpr size_t bytes(bool two = false) { return OB + (two ? 2 : 1) * BUF; }
 };
 
+// One CTA per (chunk slot, key head).  Q~ and P = Tril(Q~ K^T * Gamma) depend on the key head
+// only; each of its value heads j then forms E_j = U_j - W H_j and O_j = Diag(gamma) Q~ H_j + P E_j,
+// with the next value head's U and H^T loading meanwhile.
 template <typename T, int DK, int DV>
 __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     using S = OutSmem<T, DK, DV>;
-    const int slot = blockIdx.x, h = blockIdx.y;
+    const int slot = blockIdx.x, hk = blockIdx.y, Hk = p.H / p.vg, vg = p.vg;
     const SlotInfo si = p.slot_info[slot];
     if (si.len <= 0) return;
     const int L = si.len;
     const long long t0 = si.start;
-    const long long idx = (long long)slot * p.H + h;
+    const long long idx0 = (long long)slot * p.H + hk * vg;   // the key head's first value head
     const int tid = threadIdx.x, warp = tid >> 5;
 
     extern __shared__ __align__(128) char smem[];
     T* sQ = reinterpret_cast<T*>(smem + S::OQ);
     T* sK = reinterpret_cast<T*>(smem + S::OK);
     T* sW = reinterpret_cast<T*>(smem + S::OW);
-    T* sP = sW;
-    T* sU = reinterpret_cast<T*>(smem + S::OU);
-    T* sE = sU;
-    T* sH = reinterpret_cast<T*>(smem + S::OH);
+    T* sP = reinterpret_cast<T*>(smem + S::OP);
     float* sG = reinterpret_cast<float*>(smem + S::OG);
+    auto sU = [&](int j) { return reinterpret_cast<T*>(smem + S::OB + (j & 1) * S::BUF + S::BU); };
+    auto sH = [&](int j) { return reinterpret_cast<T*>(smem + S::OB + (j & 1) * S::BUF + S::BH); };
+    auto load_vh = [&](int j) {   // value head j's U and H^T
+        const long long idx = idx0 + j;
+        load_tile_async<T>(sU(j), S::PV, (const T*)p.Ub + idx * 64 * DV, DV, 64, DV, 64, tid, 128);
+        load_tile_async<T>(sH(j), S::PK, (const T*)p.Hb + idx * DV * DK, DK, DV, DK, DV, tid, 128);
+    };
 
-    const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;   // key-side rows
+    const long long kr0 = t0 * Hk + hk, kld = (long long)Hk * DK;   // key-side rows
     load_tile_async<T>(sQ, S::PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
-    load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx * 64 * DK, DK, 64, DK, 64, tid, 128);
-    load_tile_async<T>(sU, S::PV, (const T*)p.Ub + idx * 64 * DV, DV, 64, DV, 64, tid, 128);
-    load_tile_async<T>(sH, S::PK, (const T*)p.Hb + idx * DV * DK, DK, DV, DK, DV, tid, 128);
+    load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx0 * 64 * DK, DK, 64, DK, 64, tid, 128);
+    load_vh(0);
     cp_async_commit();
-    if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
-    cp_async_wait<0>();
+    if (vg > 1) load_vh(1);
+    cp_async_commit();
+    if (tid < 64) sG[tid] = p.Gb[idx0 * 64 + tid];
+    cp_async_wait<1>();
     __syncthreads();
 
-    // E = U - W H  (B operand H[c][j] read from H^T[j][c]); E replaces U in shared memory.
-    {
-        float e[DV / 8][4];
-        zero(e);
-        warp_gemm<true, true, DV / 8>(e, sW, S::PK, sH, S::PK, 16 * warp, 0, DK);
-#pragma unroll
-        for (int t = 0; t < DV / 8; ++t)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
-                e[t][i] = to_f(sU[r * S::PV + c]) - e[t][i];
-            }
-        if (p.Eb) frag_store_global<T, DV / 8>((T*)p.Eb + idx * 64 * DV, DV, 16 * warp, 0, e, 64);
-        frag_store<T, DV / 8>(sE, S::PV, 16 * warp, 0, e);
-    }
-    const float dh = p.d[h / p.vg];
+    const float dh = p.d[hk];
     for (int e = tid; e < 64 * DK; e += 128) {
         const int r = e / DK, c = e % DK;
         sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dh * to_f(sK[r * S::PK + c]));
     }
     __syncthreads();
-    if (!p.o) return;
-
-    {
+    if (p.o) {
         float sc[8][4];
         zero(sc);
         warp_gemm<true, true, 8>(sc, sQ, S::PK, sK, S::PK, 16 * warp, 0, DK);
@@ -363,22 +358,53 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
                 sP[r * S::PL + c] = from_f<T>(v);
             }
     }
-    __syncthreads();
+    const float e0 = expf(sG[16 * warp + frag_row(0)]);
+    const float e1 = expf(sG[16 * warp + frag_row(2)]);
 
-    float o[DV / 8][4];
-    zero(o);
-    warp_gemm<true, true, DV / 8>(o, sQ, S::PK, sH, S::PK, 16 * warp, 0, DK);
-    {
-        const float e0 = expf(sG[16 * warp + frag_row(0)]);
-        const float e1 = expf(sG[16 * warp + frag_row(2)]);
-#pragma unroll
-        for (int t = 0; t < DV / 8; ++t) {
-            o[t][0] *= e0; o[t][1] *= e0;
-            o[t][2] *= e1; o[t][3] *= e1;
+    for (int j = 0; j < vg; ++j) {
+        const long long idx = idx0 + j;
+        if (j > 0) {
+            cp_async_wait<1>();   // this value head's tiles (only the newest group may be pending)
+            __syncthreads();
         }
+        T* sE = sU(j);
+        T* sHj = sH(j);
+        // E = U - W H  (B operand H[c][jj] read from H^T[jj][c]); E replaces U.  Each warp reads
+        // and writes only its own 16 rows of U / E.
+        {
+            float e[DV / 8][4];
+            zero(e);
+            warp_gemm<true, true, DV / 8>(e, sW, S::PK, sHj, S::PK, 16 * warp, 0, DK);
+#pragma unroll
+            for (int t = 0; t < DV / 8; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = 16 * warp + frag_row(i), c = frag_col(t, i);
+                    e[t][i] = to_f(sE[r * S::PV + c]) - e[t][i];
+                }
+            if (p.Eb) frag_store_global<T, DV / 8>((T*)p.Eb + idx * 64 * DV, DV, 16 * warp, 0, e, 64);
+            frag_store<T, DV / 8>(sE, S::PV, 16 * warp, 0, e);
+        }
+        __syncthreads();   // E (and, for j = 0, P) complete
+        if (p.o) {
+            float o[DV / 8][4];
+            zero(o);
+            warp_gemm<true, true, DV / 8>(o, sQ, S::PK, sHj, S::PK, 16 * warp, 0, DK);
+#pragma unroll
+            for (int t = 0; t < DV / 8; ++t) {
+                o[t][0] *= e0; o[t][1] *= e0;
+                o[t][2] *= e1; o[t][3] *= e1;
+            }
+            warp_gemm<true, false, DV / 8>(o, sP, S::PL, sE, S::PV, 16 * warp, 0, 64);
+            frag_store_global<T, DV / 8>((T*)p.o + (t0 * p.H + hk * vg + j) * DV, (long long)p.H * DV, 16 * warp, 0,
+                                         o, L);
+        }
+        if (j + 2 < vg) {
+            __syncthreads();   // this buffer is fully read
+            load_vh(j + 2);
+        }
+        cp_async_commit();
     }
-    warp_gemm<true, false, DV / 8>(o, sP, S::PL, sE, S::PV, 16 * warp, 0, 64);
-    frag_store_global<T, DV / 8>((T*)p.o + (t0 * p.H + h) * DV, (long long)p.H * DV, 16 * warp, 0, o, L);
 }
 
 // -------------------------------------------------------------- launchers
@@ -386,7 +412,7 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
 template <typename T, int DK, int DV>
 static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int ev0) {
     const size_t sm_prep = PrepSmem<T, DK, DV>::bytes(p.p != nullptr);
-    const size_t sm_out = OutSmem<T, DK, DV>::bytes();
+    const size_t sm_out = OutSmem<T, DK, DV>::bytes(p.vg > 1);
     cudaError_t e;
     if ((e = cudaFuncSetAttribute(k_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
         return e;
@@ -417,7 +443,7 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
         if (tcp) {
             if ((e = launch_output_tc(q, s))) return e;
         } else if (q.slots > 0) {
-            k_output<T, DK, DV><<<dim3(q.slots, q.H), 128, sm_out, s>>>(q);
+            k_output<T, DK, DV><<<dim3(q.slots, q.H / q.vg), 128, sm_out, s>>>(q);   // one CTA per key head
         }
     }
     if ((e = cudaGetLastError())) return e;
@@ -443,11 +469,11 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
     return cudaErrorInvalidValue;
 }
 
-size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk) {
+size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk, bool groups) {
     if (kernel == 1) return scan_smem_bytes(is_bf16, dk, dv);
     if (use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(kernel == 0 ? 0 : 1);
 #define COMBA_SM(T, DK, DV) \
-    if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes(pk) : OutSmem<T, DK, DV>::bytes();
+    if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes(pk) : OutSmem<T, DK, DV>::bytes(groups);
     if (is_bf16) {
         COMBA_SM(bf16, 128, 128) COMBA_SM(bf16, 128, 64) COMBA_SM(bf16, 64, 128) COMBA_SM(bf16, 64, 64)
         COMBA_SM(bf16, 256, 64)

@@ -152,7 +152,8 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
 // the head reduction.  Stage events: ev0 before C^T, ev0+1 before the scan, ev0+2 before
 // the local gradients, ev0+3 before the reduction, ev0+4 after it.
 cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int ev0);
-size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false);
+// `groups`: several value heads per key head (the output kernel then double-buffers their tiles)
+size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false, bool groups = false);
 // tcgen05 kernels of the bf16 dk = dv = 128 path (chunk_tc.cu)
 cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s);
 cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s);
