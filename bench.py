@@ -59,41 +59,47 @@ def fwd_flops_per_token_head(C=64, dk=128, dv=128):
 # the tile products the kernel must form and the tensors it must read or write
 # once.  Forward saves the backward's factors (M, Atilde^T, E).
 
-def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False):
+def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
     """`tc`: the tcgen05 path (bf16, d=128), whose reverse scan reads Atilde itself, so
     the forward saves M but no Atilde^T.  `pk`: Comba-pk feedback vectors P, read by prep and
     by the local gradients, which also write dP.  At dk = 256 no chunk map is formed: the
-    scans read W, K and U (forward) or C^T (backward) and form two products per chunk."""
+    scans read W, K and U (forward) or C^T (backward) and form two products per chunk.
+    `H` counts value heads of width `dv`, `vg` of them per key head: tensors and products
+    that depend on the key head only (q, k, gates, W, M, Atilde, the Gram, Q~ K^T, dq, dk,
+    dalpha, dbeta) are counted once per (chunk, key head), however often a kernel re-reads
+    or recomputes them per value head."""
     C, es, f4 = 64, 2, 4
-    P = slots * H
+    P = slots * H            # (chunk, value head) units
+    Pk = P // vg             # (chunk, key head) units
     wide = dk > 128
     at = save and not tc and not wide
-    mp = 0 if wide else 1   # the chunk map Atilde, B^T
+    mp = 0 if wide else 1    # the chunk map Atilde, B^T
     m = {}
-    m["prep"] = dict(flops=P * (2 * C * C * (2 * dk + dv)
-                                + mp * (2 * dk * C * dk * (2 if at else 1) + 2 * dv * C * dk)),
-                     bytes=P * (C * (dk + dv) * es + 2 * C * f4 + C * (dk + dv) * es + C * f4
-                                + mp * (dk * dk * es + dv * dk * es) + (C * C * es if save else 0)
-                                + (dk * dk * es if at else 0)))
+    m["prep"] = dict(flops=Pk * (2 * C * C * 2 * dk + mp * 2 * dk * C * dk * (2 if at else 1))
+                     + P * (2 * C * C * dv + mp * 2 * dv * C * dk),
+                     bytes=Pk * (2 * C * dk * es + 3 * C * f4 + (C * C * es if save else 0)
+                                 + mp * dk * dk * es + (dk * dk * es if at else 0))
+                     + P * (2 * C * dv * es + mp * dv * dk * es))
     if wide:
-        m["scan_fwd"] = dict(flops=P * 4 * C * dk * dv, bytes=P * ((2 * C * dk + C * dv + dv * dk) * es + C * f4))
+        m["scan_fwd"] = dict(flops=P * 4 * C * dk * dv,
+                             bytes=Pk * (2 * C * dk * es + C * f4) + P * (C * dv + dv * dk) * es)
+        m["scan_bwd"] = dict(flops=P * 4 * C * dk * dv,
+                             bytes=Pk * (2 * C * dk * es + C * f4) + P * 2 * dv * dk * es)
     else:
-        m["scan_fwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
-    m["output"] = dict(flops=P * (4 * C * dk * dv + 2 * C * C * (dk + dv)),
-                       bytes=P * (3 * C * dk * es + C * dv * es + dv * dk * es + C * dv * es * (2 if save else 1)
-                                  + C * f4))
-    m["bwd_prep"] = dict(flops=P * (4 * C * C * dk + 2 * dv * C * dk),
-                         bytes=P * (3 * C * dk * es + C * dv * es + dv * dk * es + C * f4))
-    if wide:
-        m["scan_bwd"] = dict(flops=P * 4 * C * dk * dv, bytes=P * ((2 * C * dk + 2 * dv * dk) * es + C * f4))
-    else:
-        m["scan_bwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=P * ((dk * dk + 2 * dv * dk) * es + f4))
-    m["bwd_local"] = dict(flops=P * (2 * C * C * dk * 9 + 2 * C * dk * dv * 4 + 2 * C * C * dv * 4 + 4 * C ** 3),
-                          bytes=P * (C * (2 * dk + 2 * dv) * es + C * dv * es + 2 * dv * dk * es + C * C * es
-                                     + 3 * C * f4 + C * (2 * dk + dv) * es + 2 * C * f4))
+        m["scan_fwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=Pk * (dk * dk * es + f4) + P * 2 * dv * dk * es)
+        m["scan_bwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=Pk * (dk * dk * es + f4) + P * 2 * dv * dk * es)
+    m["output"] = dict(flops=Pk * 2 * C * C * dk + P * (4 * C * dk * dv + 2 * C * C * dv),
+                       bytes=Pk * (3 * C * dk * es + C * f4)
+                       + P * (C * dv * es + dv * dk * es + C * dv * es * (2 if save else 1)))
+    m["bwd_prep"] = dict(flops=Pk * 4 * C * C * dk + P * 2 * dv * C * dk,
+                         bytes=Pk * (3 * C * dk * es + C * f4) + P * (C * dv * es + dv * dk * es))
+    m["bwd_local"] = dict(flops=Pk * 2 * C * C * dk * 2
+                          + P * (2 * C * C * dk * 7 + 2 * C * dk * dv * 4 + 2 * C * C * dv * 4 + 4 * C ** 3),
+                          bytes=Pk * (2 * C * dk * es + C * C * es + 3 * C * f4 + 2 * C * dk * es + 2 * C * f4)
+                          + P * (2 * C * dv * es + C * dv * es + 2 * dv * dk * es + C * dv * es))
     if pk:
-        m["prep"]["bytes"] += P * C * dk * es
-        m["bwd_local"]["bytes"] += P * 2 * C * dk * es
+        m["prep"]["bytes"] += Pk * C * dk * es
+        m["bwd_local"]["bytes"] += Pk * 2 * C * dk * es
     m["chunk_map"] = dict(flops=0, bytes=slots * 16 + (N + 1) * 8)
     m["output_E"] = dict(flops=0, bytes=0)
     m["reduce"] = dict(flops=0, bytes=P * 8 + 8 * H)
@@ -106,14 +112,14 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 110_802, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c38997b1ac5319b7"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_487, ('scan.cu', 'common.cuh', 'params.cuh'), "bd55d18df9523763"),
-    "output": ("k_output_tc", 118_759, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c38997b1ac5319b7"),
-    "bwd_prep": ("k_bwd_prep_tc", 82_468, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c38997b1ac5319b7"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_409, ('scan.cu', 'common.cuh', 'params.cuh'), "bd55d18df9523763"),
-    "bwd_local": ("k_bwd_local_tc", 194_260, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c382ee4e8c042aa7"),
+    "prep": ("k_prep_tc", 110_760, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_169, ('scan.cu', 'common.cuh', 'params.cuh'), "6c77bca293e56549"),
+    "output": ("k_output_tc", 118_698, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
+    "bwd_prep": ("k_bwd_prep_tc", 82_499, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_249, ('scan.cu', 'common.cuh', 'params.cuh'), "6c77bca293e56549"),
+    "bwd_local": ("k_bwd_local_tc", 194_298, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "2486fcf383440d09"),
 }
-DECODE_TRAFFIC = (481_426_688, ('decode.cu', 'common.cuh', 'params.cuh'), "3956f50c494e5178")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (481_306_880, ('decode.cu', 'common.cuh', 'params.cuh'), "988ef445c98cc562")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
@@ -461,7 +467,7 @@ def run_ours(args, world, rank, local):
     vg = dv // 64 if dk == 256 else (dv // 128 if dv > 128 else 1)
     dv_u, H_u = dv // vg, H * vg
     tc = w.dtype == "bf16" and dk == 128 and dv_u == 128
-    model = stage_model(dk, dv_u, slots, H_u, N, tc=tc, pk=pk)
+    model = stage_model(dk, dv_u, slots, H_u, N, tc=tc, pk=pk, vg=vg)
     # the dominant launch: the (phase, stage) with the most time (a stage the backward skips
     # because it reuses the forward's factors is not averaged with its empty slot)
     dom_phase, dom = max(stage_ms, key=lambda ps: stage_ms[ps])
