@@ -117,7 +117,7 @@ CAPTURED_TRAFFIC = {
     "output": ("k_output_tc", 118_698, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
     "bwd_prep": ("k_bwd_prep_tc", 82_499, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
     "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_249, ('scan.cu', 'common.cuh', 'params.cuh'), "6c77bca293e56549"),
-    "bwd_local": ("k_bwd_local_tc", 194_298, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "2486fcf383440d09"),
+    "bwd_local": ("k_bwd_local_tc", 194_243, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "1123096a93568c0f"),
 }
 DECODE_TRAFFIC = (481_306_880, ('decode.cu', 'common.cuh', 'params.cuh'), "988ef445c98cc562")   # whole Bd=256 H=16 launch
 

@@ -17,7 +17,9 @@
 // An M = 64 accumulator read with tcgen05.ld.16x256b gives each warp the rows
 // 16 (w & 3) .. + 15 in exactly the m16n8 accumulator fragment layout of
 // mma.sync, so the epilogues (masks, decay factors, row and column partial
-// sums) are fragment code: warps w and w + 4 take the two column halves.
+// sums) are fragment code.  Sixteen warps: w, w + 4, w + 8 and w + 12 share a
+// TMEM lane quadrant and take the four column quarters of every accumulator
+// (128 registers a thread, so the epilogues' register tiles stay small).
 // Operands live in 128-byte-swizzled shared tiles (K-major or MN-major as
 // each product needs; no transposed copies).  Outputs are staged in shared
 // memory and written with coalesced 16-byte stores.
@@ -25,6 +27,10 @@
 
 namespace comba {
 namespace tc {
+
+constexpr int kLocalThreads = 512;            // 16 warps: four per TMEM lane quadrant
+constexpr int kQ = kLocalThreads / 128;        // column parts of each accumulator (one per warp of a quadrant)
+constexpr int NK = 16 / kQ, NL = 8 / kQ;       // m16n8 fragments per warp of 128- and 64-wide results
 
 struct LocalTcSmem {
     static constexpr uint32_t OQK = 0;             // two [128][128] tiles (consecutive units alternate): rows 0-63
@@ -38,11 +44,11 @@ struct LocalTcSmem {
     static constexpr uint32_t OP = OM + 8192;      // P [64][64]
     static constexpr uint32_t ODE = OP + 8192;     // dE [64][128]
     static constexpr uint32_t OF = ODE + 16384;    // fp32: 8 x 64 per-row vectors, row and column partials, reduction
-    static constexpr uint32_t NF = 8 * 64 + 8 * 2 * 64 + 2 * 4 * 64 + 16;
+    static constexpr uint32_t NF = 8 * 64 + 8 * kQ * 64 + 2 * 4 * 64 + 16;
     static constexpr size_t bytes() { return 1024 + OF + NF * 4; }
 };
 
-// M = 64 accumulator columns [taddr, +8 NT) of this warp's 16 rows as m16n8 fragments.
+// M = 64 accumulator columns [taddr, +8 NT) of this warp's 16 rows as m16n8 fragments (NT = 4, 2).
 __device__ __forceinline__ void tmem_frag4(uint32_t taddr, float (&a)[4][4]) {
     uint32_t r[16];
     asm volatile(
@@ -54,19 +60,14 @@ __device__ __forceinline__ void tmem_frag4(uint32_t taddr, float (&a)[4][4]) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) a[i >> 2][i & 3] = __uint_as_float(r[i]);
 }
-__device__ __forceinline__ void tmem_frag8(uint32_t taddr, float (&a)[8][4]) {
-    uint32_t r[32];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.16x256b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
+__device__ __forceinline__ void tmem_frag2(uint32_t taddr, float (&a)[2][4]) {
+    uint32_t r[8];
+    asm volatile("tcgen05.ld.sync.aligned.16x256b.x2.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr));
     asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
 #pragma unroll
-    for (int i = 0; i < 32; ++i) a[i >> 2][i & 3] = __uint_as_float(r[i]);
+    for (int i = 0; i < 8; ++i) a[i >> 2][i & 3] = __uint_as_float(r[i]);
 }
 
 // bf16 pair (row, col..col+1) of a K-major swizzled tile with `rows` allocated rows.
@@ -85,6 +86,12 @@ __device__ __forceinline__ void frag_store_sw(uint8_t* tile, int rows, int m0, i
         for (int hh = 0; hh < 2; ++hh)
             st_pair(tile, rows, m0 + frag_row(2 * hh), n0 + frag_col(t, 0), acc[t][2 * hh], acc[t][2 * hh + 1]);
 }
+template <int NT>
+__device__ __forceinline__ void tmem_frag(uint32_t taddr, float (&a)[NT][4]) {
+    static_assert(NT == 2 || NT == 4, "column quarters of 64- and 128-wide accumulators");
+    if constexpr (NT == 2) tmem_frag2(taddr, a);
+    else tmem_frag4(taddr, a);
+}
 // Row-major [64][128] bf16 staging with 16-byte chunks rotated by row (conflict-free fragment
 // writes), and its coalesced copy of rows < L to a strided global matrix.
 template <int NT>
@@ -99,7 +106,7 @@ __device__ __forceinline__ void frag_stage(uint8_t* st, int m0, int n0, const fl
         }
 }
 __device__ __forceinline__ void copy_stage_rows(bf16* g, long long ld, const uint8_t* st, int L, int tid) {
-    for (int e = tid; e < L * 16; e += 256) {
+    for (int e = tid; e < L * 16; e += kLocalThreads) {
         const int r = e >> 4, ch = e & 15;
         *reinterpret_cast<uint4*>(g + r * ld + ch * 8) =
             *reinterpret_cast<const uint4*>(st + r * 256 + (((ch + r) & 15) << 4));
@@ -134,7 +141,7 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 // M after R7; Q and K into the second of two alternating tiles at the start of the unit; the
 // per-row scalars into registers), so the loads of consecutive units overlap the tensor-core
 // and epilogue work instead of every SM loading at the same moment.
-__global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long long units) {
+__global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p, long long units) {
     using S = LocalTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar;
@@ -164,8 +171,8 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
     float* sDg = sG + 320;
     float* sEm1 = sG + 384;           // gamma_{r-1}
     float* sWs = sG + 448;            // btilde_r gamma_{r-1}
-    float* rowp = sG + 512;           // [kind][column half][row]
-    float* colp = rowp + 8 * 2 * 64;  // [kind][row block][column]
+    float* rowp = sG + 512;           // [kind][column quarter][row]
+    float* colp = rowp + 8 * kQ * 64;  // [kind][row block][column]
     float* red = colp + 2 * 4 * 64;
     const uint32_t uV = smem_u32(sV), udO = smem_u32(sdO),
                    uE = smem_u32(sE), uH = smem_u32(sHt), udH = smem_u32(sdHt), uM = smem_u32(sM),
@@ -176,7 +183,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
     auto load_qk = [&](uint8_t* dst, const UnitRef& x) {
         const bf16* qg = (const bf16*)p.q + (x.t0 * Hk + x.h / p.vg) * D;
         const bf16* kg = (const bf16*)p.k + (x.t0 * Hk + x.h / p.vg) * D;
-        for (int e = tid; e < 128 * 16; e += 256) {
+        for (int e = tid; e < 128 * 16; e += kLocalThreads) {
             const int r = e >> 4, ch = e & 15, rr = r & 63;
             const bool okr = rr < x.L;
             const bf16* src = (r < 64 ? qg : kg) + (long long)rr * Hk * D + ch * 8;
@@ -196,12 +203,12 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         return r;
     };
     auto load_tok = [&](uint8_t* dst, const void* base, const UnitRef& x) {
-        load_sw(dst, 64, D, (const bf16*)base + (x.t0 * p.H + x.h) * D, (long long)p.H * D, x.L, tid, 256);
+        load_sw(dst, 64, D, (const bf16*)base + (x.t0 * p.H + x.h) * D, (long long)p.H * D, x.L, tid, kLocalThreads);
     };
-    auto load_dH = [&](const UnitRef& x) { load_sw(sdHt, 128, D, (const bf16*)p.dHb + x.idx * D * D, D, 128, tid, 256); };
-    auto load_H = [&](const UnitRef& x) { load_sw(sHt, 128, D, (const bf16*)p.Hb + x.idx * D * D, D, 128, tid, 256); };
-    auto load_E = [&](const UnitRef& x) { load_sw(sE, 64, D, (const bf16*)p.Eb + x.idx * 64 * D, D, 64, tid, 256); };
-    auto load_M = [&](const UnitRef& x) { load_sw(sM, 64, 64, (const bf16*)p.Mb + x.idx * 4096, 64, 64, tid, 256); };
+    auto load_dH = [&](const UnitRef& x) { load_sw(sdHt, 128, D, (const bf16*)p.dHb + x.idx * D * D, D, 128, tid, kLocalThreads); };
+    auto load_H = [&](const UnitRef& x) { load_sw(sHt, 128, D, (const bf16*)p.Hb + x.idx * D * D, D, 128, tid, kLocalThreads); };
+    auto load_E = [&](const UnitRef& x) { load_sw(sE, 64, D, (const bf16*)p.Eb + x.idx * 64 * D, D, 64, tid, kLocalThreads); };
+    auto load_M = [&](const UnitRef& x) { load_sw(sM, 64, 64, (const bf16*)p.Mb + x.idx * 4096, 64, 64, tid, kLocalThreads); };
 
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
@@ -214,16 +221,16 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
     const uint32_t tmem = tbase;
     const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16);   // this warp's TMEM lanes
     MmaSync ms{smem_u32(&bar), 0};
-    const int nl0 = 32 * wc, nk0 = 64 * wc;   // this warp's columns of 64- and 128-wide results
+    const int nl0 = 8 * NL * wc, nk0 = 8 * NK * wc;   // this warp's columns of 64- and 128-wide results
     const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows
     auto put_rows = [&](int kind, float s0, float s1) {
-        if ((lane & 3) == 0) { rowp[(kind * 2 + wc) * 64 + ra] = s0; rowp[(kind * 2 + wc) * 64 + rb] = s1; }
+        if ((lane & 3) == 0) { rowp[(kind * kQ + wc) * 64 + ra] = s0; rowp[(kind * kQ + wc) * 64 + rb] = s1; }
     };
     // row dot of a 128-wide fragment tile with the bf16 tile `t` (rows r at row offset roff)
-    auto tile_rowdot = [&](const float (&acc)[8][4], const uint8_t* t, int rows, int roff, float& s0, float& s1) {
-        float prod[8][4];
+    auto tile_rowdot = [&](const float (&acc)[NK][4], const uint8_t* t, int rows, int roff, float& s0, float& s1) {
+        float prod[NK][4];
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
+        for (int j = 0; j < NK; ++j)
 #pragma unroll
             for (int hh = 0; hh < 2; ++hh) {
                 const float2 v = ld_pair(t, rows, roff + m0 + frag_row(2 * hh), nk0 + frag_col(j, 0));
@@ -290,7 +297,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             cp_async_commit();
         }
         // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
-        for (int e = tid; e < 64 * 16; e += 256) {
+        for (int e = tid; e < 64 * 16; e += kLocalThreads) {
             const int r = e >> 4, ch = e & 15;
             uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
             const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
@@ -304,7 +311,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         // <H, dH'>: the two tiles share one layout, so matching 16-byte chunks pair up
         {
             float sacc = 0.f;
-            for (int e = tid; e < 128 * 16; e += 256) {
+            for (int e = tid; e < 128 * 16; e += kLocalThreads) {
                 float hv[8], gv[8];
                 unpack8(reinterpret_cast<const uint4*>(sHt)[e], hv);
                 unpack8(reinterpret_cast<const uint4*>(sdHt)[e], gv);
@@ -331,12 +338,12 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         }
         ok = ms.finish(tid);
         if (ok && has_next) { load_dH(nxt); cp_async_commit(); }
-        float sc[4][4], dP[4][4], acc_dq[8][4], acc_dk[8][4], de[8][4];
+        float sc[NL][4], dP[NL][4], acc_dq[NK][4], acc_dk[NK][4], de[NK][4];
         if (ok) {
             // P = Tril(S * Gamma)
-            tmem_frag4(tq + 0 + nl0, sc);
+            tmem_frag<NL>(tq + 0 + nl0, sc);
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
+            for (int t = 0; t < NL; ++t)
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh) {
                     const int r = m0 + frag_row(2 * hh), c = nl0 + frag_col(t, 0);
@@ -345,7 +352,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                     const float v1 = (c + 1 <= r && r < L) ? sc[t][2 * hh + 1] * __expf(gr - sG[c + 1]) : 0.f;
                     st_pair(sP, 64, r, c, v0, v1);
                 }
-            tmem_frag4(tq + 64 + nl0, dP);
+            tmem_frag<NL>(tq + 64 + nl0, dP);
         }
         publish_smem();
 
@@ -354,32 +361,32 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
         if (ok) {
             // dQ~ part Diag(gamma) dO H^T; its row dot with Q~ is the log-decay gradient of the Q~ H term
-            tmem_frag8(tq + 128 + nk0, acc_dq);
+            tmem_frag<NK>(tq + 128 + nk0, acc_dq);
 #pragma unroll
-            for (int t = 0; t < 8; ++t) { acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb; }
+            for (int t = 0; t < NK; ++t) { acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb; }
             float s0, s1;
             tile_rowdot(acc_dq, sQK, 128, 0, s0, s1);
             put_rows(0, s0, s1);
             // dK from Kbar: Diag(gamma_C / gamma_r) E dH'^T
-            tmem_frag8(tq + 256 + nk0, acc_dk);
+            tmem_frag<NK>(tq + 256 + nk0, acc_dk);
 #pragma unroll
-            for (int t = 0; t < 8; ++t) { acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb; }
+            for (int t = 0; t < NK; ++t) { acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb; }
             tile_rowdot(acc_dk, sQK, 128, 64, s0, s1);
             put_rows(1, s0, s1);
             // Kbar dH' part of dE
-            tmem_frag8(tq + 384 + nk0, de);
+            tmem_frag<NK>(tq + 384 + nk0, de);
 #pragma unroll
-            for (int t = 0; t < 8; ++t) { de[t][0] *= sKa; de[t][1] *= sKa; de[t][2] *= sKb; de[t][3] *= sKb; }
+            for (int t = 0; t < NK; ++t) { de[t][0] *= sKa; de[t][1] *= sKa; de[t][2] *= sKb; de[t][3] *= sKb; }
         }
         ok = ok && ms.finish(tid);
         if (ok) {
-            float t2[8][4];
-            tmem_frag8(tq + 0 + nk0, t2);
+            float t2[NK][4];
+            tmem_frag<NK>(tq + 0 + nk0, t2);
 #pragma unroll
-            for (int t = 0; t < 8; ++t)
+            for (int t = 0; t < NK; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) de[t][i] += t2[t][i];
-            frag_store_sw<8>(sdE, 64, m0, nk0, de);
+            frag_store_sw<NK>(sdE, 64, m0, nk0, de);
         }
         publish_smem();
 
@@ -392,16 +399,16 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         }
         ok = ok && ms.finish(tid);
         if (ok && has_next) { load_H(nxt); cp_async_commit(); }
-        float dMa[4][4], gr[4][4];
-        float t3[8][4];
+        float dMa[NL][4], gr[NL][4];
+        float t3[NK][4];
         if (ok) {
             // dW = -dE H^T (over the dead dO tile)
-            tmem_frag8(tq + 0 + nk0, t3);
+            tmem_frag<NK>(tq + 0 + nk0, t3);
 #pragma unroll
-            for (int t = 0; t < 8; ++t)
+            for (int t = 0; t < NK; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) t3[t][i] = -t3[t][i];
-            frag_store_sw<8>(sdW, 64, m0, nk0, t3);
+            frag_store_sw<NK>(sdW, 64, m0, nk0, t3);
         }
         publish_smem();
 
@@ -409,33 +416,33 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         // columns (already read); the rest of the R3 epilogue and the dv store run meanwhile
         if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 0, udW, 64, uK, 128, 64, D, false);
         if (ok) {
-            tmem_frag4(tq + 128 + nl0, dMa);
+            tmem_frag<NL>(tq + 128 + nl0, dMa);
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
+            for (int t = 0; t < NL; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dMa[t][i] *= sBe[nl0 + frag_col(t, i)];
             // dV = Diag(beta) M^T dE ; direct dbeta = v . (M^T dE)
-            tmem_frag8(tq + 192 + nk0, t3);
+            tmem_frag<NK>(tq + 192 + nk0, t3);
             float s0, s1;
             tile_rowdot(t3, sV, 64, 0, s0, s1);
             put_rows(2, s0, s1);
             const float ba = sBe[ra], bb = sBe[rb];
 #pragma unroll
-            for (int t = 0; t < 8; ++t) { t3[t][0] *= ba; t3[t][1] *= ba; t3[t][2] *= bb; t3[t][3] *= bb; }
-            frag_stage<8>(stV, m0, nk0, t3);
-            tmem_frag4(tq + 320 + nl0, gr);
+            for (int t = 0; t < NK; ++t) { t3[t][0] *= ba; t3[t][1] *= ba; t3[t][2] *= bb; t3[t][3] *= bb; }
+            frag_stage<NK>(stV, m0, nk0, t3);
+            tmem_frag<NL>(tq + 320 + nl0, gr);
         }
         __syncthreads();
         if (ok) copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, (long long)p.H * D, stV, L, tid);
         ok = ok && ms.finish(tid);
         if (ok && has_next) { load_E(nxt); cp_async_commit(); }
         if (ok) {
-            float mb[4][4];
-            tmem_frag4(tq + 0 + nl0, mb);
+            float mb[NL][4];
+            tmem_frag<NL>(tq + 0 + nl0, mb);
             float rs0 = 0.f, rs1 = 0.f;
-            float cs[4][2];
+            float cs[NL][2];
 #pragma unroll
-            for (int t = 0; t < 4; ++t) {
+            for (int t = 0; t < NL; ++t) {
                 cs[t][0] = cs[t][1] = 0.f;
                 float ph[4], dm[4];
 #pragma unroll
@@ -461,7 +468,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             rs1 = quad_sum(rs1);
             put_rows(3, rs0, rs1);
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
+            for (int t = 0; t < NL; ++t)
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
                     const float v = col_sum8(cs[t][e]);
@@ -474,9 +481,9 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 64, uM, 64, udM, 64, 64, 64, false);
         ok = ok && ms.finish(tid);
         if (ok) {
-            float y[4][4];
-            tmem_frag4(tq + 64 + nl0, y);
-            frag_store_sw<4>(sY, 64, m0, nl0, y);
+            float y[NL][4];
+            tmem_frag<NL>(tq + 64 + nl0, y);
+            frag_store_sw<NL>(sY, 64, m0, nl0, y);
         }
         publish_smem();
 
@@ -484,12 +491,12 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 128, uY, 64, uM, 64, 64, 64, false);
         ok = ok && ms.finish(tid);
         if (ok) {
-            float da[4][4];
-            tmem_frag4(tq + 128 + nl0, da);
+            float da[NL][4];
+            tmem_frag<NL>(tq + 128 + nl0, da);
             float rb0 = 0.f, rb1 = 0.f, ra0 = 0.f, ra1 = 0.f;
-            float cs[4][2];
+            float cs[NL][2];
 #pragma unroll
-            for (int t = 0; t < 4; ++t) {
+            for (int t = 0; t < NL; ++t) {
                 cs[t][0] = cs[t][1] = 0.f;
                 float g4[4];
 #pragma unroll
@@ -515,7 +522,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             put_rows(4, rb0, rb1);
             put_rows(5, ra0, ra1);
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
+            for (int t = 0; t < NL; ++t)
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
                     const float v = col_sum8(cs[t][e]);
@@ -541,11 +548,11 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             rin = load_rows(nxt);
         }
         if (ok) {
-            float t7[8][4], s0, s1;
+            float t7[NK][4], s0, s1;
             // dq = dQ~ ; dd partial = -k . dQ~ ; dk -= d dQ~
-            tmem_frag8(tq + 0 + nk0, t7);
+            tmem_frag<NK>(tq + 0 + nk0, t7);
 #pragma unroll
-            for (int t = 0; t < 8; ++t)
+            for (int t = 0; t < NK; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     acc_dq[t][i] += t7[t][i];
@@ -553,26 +560,26 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
                 }
             tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
             put_rows(6, s0, s1);
-            tmem_frag8(tq + 128 + nk0, t7);
+            tmem_frag<NK>(tq + 128 + nk0, t7);
 #pragma unroll
-            for (int t = 0; t < 8; ++t)
+            for (int t = 0; t < NK; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) acc_dk[t][i] += t7[t][i];
             // W path: M^T dW scaled by btilde gamma_{r-1}; its row dot with k feeds dbtilde and d g_{r-1}
-            tmem_frag8(tq + 256 + nk0, t7);
+            tmem_frag<NK>(tq + 256 + nk0, t7);
             tile_rowdot(t7, sQK, 128, 64, s0, s1);
             put_rows(7, s0, s1);
             const float wa = sWs[ra], wb = sWs[rb];
 #pragma unroll
-            for (int t = 0; t < 8; ++t) {
+            for (int t = 0; t < NK; ++t) {
                 acc_dk[t][0] += wa * t7[t][0]; acc_dk[t][1] += wa * t7[t][1];
                 acc_dk[t][2] += wb * t7[t][2]; acc_dk[t][3] += wb * t7[t][3];
             }
         }
         __syncthreads();   // every row dot has read the Q~/K tile
         if (ok) {
-            frag_stage<8>(sQK, m0, nk0, acc_dq);
-            frag_stage<8>(sQK + 16384, m0, nk0, acc_dk);
+            frag_stage<NK>(sQK, m0, nk0, acc_dq);
+            frag_stage<NK>(sQK + 16384, m0, nk0, acc_dk);
         }
         __syncthreads();
         if (ok) {
@@ -582,7 +589,12 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
         }
 
         // ---------------- per-position scalars (rows 0..63, one thread each)
-        auto rsum = [&](int kind, int r) { return rowp[(kind * 2) * 64 + r] + rowp[(kind * 2 + 1) * 64 + r]; };
+        auto rsum = [&](int kind, int r) {
+            float v = 0.f;
+#pragma unroll
+            for (int j = 0; j < kQ; ++j) v += rowp[(kind * kQ + j) * 64 + r];
+            return v;
+        };
         auto csum = [&](int kind, int c) {
             return colp[(kind * 4 + 0) * 64 + c] + colp[(kind * 4 + 1) * 64 + c] + colp[(kind * 4 + 2) * 64 + c] +
                    colp[(kind * 4 + 3) * 64 + c];
@@ -605,7 +617,7 @@ __global__ void __launch_bounds__(256, 1) k_bwd_local_tc(ChunkParams p, long lon
             // last position; the Kbar terms, which reach it as (their total - their suffix), are
             // added as the exclusive prefix sum_{r < j} instead, so nothing cancels.
             float k0 = lane < L ? rsum(1, lane) : 0.f, k1 = lane + 32 < L ? rsum(1, lane + 32) : 0.f;
-            float hd = lane < 8 ? red[lane] : 0.f;
+            float hd = lane < kLocalThreads / 32 ? red[lane] : 0.f;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) hd += __shfl_xor_sync(0xffffffffu, hd, o);
 #pragma unroll
@@ -684,7 +696,7 @@ cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s) {
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     const long long units = (long long)p.slots * p.H;
     const int grid = (int)(units < nsm ? units : nsm);   // one resident CTA per SM
-    if (grid > 0) tc::k_bwd_local_tc<<<grid, 256, sm, s>>>(p, units);
+    if (grid > 0) tc::k_bwd_local_tc<<<grid, tc::kLocalThreads, sm, s>>>(p, units);
     return cudaGetLastError();
 }
 
