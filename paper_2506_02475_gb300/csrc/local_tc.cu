@@ -290,12 +290,6 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         }
         cp_async_wait<0>();
         __syncthreads();
-        // the next unit's Q/K tile streams in during this unit (its buffer was last read by the
-        // previous unit's staging copies, finished before this unit began)
-        if (has_next) {
-            load_qk(sQKn, nxt);
-            cp_async_commit();
-        }
         // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
         for (int e = tid; e < 64 * 16; e += kLocalThreads) {
             const int r = e >> 4, ch = e & 15;
@@ -307,20 +301,6 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
 #pragma unroll
             for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
             *qa = pack8(qv);
-        }
-        // <H, dH'>: the two tiles share one layout, so matching 16-byte chunks pair up
-        {
-            float sacc = 0.f;
-            for (int e = tid; e < 128 * 16; e += kLocalThreads) {
-                float hv[8], gv[8];
-                unpack8(reinterpret_cast<const uint4*>(sHt)[e], hv);
-                unpack8(reinterpret_cast<const uint4*>(sdHt)[e], gv);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) sacc = fmaf(hv[i], gv[i], sacc);
-            }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, o);
-            if (lane == 0) red[warp] = sacc;
         }
         publish_smem();
 
@@ -335,6 +315,27 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
             tc_gemm_m64<false, true>(tmem + 128, udO, 64, uH, 128, 128, D, false);     // dO H^T
             tc_gemm_m64<false, true>(tmem + 256, uE, 64, udH, 128, 128, D, false);     // E dH'^T
             tc_gemm_m64<false, false>(tmem + 384, uK, 128, udH, 128, 128, D, false);   // K dH'
+        }
+        // While R1 runs: the next unit's Q/K tile starts streaming in (its buffer was last read by
+        // the previous unit's staging copies, finished before this unit began), and <H, dH'> is
+        // formed (R1 reads the same two tiles; both only read them)
+        if (has_next) {
+            load_qk(sQKn, nxt);
+            cp_async_commit();
+        }
+        {
+            // the two tiles share one layout, so matching 16-byte chunks pair up
+            float sacc = 0.f;
+            for (int e = tid; e < 128 * 16; e += kLocalThreads) {
+                float hv[8], gv[8];
+                unpack8(reinterpret_cast<const uint4*>(sHt)[e], hv);
+                unpack8(reinterpret_cast<const uint4*>(sdHt)[e], gv);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) sacc = fmaf(hv[i], gv[i], sacc);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, o);
+            if (lane == 0) red[warp] = sacc;
         }
         ok = ms.finish(tid);
         if (ok && has_next) { load_dH(nxt); cp_async_commit(); }
@@ -360,19 +361,15 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         // the rest of the R1 epilogue runs while it computes
         if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
         if (ok) {
-            // dQ~ part Diag(gamma) dO H^T; its row dot with Q~ is the log-decay gradient of the Q~ H term
+            // dQ~ part Diag(gamma) dO H^T (its row dot with Q~, the log-decay gradient of the Q~ H
+            // term, is taken while R3 runs)
             tmem_frag<NK>(tq + 128 + nk0, acc_dq);
 #pragma unroll
             for (int t = 0; t < NK; ++t) { acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb; }
-            float s0, s1;
-            tile_rowdot(acc_dq, sQK, 128, 0, s0, s1);
-            put_rows(0, s0, s1);
             // dK from Kbar: Diag(gamma_C / gamma_r) E dH'^T
             tmem_frag<NK>(tq + 256 + nk0, acc_dk);
 #pragma unroll
             for (int t = 0; t < NK; ++t) { acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb; }
-            tile_rowdot(acc_dk, sQK, 128, 64, s0, s1);
-            put_rows(1, s0, s1);
             // Kbar dH' part of dE
             tmem_frag<NK>(tq + 384 + nk0, de);
 #pragma unroll
@@ -396,6 +393,15 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
             tc_gemm_m64<false, false>(tmem + 128, udE, 64, uV, 64, 64, D, false);       // dE V^T
             tc_gemm_m64<true, true>(tmem + 192, uM, 64, udE, 64, 128, 64, false);       // M^T dE
             tc_gemm_m64<false, false>(tmem + 320, uK, 128, uK, 128, 64, D, false);      // K K^T
+        }
+        if (ok) {
+            // while R3 runs: the row dots of the two R1 parts with Q~ and with K (used by the
+            // per-position tail only)
+            float s0, s1;
+            tile_rowdot(acc_dq, sQK, 128, 0, s0, s1);
+            put_rows(0, s0, s1);
+            tile_rowdot(acc_dk, sQK, 128, 64, s0, s1);
+            put_rows(1, s0, s1);
         }
         ok = ok && ms.finish(tid);
         if (ok && has_next) { load_H(nxt); cp_async_commit(); }
