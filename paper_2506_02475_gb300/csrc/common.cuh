@@ -501,22 +501,25 @@ __device__ __forceinline__ void unit_lower_inverse_diag16(const float* At, float
 }
 
 // (I + A)^{-1} for a strictly lower 64 x 64 A over 256 threads, in three levels: the four
-// 16 x 16 diagonal blocks (threads 0..63, one column each), then the 32 x 32 blocks
+// 16 x 16 diagonal blocks (warps 0..3, one block each, a column per lane), then the 32 x 32 blocks
 // M10 = -M11 (A10 M00) of both halves, then the 64 x 64 M21 = -M22 (A21 M11).  At is A
 // transposed with pitch 68; M has pitch `pm` and is written in full (zeros above the
 // diagonal); T holds 32 x 36 floats of scratch.
 __device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float* M, int pm, float* T, int tid) {
-    if (tid < 64) {
-        const int j = tid & 15;
-        switch (tid >> 4) {
-            case 0: unit_lower_inverse_diag16<0>(At, M, pm, j); break;
-            case 1: unit_lower_inverse_diag16<16>(At, M, pm, j); break;
-            case 2: unit_lower_inverse_diag16<32>(At, M, pm, j); break;
-            default: unit_lower_inverse_diag16<48>(At, M, pm, j); break;
+    if (tid < 128) {
+        // warp b solves diagonal block b (lanes 0..15, one column each): no divergence between blocks
+        const int j = tid & 31;
+        if (j < 16) {
+            switch (tid >> 5) {
+                case 0: unit_lower_inverse_diag16<0>(At, M, pm, j); break;
+                case 1: unit_lower_inverse_diag16<16>(At, M, pm, j); break;
+                case 2: unit_lower_inverse_diag16<32>(At, M, pm, j); break;
+                default: unit_lower_inverse_diag16<48>(At, M, pm, j); break;
+            }
         }
     } else {
         // zeros above the diagonal blocks: rows 0..47, columns past each row's block
-        for (int e = tid - 64; e < 64 * 64; e += 192) {
+        for (int e = tid - 128; e < 64 * 64; e += 128) {
             const int r = e >> 6, c = e & 63;
             if ((c >> 4) > (r >> 4)) M[r * pm + c] = 0.f;
         }
