@@ -59,10 +59,10 @@ def test_decode_workload_1024_steps_sampled_rows():
     assert rel(np64(st_gpu[rows]), st_ref) <= TOL_BF16
 
 
-@pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_decode_steps_iplr(dtype):
+@pytest.mark.parametrize("dtype,dk", [("f32", 128), ("bf16", 128), ("bf16", 256)])
+def test_decode_steps_iplr(dtype, dk):
     """Comba-iplr decode (feedback strength 2 alpha b beta) against the oracle's iplr step."""
-    Bd, H, dk, dv, steps = 6, 2, 128, 128, 5
+    Bd, H, dv, steps = 6, 2, 128, 5
     state = inputs.decode_state(Bd, H, dk, dv, seed_offset=7)
     b = np.random.default_rng(2).uniform(0, 1, H).astype(np.float32)
     st_gpu = _f32(state)

@@ -1,5 +1,6 @@
 """GPU parity on the method's degenerate gate values, forward and backward, on the tcgen05
-path (bf16, d = 128) and the fp32 path (d = 64):
+path (bf16, d = 128), the fp32 path (d = 64) and head dim 256 (bf16, dk = 256, dv = 128: two
+value heads of width 64 on the mma.sync kernels and the E-form scan):
   * alpha = 1: no decay (chunk log-decays all zero);
   * beta = 0: nothing is written, the output reads the decayed initial state only;
   * b = 0: no state feedback (gated linear attention);
@@ -31,8 +32,8 @@ CASES = {
 }
 
 
-def _workload(dtype, d, case):
-    w = inputs.make("custom", B=2, T=150, H=2, dk=d, dv=d, dtype=dtype, with_b=True, with_h0=True, with_grads=True,
+def _workload(dtype, dk, dv, case):
+    w = inputs.make("custom", B=2, T=150, H=2, dk=dk, dv=dv, dtype=dtype, with_b=True, with_h0=True, with_grads=True,
                     seed_offset=29)
     for key, val in CASES[case].items():
         if key in ("alpha", "beta"):
@@ -50,9 +51,9 @@ def _workload(dtype, d, case):
 
 
 @pytest.mark.parametrize("case", sorted(CASES))
-@pytest.mark.parametrize("dtype,d", [("bf16", 128), ("f32", 64)])
-def test_degenerate_gates(dtype, d, case):
-    w = _workload(dtype, d, case)
+@pytest.mark.parametrize("dtype,dk,dv", [("bf16", 128, 128), ("f32", 64, 64), ("bf16", 256, 128)])
+def test_degenerate_gates(dtype, dk, dv, case):
+    w = _workload(dtype, dk, dv, case)
     t = to_dev(w)
     check_fwd(w, t)
     g = gpu_bwd(t)

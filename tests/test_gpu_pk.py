@@ -116,9 +116,10 @@ def test_pk_full_size_sampled_heads():
     _check(w, p, o, hT, g, heads=[0, 15])
 
 
-@pytest.mark.parametrize("dtype,iplr", [("bf16", False), ("f32", True)])
-def test_pk_decode_steps(dtype, iplr):
-    Bd, H, dk, dv, steps = 5, 3, 128, 128, 6
+@pytest.mark.parametrize("dtype,iplr,dk,dv", [("bf16", False, 128, 128), ("f32", True, 128, 128),
+                                              ("bf16", True, 256, 256)])
+def test_pk_decode_steps(dtype, iplr, dk, dv):
+    Bd, H, steps = 5, 3, 6
     state = inputs.decode_state(Bd, H, dk, dv, seed_offset=3)
     b = np.random.default_rng(5).uniform(0, 1, H).astype(np.float32)
     tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
