@@ -92,6 +92,33 @@ __device__ __forceinline__ void tmem_frag(uint32_t taddr, float (&a)[NT][4]) {
     if constexpr (NT == 2) tmem_frag2(taddr, a);
     else tmem_frag4(taddr, a);
 }
+// Several accumulators read with one wait: tmem_issue() starts a load, tmem_wait() completes
+// every load issued before it, and tmem_take() then moves the words into floats behind an empty
+// asm per register, so that no use of them is scheduled ahead of the wait.
+template <int NT>
+__device__ __forceinline__ void tmem_issue(uint32_t taddr, uint32_t (&r)[NT * 4]) {
+    static_assert(NT == 2 || NT == 4, "column quarters of 64- and 128-wide accumulators");
+    if constexpr (NT == 2) {
+        asm volatile("tcgen05.ld.sync.aligned.16x256b.x2.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n"
+                     : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                     : "r"(taddr));
+    } else {
+        asm volatile(
+            "tcgen05.ld.sync.aligned.16x256b.x4.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+              "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+            : "r"(taddr));
+    }
+}
+__device__ __forceinline__ void tmem_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
+template <int NT>
+__device__ __forceinline__ void tmem_take(uint32_t (&r)[NT * 4], float (&a)[NT][4]) {
+#pragma unroll
+    for (int i = 0; i < NT * 4; ++i) {
+        asm volatile("" : "+r"(r[i]));
+        a[i >> 2][i & 3] = __uint_as_float(r[i]);
+    }
+}
 // Row-major [64][128] bf16 staging with 16-byte chunks rotated by row (conflict-free fragment
 // writes), and its coalesced copy of rows < L to a strided global matrix.
 template <int NT>
@@ -341,8 +368,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         if (ok && has_next) { load_dH(nxt); cp_async_commit(); }
         float sc[NL][4], dP[NL][4], acc_dq[NK][4], acc_dk[NK][4], de[NK][4];
         if (ok) {
-            // P = Tril(S * Gamma)
-            tmem_frag<NL>(tq + 0 + nl0, sc);
+            // P = Tril(S * Gamma); S and dP arrive with one wait
+            uint32_t rS[NL * 4], rP[NL * 4];
+            tmem_issue<NL>(tq + 0 + nl0, rS);
+            tmem_issue<NL>(tq + 64 + nl0, rP);
+            tmem_wait();
+            tmem_take<NL>(rS, sc);
+            tmem_take<NL>(rP, dP);
 #pragma unroll
             for (int t = 0; t < NL; ++t)
 #pragma unroll
@@ -353,7 +385,6 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
                     const float v1 = (c + 1 <= r && r < L) ? sc[t][2 * hh + 1] * __expf(gr - sG[c + 1]) : 0.f;
                     st_pair(sP, 64, r, c, v0, v1);
                 }
-            tmem_frag<NL>(tq + 64 + nl0, dP);
         }
         publish_smem();
 
@@ -361,17 +392,23 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         // the rest of the R1 epilogue runs while it computes
         if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
         if (ok) {
+            // the three other R1 products with one wait
+            uint32_t rq[NK * 4], rk[NK * 4], re[NK * 4];
+            tmem_issue<NK>(tq + 128 + nk0, rq);
+            tmem_issue<NK>(tq + 256 + nk0, rk);
+            tmem_issue<NK>(tq + 384 + nk0, re);
+            tmem_wait();
             // dQ~ part Diag(gamma) dO H^T (its row dot with Q~, the log-decay gradient of the Q~ H
             // term, is taken while R3 runs)
-            tmem_frag<NK>(tq + 128 + nk0, acc_dq);
+            tmem_take<NK>(rq, acc_dq);
 #pragma unroll
             for (int t = 0; t < NK; ++t) { acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb; }
             // dK from Kbar: Diag(gamma_C / gamma_r) E dH'^T
-            tmem_frag<NK>(tq + 256 + nk0, acc_dk);
+            tmem_take<NK>(rk, acc_dk);
 #pragma unroll
             for (int t = 0; t < NK; ++t) { acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb; }
             // Kbar dH' part of dE
-            tmem_frag<NK>(tq + 384 + nk0, de);
+            tmem_take<NK>(re, de);
 #pragma unroll
             for (int t = 0; t < NK; ++t) { de[t][0] *= sKa; de[t][1] *= sKa; de[t][2] *= sKb; de[t][3] *= sKb; }
         }
@@ -422,13 +459,19 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         // columns (already read); the rest of the R3 epilogue and the dv store run meanwhile
         if (ok && tid == 0) tc_gemm_m64<false, false>(tmem + 0, udW, 64, uK, 128, 64, D, false);
         if (ok) {
-            tmem_frag<NL>(tq + 128 + nl0, dMa);
+            // dE V^T, M^T dE and the Gram with one wait
+            uint32_t rm[NL * 4], rt[NK * 4], rg[NL * 4];
+            tmem_issue<NL>(tq + 128 + nl0, rm);
+            tmem_issue<NK>(tq + 192 + nk0, rt);
+            tmem_issue<NL>(tq + 320 + nl0, rg);
+            tmem_wait();
+            tmem_take<NL>(rm, dMa);
 #pragma unroll
             for (int t = 0; t < NL; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dMa[t][i] *= sBe[nl0 + frag_col(t, i)];
             // dV = Diag(beta) M^T dE ; direct dbeta = v . (M^T dE)
-            tmem_frag<NK>(tq + 192 + nk0, t3);
+            tmem_take<NK>(rt, t3);
             float s0, s1;
             tile_rowdot(t3, sV, 64, 0, s0, s1);
             put_rows(2, s0, s1);
@@ -436,7 +479,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
 #pragma unroll
             for (int t = 0; t < NK; ++t) { t3[t][0] *= ba; t3[t][1] *= ba; t3[t][2] *= bb; t3[t][3] *= bb; }
             frag_stage<NK>(stV, m0, nk0, t3);
-            tmem_frag<NL>(tq + 320 + nl0, gr);
+            tmem_take<NL>(rg, gr);
         }
         __syncthreads();
         if (ok) copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, (long long)p.H * D, stV, L, tid);
@@ -555,8 +598,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         }
         if (ok) {
             float t7[NK][4], s0, s1;
+            uint32_t r7a[NK * 4], r7b[NK * 4], r7c[NK * 4];
+            tmem_issue<NK>(tq + 0 + nk0, r7a);
+            tmem_issue<NK>(tq + 128 + nk0, r7b);
+            tmem_issue<NK>(tq + 256 + nk0, r7c);
+            tmem_wait();
             // dq = dQ~ ; dd partial = -k . dQ~ ; dk -= d dQ~
-            tmem_frag<NK>(tq + 0 + nk0, t7);
+            tmem_take<NK>(r7a, t7);
 #pragma unroll
             for (int t = 0; t < NK; ++t)
 #pragma unroll
@@ -566,13 +614,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
                 }
             tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
             put_rows(6, s0, s1);
-            tmem_frag<NK>(tq + 128 + nk0, t7);
+            tmem_take<NK>(r7b, t7);
 #pragma unroll
             for (int t = 0; t < NK; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) acc_dk[t][i] += t7[t][i];
             // W path: M^T dW scaled by btilde gamma_{r-1}; its row dot with k feeds dbtilde and d g_{r-1}
-            tmem_frag<NK>(tq + 256 + nk0, t7);
+            tmem_take<NK>(r7c, t7);
             tile_rowdot(t7, sQK, 128, 64, s0, s1);
             put_rows(7, s0, s1);
             const float wa = sWs[ra], wb = sWs[rb];
