@@ -703,23 +703,35 @@ __global__ void __launch_bounds__(256) k_reduce_heads(ChunkParams p) {
 }
 
 // Value-head groups: out[t, hk, :] = sum_{j < vg} in[t, hk * vg + j, :] in order j = 0, 1, ...
-// for dq, dk (D wide, storage type) and dalpha, dbeta (one float), one thread per element.
+// for dq, dk (D wide, storage type) and dalpha, dbeta (one float).  One thread per 16-byte chunk
+// of a key row (16-byte loads and stores; rows are D * sizeof(T) bytes, a multiple of 16).
 template <typename T>
 __global__ void __launch_bounds__(256) k_group_sum(const T* __restrict__ dq_v, const T* __restrict__ dk_v,
                                                    const float* __restrict__ da_v, const float* __restrict__ db_v,
                                                    T* __restrict__ dq, T* __restrict__ dk, float* __restrict__ dalpha,
                                                    float* __restrict__ dbeta, long long rows_k, int vg, int D) {
+    constexpr int V = 16 / (int)sizeof(T);   // elements per chunk
+    const int CH = D / V;                    // chunks per row
     const long long stride = (long long)gridDim.x * blockDim.x;
-    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < rows_k * D; e += stride) {
-        const long long rk = e / D, c = e - rk * D;   // key row (token * Hk + hk), column
-        float sq = 0.f, sk = 0.f;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < rows_k * CH; e += stride) {
+        const long long rk = e / CH;          // key row (token * Hk + hk)
+        const int c = (int)(e - rk * CH) * V;  // first column of the chunk
+        float sq[V], sk[V];
+#pragma unroll
+        for (int i = 0; i < V; ++i) sq[i] = sk[i] = 0.f;
         for (int j = 0; j < vg; ++j) {
             const long long iv = (rk * vg + j) * D + c;
-            sq += to_f(dq_v[iv]);
-            sk += to_f(dk_v[iv]);
+            union { uint4 u; T x[V]; } a, b;
+            a.u = *reinterpret_cast<const uint4*>(dq_v + iv);
+            b.u = *reinterpret_cast<const uint4*>(dk_v + iv);
+#pragma unroll
+            for (int i = 0; i < V; ++i) { sq[i] += to_f(a.x[i]); sk[i] += to_f(b.x[i]); }
         }
-        dq[e] = from_f<T>(sq);
-        dk[e] = from_f<T>(sk);
+        union { uint4 u; T x[V]; } oq, ov;
+#pragma unroll
+        for (int i = 0; i < V; ++i) { oq.x[i] = from_f<T>(sq[i]); ov.x[i] = from_f<T>(sk[i]); }
+        *reinterpret_cast<uint4*>(dq + rk * D + c) = oq.u;
+        *reinterpret_cast<uint4*>(dk + rk * D + c) = ov.u;
         if (c == 0) {
             float sa = 0.f, sb = 0.f;
             for (int j = 0; j < vg; ++j) { sa += da_v[rk * vg + j]; sb += db_v[rk * vg + j]; }
@@ -737,7 +749,8 @@ cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da
     int dev = 0, nsm = 0;
     cudaError_t e;
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
-    long long blocks = (rows_k * dk_ + 255) / 256;   // grid-stride: at most 8 blocks per SM
+    const long long chunks = rows_k * (dk_ / (is_bf16 ? 8 : 4));
+    long long blocks = (chunks + 255) / 256;   // grid-stride: at most 8 blocks per SM
     if (blocks > 8LL * nsm) blocks = 8LL * nsm;
     if (is_bf16)
         k_group_sum<bf16><<<(unsigned)blocks, 256, 0, s>>>((const bf16*)dq_v, (const bf16*)dk_v, da_v, db_v, (bf16*)dq,
