@@ -261,18 +261,20 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     load_tile_async<T>(sE, PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
     load_tile_async<T>(sH, PK, (const T*)p.Hb + idx * DV * DK, DK, DV, DK, DV, tid, 256);
     load_tile_async<T>(sdH, PK, (const T*)p.dHb + idx * DV * DK, DK, DV, DK, DV, tid, 256);
-    load_tile_async<T>(sM, PL, (const T*)p.Mb + idx * 4096, 64, 64, 64, 64, tid, 256);
+    // M and G are stored once per key head, at its first value head's unit
+    const long long kidx = (long long)slot * p.H + hk * p.vg;
+    load_tile_async<T>(sM, PL, (const T*)p.Mb + kidx * 4096, 64, 64, 64, 64, tid, 256);
     cp_async_commit();
     if (tid < 64) {
-        sG[tid] = p.Gb[idx * 64 + tid];
-        sGm1[tid] = tid > 0 ? p.Gb[idx * 64 + tid - 1] : 0.f;
+        sG[tid] = p.Gb[kidx * 64 + tid];
+        sGm1[tid] = tid > 0 ? p.Gb[kidx * 64 + tid - 1] : 0.f;
         const float be = tid < L ? p.beta[krow(p, t0 + tid, h)] : 0.f;
         sBe[tid] = be;
         const float al = tid < L ? p.alpha[krow(p, t0 + tid, h)] : 1.f;
         const float fsc = feedback_scale(p.iplr, al);
         sBt[tid] = bh * be * fsc;
         sAl[tid] = al;
-        const float em1 = tid > 0 ? __expf(p.Gb[idx * 64 + tid - 1]) : 1.f;
+        const float em1 = tid > 0 ? __expf(p.Gb[kidx * 64 + tid - 1]) : 1.f;
         sEm1[tid] = em1;
         sWs[tid] = bh * be * fsc * em1;
     }

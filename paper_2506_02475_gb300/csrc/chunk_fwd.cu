@@ -149,8 +149,9 @@ __device__ __forceinline__ void gemm_to_global(T* g, const T* sA, int lda, const
 }
 
 // One CTA per (chunk slot, key head).  The Gram, the UT inverse and W depend on the key head
-// only: they are formed once and written to each of its vg value heads (units slot * H + hk *
-// vg + j), which differ in V and so in U = M Diag(beta) V.
+// only: they are formed once, and W, M and the log-decays G are stored once, at the key head's
+// first value-head unit slot * H + hk * vg, where every mma.sync kernel and the dk = 256 scan read
+// them.  The vg value heads (units slot * H + hk * vg + j) differ in V and so in U = M Diag(beta) V.
 template <typename T, int DK, int DV>
 __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
     using S = PrepSmem<T, DK, DV>;
@@ -226,11 +227,9 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
         const float m = sM[r * 65 + c];
         sMw[r * S::PL + c] = from_f<T>(m * sBt[c] * expf(sGm1[c]));
         sMu[r * S::PL + c] = from_f<T>(m * sBe[c]);
-        if (p.Mb)
-            for (int j = 0; j < p.vg; ++j) ((T*)p.Mb + vidx(j) * 4096)[e] = from_f<T>(m);
+        if (p.Mb) ((T*)p.Mb + vidx(0) * 4096)[e] = from_f<T>(m);
     }
-    if (tid < 64)
-        for (int j = 0; j < p.vg; ++j) p.Gb[vidx(j) * 64 + tid] = sG[tid];
+    if (tid < 64) p.Gb[vidx(0) * 64 + tid] = sG[tid];
     __syncthreads();
 
     // W = Mw P, U = Mu V (stored) and, for the chunk's state map, their Kbar-row-scaled copies.
@@ -240,8 +239,7 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
         float acc[DK / 8][4];
         zero(acc);
         warp_gemm<true, false, DK / 8>(acc, sMw, S::PL, sF, S::PK, 16 * warp, 0, 64);
-        for (int j = 0; j < p.vg; ++j)
-            frag_store_global<T, DK / 8>((T*)p.Wb + vidx(j) * 64 * DK, DK, 16 * warp, 0, acc, 64);
+        frag_store_global<T, DK / 8>((T*)p.Wb + vidx(0) * 64 * DK, DK, 16 * warp, 0, acc, 64);
         if constexpr (kMap) {
 #pragma unroll
             for (int t = 0; t < DK / 8; ++t) { acc[t][0] *= sa; acc[t][1] *= sa; acc[t][2] *= sb; acc[t][3] *= sb; }

@@ -562,6 +562,11 @@ static bool make_map(CUtensorMap* m, const void* base, long long rows, int cols,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The same view for other kernels (scan_wide.cu).
+bool make_bf16_map(CUtensorMap* m, const void* base, long long rows, int cols, int box_rows) {
+    return make_map(m, base, rows, cols, box_rows);
+}
+
 template <int DK, int DV, bool XMN>
 static cudaError_t run_scan_tc_split(const ScanArgs& a, long long pairs, cudaStream_t s) {
     using S = ScanSplitSmem<DK, DV>;
