@@ -112,14 +112,14 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 110_760, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_169, ('scan.cu', 'common.cuh', 'params.cuh'), "6c77bca293e56549"),
-    "output": ("k_output_tc", 118_698, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
-    "bwd_prep": ("k_bwd_prep_tc", 82_499, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "33a092f58ffd7083"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_249, ('scan.cu', 'common.cuh', 'params.cuh'), "6c77bca293e56549"),
-    "bwd_local": ("k_bwd_local_tc", 194_243, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "1123096a93568c0f"),
+    "prep": ("k_prep_tc", 110_685, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "87c8dc1931f1d8d9"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_123, ('scan.cu', 'common.cuh', 'params.cuh'), "a8e4b04b79c9cb5a"),
+    "output": ("k_output_tc", 118_597, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "87c8dc1931f1d8d9"),
+    "bwd_prep": ("k_bwd_prep_tc", 82_535, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "87c8dc1931f1d8d9"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_383, ('scan.cu', 'common.cuh', 'params.cuh'), "a8e4b04b79c9cb5a"),
+    "bwd_local": ("k_bwd_local_tc", 194_446, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "0768c8a76ce490a8"),
 }
-DECODE_TRAFFIC = (481_306_880, ('decode.cu', 'common.cuh', 'params.cuh'), "988ef445c98cc562")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (481_318_912, ('decode.cu', 'common.cuh', 'params.cuh'), "5d94f1984c163f43")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
