@@ -22,8 +22,8 @@ struct Layout {
     size_t qh, kh, ga, gb, bg, dqh, dkh, dal, dbe, dbi, dar, dcr, dpa, dpc;
     // Comba-pk (COMBA_PK): the corrected queries q - d p and the zero d the chunk kernels then see
     size_t qt, dz;
-    // value-head groups (vg > 1): the backward's per-value-head dq, dk, dalpha, dbeta
-    size_t gdq, gdk, gda, gdb;
+    // value-head groups (vg > 1): the backward's per-value-head dq, dk, dalpha, dbeta (and dp)
+    size_t gdq, gdk, gda, gdb, gdp;
     size_t total;
     int slots;
     int vg;      // value heads per key head; the kernels see H * vg heads of width dv / vg
@@ -52,9 +52,9 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (s->chunk != comba::kChunk) return COMBA_ERR_UNSUPPORTED;
     const int vg = value_groups(s);
     if (s->dk == 256) {
-        // head dim 256 (bf16, plain or iplr form): value heads 64 wide, at most four per key head
+        // head dim 256 (bf16; plain, iplr or pk form): value heads 64 wide, at most four per key head
         if (s->dtype != COMBA_BF16 || s->dv < 64 || s->dv % 64 != 0 || vg > 4) return COMBA_ERR_UNSUPPORTED;
-        if (s->flags & (COMBA_GATED | COMBA_PK)) return COMBA_ERR_UNSUPPORTED;
+        if (s->flags & COMBA_GATED) return COMBA_ERR_UNSUPPORTED;
     } else if (vg > 1) {
         // dv = 256, 384 or 512 as groups of 128-wide value heads on the tcgen05 path
         if (s->dv % 128 != 0 || vg > 4 || s->dk != 128 || s->dtype != COMBA_BF16) return COMBA_ERR_UNSUPPORTED;
@@ -135,6 +135,7 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
         L.gdk = take(vrows * dk * es);
         L.gda = take(vrows * sizeof(float));
         L.gdb = take(vrows * sizeof(float));
+        if (s->flags & COMBA_PK) L.gdp = take(vrows * dk * es);
     }
     L.total = o;
     L.slots = (int)slots;
@@ -269,6 +270,7 @@ comba_status_t backward_run(const comba_shape_t* shape, const Layout& L, void* w
         p.dq = w + L.gdq; p.dkk = w + L.gdk;
         p.dalpha = reinterpret_cast<float*>(w + L.gda);
         p.dbeta = reinterpret_cast<float*>(w + L.gdb);
+        if (pk.dp) p.dpp = w + L.gdp;
     }
     const bool bf = shape->dtype == COMBA_BF16;
     comba::mark(p, 0, s);
@@ -283,8 +285,8 @@ comba_status_t backward_run(const comba_shape_t* shape, const Layout& L, void* w
         if (comba::launch_fwd(f, bf, true, s, 1) != cudaSuccess) return COMBA_ERR_CUDA;
     }
     if (comba::launch_bwd(p, bf, s, 4) != cudaSuccess) return COMBA_ERR_CUDA;
-    if (L.vg > 1 && comba::launch_group_sum(p.dq, p.dkk, p.dalpha, p.dbeta, dq, dk, dalpha, dbeta, p.Ttot, p.H, L.vg,
-                                            p.dk, bf, s) != cudaSuccess)
+    if (L.vg > 1 && comba::launch_group_sum(p.dq, p.dkk, p.dalpha, p.dbeta, pk.dp ? p.dpp : nullptr, dq, dk, dalpha,
+                                            dbeta, pk.dp, p.Ttot, p.H, L.vg, p.dk, bf, s) != cudaSuccess)
         return COMBA_ERR_CUDA;
     return COMBA_OK;
 }

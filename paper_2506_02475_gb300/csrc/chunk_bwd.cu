@@ -705,35 +705,43 @@ __global__ void __launch_bounds__(256) k_reduce_heads(ChunkParams p) {
 }
 
 // Value-head groups: out[t, hk, :] = sum_{j < vg} in[t, hk * vg + j, :] in order j = 0, 1, ...
-// for dq, dk (D wide, storage type) and dalpha, dbeta (one float).  One thread per 16-byte chunk
-// of a key row (16-byte loads and stores; rows are D * sizeof(T) bytes, a multiple of 16).
+// for dq, dk and, with Comba-pk feedback vectors, dp (D wide, storage type; dp_v null without
+// them) and dalpha, dbeta (one float).  One thread per 16-byte chunk of a key row (16-byte loads
+// and stores; rows are D * sizeof(T) bytes, a multiple of 16).
+template <typename T>
+__device__ __forceinline__ void group_sum_chunk(const T* __restrict__ in, T* __restrict__ out, long long rk, int c,
+                                                int vg, int D) {
+    constexpr int V = 16 / (int)sizeof(T);
+    float a[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) a[i] = 0.f;
+    for (int j = 0; j < vg; ++j) {
+        union { uint4 u; T x[V]; } w;
+        w.u = *reinterpret_cast<const uint4*>(in + (rk * vg + j) * D + c);
+#pragma unroll
+        for (int i = 0; i < V; ++i) a[i] += to_f(w.x[i]);
+    }
+    union { uint4 u; T x[V]; } o;
+#pragma unroll
+    for (int i = 0; i < V; ++i) o.x[i] = from_f<T>(a[i]);
+    *reinterpret_cast<uint4*>(out + rk * D + c) = o.u;
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256) k_group_sum(const T* __restrict__ dq_v, const T* __restrict__ dk_v,
                                                    const float* __restrict__ da_v, const float* __restrict__ db_v,
-                                                   T* __restrict__ dq, T* __restrict__ dk, float* __restrict__ dalpha,
-                                                   float* __restrict__ dbeta, long long rows_k, int vg, int D) {
+                                                   const T* __restrict__ dp_v, T* __restrict__ dq, T* __restrict__ dk,
+                                                   float* __restrict__ dalpha, float* __restrict__ dbeta,
+                                                   T* __restrict__ dp, long long rows_k, int vg, int D) {
     constexpr int V = 16 / (int)sizeof(T);   // elements per chunk
     const int CH = D / V;                    // chunks per row
     const long long stride = (long long)gridDim.x * blockDim.x;
     for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < rows_k * CH; e += stride) {
         const long long rk = e / CH;          // key row (token * Hk + hk)
         const int c = (int)(e - rk * CH) * V;  // first column of the chunk
-        float sq[V], sk[V];
-#pragma unroll
-        for (int i = 0; i < V; ++i) sq[i] = sk[i] = 0.f;
-        for (int j = 0; j < vg; ++j) {
-            const long long iv = (rk * vg + j) * D + c;
-            union { uint4 u; T x[V]; } a, b;
-            a.u = *reinterpret_cast<const uint4*>(dq_v + iv);
-            b.u = *reinterpret_cast<const uint4*>(dk_v + iv);
-#pragma unroll
-            for (int i = 0; i < V; ++i) { sq[i] += to_f(a.x[i]); sk[i] += to_f(b.x[i]); }
-        }
-        union { uint4 u; T x[V]; } oq, ov;
-#pragma unroll
-        for (int i = 0; i < V; ++i) { oq.x[i] = from_f<T>(sq[i]); ov.x[i] = from_f<T>(sk[i]); }
-        *reinterpret_cast<uint4*>(dq + rk * D + c) = oq.u;
-        *reinterpret_cast<uint4*>(dk + rk * D + c) = ov.u;
+        group_sum_chunk(dq_v, dq, rk, c, vg, D);
+        group_sum_chunk(dk_v, dk, rk, c, vg, D);
+        if (dp_v) group_sum_chunk(dp_v, dp, rk, c, vg, D);
         if (c == 0) {
             float sa = 0.f, sb = 0.f;
             for (int j = 0; j < vg; ++j) { sa += da_v[rk * vg + j]; sb += db_v[rk * vg + j]; }
@@ -743,9 +751,9 @@ __global__ void __launch_bounds__(256) k_group_sum(const T* __restrict__ dq_v, c
     }
 }
 
-cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da_v, const float* db_v, void* dq,
-                             void* dk, float* dalpha, float* dbeta, long long tokens, int H, int vg, int dk_,
-                             bool is_bf16, cudaStream_t s) {
+cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da_v, const float* db_v,
+                             const void* dp_v, void* dq, void* dk, float* dalpha, float* dbeta, void* dp,
+                             long long tokens, int H, int vg, int dk_, bool is_bf16, cudaStream_t s) {
     const long long rows_k = tokens * (H / vg);
     if (rows_k <= 0) return cudaSuccess;
     int dev = 0, nsm = 0;
@@ -755,11 +763,13 @@ cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da
     long long blocks = (chunks + 255) / 256;   // grid-stride: at most 8 blocks per SM
     if (blocks > 8LL * nsm) blocks = 8LL * nsm;
     if (is_bf16)
-        k_group_sum<bf16><<<(unsigned)blocks, 256, 0, s>>>((const bf16*)dq_v, (const bf16*)dk_v, da_v, db_v, (bf16*)dq,
-                                                          (bf16*)dk, dalpha, dbeta, rows_k, vg, dk_);
+        k_group_sum<bf16><<<(unsigned)blocks, 256, 0, s>>>((const bf16*)dq_v, (const bf16*)dk_v, da_v, db_v,
+                                                          (const bf16*)dp_v, (bf16*)dq, (bf16*)dk, dalpha, dbeta,
+                                                          (bf16*)dp, rows_k, vg, dk_);
     else
         k_group_sum<float><<<(unsigned)blocks, 256, 0, s>>>((const float*)dq_v, (const float*)dk_v, da_v, db_v,
-                                                           (float*)dq, (float*)dk, dalpha, dbeta, rows_k, vg, dk_);
+                                                           (const float*)dp_v, (float*)dq, (float*)dk, dalpha, dbeta,
+                                                           (float*)dp, rows_k, vg, dk_);
     return cudaGetLastError();
 }
 

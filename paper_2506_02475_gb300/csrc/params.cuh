@@ -172,10 +172,11 @@ cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, c
                                   const void* v, const void* p, const float* alpha, const float* beta,
                                   const float* b, const float* d, float* state, void* o, bool iplr, cudaStream_t s);
 // Value-head groups: sums over the vg value heads of each key head, in a fixed order, of the
-// backward's per-value-head dq, dk [tokens, H, dk] (storage type) and dalpha, dbeta [tokens, H].
-cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da_v, const float* db_v, void* dq,
-                             void* dk, float* dalpha, float* dbeta, long long tokens, int H, int vg, int dk_,
-                             bool is_bf16, cudaStream_t s);
+// backward's per-value-head dq, dk [tokens, H, dk] (storage type), dalpha, dbeta [tokens, H] and,
+// with Comba-pk feedback vectors, dp (dp_v and dp null otherwise).
+cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da_v, const float* db_v,
+                             const void* dp_v, void* dq, void* dk, float* dalpha, float* dbeta, void* dp,
+                             long long tokens, int H, int vg, int dk_, bool is_bf16, cudaStream_t s);
 // Comba-pk correction applied before the chunk kernels: qt = q - d_h p over [rows = tokens*H, dk].
 cudaError_t launch_pk_qtilde(const void* q, const void* p, const float* d, void* qt, long long rows, int H, int dk,
                              bool is_bf16, cudaStream_t s);

@@ -217,13 +217,16 @@ def test_value_head_groups(L):
 
 
 def test_head_dim_256(L):
-    """dk = 256 (bf16, plain or iplr) runs as value heads 64 wide: dv = 64 .. 256 in steps of 64."""
+    """dk = 256 (bf16; plain, iplr or pk form) runs as value heads 64 wide: dv = 64 .. 256 in steps of 64."""
     w64, w128, w256 = (ws(L, shape(dk=256, dv=d), 1) for d in (64, 128, 256))
     assert 0 < w64 < w128 < w256
     assert ws(L, shape(dk=256, dv=192), 0) > 0
     assert ws(L, shape(dk=256, dv=64, flags=4), 1) > 0
-    for kw in (dict(dv=320), dict(dv=32), dict(dv=96), dict(dtype=0), dict(flags=8), dict(flags=16)):
+    for kw in (dict(dv=320), dict(dv=32), dict(dv=96), dict(dtype=0), dict(flags=8)):
         assert ws(L, shape(dk=256, **kw)) == 0, kw
+    # Comba-pk at head dim 256: the workspace also holds q - d p and, with value-head groups, the
+    # per-value-head dp
+    assert ws(L, shape(dk=256, dv=128, flags=16), 1) > ws(L, shape(dk=256, dv=128), 1)
 
     def step(dv, dk=256):
         return L.comba_recurrent_step(4, 2, dk, dv, 1, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 0,

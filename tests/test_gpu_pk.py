@@ -73,6 +73,9 @@ CASES = [
     ("bf16", 64, 128, 1, 127, None, "splr"),
     ("f32", 64, 64, 2, 200, None, "splr"),
     ("f32", 64, 64, 1, None, [70, 0, 5, 133], "iplr"),
+    # head dim 256: one value head of width 64, then two (dp summed over them like dq and dk)
+    ("bf16", 256, 64, 2, 150, None, "splr"),
+    ("bf16", 256, 128, 1, None, [1, 63, 64, 65, 0, 90], "iplr"),
 ]
 
 
