@@ -46,7 +46,8 @@ struct ChunkParams {
     float* dd;
     float* dh0;
 
-    // workspace views (per (slot, head) pair idx = slot*H + h)
+    // workspace views (per (slot, head) pair idx = slot*H + h; with value-head groups on the
+    // mma.sync path, W, G and M are stored once per key head, at its first value head's pair)
     SlotInfo* slot_info;     // [slots]
     int* seq_first;          // [N+1] first slot of each sequence
     void* Wb;                // [pairs][64][dk]  WY factor W (storage type)
