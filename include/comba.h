@@ -47,9 +47,9 @@
  *     runs as dv / 128 value heads of width 128 that share its q, k and gates
  *     (a state's columns evolve independently), and the key-side gradients are
  *     summed over them in a fixed order.
- *   - dk = 256 (the paper's head dim 256; bf16; plain, iplr or pk form) with
- *     dv = 64, 128, 192 or 256: value heads 64 wide, the same way (with pk, dp
- *     is summed over a key head's value heads like dq and dk).
+ *   - dk = 256 (the paper's head dim 256; bf16; plain, iplr, pk or gated form)
+ *     with dv = 64, 128, 192 or 256: value heads 64 wide, the same way (with
+ *     pk, dp is summed over a key head's value heads like dq and dk).
  */
 #ifndef COMBA_H
 #define COMBA_H
@@ -79,8 +79,8 @@ typedef struct {
     int dk;                     /* key/query head dim: 64, 128 or 256             */
     int dv;                     /* value head dim: 64 or 128; with dk = 128 also  */
                                 /* 256, 384, 512; with dk = 256 64, 128, 192, 256 */
-                                /* (wider dv and dk = 256: bf16, no gated form;   */
-                                /* see "Head widths" below)                       */
+                                /* (wider dv and dk = 256: bf16; see "Head        */
+                                /* widths" below)                                 */
     int num_seqs;               /* N: == B when cu_seqlens == NULL                */
     const int32_t *cu_seqlens;  /* device int32 [N+1] or NULL                     */
     comba_dtype_t dtype;        /* storage type of q, k, v, o and their grads     */

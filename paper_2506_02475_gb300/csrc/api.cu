@@ -52,9 +52,8 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     if (s->chunk != comba::kChunk) return COMBA_ERR_UNSUPPORTED;
     const int vg = value_groups(s);
     if (s->dk == 256) {
-        // head dim 256 (bf16; plain, iplr or pk form): value heads 64 wide, at most four per key head
+        // head dim 256 (bf16; plain, iplr, pk or gated form): value heads 64 wide, at most four per key head
         if (s->dtype != COMBA_BF16 || s->dv < 64 || s->dv % 64 != 0 || vg > 4) return COMBA_ERR_UNSUPPORTED;
-        if (s->flags & COMBA_GATED) return COMBA_ERR_UNSUPPORTED;
     } else if (vg > 1) {
         // dv = 256, 384 or 512 as groups of 128-wide value heads on the tcgen05 path
         if (s->dv % 128 != 0 || vg > 4 || s->dk != 128 || s->dtype != COMBA_BF16) return COMBA_ERR_UNSUPPORTED;

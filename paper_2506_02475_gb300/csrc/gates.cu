@@ -120,9 +120,9 @@ struct ProStage {   // one slot of the prologue ring
     T q[kStageRows * DK], k[kStageRows * DK];
     float ga[kStageRows], gb[kStageRows];
 };
-template <typename T, int DK>
-struct EpiStage {   // one slot of the epilogue ring
-    T q[kStageRows * DK], dq[kStageRows * DK], k[kStageRows * DK], dk[kStageRows * DK];
+template <typename T, int DK, int NP>
+struct EpiStage {   // one slot of the epilogue ring: NP (x, dx_hat) pairs, q then k
+    T x[NP][kStageRows * DK], dx[NP][kStageRows * DK];
     float ga[kStageRows], al[kStageRows], dal[kStageRows], be[kStageRows], dbe[kStageRows];
 };
 
@@ -189,9 +189,16 @@ __global__ void __launch_bounds__(kGateThreads) k_gate_prologue(GateParams g) {
     cp_async_wait<0>();
 }
 
-template <typename T, int DK>
-__global__ void __launch_bounds__(kGateThreads) k_gate_epilogue(GateParams g) {
-    using S = EpiStage<T, DK>;
+// NP = 2: q and k in one pass.  NP = 1 (head dim 256, whose four [64][256] tiles would not fit
+// two ring slots): pass 0 takes q and the gates, pass 1 k.
+template <typename T, int DK, int NP>
+__global__ void __launch_bounds__(kGateThreads) k_gate_epilogue(GateParams g, int pass) {
+    using S = EpiStage<T, DK, NP>;
+    const bool gates = pass == 0;
+    // pair j's raw input, chunk-backward gradient and output
+    auto src = [&](int j) { return (NP == 2 ? j : pass) == 0 ? (const T*)g.q : (const T*)g.k; };
+    auto dsrc = [&](int j) { return (NP == 2 ? j : pass) == 0 ? (const T*)g.dqh : (const T*)g.dkh; };
+    auto dst = [&](int j) { return (NP == 2 ? j : pass) == 0 ? (T*)g.dq : (T*)g.dk; };
     constexpr int NS = Ring<(int)sizeof(S)>::n;
     extern __shared__ __align__(128) unsigned char gate_smem[];
     S* ring = reinterpret_cast<S*>(gate_smem);
@@ -203,16 +210,19 @@ __global__ void __launch_bounds__(kGateThreads) k_gate_epilogue(GateParams g) {
             const long long row0 = (blockIdx.x + i * gridDim.x) * kStageRows;
             const int nr = (int)(g.rows - row0 < kStageRows ? g.rows - row0 : kStageRows);
             S& st = ring[i % NS];
-            stage_rows<T, DK>(st.q, (const T*)g.q, row0, nr, tid, kGateThreads);
-            stage_rows<T, DK>(st.dq, (const T*)g.dqh, row0, nr, tid, kGateThreads);
-            stage_rows<T, DK>(st.k, (const T*)g.k, row0, nr, tid, kGateThreads);
-            stage_rows<T, DK>(st.dk, (const T*)g.dkh, row0, nr, tid, kGateThreads);
+#pragma unroll
+            for (int j = 0; j < NP; ++j) {
+                stage_rows<T, DK>(st.x[j], src(j), row0, nr, tid, kGateThreads);
+                stage_rows<T, DK>(st.dx[j], dsrc(j), row0, nr, tid, kGateThreads);
+            }
             constexpr int SC = kStageRows / 4;   // 16-byte chunks of a stage's per-row floats
-            if (tid < SC) stage_scalars(st.ga, g.g_alpha, row0, nr, tid);
-            else if (tid < 2 * SC) stage_scalars(st.al, g.alpha, row0, nr, tid - SC);
-            else if (tid < 3 * SC) stage_scalars(st.dal, g.dalpha, row0, nr, tid - 2 * SC);
-            else if (tid < 4 * SC) stage_scalars(st.be, g.beta, row0, nr, tid - 3 * SC);
-            else if (tid < 5 * SC) stage_scalars(st.dbe, g.dbeta, row0, nr, tid - 4 * SC);
+            if (gates) {
+                if (tid < SC) stage_scalars(st.ga, g.g_alpha, row0, nr, tid);
+                else if (tid < 2 * SC) stage_scalars(st.al, g.alpha, row0, nr, tid - SC);
+                else if (tid < 3 * SC) stage_scalars(st.dal, g.dalpha, row0, nr, tid - 2 * SC);
+                else if (tid < 4 * SC) stage_scalars(st.be, g.beta, row0, nr, tid - 3 * SC);
+                else if (tid < 5 * SC) stage_scalars(st.dbe, g.dbeta, row0, nr, tid - 4 * SC);
+            }
         }
         cp_async_commit();
     };
@@ -225,7 +235,7 @@ __global__ void __launch_bounds__(kGateThreads) k_gate_epilogue(GateParams g) {
         const long long row0 = (blockIdx.x + i * gridDim.x) * kStageRows;
         const int nr = (int)(g.rows - row0 < kStageRows ? g.rows - row0 : kStageRows);
         const int sr = tid - (kGateThreads - kStageRows);   // the last warps' threads: one row's gates each
-        if (sr >= 0 && sr < nr) {
+        if (gates && sr >= 0 && sr < nr) {
             const long long row = row0 + sr;
             const int h = (int)(row % g.H);
             const float z = st.ga[sr] + g.c[h], al = st.al[sr], dal = st.dal[sr], be = st.be[sr];
@@ -237,8 +247,9 @@ __global__ void __launch_bounds__(kGateThreads) k_gate_epilogue(GateParams g) {
         }
         {
             const int r = tid >> 3, l = tid & 7;
-            unnormalise_part<T, DK>(st.q + r * DK, st.dq + r * DK, (T*)g.dq + (row0 + r) * DK, r < nr, g.eps, l);
-            unnormalise_part<T, DK>(st.k + r * DK, st.dk + r * DK, (T*)g.dk + (row0 + r) * DK, r < nr, g.eps, l);
+#pragma unroll
+            for (int j = 0; j < NP; ++j)
+                unnormalise_part<T, DK>(st.x[j] + r * DK, st.dx[j] + r * DK, dst(j) + (row0 + r) * DK, r < nr, g.eps, l);
         }
     }
     cp_async_wait<0>();
@@ -303,8 +314,8 @@ __global__ void __launch_bounds__(256) k_gate_reduce(GateParams g, int nblk) {
 }
 
 // Grid-stride launch over 64-row stages: one block per SM (the ring fills shared memory).
-template <typename K>
-static cudaError_t launch_ring(K kernel, int smem, const GateParams& g, cudaStream_t s) {
+template <typename K, typename... A>
+static cudaError_t launch_ring(K kernel, int smem, const GateParams& g, cudaStream_t s, A... args) {
     int dev = 0, nsm = 0;
     cudaError_t e;
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) ||
@@ -312,7 +323,7 @@ static cudaError_t launch_ring(K kernel, int smem, const GateParams& g, cudaStre
         return e;
     const long long nstages = (g.rows + kStageRows - 1) / kStageRows;
     const long long grid = nstages < nsm ? (nstages > 0 ? nstages : 1) : nsm;
-    kernel<<<(unsigned)grid, kGateThreads, smem, s>>>(g);
+    kernel<<<(unsigned)grid, kGateThreads, smem, s>>>(g, args...);
     return cudaGetLastError();
 }
 
@@ -323,19 +334,30 @@ static cudaError_t run_prologue(const GateParams& g, cudaStream_t s) {
 }
 template <typename T, int DK>
 static cudaError_t run_epilogue(const GateParams& g, cudaStream_t s) {
-    static_assert(Ring<(int)sizeof(EpiStage<T, DK>)>::bytes <= 227 * 1024, "epilogue ring exceeds shared memory");
-    return launch_ring(k_gate_epilogue<T, DK>, Ring<(int)sizeof(EpiStage<T, DK>)>::bytes, g, s);
+    constexpr int one = Ring<(int)sizeof(EpiStage<T, DK, 2>)>::bytes;
+    if constexpr (one <= 227 * 1024) {
+        return launch_ring(k_gate_epilogue<T, DK, 2>, one, g, s, 0);
+    } else {
+        constexpr int two = Ring<(int)sizeof(EpiStage<T, DK, 1>)>::bytes;
+        static_assert(two <= 227 * 1024, "epilogue ring exceeds shared memory");
+        cudaError_t e = launch_ring(k_gate_epilogue<T, DK, 1>, two, g, s, 0);
+        return e ? e : launch_ring(k_gate_epilogue<T, DK, 1>, two, g, s, 1);
+    }
 }
 
 cudaError_t launch_gate_prologue(const GateParams& g, bool is_bf16, int dk, cudaStream_t s) {
-    if (is_bf16) return dk == 128 ? run_prologue<bf16, 128>(g, s) : run_prologue<bf16, 64>(g, s);
+    if (is_bf16) {
+        if (dk == 256) return run_prologue<bf16, 256>(g, s);
+        return dk == 128 ? run_prologue<bf16, 128>(g, s) : run_prologue<bf16, 64>(g, s);
+    }
     return dk == 128 ? run_prologue<float, 128>(g, s) : run_prologue<float, 64>(g, s);
 }
 
 cudaError_t launch_gate_epilogue(const GateParams& g, bool is_bf16, int dk, cudaStream_t s) {
     cudaError_t e;
     if (g.rows > 0) {
-        if (is_bf16) e = dk == 128 ? run_epilogue<bf16, 128>(g, s) : run_epilogue<bf16, 64>(g, s);
+        if (is_bf16) e = dk == 256 ? run_epilogue<bf16, 256>(g, s)
+                                   : (dk == 128 ? run_epilogue<bf16, 128>(g, s) : run_epilogue<bf16, 64>(g, s));
         else if (dk == 64) e = run_epilogue<float, 64>(g, s);   // the fp32 backward runs dk = dv = 64 only
         else return cudaErrorInvalidValue;
         if (e) return e;

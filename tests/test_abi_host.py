@@ -217,13 +217,14 @@ def test_value_head_groups(L):
 
 
 def test_head_dim_256(L):
-    """dk = 256 (bf16; plain, iplr or pk form) runs as value heads 64 wide: dv = 64 .. 256 in steps of 64."""
+    """dk = 256 (bf16; plain, iplr, pk or gated form) runs as value heads 64 wide: dv = 64 .. 256 in steps of 64."""
     w64, w128, w256 = (ws(L, shape(dk=256, dv=d), 1) for d in (64, 128, 256))
     assert 0 < w64 < w128 < w256
     assert ws(L, shape(dk=256, dv=192), 0) > 0
     assert ws(L, shape(dk=256, dv=64, flags=4), 1) > 0
-    for kw in (dict(dv=320), dict(dv=32), dict(dv=96), dict(dtype=0), dict(flags=8)):
+    for kw in (dict(dv=320), dict(dv=32), dict(dv=96), dict(dtype=0)):
         assert ws(L, shape(dk=256, **kw)) == 0, kw
+    assert ws(L, shape(dk=256, dv=256, flags=8), 1) > ws(L, shape(dk=256, dv=256), 1)   # gated: the prologue's outputs
     # Comba-pk at head dim 256: the workspace also holds q - d p and, with value-head groups, the
     # per-value-head dp
     assert ws(L, shape(dk=256, dv=128, flags=16), 1) > ws(L, shape(dk=256, dv=128), 1)

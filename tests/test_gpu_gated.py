@@ -95,11 +95,14 @@ def _check(w, variant, o, hT, g):
     assert not bad, (bad, errs)
 
 
-@pytest.mark.parametrize("dtype,d,lens,variant", [("bf16", 128, [130, 0, 257, 64], "splr"),
-                                                   ("bf16", 128, None, "iplr"),
-                                                   ("f32", 64, [70, 5, 133], "splr")])
-def test_gated_forward_backward(dtype, d, lens, variant):
-    w = inputs.make_gated(B=2, T=200, H=3, dk=d, dv=d, dtype=dtype, seed_offset=d + len(lens or []), lengths=lens)
+@pytest.mark.parametrize("dtype,d,dv,lens,variant", [("bf16", 128, 128, [130, 0, 257, 64], "splr"),
+                                                      ("bf16", 128, 128, None, "iplr"),
+                                                      ("f32", 64, 64, [70, 5, 133], "splr"),
+                                                      # head dim 256: two value heads of width 64, and
+                                                      # the epilogue's two passes (q, then k)
+                                                      ("bf16", 256, 128, [130, 0, 77], "splr")])
+def test_gated_forward_backward(dtype, d, dv, lens, variant):
+    w = inputs.make_gated(B=2, T=200, H=3, dk=d, dv=dv, dtype=dtype, seed_offset=d + len(lens or []), lengths=lens)
     _check(w, variant, *_run(w, variant))
 
 
