@@ -43,7 +43,7 @@
  *
  * Head widths (chunk entry points; comba_workspace_size returns 0 for the rest)
  *   - dk, dv in {64, 128}, either storage type (the fp32 backward: dk = dv = 64).
- *   - dk = 128 with dv = 256, 384 or 512 (bf16, plain or iplr form): each head
+ *   - dk = 128 with dv = 256, 384 or 512 (bf16, any of the four forms): each head
  *     runs as dv / 128 value heads of width 128 that share its q, k and gates
  *     (a state's columns evolve independently), and the key-side gradients are
  *     summed over them in a fixed order.

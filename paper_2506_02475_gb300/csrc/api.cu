@@ -29,9 +29,9 @@ struct Layout {
     int vg;      // value heads per key head; the kernels see H * vg heads of width dv / vg
 };
 
-// Value heads per key head: dv beyond 128 (a multiple of 128, dk = 128, bf16, plain or iplr
-// form) runs as dv / 128 value heads of width 128 that share the key head's q, k and gates;
-// at head dim dk = 256 the value heads are 64 wide (dv = 64 .. 256).
+// Value heads per key head: dv beyond 128 (a multiple of 128, dk = 128, bf16) runs as dv / 128
+// value heads of width 128 that share the key head's q, k (p) and gates; at head dim dk = 256 the
+// value heads are 64 wide (dv = 64 .. 256).
 int value_groups(const comba_shape_t* s) {
     if (s->dk == 256) return s->dv >= 64 ? s->dv / 64 : 1;
     return s->dv > 128 ? s->dv / 128 : 1;
@@ -57,7 +57,6 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     } else if (vg > 1) {
         // dv = 256, 384 or 512 as groups of 128-wide value heads on the tcgen05 path
         if (s->dv % 128 != 0 || vg > 4 || s->dk != 128 || s->dtype != COMBA_BF16) return COMBA_ERR_UNSUPPORTED;
-        if (s->flags & (COMBA_GATED | COMBA_PK)) return COMBA_ERR_UNSUPPORTED;
     } else if ((s->dk != 64 && s->dk != 128) || (s->dv != 64 && s->dv != 128)) {
         return COMBA_ERR_UNSUPPORTED;
     }

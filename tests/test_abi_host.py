@@ -75,7 +75,7 @@ def test_workspace_size_counts_chunks_and_heads(L):
 
 
 @pytest.mark.parametrize("kw", [dict(dk=96), dict(dv=192), dict(dv=256, dk=64), dict(dv=256, dtype=0), dict(dv=640),
-                                dict(dv=256, flags=8), dict(dv=256, flags=16), dict(chunk=32), dict(H=0), dict(B=0), dict(dtype=7),
+                                dict(chunk=32), dict(H=0), dict(B=0), dict(dtype=7),
                                 dict(B=2, N=3), dict(B=2, cu=FAKE, N=2), dict(T=-1), dict(cu=FAKE + 4, B=1, N=1)])
 def test_invalid_shapes_have_no_workspace(L, kw):
     assert ws(L, shape(**kw)) == 0
@@ -207,6 +207,9 @@ def test_value_head_groups(L):
     w128, w256, w512 = (ws(L, shape(dv=d), 1) for d in (128, 256, 512))
     assert 0 < w128 < w256 < w512
     assert ws(L, shape(dv=384), 0) > 0
+    # the gated and pk forms take value-head groups too
+    assert ws(L, shape(dv=256, flags=8), 1) > w256
+    assert ws(L, shape(dv=256, flags=16), 1) > w256
     assert ws(L, shape(dv=256, H=65535 // 2 + 1)) == 0   # value heads H * 2 beyond the head limit
 
     def step(dv, dk=128, dtype=1):

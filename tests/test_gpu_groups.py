@@ -102,3 +102,21 @@ def test_decode_dv256(dtype):
         torch.cuda.synchronize()
         assert rel(np64(o), ro) <= tol(dtype)
         assert rel(np64(st_gpu), st_ref) <= tol(dtype)
+
+
+def test_value_groups_gated():
+    """The gate and normalisation prologue with dv = 256: its q_hat, k_hat and gates serve both
+    value heads, and their gradients are summed over them before the epilogue."""
+    from test_gpu_gated import _check as gated_check, _run as gated_run
+    w = inputs.make_gated(B=2, T=150, H=2, dk=128, dv=256, dtype="bf16", seed_offset=256, lengths=[100, 0, 129])
+    gated_check(w, "splr", *gated_run(w, "splr"))
+
+
+def test_value_groups_pk():
+    """Comba-pk feedback vectors with dv = 256: dp is summed over the two value heads like dq and dk."""
+    from test_gpu_pk import _check as pk_check, _run as pk_run, _with_p
+    w = inputs.make("custom", B=2, T=170, H=2, dk=128, dv=256, dtype="bf16", with_b=True, with_h0=True,
+                    with_grads=True, seed_offset=77)
+    p, tp = _with_p(w, seed=256)
+    t = to_dev(w)
+    pk_check(w, p, *pk_run(w, t, tp))
