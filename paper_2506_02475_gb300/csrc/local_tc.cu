@@ -23,9 +23,14 @@
 // Operands live in 128-byte-swizzled shared tiles (K-major or MN-major as
 // each product needs; no transposed copies).  Outputs are staged in shared
 // memory and written with coalesced 16-byte stores.
+#include <cuda.h>
+
 #include "tc_tiles.cuh"
 
 namespace comba {
+
+bool make_bf16_token_map(CUtensorMap* m, const void* base, long long tokens, int heads, int cols);
+
 namespace tc {
 
 constexpr int kLocalThreads = 512;            // 16 warps: four per TMEM lane quadrant
@@ -132,6 +137,16 @@ __device__ __forceinline__ void frag_stage(uint8_t* st, int m0, int n0, const fl
                 __floats2bfloat162_rn(acc[t][2 * hh], acc[t][2 * hh + 1]);
         }
 }
+// Bulk tensor store of a [64][64-column] swizzled tile to (columns x, head y, tokens z ..).
+__device__ __forceinline__ void tma_store_rows(const void* tmap, int x, int y, int z, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];\n"
+                 ::"l"(tmap), "r"(x), "r"(y), "r"(z), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit_rows() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_rows_read() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_rows_done() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
+
 __device__ __forceinline__ void copy_stage_rows(bf16* g, long long ld, const uint8_t* st, int L, int tid) {
     for (int e = tid; e < L * 16; e += kLocalThreads) {
         const int r = e >> 4, ch = e & 15;
@@ -168,7 +183,9 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 // M after R7; Q and K into the second of two alternating tiles at the start of the unit; the
 // per-row scalars into registers), so the loads of consecutive units overlap the tensor-core
 // and epilogue work instead of every SM loading at the same moment.
-__global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p, long long units) {
+__global__ void __launch_bounds__(kLocalThreads, 1)
+    k_bwd_local_tc(ChunkParams p, long long units, const __grid_constant__ CUtensorMap tmDq,
+                   const __grid_constant__ CUtensorMap tmDk) {
     using S = LocalTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar;
@@ -292,6 +309,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         const long long t0 = cur.t0, idx = cur.idx;
 
         if (!pre) {
+            // a bulk store of dq, dk two units back may still read this tile
+            if (tid == 0) bulk_wait_rows_read();
+            __syncthreads();
             load_qk(sQK, cur);
             load_tok(sdO, p.dO, cur);
             load_E(cur);
@@ -329,6 +349,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
             for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
             *qa = pack8(qv);
         }
+        // the next unit's Q/K tile (loaded below, after R1's issue) may still be the source of the
+        // previous unit's bulk dq, dk stores
+        if (tid == 0) bulk_wait_rows_read();
         publish_smem();
 
         const float gL = sG[L - 1];
@@ -632,14 +655,33 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         }
         __syncthreads();   // every row dot has read the Q~/K tile
         if (ok) {
-            frag_stage<NK>(sQK, m0, nk0, acc_dq);
-            frag_stage<NK>(sQK + 16384, m0, nk0, acc_dk);
+            // a full chunk leaves by bulk tensor stores from swizzled tiles, which run behind the
+            // per-position tail; a partial one by row copies (a 64-row box would pass its end)
+            if (L == kChunk) {
+                frag_store_sw<NK>(sQK, 64, m0, nk0, acc_dq);
+                frag_store_sw<NK>(sQK + 16384, 64, m0, nk0, acc_dk);
+            } else {
+                frag_stage<NK>(sQK, m0, nk0, acc_dq);
+                frag_stage<NK>(sQK + 16384, m0, nk0, acc_dk);
+            }
         }
+        if (L == kChunk) fence_async_smem();
         __syncthreads();
         if (ok) {
-            const long long ld = (long long)p.H * D;
-            copy_stage_rows((bf16*)p.dq + (t0 * p.H + h) * D, ld, sQK, L, tid);
-            copy_stage_rows((bf16*)p.dkk + (t0 * p.H + h) * D, ld, sQK + 16384, L, tid);
+            if (L == kChunk) {
+                if (tid == 0) {
+#pragma unroll
+                    for (int half = 0; half < 2; ++half) {
+                        tma_store_rows(&tmDq, 64 * half, h, (int)t0, smem_u32(sQK) + half * 8192);
+                        tma_store_rows(&tmDk, 64 * half, h, (int)t0, smem_u32(sQK + 16384) + half * 8192);
+                    }
+                    bulk_commit_rows();
+                }
+            } else {
+                const long long ld = (long long)p.H * D;
+                copy_stage_rows((bf16*)p.dq + (t0 * p.H + h) * D, ld, sQK, L, tid);
+                copy_stage_rows((bf16*)p.dkk + (t0 * p.H + h) * D, ld, sQK + 16384, L, tid);
+            }
         }
 
         // ---------------- per-position scalars (rows 0..63, one thread each)
@@ -734,6 +776,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1) k_bwd_local_tc(ChunkParams p
         cur = nxt;
     }
     cp_async_wait<0>();   // no copy is still writing shared memory at exit
+    if (tid == 0) bulk_wait_rows_done();   // and no bulk store is still reading it
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -750,7 +793,11 @@ cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s) {
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     const long long units = (long long)p.slots * p.H;
     const int grid = (int)(units < nsm ? units : nsm);   // one resident CTA per SM
-    if (grid > 0) tc::k_bwd_local_tc<<<grid, tc::kLocalThreads, sm, s>>>(p, units);
+    CUtensorMap tq, tk;   // dq, dk [tokens][value heads][128]
+    if (!make_bf16_token_map(&tq, p.dq, p.Ttot, p.H, tc::D) ||
+        !make_bf16_token_map(&tk, p.dkk, p.Ttot, p.H, tc::D))
+        return cudaErrorInvalidValue;
+    if (grid > 0) tc::k_bwd_local_tc<<<grid, tc::kLocalThreads, sm, s>>>(p, units, tq, tk);
     return cudaGetLastError();
 }
 

@@ -567,6 +567,20 @@ bool make_bf16_map(CUtensorMap* m, const void* base, long long rows, int cols, i
     return make_map(m, base, rows, cols, box_rows);
 }
 
+// A [tokens][heads][cols] bf16 token tensor as a 3D view with a {64 columns, 1 head, 64 tokens}
+// box (one head's 64-token chunk, 128-byte rows, 128-byte swizzle).
+bool make_bf16_token_map(CUtensorMap* m, const void* base, long long tokens, int heads, int cols) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t gdim[3] = {(cuuint64_t)cols, (cuuint64_t)heads, (cuuint64_t)(tokens > 0 ? tokens : 1)};
+    cuuint64_t gstride[2] = {(cuuint64_t)cols * 2, (cuuint64_t)heads * cols * 2};
+    cuuint32_t box[3] = {64, 1, 64};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), gdim, gstride, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int DK, int DV, bool XMN>
 static cudaError_t run_scan_tc_split(const ScanArgs& a, long long pairs, cudaStream_t s) {
     using S = ScanSplitSmem<DK, DV>;
