@@ -112,14 +112,14 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 110_685, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "87c8dc1931f1d8d9"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0>", 85_123, ('scan.cu', 'common.cuh', 'params.cuh'), "a8e4b04b79c9cb5a"),
-    "output": ("k_output_tc", 118_597, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "87c8dc1931f1d8d9"),
-    "bwd_prep": ("k_bwd_prep_tc", 82_535, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "87c8dc1931f1d8d9"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_383, ('scan.cu', 'common.cuh', 'params.cuh'), "a8e4b04b79c9cb5a"),
-    "bwd_local": ("k_bwd_local_tc", 194_446, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "0768c8a76ce490a8"),
+    "prep": ("k_prep_tc", 110_874, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e70ceda23d6b45f6"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0>", 84_983, ('scan.cu', 'common.cuh', 'params.cuh'), "45bacb88f341bda6"),
+    "output": ("k_output_tc", 118_730, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e70ceda23d6b45f6"),
+    "bwd_prep": ("k_bwd_prep_tc", 82_503, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e70ceda23d6b45f6"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_324, ('scan.cu', 'common.cuh', 'params.cuh'), "45bacb88f341bda6"),
+    "bwd_local": ("k_bwd_local_tc", 194_212, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "1bd033503e34c0e0"),
 }
-DECODE_TRAFFIC = (481_318_912, ('decode.cu', 'common.cuh', 'params.cuh'), "5d94f1984c163f43")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (481_121_280, ('decode.cu', 'common.cuh', 'params.cuh'), "4d5d41608ec01898")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
