@@ -61,7 +61,9 @@ def fwd_flops_per_token_head(C=64, dk=128, dv=128):
 
 def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
     """`tc`: the tcgen05 path (bf16, d=128), whose reverse scan reads Atilde itself, so
-    the forward saves M but no Atilde^T.  `pk`: Comba-pk feedback vectors P, read by prep and
+    the forward saves M but no Atilde^T; its output kernel also forms and saves
+    Z^T = (Qhat - P W)^T, and its reverse scan forms the additive term C^T = dO^T Z from Z^T
+    and dO (no separate C-term kernel).  `pk`: Comba-pk feedback vectors P, read by prep and
     by the local gradients, which also write dP.  At dk = 256 no chunk map is formed: the
     scans read W, K and U (forward) or C^T (backward) and form two products per chunk.
     `H` counts value heads of width `dv`, `vg` of them per key head: tensors and products
@@ -93,6 +95,14 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
                        + P * (C * dv * es + dv * dk * es + C * dv * es * (2 if save else 1)))
     m["bwd_prep"] = dict(flops=Pk * 4 * C * C * dk + P * 2 * dv * C * dk,
                          bytes=Pk * (3 * C * dk * es + C * f4) + P * (C * dv * es + dv * dk * es))
+    if tc and not wide:
+        if save:   # Z^T = Qhat^T - W^T P^T, once per (chunk, key head)
+            m["output"]["flops"] += Pk * 2 * C * C * dk
+            m["output"]["bytes"] += Pk * dk * C * es
+        m["bwd_prep"] = dict(flops=0, bytes=0)
+        # reverse scan: Atilde and gamma, Z^T per key head; dO in and dH'^T out per value head
+        m["scan_bwd"] = dict(flops=P * (2 * dv * dk * dk + 2 * dv * C * dk),
+                             bytes=Pk * (dk * dk * es + f4 + dk * C * es) + P * (C * dv * es + dv * dk * es))
     m["bwd_local"] = dict(flops=Pk * 2 * C * C * dk * 2
                           + P * (2 * C * C * dk * 7 + 2 * C * dk * dv * 4 + 2 * C * C * dv * 4 + 4 * C ** 3),
                           bytes=Pk * (2 * C * dk * es + C * C * es + 3 * C * f4 + 2 * C * dk * es + 2 * C * f4)
@@ -107,17 +117,16 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per (chunk, head) unit
-# of each kernel of the bf16 d=128 path, from one ncu --set full capture of the
-# 340M-shape step (2048 units per launch), scaled to a launch by its unit count
+# of each kernel of the bf16 d=128 path, from one ncu capture of those two metrics on
+# the 340M-shape step (2048 units per launch), scaled to a launch by its unit count
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 110_874, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e70ceda23d6b45f6"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0>", 84_983, ('scan.cu', 'common.cuh', 'params.cuh'), "45bacb88f341bda6"),
-    "output": ("k_output_tc", 118_730, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e70ceda23d6b45f6"),
-    "bwd_prep": ("k_bwd_prep_tc", 82_503, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e70ceda23d6b45f6"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1>", 86_324, ('scan.cu', 'common.cuh', 'params.cuh'), "45bacb88f341bda6"),
-    "bwd_local": ("k_bwd_local_tc", 194_212, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "1bd033503e34c0e0"),
+    "prep": ("k_prep_tc", 110_806, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "52788c9a97b55452"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0,0>", 83_584, ('scan.cu', 'common.cuh', 'params.cuh'), "4362e0614f0a6aeb"),
+    "output": ("k_output_tc", 128_467, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "52788c9a97b55452"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 83_417, ('scan.cu', 'common.cuh', 'params.cuh'), "4362e0614f0a6aeb"),
+    "bwd_local": ("k_bwd_local_tc", 192_595, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "cd583d86216d3690"),
 }
 DECODE_TRAFFIC = (481_121_280, ('decode.cu', 'common.cuh', 'params.cuh'), "4d5d41608ec01898")   # whole Bd=256 H=16 launch
 
@@ -578,7 +587,10 @@ def run_ours(args, world, rank, local):
                     "all_outputs_read_back": {"value": tokens * world / (e_full_ms / 1e3), "ms_per_step": e_full_ms,
                                               "d2h_bytes_per_step": bo_full}},
             "clocks": clk,
-            "gpu_launches": 8 * args.steps,
+            # forward: chunk map, prep, scan, output; backward: (C term off the tcgen05 path), reverse
+            # scan, local gradients, per-head sums; plus q - d p per call with p, the key-head sums
+            # with value-head groups
+            "gpu_launches": (4 + (3 if tc else 4) + (2 if pk else 0) + (1 if vg > 1 else 0)) * args.steps,
             "stages_ms_per_step": {f"{p}.{s}": v / args.steps for (p, s), v in stage_ms.items()},
             "wall_s_timed": wall,
         }

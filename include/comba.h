@@ -104,7 +104,8 @@ typedef struct {
  * Saved factors (training step without recomputation).
  *   comba_chunk_fwd with COMBA_SAVE_FACTORS also keeps everything the
  *   backward needs (chunk table, W, U, log-decays, the UT inverses M, the
- *   chunk-start states H_n and E = U - W H_n) in its workspace, which must then
+ *   chunk-start states H_n, E = U - W H_n and, at dk = dv = 128 in bf16, the
+ *   factor Z = Qhat - P W of the reverse scan's additive term) in its workspace, which must then
  *   hold comba_workspace_size(shape, 1) bytes (else COMBA_ERR_WORKSPACE).
  *   comba_chunk_bwd with COMBA_REUSE_FACTORS reads them from the workspace
  *   instead of recomputing the forward chunk factors and states.  The

@@ -16,7 +16,7 @@ size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct Layout {
-    size_t err, slot_info, seq_first, W, U, G, A, B, Hs, E, M, AT, C, dH, part;
+    size_t err, slot_info, seq_first, W, U, G, A, B, Hs, E, M, AT, C, Z, dH, part;
     // gate and normalisation prologue (COMBA_GATED): its outputs, and the backward's gradients
     // w.r.t. them with the per-row contributions to da, dc
     size_t qh, kh, ga, gb, bg, dqh, dkh, dal, dbe, dbi, dar, dcr, dpa, dpc;
@@ -99,7 +99,11 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
         // Atilde^T is only materialised off the tcgen05 path (that reverse scan reads Atilde directly)
         if (has_chunk_map(s->dk) && !comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv))
             L.AT = take(pairs * dk * dk * es);
-        L.C = take(pairs * dv * dk * es);
+        // the tcgen05 path keeps Z^T (its reverse scan forms C itself); the others C^T
+        if (comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv / vg))
+            L.Z = take(pairs * dk * 64 * es);
+        else
+            L.C = take(pairs * dv * dk * es);
         L.dH = take(pairs * dv * dk * es);
         L.part = take(pairs * 2 * sizeof(float));
     }
@@ -183,7 +187,8 @@ void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* 
         p.Eb = w + L.E;
         p.Mb = w + L.M;
         p.ATb = L.AT ? w + L.AT : nullptr;
-        p.Cb = w + L.C;
+        p.Cb = L.C ? w + L.C : nullptr;
+        p.Zb = L.Z ? w + L.Z : nullptr;
         p.dHb = w + L.dH;
         p.part = reinterpret_cast<float*>(w + L.part);
     }

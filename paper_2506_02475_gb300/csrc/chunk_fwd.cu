@@ -418,7 +418,7 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
         return e;
     const bool tcp = use_tc_path(sizeof(T) == 2, DK, DV);
     ChunkParams q = p;
-    if (!save) { q.Mb = nullptr; q.ATb = nullptr; q.Eb = nullptr; }
+    if (!save) { q.Mb = nullptr; q.ATb = nullptr; q.Eb = nullptr; q.Zb = nullptr; }
     if (tcp) q.ATb = nullptr;   // the tcgen05 reverse scan reads Atilde directly
     mark(q, ev0, s);
     if (tcp) {

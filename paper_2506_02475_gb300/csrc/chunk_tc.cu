@@ -5,18 +5,19 @@
 // threads stage tiles with asynchronous copies and run the epilogues on the
 // rows they read back from TMEM (one row per thread).  Products are formed
 // transposed where that puts a 128-wide head dimension on M (W^T, U^T, E^T,
-// O^T, C^T); 64 x 64 chunk products pad M to 128 with zero rows.
+// O^T, (P W)^T); 64 x 64 chunk products pad M to 128 with zero rows.
 //
 //   k_prep_tc      Gram K K^T -> decay/btilde mask -> UT inverse M (fp32, blocked
 //                  forward substitution) -> W^T = K^T Mw^T, U^T = V^T Mu^T ->
 //                  Atilde = -K^T Diag(s) W, B^T = (Diag(s) U)^T K  (s = gamma_C/gamma_r);
 //                  with Comba-pk feedback vectors P: Gram P K^T and W^T = P^T Mw^T
 //   k_output_tc    P = Tril(Q~ K^T * Gamma), E^T = U^T - H^T W^T,
-//                  O^T = H^T Qhat^T + E^T P^T  (Qhat = Diag(gamma) Q~)
-//   k_bwd_prep_tc  C^T = dO^T (Qhat - P W)
+//                  O^T = H^T Qhat^T + E^T P^T  (Qhat = Diag(gamma) Q~); for the
+//                  backward also Z^T = Qhat^T - W^T P^T, the factor of the reverse
+//                  scan's additive term C = Z^T dO (formed by the scan itself)
 //
-// Workspace tensors of this path: W^T, U^T [pairs][128][64]; Atilde, B^T,
-// H^T, C^T, dH^T [pairs][128][128]; E [pairs][64][128] row-major; M [pairs][64][64].
+// Workspace tensors of this path: W^T, U^T, Z^T [pairs][128][64]; Atilde, B^T,
+// H^T, dH^T [pairs][128][128]; E [pairs][64][128] row-major; M [pairs][64][64].
 #include "tc_tiles.cuh"
 
 namespace comba {
@@ -253,9 +254,9 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
 struct OutTcSmem {
     static constexpr uint32_t OQK = 0;             // [128 rows][128]: rows 0-63 Q -> Q~ -> Qhat, rows 64-127 K;
                                                    // P [64][64] later over K's first half     32 KB
-    static constexpr uint32_t OW = 32768;          // W^T [128][64] (MN-major B), later E^T    16 KB
-    static constexpr uint32_t OU = OW + 16384;     // U^T [128][64], later E [64][128]         16 KB
-    static constexpr uint32_t OH = OU + 16384;     // H^T [128][128] K-major, later O staging  32 KB
+    static constexpr uint32_t OW = 32768;          // W^T [128][64] (MN-major B, then K-major A), later E [64][128]  16 KB
+    static constexpr uint32_t OU = OW + 16384;     // U^T [128][64], then E^T in place, later Z^T staging             16 KB
+    static constexpr uint32_t OH = OU + 16384;     // H^T [128][128] K-major, later O staging                        32 KB
     static constexpr uint32_t OG = OH + 32768;
     static constexpr size_t bytes() { return 1024 + OG + 64 * 4; }
 };
@@ -280,9 +281,10 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     uint8_t* sQK = sm + S::OQK;
     uint8_t* sP = sQK + 64 * 128;   // K's rows of the first 64-column half, dead after S = Q~ K^T
     uint8_t* sWt = sm + S::OW;
-    uint8_t* sEt = sWt;
     uint8_t* sUt = sm + S::OU;
-    bf16* sE = reinterpret_cast<bf16*>(sUt);   // [64][128] row-major staging of E
+    uint8_t* sEt = sUt;                        // E^T replaces U^T row by row
+    bf16* sE = reinterpret_cast<bf16*>(sWt);   // [64][128] row-major staging of E, once W^T is dead
+    uint8_t* stZ = sUt;                        // Z^T staging, once E^T is dead
     uint8_t* sHt = sm + S::OH;
     bf16* sO = reinterpret_cast<bf16*>(sHt);   // [64][136] staging of O
     float* sG = reinterpret_cast<float*>(sm + S::OG);
@@ -336,6 +338,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     }
     bool ok = ms.finish(tid);
     bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
+    bf16* Zg = p.Zb ? (bf16*)p.Zb + idx * D * 64 : nullptr;
     uint32_t ev[16];   // this thread's 32 positions of row j of E^T, packed bf16 pairs
     if (ok) {
         float d[32], v[8];
@@ -366,7 +369,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
                 unpack8(*reinterpret_cast<const uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)), u);
 #pragma unroll
                 for (int e = 0; e < 8; ++e) v[e] = u[e] - d[8 * q + e];
-                // sEt aliases sWt: every thread reads only its own row, and W^T is no longer needed
+                // in place: each thread reads and then overwrites only these 16 bytes of its own row
                 const uint4 pk = pack8(v);
                 *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * g + 8 * q, 128)) = pk;
                 const int b0 = 4 * q;
@@ -386,9 +389,19 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
         }
     }
     publish_smem();
+
+    // O^T = H^T Qhat^T + E^T P^T -> cols [128,192);  (P W)^T = W^T P^T -> cols [192,256)
+    const bool mma2 = p.o || Zg;
+    if (ok && tid == 0) {
+        if (p.o) {
+            tc_gemm<false, false>(tmem + 128, smem_u32(sHt), 128, smem_u32(sQK), 128, 64, D, false);
+            tc_gemm<false, false>(tmem + 128, smem_u32(sEt), 128, smem_u32(sP), 64, 64, 64, true);
+        }
+        if (Zg) tc_gemm<false, false>(tmem + 192, smem_u32(sWt), 128, smem_u32(sP), 64, 64, 64, false);
+    }
+    if (mma2) ok = ok && ms.finish(tid);
+    // W^T, E^T and H^T are dead: E, Z^T and O are staged over them.
     if (ok && Eg) {
-        // E [64][128] row-major over the dead U^T tile (every thread is past its U^T reads), then
-        // one 16 KB bulk copy to the workspace
 #pragma unroll
         for (int pp = 0; pp < 16; ++pp) {
             const __nv_bfloat162 two = *reinterpret_cast<const __nv_bfloat162*>(&ev[pp]);
@@ -397,194 +410,46 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
         }
         fence_async_smem();
     }
+    if (ok && Zg) {
+        // Z^T = Qhat^T - (P W)^T: row `row` (a key dimension), positions [32 half, +32); columns
+        // past a short chunk are zero because Qhat and P rows past it are
+        float d[32], v[8];
+        tmem_ld32(trow + 192 + half * 32, d);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int t = 32 * half + 8 * q + e;
+                const float qh = __bfloat162float(*reinterpret_cast<const bf16*>(sQK + sw128_offset(t, row, 128)));
+                v[e] = qh - d[8 * q + e];
+            }
+            stage_chunk<8>(stZ, row, 4 * half + q, pack8(v));
+        }
+    }
+    if (ok && p.o) {
+        float d[32];
+        tmem_ld32(trow + 128 + half * 32, d);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) sO[(32 * half + c) * 136 + row] = __float2bfloat16_rn(d[c]);
+    }
     __syncthreads();
     if (ok && Eg && tid == 0) bulk_copy_s2g(Eg, smem_u32(sE), 64 * D * 2);
-    if (!p.o) ok = false;   // E only (backward recompute): nothing more to do
-
-    // O^T = H^T Qhat^T + E^T P^T -> cols [128,192)
-    if (ok && tid == 0) {
-        tc_gemm<false, false>(tmem + 128, smem_u32(sHt), 128, smem_u32(sQK), 128, 64, D, false);
-        tc_gemm<false, false>(tmem + 128, smem_u32(sEt), 128, smem_u32(sP), 64, 64, 64, true);
-    }
-    if (p.o) {
-        ok = ok && ms.finish(tid);
-        if (ok) {
-            float d[32];
-            tmem_ld32(trow + 128 + half * 32, d);
-#pragma unroll
-            for (int c = 0; c < 32; ++c) sO[(32 * half + c) * 136 + row] = __float2bfloat16_rn(d[c]);
-        }
-        __syncthreads();
-        if (ok) {
-            bf16* Og = (bf16*)p.o + (t0 * p.H + h) * D;
-            for (int e = tid; e < L * 16; e += NTH) {
-                const int r = e >> 4, ch = e & 15;
-                *reinterpret_cast<uint4*>(Og + (long long)r * p.H * D + 8 * ch) =
-                    *reinterpret_cast<const uint4*>(sO + r * 136 + 8 * ch);
-            }
-        } else if (tid == 0) {
-            flag_error(p);
-        }
-    }
-    if (Eg && tid == 0) bulk_wait_all_reads();   // the E copy has read its staging before exit
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (warp == 0) tmem_dealloc(tmem, 256);
-}
-
-// ------------------------------------------------- reverse-scan additive term
-
-struct BPrepTcSmem {
-    static constexpr uint32_t OQ = 0;              // Q -> Q~ -> Qhat [128 alloc rows][128]   32 KB
-    static constexpr uint32_t OK = 32768;          // K [64][128], later P [128 alloc][64]    16 KB
-    static constexpr uint32_t OW = OK + 16384;     // W^T [128][64] (K-major B), later Z      16 KB
-    static constexpr uint32_t OD = OW + 16384;     // dO [64][128] (MN-major A)               16 KB
-    static constexpr uint32_t OG = OD + 16384;
-    static constexpr size_t bytes() { return 1024 + OG + 64 * 4; }
-};
-
-// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
-__global__ void __launch_bounds__(256) k_bwd_prep_tc(ChunkParams p) {
-    constexpr int NTH = 256;
-    using S = BPrepTcSmem;
-    extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar;
-    __shared__ uint32_t tbase;
-    const int slot = blockIdx.x, h = blockIdx.y;
-    const SlotInfo si = p.slot_info[slot];
-    if (si.len <= 0) return;
-    const int L = si.len;
-    const long long t0 = si.start;
-    const long long idx = (long long)slot * p.H + h;
-    const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
-    const int tid = threadIdx.x, warp = tid >> 5;
-    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sQ = sm + S::OQ;
-    uint8_t* sK = sm + S::OK;
-    uint8_t* sP = sK;
-    uint8_t* sWt = sm + S::OW;
-    uint8_t* sZ = sWt;
-    uint8_t* sdO = sm + S::OD;
-    float* sG = reinterpret_cast<float*>(sm + S::OG);
-
-    load_sw(sQ, 128, D, (const bf16*)p.q + (t0 * Hk + hk) * D, (long long)Hk * D, L, tid, NTH);
-    load_sw(sK, 64, D, (const bf16*)p.k + (t0 * Hk + hk) * D, (long long)Hk * D, L, tid, NTH);
-    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid, NTH);
-    load_sw(sdO, 64, D, (const bf16*)p.dO + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
-    cp_async_commit();
-    if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
-    if (tid == 0) {
-        mbar_init(smem_u32(&bar), 1);
-        mbar_fence_init();
-    }
-    if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
-    cp_async_wait<0>();
-    __syncthreads();
-    const float dh = p.d[hk];
-    for (int e = tid; e < 64 * 16; e += NTH) {
-        const int r = e >> 4, ch = e & 15;
-        uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
-        const uint4 ka = *reinterpret_cast<const uint4*>(sK + sw128_offset(r, 8 * ch, 64));
-        float qv[8], kv[8];
-        unpack8(*qa, qv);
-        unpack8(ka, kv);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
-        *qa = pack8(qv);
-    }
-    publish_smem();
-    const uint32_t tmem = tbase;
-    MmaSync ms{smem_u32(&bar), 0};
-    const int row = tid & 127, half = tid >> 7;   // TMEM lane, and which half of the columns
-    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-
-    if (tid == 0) tc_gemm<false, false>(tmem, smem_u32(sQ), 128, smem_u32(sK), 64, 64, D, false);   // Q~ K^T
-    bool ok = ms.finish(tid);
-    if (ok) {
-        // P [128 alloc rows][64] K-major A operand (rows >= 64 zero); Qhat = Diag(gamma) Q~ in place.
-        float d[32], v[8];
-        const float gr = row < 64 ? sG[row] : 0.f;
-        {
-            const int g = half;
-            tmem_ld32(trow + g * 32, d);
-            if (row < 64) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const int i = 32 * g + 8 * q + e;
-                        v[e] = (i <= row && row < L) ? d[8 * q + e] * __expf(gr - sG[i]) : 0.f;
-                    }
-                    *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
-                }
-            } else {
-#pragma unroll
-                for (int q = 0; q < 4; ++q)
-                    *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 128)) = make_uint4(0, 0, 0, 0);
-            }
-        }
-        for (int e = tid; e < 64 * 16; e += NTH) {
+    if (ok && Zg) copy_staged<8>(Zg, stZ, tid, NTH);
+    if (ok && p.o) {
+        bf16* Og = (bf16*)p.o + (t0 * p.H + h) * D;
+        for (int e = tid; e < L * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15;
-            uint4* qa = reinterpret_cast<uint4*>(sQ + sw128_offset(r, 8 * ch, 128));
-            float qv[8];
-            unpack8(*qa, qv);
-            const float gr = __expf(sG[r]);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) qv[i] *= gr;
-            *qa = pack8(qv);
+            *reinterpret_cast<uint4*>(Og + (long long)r * p.H * D + 8 * ch) =
+                *reinterpret_cast<const uint4*>(sO + r * 136 + 8 * ch);
         }
     }
-    publish_smem();
-    // P W -> cols [64,192)  (B = W via W^T [c][i], K-major)
-    if (ok && tid == 0) tc_gemm<false, false>(tmem + 64, smem_u32(sP), 128, smem_u32(sWt), 128, 128, 64, false);
-    ok = ok && ms.finish(tid);
-    if (ok && row < 64) {
-        // Z = Qhat - P W, written as an MN-major [64 k-rows][128] tile (B operand of dO^T Z)
-        float d[32], v[8];
-#pragma unroll
-        for (int g = 2 * half; g < 2 * half + 2; ++g) {
-            tmem_ld32(trow + 64 + g * 32, d);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                float qh[8];
-                unpack8(*reinterpret_cast<const uint4*>(sQ + sw128_offset(row, 32 * g + 8 * q, 128)), qh);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) v[e] = qh[e] - d[8 * q + e];
-                *reinterpret_cast<uint4*>(sZ + mn128_offset(32 * g + 8 * q, row, 64)) = pack8(v);
-            }
-        }
-    } else if (ok) {
-        float d[32];
-#pragma unroll
-        for (int g = 2 * half; g < 2 * half + 2; ++g) tmem_ld32(trow + 64 + g * 32, d);   // keep the warp-collective loads aligned
-    }
-    publish_smem();
-    // C^T = dO^T Z -> cols [0,128)
-    if (ok && tid == 0) tc_gemm<true, true>(tmem, smem_u32(sdO), 64, smem_u32(sZ), 64, 128, 64, false);
-    ok = ok && ms.finish(tid);
-    if (ok) {
-        // C^T staged over the dead Qhat tile, then copied out coalesced
-        float d[32];
-#pragma unroll
-        for (int g = 2 * half; g < 2 * half + 2; ++g) {
-            tmem_ld32(trow + g * 32, d);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) stage_chunk<16>(sQ, row, 4 * g + q, pack8(d + 8 * q));
-        }
-    }
-    __syncthreads();
-    if (ok) {
-        copy_staged<16>((bf16*)p.Cb + idx * D * D, sQ, tid, NTH);
-    } else if (tid == 0) {
-        flag_error(p);
-    }
+    if (!ok && tid == 0) flag_error(p);
+    if (ok && Eg && tid == 0) bulk_wait_all_reads();   // the E copy has read its staging before exit
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, 256);
 }
-
 
 }  // namespace tc
 
@@ -606,16 +471,6 @@ cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_bwd_prep_tc(const ChunkParams& p, cudaStream_t s) {
-    const size_t sm = tc::BPrepTcSmem::bytes();
-    cudaError_t e = cudaFuncSetAttribute(tc::k_bwd_prep_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-    if (e) return e;
-    if (p.slots > 0) tc::k_bwd_prep_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p);
-    return cudaGetLastError();
-}
-
-size_t tc_smem_bytes(int kernel) {
-    return kernel == 0 ? tc::PrepTcSmem::bytes() : (kernel == 1 ? tc::OutTcSmem::bytes() : tc::BPrepTcSmem::bytes());
-}
+size_t tc_smem_bytes(int kernel) { return kernel == 0 ? tc::PrepTcSmem::bytes() : tc::OutTcSmem::bytes(); }
 
 }  // namespace comba

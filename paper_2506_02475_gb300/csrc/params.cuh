@@ -59,7 +59,10 @@ struct ChunkParams {
     void* Eb;                // [pairs][64][dv]  E = U - W H (saved for the backward)
     void* Mb;                // [pairs][64][64]  UT inverse M (saved for the backward)
     void* ATb;               // [pairs][dk][dk]  Atilde^T (backward scan operand)
-    void* Cb;                // [pairs][dv][dk]  ((Qhat - P W)^T dO)^T (backward scan additive term)
+    void* Cb;                // [pairs][dv][dk]  ((Qhat - P W)^T dO)^T (backward scan additive term;
+                             //                  off the tcgen05 path)
+    void* Zb;                // [pairs][dk][64]  Z^T = (Qhat - P W)^T (tcgen05 path: the reverse scan
+                             //                  forms Z^T dO itself)
     void* dHb;               // [pairs][dv][dk]  dL/dH at chunk end, transposed
     float* part;             // [pairs][2]       per-chunk db, dd partial sums
     int* err;                // device status word (nonzero: a bounded wait gave up)
@@ -136,6 +139,11 @@ struct ScanArgs {
     int x_mn;                // X is read as an MN-major operand ([k][m] row-major, no transpose)
     int vg;                  // value heads per key head: init/fin are [N, H / vg, dk, vg * dv]
     int* err;
+    // Reverse scan on the tcgen05 path (zc = 1): the additive term of each chunk is formed in the
+    // scan as (dO^T Z)^T from Z^T [pairs][dk][64] and dO [tokens, H, dv] instead of read from Y.
+    int zc = 0;
+    const void* Z = nullptr;
+    const void* dO = nullptr;
 };
 cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s);
 size_t scan_smem_bytes(bool is_bf16, int dk, int dv);
@@ -158,7 +166,6 @@ size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false,
 // tcgen05 kernels of the bf16 dk = dv = 128 path (chunk_tc.cu)
 cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s);
 cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s);
-cudaError_t launch_bwd_prep_tc(const ChunkParams& p, cudaStream_t s);
 size_t tc_smem_bytes(int kernel);
 // tcgen05 local-gradient kernel of the same path (local_tc.cu)
 cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s);

@@ -11,7 +11,10 @@
 // with X = Atilde (forward; row-major [dk][dk], read K-major) or, in the
 // backward, Atilde read as an MN-major operand (bf16 path) or Atilde^T
 // (fp32 path); Y = B^T or C^T stored [dv][dk].  Each chunk stores the state it started
-// from (H_n^T, or dH_{n+1}^T in the backward) for the parallel kernels.
+// from (H_n^T, or dH_{n+1}^T in the backward) for the parallel kernels.  The
+// tcgen05 path's reverse scan reads no C^T: it forms C^T = dO^T Z itself from
+// the Z^T the forward's output kernel saved, one product per chunk issued ahead
+// of the sequential one (see k_scan_tc_split).
 //
 // bf16 storage: one CTA per (sequence, head), 256 threads (two per state row,
 // each holding half of the row's dk columns); the fp32 state stays in registers.
@@ -257,26 +260,37 @@ __global__ void __launch_bounds__(256, 1)
 // stores half of the chunk state, and the epilogue is half as long.  X and Y each
 // stream three chunks deep; one thread issues the MMAs while another issues the TMA
 // stores and loads, so a step's critical path is the MMA, not the issue sequence.
-template <int DK, int DV>
+// ZC (reverse scan of the tcgen05 path): the additive term C^T = dO^T Z is formed here.  Its
+// operands stream in four chunks deep in place of Y: Z^T [dk][64 positions] (K-major B) and this
+// CTA's 64 columns of dO [64 positions][64] (MN-major A).  Each chunk's C product is issued right
+// after the previous chunk's state product, into the other of two TMEM accumulators, so it runs
+// while that chunk's epilogue does; the state product then accumulates onto it.
+template <int DK, int DV, bool ZC>
 struct ScanSplitSmem {
-    static constexpr int SX = 3, SY = 3;
+    static constexpr int SX = 3, SY = 3, SZ = 4;
     static constexpr uint32_t A_BYTES = 64 * DK * 2;    // this CTA's 64 rows of S^T; two buffers
     static constexpr uint32_t X_BYTES = DK * DK * 2;
     static constexpr uint32_t Y_BYTES = 64 * DK * 2;
+    static constexpr uint32_t ZT_BYTES = DK * 64 * 2;   // ZC: Z^T
+    static constexpr uint32_t DO_BYTES = 64 * 64 * 2;   // ZC: this CTA's dO columns
     static constexpr uint32_t OX = 2 * A_BYTES;
     static constexpr uint32_t OY = OX + SX * X_BYTES;
-    static constexpr size_t bytes() { return 1024 + OY + (size_t)SY * Y_BYTES; }
+    static constexpr uint32_t OZ = OY;                  // ZC: Z^T stages, then dO stages
+    static constexpr uint32_t OD = OZ + SZ * ZT_BYTES;
+    static constexpr int NY = ZC ? SZ : SY;             // stages behind the full_y barriers
+    static constexpr size_t bytes() { return 1024 + (ZC ? OD + (size_t)SZ * DO_BYTES : OY + (size_t)SY * Y_BYTES); }
 };
 
-template <int DK, int DV, bool XMN>
+template <int DK, int DV, bool XMN, bool ZC>
 __global__ void __launch_bounds__(256, 1)
     k_scan_tc_split(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY,
-                    const __grid_constant__ CUtensorMap tmS) {
+                    const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmO) {
     static_assert(DK == 128 && DV == 128, "row split is laid out for dk = dv = 128");
-    using S = ScanSplitSmem<DK, DV>;
+    using S = ScanSplitSmem<DK, DV, ZC>;
     constexpr int NT = DK / 16;   // 8-column tiles per thread (half of the columns)
+    constexpr uint32_t TCOLS = ZC ? 2 * DK : DK;   // ZC: two accumulators, chunk it in (it & 1)
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t full_x[S::SX], full_y[S::SY];
+    __shared__ uint64_t full_x[S::SX], full_y[S::NY];
     __shared__ uint64_t mma_bar;
     __shared__ uint32_t tmem_base;
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -307,16 +321,17 @@ __global__ void __launch_bounds__(256, 1)
 
     if (tid == 0) {
         for (int s = 0; s < S::SX; ++s) mbar_init(smem_u32(&full_x[s]), 1);
-        for (int s = 0; s < S::SY; ++s) mbar_init(smem_u32(&full_y[s]), 1);
+        for (int s = 0; s < S::NY; ++s) mbar_init(smem_u32(&full_y[s]), 1);
         mbar_init(smem_u32(&mma_bar), 1);
         mbar_fence_init();
     }
-    if (warp == 0) tmem_alloc(smem_u32(&tmem_base), DK);
+    if (warp == 0) tmem_alloc(smem_u32(&tmem_base), TCOLS);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base;
     const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16) + 64 * wc;
+    auto acc_col = [&](int it) { return ZC ? (uint32_t)(it & 1) * DK : 0u; };
 
     auto chunk_of = [&](int it) { return a.reverse ? nch - 1 - it : it; };
     auto unit_of = [&](int it) { return (long long)(s0 + chunk_of(it)) * a.H + h; };
@@ -337,16 +352,64 @@ __global__ void __launch_bounds__(256, 1)
         for (int half = 0; half < DK / 64; ++half)
             tma_load_2d(smem_u + y_off(it) + half * 64 * 128, &tmY, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), fb);
     };
+    auto zt_buf = [&](int it) { return smem_u + S::OZ + (uint32_t)(it % S::SZ) * S::ZT_BYTES; };
+    auto do_buf = [&](int it) { return smem_u + S::OD + (uint32_t)(it % S::SZ) * S::DO_BYTES; };
+    auto issue_zd = [&](int it) {   // ZC: Z^T of the chunk, and its dO rows x this CTA's 64 columns
+        const uint32_t fb = smem_u32(&full_y[it % S::SZ]);
+        mbar_expect_tx(fb, S::ZT_BYTES + S::DO_BYTES);
+        tma_load_2d(zt_buf(it), &tmY, 0, (int)(unit_of(it) * DK), fb);
+        tma_load_3d(do_buf(it), &tmO, 64 * rhalf, h, (int)(start + (long long)chunk_of(it) * kChunk), fb);
+    };
     // Thread 0 issues the MMAs; thread 32 (warp 1) the TMA traffic: the chunk-state stores, the
     // X / Y loads and the bulk-group waits, so neither waits for the other's issue sequence.
     constexpr int kTma = 32;
     int nx = 0, ny = 0;
     if (tid == kTma) {
         for (; nx < S::SX - 1 && nx < nch; ++nx) issue_x(nx);
-        for (; ny < S::SY - 1 && ny < nch; ++ny) issue_y(ny);
+        if constexpr (ZC) {
+            for (; ny < S::SZ - 1 && ny < nch; ++ny) issue_zd(ny);
+        } else {
+            for (; ny < S::SY - 1 && ny < nch; ++ny) issue_y(ny);
+        }
     }
 
     constexpr uint32_t idesc = idesc_bf16_f32(64, DK) | (XMN ? 1u << 16 : 0u);
+    // ZC: C^T rows = dO^T (A: MN-major, M = this CTA's 64 dv columns) x Z (B: Z^T K-major), K = 64
+    constexpr uint32_t idesc_c = idesc_bf16_f32(64, DK) | (1u << 15);
+    auto issue_c = [&](int it) {
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks)
+            tc_mma_bf16(tmem + acc_col(it), desc_mnmajor(do_buf(it), 64, ks), desc_kmajor(zt_buf(it), DK, ks),
+                        idesc_c, ks > 0 ? 1u : 0u);
+    };
+    int cbad = 0;   // thread 0: a C product's operands never arrived
+    if constexpr (ZC) {
+        if (nch > 0) {
+            // The first chunk of the reverse scan is a sequence's last and may be short.  Its dO rows
+            // past the sequence end belong to the next sequence (or lie past the tensor): zero them,
+            // so that only this sequence's positions enter the product (its Z^T columns there are
+            // zero, but a non-finite dO elsewhere must not leak in).
+            const long long rem = len - (long long)chunk_of(0) * kChunk;
+            const int L0 = (int)(rem < kChunk ? rem : kChunk);
+            bool ok0 = true;
+            if (L0 < kChunk) {
+                ok0 = mbar_wait(smem_u32(&full_y[0]), 0);
+                if (ok0)
+                    for (int e = tid; e < (kChunk - L0) * 8; e += 256)
+                        *reinterpret_cast<uint4*>(smem + S::OD + (L0 + (e >> 3)) * 128 + (e & 7) * 16) =
+                            make_uint4(0, 0, 0, 0);
+                fence_async_smem();
+                __syncthreads();
+                tc_fence_after();
+            }
+            if (tid == 0) {
+                if (ok0 && mbar_wait(smem_u32(&full_y[0]), 0))
+                    issue_c(0);
+                else
+                    cbad = 1;
+            }
+        }
+    }
     auto log_decay = [&](int it) {
         const int c = chunk_of(it);
         const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
@@ -370,37 +433,57 @@ __global__ void __launch_bounds__(256, 1)
         __syncthreads();
         tc_fence_after();
 
-        int bad = 0;
+        int bad = cbad;
         if (tid == 0) {
-            if (mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
+            if (!cbad && mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
 #pragma unroll
                 for (int ks = 0; ks < DK / 16; ++ks) {
                     const int half = ks >> 2, sub = ks & 3;
                     const uint64_t ad = smem_desc_sw128(a_buf(it) + half * 64 * 128 + sub * 32);
                     const uint64_t bd = XMN ? desc_mnmajor(x_buf(it), DK, ks)
                                             : smem_desc_sw128(x_buf(it) + half * DK * 128 + sub * 32);
-                    tc_mma_bf16(tmem, ad, bd, idesc, ks > 0 ? 1u : 0u);
+                    tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc, (ZC || ks > 0) ? 1u : 0u);
                 }
             } else {
                 bad = 1;
             }
             tc_commit(smem_u32(&mma_bar));
+            if constexpr (ZC) {
+                // the next chunk's C product, into the other accumulator (read back two chunks ago)
+                if (!bad && it + 1 < nch) {
+                    if (mbar_wait(smem_u32(&full_y[(it + 1) % S::SZ]), ((it + 1) / S::SZ) & 1))
+                        issue_c(it + 1);
+                    else
+                        bad = cbad = 1;
+                }
+            }
         } else if (tid == kTma) {
 #pragma unroll
             for (int half = 0; half < DK / 64; ++half)
                 tma_store_2d(&tmS, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), a_buf(it) + half * 64 * 128);
             bulk_commit();
             if (nx < nch) issue_x(nx++);
-            if (ny < nch) issue_y(ny++);
+            if constexpr (ZC) {
+                // its stage last held chunk it - 1, whose C product the commit of chunk it - 1 covered
+                if (ny < nch) issue_zd(ny++);
+            } else {
+                if (ny < nch) issue_y(ny++);
+            }
         }
         if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
-        if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1)) bad = 1;
+        if constexpr (!ZC)
+            if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1)) bad = 1;
         if (tid == kTma) bulk_wait_read<1>();
         if (__syncthreads_or(bad)) {
             if (tid == kTma) {
                 if (a.err) atomicExch(a.err, 1);
                 for (int c = it; c < nx; ++c) mbar_wait(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
-                for (int c = it; c < ny; ++c) mbar_wait(smem_u32(&full_y[c % S::SY]), (c / S::SY) & 1);
+                for (int c = it; c < ny; ++c) mbar_wait(smem_u32(&full_y[c % S::NY]), (c / S::NY) & 1);
+            }
+            if (ZC && tid == 0) {
+                // a C product issued after the last commit must finish before TMEM is released
+                tc_commit(smem_u32(&mma_bar));
+                mbar_wait(smem_u32(&mma_bar), (it + 1) & 1);
             }
             break;
         }
@@ -415,22 +498,29 @@ __global__ void __launch_bounds__(256, 1)
               "=r"(d[8]), "=r"(d[9]), "=r"(d[10]), "=r"(d[11]), "=r"(d[12]), "=r"(d[13]), "=r"(d[14]), "=r"(d[15]),
               "=r"(d[16]), "=r"(d[17]), "=r"(d[18]), "=r"(d[19]), "=r"(d[20]), "=r"(d[21]), "=r"(d[22]), "=r"(d[23]),
               "=r"(d[24]), "=r"(d[25]), "=r"(d[26]), "=r"(d[27]), "=r"(d[28]), "=r"(d[29]), "=r"(d[30]), "=r"(d[31])
-            : "r"(tq));
-        const uint8_t* sY = smem + y_off(it);
+            : "r"(tq + acc_col(it)));
         __nv_bfloat162 yv[NT][2];
+        if constexpr (!ZC) {
+            const uint8_t* sY = smem + y_off(it);
 #pragma unroll
-        for (int t = 0; t < NT; ++t)
+            for (int t = 0; t < NT; ++t)
 #pragma unroll
-            for (int hh = 0; hh < 2; ++hh)
-                yv[t][hh] = *reinterpret_cast<const __nv_bfloat162*>(sY + sw128_offset(r0 + 8 * hh, cq + 8 * t, 64));
+                for (int hh = 0; hh < 2; ++hh)
+                    yv[t][hh] = *reinterpret_cast<const __nv_bfloat162*>(sY + sw128_offset(r0 + 8 * hh, cq + 8 * t, 64));
+        }
         tmem_wait_ld();
 #pragma unroll
         for (int t = 0; t < NT; ++t)
 #pragma unroll
             for (int hh = 0; hh < 2; ++hh) {
-                const float2 yf = __bfloat1622float2(yv[t][hh]);
-                st[t][2 * hh] = fmaf(gam, st[t][2 * hh], __uint_as_float(d[4 * t + 2 * hh]) + yf.x);
-                st[t][2 * hh + 1] = fmaf(gam, st[t][2 * hh + 1], __uint_as_float(d[4 * t + 2 * hh + 1]) + yf.y);
+                if constexpr (ZC) {   // the accumulator already holds C
+                    st[t][2 * hh] = fmaf(gam, st[t][2 * hh], __uint_as_float(d[4 * t + 2 * hh]));
+                    st[t][2 * hh + 1] = fmaf(gam, st[t][2 * hh + 1], __uint_as_float(d[4 * t + 2 * hh + 1]));
+                } else {
+                    const float2 yf = __bfloat1622float2(yv[t][hh]);
+                    st[t][2 * hh] = fmaf(gam, st[t][2 * hh], __uint_as_float(d[4 * t + 2 * hh]) + yf.x);
+                    st[t][2 * hh + 1] = fmaf(gam, st[t][2 * hh + 1], __uint_as_float(d[4 * t + 2 * hh + 1]) + yf.y);
+                }
             }
         tc_fence_before();
     }
@@ -438,7 +528,7 @@ __global__ void __launch_bounds__(256, 1)
     if (tid == kTma) bulk_wait_all();
     __syncthreads();
     tc_fence_after();
-    if (warp == 0) tmem_dealloc(tmem, DK);
+    if (warp == 0) tmem_dealloc(tmem, TCOLS);
     if (a.fin) {
         float* fin = a.fin + state_off(a, n, h, DK, DV);
 #pragma unroll
@@ -581,23 +671,36 @@ bool make_bf16_token_map(CUtensorMap* m, const void* base, long long tokens, int
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int DK, int DV, bool XMN>
+template <int DK, int DV, bool XMN, bool ZC>
 static cudaError_t run_scan_tc_split(const ScanArgs& a, long long pairs, cudaStream_t s) {
-    using S = ScanSplitSmem<DK, DV>;
-    CUtensorMap tx, ty, ts;
-    if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, 64) ||
-        !make_map(&ts, a.Sout, pairs * DV, DK, 64))
+    using S = ScanSplitSmem<DK, DV, ZC>;
+    CUtensorMap tx, ty, ts, to;
+    if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ts, a.Sout, pairs * DV, DK, 64))
         return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(k_scan_tc_split<DK, DV, XMN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)S::bytes());
+    if (ZC) {
+        // Z^T [pairs * dk][64] with a [dk][64] box; dO [tokens][heads][dv] with a {64, 1, 64} box
+        if (!a.Z || !a.dO || !make_map(&ty, a.Z, pairs * DK, 64, DK) || !make_bf16_token_map(&to, a.dO, a.Ttot, a.H, DV))
+            return cudaErrorInvalidValue;
+    } else {
+        if (!make_map(&ty, a.Y, pairs * DV, DK, 64)) return cudaErrorInvalidValue;
+        to = ty;   // not read
+    }
+    cudaError_t e = cudaFuncSetAttribute(k_scan_tc_split<DK, DV, XMN, ZC>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)S::bytes());
     if (e) return e;
-    k_scan_tc_split<DK, DV, XMN><<<dim3(2 * a.N, a.H), 256, S::bytes(), s>>>(a, tx, ty, ts);
+    k_scan_tc_split<DK, DV, XMN, ZC><<<dim3(2 * a.N, a.H), 256, S::bytes(), s>>>(a, tx, ty, ts, to);
     return cudaGetLastError();
 }
 
 template <int DK, int DV, bool XMN>
 static cudaError_t run_scan_tc(const ScanArgs& a, long long pairs, cudaStream_t s) {
-    if constexpr (DK == 128 && DV == 128) return run_scan_tc_split<DK, DV, XMN>(a, pairs, s);
+    if constexpr (DK == 128 && DV == 128) {
+        if constexpr (XMN) {
+            if (a.zc) return run_scan_tc_split<DK, DV, true, true>(a, pairs, s);
+        }
+        return run_scan_tc_split<DK, DV, XMN, false>(a, pairs, s);
+    }
+    if (a.zc) return cudaErrorInvalidValue;
     using S = ScanTcSmem<DK, DV>;
     CUtensorMap tx, ty, ts;
     if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, DV) ||
@@ -634,7 +737,8 @@ cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long lo
 size_t scan_smem_bytes(bool is_bf16, int dk, int dv) {
     if (dk == 256) return is_bf16 && dv == 64 ? scan_wide_smem_bytes() : 0;
     if (is_bf16) {
-        if (dk == 128) return dv == 128 ? ScanSplitSmem<128, 128>::bytes() : ScanTcSmem<128, 64>::bytes();
+        if (dk == 128)   // the reverse (ZC) variant is the larger
+            return dv == 128 ? ScanSplitSmem<128, 128, true>::bytes() : ScanTcSmem<128, 64>::bytes();
         return dv == 128 ? ScanTcSmem<64, 128>::bytes() : ScanTcSmem<64, 64>::bytes();
     }
     return dk == 128 ? ScanSimtSmem<128>::bytes() : ScanSimtSmem<64>::bytes();

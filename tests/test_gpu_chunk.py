@@ -110,6 +110,31 @@ def test_varlen_small_with_empty_and_ragged_sequences(dtype, d):
     check_bwd(w, t)
 
 
+def test_nonfinite_dO_stays_inside_its_packed_sequence():
+    """Packed sequences [100, 70, 129] with dO = +inf on every token of the middle one: the
+    other sequences' token gradients and dh0 stay finite and match the oracle.  Their short
+    last chunks cover the next sequence's (or no) tokens, so every kernel that reads a chunk
+    tile, the reverse scan's dO tile included, must mask the rows past the sequence end."""
+    lens = [100, 70, 129]
+    w = inputs.make("custom", H=2, dk=128, dv=128, dtype="bf16", with_b=True, with_h0=True, with_grads=True,
+                    lengths=lens, seed_offset=41)
+    cu = w.cu_seqlens
+    mid = slice(int(cu[1]), int(cu[2]))
+    keep = np.ones(int(cu[-1]), bool)
+    keep[mid] = False
+    dO_ref = w.dO.copy()
+    dO_ref[mid] = 0.0
+    w.dO[mid] = np.inf
+    g = gpu_bwd(to_dev(w))
+    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, dO_ref, h0=w.h0, dhT=w.dhT, cu_seqlens=cu)
+    for key in ("dq", "dk", "dv", "dalpha", "dbeta"):
+        x, ref = g[key][keep], r[key][keep]
+        assert np.all(np.isfinite(x)), key
+        assert rel(x, ref) <= tol(w.dtype), key
+    x, ref = g["dh0"][[0, 2]], r["dh0"][[0, 2]]
+    assert np.all(np.isfinite(x)) and rel(x, ref) <= tol(w.dtype)
+
+
 def test_backward_is_bitwise_deterministic():
     w = inputs.make("custom", B=2, T=260, H=2, dk=128, dv=128, dtype="bf16", with_b=True, with_h0=True,
                     with_grads=True, seed_offset=5)
