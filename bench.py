@@ -61,9 +61,9 @@ def fwd_flops_per_token_head(C=64, dk=128, dv=128):
 
 def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
     """`tc`: the tcgen05 path (bf16, d=128), whose reverse scan reads Atilde itself, so
-    the forward saves M but no Atilde^T; its output kernel also forms and saves
-    Z^T = (Qhat - P W)^T, and its reverse scan forms the additive term C^T = dO^T Z from Z^T
-    and dO (no separate C-term kernel).  `pk`: Comba-pk feedback vectors P, read by prep and
+    the forward saves M but no Atilde^T; its scans form their additive terms themselves:
+    B^T = U_s^T K from the U_s^T = (Diag(s) U)^T that prep writes in place of B^T, and
+    C^T = dO^T Z from the Z^T that the output kernel saves (no separate C-term kernel).  `pk`: Comba-pk feedback vectors P, read by prep and
     by the local gradients, which also write dP.  At dk = 256 no chunk map is formed: the
     scans read W, K and U (forward) or C^T (backward) and form two products per chunk.
     `H` counts value heads of width `dv`, `vg` of them per key head: tensors and products
@@ -96,6 +96,12 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
     m["bwd_prep"] = dict(flops=Pk * 4 * C * C * dk + P * 2 * dv * C * dk,
                          bytes=Pk * (3 * C * dk * es + C * f4) + P * (C * dv * es + dv * dk * es))
     if tc and not wide:
+        # prep writes U_s^T = (Diag(s) U)^T instead of forming B^T; the forward scan forms
+        # B^T = U_s^T K from it and the keys
+        m["prep"]["flops"] -= P * 2 * dv * C * dk
+        m["prep"]["bytes"] += P * (C * dv * es - dv * dk * es)
+        m["scan_fwd"] = dict(flops=P * (2 * dv * dk * dk + 2 * dv * C * dk),
+                             bytes=Pk * (dk * dk * es + f4 + C * dk * es) + P * (dv * C * es + dv * dk * es))
         if save:   # Z^T = Qhat^T - W^T P^T, once per (chunk, key head)
             m["output"]["flops"] += Pk * 2 * C * C * dk
             m["output"]["bytes"] += Pk * dk * C * es

@@ -16,7 +16,7 @@ size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct Layout {
-    size_t err, slot_info, seq_first, W, U, G, A, B, Hs, E, M, AT, C, Z, dH, part;
+    size_t err, slot_info, seq_first, W, U, G, A, B, Us, Hs, E, M, AT, C, Z, dH, part;
     // gate and normalisation prologue (COMBA_GATED): its outputs, and the backward's gradients
     // w.r.t. them with the per-row contributions to da, dc
     size_t qh, kh, ga, gb, bg, dqh, dkh, dal, dbe, dbi, dar, dcr, dpa, dpc;
@@ -88,9 +88,14 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
     L.W = take(pairs * 64 * dk * es);
     L.U = take(pairs * 64 * dv * es);
     L.G = take(pairs * 64 * sizeof(float));
+    const bool tcp = comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv / vg);
     if (has_chunk_map(s->dk)) {
         L.A = take(pairs * dk * dk * es);
-        L.B = take(pairs * dv * dk * es);
+        // the tcgen05 path keeps U_s^T (its forward scan forms B^T itself); the others B^T
+        if (tcp)
+            L.Us = take(pairs * dv * 64 * es);
+        else
+            L.B = take(pairs * dv * dk * es);
     }
     L.Hs = take(pairs * dv * dk * es);
     if (backward) {
@@ -100,7 +105,7 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
         if (has_chunk_map(s->dk) && !comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv))
             L.AT = take(pairs * dk * dk * es);
         // the tcgen05 path keeps Z^T (its reverse scan forms C itself); the others C^T
-        if (comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv / vg))
+        if (tcp)
             L.Z = take(pairs * dk * 64 * es);
         else
             L.C = take(pairs * dv * dk * es);
@@ -182,6 +187,7 @@ void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* 
     // (offset 0 is the status word, so a zero offset marks a region that is not allocated)
     p.Ab = L.A ? w + L.A : nullptr;
     p.Bb = L.B ? w + L.B : nullptr;
+    p.Usb = L.Us ? w + L.Us : nullptr;
     p.Hb = w + L.Hs;
     if (backward_layout) {
         p.Eb = w + L.E;

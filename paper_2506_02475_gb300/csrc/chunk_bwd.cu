@@ -801,10 +801,10 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     a.X = tcp ? p.Ab : p.ATb;   // tcgen05 path: Atilde read as an MN-major operand
     a.x_mn = tcp ? 1 : 0;
     a.W = p.Wb; a.K = p.k;      // dk = 256: dH = gamma dH' + C - W^T Kbar dH' per chunk
-    if (tcp) {
-        a.zc = 1;
-        a.Z = p.Zb;
-        a.dO = p.dO;
+    if (tcp) {   // C^T = dO^T Z formed in the scan
+        a.ym = 1;
+        a.F = p.Zb;
+        a.tok = p.dO;
         a.Y = nullptr;
     }
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)p.slots * p.H, s))) return e;

@@ -434,6 +434,12 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     a.Gb = q.Gb; a.init = q.h0; a.fin = q.hT; a.Sout = q.Hb; a.X = q.Ab; a.Y = q.Bb; a.reverse = 0; a.x_mn = 0;
     a.W = q.Wb; a.K = q.k;
     if (DK == 256) a.Y = q.Ub;   // the wide scan forms E = U - W H itself
+    if (tcp) {                   // B^T = U_s^T K formed in the scan
+        a.ym = 2;
+        a.F = q.Usb;
+        a.tok = q.k;
+        a.Y = nullptr;
+    }
     a.err = q.err;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)q.slots * q.H, s))) return e;
     mark(q, ev0 + 2, s);

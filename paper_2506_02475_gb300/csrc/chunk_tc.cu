@@ -9,14 +9,15 @@
 //
 //   k_prep_tc      Gram K K^T -> decay/btilde mask -> UT inverse M (fp32, blocked
 //                  forward substitution) -> W^T = K^T Mw^T, U^T = V^T Mu^T ->
-//                  Atilde = -K^T Diag(s) W, B^T = (Diag(s) U)^T K  (s = gamma_C/gamma_r);
+//                  Atilde = -K^T Diag(s) W  (s = gamma_C/gamma_r), and U_s^T = (Diag(s) U)^T
+//                  for the forward scan, which forms B^T = U_s^T K itself;
 //                  with Comba-pk feedback vectors P: Gram P K^T and W^T = P^T Mw^T
 //   k_output_tc    P = Tril(Q~ K^T * Gamma), E^T = U^T - H^T W^T,
 //                  O^T = H^T Qhat^T + E^T P^T  (Qhat = Diag(gamma) Q~); for the
 //                  backward also Z^T = Qhat^T - W^T P^T, the factor of the reverse
 //                  scan's additive term C = Z^T dO (formed by the scan itself)
 //
-// Workspace tensors of this path: W^T, U^T, Z^T [pairs][128][64]; Atilde, B^T,
+// Workspace tensors of this path: W^T, U^T, U_s^T, Z^T [pairs][128][64]; Atilde,
 // H^T, dH^T [pairs][128][128]; E [pairs][64][128] row-major; M [pairs][64][64].
 #include "tc_tiles.cuh"
 
@@ -204,20 +205,19 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
     }
     publish_smem();
 
-    // Atilde = -K^T (Diag(s) W) -> cols [0,128);  B^T = (Diag(s) U)^T K -> cols [128,256).
-    if (ok && tid == 0) {
-        tc_gemm<true, false>(tmem, smem_u32(sKk), 128, smem_u32(sWt), 128, 128, 64, false);
-        tc_gemm<false, true>(tmem + 128, smem_u32(sUt), 128, smem_u32(sKk), 128, 128, 64, false);
-    }
+    // Atilde = -K^T (Diag(s) W) -> cols [0,128)
+    if (ok && tid == 0) tc_gemm<true, false>(tmem, smem_u32(sKk), 128, smem_u32(sWt), 128, 128, 64, false);
     if (ok) {
-        // W^T, U^T out while the tensor core works
+        // W^T, U^T and U_s^T (un-swizzled row by row) out while the tensor core works
         copy_staged<8>((bf16*)p.Wb + idx * D * 64, stW, tid, NTH);
         copy_staged<8>((bf16*)p.Ub + idx * D * 64, stU, tid, NTH);
+        uint4* us = reinterpret_cast<uint4*>((bf16*)p.Usb + idx * D * 64);
+        for (int e = tid; e < 128 * 8; e += NTH)
+            us[e] = *reinterpret_cast<const uint4*>(sUt + sw128_offset(e >> 3, 8 * (e & 7), 128));
     }
     ok = ok && ms.finish(tid);
-    // Atilde over the dead K tile, B^T over the dead V/Mw/Mu tiles (their copies are done)
+    // Atilde over the dead K tile
     uint8_t* stA = sK;
-    uint8_t* stB = sV;
     if (ok) {
         float d[32], v[8];
 #pragma unroll
@@ -230,18 +230,9 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
                 stage_chunk<16>(stA, row, 4 * g + q, pack8(v));
             }
         }
-#pragma unroll
-        for (int g = 2 * half; g < 2 * half + 2; ++g) {
-            tmem_ld32(trow + 128 + g * 32, d);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) stage_chunk<16>(stB, row, 4 * g + q, pack8(d + 8 * q));
-        }
     }
     __syncthreads();
-    if (ok) {
-        copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
-        copy_staged<16>((bf16*)p.Bb + idx * D * D, stB, tid, NTH);
-    }
+    if (ok) copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
     if (!ok && tid == 0) flag_error(p);
     tc_fence_before();
     __syncthreads();

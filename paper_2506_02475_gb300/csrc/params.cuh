@@ -54,7 +54,10 @@ struct ChunkParams {
     void* Ub;                // [pairs][64][dv]  WY factor U
     float* Gb;               // [pairs][64]      chunk-local log-cumsum of alpha
     void* Ab;                // [pairs][dk][dk]  Atilde = -Kbar^T W (forward scan operand)
-    void* Bb;                // [pairs][dv][dk]  (Kbar^T U)^T (forward scan additive term)
+    void* Bb;                // [pairs][dv][dk]  (Kbar^T U)^T (forward scan additive term; off the
+                             //                  tcgen05 path)
+    void* Usb;               // [pairs][dv][64]  U_s^T = (Diag(s) U)^T, s_r = gamma_C / gamma_r (tcgen05
+                             //                  path: the forward scan forms B^T = U_s^T K itself)
     void* Hb;                // [pairs][dv][dk]  chunk-start state, transposed
     void* Eb;                // [pairs][64][dv]  E = U - W H (saved for the backward)
     void* Mb;                // [pairs][64][64]  UT inverse M (saved for the backward)
@@ -139,11 +142,13 @@ struct ScanArgs {
     int x_mn;                // X is read as an MN-major operand ([k][m] row-major, no transpose)
     int vg;                  // value heads per key head: init/fin are [N, H / vg, dk, vg * dv]
     int* err;
-    // Reverse scan on the tcgen05 path (zc = 1): the additive term of each chunk is formed in the
-    // scan as (dO^T Z)^T from Z^T [pairs][dk][64] and dO [tokens, H, dv] instead of read from Y.
-    int zc = 0;
-    const void* Z = nullptr;
-    const void* dO = nullptr;
+    // tcgen05 path (dk = dv = 128): the scan forms each chunk's additive term itself instead of
+    // reading Y, as a product of a workspace factor F and a token tensor `tok`:
+    //   ym = 2 (forward):  B^T = U_s^T K,  F = U_s^T [pairs][dv][64], tok = keys [tokens, H / vg, dk]
+    //   ym = 1 (reverse):  C^T = dO^T Z,   F = Z^T [pairs][dk][64],   tok = dO [tokens, H, dv]
+    int ym = 0;
+    const void* F = nullptr;
+    const void* tok = nullptr;
 };
 cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long long pairs, cudaStream_t s);
 size_t scan_smem_bytes(bool is_bf16, int dk, int dv);

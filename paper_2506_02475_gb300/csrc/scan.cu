@@ -12,9 +12,10 @@
 // backward, Atilde read as an MN-major operand (bf16 path) or Atilde^T
 // (fp32 path); Y = B^T or C^T stored [dv][dk].  Each chunk stores the state it started
 // from (H_n^T, or dH_{n+1}^T in the backward) for the parallel kernels.  The
-// tcgen05 path's reverse scan reads no C^T: it forms C^T = dO^T Z itself from
-// the Z^T the forward's output kernel saved, one product per chunk issued ahead
-// of the sequential one (see k_scan_tc_split).
+// tcgen05 path reads no Y: its scans form B^T = U_s^T K (U_s = Diag(s) U, saved
+// by prep) and C^T = dO^T Z (Z^T saved by the forward's output kernel)
+// themselves, one product per chunk issued ahead of the sequential one (see
+// k_scan_tc_split).
 //
 // bf16 storage: one CTA per (sequence, head), 256 threads (two per state row,
 // each holding half of the row's dk columns); the fp32 state stays in registers.
@@ -25,7 +26,8 @@
 // sit on the chunk-to-chunk path; it drains while the next chunks compute).
 // X and Y stream in by TMA through mbarrier pipelines (3 and 2 stages); one
 // thread issues the tcgen05 MMAs (M = 128, N = dk, K = dk) into a TMEM
-// accumulator that all threads read back with tcgen05.ld.
+// accumulator that all threads read back with tcgen05.ld (shapes other than
+// dk = dv = 128; that one runs the row-split kernel below).
 // fp32 storage: the same recurrence with FMA tile products (tolerance 1e-4).
 #include <cuda.h>
 
@@ -251,46 +253,49 @@ __global__ void __launch_bounds__(256, 1)
     }
 }
 
-// Row-split variant (dk = dv = 128): two CTAs per (sequence, head), each owning 64 of
-// the state's dv rows (rows are independent under S^T <- gamma S^T + S^T X^T + Y).
-// The MMA is M = 64 (this CTA's rows) x N = dk x K = dk against the full X; read
-// back with tcgen05.ld.16x256b, the accumulator arrives in the m16n8 fragment
-// layout, so each thread keeps 32 state values (rows 16 (w & 3) + g, + 8; columns
-// 64 (w >> 2) + 8 t + 2 q, + 1).  Per chunk each SM loads X plus half of Y and
-// stores half of the chunk state, and the epilogue is half as long.  X and Y each
-// stream three chunks deep; one thread issues the MMAs while another issues the TMA
-// stores and loads, so a step's critical path is the MMA, not the issue sequence.
-// ZC (reverse scan of the tcgen05 path): the additive term C^T = dO^T Z is formed here.  Its
-// operands stream in four chunks deep in place of Y: Z^T [dk][64 positions] (K-major B) and this
-// CTA's 64 columns of dO [64 positions][64] (MN-major A).  Each chunk's C product is issued right
-// after the previous chunk's state product, into the other of two TMEM accumulators, so it runs
-// while that chunk's epilogue does; the state product then accumulates onto it.
-template <int DK, int DV, bool ZC>
+// Row-split variant (dk = dv = 128, the tcgen05 path): two CTAs per (sequence, head), each
+// owning 64 of the state's dv rows (rows are independent under S^T <- gamma S^T + S^T X^T + Y).
+// The MMA is M = 64 (this CTA's rows) x N = dk x K = dk against the full X; read back with
+// tcgen05.ld.16x256b, the accumulator arrives in the m16n8 fragment layout, so each thread
+// keeps 32 state values (rows 16 (w & 3) + g, + 8; columns 64 (w >> 2) + 8 t + 2 q, + 1).
+// Per chunk each SM loads X and stores half of the chunk state, and the epilogue is half as
+// long.  One thread issues the MMAs while another issues the TMA stores and loads, so a
+// step's critical path is the MMA, not the issue sequence.
+//
+// The additive term Y is not read: this kernel forms its rows as one more product per chunk,
+// K = 64 positions, from a workspace factor F and a token tensor T of the chunk:
+//   forward (YM = 2):  B^T = U_s^T K,  F = U_s^T = (Diag(s) U)^T [dv][64] (this CTA's 64 rows,
+//                      K-major A), T = the chunk's keys [64][dk] (MN-major B);
+//   reverse (YM = 1):  C^T = dO^T Z,   F = Z^T [dk][64] (K-major B), T = this CTA's 64 columns
+//                      of dO [64][64] (MN-major A).
+// F and T stream in four chunks deep.  Each chunk's product is issued right after the previous
+// chunk's state product, into the other of two TMEM accumulators, so it runs while that
+// chunk's epilogue does; the state product then accumulates onto it.  The rows of T past a
+// short chunk's end (the next sequence's tokens, or past the tensor) are zeroed first, so
+// nothing from outside the sequence enters its sums.
+template <int DK, int DV, int YM>
 struct ScanSplitSmem {
-    static constexpr int SX = 3, SY = 3, SZ = 4;
-    static constexpr uint32_t A_BYTES = 64 * DK * 2;    // this CTA's 64 rows of S^T; two buffers
+    static constexpr int SX = 3, SF = 4;
+    static constexpr uint32_t A_BYTES = 64 * DK * 2;                 // this CTA's 64 rows of S^T; two buffers
     static constexpr uint32_t X_BYTES = DK * DK * 2;
-    static constexpr uint32_t Y_BYTES = 64 * DK * 2;
-    static constexpr uint32_t ZT_BYTES = DK * 64 * 2;   // ZC: Z^T
-    static constexpr uint32_t DO_BYTES = 64 * 64 * 2;   // ZC: this CTA's dO columns
+    static constexpr uint32_t F_BYTES = (YM == 1 ? DK : 64) * 64 * 2;   // Z^T, or this CTA's rows of U_s^T
+    static constexpr uint32_t T_BYTES = 64 * (YM == 1 ? 64 : DK) * 2;   // this CTA's dO columns, or K
     static constexpr uint32_t OX = 2 * A_BYTES;
-    static constexpr uint32_t OY = OX + SX * X_BYTES;
-    static constexpr uint32_t OZ = OY;                  // ZC: Z^T stages, then dO stages
-    static constexpr uint32_t OD = OZ + SZ * ZT_BYTES;
-    static constexpr int NY = ZC ? SZ : SY;             // stages behind the full_y barriers
-    static constexpr size_t bytes() { return 1024 + (ZC ? OD + (size_t)SZ * DO_BYTES : OY + (size_t)SY * Y_BYTES); }
+    static constexpr uint32_t OF = OX + SX * X_BYTES;
+    static constexpr uint32_t OT = OF + SF * F_BYTES;
+    static constexpr size_t bytes() { return 1024 + OT + (size_t)SF * T_BYTES; }
 };
 
-template <int DK, int DV, bool XMN, bool ZC>
+template <int DK, int DV, bool XMN, int YM>
 __global__ void __launch_bounds__(256, 1)
-    k_scan_tc_split(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmY,
-                    const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmO) {
+    k_scan_tc_split(ScanArgs a, const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmF,
+                    const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmT) {
     static_assert(DK == 128 && DV == 128, "row split is laid out for dk = dv = 128");
-    using S = ScanSplitSmem<DK, DV, ZC>;
+    static_assert(YM == 1 || YM == 2, "the additive term is formed in the scan");
+    using S = ScanSplitSmem<DK, DV, YM>;
     constexpr int NT = DK / 16;   // 8-column tiles per thread (half of the columns)
-    constexpr uint32_t TCOLS = ZC ? 2 * DK : DK;   // ZC: two accumulators, chunk it in (it & 1)
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t full_x[S::SX], full_y[S::NY];
+    __shared__ uint64_t full_x[S::SX], full_f[S::SF];
     __shared__ uint64_t mma_bar;
     __shared__ uint32_t tmem_base;
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -321,23 +326,24 @@ __global__ void __launch_bounds__(256, 1)
 
     if (tid == 0) {
         for (int s = 0; s < S::SX; ++s) mbar_init(smem_u32(&full_x[s]), 1);
-        for (int s = 0; s < S::NY; ++s) mbar_init(smem_u32(&full_y[s]), 1);
+        for (int s = 0; s < S::SF; ++s) mbar_init(smem_u32(&full_f[s]), 1);
         mbar_init(smem_u32(&mma_bar), 1);
         mbar_fence_init();
     }
-    if (warp == 0) tmem_alloc(smem_u32(&tmem_base), TCOLS);
+    if (warp == 0) tmem_alloc(smem_u32(&tmem_base), 2 * DK);   // two accumulators: chunk it in (it & 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base;
     const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16) + 64 * wc;
-    auto acc_col = [&](int it) { return ZC ? (uint32_t)(it & 1) * DK : 0u; };
+    auto acc_col = [&](int it) { return (uint32_t)(it & 1) * DK; };
 
     auto chunk_of = [&](int it) { return a.reverse ? nch - 1 - it : it; };
     auto unit_of = [&](int it) { return (long long)(s0 + chunk_of(it)) * a.H + h; };
     auto a_buf = [&](int it) { return smem_u + (uint32_t)(it & 1) * S::A_BYTES; };
     auto x_buf = [&](int it) { return smem_u + S::OX + (uint32_t)(it % S::SX) * S::X_BYTES; };
-    auto y_off = [&](int it) { return S::OY + (uint32_t)(it % S::SY) * S::Y_BYTES; };
+    auto f_off = [&](int it) { return S::OF + (uint32_t)(it % S::SF) * S::F_BYTES; };
+    auto t_off = [&](int it) { return S::OT + (uint32_t)(it % S::SF) * S::T_BYTES; };
     auto issue_x = [&](int it) {
         const uint32_t fb = smem_u32(&full_x[it % S::SX]);
         mbar_expect_tx(fb, S::X_BYTES);
@@ -345,71 +351,57 @@ __global__ void __launch_bounds__(256, 1)
         for (int half = 0; half < DK / 64; ++half)
             tma_load_2d(x_buf(it) + half * DK * 128, &tmX, half * 64, (int)(unit_of(it) * DK), fb);
     };
-    auto issue_y = [&](int it) {
-        const uint32_t fb = smem_u32(&full_y[it % S::SY]);
-        mbar_expect_tx(fb, S::Y_BYTES);
+    auto issue_f = [&](int it) {   // F and T of the chunk
+        const uint32_t fb = smem_u32(&full_f[it % S::SF]);
+        mbar_expect_tx(fb, S::F_BYTES + S::T_BYTES);
+        const int tok = (int)(start + (long long)chunk_of(it) * kChunk);
+        if constexpr (YM == 1) {
+            tma_load_2d(smem_u + f_off(it), &tmF, 0, (int)(unit_of(it) * DK), fb);
+            tma_load_3d(smem_u + t_off(it), &tmT, 64 * rhalf, h, tok, fb);
+        } else {
+            tma_load_2d(smem_u + f_off(it), &tmF, 0, (int)(unit_of(it) * DV + 64 * rhalf), fb);
 #pragma unroll
-        for (int half = 0; half < DK / 64; ++half)
-            tma_load_2d(smem_u + y_off(it) + half * 64 * 128, &tmY, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), fb);
-    };
-    auto zt_buf = [&](int it) { return smem_u + S::OZ + (uint32_t)(it % S::SZ) * S::ZT_BYTES; };
-    auto do_buf = [&](int it) { return smem_u + S::OD + (uint32_t)(it % S::SZ) * S::DO_BYTES; };
-    auto issue_zd = [&](int it) {   // ZC: Z^T of the chunk, and its dO rows x this CTA's 64 columns
-        const uint32_t fb = smem_u32(&full_y[it % S::SZ]);
-        mbar_expect_tx(fb, S::ZT_BYTES + S::DO_BYTES);
-        tma_load_2d(zt_buf(it), &tmY, 0, (int)(unit_of(it) * DK), fb);
-        tma_load_3d(do_buf(it), &tmO, 64 * rhalf, h, (int)(start + (long long)chunk_of(it) * kChunk), fb);
+            for (int half = 0; half < DK / 64; ++half)   // the key head's keys, two 64-column halves
+                tma_load_3d(smem_u + t_off(it) + half * 64 * 128, &tmT, 64 * half, h / a.vg, tok, fb);
+        }
     };
     // Thread 0 issues the MMAs; thread 32 (warp 1) the TMA traffic: the chunk-state stores, the
-    // X / Y loads and the bulk-group waits, so neither waits for the other's issue sequence.
+    // X / F / T loads and the bulk-group waits, so neither waits for the other's issue sequence.
     constexpr int kTma = 32;
-    int nx = 0, ny = 0;
+    int nx = 0, nf = 0;
     if (tid == kTma) {
         for (; nx < S::SX - 1 && nx < nch; ++nx) issue_x(nx);
-        if constexpr (ZC) {
-            for (; ny < S::SZ - 1 && ny < nch; ++ny) issue_zd(ny);
-        } else {
-            for (; ny < S::SY - 1 && ny < nch; ++ny) issue_y(ny);
-        }
+        for (; nf < S::SF - 1 && nf < nch; ++nf) issue_f(nf);
     }
 
     constexpr uint32_t idesc = idesc_bf16_f32(64, DK) | (XMN ? 1u << 16 : 0u);
-    // ZC: C^T rows = dO^T (A: MN-major, M = this CTA's 64 dv columns) x Z (B: Z^T K-major), K = 64
-    constexpr uint32_t idesc_c = idesc_bf16_f32(64, DK) | (1u << 15);
-    auto issue_c = [&](int it) {
+    // additive-term product: A = dO^T (MN-major) for YM = 1, U_s^T (K-major) for YM = 2; B = Z^T
+    // (K-major) for YM = 1, K (MN-major) for YM = 2
+    constexpr uint32_t idesc_y = idesc_bf16_f32(64, DK) | (YM == 1 ? 1u << 15 : 1u << 16);
+    // Thread 0: wait for the chunk's F and T, zero T's rows past a short chunk, issue the product.
+    auto issue_y = [&](int it) {
+        if (!mbar_wait(smem_u32(&full_f[it % S::SF]), (it / S::SF) & 1)) return false;
+        const long long rem = len - (long long)chunk_of(it) * kChunk;
+        if (rem < kChunk) {
+            uint8_t* tb = smem + t_off(it);
+            for (int e = (int)rem * 8; e < kChunk * 8; ++e)
 #pragma unroll
-        for (int ks = 0; ks < 4; ++ks)
-            tc_mma_bf16(tmem + acc_col(it), desc_mnmajor(do_buf(it), 64, ks), desc_kmajor(zt_buf(it), DK, ks),
-                        idesc_c, ks > 0 ? 1u : 0u);
-    };
-    int cbad = 0;   // thread 0: a C product's operands never arrived
-    if constexpr (ZC) {
-        if (nch > 0) {
-            // The first chunk of the reverse scan is a sequence's last and may be short.  Its dO rows
-            // past the sequence end belong to the next sequence (or lie past the tensor): zero them,
-            // so that only this sequence's positions enter the product (its Z^T columns there are
-            // zero, but a non-finite dO elsewhere must not leak in).
-            const long long rem = len - (long long)chunk_of(0) * kChunk;
-            const int L0 = (int)(rem < kChunk ? rem : kChunk);
-            bool ok0 = true;
-            if (L0 < kChunk) {
-                ok0 = mbar_wait(smem_u32(&full_y[0]), 0);
-                if (ok0)
-                    for (int e = tid; e < (kChunk - L0) * 8; e += 256)
-                        *reinterpret_cast<uint4*>(smem + S::OD + (L0 + (e >> 3)) * 128 + (e & 7) * 16) =
-                            make_uint4(0, 0, 0, 0);
-                fence_async_smem();
-                __syncthreads();
-                tc_fence_after();
-            }
-            if (tid == 0) {
-                if (ok0 && mbar_wait(smem_u32(&full_y[0]), 0))
-                    issue_c(0);
-                else
-                    cbad = 1;
-            }
+                for (int half = 0; half < (YM == 1 ? 1 : DK / 64); ++half)
+                    *reinterpret_cast<uint4*>(tb + half * 64 * 128 + e * 16) = make_uint4(0, 0, 0, 0);
+            fence_async_smem();
         }
-    }
+        const uint32_t fa = smem_u + f_off(it), ta = smem_u + t_off(it);
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+            const uint64_t ad = YM == 1 ? desc_mnmajor(ta, 64, ks) : desc_kmajor(fa, 64, ks);
+            const uint64_t bd = YM == 1 ? desc_kmajor(fa, DK, ks) : desc_mnmajor(ta, 64, ks);
+            tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc_y, ks > 0 ? 1u : 0u);
+        }
+        return true;
+    };
+    int ybad = 0;   // thread 0: a chunk's F / T never arrived
+    if (tid == 0 && nch > 0 && !issue_y(0)) ybad = 1;
+
     auto log_decay = [&](int it) {
         const int c = chunk_of(it);
         const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
@@ -433,55 +425,42 @@ __global__ void __launch_bounds__(256, 1)
         __syncthreads();
         tc_fence_after();
 
-        int bad = cbad;
+        int bad = ybad;
         if (tid == 0) {
-            if (!cbad && mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
+            if (!ybad && mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
 #pragma unroll
                 for (int ks = 0; ks < DK / 16; ++ks) {
                     const int half = ks >> 2, sub = ks & 3;
                     const uint64_t ad = smem_desc_sw128(a_buf(it) + half * 64 * 128 + sub * 32);
                     const uint64_t bd = XMN ? desc_mnmajor(x_buf(it), DK, ks)
                                             : smem_desc_sw128(x_buf(it) + half * DK * 128 + sub * 32);
-                    tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc, (ZC || ks > 0) ? 1u : 0u);
+                    tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc, 1u);   // onto the additive term
                 }
             } else {
                 bad = 1;
             }
             tc_commit(smem_u32(&mma_bar));
-            if constexpr (ZC) {
-                // the next chunk's C product, into the other accumulator (read back two chunks ago)
-                if (!bad && it + 1 < nch) {
-                    if (mbar_wait(smem_u32(&full_y[(it + 1) % S::SZ]), ((it + 1) / S::SZ) & 1))
-                        issue_c(it + 1);
-                    else
-                        bad = cbad = 1;
-                }
-            }
+            // the next chunk's additive term, into the other accumulator (read back a chunk ago)
+            if (!bad && it + 1 < nch && !issue_y(it + 1)) bad = ybad = 1;
         } else if (tid == kTma) {
 #pragma unroll
             for (int half = 0; half < DK / 64; ++half)
                 tma_store_2d(&tmS, half * 64, (int)(unit_of(it) * DV + 64 * rhalf), a_buf(it) + half * 64 * 128);
             bulk_commit();
             if (nx < nch) issue_x(nx++);
-            if constexpr (ZC) {
-                // its stage last held chunk it - 1, whose C product the commit of chunk it - 1 covered
-                if (ny < nch) issue_zd(ny++);
-            } else {
-                if (ny < nch) issue_y(ny++);
-            }
+            // its stage last held chunk it - 1, whose product the commit of chunk it - 1 covered
+            if (nf < nch) issue_f(nf++);
         }
         if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
-        if constexpr (!ZC)
-            if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1)) bad = 1;
         if (tid == kTma) bulk_wait_read<1>();
         if (__syncthreads_or(bad)) {
             if (tid == kTma) {
                 if (a.err) atomicExch(a.err, 1);
                 for (int c = it; c < nx; ++c) mbar_wait(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
-                for (int c = it; c < ny; ++c) mbar_wait(smem_u32(&full_y[c % S::NY]), (c / S::NY) & 1);
+                for (int c = it; c < nf; ++c) mbar_wait(smem_u32(&full_f[c % S::SF]), (c / S::SF) & 1);
             }
-            if (ZC && tid == 0) {
-                // a C product issued after the last commit must finish before TMEM is released
+            if (tid == 0) {
+                // a product issued after the last commit must finish before TMEM is released
                 tc_commit(smem_u32(&mma_bar));
                 mbar_wait(smem_u32(&mma_bar), (it + 1) & 1);
             }
@@ -489,7 +468,7 @@ __global__ void __launch_bounds__(256, 1)
         }
         tc_fence_after();
 
-        // S^T <- gamma S^T + (S^T X^T) + Y  on this thread's 32 values
+        // S^T <- gamma S^T + (Y + S^T X^T)  on this thread's 32 values
         uint32_t d[32];
         asm volatile(
             "tcgen05.ld.sync.aligned.16x256b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
@@ -499,36 +478,18 @@ __global__ void __launch_bounds__(256, 1)
               "=r"(d[16]), "=r"(d[17]), "=r"(d[18]), "=r"(d[19]), "=r"(d[20]), "=r"(d[21]), "=r"(d[22]), "=r"(d[23]),
               "=r"(d[24]), "=r"(d[25]), "=r"(d[26]), "=r"(d[27]), "=r"(d[28]), "=r"(d[29]), "=r"(d[30]), "=r"(d[31])
             : "r"(tq + acc_col(it)));
-        __nv_bfloat162 yv[NT][2];
-        if constexpr (!ZC) {
-            const uint8_t* sY = smem + y_off(it);
-#pragma unroll
-            for (int t = 0; t < NT; ++t)
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh)
-                    yv[t][hh] = *reinterpret_cast<const __nv_bfloat162*>(sY + sw128_offset(r0 + 8 * hh, cq + 8 * t, 64));
-        }
         tmem_wait_ld();
 #pragma unroll
         for (int t = 0; t < NT; ++t)
 #pragma unroll
-            for (int hh = 0; hh < 2; ++hh) {
-                if constexpr (ZC) {   // the accumulator already holds C
-                    st[t][2 * hh] = fmaf(gam, st[t][2 * hh], __uint_as_float(d[4 * t + 2 * hh]));
-                    st[t][2 * hh + 1] = fmaf(gam, st[t][2 * hh + 1], __uint_as_float(d[4 * t + 2 * hh + 1]));
-                } else {
-                    const float2 yf = __bfloat1622float2(yv[t][hh]);
-                    st[t][2 * hh] = fmaf(gam, st[t][2 * hh], __uint_as_float(d[4 * t + 2 * hh]) + yf.x);
-                    st[t][2 * hh + 1] = fmaf(gam, st[t][2 * hh + 1], __uint_as_float(d[4 * t + 2 * hh + 1]) + yf.y);
-                }
-            }
+            for (int i = 0; i < 4; ++i) st[t][i] = fmaf(gam, st[t][i], __uint_as_float(d[4 * t + i]));
         tc_fence_before();
     }
 
     if (tid == kTma) bulk_wait_all();
     __syncthreads();
     tc_fence_after();
-    if (warp == 0) tmem_dealloc(tmem, TCOLS);
+    if (warp == 0) tmem_dealloc(tmem, 2 * DK);
     if (a.fin) {
         float* fin = a.fin + state_off(a, n, h, DK, DV);
 #pragma unroll
@@ -671,36 +632,37 @@ bool make_bf16_token_map(CUtensorMap* m, const void* base, long long tokens, int
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int DK, int DV, bool XMN, bool ZC>
+template <int DK, int DV, bool XMN, int YM>
 static cudaError_t run_scan_tc_split(const ScanArgs& a, long long pairs, cudaStream_t s) {
-    using S = ScanSplitSmem<DK, DV, ZC>;
-    CUtensorMap tx, ty, ts, to;
-    if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ts, a.Sout, pairs * DV, DK, 64))
+    using S = ScanSplitSmem<DK, DV, YM>;
+    CUtensorMap tx, tf, ts, tt;
+    if (!a.F || !a.tok || !make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ts, a.Sout, pairs * DV, DK, 64))
         return cudaErrorInvalidValue;
-    if (ZC) {
-        // Z^T [pairs * dk][64] with a [dk][64] box; dO [tokens][heads][dv] with a {64, 1, 64} box
-        if (!a.Z || !a.dO || !make_map(&ty, a.Z, pairs * DK, 64, DK) || !make_bf16_token_map(&to, a.dO, a.Ttot, a.H, DV))
+    if (YM == 1) {
+        // Z^T [pairs * dk][64] with a [dk][64] box; dO [tokens][heads][dv], {64, 1, 64} boxes
+        if (!make_map(&tf, a.F, pairs * DK, 64, DK) || !make_bf16_token_map(&tt, a.tok, a.Ttot, a.H, DV))
             return cudaErrorInvalidValue;
     } else {
-        if (!make_map(&ty, a.Y, pairs * DV, DK, 64)) return cudaErrorInvalidValue;
-        to = ty;   // not read
+        // U_s^T [pairs * dv][64] with a [64][64] box; keys [tokens][key heads][dk], {64, 1, 64} boxes
+        if (!make_map(&tf, a.F, pairs * DV, 64, 64) || !make_bf16_token_map(&tt, a.tok, a.Ttot, a.H / a.vg, DK))
+            return cudaErrorInvalidValue;
     }
-    cudaError_t e = cudaFuncSetAttribute(k_scan_tc_split<DK, DV, XMN, ZC>,
+    cudaError_t e = cudaFuncSetAttribute(k_scan_tc_split<DK, DV, XMN, YM>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)S::bytes());
     if (e) return e;
-    k_scan_tc_split<DK, DV, XMN, ZC><<<dim3(2 * a.N, a.H), 256, S::bytes(), s>>>(a, tx, ty, ts, to);
+    k_scan_tc_split<DK, DV, XMN, YM><<<dim3(2 * a.N, a.H), 256, S::bytes(), s>>>(a, tx, tf, ts, tt);
     return cudaGetLastError();
 }
 
 template <int DK, int DV, bool XMN>
 static cudaError_t run_scan_tc(const ScanArgs& a, long long pairs, cudaStream_t s) {
     if constexpr (DK == 128 && DV == 128) {
-        if constexpr (XMN) {
-            if (a.zc) return run_scan_tc_split<DK, DV, true, true>(a, pairs, s);
-        }
-        return run_scan_tc_split<DK, DV, XMN, false>(a, pairs, s);
+        // the tcgen05 path forms its additive term in the scan: C^T = dO^T Z (reverse, Atilde read
+        // MN-major) or B^T = U_s^T K (forward)
+        if (a.ym != (XMN ? 1 : 2)) return cudaErrorInvalidValue;
+        return run_scan_tc_split<DK, DV, XMN, XMN ? 1 : 2>(a, pairs, s);
     }
-    if (a.zc) return cudaErrorInvalidValue;
+    if (a.ym) return cudaErrorInvalidValue;
     using S = ScanTcSmem<DK, DV>;
     CUtensorMap tx, ty, ts;
     if (!make_map(&tx, a.X, pairs * DK, DK, DK) || !make_map(&ty, a.Y, pairs * DV, DK, DV) ||
@@ -737,8 +699,8 @@ cudaError_t launch_scan(const ScanArgs& a, bool is_bf16, int dk, int dv, long lo
 size_t scan_smem_bytes(bool is_bf16, int dk, int dv) {
     if (dk == 256) return is_bf16 && dv == 64 ? scan_wide_smem_bytes() : 0;
     if (is_bf16) {
-        if (dk == 128)   // the reverse (ZC) variant is the larger
-            return dv == 128 ? ScanSplitSmem<128, 128, true>::bytes() : ScanTcSmem<128, 64>::bytes();
+        if (dk == 128)   // both directions of the row split take the same shared memory
+            return dv == 128 ? ScanSplitSmem<128, 128, 1>::bytes() : ScanTcSmem<128, 64>::bytes();
         return dv == 128 ? ScanTcSmem<64, 128>::bytes() : ScanTcSmem<64, 64>::bytes();
     }
     return dk == 128 ? ScanSimtSmem<128>::bytes() : ScanSimtSmem<64>::bytes();

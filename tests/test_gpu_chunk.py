@@ -110,11 +110,12 @@ def test_varlen_small_with_empty_and_ragged_sequences(dtype, d):
     check_bwd(w, t)
 
 
-def test_nonfinite_dO_stays_inside_its_packed_sequence():
-    """Packed sequences [100, 70, 129] with dO = +inf on every token of the middle one: the
-    other sequences' token gradients and dh0 stay finite and match the oracle.  Their short
-    last chunks cover the next sequence's (or no) tokens, so every kernel that reads a chunk
-    tile, the reverse scan's dO tile included, must mask the rows past the sequence end."""
+def test_nonfinite_inputs_stay_inside_their_packed_sequence():
+    """Packed sequences [100, 70, 129] with k and dO = +inf on every token of the middle one:
+    the other sequences' outputs, final states, token gradients and dh0 stay finite and match
+    the oracle.  Their short last chunks cover the next sequence's (or no) tokens, so every
+    kernel that reads a chunk tile, the scans' key and dO tiles included, must mask the rows
+    past the sequence end."""
     lens = [100, 70, 129]
     w = inputs.make("custom", H=2, dk=128, dv=128, dtype="bf16", with_b=True, with_h0=True, with_grads=True,
                     lengths=lens, seed_offset=41)
@@ -122,11 +123,18 @@ def test_nonfinite_dO_stays_inside_its_packed_sequence():
     mid = slice(int(cu[1]), int(cu[2]))
     keep = np.ones(int(cu[-1]), bool)
     keep[mid] = False
-    dO_ref = w.dO.copy()
+    k_ref, dO_ref = w.k.copy(), w.dO.copy()
+    k_ref[mid] = 0.0
     dO_ref[mid] = 0.0
+    w.k[mid] = np.inf
     w.dO[mid] = np.inf
-    g = gpu_bwd(to_dev(w))
-    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, dO_ref, h0=w.h0, dhT=w.dhT, cu_seqlens=cu)
+    t = to_dev(w)
+    o, hT = gpu_fwd(t)
+    ro, rhT = oracle.fwd(w.q, k_ref, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0, cu_seqlens=cu)
+    assert np.all(np.isfinite(o[keep])) and rel(o[keep], ro[keep]) <= tol(w.dtype)
+    assert np.all(np.isfinite(hT[[0, 2]])) and rel(hT[[0, 2]], rhT[[0, 2]]) <= tol(w.dtype)
+    g = gpu_bwd(t)
+    r = oracle.bwd(w.q, k_ref, w.v, w.alpha, w.beta, w.b, w.d, dO_ref, h0=w.h0, dhT=w.dhT, cu_seqlens=cu)
     for key in ("dq", "dk", "dv", "dalpha", "dbeta"):
         x, ref = g[key][keep], r[key][keep]
         assert np.all(np.isfinite(x)), key
