@@ -273,6 +273,15 @@ __global__ void __launch_bounds__(256, 1)
 // chunk's epilogue does; the state product then accumulates onto it.  The rows of T past a
 // short chunk's end (the next sequence's tokens, or past the tensor) are zeroed first, so
 // nothing from outside the sequence enters its sums.
+// Zero rows [from, 64) of `halves` consecutive [64][128 B] tiles and make the writes visible to
+// the tensor core (one thread; kept out of line, off the scans' per-chunk issue path).
+static __device__ __noinline__ void zero_tile_rows(uint8_t* tile, int from, int halves) {
+    for (int half = 0; half < halves; ++half)
+        for (int e = from * 8; e < 64 * 8; ++e)
+            *reinterpret_cast<uint4*>(tile + half * 64 * 128 + e * 16) = make_uint4(0, 0, 0, 0);
+    fence_async_smem();
+}
+
 template <int DK, int DV, int YM>
 struct ScanSplitSmem {
     static constexpr int SX = 3, SF = 4;
@@ -378,18 +387,12 @@ __global__ void __launch_bounds__(256, 1)
     // additive-term product: A = dO^T (MN-major) for YM = 1, U_s^T (K-major) for YM = 2; B = Z^T
     // (K-major) for YM = 1, K (MN-major) for YM = 2
     constexpr uint32_t idesc_y = idesc_bf16_f32(64, DK) | (YM == 1 ? 1u << 15 : 1u << 16);
-    // Thread 0: wait for the chunk's F and T, zero T's rows past a short chunk, issue the product.
+    // Thread 0: the rows of T past a short chunk's end are zeroed before its product is issued.
+    // Only a sequence's last chunk can be short: the reverse scan's first step, the forward's last.
+    auto zero_tail = [&](int it) {
+        zero_tile_rows(smem + t_off(it), (int)(len - (long long)chunk_of(it) * kChunk), YM == 1 ? 1 : DK / 64);
+    };
     auto issue_y = [&](int it) {
-        if (!mbar_wait(smem_u32(&full_f[it % S::SF]), (it / S::SF) & 1)) return false;
-        const long long rem = len - (long long)chunk_of(it) * kChunk;
-        if (rem < kChunk) {
-            uint8_t* tb = smem + t_off(it);
-            for (int e = (int)rem * 8; e < kChunk * 8; ++e)
-#pragma unroll
-                for (int half = 0; half < (YM == 1 ? 1 : DK / 64); ++half)
-                    *reinterpret_cast<uint4*>(tb + half * 64 * 128 + e * 16) = make_uint4(0, 0, 0, 0);
-            fence_async_smem();
-        }
         const uint32_t fa = smem_u + f_off(it), ta = smem_u + t_off(it);
 #pragma unroll
         for (int ks = 0; ks < 4; ++ks) {
@@ -397,10 +400,18 @@ __global__ void __launch_bounds__(256, 1)
             const uint64_t bd = YM == 1 ? desc_kmajor(fa, DK, ks) : desc_mnmajor(ta, 64, ks);
             tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc_y, ks > 0 ? 1u : 0u);
         }
-        return true;
     };
+    auto wait_f = [&](int it) { return mbar_wait(smem_u32(&full_f[it % S::SF]), (it / S::SF) & 1); };
+    const bool tail_short = (len & (kChunk - 1)) != 0;
     int ybad = 0;   // thread 0: a chunk's F / T never arrived
-    if (tid == 0 && nch > 0 && !issue_y(0)) ybad = 1;
+    if (tid == 0 && nch > 0) {
+        if (!wait_f(0)) {
+            ybad = 1;
+        } else {
+            if (tail_short && (YM == 1 || nch == 1)) zero_tail(0);
+            issue_y(0);
+        }
+    }
 
     auto log_decay = [&](int it) {
         const int c = chunk_of(it);
@@ -441,7 +452,15 @@ __global__ void __launch_bounds__(256, 1)
             }
             tc_commit(smem_u32(&mma_bar));
             // the next chunk's additive term, into the other accumulator (read back a chunk ago)
-            if (!bad && it + 1 < nch && !issue_y(it + 1)) bad = ybad = 1;
+            if (!bad && it + 1 < nch) {
+                if (!wait_f(it + 1)) {
+                    bad = ybad = 1;
+                } else {
+                    if constexpr (YM == 2)
+                        if (tail_short && it + 2 == nch) zero_tail(it + 1);
+                    issue_y(it + 1);
+                }
+            }
         } else if (tid == kTma) {
 #pragma unroll
             for (int half = 0; half < DK / 64; ++half)
