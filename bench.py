@@ -128,13 +128,13 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 110_806, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "52788c9a97b55452"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0,0>", 83_584, ('scan.cu', 'common.cuh', 'params.cuh'), "4362e0614f0a6aeb"),
-    "output": ("k_output_tc", 128_467, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "52788c9a97b55452"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 83_417, ('scan.cu', 'common.cuh', 'params.cuh'), "4362e0614f0a6aeb"),
-    "bwd_local": ("k_bwd_local_tc", 192_595, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "cd583d86216d3690"),
+    "prep": ("k_prep_tc", 94_652, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "184b25a35eec3b9f"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_498, ('scan.cu', 'common.cuh', 'params.cuh'), "b672e4ffeaab0e2a"),
+    "output": ("k_output_tc", 130_018, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "184b25a35eec3b9f"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_647, ('scan.cu', 'common.cuh', 'params.cuh'), "b672e4ffeaab0e2a"),
+    "bwd_local": ("k_bwd_local_tc", 193_677, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "a8c1b350393300fe"),
 }
-DECODE_TRAFFIC = (481_121_280, ('decode.cu', 'common.cuh', 'params.cuh'), "4d5d41608ec01898")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (481_437_952, ('decode.cu', 'common.cuh', 'params.cuh'), "12709e39ee4a0b73")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
