@@ -65,7 +65,8 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
     B^T = U_s^T K from the U_s^T = (Diag(s) U)^T that prep writes in place of B^T, and
     C^T = dO^T Z from the Z^T that the output kernel saves (no separate C-term kernel).  `pk`: Comba-pk feedback vectors P, read by prep and
     by the local gradients, which also write dP.  At dk = 256 no chunk map is formed: the
-    scans read W, K and U (forward) or C^T (backward) and form two products per chunk.
+    scans read W, K and U (forward) or Z and dO (backward, forming C^T = dO^T Z) and form
+    two products per chunk.
     `H` counts value heads of width `dv`, `vg` of them per key head: tensors and products
     that depend on the key head only (q, k, gates, W, M, Atilde, the Gram, Q~ K^T, dq, dk,
     dalpha, dbeta) are counted once per (chunk, key head), however often a kernel re-reads
@@ -85,8 +86,9 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
     if wide:
         m["scan_fwd"] = dict(flops=P * 4 * C * dk * dv,
                              bytes=Pk * (2 * C * dk * es + C * f4) + P * (C * dv + dv * dk) * es)
-        m["scan_bwd"] = dict(flops=P * 4 * C * dk * dv,
-                             bytes=Pk * (2 * C * dk * es + C * f4) + P * 2 * dv * dk * es)
+        # reverse: W, K, Z per key head; dO in and dH'^T out per value head; C^T = dO^T Z formed inside
+        m["scan_bwd"] = dict(flops=P * 6 * C * dk * dv,
+                             bytes=Pk * (3 * C * dk * es + C * f4) + P * (C * dv + dv * dk) * es)
     else:
         m["scan_fwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=Pk * (dk * dk * es + f4) + P * 2 * dv * dk * es)
         m["scan_bwd"] = dict(flops=P * 2 * dv * dk * dk, bytes=Pk * (dk * dk * es + f4) + P * 2 * dv * dk * es)
@@ -95,6 +97,11 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
                        + P * (C * dv * es + dv * dk * es + C * dv * es * (2 if save else 1)))
     m["bwd_prep"] = dict(flops=Pk * 4 * C * C * dk + P * 2 * dv * C * dk,
                          bytes=Pk * (3 * C * dk * es + C * f4) + P * (C * dv * es + dv * dk * es))
+    if wide:   # the output kernel saves Z once per key head; no C-term kernel
+        if save:
+            m["output"]["flops"] += Pk * 2 * C * C * dk
+            m["output"]["bytes"] += Pk * C * dk * es
+        m["bwd_prep"] = dict(flops=0, bytes=0)
     if tc and not wide:
         # prep writes U_s^T = (Diag(s) U)^T instead of forming B^T; the forward scan forms
         # B^T = U_s^T K from it and the keys
@@ -128,13 +135,13 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 94_652, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "184b25a35eec3b9f"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_498, ('scan.cu', 'common.cuh', 'params.cuh'), "b672e4ffeaab0e2a"),
-    "output": ("k_output_tc", 130_018, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "184b25a35eec3b9f"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_647, ('scan.cu', 'common.cuh', 'params.cuh'), "b672e4ffeaab0e2a"),
-    "bwd_local": ("k_bwd_local_tc", 193_677, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "a8c1b350393300fe"),
+    "prep": ("k_prep_tc", 94_639, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "baad78d9ff3e50a2"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_455, ('scan.cu', 'common.cuh', 'params.cuh'), "7a7f118563435027"),
+    "output": ("k_output_tc", 130_166, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "baad78d9ff3e50a2"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_799, ('scan.cu', 'common.cuh', 'params.cuh'), "7a7f118563435027"),
+    "bwd_local": ("k_bwd_local_tc", 193_945, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "eae3896024836c81"),
 }
-DECODE_TRAFFIC = (481_437_952, ('decode.cu', 'common.cuh', 'params.cuh'), "12709e39ee4a0b73")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (481_069_568, ('decode.cu', 'common.cuh', 'params.cuh'), "608792102ddc3411")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
@@ -593,10 +600,10 @@ def run_ours(args, world, rank, local):
                     "all_outputs_read_back": {"value": tokens * world / (e_full_ms / 1e3), "ms_per_step": e_full_ms,
                                               "d2h_bytes_per_step": bo_full}},
             "clocks": clk,
-            # forward: chunk map, prep, scan, output; backward: (C term off the tcgen05 path), reverse
+            # forward: chunk map, prep, scan, output; backward: (C term at dk = 64), reverse
             # scan, local gradients, per-head sums; plus q - d p per call with p, the key-head sums
             # with value-head groups
-            "gpu_launches": (4 + (3 if tc else 4) + (2 if pk else 0) + (1 if vg > 1 else 0)) * args.steps,
+            "gpu_launches": (4 + (3 if tc or dk == 256 else 4) + (2 if pk else 0) + (1 if vg > 1 else 0)) * args.steps,
             "stages_ms_per_step": {f"{p}.{s}": v / args.steps for (p, s), v in stage_ms.items()},
             "wall_s_timed": wall,
         }

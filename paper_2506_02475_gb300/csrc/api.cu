@@ -104,8 +104,9 @@ comba_status_t plan(const comba_shape_t* s, int backward, Layout* out) {
         // Atilde^T is only materialised off the tcgen05 path (that reverse scan reads Atilde directly)
         if (has_chunk_map(s->dk) && !comba::use_tc_path(s->dtype == COMBA_BF16, s->dk, s->dv))
             L.AT = take(pairs * dk * dk * es);
-        // the tcgen05 path keeps Z^T (its reverse scan forms C itself); the others C^T
-        if (tcp)
+        // the tcgen05 path keeps Z^T, head dim 256 Z (their reverse scans form C themselves); the
+        // others C^T
+        if (tcp || s->dk == 256)
             L.Z = take(pairs * dk * 64 * es);
         else
             L.C = take(pairs * dv * dk * es);

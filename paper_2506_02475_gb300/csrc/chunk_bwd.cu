@@ -788,9 +788,10 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
         return e;
     const bool tcp = use_tc_path(sizeof(T) == 2, DK, DV);
     mark(p, ev0, s);
-    // tcgen05 path: no separate additive-term kernel; the forward's output kernel stored Z^T and
-    // the reverse scan forms C^T = dO^T Z per chunk
-    if (!tcp && p.slots > 0)
+    // tcgen05 path and head dim 256: no separate additive-term kernel; the forward's output kernel
+    // stored Z (Z^T on the tcgen05 path) and the reverse scan forms C^T = dO^T Z per chunk
+    const bool zc = tcp || DK == 256;
+    if (!zc && p.slots > 0)
         k_bwd_prep<T, DK, DV><<<dim3(p.slots, p.H / p.vg), 128, sm_prep, s>>>(p);   // one CTA per key head
     if ((e = cudaGetLastError())) return e;
     mark(p, ev0 + 1, s);
@@ -801,7 +802,7 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     a.X = tcp ? p.Ab : p.ATb;   // tcgen05 path: Atilde read as an MN-major operand
     a.x_mn = tcp ? 1 : 0;
     a.W = p.Wb; a.K = p.k;      // dk = 256: dH = gamma dH' + C - W^T Kbar dH' per chunk
-    if (tcp) {   // C^T = dO^T Z formed in the scan
+    if (zc) {   // C^T = dO^T Z formed in the scan
         a.ym = 1;
         a.F = p.Zb;
         a.tok = p.dO;
@@ -838,7 +839,7 @@ cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int e
 }
 
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk) {
-    if (kernel == 0 && use_tc_path(is_bf16, dk, dv)) return 0;   // no additive-term kernel there
+    if (kernel == 0 && (use_tc_path(is_bf16, dk, dv) || dk == 256)) return 0;   // no additive-term kernel there
     if (kernel == 1 && use_tc_path(is_bf16, dk, dv) && !pk) return local_tc_smem_bytes();
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? BPrepSmem<T, DK, DV>::bytes() : LocalSmem<T, DK, DV>::bytes();

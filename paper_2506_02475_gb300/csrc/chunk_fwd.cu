@@ -7,7 +7,8 @@
 //                 Atilde = -Kbar^T W, B = Kbar^T U (the inter-chunk state
 //                 equation with Kbar = Diag(gamma_C / gamma_r) K)
 //   (scan.cu)   : the sequential scan of those maps
-//   k_output    : per chunk, E = U - W H_n and the output equation
+//   k_output    : per chunk, E = U - W H_n and the output equation (at head dim 256 with the
+//                 backward's workspace also Z = Diag(gamma) Q~ - P W for the reverse scan)
 //                 O = Diag(gamma) Q~ H_n + Tril(Q~ K^T * Gamma) E, Q~ = Q - d K
 #include "params.cuh"
 
@@ -343,7 +344,10 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
         sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dh * to_f(sK[r * S::PK + c]));
     }
     __syncthreads();
-    if (p.o) {
+    // head dim 256 with the backward's workspace: Z = Diag(gamma) Q~ - P W is saved for the reverse
+    // scan, which forms the additive term C^T = dO^T Z itself
+    const bool zout = DK == 256 && p.Zb != nullptr;
+    if (p.o || zout) {
         float sc[8][4];
         zero(sc);
         warp_gemm<true, true, 8>(sc, sQ, S::PK, sK, S::PK, 16 * warp, 0, DK);
@@ -358,6 +362,28 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     }
     const float e0 = expf(sG[16 * warp + frag_row(0)]);
     const float e1 = expf(sG[16 * warp + frag_row(2)]);
+    if constexpr (DK == 256) {
+        if (zout) {
+            // Z [64][dk] at the key head's first value head (like W); each warp its own 16 rows, whose
+            // P rows it wrote itself.  Rows past a short chunk are zero (Q~ and P rows are).
+            __syncwarp();
+            T* zg = (T*)p.Zb + idx0 * 64 * DK;
+#pragma unroll 1
+            for (int n0 = 0; n0 < DK; n0 += 128) {
+                float z[16][4];
+                zero(z);
+                warp_gemm<true, false, 16>(z, sP, S::PL, sW, S::PK, 16 * warp, n0, 64);
+#pragma unroll
+                for (int t = 0; t < 16; ++t)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int r = 16 * warp + frag_row(i), c = n0 + frag_col(t, i);
+                        z[t][i] = (i < 2 ? e0 : e1) * to_f(sQ[r * S::PK + c]) - z[t][i];
+                    }
+                frag_store_global<T, 16>(zg, DK, 16 * warp, n0, z, 64);
+            }
+        }
+    }
 
     for (int j = 0; j < vg; ++j) {
         const long long idx = idx0 + j;

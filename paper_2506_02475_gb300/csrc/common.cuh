@@ -302,6 +302,15 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, int 
 }
 
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
+
+// Zero rows [from, 64) of `halves` consecutive [64][128 B] tiles and make the writes visible to
+// the tensor core (one thread; kept out of line, off the scans' per-chunk issue path).
+static __device__ __noinline__ void zero_tile_rows(uint8_t* tile, int from, int halves) {
+    for (int half = 0; half < halves; ++half)
+        for (int e = from * 8; e < 64 * 8; ++e)
+            *reinterpret_cast<uint4*>(tile + half * 64 * 128 + e * 16) = make_uint4(0, 0, 0, 0);
+    fence_async_smem();
+}
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
 

@@ -64,8 +64,9 @@ struct ChunkParams {
     void* ATb;               // [pairs][dk][dk]  Atilde^T (backward scan operand)
     void* Cb;                // [pairs][dv][dk]  ((Qhat - P W)^T dO)^T (backward scan additive term;
                              //                  off the tcgen05 path)
-    void* Zb;                // [pairs][dk][64]  Z^T = (Qhat - P W)^T (tcgen05 path: the reverse scan
-                             //                  forms Z^T dO itself)
+    void* Zb;                // [pairs][dk][64]  Z^T = (Qhat - P W)^T (tcgen05 path), or [pairs][64][dk]
+                             //                  Z at head dim 256 (once per key head, at its first value
+                             //                  head's pair): the reverse scan forms C^T = dO^T Z itself
     void* dHb;               // [pairs][dv][dk]  dL/dH at chunk end, transposed
     float* part;             // [pairs][2]       per-chunk db, dd partial sums
     int* err;                // device status word (nonzero: a bounded wait gave up)
@@ -146,6 +147,7 @@ struct ScanArgs {
     // reading Y, as a product of a workspace factor F and a token tensor `tok`:
     //   ym = 2 (forward):  B^T = U_s^T K,  F = U_s^T [pairs][dv][64], tok = keys [tokens, H / vg, dk]
     //   ym = 1 (reverse):  C^T = dO^T Z,   F = Z^T [pairs][dk][64],   tok = dO [tokens, H, dv]
+    // and at dk = 256 (k_scan_wide) ym = 1 with F = Z [pairs][64][dk] (key-head pairs).
     int ym = 0;
     const void* F = nullptr;
     const void* tok = nullptr;

@@ -273,15 +273,6 @@ __global__ void __launch_bounds__(256, 1)
 // chunk's epilogue does; the state product then accumulates onto it.  The rows of T past a
 // short chunk's end (the next sequence's tokens, or past the tensor) are zeroed first, so
 // nothing from outside the sequence enters its sums.
-// Zero rows [from, 64) of `halves` consecutive [64][128 B] tiles and make the writes visible to
-// the tensor core (one thread; kept out of line, off the scans' per-chunk issue path).
-static __device__ __noinline__ void zero_tile_rows(uint8_t* tile, int from, int halves) {
-    for (int half = 0; half < halves; ++half)
-        for (int e = from * 8; e < 64 * 8; ++e)
-            *reinterpret_cast<uint4*>(tile + half * 64 * 128 + e * 16) = make_uint4(0, 0, 0, 0);
-    fence_async_smem();
-}
-
 template <int DK, int DV, int YM>
 struct ScanSplitSmem {
     static constexpr int SX = 3, SF = 4;

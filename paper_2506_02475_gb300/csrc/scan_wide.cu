@@ -5,14 +5,22 @@
 // together.  So this scan applies section 3.3's chunk equations directly, two
 // products per chunk:
 //     forward:   E = U - W H,            H' = gamma_C H + Kbar^T E
-//     backward:  R = Kbar dH',           dH = gamma_C dH' + C - W^T R
+//     backward:  R = Kbar dH',           dH = gamma_C dH' + C - W^T R,   C = Z^T dO
 // with Kbar = Diag(s) K, s_r = gamma_C / gamma_r for positions r < L (zero past
 // the chunk).  Both run transposed over one value head's 64 state rows (dv):
 //     Pt = (Z - S^T F1^T) Diag(s),       S^T <- gamma_C S^T + Pt F2 + Y
 // forward:  F1 = W, F2 = K, Z = U^T, Y = 0 (Pt = E^T Diag(s));
 // backward: F1 = K, F2 = W, Z = 0,   Y = C^T (Pt = -R^T).
-// W rows past the chunk are zero (prep zero-fills its key rows); key rows past
-// the chunk (the next tokens, or the fill value past the tensor) meet s_r = 0.
+// The backward forms Y itself: C^T = dO^T Z (M = 64, N = 256, K = 64) from the
+// chunk's Z = Diag(gamma) Q~ - P W (saved by the forward's output kernel once per
+// key head) and this value head's dO, issued right after the first product into
+// the second product's accumulator, so it runs while Pt is formed and the second
+// product accumulates onto it.
+// W rows past the chunk are zero (prep zero-fills its key rows).  Key rows past
+// a short chunk (the next sequence's tokens, or the fill value past the tensor)
+// meet s_r = 0, but are zeroed in shared memory all the same, so that a
+// non-finite key elsewhere cannot reach this sequence (0 * inf); so are the dO
+// rows there in the backward.
 //
 // One CTA per (sequence, value head), 256 threads.  Both products run on the
 // tensor core (tcgen05, M = 64): S^T F1^T (N = 64, K = 256) and Pt F2 (N = 256,
@@ -23,8 +31,9 @@
 // (64 fp32 values a thread) across the whole sequence.  One thread issues the
 // MMAs; another issues the TMA traffic: F1 single-buffered and refilled as soon
 // as the first product has read it, F2 and Z / Y double-buffered a chunk
-// ahead, and each chunk's starting state (H_n^T, or dH_{n+1}^T in the backward)
-// stored in bf16 by a bulk tensor copy from the A-operand tile.
+// ahead (the backward's stage also holds Z and the dO tile), and each chunk's
+// starting state (H_n^T, or dH_{n+1}^T in the backward) stored in bf16 by a bulk
+// tensor copy from the A-operand tile.
 #include <cuda.h>
 
 #include "params.cuh"
@@ -32,18 +41,21 @@
 namespace comba {
 
 bool make_bf16_map(CUtensorMap* m, const void* base, long long rows, int cols, int box_rows);
+bool make_bf16_token_map(CUtensorMap* m, const void* base, long long tokens, int heads, int cols);
 
 namespace {
 
 constexpr int kWideDK = 256, kWideDV = 64;
+
 
 struct WideSmem {
     static constexpr uint32_t T_BYTES = 64 * kWideDK * 2;   // a [64][256] bf16 tile: four 64-column halves
     static constexpr uint32_t OA = 0;                       // S^T: A operand of the first product, stored state
     static constexpr uint32_t OP = OA + T_BYTES;            // Pt: A operand of the second product [64][64]
     static constexpr uint32_t OF1 = OP + 8192;              // F1 (one buffer)
-    static constexpr uint32_t OST = OF1 + T_BYTES;          // two stages: F2, then Z (U, [64][64]) or Y (C^T)
-    __host__ __device__ static constexpr uint32_t z_bytes(bool reverse) { return reverse ? T_BYTES : 8192; }
+    static constexpr uint32_t OST = OF1 + T_BYTES;          // two stages: F2, then U [64][64] (forward) or
+                                                            // Z [64][256] and dO [64][64] (backward)
+    __host__ __device__ static constexpr uint32_t z_bytes(bool reverse) { return reverse ? T_BYTES + 8192 : 8192; }
     __host__ __device__ static constexpr uint32_t stage_bytes(bool reverse) { return T_BYTES + z_bytes(reverse); }
     __host__ __device__ static constexpr size_t bytes(bool reverse) { return 1024 + OST + 2 * stage_bytes(reverse); }
 };
@@ -99,7 +111,8 @@ __device__ __forceinline__ void tmem_frags(uint32_t taddr, uint32_t (&r)[NT * 4]
 
 __global__ void __launch_bounds__(256, 1)
     k_scan_wide(ScanArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmK,
-                const __grid_constant__ CUtensorMap tmZ, const __grid_constant__ CUtensorMap tmS) {
+                const __grid_constant__ CUtensorMap tmZ, const __grid_constant__ CUtensorMap tmS,
+                const __grid_constant__ CUtensorMap tmO) {
     using S = WideSmem;
     constexpr int DK = kWideDK, DV = kWideDV, NT = DK / 16;   // 16 8-column state tiles a thread
     constexpr int kTma = 32;                                  // the thread that issues the TMA traffic
@@ -184,8 +197,9 @@ __global__ void __launch_bounds__(256, 1)
         if (rev) {
             load_w(uF2(it), it, bar);
 #pragma unroll
-            for (int half = 0; half < 4; ++half)
-                tma_load_2d(uZ(it) + half * 8192, &tmZ, 64 * half, (int)(unit_of(it) * 64), bar);   // C^T
+            for (int half = 0; half < 4; ++half)   // Z, stored at the key head's unit
+                tma_load_2d(uZ(it) + half * 8192, &tmZ, 64 * half, (int)(kunit_of(it) * 64), bar);
+            tma_load_3d(uZ(it) + S::T_BYTES, &tmO, 0, h, (int)(start + (long long)chunk_of(it) * kChunk), bar);   // dO
         } else {
             load_k(uF2(it), it, bar);
             tma_load_2d(uZ(it), &tmZ, 0, (int)(unit_of(it) * 64), bar);                              // U
@@ -212,6 +226,7 @@ __global__ void __launch_bounds__(256, 1)
     if (nch > 0) load_g(0);
 
     bool failed = false;
+    int n2 = 0;   // thread 0: commits to mma2_bar so far
     for (int it = 0; it < nch; ++it) {
         const int L = len_of(it);
         float g[8];
@@ -237,9 +252,25 @@ __global__ void __launch_bounds__(256, 1)
 
         int bad = 0;
         if (tid == 0) {
-            if (mbar_wait(smem_u32(&full_f1), it & 1)) tc_gemm_m64<false, false>(tmem, uA, 64, uF1, 64, 64, DK, false);
-            else bad = 1;
+            if (mbar_wait(smem_u32(&full_f1), it & 1)) {
+                // backward: F1 holds the keys; the first chunk of the reverse scan may be short
+                if (rev && it == 0 && L < kChunk) zero_tile_rows(smem + S::OF1, L, 4);
+                tc_gemm_m64<false, false>(tmem, uA, 64, uF1, 64, 64, DK, false);
+            } else {
+                bad = 1;
+            }
             tc_commit(smem_u32(&mma1_bar));
+            if (rev && !bad) {
+                // C^T = dO^T Z into the second product's columns (read back in the previous chunk's update)
+                if (mbar_wait(smem_u32(&full_st[it & 1]), (it >> 1) & 1)) {
+                    // the reverse scan's first chunk is a sequence's last and may be short: its dO rows
+                    // past the sequence end (the next sequence's, or past the tensor) must not enter
+                    if (it == 0 && L < kChunk) zero_tile_rows(smem + (uZ(it) - su) + S::T_BYTES, L, 1);
+                    tc_gemm_m64<true, true>(tmem + 64, uZ(it) + S::T_BYTES, 64, uZ(it), 64, DK, 64, false);
+                } else {
+                    bad = 1;
+                }
+            }
         } else if (tid == kTma) {
 #pragma unroll
             for (int half = 0; half < 4; ++half) tma_store_tile(&tmS, 64 * half, (int)(unit_of(it) * 64), uA + half * 8192);
@@ -284,29 +315,24 @@ __global__ void __launch_bounds__(256, 1)
         __syncthreads();
         tc_fence_after();
         if (tid == 0) {
-            tc_gemm_m64<false, true>(tmem + 64, uP, 64, uF2(it), 64, DK, 64, false);
+            // forward: F2 holds the keys; the last chunk may be short
+            if (!rev && it + 1 == nch && L < kChunk) zero_tile_rows(smem + (uF2(it) - su), L, 4);
+            tc_gemm_m64<false, true>(tmem + 64, uP, 64, uF2(it), 64, DK, 64, rev);   // onto C^T (backward)
             tc_commit(smem_u32(&mma2_bar));
+            ++n2;
         }
         if (!mbar_wait(smem_u32(&mma2_bar), it & 1)) bad = 1;
         tc_fence_after();
 
-        // S^T <- gamma_C S^T + Pt F2 + Y
+        // S^T <- gamma_C S^T + Pt F2 + Y  (the accumulator holds Y as well)
         if (!bad) {
             uint32_t d[4 * NT];
             tmem_frags<NT>(tq + 64 + 128 * wc, d);
             const float gam = __expf(gL);
-            const uint8_t* y = smem + (uZ(it) - su);
 #pragma unroll
             for (int t = 0; t < NT; ++t)
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    float2 yf = make_float2(0.f, 0.f);
-                    if (rev)   // C^T
-                        yf = __bfloat1622float2(
-                            *reinterpret_cast<const __nv_bfloat162*>(y + sw128_offset(r0 + 8 * hh, cq + 8 * t, 64)));
-                    st[t][2 * hh] = fmaf(gam, st[t][2 * hh], __uint_as_float(d[4 * t + 2 * hh]) + yf.x);
-                    st[t][2 * hh + 1] = fmaf(gam, st[t][2 * hh + 1], __uint_as_float(d[4 * t + 2 * hh + 1]) + yf.y);
-                }
+                for (int i = 0; i < 4; ++i) st[t][i] = fmaf(gam, st[t][i], __uint_as_float(d[4 * t + i]));
         }
         tc_fence_before();
         if (__syncthreads_or(bad)) {   // this stage and Pt are fully read
@@ -316,6 +342,11 @@ __global__ void __launch_bounds__(256, 1)
         if (tid == kTma && it + 2 < nch) issue_stage(it + 2);
     }
 
+    if (failed && tid == 0) {
+        // a C^T product issued after the last commit finishes before TMEM is released
+        tc_commit(smem_u32(&mma2_bar));
+        mbar_wait(smem_u32(&mma2_bar), n2 & 1);
+    }
     if (failed && tid == kTma) {
         // a bounded wait gave up: record it, and let the last load issued to each barrier land
         // (bounded waits again) before this CTA's shared memory is released
@@ -345,16 +376,24 @@ cudaError_t launch_scan_wide(const ScanArgs& a, cudaStream_t s) {
     const bool rev = a.reverse != 0;
     const long long pairs = (long long)a.slots * a.H;
     const int Hk = a.H / a.vg;
-    CUtensorMap tw, tk, tz, ts;
+    CUtensorMap tw, tk, tz, ts, to;
     const long long krows = a.Ttot > 0 ? a.Ttot : 1;   // a valid view even when no token exists
     const long long prow = pairs > 0 ? pairs * 64 : 64;
+    // backward: Z [pairs * 64][dk] (key-head units) and dO [tokens][value heads][64]; forward: U
+    if (rev && (a.ym != 1 || !a.F || !a.tok)) return cudaErrorInvalidValue;
     if (!make_bf16_map(&tw, a.W, prow, kWideDK, 64) || !make_bf16_map(&tk, a.K, krows, Hk * kWideDK, 64) ||
-        !make_bf16_map(&tz, a.Y, prow, rev ? kWideDK : kWideDV, 64) || !make_bf16_map(&ts, a.Sout, prow, kWideDK, 64))
+        !make_bf16_map(&tz, rev ? a.F : a.Y, prow, rev ? kWideDK : kWideDV, 64) ||
+        !make_bf16_map(&ts, a.Sout, prow, kWideDK, 64))
         return cudaErrorInvalidValue;
+    if (rev) {
+        if (!make_bf16_token_map(&to, a.tok, krows, a.H, kWideDV)) return cudaErrorInvalidValue;
+    } else {
+        to = tz;   // not read
+    }
     const size_t sm = WideSmem::bytes(rev);
     cudaError_t e = cudaFuncSetAttribute(k_scan_wide, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
-    if (a.N > 0 && a.H > 0) k_scan_wide<<<dim3(a.N, a.H), 256, sm, s>>>(a, tw, tk, tz, ts);
+    if (a.N > 0 && a.H > 0) k_scan_wide<<<dim3(a.N, a.H), 256, sm, s>>>(a, tw, tk, tz, ts, to);
     return cudaGetLastError();
 }
 

@@ -110,14 +110,15 @@ def test_varlen_small_with_empty_and_ragged_sequences(dtype, d):
     check_bwd(w, t)
 
 
-def test_nonfinite_inputs_stay_inside_their_packed_sequence():
+@pytest.mark.parametrize("dk,dv", [(128, 128), (256, 128)])
+def test_nonfinite_inputs_stay_inside_their_packed_sequence(dk, dv):
     """Packed sequences [100, 70, 129] with k and dO = +inf on every token of the middle one:
     the other sequences' outputs, final states, token gradients and dh0 stay finite and match
     the oracle.  Their short last chunks cover the next sequence's (or no) tokens, so every
     kernel that reads a chunk tile, the scans' key and dO tiles included, must mask the rows
-    past the sequence end."""
+    past the sequence end.  Head dim 128 (tcgen05 kernels) and 256 (two value heads of 64)."""
     lens = [100, 70, 129]
-    w = inputs.make("custom", H=2, dk=128, dv=128, dtype="bf16", with_b=True, with_h0=True, with_grads=True,
+    w = inputs.make("custom", H=2, dk=dk, dv=dv, dtype="bf16", with_b=True, with_h0=True, with_grads=True,
                     lengths=lens, seed_offset=41)
     cu = w.cu_seqlens
     mid = slice(int(cu[1]), int(cu[2]))
