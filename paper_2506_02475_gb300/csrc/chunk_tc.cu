@@ -74,6 +74,20 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
     // P K^T, and K (rows 64..127) is the operand of every later product that takes K.
     const bool pk = p.p != nullptr;
     const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
+    // The per-position gates go first: the first barrier waits on them, and loads issued behind
+    // the tiles' cp.async traffic would queue behind it.
+    const int lane = tid & 31;
+    const float* ag = p.alpha + t0 * Hk + hk;
+    float a0 = 1.f, a1 = 1.f, bev = 0.f, alv = 1.f, bh = 1.f;
+    if (warp == 0) {
+        a0 = lane < L ? ag[(long long)lane * Hk] : 1.f;
+        a1 = lane + 32 < L ? ag[(long long)(lane + 32) * Hk] : 1.f;
+    }
+    if (tid < 64) {
+        bev = tid < L ? p.beta[(t0 + tid) * Hk + hk] : 0.f;
+        alv = tid < L ? ag[(long long)tid * Hk] : 1.f;
+        bh = p.b ? p.b[hk] : 1.f;
+    }
     {
         const bf16* kg = (const bf16*)p.k + (t0 * Hk + hk) * D;
         const bf16* fg = pk ? (const bf16*)p.p + (t0 * Hk + hk) * D : kg;
@@ -88,12 +102,10 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
     const uint8_t* sKk = pk ? sK + 64 * 128 : sK;   // the 64 key rows (rows 64.. of each K-half for pk)
     load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
     cp_async_commit();
-    if (warp == 0) chunk_log_cumsum(p.alpha + t0 * Hk + hk, Hk, L, sG, sGm1);
+    if (warp == 0) chunk_log_cumsum_vals(a0, a1, L, sG, sGm1);
     if (tid < 64) {
-        const float be = tid < L ? p.beta[(t0 + tid) * Hk + hk] : 0.f;
-        sBe[tid] = be;
-        const float al = tid < L ? p.alpha[(t0 + tid) * Hk + hk] : 1.f;
-        sBt[tid] = (p.b ? p.b[hk] : 1.f) * be * feedback_scale(p.iplr, al);
+        sBe[tid] = bev;
+        sBt[tid] = bh * bev * feedback_scale(p.iplr, alv);
     }
     __syncthreads();   // sG, sGm1, sBt complete
     if (tid < 64) sWs[tid] = sBt[tid] * expf(sGm1[tid]);

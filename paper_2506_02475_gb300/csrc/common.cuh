@@ -238,10 +238,11 @@ __host__ __device__ constexpr size_t align128(size_t off) { return (off + 127) &
 // Inclusive prefix sum of log(alpha) over a chunk (warp-wide; lane handles
 // positions lane and lane + 32).  Positions >= L contribute 0, so G stays
 // finite there.  Writes G[p] and Gm1[p] = G[p-1] (Gm1[0] = 0).
-__device__ __forceinline__ void chunk_log_cumsum(const float* alpha, long long stride, int L, float* G, float* Gm1) {
+// chunk_log_cumsum_vals takes the lane's alpha values (positions lane, lane + 32) already loaded.
+__device__ __forceinline__ void chunk_log_cumsum_vals(float a0, float a1, int L, float* G, float* Gm1) {
     const int lane = threadIdx.x & 31;
-    float x0 = lane < L ? logf(alpha[(long long)lane * stride]) : 0.f;
-    float x1 = lane + 32 < L ? logf(alpha[(long long)(lane + 32) * stride]) : 0.f;
+    float x0 = lane < L ? logf(a0) : 0.f;
+    float x1 = lane + 32 < L ? logf(a1) : 0.f;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
         const float y0 = __shfl_up_sync(0xffffffffu, x0, o);
@@ -256,6 +257,12 @@ __device__ __forceinline__ void chunk_log_cumsum(const float* alpha, long long s
     const float p1 = __shfl_up_sync(0xffffffffu, x1, 1);
     Gm1[lane] = lane == 0 ? 0.f : p0;
     Gm1[lane + 32] = lane == 0 ? tot0 : p1;
+}
+__device__ __forceinline__ void chunk_log_cumsum(const float* alpha, long long stride, int L, float* G, float* Gm1) {
+    const int lane = threadIdx.x & 31;
+    const float a0 = lane < L ? alpha[(long long)lane * stride] : 1.f;
+    const float a1 = lane + 32 < L ? alpha[(long long)(lane + 32) * stride] : 1.f;
+    chunk_log_cumsum_vals(a0, a1, L, G, Gm1);
 }
 
 // ------------------------------------------- sm_100-family async primitives
