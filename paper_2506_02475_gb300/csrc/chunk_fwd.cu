@@ -188,16 +188,27 @@ __global__ void __launch_bounds__(128) k_prep(ChunkParams p) {
         load_tile_async<T>(sV, S::PV, (const T*)p.v + (t0 * p.H + hk * p.vg + j) * DV, (long long)p.H * DV, 64, DV,
                            L, tid, 128);
     };
+    // The per-position gates go first, so that their loads do not queue behind the tiles' cp.async
+    // traffic; the log-cumsum then runs while the tiles arrive.
+    const int lane = tid & 31;
+    float a0 = 1.f, a1 = 1.f, bev = 0.f, alv = 1.f, bh = 1.f;
+    if (warp == 0) {
+        a0 = lane < L ? p.alpha[kr0 + (long long)lane * Hk] : 1.f;
+        a1 = lane + 32 < L ? p.alpha[kr0 + (long long)(lane + 32) * Hk] : 1.f;
+    }
+    if (tid < 64) {
+        bev = tid < L ? p.beta[kr0 + (long long)tid * Hk] : 0.f;
+        alv = tid < L ? p.alpha[kr0 + (long long)tid * Hk] : 1.f;
+        bh = p.b ? p.b[hk] : 1.f;
+    }
     load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
     if (p.p) load_tile_async<T>(sF, S::PK, (const T*)p.p + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_v(0);
     cp_async_commit();
-    if (warp == 0) chunk_log_cumsum(p.alpha + kr0, Hk, L, sG, sGm1);
+    if (warp == 0) chunk_log_cumsum_vals(a0, a1, L, sG, sGm1);
     if (tid < 64) {
-        const float be = tid < L ? p.beta[kr0 + (long long)tid * Hk] : 0.f;
-        sBe[tid] = be;
-        const float al = tid < L ? p.alpha[kr0 + (long long)tid * Hk] : 1.f;
-        sBt[tid] = (p.b ? p.b[hk] : 1.f) * be * feedback_scale(p.iplr, al);
+        sBe[tid] = bev;
+        sBt[tid] = bh * bev * feedback_scale(p.iplr, alv);
     }
     cp_async_wait<0>();
     __syncthreads();
@@ -327,6 +338,7 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     };
 
     const long long kr0 = t0 * Hk + hk, kld = (long long)Hk * DK;   // key-side rows
+    const float dh = p.d[hk];   // loaded ahead of the tiles' cp.async traffic
     load_tile_async<T>(sQ, S::PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx0 * 64 * DK, DK, 64, DK, 64, tid, 128);
@@ -338,7 +350,6 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     cp_async_wait<1>();
     __syncthreads();
 
-    const float dh = p.d[hk];
     for (int e = tid; e < 64 * DK; e += 128) {
         const int r = e / DK, c = e % DK;
         sQ[r * S::PK + c] = from_f<T>(to_f(sQ[r * S::PK + c]) - dh * to_f(sK[r * S::PK + c]));

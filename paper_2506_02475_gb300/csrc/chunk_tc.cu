@@ -292,6 +292,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     bf16* sO = reinterpret_cast<bf16*>(sHt);   // [64][136] staging of O
     float* sG = reinterpret_cast<float*>(sm + S::OG);
 
+    const float dh = p.d[hk];   // loaded ahead of the tiles' cp.async traffic
     {
         // Q into rows 0-63 and K into rows 64-127 of one K-major tile (rows past the chunk zero)
         const bf16* qg = (const bf16*)p.q + (t0 * Hk + hk) * D;
@@ -316,7 +317,6 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     cp_async_wait<0>();
     __syncthreads();
     // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
-    const float dh = p.d[hk];
     for (int e = tid; e < 64 * 16; e += NTH) {
         const int r = e >> 4, ch = e & 15;
         uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
