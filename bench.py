@@ -135,13 +135,13 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 94_639, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "baad78d9ff3e50a2"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_455, ('scan.cu', 'common.cuh', 'params.cuh'), "7a7f118563435027"),
-    "output": ("k_output_tc", 130_166, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "baad78d9ff3e50a2"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_799, ('scan.cu', 'common.cuh', 'params.cuh'), "7a7f118563435027"),
-    "bwd_local": ("k_bwd_local_tc", 193_945, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "eae3896024836c81"),
+    "prep": ("k_prep_tc", 94_684, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e9834dbb5b984f52"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_492, ('scan.cu', 'common.cuh', 'params.cuh'), "719c2e63f7fb0962"),
+    "output": ("k_output_tc", 130_177, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "e9834dbb5b984f52"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_777, ('scan.cu', 'common.cuh', 'params.cuh'), "719c2e63f7fb0962"),
+    "bwd_local": ("k_bwd_local_tc", 193_688, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "ae17b319a7584d5f"),
 }
-DECODE_TRAFFIC = (481_069_568, ('decode.cu', 'common.cuh', 'params.cuh'), "608792102ddc3411")   # whole Bd=256 H=16 launch
+DECODE_TRAFFIC = (481_439_744, ('decode.cu', 'common.cuh', 'params.cuh'), "2df9a51b0d0f5a9d")   # whole Bd=256 H=16 launch
 
 
 def sources_hash(files):
