@@ -292,7 +292,8 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     bf16* sO = reinterpret_cast<bf16*>(sHt);   // [64][136] staging of O
     float* sG = reinterpret_cast<float*>(sm + S::OG);
 
-    const float dh = p.d[hk];   // loaded ahead of the tiles' cp.async traffic
+    const float dh = p.d[hk];   // loaded ahead of the tiles' cp.async traffic, as are the log-decays
+    const float gv = tid < 64 ? p.Gb[idx * 64 + tid] : 0.f;
     {
         // Q into rows 0-63 and K into rows 64-127 of one K-major tile (rows past the chunk zero)
         const bf16* qg = (const bf16*)p.q + (t0 * Hk + hk) * D;
@@ -308,7 +309,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     load_sw(sUt, 128, 64, (const bf16*)p.Ub + idx * D * 64, 64, 128, tid, NTH);
     load_sw(sHt, 128, D, (const bf16*)p.Hb + idx * D * D, D, 128, tid, NTH);
     cp_async_commit();
-    if (tid < 64) sG[tid] = p.Gb[idx * 64 + tid];
+    if (tid < 64) sG[tid] = gv;
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
         mbar_fence_init();
