@@ -254,6 +254,20 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     const long long kr0 = krow(p, t0, h), kld = (long long)(p.H / p.vg) * DK;
     const float bh = p.b ? p.b[hk] : 1.f;
     const float dh = p.d[hk];
+    // M and G are stored once per key head, at its first value head's unit
+    const long long kidx = (long long)slot * p.H + hk * p.vg;
+    // At head dims up to 128 the per-row scalars go ahead of the tiles' cp.async traffic, whose
+    // queue their loads would otherwise wait behind.  At head dim 256 (a larger kernel) holding
+    // them across the tile loads measured slower, so there they follow the tiles as before.
+    float rg = 0.f, rgm1 = 0.f, rbe = 0.f, ral = 1.f;
+    if constexpr (DK <= 128) {
+        if (tid < 64) {
+            rg = p.Gb[kidx * 64 + tid];
+            rgm1 = tid > 0 ? p.Gb[kidx * 64 + tid - 1] : 0.f;
+            rbe = tid < L ? p.beta[krow(p, t0 + tid, h)] : 0.f;
+            ral = tid < L ? p.alpha[krow(p, t0 + tid, h)] : 1.f;
+        }
+    }
     load_tile_async<T>(sK, PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 256);
     load_tile_async<T>(sQ, PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 256);
     load_tile_async<T>(sV, PV, (const T*)p.v + (t0 * p.H + h) * DV, (long long)p.H * DV, 64, DV, L, tid, 256);
@@ -261,22 +275,34 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     load_tile_async<T>(sE, PV, (const T*)p.Eb + idx * 64 * DV, DV, 64, DV, 64, tid, 256);
     load_tile_async<T>(sH, PK, (const T*)p.Hb + idx * DV * DK, DK, DV, DK, DV, tid, 256);
     load_tile_async<T>(sdH, PK, (const T*)p.dHb + idx * DV * DK, DK, DV, DK, DV, tid, 256);
-    // M and G are stored once per key head, at its first value head's unit
-    const long long kidx = (long long)slot * p.H + hk * p.vg;
     load_tile_async<T>(sM, PL, (const T*)p.Mb + kidx * 4096, 64, 64, 64, 64, tid, 256);
     cp_async_commit();
-    if (tid < 64) {
-        sG[tid] = p.Gb[kidx * 64 + tid];
-        sGm1[tid] = tid > 0 ? p.Gb[kidx * 64 + tid - 1] : 0.f;
-        const float be = tid < L ? p.beta[krow(p, t0 + tid, h)] : 0.f;
-        sBe[tid] = be;
-        const float al = tid < L ? p.alpha[krow(p, t0 + tid, h)] : 1.f;
-        const float fsc = feedback_scale(p.iplr, al);
-        sBt[tid] = bh * be * fsc;
-        sAl[tid] = al;
-        const float em1 = tid > 0 ? __expf(p.Gb[kidx * 64 + tid - 1]) : 1.f;
-        sEm1[tid] = em1;
-        sWs[tid] = bh * be * fsc * em1;
+    if constexpr (DK <= 128) {
+        if (tid < 64) {
+            sG[tid] = rg;
+            sGm1[tid] = rgm1;
+            sBe[tid] = rbe;
+            const float fsc = feedback_scale(p.iplr, ral);
+            sBt[tid] = bh * rbe * fsc;
+            sAl[tid] = ral;
+            const float em1 = tid > 0 ? __expf(rgm1) : 1.f;
+            sEm1[tid] = em1;
+            sWs[tid] = bh * rbe * fsc * em1;
+        }
+    } else {
+        if (tid < 64) {
+            sG[tid] = p.Gb[kidx * 64 + tid];
+            sGm1[tid] = tid > 0 ? p.Gb[kidx * 64 + tid - 1] : 0.f;
+            const float be = tid < L ? p.beta[krow(p, t0 + tid, h)] : 0.f;
+            sBe[tid] = be;
+            const float al = tid < L ? p.alpha[krow(p, t0 + tid, h)] : 1.f;
+            const float fsc = feedback_scale(p.iplr, al);
+            sBt[tid] = bh * be * fsc;
+            sAl[tid] = al;
+            const float em1 = tid > 0 ? __expf(p.Gb[kidx * 64 + tid - 1]) : 1.f;
+            sEm1[tid] = em1;
+            sWs[tid] = bh * be * fsc * em1;
+        }
     }
     cp_async_wait<0>();
     __syncthreads();

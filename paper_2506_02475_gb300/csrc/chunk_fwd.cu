@@ -338,7 +338,8 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     };
 
     const long long kr0 = t0 * Hk + hk, kld = (long long)Hk * DK;   // key-side rows
-    const float dh = p.d[hk];   // loaded ahead of the tiles' cp.async traffic
+    const float dh = p.d[hk];   // loaded ahead of the tiles' cp.async traffic, as are the log-decays
+    const float gv = tid < 64 ? p.Gb[idx0 * 64 + tid] : 0.f;
     load_tile_async<T>(sQ, S::PK, (const T*)p.q + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sK, S::PK, (const T*)p.k + kr0 * DK, kld, 64, DK, L, tid, 128);
     load_tile_async<T>(sW, S::PK, (const T*)p.Wb + idx0 * 64 * DK, DK, 64, DK, 64, tid, 128);
@@ -346,7 +347,7 @@ __global__ void __launch_bounds__(128) k_output(ChunkParams p) {
     cp_async_commit();
     if (vg > 1) load_vh(1);
     cp_async_commit();
-    if (tid < 64) sG[tid] = p.Gb[idx0 * 64 + tid];
+    if (tid < 64) sG[tid] = gv;
     cp_async_wait<1>();
     __syncthreads();
 
