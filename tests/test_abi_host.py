@@ -74,6 +74,20 @@ def test_workspace_size_counts_chunks_and_heads(L):
     assert ws(L, shape(B=1, T=65536, N=12, cu=FAKE)) > ws(L, shape(B=1, T=65536, N=1))
 
 
+def test_workspace_per_unit_on_the_tcgen05_path(L):
+    """bf16 dk = dv = 128, one (chunk, head) unit per 64 tokens: the forward keeps W^T, U^T,
+    U_s^T (16 KB each), the log-decays (256 B), Atilde and the chunk state H^T (32 KB each) per
+    unit, and no B^T (its scan forms B^T = U_s^T K itself); the backward adds E (16 KB), M
+    (8 KB), Z^T (16 KB, for the C term its scan forms), dH'^T (32 KB) and two per-unit floats,
+    and no C^T.  32 more units (and their 16-byte slot records) keep every sub-buffer a whole
+    number of 256-byte alignment steps, so the differences are exact."""
+    fwd_unit = 3 * 16384 + 256 + 2 * 32768
+    bwd_unit = fwd_unit + 16384 + 8192 + 16384 + 32768 + 8
+    for backward, unit in ((0, fwd_unit), (1, bwd_unit)):
+        d = ws(L, shape(B=1, T=64 * 64, H=1), backward) - ws(L, shape(B=1, T=64 * 32, H=1), backward)
+        assert d == 32 * (unit + 16), (backward, d)
+
+
 @pytest.mark.parametrize("kw", [dict(dk=96), dict(dv=192), dict(dv=256, dk=64), dict(dv=256, dtype=0), dict(dv=640),
                                 dict(chunk=32), dict(H=0), dict(B=0), dict(dtype=7),
                                 dict(B=2, N=3), dict(B=2, cu=FAKE, N=2), dict(T=-1), dict(cu=FAKE + 4, B=1, N=1)])
