@@ -12,7 +12,7 @@
  * the paper's recurrent listing does (appendix B.1).  Equivalently
  *     e_t = beta_t v_t - btilde_t H_{t-1}^T k_t,  H_t = alpha_t H_{t-1} + k_t e_t^T,
  *     o_t = H_t^T (q_t - d k_t).
- * There is no query scale.  Training uses the chunk-wise form of section 3.3
+ * There is no query scale.  Training uses the chunk-wise form of section 3.2
  * (WY representation with a single UT inverse per chunk, Eq. "prepare WY_M",
  * then the inter-chunk state and output equations); inference uses the
  * one-token recurrence.
@@ -221,7 +221,7 @@ comba_status_t comba_chunk_bwd_pk(const comba_shape_t *shape,
 size_t comba_workspace_size(const comba_shape_t *shape, int backward);
 
 /*
- * Chunk-parallel forward (section 3.3).  Per chunk of 64 tokens: the
+ * Chunk-parallel forward (section 3.2).  Per chunk of 64 tokens: the
  * decay-masked, btilde-scaled Gram matrix, its unit-lower-triangular inverse
  * M = (I + strict_lower(Diag(btilde)(A^{(i-1)/j} * K K^T)))^{-1}, the WY/UT
  * factors W = M Diag(btilde*gamma_{r-1}) K and U = M Diag(beta) V

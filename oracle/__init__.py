@@ -8,7 +8,7 @@ never calls the CUDA library.
 Eq. "comba-S"; feedback strength of section 3.1; recurrent listing of
 appendix B.1) in double precision, with exact back-propagation through time
 for the gradients.  ``chunked.py`` is a separate fp64 NumPy statement of the
-paper's chunk-wise algorithm (section 3.3: WY representation, UT transform,
+paper's chunk-wise algorithm (section 3.2: WY representation, UT transform,
 inter-chunk state and output equations); it is used only to pin the paper's
 chunk algebra against the recurrence.
 

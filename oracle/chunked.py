@@ -1,6 +1,6 @@
 """The paper's chunk-wise Comba algorithm in plain fp64 NumPy (test infrastructure only).
 
-Section 3.3 ("Comba with Chunk-wise Parallel") states the chunk form; this
+Section 3.2 ("Comba with Chunk-wise Parallel") states the chunk form; this
 module follows it step by step, in the paper's orientation S (dv x dk), so
 that tests can check that the paper's chunk equations, under this package's
 reading of their notation, reproduce the token recurrence of ``comba_oracle.c``.

@@ -1,6 +1,6 @@
 // Chunk-parallel Comba backward.  The paper prints no backward pass; these
 // kernels evaluate the exact chain-rule derivatives of the chunk form of
-// section 3.3 (Eq. "prepare WY_M", the inter-chunk state equation and the
+// section 3.2 (Eq. "prepare WY_M", the inter-chunk state equation and the
 // output equation), with chunk-local log-decays g_r = sum_{j<=r} log alpha_j.
 // With dH' = dL/dH at a chunk's end, P = Tril(Q~K^T * Gamma), Qhat =
 // Diag(gamma) Q~ and Kbar = Diag(gamma_C/gamma_r) K:

@@ -1,4 +1,4 @@
-// Chunk-parallel Comba forward (section 3.3 of the paper):
+// Chunk-parallel Comba forward (section 3.2 of the paper):
 //   k_chunk_map : chunk slots of (packed) sequences
 //   k_prep      : per chunk, the decay-masked btilde-scaled Gram matrix, its
 //                 UT inverse M, the WY factors W = M Diag(btilde gamma_{r-1}) K

@@ -1,6 +1,6 @@
 // Sequential inter-chunk scan, shared by the forward and the backward.
 //
-// Folding each chunk of section 3.3's state equation into one affine map,
+// Folding each chunk of section 3.2's state equation into one affine map,
 //     H_{n+1} = gamma_n H_n + Atilde_n H_n + B_n,
 //     Atilde_n = -Kbar_n^T W_n,  B_n = Kbar_n^T U_n,  gamma_n = gamma_C of chunk n,
 // leaves a single dense product on the sequential path.  The backward's

@@ -2,7 +2,7 @@
 //
 // At dk = 256 a chunk's folded map Atilde = -Kbar^T W is 256 x 256 (128 KB in
 // bf16): writing and reading it per (chunk, head) would cost twice W and K
-// together.  So this scan applies section 3.3's chunk equations directly, two
+// together.  So this scan applies section 3.2's chunk equations directly, two
 // products per chunk:
 //     forward:   E = U - W H,            H' = gamma_C H + Kbar^T E
 //     backward:  R = Kbar dH',           dH = gamma_C dH' + C - W^T R,   C = Z^T dO

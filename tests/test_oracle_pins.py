@@ -185,7 +185,7 @@ def test_transition_spectrum_and_state_norm_bound():
 
 @pytest.mark.parametrize("C", [1, 4, 16, 64])
 def test_paper_chunk_equations_equal_recurrence(C):
-    """Section 3.3: the WY/UT chunk form (single inverse M, W, U, inter-chunk state and
+    """Section 3.2: the WY/UT chunk form (single inverse M, W, U, inter-chunk state and
     output equations) under the stated readings reproduces the token recurrence,
     including short last chunks and several packed sequences."""
     rng = np.random.default_rng(7)
