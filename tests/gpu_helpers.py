@@ -1,21 +1,21 @@
 """Helpers shared by the GPU parity tests: move a seeded workload to the GPU,
 run the library through its binding, and compare with the fp64 oracle.
 
-Error metric (per output tensor): max-norm relative error
+Error metric (per output tensor, every tensor alike): max-norm relative error
     rel = max_i |x_i - r_i| / max_i |r_i|.
 Tolerances: 1e-4 for the fp32 storage path, 2e-2 for bf16 storage with fp32
 state and accumulation.
 
-The per-head parameter gradients db and dd are sums over every token of the
-batch of per-token contributions c_t (dd: -k_t . dq~_t, from the output
-correction q~ = q - d k; db: beta_t dbtilde_t, from btilde = b beta).  Their
-error is measured on the scale of that sum, max_h |x_h - r_h| / sum_t |c_t|:
-the bound a sum meets when each contribution meets the tolerance.  The plain
-relative error of such a sum is ill-conditioned (at the 340M layer shape the
-sum is about 1/4000 of sum_t |c_t|).  The contributions come from the
-oracle's outputs alone: c_t(dd) = -k_t . dq_t, and
-c_t(db) = (beta_t dbeta_t - v_t . dv_t) / b, since dbeta = v . de + b dbtilde
-and dv = beta de.
+The per-head parameter gradients db and dd are tensors [H] like any other and
+take the same metric over their heads.  Each head's value is a sum over every
+token of the batch of per-token contributions c_t (dd: -k_t . dq~_t, from the
+output correction q~ = q - d k; db: beta_t dbtilde_t, from btilde = b beta),
+and a head whose sum happens to cancel to near zero has a large error of its
+own (its elementwise relative error), the same as a near-zero element of any
+other tensor.  `param_grad_report` gives those per-head figures and the error
+on the scale sum_t |c_t| of the contributions, for reporting next to the
+metric: c_t(dd) = -k_t . dq_t, c_t(db) = (beta_t dbeta_t - v_t . dv_t) / b,
+both from the oracle's outputs alone (dbeta = v . de + b dbtilde, dv = beta de).
 """
 import numpy as np
 import torch
@@ -52,10 +52,21 @@ def rel_sum(x, ref, scale):
     return float(np.max(np.abs(x - ref) / np.maximum(scale, 1e-300)))
 
 
-def param_grad_errors(g, ref, k, v, beta, b):
-    """dd and db errors on the summation scale."""
+def param_grad_errors(g, ref):
+    """dd and db: the max-norm relative error over their heads, as for every tensor."""
+    return {key: rel(g[key], ref[key]) for key in ("dd", "db")}
+
+
+def param_grad_report(g, ref, k, v, beta, b):
+    """Context for dd and db (not a bound): the worst per-head relative error, and the error
+    on the summation scale sum_t |c_t|."""
     sc = param_grad_scales(k, v, beta, b, ref)
-    return {key: rel_sum(g[key], ref[key], sc[key]) for key in ("dd", "db")}
+    out = {}
+    for key in ("dd", "db"):
+        x, r = (np.asarray(a, np.float64).reshape(-1) for a in (g[key], ref[key]))
+        out[key + "_per_head_max"] = float(np.max(np.abs(x - r) / np.maximum(np.abs(r), 1e-300)))
+        out[key + "_sum_scale"] = rel_sum(x, r, sc[key])
+    return out
 
 
 def tol(dtype):

@@ -4,14 +4,14 @@ Every comparison runs the CUDA library through its C ABI (ctypes binding) on
 seeded synthetic inputs and the oracle on the very same values.  Small cases
 span several 64-token chunks with ragged tails; the full-size workloads run
 the whole problem on the GPU exactly as the benchmark does, and are compared
-on every (sequence) unit of sampled heads, which the oracle can afford.
+on every sequence and head (the oracle takes seconds on a many-core host).
 """
 import numpy as np
 import pytest
 import torch
 
 import oracle
-from gpu_helpers import np64, param_grad_errors, rel, to_dev, tol
+from gpu_helpers import np64, param_grad_errors, param_grad_report, rel, to_dev, tol
 from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, inputs
 
 pytestmark = pytest.mark.gpu
@@ -49,9 +49,9 @@ def check_bwd(w, t=None):
     g = gpu_bwd(t)
     r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens)
     errs = {key: rel(g[key], r[key]) for key in GRADS}
-    errs.update(param_grad_errors(g, r, w.k, w.v, w.beta, w.b))
+    errs.update(param_grad_errors(g, r))
     bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
-    assert not bad, (bad, errs)
+    assert not bad, (bad, errs, param_grad_report(g, r, w.k, w.v, w.beta, w.b))
     return errs
 
 
@@ -157,27 +157,13 @@ def test_backward_is_bitwise_deterministic():
     assert np.array_equal(o1, o2) and np.array_equal(h1, h2)
 
 
-def _head_slice(w, h):
-    """The workload restricted to head h (every sequence), for the oracle."""
-    def tok(x):
-        return None if x is None else np.ascontiguousarray(x[..., h:h + 1, :])
-
-    def gate(x):
-        return np.ascontiguousarray(x[..., h:h + 1])
-
-    def st(x):
-        return None if x is None else np.ascontiguousarray(x[:, h:h + 1])
-
-    return dict(q=tok(w.q), k=tok(w.k), v=tok(w.v), alpha=gate(w.alpha), beta=gate(w.beta),
-                b=None if w.b is None else w.b[h:h + 1], d=w.d[h:h + 1], h0=st(w.h0), dO=tok(w.dO), dhT=st(w.dhT),
-                cu_seqlens=w.cu_seqlens)
-
-
-@pytest.mark.parametrize("name,heads", [("lm340m", [0, 7]), ("lm1p3b", [0, 15]), ("varlen64k", [5])])
-def test_full_size_workload_sampled_heads(name, heads):
+@pytest.mark.parametrize("name", ["lm340m", "lm1p3b", "varlen64k"])
+def test_full_size_workload(name):
     """The full workload on the GPU in the benchmark's launch configuration (forward
-    saving its factors, backward reusing them); every sequence of the sampled heads
-    against the oracle, forward and backward."""
+    saving its factors, backward reusing them), every output against the oracle over
+    the whole workload (every sequence and head), forward and backward.  dd and db are
+    checked over all their heads like every other tensor; their per-head figures are
+    printed for context."""
     from paper_2506_02475_gb300 import comba_workspace_size
     w = inputs.make(name)
     t = to_dev(w)
@@ -188,24 +174,19 @@ def test_full_size_workload_sampled_heads(name, heads):
     g = comba_chunk_bwd(t["q"], t["k"], t["v"], t["alpha"], t["beta"], t["d"], t["dO"], b=t["b"], h0=t["h0"],
                         dhT=t["dhT"], cu_seqlens=t["cu_seqlens"], workspace=ws, reuse_factors=True)
     torch.cuda.synchronize()
-    for h in heads:
-        s = _head_slice(w, h)
-        ro, rhT = oracle.fwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], h0=s["h0"],
-                             cu_seqlens=s["cu_seqlens"])
-        assert rel(np64(o[..., h:h + 1, :]), ro) <= tol(w.dtype)
-        assert rel(np64(hT[:, h:h + 1]), rhT) <= tol(w.dtype)
-        r = oracle.bwd(s["q"], s["k"], s["v"], s["alpha"], s["beta"], s["b"], s["d"], s["dO"], h0=s["h0"],
-                       dhT=s["dhT"], cu_seqlens=s["cu_seqlens"])
-        errs = {}
-        for key in ("dq", "dk", "dv"):
-            errs[key] = rel(np64(g[key][..., h:h + 1, :]), r[key])
-        for key in ("dalpha", "dbeta"):
-            errs[key] = rel(np64(g[key][..., h:h + 1]), r[key])
-        errs["dh0"] = rel(np64(g["dh0"][:, h:h + 1]), r["dh0"])
-        errs.update(param_grad_errors({"dd": np64(g["dd"][h:h + 1]), "db": np64(g["db"][h:h + 1])}, r,
-                                      s["k"], s["v"], s["beta"], s["b"]))
-        bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
-        assert not bad, (name, h, bad, errs)
+    g = {key: np64(val) for key, val in g.items()}
+    o, hT = np64(o), np64(hT)
+    del t, ws
+    ro, rhT = oracle.fwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0, cu_seqlens=w.cu_seqlens)
+    errs = {"o": rel(o, ro), "hT": rel(hT, rhT)}
+    del ro, rhT
+    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens)
+    errs.update({key: rel(g[key], r[key]) for key in GRADS})
+    errs.update(param_grad_errors(g, r))
+    ctx = param_grad_report(g, r, w.k, w.v, w.beta, w.b)
+    print(name, {k_: f"{e:.2e}" for k_, e in errs.items()}, "context:", {k_: f"{e:.2e}" for k_, e in ctx.items()})
+    bad = {k_: e for k_, e in errs.items() if not e <= tol(w.dtype)}
+    assert not bad, (name, bad, errs, ctx)
 
 
 @pytest.mark.parametrize("dtype,d,lens", [("bf16", 128, None), ("f32", 64, None), ("bf16", 64, [70, 0, 129, 5])])
@@ -232,7 +213,7 @@ def test_backward_reusing_saved_forward_factors(dtype, d, lens):
     r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens)
     for key in GRADS:
         assert rel(g[key], r[key]) <= tol(w.dtype), key
-    for key, e in param_grad_errors(g, r, w.k, w.v, w.beta, w.b).items():
+    for key, e in param_grad_errors(g, r).items():
         assert e <= tol(w.dtype), key
 
 
@@ -263,9 +244,7 @@ def test_iplr_variant_forward_backward(dtype, d, lens):
     for key in GRADS:
         assert np.array_equal(gn[key], np64(g2[key])), key          # reuse == recompute, bitwise
         assert rel(gn[key], r[key]) <= tol(dtype), (key, rel(gn[key], r[key]))
-    # db, dd on their summation scale: with btilde' = 2 alpha b beta, (beta dbeta - v.dv) / b is still
-    # the per-token contribution beta dbtilde' (2 alpha)
-    for key, e in param_grad_errors(gn, r, w.k, w.v, w.beta, w.b).items():
+    for key, e in param_grad_errors(gn, r).items():
         assert e <= tol(dtype), (key, e)
     # and it is not the SPLR result
     ro_s, _ = oracle.fwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0, cu_seqlens=w.cu_seqlens)

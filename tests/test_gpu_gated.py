@@ -5,8 +5,7 @@ import numpy as np
 import pytest
 import torch
 
-import oracle
-from gpu_helpers import np64, rel, rel_sum, tol
+from gpu_helpers import np64, rel, tol
 from oracle import gated
 from paper_2506_02475_gb300 import comba_chunk_bwd_gated, comba_chunk_fwd_gated, inputs
 
@@ -51,22 +50,6 @@ def _run(w, variant):
     return np64(o), np64(hT), g
 
 
-def _head(w, h):
-    """The raw workload restricted to head h (every sequence), for the oracle."""
-    def tok(x):
-        return None if x is None else np.ascontiguousarray(x[..., h:h + 1, :])
-
-    def gate(x):
-        return np.ascontiguousarray(x[..., h:h + 1])
-
-    def st(x):
-        return None if x is None else np.ascontiguousarray(x[:, h:h + 1])
-
-    return inputs.GatedWorkload(dtype=w.dtype, q=tok(w.q), k=tok(w.k), v=tok(w.v), g_alpha=gate(w.g_alpha),
-                                g_beta=gate(w.g_beta), a=w.a[h:h + 1], c=w.c[h:h + 1], b_raw=w.b_raw[h:h + 1],
-                                d=w.d[h:h + 1], h0=st(w.h0), dO=tok(w.dO), dhT=st(w.dhT), cu_seqlens=w.cu_seqlens)
-
-
 def _check(w, variant, o, hT, g):
     """Every output against the oracle composition on w (all of its heads)."""
     raw = (w.q, w.k, w.v, w.g_alpha, w.g_beta, w.a, w.c, w.b_raw, w.d)
@@ -76,23 +59,12 @@ def _check(w, variant, o, hT, g):
     errs = {"o": rel(o, ro), "hT": rel(hT, rhT)}
     for key in ("dq", "dk", "dv", "dg_alpha", "dg_beta", "dh0"):
         errs[key] = rel(g[key], r[key])
-    # per-head sums on the scale of their per-token contributions, all from the oracle
-    qh, kh, al, be, b = gated.prologue(w.q, w.k, w.g_alpha, w.g_beta, w.a, w.c, w.b_raw)
-    inner = oracle.bwd(qh, kh, w.v, al, be, b, w.d, w.dO, h0=w.h0, dhT=w.dhT, cu_seqlens=w.cu_seqlens,
-                       variant=variant)
-    z = w.g_alpha.astype(np.float64) + w.c
-    H = w.g_alpha.shape[-1]
-    scale = {
-        "da": np.abs(inner["dalpha"] * al * gated.softplus(z)).reshape(-1, H).sum(0),
-        "dc": np.abs(r["dg_alpha"]).reshape(-1, H).sum(0),
-        "dd": np.abs(np.einsum("...hd,...hd->...h", kh, inner["dq"])).reshape(-1, H).sum(0),
-        "db_raw": (np.abs(be * inner["dbeta"] - np.einsum("...hd,...hd->...h", w.v, inner["dv"])).reshape(-1, H)
-                   .sum(0) * (1.0 - b)),
-    }
-    for key, sc in scale.items():
-        errs[key] = rel_sum(g[key], r[key], sc)
+    # the per-head parameter gradients take the max-norm error over their heads like every tensor
+    for key in ("da", "dc", "dd", "db_raw"):
+        errs[key] = rel(g[key], r[key])
     bad = {key: e for key, e in errs.items() if not e <= tl}
     assert not bad, (bad, errs)
+    return errs
 
 
 @pytest.mark.parametrize("dtype,d,dv,lens,variant", [("bf16", 128, 128, [130, 0, 257, 64], "splr"),
@@ -113,14 +85,9 @@ def test_gated_many_heads():
     _check(w, "splr", *_run(w, "splr"))
 
 
-def test_gated_full_size_sampled_heads():
+def test_gated_full_size():
     """B=4 T=4096 H=16 d=128 bf16 (the gated benchmark's shape and launch configuration):
-    every sequence of two sampled heads against the oracle, forward and backward."""
+    every output against the oracle over the whole workload, forward and backward."""
     w = inputs.make_gated(B=4, T=4096, H=16, dk=128, dv=128, dtype="bf16")
     o, hT, g = _run(w, "splr")
-    for h in (0, 15):
-        sl = lambda x: x[..., h:h + 1, :]
-        gs = {key: (g[key][..., h:h + 1, :] if g[key].ndim == 4 and key != "dh0" else
-                    g[key][:, h:h + 1] if key == "dh0" else
-                    g[key][..., h:h + 1] if g[key].ndim == 3 else g[key][h:h + 1]) for key in g}
-        _check(_head(w, h), "splr", sl(o), hT[:, h:h + 1], gs)
+    print("gated lm1p3b", {k_: f"{e:.2e}" for k_, e in _check(w, "splr", o, hT, g).items()})

@@ -1,13 +1,13 @@
 """GPU parity of the Comba-pk form (appendix B.3; comba_chunk_fwd_pk / _bwd_pk /
 comba_recurrent_step_pk) against the oracle with feedback vectors p: x = H^T p, e = beta v -
-btilde x, H <- alpha H + k e^T, o = H^T (q - d p).  dd and db are compared on the scale of
-their per-token contributions (dd: -p . dq)."""
+btilde x, H <- alpha H + k e^T, o = H^T (q - d p).  dd and db take the max-norm relative
+error over their heads like every other tensor."""
 import numpy as np
 import pytest
 import torch
 
 import oracle
-from gpu_helpers import np64, param_grad_errors, rel, tol, to_dev
+from gpu_helpers import np64, param_grad_errors, param_grad_report, rel, tol, to_dev
 from paper_2506_02475_gb300 import (comba_chunk_bwd_pk, comba_chunk_fwd_pk, comba_recurrent_step_pk,
                                     comba_workspace_size, inputs)
 from paper_2506_02475_gb300 import binding
@@ -58,11 +58,12 @@ def _check(w, p, o, hT, g, variant="splr", heads=None):
     for key in ("dalpha", "dbeta"):
         errs[key] = rel(sl(g[key], -1), r[key])
     errs["dh0"] = rel(sl(g["dh0"], 1), r["dh0"])
-    # dd sums -p . dq over tokens: its scale takes p where the plain form takes k
-    errs.update(param_grad_errors({"dd": sl(g["dd"], 0), "db": sl(g["db"], 0)}, r, ref_in["p"], ref_in["v"],
-                                  ref_in["beta"], ref_in["b"]))
+    gp = {"dd": sl(g["dd"], 0), "db": sl(g["db"], 0)}
+    errs.update(param_grad_errors(gp, r))
     bad = {key: e for key, e in errs.items() if not e <= tl}
-    assert not bad, (bad, errs)
+    # context for dd (a sum of -p . dq over tokens: its scale takes p where the plain form takes k)
+    assert not bad, (bad, errs, param_grad_report(gp, r, ref_in["p"], ref_in["v"], ref_in["beta"], ref_in["b"]))
+    return errs
 
 
 CASES = [
@@ -109,14 +110,15 @@ def test_pk_with_p_equal_to_k_matches_the_plain_form_on_the_gpu():
         assert rel(g[key], np64(g0[key])) <= tl, key
 
 
-def test_pk_full_size_sampled_heads():
-    """B=4 T=4096 H=16 d=128 bf16 in the benchmark's configuration; heads 0 and 15, every
-    sequence, forward and backward against the oracle."""
+def test_pk_full_size():
+    """B=4 T=4096 H=16 d=128 bf16 in the benchmark's configuration; every output against the
+    oracle over the whole workload, forward and backward."""
     w = inputs.make("lm1p3b")
     p, tp = _with_p(w, seed=0)
     t = to_dev(w)
     o, hT, g = _run(w, t, tp)
-    _check(w, p, o, hT, g, heads=[0, 15])
+    del t, tp
+    print("lm1p3b pk", {k_: f"{e:.2e}" for k_, e in _check(w, p, o, hT, g).items()})
 
 
 @pytest.mark.parametrize("dtype,iplr,dk,dv", [("bf16", False, 128, 128), ("f32", True, 128, 128),

@@ -6,7 +6,7 @@ import pytest
 import torch
 
 import oracle
-from gpu_helpers import np64, param_grad_errors, rel, tol, to_dev
+from gpu_helpers import np64, param_grad_errors, param_grad_report, rel, tol, to_dev
 from paper_2506_02475_gb300 import comba_chunk_bwd, comba_chunk_fwd, comba_recurrent_step, comba_workspace_size, inputs
 from test_gpu_chunk import GRADS, check_bwd, check_fwd
 
@@ -17,8 +17,10 @@ pytestmark = pytest.mark.gpu
                                             (192, 1, None, [1, 63, 64, 65, 0, 200, 7]),
                                             (256, 1, None, [129, 3, 64])])
 def test_head_dim_256_forward_backward(dv, B, T, lengths):
+    # four heads: the per-head sums db and dd are checked with the max-norm over their heads, which
+    # over two heads of a few hundred tokens rests on two sums that may both nearly cancel
     kw = dict(lengths=lengths) if lengths else dict(B=B, T=T)
-    w = inputs.make("custom", H=2, dk=256, dv=dv, dtype="bf16", with_b=True, with_h0=True, with_grads=True,
+    w = inputs.make("custom", H=4, dk=256, dv=dv, dtype="bf16", with_b=True, with_h0=True, with_grads=True,
                     seed_offset=dv + (len(lengths) if lengths else T), **kw)
     t = to_dev(w)
     check_fwd(w, t)
@@ -39,7 +41,7 @@ def test_head_dim_256_iplr():
     g = {key: np64(val) for key, val in g.items()}
     errs = {"o": rel(np64(o), ro), "hT": rel(np64(hT), rhT)}
     errs.update({key: rel(g[key], r[key]) for key in GRADS})
-    errs.update(param_grad_errors(g, r, w.k, w.v, w.beta, w.b))
+    errs.update(param_grad_errors(g, r))
     bad = {key: e for key, e in errs.items() if not e <= tol("bf16")}
     assert not bad, (bad, errs)
 
@@ -68,9 +70,9 @@ def test_head_dim_256_reuse_equals_recompute():
         assert np.array_equal(np64(g1[key]), np64(g2[key])), key
 
 
-def test_head_dim_256_full_size_sampled_heads():
+def test_head_dim_256_full_size():
     """B=4 T=4096 H=8 dk=dv=256 (the head-dim-256 benchmark shape) in the benchmark's
-    configuration; heads 0 and 7 (every sequence) against the oracle."""
+    configuration; every output against the oracle over the whole workload."""
     w = inputs.make("lm1p3b_d256")
     t = to_dev(w)
     ws = torch.empty(comba_workspace_size(t["q"], t["v"], None, backward=True), dtype=torch.uint8, device="cuda")
@@ -78,24 +80,19 @@ def test_head_dim_256_full_size_sampled_heads():
     o, hT = comba_chunk_fwd(*args, b=t["b"], h0=t["h0"], output_final_state=True, workspace=ws, save_factors=True)
     g = comba_chunk_bwd(*args, t["dO"], b=t["b"], h0=t["h0"], dhT=t["dhT"], workspace=ws, reuse_factors=True)
     torch.cuda.synchronize()
-    for h in (0, 7):
-        sl = lambda x: np.ascontiguousarray(x[..., h:h + 1, :])
-        sg = lambda x: np.ascontiguousarray(x[..., h:h + 1])
-        st = lambda x: None if x is None else np.ascontiguousarray(x[:, h:h + 1])
-        bh = None if w.b is None else w.b[h:h + 1]
-        ro, rhT = oracle.fwd(sl(w.q), sl(w.k), sl(w.v), sg(w.alpha), sg(w.beta), bh, w.d[h:h + 1], h0=st(w.h0))
-        r = oracle.bwd(sl(w.q), sl(w.k), sl(w.v), sg(w.alpha), sg(w.beta), bh, w.d[h:h + 1], sl(w.dO),
-                       h0=st(w.h0), dhT=st(w.dhT))
-        errs = {"o": rel(np64(o[..., h:h + 1, :]), ro), "hT": rel(np64(hT[:, h:h + 1]), rhT)}
-        for key in ("dq", "dk", "dv"):
-            errs[key] = rel(np64(g[key][..., h:h + 1, :]), r[key])
-        for key in ("dalpha", "dbeta"):
-            errs[key] = rel(np64(g[key][..., h:h + 1]), r[key])
-        errs["dh0"] = rel(np64(g["dh0"][:, h:h + 1]), r["dh0"])
-        errs.update(param_grad_errors({"dd": np64(g["dd"][h:h + 1]), "db": np64(g["db"][h:h + 1])}, r, sl(w.k),
-                                      sl(w.v), sg(w.beta), bh))
-        bad = {key: e for key, e in errs.items() if not e <= tol("bf16")}
-        assert not bad, (h, bad, errs)
+    g = {key: np64(val) for key, val in g.items()}
+    o, hT = np64(o), np64(hT)
+    del t, ws
+    ro, rhT = oracle.fwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, h0=w.h0)
+    errs = {"o": rel(o, ro), "hT": rel(hT, rhT)}
+    del ro, rhT
+    r = oracle.bwd(w.q, w.k, w.v, w.alpha, w.beta, w.b, w.d, w.dO, h0=w.h0, dhT=w.dhT)
+    errs.update({key: rel(g[key], r[key]) for key in GRADS})
+    errs.update(param_grad_errors(g, r))
+    ctx = param_grad_report(g, r, w.k, w.v, w.beta, w.b)
+    print("lm1p3b_d256", {k_: f"{e:.2e}" for k_, e in errs.items()}, "context:", {k_: f"{e:.2e}" for k_, e in ctx.items()})
+    bad = {key: e for key, e in errs.items() if not e <= tol("bf16")}
+    assert not bad, (bad, errs, ctx)
 
 
 @pytest.mark.parametrize("dtype,dv", [("bf16", 256), ("bf16", 64), ("f32", 128)])
