@@ -67,7 +67,7 @@ typedef enum {
     COMBA_ERR_UNSUPPORTED = 2,  /* valid but not implemented (head dim, chunk size) */
     COMBA_ERR_WORKSPACE = 3,    /* workspace NULL or smaller than required         */
     COMBA_ERR_CUDA = 4,         /* a CUDA launch or query failed                    */
-    COMBA_ERR_TIMEOUT = 5       /* reserved: a bounded device-side wait gave up     */
+    COMBA_ERR_TIMEOUT = 5       /* a device-side wait gave up (comba_workspace_status) */
 } comba_status_t;
 
 typedef enum { COMBA_F32 = 0, COMBA_BF16 = 1 } comba_dtype_t;
@@ -95,6 +95,14 @@ typedef struct {
      * it).  Fewer handles than needed is COMBA_ERR_INVALID_ARG. */
     void **stage_events;
     int num_stage_events;
+    /* Limit of each device-side wait of the call's kernels (tensor-core
+     * completion, TMA arrival), in nanoseconds of the GPU's global timer;
+     * 0 = the default of one second; values above 4e9 count as 4e9.  A wait
+     * that runs past it gives up: the kernel lets its copies and products in
+     * flight land, skips the rest of its work, marks the workspace's status
+     * word and returns (see comba_workspace_status).  The outputs of such a
+     * call are then incomplete. */
+    unsigned int wait_limit_ns;
 } comba_shape_t;
 
 #define COMBA_FWD_EVENTS 5
@@ -185,6 +193,18 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t *shape,
  * the mma.sync one for every shape.
  */
 #define COMBA_PK 16
+
+/*
+ * Diagnostic flag of comba_chunk_fwd and comba_chunk_bwd (bf16, dk = dv = 128,
+ * the tcgen05 kernels): the first tensor-core completion wait of every CTA of
+ * the prep, output and local-gradient kernels waits on a barrier that nothing
+ * arrives at, so it runs out after shape->wait_limit_ns.  The kernel then lets
+ * its products land, skips its work and marks the workspace's status word, so
+ * that a test can watch a device-side timeout reach the host
+ * (comba_workspace_status) without faulting or hanging the GPU.  The call's
+ * outputs are then meaningless.  Not for production use.
+ */
+#define COMBA_DIAG_STALL 32
 
 /*
  * The pk forward: as comba_chunk_fwd plus p [B,T,H,dk] (storage type, required).
@@ -305,17 +325,19 @@ comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtyp
  * device memory (e.g. code running inside a framework's execute step that
  * forbids allocation, or a latency-critical loop that must not reach an
  * allocator).  The paper has no counterpart; this is a deployment variant of
- * comba_chunk_fwd with identical arguments minus the workspace and identical
- * results.
+ * comba_chunk_fwd with the same arguments minus the workspace, and bitwise
+ * the same o and hT.  shape->flags may be 0 or COMBA_IPLR; any other flag
+ * (saved factors, the gated or pk forms) returns COMBA_ERR_INVALID_ARG.
  *
  * Scratch comes from one file-scope device array of COMBA_STATIC_SCRATCH_BYTES
  * that every GPU loading this library holds until the process exits.  Shapes
  * whose comba_workspace_size(shape, 0) exceeds it return COMBA_ERR_WORKSPACE
- * without launching anything.  The first call on a device looks up the
- * array's device address (with that device current); make that first call
- * before any stream capture.  All calls share the array: calls whose kernels
- * may overlap on the GPU race on it and must be serialised by the caller.
- * Nothing in it needs to start zeroed.  No allocation is made.
+ * without launching anything.  Each call looks up the array's device address
+ * on the current device (cudaGetSymbolAddress); the first call on a device
+ * also loads the library's device code there, so make it before any stream
+ * capture.  All calls share the array: calls whose kernels may overlap on
+ * the GPU race on it and must be serialised by the caller.  Nothing in it
+ * needs to start zeroed.  No allocation is made.
  */
 #define COMBA_STATIC_SCRATCH_BYTES (32u << 20)
 comba_status_t comba_chunk_fwd_noalloc(const comba_shape_t *shape,
@@ -323,6 +345,22 @@ comba_status_t comba_chunk_fwd_noalloc(const comba_shape_t *shape,
                                        const float *alpha, const float *beta,
                                        const float *b, const float *d, const float *h0,
                                        void *o, float *hT, void *stream);
+
+/*
+ * Status of the device-side waits of the calls that last used `workspace`.
+ * Every kernel wait is bounded in time (comba_shape_t.wait_limit_ns); a wait
+ * that gives up sets the status word in the workspace's first 4 bytes.  The
+ * word is cleared by the first kernel of every forward call and of every
+ * backward call that recomputes the forward's factors; a backward that reuses
+ * saved factors adds to what its forward set.  This call waits for `stream`
+ * (cudaStreamSynchronize), copies the word back with one cudaMemcpyAsync into
+ * a host variable, and returns COMBA_ERR_TIMEOUT when it is set, COMBA_OK when
+ * it is clear, COMBA_ERR_CUDA when the stream or the copy failed.  The word is
+ * left as it is.  `workspace` NULL reads the word of the static scratch of
+ * comba_chunk_fwd_noalloc on the current device.  Nothing is allocated.
+ * (No counterpart in the paper: the hot-path boundary's error reporting.)
+ */
+comba_status_t comba_workspace_status(const void *workspace, void *stream);
 
 /* Static, human-readable name of a status code. */
 const char *comba_status_string(comba_status_t status);

@@ -16,6 +16,7 @@ from .binding import (  # noqa: F401
     comba_recurrent_step,
     comba_recurrent_step_pk,
     comba_workspace_size,
+    comba_workspace_status,
     lib,
     library_path,
 )

@@ -22,6 +22,7 @@ _lock = threading.Lock()
 
 COMBA_F32, COMBA_BF16 = 0, 1
 COMBA_SAVE_FACTORS, COMBA_REUSE_FACTORS, COMBA_IPLR, COMBA_GATED, COMBA_PK = 1, 2, 4, 8, 16
+COMBA_ERR_TIMEOUT = 5
 _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "workspace missing or too small",
            4: "CUDA error", 5: "device-side wait timed out"}
 
@@ -37,7 +38,7 @@ class _Shape(ctypes.Structure):
                 ("dv", ctypes.c_int), ("num_seqs", ctypes.c_int), ("cu_seqlens", ctypes.c_void_p),
                 ("dtype", ctypes.c_int), ("chunk", ctypes.c_int), ("flags", ctypes.c_int),
                 ("stage_events", ctypes.c_void_p),
-                ("num_stage_events", ctypes.c_int)]
+                ("num_stage_events", ctypes.c_int), ("wait_limit_ns", ctypes.c_uint)]
 
 
 def library_path() -> str:
@@ -74,6 +75,8 @@ def lib():
         L.comba_chunk_bwd_pk.restype = I
         L.comba_recurrent_step_pk.argtypes = [I, I, I, I, I] + [P] * 10 + [I, P]
         L.comba_recurrent_step_pk.restype = I
+        L.comba_workspace_status.argtypes = [P, P]
+        L.comba_workspace_status.restype = I
         L.comba_status_string.argtypes = [I]
         L.comba_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -112,11 +115,12 @@ def _check(name, t, dtype=None, shape=None, device=None):
         raise ValueError(f"{name} is on {t.device}, expected {device}")
 
 
-def make_shape(q, v, cu_seqlens=None, stage_events=None, flags=0):
+def make_shape(q, v, cu_seqlens=None, stage_events=None, flags=0, wait_limit_ns=0):
     """Build the C shape struct from q [B,T,H,dk] (or packed [Ttot,H,dk]) and v.
 
     ``stage_events`` (optional): sequence of raw cudaEvent_t handles (ints) recorded at
-    kernel boundaries (instrumentation; see include/comba.h)."""
+    kernel boundaries (instrumentation; see include/comba.h).  ``wait_limit_ns``: limit of
+    each device-side wait in nanoseconds (0: the library's default of one second)."""
     if q.dim() == 3:
         q = q.unsqueeze(0)
         v = v.unsqueeze(0)
@@ -133,6 +137,7 @@ def make_shape(q, v, cu_seqlens=None, stage_events=None, flags=0):
     s.dtype = _dtype_code(q)
     s.chunk = 64
     s.flags = flags
+    s.wait_limit_ns = wait_limit_ns
     if stage_events is not None:
         arr = (ctypes.c_void_p * len(stage_events))(*stage_events)
         s._events_keepalive = arr
@@ -179,7 +184,7 @@ def _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens):
 
 def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, output_final_state=False,
                     o=None, hT=None, workspace=None, stream=None, stage_events=None, save_factors=False,
-                    iplr=False):
+                    iplr=False, wait_limit_ns=0):
     """Chunk-parallel forward.  Returns ``(o, hT)`` (``hT`` is None unless requested).
 
     ``save_factors=True`` keeps the backward's chunk factors in ``workspace`` (which must
@@ -188,7 +193,7 @@ def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, o
     transition alpha (I - 2 btilde k k^T)."""
     N, H, dk, dv = _check_inputs(q, k, v, alpha, beta, b, d, h0, cu_seqlens)
     shape = make_shape(q, v, cu_seqlens, stage_events,
-                       (COMBA_SAVE_FACTORS if save_factors else 0) | (COMBA_IPLR if iplr else 0))
+                       (COMBA_SAVE_FACTORS if save_factors else 0) | (COMBA_IPLR if iplr else 0), wait_limit_ns)
     L = lib()
     nbytes = L.comba_workspace_size(ctypes.byref(shape), 1 if save_factors else 0)
     if nbytes == 0:
@@ -208,7 +213,7 @@ def comba_chunk_fwd(q, k, v, alpha, beta, d, b=None, h0=None, cu_seqlens=None, o
 
 def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_seqlens=None, want_dh0=True,
                     want_db=True, out=None, workspace=None, stream=None, stage_events=None, reuse_factors=False,
-                    iplr=False):
+                    iplr=False, wait_limit_ns=0):
     """Chunk-parallel backward.  Returns a dict with dq, dk, dv, dalpha, dbeta, dd, db, dh0.
 
     ``reuse_factors=True`` requires ``workspace`` to hold the factors of a
@@ -219,7 +224,7 @@ def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_s
     if reuse_factors and workspace is None:
         raise ValueError("reuse_factors=True needs the workspace of the saving forward call")
     shape = make_shape(q, v, cu_seqlens, stage_events,
-                       (COMBA_REUSE_FACTORS if reuse_factors else 0) | (COMBA_IPLR if iplr else 0))
+                       (COMBA_REUSE_FACTORS if reuse_factors else 0) | (COMBA_IPLR if iplr else 0), wait_limit_ns)
     L = lib()
     nbytes = L.comba_workspace_size(ctypes.byref(shape), 1)
     if nbytes == 0:
@@ -243,6 +248,16 @@ def comba_chunk_bwd(q, k, v, alpha, beta, d, dO, b=None, h0=None, dhT=None, cu_s
     if st != 0:
         raise CombaError("comba_chunk_bwd", st)
     return g
+
+
+def comba_workspace_status(workspace=None, stream=None) -> int:
+    """Status word of the calls that last used ``workspace`` (None: the static scratch of the
+    allocation-free forward): 0 (COMBA_OK), or 5 (COMBA_ERR_TIMEOUT) when a device-side wait of
+    one of their kernels gave up.  Waits for ``stream`` first."""
+    st = lib().comba_workspace_status(_ptr(workspace), _stream(stream))
+    if st not in (0, COMBA_ERR_TIMEOUT):
+        raise CombaError("comba_workspace_status", st)
+    return st
 
 
 def comba_recurrent_step(q, k, v, alpha, beta, d, state, b=None, o=None, stream=None, iplr=False):

@@ -177,9 +177,12 @@ void fill_common(ChunkParams& p, const comba_shape_t* s, const Layout& L, void* 
     p.cu = s->cu_seqlens;
     p.slots = L.slots;
     p.iplr = (s->flags & COMBA_IPLR) != 0;
+    p.stall = (s->flags & COMBA_DIAG_STALL) != 0;
     p.ev = reinterpret_cast<cudaEvent_t*>(s->stage_events);
     p.nev = s->stage_events ? s->num_stage_events : 0;
     p.err = reinterpret_cast<int*>(w + L.err);
+    const uint32_t lim = s->wait_limit_ns ? s->wait_limit_ns : comba::kDefaultWaitNs;
+    p.wait_ns = lim < comba::kMaxWaitNs ? lim : comba::kMaxWaitNs;
     p.slot_info = reinterpret_cast<comba::SlotInfo*>(w + L.slot_info);
     p.seq_first = reinterpret_cast<int*>(w + L.seq_first);
     p.Wb = w + L.W;
@@ -230,6 +233,21 @@ size_t comba_workspace_size(const comba_shape_t* shape, int backward) {
     Layout L;
     if (plan(shape, backward, &L) != COMBA_OK) return 0;
     return L.total;
+}
+
+comba_status_t comba_workspace_status(const void* workspace, void* stream) {
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const void* word = workspace;   // the status word is the workspace's first 4 bytes (Layout::err = 0)
+    if (!word) {
+        void* scratch = nullptr;
+        if (comba::static_scratch_address(&scratch) != cudaSuccess) return COMBA_ERR_CUDA;
+        word = scratch;
+    }
+    int host = 0;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (cudaMemcpyAsync(&host, word, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess) return COMBA_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return COMBA_ERR_CUDA;
+    return host ? COMBA_ERR_TIMEOUT : COMBA_OK;
 }
 
 }  // extern "C"
@@ -335,7 +353,7 @@ comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const 
     const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
     comba_status_t st = plan(shape, save ? 1 : 0, &L);
     if (st != COMBA_OK) return st;
-    if (shape->flags & ~(COMBA_SAVE_FACTORS | COMBA_IPLR)) return COMBA_ERR_INVALID_ARG;
+    if (shape->flags & ~(COMBA_SAVE_FACTORS | COMBA_IPLR | COMBA_DIAG_STALL)) return COMBA_ERR_INVALID_ARG;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(o);
     COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
@@ -353,7 +371,7 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     Layout L;
     comba_status_t st = plan(shape, 1, &L);
     if (st != COMBA_OK) return st;
-    if (shape->flags & ~(COMBA_REUSE_FACTORS | COMBA_IPLR)) return COMBA_ERR_INVALID_ARG;
+    if (shape->flags & ~(COMBA_REUSE_FACTORS | COMBA_IPLR | COMBA_DIAG_STALL)) return COMBA_ERR_INVALID_ARG;
     COMBA_REQUIRE(q); COMBA_REQUIRE(k); COMBA_REQUIRE(v); COMBA_REQUIRE(alpha); COMBA_REQUIRE(beta);
     COMBA_REQUIRE(d); COMBA_REQUIRE(dO);
     COMBA_REQUIRE(dq); COMBA_REQUIRE(dk); COMBA_REQUIRE(dv); COMBA_REQUIRE(dalpha); COMBA_REQUIRE(dbeta);

@@ -825,6 +825,7 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     a.H = p.H; a.vg = p.vg; a.N = p.N; a.T = p.T; a.slots = p.slots; a.Ttot = p.Ttot; a.cu = p.cu;
     a.seq_first = p.seq_first;
     a.Gb = p.Gb; a.init = p.dhT; a.fin = p.dh0; a.Sout = p.dHb; a.Y = p.Cb; a.reverse = 1; a.err = p.err;
+    a.wait_ns = p.wait_ns;
     a.X = tcp ? p.Ab : p.ATb;   // tcgen05 path: Atilde read as an MN-major operand
     a.x_mn = tcp ? 1 : 0;
     a.W = p.Wb; a.K = p.k;      // dk = 256: dH = gamma dH' + C - W^T Kbar dH' per chunk

@@ -479,6 +479,7 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
         a.Y = nullptr;
     }
     a.err = q.err;
+    a.wait_ns = q.wait_ns;
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)q.slots * q.H, s))) return e;
     mark(q, ev0 + 2, s);
     if (q.o || q.Eb) {

@@ -38,11 +38,11 @@ struct PrepTcSmem {
 };
 
 // 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
-__global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
+__global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p) {
     constexpr int NTH = 256;
     using S = PrepTcSmem;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar;
+    __shared__ uint64_t bar, stall_bar;   // stall_bar: nothing arrives (COMBA_DIAG_STALL)
     __shared__ uint32_t tbase;
     const int slot = blockIdx.x, h = blockIdx.y;
     const SlotInfo si = p.slot_info[slot];
@@ -111,13 +111,14 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
     if (tid < 64) sWs[tid] = sBt[tid] * expf(sGm1[tid]);
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
+        mbar_init(smem_u32(&stall_bar), 1);
         mbar_fence_init();
     }
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
     cp_async_wait<0>();
     publish_smem();
     const uint32_t tmem = tbase;
-    MmaSync ms{smem_u32(&bar), 0};
+    MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
     const int row = tid & 127, half = tid >> 7;   // TMEM lane / accumulator row, and which column half
     const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     bool ok = true;
@@ -245,7 +246,10 @@ __global__ void __launch_bounds__(256) k_prep_tc(ChunkParams p) {
     }
     __syncthreads();
     if (ok) copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
-    if (!ok && tid == 0) flag_error(p);
+    if (!ok) {
+        if (tid == 0) flag_error(p);
+        ms.drain(tid);
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -270,7 +274,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     constexpr int NTH = 256;
     using S = OutTcSmem;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar;
+    __shared__ uint64_t bar, stall_bar;   // stall_bar: nothing arrives (COMBA_DIAG_STALL)
     __shared__ uint32_t tbase;
     const int slot = blockIdx.x, h = blockIdx.y;
     const SlotInfo si = p.slot_info[slot];
@@ -312,6 +316,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     if (tid < 64) sG[tid] = gv;
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
+        mbar_init(smem_u32(&stall_bar), 1);
         mbar_fence_init();
     }
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
@@ -331,7 +336,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     }
     publish_smem();
     const uint32_t tmem = tbase;
-    MmaSync ms{smem_u32(&bar), 0};
+    MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
     const int row = tid & 127, half = tid >> 7;   // TMEM lane, and which 32 of each 64 columns
     const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
 
@@ -447,7 +452,10 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
                 *reinterpret_cast<const uint4*>(sO + r * 136 + 8 * ch);
         }
     }
-    if (!ok && tid == 0) flag_error(p);
+    if (!ok) {
+        if (tid == 0) flag_error(p);
+        ms.drain(tid);
+    }
     if (ok && Eg && tid == 0) bulk_wait_all_reads();   // the E copy has read its staging before exit
     tc_fence_before();
     __syncthreads();

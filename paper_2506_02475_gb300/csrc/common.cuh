@@ -267,10 +267,24 @@ __device__ __forceinline__ void chunk_log_cumsum(const float* alpha, long long s
 
 // ------------------------------------------- sm_100-family async primitives
 // mbarrier, TMA (cp.async.bulk.tensor), and tcgen05 (5th-generation tensor
-// cores with TMEM accumulators).  Every wait is bounded: it gives up after
-// kSpinLimit polls and reports failure instead of hanging.
+// cores with TMEM accumulators).  Every wait is bounded in time (%globaltimer,
+// nanoseconds) and reports failure instead of hanging.  A kernel's own waits
+// take the per-call limit of its launch parameters (kDefaultWaitNs unless the
+// caller sets one, at most kMaxWaitNs); a kernel that gave up then lets every copy and product it
+// has in flight finish with mbar_drain, whose limit is fixed, so that nothing
+// still writes its shared memory or TMEM when the kernel releases them.
 
-constexpr long long kSpinLimit = 1LL << 26;
+constexpr uint32_t kDefaultWaitNs = 1000000000u;   // 1 s
+constexpr uint32_t kDrainWaitNs = 2000000000u;     // 2 s
+// Limits are at most kMaxWaitNs, so that the low 32 bits of %globaltimer measure them
+// without ambiguity (they wrap every 4.29 s).
+constexpr uint32_t kMaxWaitNs = 4000000000u;
+
+__device__ __forceinline__ uint32_t global_ns_lo() {
+    uint32_t t;
+    asm volatile("{\n .reg .u64 t64;\n mov.u64 t64, %%globaltimer;\n cvt.u32.u64 %0, t64;\n}\n" : "=r"(t));
+    return t;
+}
 
 __device__ __forceinline__ void mbar_init(uint32_t mbar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(mbar), "r"(count) : "memory");
@@ -279,17 +293,44 @@ __device__ __forceinline__ void mbar_fence_init() { asm volatile("fence.mbarrier
 __device__ __forceinline__ void mbar_expect_tx(uint32_t mbar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(mbar), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity) {
-    for (long long it = 0; it < kSpinLimit; ++it) {
-        uint32_t ok;
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(ok)
-            : "r"(mbar), "r"(parity)
-            : "memory");
-        if (ok) return true;
+__device__ __forceinline__ bool mbar_try(uint32_t mbar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(mbar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Wait for the phase of parity `parity` to complete; false once `limit_ns` have passed without it.
+// The clock is first read after 64 polls (a wait that ends sooner never touches it), then every 64
+// polls, which keeps both the fast path and the loop's registers lean.
+__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity, uint32_t limit_ns) {
+    uint32_t t0 = 0;
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try(mbar, parity)) return true;
+        if ((i & 63) == 0) {
+            const uint32_t t = global_ns_lo();
+            if (i == 64)
+                t0 = t;
+            else if (t - t0 > limit_ns)
+                return false;
+        }
     }
+}
+// A wait bounded by a poll count instead of the clock, for the tensor-core completion waits of the
+// chunk kernels (prep, output, local gradients), where reading %globaltimer anywhere in the loop
+// measurably slows the kernel: one try_wait takes at least ~16 ns, so `limit_ns / 16` polls
+// last no less than the limit.
+__device__ __forceinline__ bool mbar_wait_polls(uint32_t mbar, uint32_t parity, uint32_t limit_ns) {
+    const long long polls = (long long)(limit_ns >> 4) + 1;
+    for (long long it = 0; it < polls; ++it)
+        if (mbar_try(mbar, parity)) return true;
     return false;
+}
+// The wait of a kernel's give-up path: its copies and products in flight must land first.
+__device__ __forceinline__ bool mbar_drain(uint32_t mbar, uint32_t parity) {
+    return mbar_wait(mbar, parity, kDrainWaitNs);
 }
 
 // 2D tiled TMA load of box (x, y) into shared memory, completing on `mbar`.

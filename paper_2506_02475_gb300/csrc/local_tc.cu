@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                    const __grid_constant__ CUtensorMap tmDk) {
     using S = LocalTcSmem;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar;
+    __shared__ uint64_t bar, stall_bar;   // stall_bar: nothing arrives (COMBA_DIAG_STALL)
     __shared__ uint32_t tbase;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wr = warp & 3, wc = warp >> 2, m0 = 16 * wr;
@@ -256,6 +256,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
 
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
+        mbar_init(smem_u32(&stall_bar), 1);
         mbar_fence_init();
     }
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 512);
@@ -264,7 +265,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     tc_fence_after();
     const uint32_t tmem = tbase;
     const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16);   // this warp's TMEM lanes
-    MmaSync ms{smem_u32(&bar), 0};
+    MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
     const int nl0 = 8 * NL * wc, nk0 = 8 * NK * wc;   // this warp's columns of 64- and 128-wide results
     const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows
     auto put_rows = [&](int kind, float s0, float s1) {
@@ -777,6 +778,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     }
     cp_async_wait<0>();   // no copy is still writing shared memory at exit
     if (tid == 0) bulk_wait_rows_done();   // and no bulk store is still reading it
+    if (!ok) ms.drain(tid);               // nor a product still writing TMEM after a wait gave up
     tc_fence_before();
     __syncthreads();
     tc_fence_after();

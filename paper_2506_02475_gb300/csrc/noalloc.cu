@@ -8,53 +8,52 @@
 //
 // The array is COMBA_STATIC_SCRATCH_BYTES (32 MiB) and exists on every GPU
 // that loads this library, for the life of the process.  Its device address
-// is looked up once per device (cudaGetSymbolAddress, with that device
-// current) on the first call made there.  All calls share the one array and
+// is looked up on every call (cudaGetSymbolAddress, with the caller's device
+// current): the lookup is cheap and cannot go stale when a context is torn
+// down and re-created.  All calls share the one array and
 // it keeps whatever the last call left: the forward writes every scratch byte
 // before reading it, so nothing needs clearing, but two calls whose kernels
 // overlap on the GPU (different streams, or different host threads) race on
 // it and must be serialised by the caller.
 #include <cuda_runtime.h>
 
-#include <mutex>
-
 #include "../../include/comba.h"
+#include "params.cuh"
 
 namespace {
 
 static __device__ __align__(256) unsigned char g_static_scratch[COMBA_STATIC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
+}  // namespace
 
-// Device address of the static scratch on the current device (looked up once).
-comba_status_t static_scratch(void** out) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return COMBA_ERR_CUDA;
-    if (dev < 0 || dev >= kMaxDevices) return COMBA_ERR_UNSUPPORTED;
-    std::lock_guard<std::mutex> lock(g_mutex);
-    if (!g_scratch_addr[dev]) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) return COMBA_ERR_CUDA;
-        g_scratch_addr[dev] = p;
-    }
-    *out = g_scratch_addr[dev];
-    return COMBA_OK;
+namespace comba {
+
+// Device address of the static scratch on the current device.  In host code
+// the array's name is only a host-side stand-in, so the address is asked of
+// the runtime each time.
+cudaError_t static_scratch_address(void** out) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess) return e;
+    if (!p) return cudaErrorInvalidSymbol;
+    *out = p;
+    return cudaSuccess;
 }
 
-}  // namespace
+}  // namespace comba
 
 extern "C" comba_status_t comba_chunk_fwd_noalloc(const comba_shape_t* shape, const void* q, const void* k,
                                                   const void* v, const float* alpha, const float* beta,
                                                   const float* b, const float* d, const float* h0, void* o,
                                                   float* hT, void* stream) {
+    // Only the plain and iplr forms run here: saved factors would land in the shared array where no
+    // caller can reach them, and the gated and pk forms have entry points of their own.
+    if (shape && (shape->flags & ~COMBA_IPLR)) return COMBA_ERR_INVALID_ARG;
     const size_t need = comba_workspace_size(shape, 0);
     if (need > (size_t)COMBA_STATIC_SCRATCH_BYTES) return COMBA_ERR_WORKSPACE;
     void* scratch = nullptr;
     if (need > 0) {
-        const comba_status_t st = static_scratch(&scratch);
-        if (st != COMBA_OK) return st;
+        if (comba::static_scratch_address(&scratch) != cudaSuccess) return COMBA_ERR_CUDA;
     }
     // need == 0 means an invalid shape: the regular entry point reports why before launching anything.
     return comba_chunk_fwd(shape, q, k, v, alpha, beta, b, d, h0, o, hT, scratch, (size_t)COMBA_STATIC_SCRATCH_BYTES,

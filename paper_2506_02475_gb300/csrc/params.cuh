@@ -70,6 +70,8 @@ struct ChunkParams {
     void* dHb;               // [pairs][dv][dk]  dL/dH at chunk end, transposed
     float* part;             // [pairs][2]       per-chunk db, dd partial sums
     int* err;                // device status word (nonzero: a bounded wait gave up)
+    uint32_t wait_ns;        // limit of each device-side wait (kDefaultWaitNs unless set)
+    int stall;               // COMBA_DIAG_STALL: the tcgen05 chunk kernels' first completion wait runs out
 
     // optional stage-boundary events (instrumentation)
     cudaEvent_t* ev;
@@ -143,6 +145,7 @@ struct ScanArgs {
     int x_mn;                // X is read as an MN-major operand ([k][m] row-major, no transpose)
     int vg;                  // value heads per key head: init/fin are [N, H / vg, dk, vg * dv]
     int* err;
+    uint32_t wait_ns;        // limit of each device-side wait
     // tcgen05 path (dk = dv = 128): the scan forms each chunk's additive term itself instead of
     // reading Y, as a product of a workspace factor F and a token tensor `tok`:
     //   ym = 2 (forward):  B^T = U_s^T K,  F = U_s^T [pairs][dv][64], tok = keys [tokens, H / vg, dk]
@@ -192,6 +195,9 @@ cudaError_t launch_recurrent_step(int Bd, int H, int dk, int dv, bool is_bf16, c
 cudaError_t launch_group_sum(const void* dq_v, const void* dk_v, const float* da_v, const float* db_v,
                              const void* dp_v, void* dq, void* dk, float* dalpha, float* dbeta, void* dp,
                              long long tokens, int H, int vg, int dk_, bool is_bf16, cudaStream_t s);
+// Device address of the static scratch of comba_chunk_fwd_noalloc on the current device
+// (noalloc.cu); its first 4 bytes are that entry point's status word.
+cudaError_t static_scratch_address(void** out);
 // Comba-pk correction applied before the chunk kernels: qt = q - d_h p over [rows = tokens*H, dk].
 cudaError_t launch_pk_qtilde(const void* q, const void* p, const float* d, void* qt, long long rows, int H, int dk,
                              bool is_bf16, cudaStream_t s);

@@ -178,7 +178,7 @@ __global__ void __launch_bounds__(256, 1)
 
         int bad = 0;
         if (tid == 0) {
-            if (mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
+            if (mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1, a.wait_ns)) {
 #pragma unroll
                 for (int ks = 0; ks < DK / 16; ++ks) {
                     const int half = ks >> 2, sub = ks & 3;
@@ -201,17 +201,19 @@ __global__ void __launch_bounds__(256, 1)
             if (nx < nch) issue_x(nx++);
             if (ny < nch) issue_y(ny++);
         }
-        if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
-        if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1)) bad = 1;
+        if (!mbar_wait(smem_u32(&mma_bar), it & 1, a.wait_ns)) bad = 1;
+        if (!mbar_wait(smem_u32(&full_y[it % S::SY]), (it / S::SY) & 1, a.wait_ns)) bad = 1;
         // Before the next chunk packs into the other A buffer, the store issued one chunk ago
         // (from that buffer) must have finished reading it.
         if (tid == 0) bulk_wait_read<1>();
         if (__syncthreads_or(bad)) {
             if (tid == 0) {
                 if (a.err) atomicExch(a.err, 1);
-                // drain the loads still in flight into this CTA's shared memory (bounded waits)
-                for (int c = it; c < nx; ++c) mbar_wait(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
-                for (int c = it; c < ny; ++c) mbar_wait(smem_u32(&full_y[c % S::SY]), (c / S::SY) & 1);
+                // drain the loads still in flight into this CTA's shared memory, and the chunk's
+                // product (its commit, phase it, is the last) before TMEM is released
+                for (int c = it; c < nx; ++c) mbar_drain(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
+                for (int c = it; c < ny; ++c) mbar_drain(smem_u32(&full_y[c % S::SY]), (c / S::SY) & 1);
+                mbar_drain(smem_u32(&mma_bar), it & 1);
             }
             break;
         }
@@ -392,7 +394,7 @@ __global__ void __launch_bounds__(256, 1)
             tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc_y, ks > 0 ? 1u : 0u);
         }
     };
-    auto wait_f = [&](int it) { return mbar_wait(smem_u32(&full_f[it % S::SF]), (it / S::SF) & 1); };
+    auto wait_f = [&](int it) { return mbar_wait(smem_u32(&full_f[it % S::SF]), (it / S::SF) & 1, a.wait_ns); };
     const bool tail_short = (len & (kChunk - 1)) != 0;
     int ybad = 0;   // thread 0: a chunk's F / T never arrived
     if (tid == 0 && nch > 0) {
@@ -429,7 +431,7 @@ __global__ void __launch_bounds__(256, 1)
 
         int bad = ybad;
         if (tid == 0) {
-            if (!ybad && mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1)) {
+            if (!ybad && mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1, a.wait_ns)) {
 #pragma unroll
                 for (int ks = 0; ks < DK / 16; ++ks) {
                     const int half = ks >> 2, sub = ks & 3;
@@ -461,18 +463,21 @@ __global__ void __launch_bounds__(256, 1)
             // its stage last held chunk it - 1, whose product the commit of chunk it - 1 covered
             if (nf < nch) issue_f(nf++);
         }
-        if (!mbar_wait(smem_u32(&mma_bar), it & 1)) bad = 1;
+        if (!mbar_wait(smem_u32(&mma_bar), it & 1, a.wait_ns)) bad = 1;
         if (tid == kTma) bulk_wait_read<1>();
         if (__syncthreads_or(bad)) {
             if (tid == kTma) {
                 if (a.err) atomicExch(a.err, 1);
-                for (int c = it; c < nx; ++c) mbar_wait(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
-                for (int c = it; c < nf; ++c) mbar_wait(smem_u32(&full_f[c % S::SF]), (c / S::SF) & 1);
+                for (int c = it; c < nx; ++c) mbar_drain(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
+                for (int c = it; c < nf; ++c) mbar_drain(smem_u32(&full_f[c % S::SF]), (c / S::SF) & 1);
             }
             if (tid == 0) {
-                // a product issued after the last commit must finish before TMEM is released
+                // the products must finish before TMEM is released: chunk it's (phase it, which may
+                // still be pending: a parity wait is only exact on the pending phase), then one more
+                // commit for the additive term issued after it
+                mbar_drain(smem_u32(&mma_bar), it & 1);
                 tc_commit(smem_u32(&mma_bar));
-                mbar_wait(smem_u32(&mma_bar), (it + 1) & 1);
+                mbar_drain(smem_u32(&mma_bar), (it + 1) & 1);
             }
             break;
         }

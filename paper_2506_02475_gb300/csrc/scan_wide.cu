@@ -252,7 +252,7 @@ __global__ void __launch_bounds__(256, 1)
 
         int bad = 0;
         if (tid == 0) {
-            if (mbar_wait(smem_u32(&full_f1), it & 1)) {
+            if (mbar_wait(smem_u32(&full_f1), it & 1, a.wait_ns)) {
                 // backward: F1 holds the keys; the first chunk of the reverse scan may be short
                 if (rev && it == 0 && L < kChunk) zero_tile_rows(smem + S::OF1, L, 4);
                 tc_gemm_m64<false, false>(tmem, uA, 64, uF1, 64, 64, DK, false);
@@ -262,7 +262,7 @@ __global__ void __launch_bounds__(256, 1)
             tc_commit(smem_u32(&mma1_bar));
             if (rev && !bad) {
                 // C^T = dO^T Z into the second product's columns (read back in the previous chunk's update)
-                if (mbar_wait(smem_u32(&full_st[it & 1]), (it >> 1) & 1)) {
+                if (mbar_wait(smem_u32(&full_st[it & 1]), (it >> 1) & 1, a.wait_ns)) {
                     // the reverse scan's first chunk is a sequence's last and may be short: its dO rows
                     // past the sequence end (the next sequence's, or past the tensor) must not enter
                     if (it == 0 && L < kChunk) zero_tile_rows(smem + (uZ(it) - su) + S::T_BYTES, L, 1);
@@ -276,8 +276,8 @@ __global__ void __launch_bounds__(256, 1)
             for (int half = 0; half < 4; ++half) tma_store_tile(&tmS, 64 * half, (int)(unit_of(it) * 64), uA + half * 8192);
             bulk_commit_group();
         }
-        if (!mbar_wait(smem_u32(&mma1_bar), it & 1)) bad = 1;
-        if (!mbar_wait(smem_u32(&full_st[it & 1]), (it >> 1) & 1)) bad = 1;
+        if (!mbar_wait(smem_u32(&mma1_bar), it & 1, a.wait_ns)) bad = 1;
+        if (!mbar_wait(smem_u32(&full_st[it & 1]), (it >> 1) & 1, a.wait_ns)) bad = 1;
         if (__syncthreads_or(bad)) {
             failed = true;
             break;
@@ -321,7 +321,7 @@ __global__ void __launch_bounds__(256, 1)
             tc_commit(smem_u32(&mma2_bar));
             ++n2;
         }
-        if (!mbar_wait(smem_u32(&mma2_bar), it & 1)) bad = 1;
+        if (!mbar_wait(smem_u32(&mma2_bar), it & 1, a.wait_ns)) bad = 1;
         tc_fence_after();
 
         // S^T <- gamma_C S^T + Pt F2 + Y  (the accumulator holds Y as well)
@@ -343,18 +343,21 @@ __global__ void __launch_bounds__(256, 1)
     }
 
     if (failed && tid == 0) {
-        // a C^T product issued after the last commit finishes before TMEM is released
+        // every product finishes before TMEM is released: first the last committed phase of the
+        // second barrier (it may be the pending one; a parity wait is only exact on that phase),
+        // then one more commit covers the first product and a C^T product issued since
+        if (n2 > 0) mbar_drain(smem_u32(&mma2_bar), (n2 - 1) & 1);
         tc_commit(smem_u32(&mma2_bar));
-        mbar_wait(smem_u32(&mma2_bar), n2 & 1);
+        mbar_drain(smem_u32(&mma2_bar), n2 & 1);
     }
     if (failed && tid == kTma) {
         // a bounded wait gave up: record it, and let the last load issued to each barrier land
         // (bounded waits again) before this CTA's shared memory is released
         if (a.err) atomicExch(a.err, 1);
-        if (nf1 > 0) mbar_wait(smem_u32(&full_f1), (nf1 - 1) & 1);
+        if (nf1 > 0) mbar_drain(smem_u32(&full_f1), (nf1 - 1) & 1);
         for (int b = 0; b < 2; ++b) {
             const int k = nst - 1 - ((nst - 1 - b) & 1);   // the latest stage issued to barrier b
-            if (k >= 0) mbar_wait(smem_u32(&full_st[b]), (k >> 1) & 1);
+            if (k >= 0) mbar_drain(smem_u32(&full_st[b]), (k >> 1) & 1);
         }
     }
     if (tid == kTma) bulk_wait_all_groups();

@@ -45,16 +45,26 @@ __device__ __forceinline__ void unpack8(uint4 u, float* v) {
 
 // One-barrier MMA completion tracker (all threads keep the same phase).
 struct MmaSync {
-    uint32_t bar;
+    uint32_t bar;        // the barrier the products commit to
+    uint32_t wbar;       // the barrier waited on: `bar`, or (COMBA_DIAG_STALL) one nothing arrives at
     uint32_t phase;
+    uint32_t limit_ns;
     // Thread 0 has issued MMAs; commit, wait everywhere, and report failure uniformly.
     __device__ __forceinline__ bool finish(int tid) {
         if (tid == 0) tc_commit(bar);
-        const bool ok = mbar_wait(bar, phase);
+        const bool ok = mbar_wait_polls(wbar, phase, limit_ns);
         phase ^= 1;
         const bool any_bad = __syncthreads_or(!ok);
         tc_fence_after();
         return !any_bad;
+    }
+    // After a failed finish (the kernel then issues no further product): the commit whose wait
+    // gave up covers every product thread 0 has issued, so waiting (again) for that phase means
+    // nothing writes TMEM once the kernel releases it.  `phase` has moved past it, and a parity
+    // wait on the phase still pending is the right one.  Called by every thread ahead of the
+    // kernel's exit barrier.
+    __device__ __forceinline__ void drain(int tid) {
+        if (tid == 0) mbar_drain(bar, phase ^ 1);
     }
 };
 

@@ -251,3 +251,27 @@ def test_head_dim_256(L):
                                       None)
     assert step(384) == UNSUPPORTED
     assert step(256, dk=64) == UNSUPPORTED
+
+
+def test_noalloc_forward_takes_only_the_plain_and_iplr_forms(L):
+    """The allocation-free forward rejects flags it cannot honour (saved factors would sit in the
+    shared static array out of the caller's reach; gated and pk have entry points of their own)
+    before any CUDA call."""
+    fn = L.comba_chunk_fwd_noalloc
+    for flags in (1, 2, 8, 16, 1 | 4):
+        s = shape(flags=flags)
+        assert fn(ctypes.byref(s), *([FAKE] * 7), None, FAKE, None, None) == INVALID, flags
+    s = shape(B=8, T=4096, H=16)
+    assert fn(ctypes.byref(s), *([FAKE] * 7), None, FAKE, None, None) == WORKSPACE
+
+
+def test_diagnostic_stall_flag_is_accepted_only_by_the_plain_chunk_calls(L):
+    """COMBA_DIAG_STALL (32) is a flag of comba_chunk_fwd / comba_chunk_bwd: with it, validation goes
+    on to the workspace check (it is accepted); an unknown bit next to it, and the allocation-free
+    forward, reject it before any CUDA call."""
+    assert fwd(L, shape(flags=32)) == WORKSPACE
+    assert fwd(L, shape(flags=1 | 32)) == WORKSPACE
+    assert fwd(L, shape(flags=32 | 64)) == INVALID
+    fn = L.comba_chunk_fwd_noalloc
+    s = shape(flags=32)
+    assert fn(ctypes.byref(s), *([FAKE] * 7), None, FAKE, None, None) == INVALID
