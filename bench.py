@@ -15,6 +15,9 @@ backward needs (COMBA_SAVE_FACTORS) and the backward reuses them.
 Prints one JSON line (rank 0).  Under torchrun each rank runs an independent
 replica of the workload (the op shards over sequences and heads with no
 data-path collective); value = tokens of all ranks / max-over-ranks time.
+The training-step line nests the decode measurement (Bd=256, H=16, d=128,
+1024 sequential token steps) under "decode" unless --no-decode; its "e2e"
+uploads every input and reads every output back each step.
 ``--impl reference`` times the fp64 CPU oracle on bounded samples instead.
 """
 from __future__ import annotations
@@ -51,6 +54,23 @@ def load_peaks():
 def fwd_flops_per_token_head(C=64, dk=128, dv=128):
     """Five C^2 d GEMMs (K K^T, M K, M V, Q~K^T, P E) and three C d^2 (W H, Q~ H, Kbar^T E)."""
     return 2 * C * (3 * dk + 2 * dv) + 6 * dk * dv
+
+
+def compulsory_bytes(dk, dv, token_heads, state_elems, es=2):
+    """Bytes a training step must move at least once (inputs read once, outputs written once):
+    forward q, k, v, alpha, beta in, o out, h0 in, hT out; backward q, k, v, alpha, beta, dO in,
+    dq, dk, dv, dalpha, dbeta out, h0 and dhT in, dh0 out.  At dk = dv = 128 in bf16 that is
+    1032 B (forward) and 1808 B (backward) per (token, head), plus the fp32 states.  `per_stage`
+    gives the share each kernel of the tcgen05 path must touch itself: prep reads k, v and the
+    gates; the output kernel reads q, k and alpha and writes o; the local-gradient kernel reads
+    every backward input and writes every token gradient."""
+    tok_fwd = (2 * dk + dv) * es + 8 + dv * es
+    tok_bwd = (2 * dk + dv) * es + 8 + dv * es + (2 * dk + dv) * es + 8
+    fwd = token_heads * tok_fwd + 2 * state_elems * 4
+    bwd = token_heads * tok_bwd + 3 * state_elems * 4
+    per_stage = {"prep": token_heads * ((dk + dv) * es + 8), "output": token_heads * ((2 * dk + dv) * es + 4),
+                 "scan_fwd": 2 * state_elems * 4, "scan_bwd": 2 * state_elems * 4, "bwd_local": token_heads * tok_bwd}
+    return fwd, bwd, per_stage
 
 
 # --------------------------------------------------------------- kernel model
@@ -510,6 +530,15 @@ def run_ours(args, world, rank, local):
                  "algorithmic_bytes": mdl["bytes"], "traffic": traffic,
                  "traffic_source": "ncu capture of the 340M-shape step, scaled by units" if traffic else None,
                  "peak_source": peak_src + " (burst)"})
+    # the same kernel and the whole step on compulsory bytes only (the step's inputs read once and
+    # its outputs written once; none of this design's intermediates)
+    c_fwd, c_bwd, c_stage = compulsory_bytes(dk, dv, tokens * H, N * H * dk * dv)
+    cb = c_stage.get(dom)
+    roof["compulsory_bytes"] = cb
+    roof["frac_compulsory"] = None if cb is None else cb / (launch_ms / 1e3) / 1e9 / peaks["hbm_gbs"]
+    roof["step_compulsory"] = {"bytes": c_fwd + c_bwd, "achieved_gbs": (c_fwd + c_bwd) / (ms / 1e3) / 1e9,
+                               "frac": (c_fwd + c_bwd) / (ms / 1e3) / 1e9 / peaks["hbm_gbs"],
+                               "floor_ms": (c_fwd + c_bwd) / (peaks["hbm_gbs"] * 1e9) * 1e3}
 
     # ---- end to end through the public API with host buffers.  Every step copies all its
     # inputs from pinned host memory and reads its result back: the per-sequence and per-head
@@ -593,12 +622,14 @@ def run_ours(args, world, rank, local):
             "tflops": tflops, "pct_bf16_peak": tflops / peaks["bf16_tflops"] * 100,
             "roofline": roof,
             "cpu_baseline": cpu,
-            "e2e": {"value": tokens * world / (e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": bi,
-                    "d2h_bytes_per_step": bo, "ms_per_step": e_ms,
-                    "result_read_back": list(RESULT),
-                    "copies": "pinned host buffers; upload and download on their own streams, double-buffered",
-                    "all_outputs_read_back": {"value": tokens * world / (e_full_ms / 1e3), "ms_per_step": e_full_ms,
-                                              "d2h_bytes_per_step": bo_full}},
+            "e2e": {"value": tokens * world / (e_full_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": bi,
+                    "d2h_bytes_per_step": bo_full, "ms_per_step": e_full_ms,
+                    "read_back": list(all_keys),
+                    "copies": "pinned host buffers; every input uploaded and every output read back each step; "
+                              "upload and download on their own streams, double-buffered",
+                    "results_only_read_back": {"value": tokens * world / (e_ms / 1e3), "ms_per_step": e_ms,
+                                               "d2h_bytes_per_step": bo, "read_back": list(RESULT),
+                                               "note": "o and the token gradients left on the device"}},
             "clocks": clk,
             # forward: chunk map, prep, scan, output; backward: (C term at dk = 64), reverse
             # scan, local gradients, per-head sums; plus q - d p per call with p, the key-head sums
@@ -607,6 +638,11 @@ def run_ours(args, world, rank, local):
             "stages_ms_per_step": {f"{p}.{s}": v / args.steps for (p, s), v in stage_ms.items()},
             "wall_s_timed": wall,
         }
+    # the recurrent decode step (Bd=256, H=16, d=128) measured in the same run, its own line nested
+    dec = None if args.no_decode else measure_decode(args, world, rank, dist, dev, peaks, peak_src)
+    if rank == 0:
+        if dec is not None:
+            line["decode"] = dec
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
@@ -752,10 +788,21 @@ def run_decode(args, world, rank, local):
     import torch
     dist = dist_init(world, local, "nccl")
     torch.cuda.set_device(local)
-    from paper_2506_02475_gb300 import comba_recurrent_step, inputs, shard
     peaks, peak_src = load_peaks()
+    line = measure_decode(args, world, rank, dist, torch.device("cuda", local), peaks, peak_src)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def measure_decode(args, world, rank, dist, dev, peaks, peak_src):
+    """The decode workload (Bd=256, H=16, d=128, 1024 sequential token steps per timed step):
+    device-resident timing, the end-to-end leg and the oracle on the host; returns the JSON
+    line's dict on rank 0 (None elsewhere)."""
+    import torch
+    from paper_2506_02475_gb300 import comba_recurrent_step, inputs, shard
     Bd, H, dk, dv = 256, 16, 128, 128
-    dev = torch.device("cuda", local)
     off = shard.rank_seed_offset(rank)
     state = torch.from_numpy(inputs.decode_state(Bd, H, dk, dv, seed_offset=off)).to(dev)
     toks = []
@@ -841,7 +888,7 @@ def run_decode(args, world, rank, local):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = decode_cpu_baseline(Bd, H, dk, dv)
     if rank == 0:
-        print(json.dumps({
+        return {
             "metric": DECODE_METRIC, "value": Bd * steps * world / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "fp32-state/bf16-tokens", "data": "synthetic",
@@ -856,9 +903,8 @@ def run_decode(args, world, rank, local):
                     "d2h_bytes_per_step": bo, "ms_per_token_step": e_ms / steps,
                     "copies": "q, k, v, alpha, beta uploaded from pinned host memory and o read back every token "
                               "step (own streams, double-buffered); the state stays on the device"},
-            "clocks": clk, "gpu_launches": steps * args.steps}), flush=True)
-    if dist:
-        dist.destroy_process_group()
+            "clocks": clk, "gpu_launches": steps * args.steps}
+    return None
 
 
 # --------------------------------------------------------------- reference
@@ -921,6 +967,8 @@ def main():
     ap.add_argument("--workload", default="lm1p3b",
                     choices=["lm1p3b", "lm340m", "varlen64k", "lm1p3b_v256", "lm1p3b_d256", "decode"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode", action="store_true",
+                    help="leave out the decode measurement nested in the training-step line")
     ap.add_argument("--gated", action="store_true",
                     help="raw q, k and gate pre-activations through the gate and normalisation prologue")
     ap.add_argument("--variant", default="splr", choices=["splr", "iplr", "pk"],
