@@ -439,31 +439,43 @@ __device__ __forceinline__ uint64_t desc_mnmajor(uint32_t base, int krows, int k
     return smem_desc(base + ks * 2048, krows * 128, 1024);
 }
 
-// D[tmem, 128 x N fp32] (+)= A[128 x K] * B[K x N] on bf16 smem tiles, issued by one
-// thread.  AMN/BMN select MN-major operand tiles; a_ext/b_ext are the tiles'
-// allocated row counts (see above).  K % 16 == 0.
+// Step from the k-step-0 descriptor of a tile to that of k-step ks, in the descriptor's
+// address units (16 bytes): a K-major tile advances 32 B inside a 64-element K half and
+// rows x 128 B from one half to the next; an MN-major one advances 16 K-rows x 128 B.  Adding
+// it to the 64-bit descriptor touches only the 14-bit start-address field, which cannot carry
+// out: shared-memory addresses stay below 2^18 bytes.  With the descriptors formed once per
+// product, issuing a k-step costs two 64-bit adds instead of rebuilding both descriptors.
+template <bool MN>
+__device__ __forceinline__ uint64_t desc_step(int ext, int ks) {
+    return MN ? (uint64_t)(ks * 128) : (uint64_t)((ks >> 2) * ext * 8 + (ks & 3) * 2);
+}
+
+// D[tmem, M x N fp32] (+)= A[M x K] * B[K x N] on bf16 smem tiles, issued by one thread.
+// AMN/BMN select MN-major operand tiles; a_ext/b_ext are the tiles' allocated row counts (see
+// above).  K % 16 == 0.
+template <int M, bool AMN, bool BMN>
+__device__ __forceinline__ void tc_gemm_mk(uint32_t tmem, uint32_t a, int a_ext, uint32_t b, int b_ext, int N, int K,
+                                           bool accumulate) {
+    const uint32_t idesc = idesc_bf16_f32(M, N) | (AMN ? 1u << 15 : 0u) | (BMN ? 1u << 16 : 0u);
+    const uint64_t a0 = AMN ? desc_mnmajor(a, a_ext, 0) : desc_kmajor(a, a_ext, 0);
+    const uint64_t b0 = BMN ? desc_mnmajor(b, b_ext, 0) : desc_kmajor(b, b_ext, 0);
+#pragma unroll
+    for (int ks = 0; ks < K / 16; ++ks)
+        tc_mma_bf16(tmem, a0 + desc_step<AMN>(a_ext, ks), b0 + desc_step<BMN>(b_ext, ks), idesc,
+                    (accumulate || ks > 0) ? 1u : 0u);
+}
+// M = 128: D row m in TMEM lane m.
 template <bool AMN, bool BMN>
 __device__ __forceinline__ void tc_gemm(uint32_t tmem, uint32_t a, int a_ext, uint32_t b, int b_ext, int N, int K,
                                         bool accumulate) {
-    const uint32_t idesc = idesc_bf16_f32(128, N) | (AMN ? 1u << 15 : 0u) | (BMN ? 1u << 16 : 0u);
-    for (int ks = 0; ks < K / 16; ++ks) {
-        const uint64_t ad = AMN ? desc_mnmajor(a, a_ext, ks) : desc_kmajor(a, a_ext, ks);
-        const uint64_t bd = BMN ? desc_mnmajor(b, b_ext, ks) : desc_kmajor(b, b_ext, ks);
-        tc_mma_bf16(tmem, ad, bd, idesc, (accumulate || ks > 0) ? 1u : 0u);
-    }
+    tc_gemm_mk<128, AMN, BMN>(tmem, a, a_ext, b, b_ext, N, K, accumulate);
 }
-
-// Same with M = 64: D row m lives in TMEM lane 32*(m/16) + m%16 (lanes 0-15 of
-// each warp's quadrant), column n in column n.
+// M = 64: D row m lives in TMEM lane 32*(m/16) + m%16 (lanes 0-15 of each warp's quadrant),
+// column n in column n.
 template <bool AMN, bool BMN>
 __device__ __forceinline__ void tc_gemm_m64(uint32_t tmem, uint32_t a, int a_ext, uint32_t b, int b_ext, int N, int K,
                                             bool accumulate) {
-    const uint32_t idesc = idesc_bf16_f32(64, N) | (AMN ? 1u << 15 : 0u) | (BMN ? 1u << 16 : 0u);
-    for (int ks = 0; ks < K / 16; ++ks) {
-        const uint64_t ad = AMN ? desc_mnmajor(a, a_ext, ks) : desc_kmajor(a, a_ext, ks);
-        const uint64_t bd = BMN ? desc_mnmajor(b, b_ext, ks) : desc_kmajor(b, b_ext, ks);
-        tc_mma_bf16(tmem, ad, bd, idesc, (accumulate || ks > 0) ? 1u : 0u);
-    }
+    tc_gemm_mk<64, AMN, BMN>(tmem, a, a_ext, b, b_ext, N, K, accumulate);
 }
 
 // Byte offset of element (mn, k) of an MN-major bf16 tile (allocated K extent krows).

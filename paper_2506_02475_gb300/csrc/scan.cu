@@ -179,14 +179,12 @@ __global__ void __launch_bounds__(256, 1)
         int bad = 0;
         if (tid == 0) {
             if (mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1, a.wait_ns)) {
+                const uint64_t a0 = desc_kmajor(a_buf(it), 128, 0);
+                const uint64_t b0 = XMN ? desc_mnmajor(x_buf(it), DK, 0) : desc_kmajor(x_buf(it), DK, 0);
 #pragma unroll
-                for (int ks = 0; ks < DK / 16; ++ks) {
-                    const int half = ks >> 2, sub = ks & 3;
-                    const uint64_t ad = smem_desc_sw128(a_buf(it) + half * 128 * 128 + sub * 32);
-                    const uint64_t bd = XMN ? desc_mnmajor(x_buf(it), DK, ks)
-                                            : smem_desc_sw128(x_buf(it) + half * DK * 128 + sub * 32);
-                    tc_mma_bf16(tmem, ad, bd, idesc, ks > 0 ? 1u : 0u);
-                }
+                for (int ks = 0; ks < DK / 16; ++ks)
+                    tc_mma_bf16(tmem, a0 + desc_step<false>(128, ks), b0 + desc_step<XMN>(DK, ks), idesc,
+                                ks > 0 ? 1u : 0u);
             } else {
                 bad = 1;
             }
@@ -387,12 +385,12 @@ __global__ void __launch_bounds__(256, 1)
     };
     auto issue_y = [&](int it) {
         const uint32_t fa = smem_u + f_off(it), ta = smem_u + t_off(it);
+        const uint64_t a0 = YM == 1 ? desc_mnmajor(ta, 64, 0) : desc_kmajor(fa, 64, 0);
+        const uint64_t b0 = YM == 1 ? desc_kmajor(fa, DK, 0) : desc_mnmajor(ta, 64, 0);
 #pragma unroll
-        for (int ks = 0; ks < 4; ++ks) {
-            const uint64_t ad = YM == 1 ? desc_mnmajor(ta, 64, ks) : desc_kmajor(fa, 64, ks);
-            const uint64_t bd = YM == 1 ? desc_kmajor(fa, DK, ks) : desc_mnmajor(ta, 64, ks);
-            tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc_y, ks > 0 ? 1u : 0u);
-        }
+        for (int ks = 0; ks < 4; ++ks)
+            tc_mma_bf16(tmem + acc_col(it), a0 + desc_step<YM == 1>(64, ks), b0 + desc_step<YM != 1>(DK, ks), idesc_y,
+                        ks > 0 ? 1u : 0u);
     };
     auto wait_f = [&](int it) { return mbar_wait(smem_u32(&full_f[it % S::SF]), (it / S::SF) & 1, a.wait_ns); };
     const bool tail_short = (len & (kChunk - 1)) != 0;
@@ -432,14 +430,12 @@ __global__ void __launch_bounds__(256, 1)
         int bad = ybad;
         if (tid == 0) {
             if (!ybad && mbar_wait(smem_u32(&full_x[it % S::SX]), (it / S::SX) & 1, a.wait_ns)) {
+                const uint64_t a0 = desc_kmajor(a_buf(it), 64, 0);
+                const uint64_t b0 = XMN ? desc_mnmajor(x_buf(it), DK, 0) : desc_kmajor(x_buf(it), DK, 0);
 #pragma unroll
-                for (int ks = 0; ks < DK / 16; ++ks) {
-                    const int half = ks >> 2, sub = ks & 3;
-                    const uint64_t ad = smem_desc_sw128(a_buf(it) + half * 64 * 128 + sub * 32);
-                    const uint64_t bd = XMN ? desc_mnmajor(x_buf(it), DK, ks)
-                                            : smem_desc_sw128(x_buf(it) + half * DK * 128 + sub * 32);
-                    tc_mma_bf16(tmem + acc_col(it), ad, bd, idesc, 1u);   // onto the additive term
-                }
+                for (int ks = 0; ks < DK / 16; ++ks)   // onto the additive term
+                    tc_mma_bf16(tmem + acc_col(it), a0 + desc_step<false>(64, ks), b0 + desc_step<XMN>(DK, ks), idesc,
+                                1u);
             } else {
                 bad = 1;
             }

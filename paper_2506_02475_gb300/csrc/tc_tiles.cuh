@@ -52,6 +52,10 @@ struct MmaSync {
     // Thread 0 has issued MMAs; commit, wait everywhere, and report failure uniformly.
     __device__ __forceinline__ bool finish(int tid) {
         if (tid == 0) tc_commit(bar);
+        return wait(tid);
+    }
+    // The same when thread 0 has committed already (tc_commit(bar) right behind its products).
+    __device__ __forceinline__ bool wait(int tid) {
         const bool ok = mbar_wait_polls(wbar, phase, limit_ns);
         phase ^= 1;
         const bool any_bad = __syncthreads_or(!ok);
