@@ -10,11 +10,14 @@
 //   R0  S = Q~ K^T, dP = dO E^T      (its own barrier; R1 is issued right behind)
 //   R1  dO H^T, E dH'^T, K dH'      (runs while the warps form P from R0)
 //   R2  P^T dO                       (behind R1, one wait: dE = Kbar dH' + P^T dO)
-//   R3  M^T dE, K K^T, dPhat K, dPhat^T Q~
-//   R4  (M^T dE) H^T = -M^T dW       (dW = -dE H^T)
+//   R3  M^T dE, dPhat^T Q~
+//   R4  (M^T dE) H^T = -M^T dW (dW = -dE H^T), K K^T, dPhat K
 //   R5  (M^T dE) U^T + (M^T dW) W^T  (= M^T dM M^T, so dA needs neither dM nor a
 //                                     second product with M)
 //   R6  dG K + dG^T K onto dPhat^T Q~
+//
+// Each epilogue first forms what the next round reads and lets it be issued, then does the rest
+// of its work while that round runs.
 //
 // An M = 64 accumulator read with tcgen05.ld.16x256b gives each warp the rows
 // 16 (w & 3) .. + 15 in exactly the m16n8 accumulator fragment layout of
@@ -77,21 +80,44 @@ __device__ __forceinline__ void tmem_frag2(uint32_t taddr, float (&a)[2][4]) {
     for (int i = 0; i < 8; ++i) a[i >> 2][i & 3] = __uint_as_float(r[i]);
 }
 
-// bf16 pair (row, col..col+1) of a K-major swizzled tile with `rows` allocated rows.
-__device__ __forceinline__ void st_pair(uint8_t* tile, int rows, int r, int c, float x, float y) {
-    *reinterpret_cast<__nv_bfloat162*>(tile + sw128_offset(r, c, rows)) = __floats2bfloat162_rn(x, y);
+__device__ __forceinline__ uint32_t pack_bf2(float x, float y) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(x, y);
+    return *reinterpret_cast<uint32_t*>(&v);
 }
-__device__ __forceinline__ float2 ld_pair(const uint8_t* tile, int rows, int r, int c) {
-    return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(tile + sw128_offset(r, c, rows)));
+__device__ __forceinline__ void stsm_x4(const void* p, uint32_t r0, uint32_t r1, uint32_t r2, uint32_t r3) {
+    asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1,%2,%3,%4};\n" ::"r"(smem_u32(p)), "r"(r0),
+                 "r"(r1), "r"(r2), "r"(r3)
+                 : "memory");
 }
+// The m16n8 accumulator fragment is the layout of four 8 x 8 b16 matrices of ldmatrix / stmatrix
+// (thread l: row l / 4, columns 2 (l % 4) and + 1), so a warp moves its 16 rows x 16 columns of a
+// fragment tile with one x4 instruction: matrices (rows 0-7, n8 tile t), (rows 8-15, t), (rows
+// 0-7, t + 1), (rows 8-15, t + 1), lane l addressing row (l & 7) + 8 ((l >> 3) & 1) of matrix
+// l >> 3 (a 16-byte chunk, which the swizzle or the staging rotation keeps whole).
+__device__ __forceinline__ int frag_mrow(int m0) { return m0 + (threadIdx.x & 7) + (((threadIdx.x >> 3) & 1) << 3); }
+__device__ __forceinline__ int frag_mcol(int n0, int t) { return n0 + 8 * (t + ((threadIdx.x >> 4) & 1)); }
 // Fragment tile into a K-major swizzled tile (columns n0 + 8 t + ...).
 template <int NT>
 __device__ __forceinline__ void frag_store_sw(uint8_t* tile, int rows, int m0, int n0, const float (&acc)[NT][4]) {
+    static_assert(NT % 2 == 0, "pairs of n8 tiles");
+    const int mr = frag_mrow(m0);
 #pragma unroll
-    for (int t = 0; t < NT; ++t)
+    for (int t = 0; t < NT; t += 2)
+        stsm_x4(tile + sw128_offset(mr, frag_mcol(n0, t), rows), pack_bf2(acc[t][0], acc[t][1]),
+                pack_bf2(acc[t][2], acc[t][3]), pack_bf2(acc[t + 1][0], acc[t + 1][1]),
+                pack_bf2(acc[t + 1][2], acc[t + 1][3]));
+}
+// The same tile read back as packed bf16 pairs: w[2 t] = (row g, tile t), w[2 t + 1] = (row g + 8, t).
+template <int NT>
+__device__ __forceinline__ void frag_load_sw(const uint8_t* tile, int rows, int m0, int n0, uint32_t (&w)[2 * NT]) {
+    static_assert(NT % 2 == 0, "pairs of n8 tiles");
+    const int mr = frag_mrow(m0);
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh)
-            st_pair(tile, rows, m0 + frag_row(2 * hh), n0 + frag_col(t, 0), acc[t][2 * hh], acc[t][2 * hh + 1]);
+    for (int t = 0; t < NT; t += 2) {
+        uint32_t r[4];
+        ldsm_x4(r, tile + sw128_offset(mr, frag_mcol(n0, t), rows));
+        w[2 * t] = r[0]; w[2 * t + 1] = r[1]; w[2 * t + 2] = r[2]; w[2 * t + 3] = r[3];
+    }
 }
 template <int NT>
 __device__ __forceinline__ void tmem_frag(uint32_t taddr, float (&a)[NT][4]) {
@@ -130,14 +156,12 @@ __device__ __forceinline__ void tmem_take(uint32_t (&r)[NT * 4], float (&a)[NT][
 // writes), and its coalesced copy of rows < L to a strided global matrix.
 template <int NT>
 __device__ __forceinline__ void frag_stage(uint8_t* st, int m0, int n0, const float (&acc)[NT][4]) {
+    const int r = frag_mrow(m0);
 #pragma unroll
-    for (int t = 0; t < NT; ++t)
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const int r = m0 + frag_row(2 * hh), c = n0 + frag_col(t, 0);
-            *reinterpret_cast<__nv_bfloat162*>(st + r * 256 + ((((c >> 3) + r) & 15) << 4) + (c & 7) * 2) =
-                __floats2bfloat162_rn(acc[t][2 * hh], acc[t][2 * hh + 1]);
-        }
+    for (int t = 0; t < NT; t += 2)
+        stsm_x4(st + r * 256 + ((((frag_mcol(n0, t) >> 3) + r) & 15) << 4), pack_bf2(acc[t][0], acc[t][1]),
+                pack_bf2(acc[t][2], acc[t][3]), pack_bf2(acc[t + 1][0], acc[t + 1][1]),
+                pack_bf2(acc[t + 1][2], acc[t + 1][3]));
 }
 // Bulk tensor store of a [64][64-column] swizzled tile to (columns x, head y, tokens z ..).
 __device__ __forceinline__ void tma_store_rows(const void* tmap, int x, int y, int z, uint32_t src) {
@@ -181,9 +205,9 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 
 // Persistent: CTA b handles units b, b + G, b + 2G, ... (G = gridDim.x, about one CTA per SM).
 // While unit u computes, the tiles of unit u + G stream into buffers as soon as their last
-// reader in unit u has finished (M after R3, E after the dv copy and H^T after R4, dH'^T and
-// dO after R5, V after R6; Q and K into the second of two alternating tiles at the start of the
-// unit; the per-row scalars into registers), so the loads of consecutive units overlap the
+// reader in unit u has finished (M after R3, H^T after R4, E (after the dv copy), dH'^T, dO and
+// Q/K (into the second of two alternating tiles, which holds M^T dE until then) after R5, V after
+// R6; the per-row scalars into registers), so the loads of consecutive units overlap the
 // tensor-core and epilogue work instead of every SM loading at the same moment.  U^T and W^T of
 // the unit itself load into the dH'^T tile once R1 has read it.
 __global__ void __launch_bounds__(kLocalThreads, 1)
@@ -207,7 +231,6 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     uint8_t* sdPh = sdE;              // dPhat [64][64], from R0's epilogue until R3
     uint8_t* sdEt = sE;               // dE [64][128], after R1 (E's readers) until R3
     uint8_t* stV = sE;                // dv staging, after R3
-    uint8_t* sMdE = sdE;              // M^T dE [64][128], after R3 until R5
     uint8_t* sMdW = sdO;              // M^T dW [64][128], after R2 (dO's readers) until R5
     uint8_t* sUt = sdHt;              // U^T, W^T [128][64] each, after R1 (dH'^T's readers) until R5
     uint8_t* sWt = sdHt + 16384;
@@ -225,7 +248,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     float* red = colp + 2 * 4 * 64;
     const uint32_t udO = smem_u32(sdO), uE = smem_u32(sE), uH = smem_u32(sHt), udH = smem_u32(sdHt),
                    uM = smem_u32(sM), uP = smem_u32(sP), udE = smem_u32(sdEt), udPh = smem_u32(sdPh),
-                   uMdE = smem_u32(sMdE), uMdW = smem_u32(sMdW), uUt = smem_u32(sUt), uWt = smem_u32(sWt),
+                   uMdW = smem_u32(sMdW), uUt = smem_u32(sUt), uWt = smem_u32(sWt),
                    udG = smem_u32(sdG);
 
     const int Hk = p.H / p.vg;   // key heads: q, k, alpha, beta, b, d of value head h are key head h / vg's
@@ -280,12 +303,14 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     };
     // row dot of a 128-wide fragment tile with the bf16 tile `t` (rows r at row offset roff)
     auto tile_rowdot = [&](const float (&acc)[NK][4], const uint8_t* t, int rows, int roff, float& s0, float& s1) {
+        uint32_t w[2 * NK];
+        frag_load_sw<NK>(t, rows, roff + m0, nk0, w);
         float prod[NK][4];
 #pragma unroll
         for (int j = 0; j < NK; ++j)
 #pragma unroll
             for (int hh = 0; hh < 2; ++hh) {
-                const float2 v = ld_pair(t, rows, roff + m0 + frag_row(2 * hh), nk0 + frag_col(j, 0));
+                const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[2 * j + hh]));
                 prod[j][2 * hh] = acc[j][2 * hh] * v.x;
                 prod[j][2 * hh + 1] = acc[j][2 * hh + 1] * v.y;
             }
@@ -312,6 +337,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         uint8_t* sKt = sQK + 64 * 128;   // K: rows 64-127 of the 128-row tile
         const uint32_t uQK = smem_u32(sQK), uK = smem_u32(sKt);
+        // M^T dE [64][128] (after R3 until R5) in the other Q/K tile, which takes the next unit's
+        // Q and K only after R5
+        uint8_t* sMdE = sQKn;
+        const uint32_t uMdE = smem_u32(sMdE);
         const bool has_next = nxt.L > 0;
         const int L = cur.L, h = cur.h;
         const long long t0 = cur.t0, idx = cur.idx;
@@ -357,8 +386,8 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
             *qa = pack8(qv);
         }
-        // the next unit's Q/K tile (loaded below, after R1's issue) may still be the source of the
-        // previous unit's bulk dq, dk stores
+        // the other Q/K tile (M^T dE from R3 on, then the next unit's Q/K) may still be the source
+        // of the previous unit's bulk dq, dk stores
         if (tid == 0) bulk_wait_rows_read();
         publish_smem();
 
@@ -376,13 +405,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             tc_gemm_m64<false, true>(tmem + 256, uE, 64, udH, 128, 128, D, false);     // E dH'^T
             tc_gemm_m64<false, false>(tmem + 384, uK, 128, udH, 128, 128, D, false);   // K dH'
         }
-        // While R0 runs: the next unit's Q/K tile starts streaming in (its buffer was last read by
-        // the previous unit's staging copies, finished before this unit began), and <H, dH'> is
-        // formed (R1 reads the same two tiles; both only read them)
-        if (has_next) {
-            load_qk(sQKn, nxt);
-            cp_async_commit();
-        }
+        // While R0 runs: <H, dH'> (R1 reads the same two tiles; both only read them)
         {
             // the two tiles share one layout, so matching 16-byte chunks pair up
             float sacc = 0.f;
@@ -397,41 +420,53 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             for (int o = 16; o > 0; o >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, o);
             if (lane == 0) red[warp] = sacc;
         }
-        float acc_dq[NK][4], acc_dk[NK][4], de[NK][4];
+        float acc_dq[NK][4], acc_dk[NK][4];
         {
             const bool ok0 = mbar_wait_polls(smem_u32(&bar0), ph0, p.wait_ns);
             ph0 ^= 1;
             ok = !__syncthreads_or(!ok0);
             tc_fence_after();
         }
+        // Each epilogue below first forms what the next round reads (P, dE, M^T dE, M^T dW, dG),
+        // publishes it and lets thread 0 issue that round, then does the rest of its work (row and
+        // column partials, dv, the dq / dk parts) while the tensor core runs.
+        float sc[NL][4], dP[NL][4];
         if (ok) {
             // P = Tril(S * Gamma); S and dP arrive with one wait
-            float sc[NL][4], dP[NL][4];
             uint32_t rS[NL * 4], rP[NL * 4];
             tmem_issue<NL>(tq + 0 + nl0, rS);
             tmem_issue<NL>(tq + 64 + nl0, rP);
             tmem_wait();
             tmem_take<NL>(rS, sc);
             tmem_take<NL>(rP, dP);
+            float pv[NL][4];
 #pragma unroll
             for (int t = 0; t < NL; ++t)
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    const int r = m0 + frag_row(2 * hh), c = nl0 + frag_col(t, 0);
-                    const float gr = sG[r];
-                    const float v0 = (c <= r && r < L) ? sc[t][2 * hh] * __expf(gr - sG[c]) : 0.f;
-                    const float v1 = (c + 1 <= r && r < L) ? sc[t][2 * hh + 1] * __expf(gr - sG[c + 1]) : 0.f;
-                    st_pair(sP, 64, r, c, v0, v1);
+                for (int i = 0; i < 4; ++i) {
+                    const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
+                    pv[t][i] = (c <= r && r < L) ? sc[t][i] * __expf(sG[r] - sG[c]) : 0.f;
                 }
+            frag_store_sw<NL>(sP, 64, m0, nl0, pv);
+        }
+        publish_smem();
+
+        // ---------------- R2: P^T dO (dE = Kbar dH' + P^T dO) into the S and dP columns (read), behind
+        // R1; one commit covers both.  The commit is made even when R0's wait gave up, so that the
+        // give-up path finds R1 tracked on this barrier.
+        if (tid == 0) {
+            if (ok) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
+            tc_commit(smem_u32(&bar));
+        }
+        if (ok) {
             // dPhat = dP * Gamma (an R3 operand) and dP * P into the log-decay gradient; the
             // diagonal's decay factor is exactly 1 (no g-dependence), so it is left out rather
             // than added and cancelled
             float rs0 = 0.f, rs1 = 0.f;
-            float cs[NL][2];
+            float cs[NL][2], ph[NL][4];
 #pragma unroll
             for (int t = 0; t < NL; ++t) {
                 cs[t][0] = cs[t][1] = 0.f;
-                float ph[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
@@ -440,12 +475,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                     const float w = c < r ? dP[t][i] * sc[t][i] * gam : 0.f;
                     if (i < 2) rs0 += w; else rs1 += w;
                     cs[t][i & 1] += w;
-                    ph[i] = dP[t][i] * gam;
+                    ph[t][i] = dP[t][i] * gam;
                 }
-                const int c0 = nl0 + frag_col(t, 0);
-                st_pair(sdPh, 64, m0 + frag_row(0), c0, ph[0], ph[1]);
-                st_pair(sdPh, 64, m0 + frag_row(2), c0, ph[2], ph[3]);
             }
+            frag_store_sw<NL>(sdPh, 64, m0, nl0, ph);
             rs0 = quad_sum(rs0);
             rs1 = quad_sum(rs1);
             put_rows(3, rs0, rs1);
@@ -457,14 +490,8 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                     if ((lane >> 2) == 0) colp[(0 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
                 }
         }
-        publish_smem();
-
-        // ---------------- R2: P^T dO (dE = Kbar dH' + P^T dO) into the S and dP columns (read), behind
-        // R1; one commit covers both.  The commit is made even when R0's wait gave up, so that the
-        // give-up path finds R1 tracked on this barrier.
-        if (ok && tid == 0) tc_gemm_m64<true, true>(tmem + 0, uP, 64, udO, 64, 128, 64, false);
         {
-            const bool ok2 = ms.finish(tid);
+            const bool ok2 = ms.wait(tid);
             ok = ok && ok2;
         }
         // this unit's U^T, W^T (read by R5) into the dead dH'^T tile
@@ -474,25 +501,14 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         cp_async_commit();   // group A
         if (ok) {
-            // the three R1 products and R2's with one wait
-            uint32_t rq[NK * 4], rk[NK * 4], re[NK * 4];
-            tmem_issue<NK>(tq + 128 + nk0, rq);
-            tmem_issue<NK>(tq + 256 + nk0, rk);
+            // dE = Kbar dH' + P^T dO (over the dead E tile: an R3 operand)
+            float de[NK][4], t2[NK][4];
+            uint32_t re[NK * 4], rt[NK * 4];
             tmem_issue<NK>(tq + 384 + nk0, re);
+            tmem_issue<NK>(tq + 0 + nk0, rt);
             tmem_wait();
-            // dQ~ part Diag(gamma) dO H^T (its row dot with Q~, the log-decay gradient of the Q~ H
-            // term, is taken while R3 runs)
-            tmem_take<NK>(rq, acc_dq);
-#pragma unroll
-            for (int t = 0; t < NK; ++t) { acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb; }
-            // dK from Kbar: Diag(gamma_C / gamma_r) E dH'^T
-            tmem_take<NK>(rk, acc_dk);
-#pragma unroll
-            for (int t = 0; t < NK; ++t) { acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb; }
-            // Kbar dH' part of dE
             tmem_take<NK>(re, de);
-            float t2[NK][4];
-            tmem_frag<NK>(tq + 0 + nk0, t2);
+            tmem_take<NK>(rt, t2);
 #pragma unroll
             for (int t = 0; t < NK; ++t) {
                 de[t][0] = fmaf(de[t][0], sKa, t2[t][0]); de[t][1] = fmaf(de[t][1], sKa, t2[t][1]);
@@ -502,38 +518,46 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         publish_smem();
 
-        // ---------------- R3: M^T dE, K K^T, dPhat K, dPhat^T Q~
-        if (ok && tid == 0) {
-            tc_gemm_m64<true, true>(tmem + 0, uM, 64, udE, 64, 128, 64, false);        // M^T dE
-            tc_gemm_m64<false, false>(tmem + 128, uK, 128, uK, 128, 64, D, false);     // K K^T
-            tc_gemm_m64<false, true>(tmem + 256, udPh, 64, uK, 128, 128, 64, false);   // dPhat K
-            tc_gemm_m64<true, true>(tmem + 384, udPh, 64, uQK, 128, 128, 64, false);   // dPhat^T Q~
+        // ---------------- R3: M^T dE, dPhat^T Q~ (into the columns dE was read from)
+        if (tid == 0) {
+            if (ok) {
+                tc_gemm_m64<true, true>(tmem + 0, uM, 64, udE, 64, 128, 64, false);        // M^T dE
+                tc_gemm_m64<true, true>(tmem + 384, udPh, 64, uQK, 128, 128, 64, false);   // dPhat^T Q~
+            }
+            tc_commit(smem_u32(&bar));
         }
         if (ok) {
-            // while R3 runs: the row dots of the two R1 parts with Q~ and with K (used by the
+            // the other two R1 products: dQ~ part Diag(gamma) dO H^T and dK from Kbar,
+            // Diag(gamma_C / gamma_r) E dH'^T, with their row dots with Q~ and with K (used by the
             // per-position tail only)
+            uint32_t rq[NK * 4], rk[NK * 4];
+            tmem_issue<NK>(tq + 128 + nk0, rq);
+            tmem_issue<NK>(tq + 256 + nk0, rk);
+            tmem_wait();
+            tmem_take<NK>(rq, acc_dq);
+            tmem_take<NK>(rk, acc_dk);
+#pragma unroll
+            for (int t = 0; t < NK; ++t) {
+                acc_dq[t][0] *= eGa; acc_dq[t][1] *= eGa; acc_dq[t][2] *= eGb; acc_dq[t][3] *= eGb;
+                acc_dk[t][0] *= sKa; acc_dk[t][1] *= sKa; acc_dk[t][2] *= sKb; acc_dk[t][3] *= sKb;
+            }
             float s0, s1;
             tile_rowdot(acc_dq, sQK, 128, 0, s0, s1);
             put_rows(0, s0, s1);
             tile_rowdot(acc_dk, sQK, 128, 64, s0, s1);
             put_rows(1, s0, s1);
         }
-        ok = ok && ms.finish(tid);
+        {
+            const bool ok3 = ms.wait(tid);
+            ok = ok && ok3;
+        }
         if (ok && has_next) load_M(nxt);   // M's last reader was R3
         cp_async_commit();                  // group B
-        float gr[NL][4];
         if (ok) {
+            // M^T dE, unscaled and in bf16, over the dead dE tile: the R4 / R5 operand; and
+            // dV = Diag(beta) M^T dE staged over the dead E tile, direct dbeta = v . (M^T dE)
             float t3[NK][4], s0, s1;
-            {
-                // M^T dE: dV = Diag(beta) M^T dE, direct dbeta = v . (M^T dE); it stays, unscaled and
-                // in bf16, over the dead dE tile as the R4 / R5 operand
-                uint32_t rt[NK * 4], rg[NL * 4];
-                tmem_issue<NK>(tq + 0 + nk0, rt);
-                tmem_issue<NL>(tq + 128 + nl0, rg);
-                tmem_wait();
-                tmem_take<NK>(rt, t3);
-                tmem_take<NL>(rg, gr);
-            }
+            tmem_frag<NK>(tq + 0 + nk0, t3);
             frag_store_sw<NK>(sMdE, 64, m0, nk0, t3);
             tile_rowdot(t3, sV, 64, 0, s0, s1);
             put_rows(2, s0, s1);
@@ -541,39 +565,52 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
 #pragma unroll
             for (int t = 0; t < NK; ++t) { t3[t][0] *= ba; t3[t][1] *= ba; t3[t][2] *= bb; t3[t][3] *= bb; }
             frag_stage<NK>(stV, m0, nk0, t3);
-            // dq = dQ~ complete: dd partial = -k . dQ~ ; dk -= d dQ~
-            tmem_frag<NK>(tq + 256 + nk0, t3);
-#pragma unroll
-            for (int t = 0; t < NK; ++t)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    acc_dq[t][i] += t3[t][i];
-                    acc_dk[t][i] -= dh * acc_dq[t][i];
-                }
-            tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
-            put_rows(6, s0, s1);
         }
         publish_smem();
 
-        // ---------------- R4: (M^T dE) H^T = -M^T dW (dW = -dE H^T); the dv rows leave meanwhile
-        if (ok && tid == 0) tc_gemm_m64<false, true>(tmem + 0, uMdE, 64, uH, 128, 128, D, false);
-        if (ok) copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, (long long)p.H * D, stV, L, tid);
-        ok = ok && ms.finish(tid);
-        if (ok && has_next) {
-            load_E(nxt);    // the dv staging above was its last use
-            load_H(nxt);    // R4 was H^T's last reader
+        // ---------------- R4: (M^T dE) H^T = -M^T dW (dW = -dE H^T) into M^T dE's columns (read), and
+        // K K^T, dPhat K into the columns of the two R1 products read above
+        if (tid == 0) {
+            if (ok) {
+                tc_gemm_m64<false, true>(tmem + 0, uMdE, 64, uH, 128, 128, D, false);
+                tc_gemm_m64<false, false>(tmem + 128, uK, 128, uK, 128, 64, D, false);     // K K^T
+                tc_gemm_m64<false, true>(tmem + 256, udPh, 64, uK, 128, 128, 64, false);   // dPhat K
+            }
+            tc_commit(smem_u32(&bar));
         }
-        cp_async_commit();   // group C
+        if (ok) copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, (long long)p.H * D, stV, L, tid);   // dv rows
+        {
+            const bool ok4 = ms.wait(tid);
+            ok = ok && ok4;
+        }
+        if (ok && has_next) load_H(nxt);   // R4 was H^T's last reader
+        cp_async_commit();                  // group C
+        float t4[NK][4];
         if (ok) {
-            // W path: M^T dW scaled by btilde gamma_{r-1} goes to dk; its row dot with k feeds dbtilde
-            // and d g_{r-1}; M^T dW in bf16 over the dead dO tile as the R5 operand
-            float t4[NK][4], s0, s1;
+            // M^T dW in bf16 over the dead dO tile: the R5 operand
             tmem_frag<NK>(tq + 0 + nk0, t4);
 #pragma unroll
             for (int t = 0; t < NK; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) t4[t][i] = -t4[t][i];
             frag_store_sw<NK>(sMdW, 64, m0, nk0, t4);
+        }
+        cp_async_wait<2>();   // group A (U^T, W^T) has landed; B and C may still be in flight
+        publish_smem();
+
+        // ---------------- R5: M^T dM M^T = (M^T dE) U^T + (M^T dW) W^T, with dM = dE (Diag(beta) V)^T +
+        // dW (Diag(btilde gamma_{-1}) K)^T, U = M Diag(beta) V and W = M Diag(btilde gamma_{-1}) K
+        if (tid == 0) {
+            if (ok) {
+                tc_gemm_m64<false, true>(tmem + 192, uMdE, 64, uUt, 128, 64, D, false);
+                tc_gemm_m64<false, true>(tmem + 192, uMdW, 64, uWt, 128, 64, D, true);
+            }
+            tc_commit(smem_u32(&bar));
+        }
+        if (ok) {
+            // W path: M^T dW scaled by btilde gamma_{r-1} goes to dk; its row dot with k feeds dbtilde
+            // and d g_{r-1}
+            float s0, s1;
             tile_rowdot(t4, sQK, 128, 64, s0, s1);
             put_rows(7, s0, s1);
             const float wa = sWs[ra], wb = sWs[rb];
@@ -582,49 +619,85 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 acc_dk[t][0] += wa * t4[t][0]; acc_dk[t][1] += wa * t4[t][1];
                 acc_dk[t][2] += wb * t4[t][2]; acc_dk[t][3] += wb * t4[t][3];
             }
+            // dq = dQ~ complete (dPhat K from R4): dd partial = -k . dQ~ ; dk -= d dQ~
+            tmem_frag<NK>(tq + 256 + nk0, t4);
+#pragma unroll
+            for (int t = 0; t < NK; ++t)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    acc_dq[t][i] += t4[t][i];
+                    acc_dk[t][i] -= dh * acc_dq[t][i];
+                }
+            tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
+            put_rows(6, s0, s1);
         }
-        cp_async_wait<2>();   // group A (U^T, W^T) has landed; B and C may still be in flight
-        publish_smem();
-
-        // ---------------- R5: M^T dM M^T = (M^T dE) U^T + (M^T dW) W^T, with dM = dE (Diag(beta) V)^T +
-        // dW (Diag(btilde gamma_{-1}) K)^T, U = M Diag(beta) V and W = M Diag(btilde gamma_{-1}) K
-        if (ok && tid == 0) {
-            tc_gemm_m64<false, true>(tmem + 128, uMdE, 64, uUt, 128, 64, D, false);
-            tc_gemm_m64<false, true>(tmem + 128, uMdW, 64, uWt, 128, 64, D, true);
+        {
+            const bool ok5 = ms.wait(tid);
+            ok = ok && ok5;
         }
-        ok = ok && ms.finish(tid);
         if (ok && has_next) {
+            load_E(nxt);               // the dv rows (copied before R4's wait) were the E tile's last use
             load_dH(nxt);              // U^T and W^T are dead
             load_tok(sdO, p.dO, nxt);  // M^T dW is dead
+            load_qk(sQKn, nxt);        // M^T dE is dead (the previous unit's dq, dk stores have read
+                                       // this tile: the prologue waited for them)
         }
         cp_async_commit();   // group D
         if (ok) {
-            // dA = -(M^T dM M^T) on the strict lower triangle -> dG
-            float da[NL][4];
-            tmem_frag<NL>(tq + 128 + nl0, da);
-            float rb0 = 0.f, rb1 = 0.f, ra0 = 0.f, ra1 = 0.f;
-            float cs[NL][2];
+            // dA = -(M^T dM M^T) on the strict lower triangle -> dG (the R6 operand)
+            float dA[NL][4];
+            tmem_frag<NL>(tq + 192 + nl0, dA);
+            float g4[NL][4];
 #pragma unroll
-            for (int t = 0; t < NL; ++t) {
-                cs[t][0] = cs[t][1] = 0.f;
-                float g4[4];
+            for (int t = 0; t < NL; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
                     const bool strict = c < r && r < L;
                     const float gm = strict ? __expf(sGm1[r] - sG[c]) : 0.f;
-                    const float a = -da[t][i];
-                    const float uu = a * gm * gr[t][i];   // contributes to dbtilde_r
-                    // dA * Aval into the log-decay gradient; on the first sub-diagonal the decay
-                    // factor gamma_{r-1}/gamma_c is exactly 1, so it is left out (it would cancel)
+                    g4[t][i] = -dA[t][i] * sBt[r] * gm;
+                }
+            frag_store_sw<NL>(sdG, 64, m0, nl0, g4);
+        }
+        publish_smem();
+
+        // ---------------- R6: dK += dPhat^T Q~ (already in TMEM) + dG K + dG^T K
+        if (tid == 0) {
+            if (ok) {
+                tc_gemm_m64<false, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
+                tc_gemm_m64<true, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
+            }
+            tc_commit(smem_u32(&bar));
+        }
+        if (ok) {
+            // the R5 epilogue's partials, from dA and K K^T read again (R6 writes neither's
+            // columns): dA * Gram into dbtilde_r, dA * Aval into the log-decay gradient (on the
+            // first sub-diagonal the decay factor gamma_{r-1}/gamma_c is exactly 1, so it is left
+            // out: it would cancel)
+            float dA[NL][4], gr[NL][4];
+            {
+                uint32_t ra_[NL * 4], rg[NL * 4];
+                tmem_issue<NL>(tq + 192 + nl0, ra_);
+                tmem_issue<NL>(tq + 128 + nl0, rg);
+                tmem_wait();
+                tmem_take<NL>(ra_, dA);
+                tmem_take<NL>(rg, gr);
+            }
+            float rb0 = 0.f, rb1 = 0.f, ra0 = 0.f, ra1 = 0.f;
+            float cs[NL][2];
+#pragma unroll
+            for (int t = 0; t < NL; ++t) {
+                cs[t][0] = cs[t][1] = 0.f;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
+                    const bool strict = c < r && r < L;
+                    const float gm = strict ? __expf(sGm1[r] - sG[c]) : 0.f;
+                    const float uu = -dA[t][i] * gm * gr[t][i];   // contributes to dbtilde_r
                     const float w = c + 1 < r ? uu * sBt[r] : 0.f;
                     if (i < 2) { rb0 += uu; ra0 += w; } else { rb1 += uu; ra1 += w; }
                     cs[t][i & 1] += w;
-                    g4[i] = a * sBt[r] * gm;
                 }
-                const int c0 = nl0 + frag_col(t, 0);
-                st_pair(sdG, 64, m0 + frag_row(0), c0, g4[0], g4[1]);
-                st_pair(sdG, 64, m0 + frag_row(2), c0, g4[2], g4[3]);
             }
             rb0 = quad_sum(rb0); rb1 = quad_sum(rb1);
             ra0 = quad_sum(ra0); ra1 = quad_sum(ra1);
@@ -638,14 +711,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                     if ((lane >> 2) == 0) colp[(1 * 4 + wr) * 64 + nl0 + 8 * t + 2 * (lane & 3) + e] = v;
                 }
         }
-        publish_smem();
-
-        // ---------------- R6: dK += dPhat^T Q~ (already in TMEM) + dG K + dG^T K
-        if (ok && tid == 0) {
-            tc_gemm_m64<false, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
-            tc_gemm_m64<true, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
+        {
+            const bool ok6 = ms.wait(tid);
+            ok = ok && ok6;
         }
-        ok = ok && ms.finish(tid);
         if (ok && has_next) {
             load_tok(sV, p.v, nxt);   // dG (over V) is dead
             rin = load_rows(nxt);
