@@ -372,9 +372,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             sEm1[tid] = em1;
             sWs[tid] = bh * rin.be * fsc * em1;
         }
+        // Q~ = Q - d K (rows < 64; rows >= L are zero in both).  load_qk gives thread tid the Q/K
+        // chunks tid + 512 j, so the Q chunk and the K chunk (1024 further) that a thread updates
+        // here are its own copies: waiting for them takes no barrier.
         cp_async_wait<0>();
-        __syncthreads();
-        // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
         for (int e = tid; e < 64 * 16; e += kLocalThreads) {
             const int r = e >> 4, ch = e & 15;
             uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
@@ -430,24 +431,28 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         // Each epilogue below first forms what the next round reads (P, dE, M^T dE, M^T dW, dG),
         // publishes it and lets thread 0 issue that round, then does the rest of its work (row and
         // column partials, dv, the dq / dk parts) while the tensor core runs.
-        float sc[NL][4], dP[NL][4];
+        float sc[NL][4], ph[NL][4];
         if (ok) {
-            // P = Tril(S * Gamma); S and dP arrive with one wait
+            // P = Tril(S * Gamma) (the R2 operand) and dPhat = dP * Gamma (an R3 operand); S and dP
+            // arrive with one wait
             uint32_t rS[NL * 4], rP[NL * 4];
             tmem_issue<NL>(tq + 0 + nl0, rS);
             tmem_issue<NL>(tq + 64 + nl0, rP);
             tmem_wait();
             tmem_take<NL>(rS, sc);
-            tmem_take<NL>(rP, dP);
+            tmem_take<NL>(rP, ph);
             float pv[NL][4];
 #pragma unroll
             for (int t = 0; t < NL; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
-                    pv[t][i] = (c <= r && r < L) ? sc[t][i] * __expf(sG[r] - sG[c]) : 0.f;
+                    const float gam = (c <= r && r < L) ? __expf(sG[r] - sG[c]) : 0.f;
+                    pv[t][i] = sc[t][i] * gam;
+                    ph[t][i] *= gam;
                 }
             frag_store_sw<NL>(sP, 64, m0, nl0, pv);
+            frag_store_sw<NL>(sdPh, 64, m0, nl0, ph);
         }
         publish_smem();
 
@@ -459,26 +464,21 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             tc_commit(smem_u32(&bar));
         }
         if (ok) {
-            // dPhat = dP * Gamma (an R3 operand) and dP * P into the log-decay gradient; the
-            // diagonal's decay factor is exactly 1 (no g-dependence), so it is left out rather
-            // than added and cancelled
+            // dP * P = dPhat * S into the log-decay gradient; the diagonal's decay factor is exactly
+            // 1 (no g-dependence), so it is left out rather than added and cancelled
             float rs0 = 0.f, rs1 = 0.f;
-            float cs[NL][2], ph[NL][4];
+            float cs[NL][2];
 #pragma unroll
             for (int t = 0; t < NL; ++t) {
                 cs[t][0] = cs[t][1] = 0.f;
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = m0 + frag_row(i), c = nl0 + frag_col(t, i);
-                    const bool incl = c <= r && r < L;
-                    const float gam = incl ? __expf(sG[r] - sG[c]) : 0.f;
-                    const float w = c < r ? dP[t][i] * sc[t][i] * gam : 0.f;
+                    const float w = c < r ? ph[t][i] * sc[t][i] : 0.f;
                     if (i < 2) rs0 += w; else rs1 += w;
                     cs[t][i & 1] += w;
-                    ph[t][i] = dP[t][i] * gam;
                 }
             }
-            frag_store_sw<NL>(sdPh, 64, m0, nl0, ph);
             rs0 = quad_sum(rs0);
             rs1 = quad_sum(rs1);
             put_rows(3, rs0, rs1);
