@@ -140,6 +140,12 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
                           + P * (2 * C * C * dk * 7 + 2 * C * dk * dv * 4 + 2 * C * C * dv * 4 + 4 * C ** 3),
                           bytes=Pk * (2 * C * dk * es + C * C * es + 3 * C * f4 + 2 * C * dk * es + 2 * C * f4)
                           + P * (2 * C * dv * es + C * dv * es + 2 * dv * dk * es + C * dv * es))
+    if tc and not pk:
+        # the tcgen05 local-gradient kernel: S, K K^T per key head; per value head R1 (three
+        # C x dk x dv products), (M^T dE) H^T, P^T dO, M^T dE, dPhat K, dPhat^T Q~, dA from
+        # (M^T dE) U^T + (M^T dW) W^T and dG K, dG^T K; it also reads U^T and W^T
+        m["bwd_local"]["flops"] = Pk * 2 * 2 * C * C * dk + P * 2 * (4 * C * dk * dv + 5 * C * C * dk + 4 * C * C * dv)
+        m["bwd_local"]["bytes"] += P * (C * dv + C * dk) * es
     if pk:
         m["prep"]["bytes"] += Pk * C * dk * es
         m["bwd_local"]["bytes"] += Pk * 2 * C * dk * es
