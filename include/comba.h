@@ -222,7 +222,8 @@ comba_status_t comba_chunk_fwd_pk(const comba_shape_t *shape,
  * (storage type, written).  dk then holds only the gradient through the state
  * write; dd = -sum_t p_t . dq_t.  shape->flags must contain COMBA_PK and may add
  * COMBA_REUSE_FACTORS (after a pk forward with COMBA_SAVE_FACTORS on the same
- * workspace) and COMBA_IPLR.
+ * workspace and inputs; the backward then also reuses that forward's q - d p) and
+ * COMBA_IPLR.
  */
 comba_status_t comba_chunk_bwd_pk(const comba_shape_t *shape,
                                   const void *q, const void *k, const void *v, const void *p,

@@ -447,11 +447,15 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t* shape, const void* q, 
 }
 
 // Comba-pk: q - d p into the workspace and a zeroed d for the chunk kernels.
+// `reuse`: a backward reusing the saved factors of a forward on the same inputs and workspace,
+// which already holds q - d p and the zero d.
 static comba_status_t pk_prologue(const comba_shape_t* shape, const Layout& L, void* workspace, const void* q,
-                                  const void* p, const float* d, cudaStream_t s, void** qt, float** dz) {
+                                  const void* p, const float* d, cudaStream_t s, void** qt, float** dz,
+                                  bool reuse = false) {
     char* w = static_cast<char*>(workspace);
     *qt = w + L.qt;
     *dz = reinterpret_cast<float*>(w + L.dz);
+    if (reuse) return COMBA_OK;
     if (cudaMemsetAsync(*dz, 0, (size_t)shape->H * sizeof(float), s) != cudaSuccess) return COMBA_ERR_CUDA;
     if (comba::launch_pk_qtilde(q, p, d, *qt, (long long)shape->B * shape->T * shape->H, shape->H, shape->dk,
                                 shape->dtype == COMBA_BF16, s) != cudaSuccess)
@@ -503,7 +507,9 @@ comba_status_t comba_chunk_bwd_pk(const comba_shape_t* shape, const void* q, con
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
     void* qt;
     float* dz;
-    if ((st = pk_prologue(shape, L, workspace, q, p, d, s, &qt, &dz)) != COMBA_OK) return st;
+    if ((st = pk_prologue(shape, L, workspace, q, p, d, s, &qt, &dz, (shape->flags & COMBA_REUSE_FACTORS) != 0)) !=
+        COMBA_OK)
+        return st;
     PkArgs pk;
     pk.p = p; pk.d = d; pk.dp = dp;
     return backward_run(shape, L, workspace, qt, k, v, alpha, beta, b, dz, h0, dO, dhT, dq, dk, dv, dalpha, dbeta, db,

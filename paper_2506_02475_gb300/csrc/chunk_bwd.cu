@@ -837,11 +837,9 @@ static cudaError_t run_bwd(const ChunkParams& p, cudaStream_t s, int ev0) {
     }
     if ((e = launch_scan(a, sizeof(T) == 2, DK, DV, (long long)p.slots * p.H, s))) return e;
     mark(p, ev0 + 2, s);
-    if (tcp && !pk) {
-        if ((e = launch_bwd_local_tc(p, s))) return e;
+    if (tcp) {
+        if ((e = launch_bwd_local_tc(p, s))) return e;   // with or without Comba-pk feedback vectors
     } else if (p.slots > 0) {
-        // the mma.sync local kernel also serves Comba-pk on the tcgen05 path: it reads the same
-        // row-major E, M and transposed chunk states
         local<<<dim3(p.slots, p.H), 256, sm_loc, s>>>(p);
     }
     if ((e = cudaGetLastError())) return e;
@@ -867,7 +865,7 @@ cudaError_t launch_bwd(const ChunkParams& p, bool is_bf16, cudaStream_t s, int e
 
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk) {
     if (kernel == 0 && (use_tc_path(is_bf16, dk, dv) || dk == 256)) return 0;   // no additive-term kernel there
-    if (kernel == 1 && use_tc_path(is_bf16, dk, dv) && !pk) return local_tc_smem_bytes();
+    if (kernel == 1 && use_tc_path(is_bf16, dk, dv)) return local_tc_smem_bytes();
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? BPrepSmem<T, DK, DV>::bytes() : LocalSmem<T, DK, DV>::bytes();
     if (is_bf16) {

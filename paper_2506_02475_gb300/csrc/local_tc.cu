@@ -210,9 +210,17 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 // R6; the per-row scalars into registers), so the loads of consecutive units overlap the
 // tensor-core and epilogue work instead of every SM loading at the same moment.  U^T and W^T of
 // the unit itself load into the dH'^T tile once R1 has read it.
+//
+// PK: Comba-pk feedback vectors P (p.p, shaped like K).  They replace K as the Gram's left factor
+// (P K^T, formed in R5 here), in W = M Diag(btilde gamma_{-1}) P and in the correction q - d p
+// (applied to q before the chunk kernels, which see d = 0): the W path and the Gram's left factor
+// go to dp instead of dk (dp = dG K + Diag(btilde gamma_{-1}) M^T dW - d dq, finished from TMEM
+// at the end), dk takes dG^T P, and the row dots of dd and of the W path take p.  The P tile
+// lives over the M and P-matrix tiles from R3 to R6; the next unit's M then loads after R6.
+template <bool PK>
 __global__ void __launch_bounds__(kLocalThreads, 1)
     k_bwd_local_tc(ChunkParams p, long long units, const __grid_constant__ CUtensorMap tmDq,
-                   const __grid_constant__ CUtensorMap tmDk) {
+                   const __grid_constant__ CUtensorMap tmDk, const __grid_constant__ CUtensorMap tmDp) {
     using S = LocalTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar, bar0, stall_bar;   // bar0: R0; stall_bar: nothing arrives (COMBA_DIAG_STALL)
@@ -235,6 +243,8 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     uint8_t* sUt = sdHt;              // U^T, W^T [128][64] each, after R1 (dH'^T's readers) until R5
     uint8_t* sWt = sdHt + 16384;
     uint8_t* sdG = sV + 8192;         // dG [64][64], after R3 until R6
+    uint8_t* sPf = sM;                // Comba-pk: P [64][128] over the M and P-matrix tiles, R3 to R6
+    uint8_t* stP = sdE;               // Comba-pk: dp staging, at the end (dPhat is dead)
     float* sG = reinterpret_cast<float*>(sm + S::OF);
     float* sGm1 = sG + 64;
     float* sBe = sG + 128;
@@ -249,7 +259,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     const uint32_t udO = smem_u32(sdO), uE = smem_u32(sE), uH = smem_u32(sHt), udH = smem_u32(sdHt),
                    uM = smem_u32(sM), uP = smem_u32(sP), udE = smem_u32(sdEt), udPh = smem_u32(sdPh),
                    uMdW = smem_u32(sMdW), uUt = smem_u32(sUt), uWt = smem_u32(sWt),
-                   udG = smem_u32(sdG);
+                   udG = smem_u32(sdG), uPf = smem_u32(sPf);
 
     const int Hk = p.H / p.vg;   // key heads: q, k, alpha, beta, b, d of value head h are key head h / vg's
     auto load_qk = [&](uint8_t* dst, const UnitRef& x) {
@@ -281,6 +291,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     auto load_H = [&](const UnitRef& x) { load_sw(sHt, 128, D, (const bf16*)p.Hb + x.idx * D * D, D, 128, tid, kLocalThreads); };
     auto load_E = [&](const UnitRef& x) { load_sw(sE, 64, D, (const bf16*)p.Eb + x.idx * 64 * D, D, 64, tid, kLocalThreads); };
     auto load_M = [&](const UnitRef& x) { load_sw(sM, 64, 64, (const bf16*)p.Mb + x.idx * 4096, 64, 64, tid, kLocalThreads); };
+    auto load_pf = [&](const UnitRef& x) {
+        load_sw(sPf, 64, D, (const bf16*)p.p + (x.t0 * Hk + x.h / p.vg) * D, (long long)Hk * D, x.L, tid, kLocalThreads);
+    };
 
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
@@ -551,7 +564,11 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             const bool ok3 = ms.wait(tid);
             ok = ok && ok3;
         }
-        if (ok && has_next) load_M(nxt);   // M's last reader was R3
+        if constexpr (PK) {
+            if (ok) load_pf(cur);           // over M (its last reader was R3) and the P matrix
+        } else {
+            if (ok && has_next) load_M(nxt);   // M's last reader was R3
+        }
         cp_async_commit();                  // group B
         if (ok) {
             // M^T dE, unscaled and in bf16, over the dead dE tile: the R4 / R5 operand; and
@@ -573,7 +590,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         if (tid == 0) {
             if (ok) {
                 tc_gemm_m64<false, true>(tmem + 0, uMdE, 64, uH, 128, 128, D, false);
-                tc_gemm_m64<false, false>(tmem + 128, uK, 128, uK, 128, 64, D, false);     // K K^T
+                if constexpr (!PK) tc_gemm_m64<false, false>(tmem + 128, uK, 128, uK, 128, 64, D, false);   // K K^T
                 tc_gemm_m64<false, true>(tmem + 256, udPh, 64, uK, 128, 128, 64, false);   // dPhat K
             }
             tc_commit(smem_u32(&bar));
@@ -595,7 +612,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 for (int i = 0; i < 4; ++i) t4[t][i] = -t4[t][i];
             frag_store_sw<NK>(sMdW, 64, m0, nk0, t4);
         }
-        cp_async_wait<2>();   // group A (U^T, W^T) has landed; B and C may still be in flight
+        // group A (U^T, W^T) has landed, and with Comba-pk group B (P); the next unit's tiles may still
+        // be in flight
+        if constexpr (PK) cp_async_wait<1>();
+        else cp_async_wait<2>();
         publish_smem();
 
         // ---------------- R5: M^T dM M^T = (M^T dE) U^T + (M^T dW) W^T, with dM = dE (Diag(beta) V)^T +
@@ -604,6 +624,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             if (ok) {
                 tc_gemm_m64<false, true>(tmem + 192, uMdE, 64, uUt, 128, 64, D, false);
                 tc_gemm_m64<false, true>(tmem + 192, uMdW, 64, uWt, 128, 64, D, true);
+                if constexpr (PK) tc_gemm_m64<false, false>(tmem + 128, uPf, 64, uK, 128, 64, D, false);   // P K^T
             }
             tc_commit(smem_u32(&bar));
         }
@@ -611,14 +632,18 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             // W path: M^T dW scaled by btilde gamma_{r-1} goes to dk; its row dot with k feeds dbtilde
             // and d g_{r-1}
             float s0, s1;
-            tile_rowdot(t4, sQK, 128, 64, s0, s1);
-            put_rows(7, s0, s1);
-            const float wa = sWs[ra], wb = sWs[rb];
+            if constexpr (PK) {
+                tile_rowdot(t4, sPf, 64, 0, s0, s1);   // with p; M^T dW stays in TMEM for dp
+            } else {
+                tile_rowdot(t4, sQK, 128, 64, s0, s1);
+                const float wa = sWs[ra], wb = sWs[rb];
 #pragma unroll
-            for (int t = 0; t < NK; ++t) {
-                acc_dk[t][0] += wa * t4[t][0]; acc_dk[t][1] += wa * t4[t][1];
-                acc_dk[t][2] += wb * t4[t][2]; acc_dk[t][3] += wb * t4[t][3];
+                for (int t = 0; t < NK; ++t) {
+                    acc_dk[t][0] += wa * t4[t][0]; acc_dk[t][1] += wa * t4[t][1];
+                    acc_dk[t][2] += wb * t4[t][2]; acc_dk[t][3] += wb * t4[t][3];
+                }
             }
+            put_rows(7, s0, s1);
             // dq = dQ~ complete (dPhat K from R4): dd partial = -k . dQ~ ; dk -= d dQ~
             tmem_frag<NK>(tq + 256 + nk0, t4);
 #pragma unroll
@@ -626,9 +651,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     acc_dq[t][i] += t4[t][i];
-                    acc_dk[t][i] -= dh * acc_dq[t][i];
+                    if constexpr (!PK) acc_dk[t][i] -= dh * acc_dq[t][i];
                 }
-            tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
+            if constexpr (PK) tile_rowdot(acc_dq, sPf, 64, 0, s0, s1);   // dd = -p . dq
+            else tile_rowdot(acc_dq, sQK, 128, 64, s0, s1);
             put_rows(6, s0, s1);
         }
         {
@@ -661,11 +687,17 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         publish_smem();
 
-        // ---------------- R6: dK += dPhat^T Q~ (already in TMEM) + dG K + dG^T K
+        // ---------------- R6: dK += dPhat^T Q~ (already in TMEM) + dG K + dG^T K; with Comba-pk dG K is
+        // dp's (into the dPhat K columns, read) and dk takes dG^T P
         if (tid == 0) {
             if (ok) {
-                tc_gemm_m64<false, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
-                tc_gemm_m64<true, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
+                if constexpr (PK) {
+                    tc_gemm_m64<false, true>(tmem + 256, udG, 64, uK, 128, 128, 64, false);
+                    tc_gemm_m64<true, true>(tmem + 384, udG, 64, uPf, 64, 128, 64, true);
+                } else {
+                    tc_gemm_m64<false, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
+                    tc_gemm_m64<true, true>(tmem + 384, udG, 64, uK, 128, 128, 64, true);
+                }
             }
             tc_commit(smem_u32(&bar));
         }
@@ -717,6 +749,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         if (ok && has_next) {
             load_tok(sV, p.v, nxt);   // dG (over V) is dead
+            if constexpr (PK) load_M(nxt);   // P (over M) is dead
             rin = load_rows(nxt);
         }
         cp_async_commit();   // group E
@@ -739,6 +772,25 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 frag_stage<NK>(sQK, m0, nk0, acc_dq);
                 frag_stage<NK>(sQK + 16384, m0, nk0, acc_dk);
             }
+            if constexpr (PK) {
+                // dp = dG K + Diag(btilde gamma_{-1}) M^T dW - d dq, the first two still in TMEM (R4 left
+                // (M^T dE) H^T = -M^T dW there)
+                float dpv[NK][4], t7[NK][4];
+                uint32_t rg[NK * 4], rw[NK * 4];
+                tmem_issue<NK>(tq + 256 + nk0, rg);
+                tmem_issue<NK>(tq + 0 + nk0, rw);
+                tmem_wait();
+                tmem_take<NK>(rg, dpv);
+                tmem_take<NK>(rw, t7);
+                const float wa = sWs[ra], wb = sWs[rb], dfb = p.d_fb[h / p.vg];
+#pragma unroll
+                for (int t = 0; t < NK; ++t)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        dpv[t][i] -= (i < 2 ? wa : wb) * t7[t][i] + dfb * acc_dq[t][i];
+                if (L == kChunk) frag_store_sw<NK>(stP, 64, m0, nk0, dpv);
+                else frag_stage<NK>(stP, m0, nk0, dpv);
+            }
         }
         if (L == kChunk) fence_async_smem();
         __syncthreads();
@@ -749,6 +801,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                     for (int half = 0; half < 2; ++half) {
                         tma_store_rows(&tmDq, 64 * half, h, (int)t0, smem_u32(sQK) + half * 8192);
                         tma_store_rows(&tmDk, 64 * half, h, (int)t0, smem_u32(sQK + 16384) + half * 8192);
+                        if constexpr (PK) tma_store_rows(&tmDp, 64 * half, h, (int)t0, smem_u32(stP) + half * 8192);
                     }
                     bulk_commit_rows();
                 }
@@ -756,6 +809,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 const long long ld = (long long)p.H * D;
                 copy_stage_rows((bf16*)p.dq + (t0 * p.H + h) * D, ld, sQK, L, tid);
                 copy_stage_rows((bf16*)p.dkk + (t0 * p.H + h) * D, ld, sQK + 16384, L, tid);
+                if constexpr (PK) copy_stage_rows((bf16*)p.dpp + (t0 * p.H + h) * D, ld, stP, L, tid);
             }
         }
 
@@ -863,17 +917,24 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
 
 cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s) {
     const size_t sm = tc::LocalTcSmem::bytes();
-    cudaError_t e = cudaFuncSetAttribute(tc::k_bwd_local_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    const bool pk = p.p != nullptr;
+    auto kern = pk ? tc::k_bwd_local_tc<true> : tc::k_bwd_local_tc<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     const long long units = (long long)p.slots * p.H;
     const int grid = (int)(units < nsm ? units : nsm);   // one resident CTA per SM
-    CUtensorMap tq, tk;   // dq, dk [tokens][value heads][128]
+    CUtensorMap tq, tk, tp;   // dq, dk (and dp) [tokens][value heads][128]
     if (!make_bf16_token_map(&tq, p.dq, p.Ttot, p.H, tc::D) ||
         !make_bf16_token_map(&tk, p.dkk, p.Ttot, p.H, tc::D))
         return cudaErrorInvalidValue;
-    if (grid > 0) tc::k_bwd_local_tc<<<grid, tc::kLocalThreads, sm, s>>>(p, units, tq, tk);
+    if (pk) {
+        if (!p.dpp || !make_bf16_token_map(&tp, p.dpp, p.Ttot, p.H, tc::D)) return cudaErrorInvalidValue;
+    } else {
+        tp = tq;   // not used
+    }
+    if (grid > 0) kern<<<grid, tc::kLocalThreads, sm, s>>>(p, units, tq, tk, tp);
     return cudaGetLastError();
 }
 
