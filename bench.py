@@ -161,11 +161,11 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 94_748, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "9d79a929b96fdafe"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_505, ('scan.cu', 'common.cuh', 'params.cuh'), "719c2e63f7fb0962"),
-    "output": ("k_output_tc", 130_306, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "9d79a929b96fdafe"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_758, ('scan.cu', 'common.cuh', 'params.cuh'), "719c2e63f7fb0962"),
-    "bwd_local": ("k_bwd_local_tc", 193_601, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "ae17b319a7584d5f"),
+    "prep": ("k_prep_tc", 94_609, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c1622ec1d7a80419"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_570, ('scan.cu', 'common.cuh', 'params.cuh'), "da98cd7442c7cea5"),
+    "output": ("k_output_tc", 130_248, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "c1622ec1d7a80419"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_733, ('scan.cu', 'common.cuh', 'params.cuh'), "da98cd7442c7cea5"),
+    "bwd_local": ("k_bwd_local_tc", 228_351, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "05aeef4842d50ddd"),
 }
 DECODE_TRAFFIC = (481_439_744, ('decode.cu', 'common.cuh', 'params.cuh'), "2df9a51b0d0f5a9d")   # whole Bd=256 H=16 launch
 
