@@ -35,6 +35,7 @@
 namespace comba {
 
 bool make_bf16_token_map(CUtensorMap* m, const void* base, long long tokens, int heads, int cols);
+bool make_bf16_map(CUtensorMap* m, const void* base, long long rows, int cols, int box_rows);
 
 namespace tc {
 
@@ -217,13 +218,26 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 // go to dp instead of dk (dp = dG K + Diag(btilde gamma_{-1}) M^T dW - d dq, finished from TMEM
 // at the end), dk takes dG^T P, and the row dots of dd and of the W path take p.  The P tile
 // lives over the M and P-matrix tiles from R3 to R6; the next unit's M then loads after R6.
+// Tensor maps of the kernel's TMA traffic (128-byte swizzle, 64-column boxes): the dq, dk, dp
+// stores and every tile load.  Token tensors [tokens][heads][128] take {64, 1, 64} boxes; the
+// workspace tiles are 2D views [units * rows][cols] with boxes of a tile's rows.
+struct LocalMaps {
+    CUtensorMap dq, dk, dp;           // stores
+    CUtensorMap q, k, p, v, dO;       // token tiles (q, k, p per key head; v, dO per value head)
+    CUtensorMap e, h, dh, m, u, w;    // workspace: E [64][128], H^T, dH'^T [128][128], M [64][64],
+                                      // U^T, W^T [128][64]
+};
+
 template <bool PK>
 __global__ void __launch_bounds__(kLocalThreads, 1)
-    k_bwd_local_tc(ChunkParams p, long long units, const __grid_constant__ CUtensorMap tmDq,
-                   const __grid_constant__ CUtensorMap tmDk, const __grid_constant__ CUtensorMap tmDp) {
+    k_bwd_local_tc(ChunkParams p, long long units, const __grid_constant__ LocalMaps mp) {
     using S = LocalTcSmem;
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar, bar0, stall_bar;   // bar0: R0; stall_bar: nothing arrives (COMBA_DIAG_STALL)
+    // TMA arrival: ldn[0..3] a unit's tiles, in the four groups the previous unit prefetches them in
+    // (M; H^T; E, dH'^T, dO, Q/K; V, and with Comba-pk M), ldu its U^T / W^T, ldp its P (Comba-pk).
+    // Each completes one phase per unit that has rows.
+    __shared__ uint64_t ldn[4], ldu, ldp;
     __shared__ uint32_t tbase;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wr = warp & 3, wc = warp >> 2, m0 = 16 * wr;
@@ -262,16 +276,64 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                    udG = smem_u32(sdG), uPf = smem_u32(sPf);
 
     const int Hk = p.H / p.vg;   // key heads: q, k, alpha, beta, b, d of value head h are key head h / vg's
-    auto load_qk = [&](uint8_t* dst, const UnitRef& x) {
-        const bf16* qg = (const bf16*)p.q + (x.t0 * Hk + x.h / p.vg) * D;
-        const bf16* kg = (const bf16*)p.k + (x.t0 * Hk + x.h / p.vg) * D;
-        for (int e = tid; e < 128 * 16; e += kLocalThreads) {
-            const int r = e >> 4, ch = e & 15, rr = r & 63;
-            const bool okr = rr < x.L;
-            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * Hk * D + ch * 8;
-            cp_async16(dst + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
+    // TMA issue (thread kTma).  Q rows 0-63 and K rows 64-127 of a 128-row tile: K halves 16 KB apart.
+    constexpr int kTma = 32;
+    auto tma_qk = [&](uint8_t* dst, const UnitRef& x, uint32_t mb) {
+        const int hk = x.h / p.vg, t0x = (int)x.t0;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            tma_load_3d(smem_u32(dst) + half * 16384, &mp.q, 64 * half, hk, t0x, mb);
+            tma_load_3d(smem_u32(dst) + 8192 + half * 16384, &mp.k, 64 * half, hk, t0x, mb);
         }
     };
+    auto tma_tok = [&](uint8_t* dst, const CUtensorMap* m, int head, const UnitRef& x, uint32_t mb) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) tma_load_3d(smem_u32(dst) + half * 8192, m, 64 * half, head, (int)x.t0, mb);
+    };
+    auto tma_e = [&](const UnitRef& x, uint32_t mb) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) tma_load_2d(smem_u32(sE) + half * 8192, &mp.e, 64 * half, (int)(x.idx * 64), mb);
+    };
+    auto tma_sq = [&](uint8_t* dst, const CUtensorMap* m, const UnitRef& x, uint32_t mb) {   // H^T or dH'^T
+#pragma unroll
+        for (int half = 0; half < 2; ++half) tma_load_2d(smem_u32(dst) + half * 16384, m, 64 * half, (int)(x.idx * 128), mb);
+    };
+    auto tma_m = [&](const UnitRef& x, uint32_t mb) { tma_load_2d(smem_u32(sM), &mp.m, 0, (int)(x.idx * 64), mb); };
+    // a unit's four tile groups (phase completions of ldn[0..3])
+    auto issue_n0 = [&](const UnitRef& x, bool m_here) {
+        const uint32_t mb = smem_u32(&ldn[0]);
+        mbar_expect_tx(mb, m_here ? 8192u : 0u);
+        if (m_here) tma_m(x, mb);
+    };
+    auto issue_n1 = [&](const UnitRef& x) {
+        const uint32_t mb = smem_u32(&ldn[1]);
+        mbar_expect_tx(mb, 32768u);
+        tma_sq(sHt, &mp.h, x, mb);
+    };
+    auto issue_n2 = [&](uint8_t* qk, const UnitRef& x) {
+        const uint32_t mb = smem_u32(&ldn[2]);
+        mbar_expect_tx(mb, 16384u + 32768u + 16384u + 32768u);
+        tma_e(x, mb);
+        tma_sq(sdHt, &mp.dh, x, mb);
+        tma_tok(sdO, &mp.dO, x.h, x, mb);
+        tma_qk(qk, x, mb);
+    };
+    auto issue_n3 = [&](const UnitRef& x, bool m_here) {
+        const uint32_t mb = smem_u32(&ldn[3]);
+        mbar_expect_tx(mb, 16384u + (m_here ? 8192u : 0u));
+        tma_tok(sV, &mp.v, x.h, x, mb);
+        if (m_here) tma_m(x, mb);
+    };
+    // rows L..63 of a token tile hold the next sequence's tokens (or the zero fill past the tensor):
+    // zeroed by all threads after the tile has landed (a sequence's last chunk only)
+    auto zero_rows = [&](uint8_t* t, int rows, int L) {
+        for (int e = tid; e < (64 - L) * 16; e += kLocalThreads) {
+            const int r = L + (e >> 4), ch = e & 15;
+            *reinterpret_cast<uint4*>(t + sw128_offset(r, 8 * ch, rows)) = make_uint4(0, 0, 0, 0);
+        }
+    };
+    uint32_t pend = 0;   // thread kTma: barriers with loads issued and not yet waited on (bit i: ldn[i],
+                         // 4: ldu, 5: ldp), drained on the give-up path
     // per-row scalars of a unit (rows tid < 64): log-decay G_r, G_{r-1}, beta, alpha
     struct RowIn { float g, gm1, be, al; };
     auto load_rows = [&](const UnitRef& x) {
@@ -284,21 +346,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         return r;
     };
-    auto load_tok = [&](uint8_t* dst, const void* base, const UnitRef& x) {
-        load_sw(dst, 64, D, (const bf16*)base + (x.t0 * p.H + x.h) * D, (long long)p.H * D, x.L, tid, kLocalThreads);
-    };
-    auto load_dH = [&](const UnitRef& x) { load_sw(sdHt, 128, D, (const bf16*)p.dHb + x.idx * D * D, D, 128, tid, kLocalThreads); };
-    auto load_H = [&](const UnitRef& x) { load_sw(sHt, 128, D, (const bf16*)p.Hb + x.idx * D * D, D, 128, tid, kLocalThreads); };
-    auto load_E = [&](const UnitRef& x) { load_sw(sE, 64, D, (const bf16*)p.Eb + x.idx * 64 * D, D, 64, tid, kLocalThreads); };
-    auto load_M = [&](const UnitRef& x) { load_sw(sM, 64, 64, (const bf16*)p.Mb + x.idx * 4096, 64, 64, tid, kLocalThreads); };
-    auto load_pf = [&](const UnitRef& x) {
-        load_sw(sPf, 64, D, (const bf16*)p.p + (x.t0 * Hk + x.h / p.vg) * D, (long long)Hk * D, x.L, tid, kLocalThreads);
-    };
-
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
         mbar_init(smem_u32(&bar0), 1);
         mbar_init(smem_u32(&stall_bar), 1);
+        for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&ldn[i]), 1);
+        mbar_init(smem_u32(&ldu), 1);
+        mbar_init(smem_u32(&ldp), 1);
         mbar_fence_init();
     }
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 512);
@@ -332,6 +386,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
 
     bool ok = true;
     bool pre = false;   // this unit's tiles and row scalars were requested by the previous unit
+    uint32_t lph = 0;   // phase parity of the TMA barriers for the current unit
     long long u = blockIdx.x;
     UnitRef cur = u < units ? unit_ref(p, u) : UnitRef{0, 0, 0, 0};
     RowIn rin{0.f, 0.f, 0.f, 1.f};
@@ -362,14 +417,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             // a bulk store of dq, dk two units back may still read this tile
             if (tid == 0) bulk_wait_rows_read();
             __syncthreads();
-            load_qk(sQK, cur);
-            load_tok(sdO, p.dO, cur);
-            load_E(cur);
-            load_H(cur);
-            load_dH(cur);
-            load_tok(sV, p.v, cur);
-            load_M(cur);
-            cp_async_commit();
+            if (tid == kTma) {
+                issue_n0(cur, true);
+                issue_n1(cur);
+                issue_n2(sQK, cur);
+                issue_n3(cur, false);
+                pend |= 15u;
+            }
             rin = load_rows(cur);
         }
         const float bh = p.b ? p.b[h / p.vg] : 1.f;
@@ -385,11 +439,32 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             sEm1[tid] = em1;
             sWs[tid] = bh * rin.be * fsc * em1;
         }
-        // Q~ = Q - d K (rows < 64; rows >= L are zero in both).  load_qk gives thread tid the Q/K
-        // chunks tid + 512 j, so the Q chunk and the K chunk (1024 further) that a thread updates
-        // here are its own copies: waiting for them takes no barrier.
-        cp_async_wait<0>();
-        for (int e = tid; e < 64 * 16; e += kLocalThreads) {
+        // the unit's tiles have landed (all four groups)
+        {
+            bool okl = true;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) okl = mbar_wait_polls(smem_u32(&ldn[i]), lph, p.wait_ns) && okl;
+            if (okl && tid == kTma) pend &= ~15u;
+            ok = !__syncthreads_or(!okl);
+            if (!ok) {   // give up on the unit: let its copies finish before leaving
+                if (tid == kTma) {
+                    for (int i = 0; i < 4; ++i)
+                        if (pend & (1u << i)) mbar_drain(smem_u32(&ldn[i]), lph);
+                    pend = 0;
+                }
+                if (tid == 0) flag_error(p);
+                break;
+            }
+        }
+        // rows past a short chunk: zero in Q, K, dO and V (Q~ below covers rows < L only)
+        if (L < kChunk) {
+            zero_rows(sQK, 128, L);
+            zero_rows(sQK + 64 * 128, 128, L);
+            zero_rows(sdO, 64, L);
+            zero_rows(sV, 64, L);
+        }
+        // Q~ = Q - d K (rows < L)
+        for (int e = tid; e < L * 16; e += kLocalThreads) {
             const int r = e >> 4, ch = e & 15;
             uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
             const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
@@ -508,11 +583,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             ok = ok && ok2;
         }
         // this unit's U^T, W^T (read by R5) into the dead dH'^T tile
-        if (ok) {
-            load_sw(sUt, 128, 64, (const bf16*)p.Ub + idx * D * 64, 64, 128, tid, kLocalThreads);
-            load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid, kLocalThreads);
+        if (ok && tid == kTma) {
+            const uint32_t mb = smem_u32(&ldu);
+            mbar_expect_tx(mb, 32768u);
+            tma_load_2d(uUt, &mp.u, 0, (int)(idx * 128), mb);
+            tma_load_2d(uWt, &mp.w, 0, (int)(idx * 128), mb);
+            pend |= 16u;
         }
-        cp_async_commit();   // group A
         if (ok) {
             // dE = Kbar dH' + P^T dO (over the dead E tile: an R3 operand)
             float de[NK][4], t2[NK][4];
@@ -564,12 +641,17 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             const bool ok3 = ms.wait(tid);
             ok = ok && ok3;
         }
-        if constexpr (PK) {
-            if (ok) load_pf(cur);           // over M (its last reader was R3) and the P matrix
-        } else {
-            if (ok && has_next) load_M(nxt);   // M's last reader was R3
+        if (ok && tid == kTma) {
+            if constexpr (PK) {
+                // this unit's P over M (its last reader was R3) and the P matrix; the next unit's M
+                // comes after R6
+                const uint32_t mb = smem_u32(&ldp);
+                mbar_expect_tx(mb, 16384u);
+                tma_tok(sPf, &mp.p, h / p.vg, cur, mb);
+                pend |= 32u;
+            }
+            if (has_next) { issue_n0(nxt, !PK); pend |= 1u; }   // M's last reader was R3
         }
-        cp_async_commit();                  // group B
         if (ok) {
             // M^T dE, unscaled and in bf16, over the dead dE tile: the R4 / R5 operand; and
             // dV = Diag(beta) M^T dE staged over the dead E tile, direct dbeta = v . (M^T dE)
@@ -600,8 +682,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             const bool ok4 = ms.wait(tid);
             ok = ok && ok4;
         }
-        if (ok && has_next) load_H(nxt);   // R4 was H^T's last reader
-        cp_async_commit();                  // group C
+        if (ok && has_next && tid == kTma) { issue_n1(nxt); pend |= 2u; }   // R4 was H^T's last reader
         float t4[NK][4];
         if (ok) {
             // M^T dW in bf16 over the dead dO tile: the R5 operand
@@ -612,11 +693,18 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 for (int i = 0; i < 4; ++i) t4[t][i] = -t4[t][i];
             frag_store_sw<NK>(sMdW, 64, m0, nk0, t4);
         }
-        // group A (U^T, W^T) has landed, and with Comba-pk group B (P); the next unit's tiles may still
-        // be in flight
-        if constexpr (PK) cp_async_wait<1>();
-        else cp_async_wait<2>();
-        publish_smem();
+        // U^T, W^T have landed, and with Comba-pk P (its rows past a short chunk zeroed)
+        {
+            bool okl = ok && mbar_wait_polls(smem_u32(&ldu), lph, p.wait_ns);
+            if constexpr (PK) okl = okl && mbar_wait_polls(smem_u32(&ldp), lph, p.wait_ns);
+            if (okl && tid == kTma) pend &= ~48u;
+            if constexpr (PK)
+                if (okl && L < kChunk) zero_rows(sPf, 64, L);
+            fence_async_smem();
+            tc_fence_before();
+            ok = ok && !__syncthreads_or(!okl);
+            tc_fence_after();
+        }
 
         // ---------------- R5: M^T dM M^T = (M^T dE) U^T + (M^T dW) W^T, with dM = dE (Diag(beta) V)^T +
         // dW (Diag(btilde gamma_{-1}) K)^T, U = M Diag(beta) V and W = M Diag(btilde gamma_{-1}) K
@@ -661,14 +749,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             const bool ok5 = ms.wait(tid);
             ok = ok && ok5;
         }
-        if (ok && has_next) {
-            load_E(nxt);               // the dv rows (copied before R4's wait) were the E tile's last use
-            load_dH(nxt);              // U^T and W^T are dead
-            load_tok(sdO, p.dO, nxt);  // M^T dW is dead
-            load_qk(sQKn, nxt);        // M^T dE is dead (the previous unit's dq, dk stores have read
-                                       // this tile: the prologue waited for them)
-        }
-        cp_async_commit();   // group D
+        // the next unit's E (the dv rows, copied before R4's wait, were the E tile's last use), dH'^T
+        // (U^T and W^T are dead), dO (M^T dW is dead) and Q/K (M^T dE is dead; the previous unit's
+        // dq, dk stores have read this tile: the prologue waited for them)
+        if (ok && has_next && tid == kTma) { issue_n2(sQKn, nxt); pend |= 4u; }
         if (ok) {
             // dA = -(M^T dM M^T) on the strict lower triangle -> dG (the R6 operand)
             float dA[NL][4];
@@ -748,11 +832,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             ok = ok && ok6;
         }
         if (ok && has_next) {
-            load_tok(sV, p.v, nxt);   // dG (over V) is dead
-            if constexpr (PK) load_M(nxt);   // P (over M) is dead
+            if (tid == kTma) { issue_n3(nxt, PK); pend |= 8u; }   // dG (over V) is dead, and P (over M)
             rin = load_rows(nxt);
         }
-        cp_async_commit();   // group E
         if (ok) {
             float t6[NK][4];
             tmem_frag<NK>(tq + 384 + nk0, t6);
@@ -799,9 +881,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 if (tid == 0) {
 #pragma unroll
                     for (int half = 0; half < 2; ++half) {
-                        tma_store_rows(&tmDq, 64 * half, h, (int)t0, smem_u32(sQK) + half * 8192);
-                        tma_store_rows(&tmDk, 64 * half, h, (int)t0, smem_u32(sQK + 16384) + half * 8192);
-                        if constexpr (PK) tma_store_rows(&tmDp, 64 * half, h, (int)t0, smem_u32(stP) + half * 8192);
+                        tma_store_rows(&mp.dq, 64 * half, h, (int)t0, smem_u32(sQK) + half * 8192);
+                        tma_store_rows(&mp.dk, 64 * half, h, (int)t0, smem_u32(sQK + 16384) + half * 8192);
+                        if constexpr (PK) tma_store_rows(&mp.dp, 64 * half, h, (int)t0, smem_u32(stP) + half * 8192);
                     }
                     bulk_commit_rows();
                 }
@@ -901,10 +983,18 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         __syncthreads();   // the staging tile read above takes the Q/K copies of the unit after next
         pre = has_next;
+        lph ^= 1;
         u = un;
         cur = nxt;
     }
-    cp_async_wait<0>();   // no copy is still writing shared memory at exit
+    // no tile copy is still writing shared memory at exit (after a give-up, the next unit's tiles are
+    // in the phase after this one's, U^T / W^T and P in this one's)
+    if (tid == kTma && pend) {
+        for (int i = 0; i < 4; ++i)
+            if (pend & (1u << i)) mbar_drain(smem_u32(&ldn[i]), lph);
+        if (pend & 16u) mbar_drain(smem_u32(&ldu), lph ^ 1);
+        if (pend & 32u) mbar_drain(smem_u32(&ldp), lph ^ 1);
+    }
     if (tid == 0) bulk_wait_rows_done();   // and no bulk store is still reading it
     if (!ok) ms.drain(tid);               // nor a product still writing TMEM after a wait gave up
     tc_fence_before();
@@ -925,16 +1015,29 @@ cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s) {
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     const long long units = (long long)p.slots * p.H;
     const int grid = (int)(units < nsm ? units : nsm);   // one resident CTA per SM
-    CUtensorMap tq, tk, tp;   // dq, dk (and dp) [tokens][value heads][128]
-    if (!make_bf16_token_map(&tq, p.dq, p.Ttot, p.H, tc::D) ||
-        !make_bf16_token_map(&tk, p.dkk, p.Ttot, p.H, tc::D))
-        return cudaErrorInvalidValue;
+    tc::LocalMaps mp;
+    const int Hk = p.H / p.vg;
+    bool good = make_bf16_token_map(&mp.dq, p.dq, p.Ttot, p.H, tc::D) &&
+                make_bf16_token_map(&mp.dk, p.dkk, p.Ttot, p.H, tc::D) &&
+                make_bf16_token_map(&mp.q, p.q, p.Ttot, Hk, tc::D) &&
+                make_bf16_token_map(&mp.k, p.k, p.Ttot, Hk, tc::D) &&
+                make_bf16_token_map(&mp.v, p.v, p.Ttot, p.H, tc::D) &&
+                make_bf16_token_map(&mp.dO, p.dO, p.Ttot, p.H, tc::D) &&
+                make_bf16_map(&mp.e, p.Eb, units * 64, tc::D, 64) &&
+                make_bf16_map(&mp.h, p.Hb, units * tc::D, tc::D, tc::D) &&
+                make_bf16_map(&mp.dh, p.dHb, units * tc::D, tc::D, tc::D) &&
+                make_bf16_map(&mp.m, p.Mb, units * 64, 64, 64) &&
+                make_bf16_map(&mp.u, p.Ub, units * tc::D, 64, tc::D) &&
+                make_bf16_map(&mp.w, p.Wb, units * tc::D, 64, tc::D);
     if (pk) {
-        if (!p.dpp || !make_bf16_token_map(&tp, p.dpp, p.Ttot, p.H, tc::D)) return cudaErrorInvalidValue;
+        good = good && p.dpp && make_bf16_token_map(&mp.dp, p.dpp, p.Ttot, p.H, tc::D) &&
+               make_bf16_token_map(&mp.p, p.p, p.Ttot, Hk, tc::D);
     } else {
-        tp = tq;   // not used
+        mp.dp = mp.dq;   // not used
+        mp.p = mp.q;
     }
-    if (grid > 0) kern<<<grid, tc::kLocalThreads, sm, s>>>(p, units, tq, tk, tp);
+    if (!good) return cudaErrorInvalidValue;
+    if (grid > 0) kern<<<grid, tc::kLocalThreads, sm, s>>>(p, units, mp);
     return cudaGetLastError();
 }
 
