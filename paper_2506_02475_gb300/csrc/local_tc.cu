@@ -42,6 +42,7 @@ namespace tc {
 constexpr int kLocalThreads = 512;            // 16 warps: four per TMEM lane quadrant
 constexpr int kQ = kLocalThreads / 128;        // column parts of each accumulator (one per warp of a quadrant)
 constexpr int NK = 16 / kQ, NL = 8 / kQ;       // m16n8 fragments per warp of 128- and 64-wide results
+constexpr int kTail = kLocalThreads - 64;     // the last two warps take the per-position tail
 
 struct LocalTcSmem {
     static constexpr uint32_t OQK = 0;             // two [128][128] tiles (consecutive units alternate): rows 0-63
@@ -173,6 +174,9 @@ __device__ __forceinline__ void tma_store_rows(const void* tmap, int x, int y, i
 __device__ __forceinline__ void bulk_commit_rows() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_rows_read() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_rows_done() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
+
+// Named barrier 1: the two tail warps only.
+__device__ __forceinline__ void tail_sync() { asm volatile("bar.sync 1, 64;\n" ::: "memory"); }
 
 __device__ __forceinline__ void copy_stage_rows(bf16* g, long long ld, const uint8_t* st, int L, int tid) {
     for (int e = tid; e < L * 16; e += kLocalThreads) {
@@ -334,10 +338,12 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     };
     uint32_t pend = 0;   // thread kTma: barriers with loads issued and not yet waited on (bit i: ldn[i],
                          // 4: ldu, 5: ldp), drained on the give-up path
-    // per-row scalars of a unit (rows tid < 64): log-decay G_r, G_{r-1}, beta, alpha
-    struct RowIn { float g, gm1, be, al; };
+    // a unit's scalars, requested a unit ahead: per row (threads tid < 64) the log-decay G_r,
+    // G_{r-1}, beta and alpha; per head (every thread) b, d and, with Comba-pk, the feedback d
+    struct RowIn { float g, gm1, be, al, bh, dh, dfb; };
     auto load_rows = [&](const UnitRef& x) {
-        RowIn r{0.f, 0.f, 0.f, 1.f};
+        const int hk = x.h / p.vg;
+        RowIn r{0.f, 0.f, 0.f, 1.f, p.b ? p.b[hk] : 1.f, p.d[hk], PK ? p.d_fb[hk] : 0.f};
         if (tid < 64) {
             r.g = p.Gb[x.idx * 64 + tid];
             r.gm1 = tid > 0 ? p.Gb[x.idx * 64 + tid - 1] : 0.f;
@@ -387,9 +393,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     bool ok = true;
     bool pre = false;   // this unit's tiles and row scalars were requested by the previous unit
     uint32_t lph = 0;   // phase parity of the TMA barriers for the current unit
+    bool early = false; // thread 0: this unit's dP and R1 products were issued during the previous unit's tail
     long long u = blockIdx.x;
     UnitRef cur = u < units ? unit_ref(p, u) : UnitRef{0, 0, 0, 0};
-    RowIn rin{0.f, 0.f, 0.f, 1.f};
+    RowIn rin{0.f, 0.f, 0.f, 1.f, 1.f, 0.f, 0.f};
     for (int it = 0; u < units && ok; ++it) {
         const long long un = u + gridDim.x;
         UnitRef nxt{0, 0, 0, 0};
@@ -426,8 +433,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             }
             rin = load_rows(cur);
         }
-        const float bh = p.b ? p.b[h / p.vg] : 1.f;
-        const float dh = p.d[h / p.vg];
+        const float bh = rin.bh;
+        const float dh = rin.dh;
+        const float dfb = rin.dfb;
         if (tid < 64) {
             sG[tid] = rin.g;
             sGm1[tid] = rin.gm1;
@@ -452,7 +460,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                         if (pend & (1u << i)) mbar_drain(smem_u32(&ldn[i]), lph);
                     pend = 0;
                 }
-                if (tid == 0) flag_error(p);
+                if (tid == 0) {
+                    if (early) {   // products issued ahead for this unit: track and drain them
+                        tc_commit(smem_u32(&bar0));
+                        mbar_drain(smem_u32(&bar0), ph0);
+                    }
+                    flag_error(p);
+                }
                 break;
             }
         }
@@ -488,11 +502,13 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         // E dH'^T, K dH', so that the tensor core runs R1 while the warps form P from R0
         if (tid == 0) {
             tc_gemm_m64<false, false>(tmem + 0, uQK, 128, uK, 128, 64, D, false);      // S = Q~ K^T
-            tc_gemm_m64<false, false>(tmem + 64, udO, 64, uE, 64, 64, D, false);       // dP = dO E^T
-            tc_commit(smem_u32(&bar0));
-            tc_gemm_m64<false, true>(tmem + 128, udO, 64, uH, 128, 128, D, false);     // dO H^T
-            tc_gemm_m64<false, true>(tmem + 256, uE, 64, udH, 128, 128, D, false);     // E dH'^T
-            tc_gemm_m64<false, false>(tmem + 384, uK, 128, udH, 128, 128, D, false);   // K dH'
+            if (!early) tc_gemm_m64<false, false>(tmem + 64, udO, 64, uE, 64, 64, D, false);   // dP = dO E^T
+            tc_commit(smem_u32(&bar0));   // (with products issued ahead, it covers those too)
+            if (!early) {
+                tc_gemm_m64<false, true>(tmem + 128, udO, 64, uH, 128, 128, D, false);     // dO H^T
+                tc_gemm_m64<false, true>(tmem + 256, uE, 64, udH, 128, 128, D, false);     // E dH'^T
+                tc_gemm_m64<false, false>(tmem + 384, uK, 128, udH, 128, 128, D, false);   // K dH'
+            }
         }
         // While R0 runs: <H, dH'> (R1 reads the same two tiles; both only read them)
         {
@@ -864,7 +880,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 tmem_wait();
                 tmem_take<NK>(rg, dpv);
                 tmem_take<NK>(rw, t7);
-                const float wa = sWs[ra], wb = sWs[rb], dfb = p.d_fb[h / p.vg];
+                const float wa = sWs[ra], wb = sWs[rb];
 #pragma unroll
                 for (int t = 0; t < NK; ++t)
 #pragma unroll
@@ -875,7 +891,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             }
         }
         if (L == kChunk) fence_async_smem();
+        tc_fence_before();   // every TMEM read of this unit is done: the next unit's products may follow
         __syncthreads();
+        tc_fence_after();
         if (ok) {
             if (L == kChunk) {
                 if (tid == 0) {
@@ -894,8 +912,25 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 if constexpr (PK) copy_stage_rows((bf16*)p.dpp + (t0 * p.H + h) * D, ld, stP, L, tid);
             }
         }
+        // The next unit's dP = dO E^T and R1 products (their tiles are in), issued while the tensor core
+        // would idle through this unit's tail, which the last two warps run; warp 0 may wait here
+        // for room in the tensor core's queue.  A short next chunk (rows to zero first) waits for its
+        // own prologue.
+        if (tid == 0) {
+            early = false;
+            if (ok && has_next && nxt.L == kChunk && mbar_wait_polls(smem_u32(&ldn[1]), lph ^ 1, p.wait_ns) &&
+                mbar_wait_polls(smem_u32(&ldn[2]), lph ^ 1, p.wait_ns)) {
+                const uint32_t uKn = smem_u32(sQKn) + 64 * 128;
+                tc_gemm_m64<false, false>(tmem + 64, udO, 64, uE, 64, 64, D, false);       // dP = dO E^T
+                tc_gemm_m64<false, true>(tmem + 128, udO, 64, uH, 128, 128, D, false);     // dO H^T
+                tc_gemm_m64<false, true>(tmem + 256, uE, 64, udH, 128, 128, D, false);     // E dH'^T
+                tc_gemm_m64<false, false>(tmem + 384, uKn, 128, udH, 128, 128, D, false);  // K dH'
+                early = true;
+            }
+        }
 
-        // ---------------- per-position scalars (rows 0..63, one thread each)
+        // ---------------- per-position scalars (rows 0..63, one thread each of the last two warps,
+        // which meet alone at named barrier 1; the rest of the block goes on to the unit's end)
         auto rsum = [&](int kind, int r) {
             float v = 0.f;
 #pragma unroll
@@ -906,79 +941,80 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             return colp[(kind * 4 + 0) * 64 + c] + colp[(kind * 4 + 1) * 64 + c] + colp[(kind * 4 + 2) * 64 + c] +
                    colp[(kind * 4 + 3) * 64 + c];
         };
-        if (ok && tid < 64) {
-            const int r = tid;
-            float g = 0.f;
-            if (r < L) {
-                g = rsum(0, r) + rsum(3, r) - csum(0, r) - csum(1, r);   // Kbar terms: prefix sum below
-                if (r + 1 < L) {
-                    g += rsum(5, r + 1);
-                    g += sWs[r + 1] * rsum(7, r + 1);
-                }
-            }
-            sDg[r] = g;
-        }
-        __syncthreads();
-        if (ok && warp == 0) {
-            // d log alpha_j = sum_{r >= j} dg_r (a suffix sum inside the chunk) plus gamma_C <H, dH'> at the
-            // last position; the Kbar terms, which reach it as (their total - their suffix), are
-            // added as the exclusive prefix sum_{r < j} instead, so nothing cancels.
-            float k0 = lane < L ? rsum(1, lane) : 0.f, k1 = lane + 32 < L ? rsum(1, lane + 32) : 0.f;
-            float hd = lane < kLocalThreads / 32 ? red[lane] : 0.f;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) hd += __shfl_xor_sync(0xffffffffu, hd, o);
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {   // inclusive prefix sums of the Kbar terms
-                const float y0 = __shfl_up_sync(0xffffffffu, k0, o);
-                const float y1 = __shfl_up_sync(0xffffffffu, k1, o);
-                if (lane >= o) { k0 += y0; k1 += y1; }
-            }
-            const float half0 = __shfl_sync(0xffffffffu, k0, 31);
-            k1 += half0;
-            const float e0p = __shfl_up_sync(0xffffffffu, k0, 1), e1p = __shfl_up_sync(0xffffffffu, k1, 1);
-            const float e0 = lane == 0 ? 0.f : e0p, e1 = lane == 0 ? half0 : e1p;   // exclusive prefixes
-            float x0 = sDg[lane], x1 = sDg[lane + 32];   // zero past L
-            const float last = __expf(gL) * hd;
-            if (L - 1 == lane) x0 += last;
-            if (L - 1 == lane + 32) x1 += last;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const float y0 = __shfl_down_sync(0xffffffffu, x0, o);
-                const float y1 = __shfl_down_sync(0xffffffffu, x1, o);
-                if (lane + o < 32) { x0 += y0; x1 += y1; }
-            }
-            x0 += __shfl_sync(0xffffffffu, x1, 0);
-            sDg[lane] = x0 + e0;
-            sDg[lane + 32] = x1 + e1;
-        }
-        __syncthreads();
-        if (ok && tid < 64) {
-            const int r = tid;
-            float dbt = 0.f, db_c = 0.f, dd_c = 0.f;
-            if (r < L) {
-                dbt = rsum(4, r) + sEm1[r] * rsum(7, r);
-                // dbt is the gradient of btilde_r = b beta_r f_r (f_r = 1, or 2 alpha_r for iplr)
-                const float fr = feedback_scale(p.iplr, sAl[r]);
-                p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r] + (p.iplr ? 2.f * bh * sBe[r] * dbt : 0.f);
-                p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * fr * dbt;
-                db_c = sBe[r] * fr * dbt;
-                dd_c = -rsum(6, r);
-            }
-            // fixed-order reduction of the two per-chunk partials over 64 rows
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                db_c += __shfl_xor_sync(0xffffffffu, db_c, o);
-                dd_c += __shfl_xor_sync(0xffffffffu, dd_c, o);
-            }
-            if (lane == 0) { red[warp * 2] = db_c; red[warp * 2 + 1] = dd_c; }
-        }
-        __syncthreads();
-        if (tid == 0) {
+        if (tid >= kTail) {
+            const int r = tid - kTail;
             if (ok) {
-                p.part[idx * 2] = red[0] + red[2];
-                p.part[idx * 2 + 1] = red[1] + red[3];
-            } else {
-                flag_error(p);
+                float g = 0.f;
+                if (r < L) {
+                    g = rsum(0, r) + rsum(3, r) - csum(0, r) - csum(1, r);   // Kbar terms: prefix sum below
+                    if (r + 1 < L) {
+                        g += rsum(5, r + 1);
+                        g += sWs[r + 1] * rsum(7, r + 1);
+                    }
+                }
+                sDg[r] = g;
+            }
+            tail_sync();
+            if (ok && warp == kTail / 32) {
+                // d log alpha_j = sum_{r >= j} dg_r (a suffix sum inside the chunk) plus gamma_C <H, dH'> at the
+                // last position; the Kbar terms, which reach it as (their total - their suffix), are
+                // added as the exclusive prefix sum_{r < j} instead, so nothing cancels.
+                float k0 = lane < L ? rsum(1, lane) : 0.f, k1 = lane + 32 < L ? rsum(1, lane + 32) : 0.f;
+                float hd = lane < kLocalThreads / 32 ? red[lane] : 0.f;
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) hd += __shfl_xor_sync(0xffffffffu, hd, o);
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {   // inclusive prefix sums of the Kbar terms
+                    const float y0 = __shfl_up_sync(0xffffffffu, k0, o);
+                    const float y1 = __shfl_up_sync(0xffffffffu, k1, o);
+                    if (lane >= o) { k0 += y0; k1 += y1; }
+                }
+                const float half0 = __shfl_sync(0xffffffffu, k0, 31);
+                k1 += half0;
+                const float e0p = __shfl_up_sync(0xffffffffu, k0, 1), e1p = __shfl_up_sync(0xffffffffu, k1, 1);
+                const float e0 = lane == 0 ? 0.f : e0p, e1 = lane == 0 ? half0 : e1p;   // exclusive prefixes
+                float x0 = sDg[lane], x1 = sDg[lane + 32];   // zero past L
+                const float last = __expf(gL) * hd;
+                if (L - 1 == lane) x0 += last;
+                if (L - 1 == lane + 32) x1 += last;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const float y0 = __shfl_down_sync(0xffffffffu, x0, o);
+                    const float y1 = __shfl_down_sync(0xffffffffu, x1, o);
+                    if (lane + o < 32) { x0 += y0; x1 += y1; }
+                }
+                x0 += __shfl_sync(0xffffffffu, x1, 0);
+                sDg[lane] = x0 + e0;
+                sDg[lane + 32] = x1 + e1;
+            }
+            tail_sync();
+            if (ok) {
+                float dbt = 0.f, db_c = 0.f, dd_c = 0.f;
+                if (r < L) {
+                    dbt = rsum(4, r) + sEm1[r] * rsum(7, r);
+                    // dbt is the gradient of btilde_r = b beta_r f_r (f_r = 1, or 2 alpha_r for iplr)
+                    const float fr = feedback_scale(p.iplr, sAl[r]);
+                    p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r] + (p.iplr ? 2.f * bh * sBe[r] * dbt : 0.f);
+                    p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * fr * dbt;
+                    db_c = sBe[r] * fr * dbt;
+                    dd_c = -rsum(6, r);
+                }
+                // fixed-order reduction of the two per-chunk partials over 64 rows
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    db_c += __shfl_xor_sync(0xffffffffu, db_c, o);
+                    dd_c += __shfl_xor_sync(0xffffffffu, dd_c, o);
+                }
+                if (lane == 0) { red[(warp - kTail / 32) * 2] = db_c; red[(warp - kTail / 32) * 2 + 1] = dd_c; }
+            }
+            tail_sync();
+            if (r == 0) {
+                if (ok) {
+                    p.part[idx * 2] = red[0] + red[2];
+                    p.part[idx * 2 + 1] = red[1] + red[3];
+                } else {
+                    flag_error(p);
+                }
             }
         }
         __syncthreads();   // the staging tile read above takes the Q/K copies of the unit after next
