@@ -19,9 +19,15 @@
 //
 // Workspace tensors of this path: W^T, U^T, U_s^T, Z^T [pairs][128][64]; Atilde,
 // H^T, dH^T [pairs][128][128]; E [pairs][64][128] row-major; M [pairs][64][64].
+#include <cuda.h>
+
 #include "tc_tiles.cuh"
 
 namespace comba {
+
+bool make_bf16_token_map(CUtensorMap* m, const void* base, long long tokens, int heads, int cols);
+bool make_bf16_map(CUtensorMap* m, const void* base, long long rows, int cols, int box_rows);
+
 namespace tc {
 
 // ------------------------------------------------------------------ prep
@@ -263,18 +269,29 @@ struct OutTcSmem {
                                                    // P [64][64] later over K's first half     32 KB
     static constexpr uint32_t OW = 32768;          // W^T [128][64] (MN-major B, then K-major A), later E [64][128]  16 KB
     static constexpr uint32_t OU = OW + 16384;     // U^T [128][64], then E^T in place, later Z^T staging             16 KB
-    static constexpr uint32_t OH = OU + 16384;     // H^T [128][128] K-major, later O staging                        32 KB
+    static constexpr uint32_t OH = OU + 16384;     // H^T [128][128] K-major, later O staging [64][128]              32 KB
     static constexpr uint32_t OG = OH + 32768;
     static constexpr size_t bytes() { return 1024 + OG + 64 * 4; }
 };
 
+// Tensor maps of the output kernel: token tiles {64 columns, 1 head, 64 tokens} of q, k (key heads)
+// and o (value heads); workspace tiles of W^T, U^T, Z^T ([pairs * 128][64], 128-row boxes) and
+// H^T ([pairs * 128][128], 128-row boxes of 64 columns).  All 128-byte swizzled.
+struct OutMaps {
+    CUtensorMap q, k, o, w, u, h, z;
+};
 
 // 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
-__global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
+// Tiles arrive by TMA in two groups: Q and K (all that Q~, S = Q~ K^T and P need), then H^T, W^T
+// and U^T, so that Q~, S and P overlap the larger load.  O and Z^T leave by bulk tensor stores
+// and E by a bulk copy, from staging tiles over the dead inputs.
+__global__ void __launch_bounds__(256) k_output_tc(ChunkParams p, const __grid_constant__ OutMaps mp) {
     constexpr int NTH = 256;
     using S = OutTcSmem;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar, stall_bar;   // stall_bar: nothing arrives (COMBA_DIAG_STALL)
+    // ldA: Q/K landed; ldB: H^T, W^T, U^T landed; barS: S; barE: H^T W^T; bar: the second products;
+    // stall_bar: nothing arrives (COMBA_DIAG_STALL)
+    __shared__ uint64_t ldA, ldB, barS, barE, bar, stall_bar;
     __shared__ uint32_t tbase;
     const int slot = blockIdx.x, h = blockIdx.y;
     const SlotInfo si = p.slot_info[slot];
@@ -282,7 +299,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     const int L = si.len;
     const long long t0 = si.start;
     const long long idx = (long long)slot * p.H + h;
-    const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
+    const int hk = h / p.vg;   // key head of value head h
     const int tid = threadIdx.x, warp = tid >> 5;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQK = sm + S::OQK;
@@ -291,39 +308,58 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
     uint8_t* sUt = sm + S::OU;
     uint8_t* sEt = sUt;                        // E^T replaces U^T row by row
     bf16* sE = reinterpret_cast<bf16*>(sWt);   // [64][128] row-major staging of E, once W^T is dead
-    uint8_t* stZ = sUt;                        // Z^T staging, once E^T is dead
+    uint8_t* stZ = sUt;                        // Z^T staging (128-byte swizzled), once E^T is dead
     uint8_t* sHt = sm + S::OH;
-    bf16* sO = reinterpret_cast<bf16*>(sHt);   // [64][136] staging of O
+    uint8_t* stO = sHt;                        // O staging: two [64][64] swizzled halves, once H^T is dead
     float* sG = reinterpret_cast<float*>(sm + S::OG);
+    const uint32_t uA = smem_u32(&ldA), uB = smem_u32(&ldB);
 
-    const float dh = p.d[hk];   // loaded ahead of the tiles' cp.async traffic, as are the log-decays
-    const float gv = tid < 64 ? p.Gb[idx * 64 + tid] : 0.f;
-    {
-        // Q into rows 0-63 and K into rows 64-127 of one K-major tile (rows past the chunk zero)
-        const bf16* qg = (const bf16*)p.q + (t0 * Hk + hk) * D;
-        const bf16* kg = (const bf16*)p.k + (t0 * Hk + hk) * D;
-        for (int e = tid; e < 128 * 16; e += NTH) {
-            const int r = e >> 4, ch = e & 15, rr = r & 63;
-            const bool okr = rr < L;
-            const bf16* src = (r < 64 ? qg : kg) + (long long)rr * Hk * D + ch * 8;
-            cp_async16(sQK + sw128_offset(r, ch * 8, 128), okr ? (const void*)src : (const void*)qg, okr);
-        }
-    }
-    load_sw(sWt, 128, 64, (const bf16*)p.Wb + idx * D * 64, 64, 128, tid, NTH);
-    load_sw(sUt, 128, 64, (const bf16*)p.Ub + idx * D * 64, 64, 128, tid, NTH);
-    load_sw(sHt, 128, D, (const bf16*)p.Hb + idx * D * D, D, 128, tid, NTH);
-    cp_async_commit();
-    if (tid < 64) sG[tid] = gv;
     if (tid == 0) {
+        mbar_init(uA, 1);
+        mbar_init(uB, 1);
+        mbar_init(smem_u32(&barS), 1);
+        mbar_init(smem_u32(&barE), 1);
         mbar_init(smem_u32(&bar), 1);
         mbar_init(smem_u32(&stall_bar), 1);
         mbar_fence_init();
     }
+    const float dh = p.d[hk];
+    const float gv = tid < 64 ? p.Gb[idx * 64 + tid] : 0.f;
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
-    cp_async_wait<0>();
+    tc_fence_before();
     __syncthreads();
-    // Q~ = Q - d K (rows < 64; rows >= L are zero in both)
-    for (int e = tid; e < 64 * 16; e += NTH) {
+    tc_fence_after();
+    if (tid == 0) {
+        mbar_expect_tx(uA, 32768u);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            tma_load_3d(smem_u32(sQK) + half * 16384, &mp.q, 64 * half, hk, (int)t0, uA);
+            tma_load_3d(smem_u32(sQK) + 8192 + half * 16384, &mp.k, 64 * half, hk, (int)t0, uA);
+        }
+        mbar_expect_tx(uB, 65536u);
+        tma_load_2d(smem_u32(sWt), &mp.w, 0, (int)(idx * 128), uB);
+        tma_load_2d(smem_u32(sUt), &mp.u, 0, (int)(idx * 128), uB);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) tma_load_2d(smem_u32(sHt) + half * 16384, &mp.h, 64 * half, (int)(idx * 128), uB);
+    }
+    if (tid < 64) sG[tid] = gv;
+    const uint32_t tmem = tbase;
+    MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
+    const int row = tid & 127, half = tid >> 7;   // TMEM lane, and which 32 of each 64 columns
+    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+
+    // Q and K in; rows past a short chunk hold the next sequence's tokens: zero them
+    const bool okA = mbar_wait_polls(uA, 0, p.wait_ns);
+    if (L < kChunk) {
+        for (int e = tid; okA && e < (64 - L) * 16; e += NTH) {
+            const int r = L + (e >> 4), ch = e & 15;
+            *reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128)) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128)) = make_uint4(0, 0, 0, 0);
+        }
+        __syncthreads();
+    }
+    // Q~ = Q - d K (rows < L)
+    for (int e = tid; okA && e < L * 16; e += NTH) {
         const int r = e >> 4, ch = e & 15;
         uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
         const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
@@ -334,70 +370,79 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
         for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
         *qa = pack8(qv);
     }
-    publish_smem();
-    const uint32_t tmem = tbase;
-    MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
-    const int row = tid & 127, half = tid >> 7;   // TMEM lane, and which 32 of each 64 columns
-    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    fence_async_smem();
+    tc_fence_before();
+    bool ok = !__syncthreads_or(!okA);
+    tc_fence_after();
 
-    // [Q~; K] K^T -> cols [0,64) (lanes 0-63: S = Q~ K^T; lanes 64-127 unused);  E^T' = H^T W^T -> cols [64,128)
+    // [Q~; K] K^T -> cols [0,64) (lanes 0-63: S = Q~ K^T; lanes 64-127 unused), then, once H^T, W^T
+    // and U^T are in, E^T' = H^T W^T -> cols [64,128), each on its own barrier
     if (tid == 0) {
-        tc_gemm<false, false>(tmem, smem_u32(sQK), 128, smem_u32(sQK) + 64 * 128, 128, 64, D, false);
-        tc_gemm<false, true>(tmem + 64, smem_u32(sHt), 128, smem_u32(sWt), 128, 64, D, false);
+        if (ok) tc_gemm<false, false>(tmem, smem_u32(sQK), 128, smem_u32(sQK) + 64 * 128, 128, 64, D, false);
+        tc_commit(smem_u32(&barS));
     }
-    bool ok = ms.finish(tid);
+    bool okB = mbar_wait_polls(uB, 0, p.wait_ns);
+    if (tid == 0) {
+        if (ok && okB) tc_gemm<false, true>(tmem + 64, smem_u32(sHt), 128, smem_u32(sWt), 128, 64, D, false);
+        tc_commit(smem_u32(&barE));
+    }
     bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
-    bf16* Zg = p.Zb ? (bf16*)p.Zb + idx * D * 64 : nullptr;
+    const bool Zg = p.Zb != nullptr;
     uint32_t ev[16];   // this thread's 32 positions of row j of E^T, packed bf16 pairs
-    if (ok) {
-        float d[32], v[8];
-        // P = Tril(S * Gamma) into a K-major [64][64] tile (B operand of E^T P^T)
-        {
-            const int g = half;
-            tmem_ld32(trow + g * 32, d);
-            if (row < 64) {
-                const float gr = sG[row];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const int i = 32 * g + 8 * q + e;
-                        v[e] = (i <= row && row < L) ? d[8 * q + e] * __expf(gr - sG[i]) : 0.f;
-                    }
-                    *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * g + 8 * q, 64)) = pack8(v);
-                }
-            }
-        }
-        // E^T = U^T - H^T W^T  (half of row j of E^T per thread)
-        {
-            const int g = half;
-            tmem_ld32(trow + 64 + g * 32, d);
+    const bool okS = mbar_wait_polls(smem_u32(&barS), 0, p.wait_ns);
+    tc_fence_after();
+    if (ok && okS) {
+        if (row < 64) {
+            // P = Tril(S * Gamma) into a K-major [64][64] tile (B operand of E^T P^T), over K
+            float d[32], v[8];
+            tmem_ld32(trow + half * 32, d);
+            const float gr = sG[row];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                float u[8];
-                unpack8(*reinterpret_cast<const uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)), u);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) v[e] = u[e] - d[8 * q + e];
-                // in place: each thread reads and then overwrites only these 16 bytes of its own row
-                const uint4 pk = pack8(v);
-                *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * g + 8 * q, 128)) = pk;
-                const int b0 = 4 * q;
-                ev[b0] = pk.x; ev[b0 + 1] = pk.y; ev[b0 + 2] = pk.z; ev[b0 + 3] = pk.w;
+                for (int e = 0; e < 8; ++e) {
+                    const int i = 32 * half + 8 * q + e;
+                    v[e] = (i <= row && row < L) ? d[8 * q + e] * __expf(gr - sG[i]) : 0.f;
+                }
+                *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * half + 8 * q, 64)) = pack8(v);
+            }
+        } else {
+            // the warps of TMEM lanes 64-127 (no S rows): Qhat = Diag(gamma) Q~ in place
+            for (int e = (tid & 63) + 64 * half; e < 64 * 16; e += 128) {
+                const int r = e >> 4, ch = e & 15;
+                uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
+                float qv[8];
+                unpack8(*qa, qv);
+                const float gr = __expf(sG[r]);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) qv[i] *= gr;
+                *qa = pack8(qv);
             }
         }
-        // Qhat = Diag(gamma) Q~ in place
-        for (int e = tid; e < 64 * 16; e += NTH) {
-            const int r = e >> 4, ch = e & 15;
-            uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
-            float qv[8];
-            unpack8(*qa, qv);
-            const float gr = __expf(sG[r]);
+    }
+    const bool okE = mbar_wait_polls(smem_u32(&barE), 0, p.wait_ns) && okB;
+    tc_fence_after();
+    if (ok && okE) {
+        // E^T = U^T - H^T W^T  (half of row j of E^T per thread)
+        float d[32], v[8];
+        tmem_ld32(trow + 64 + half * 32, d);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) qv[i] *= gr;
-            *qa = pack8(qv);
+        for (int q = 0; q < 4; ++q) {
+            float u[8];
+            unpack8(*reinterpret_cast<const uint4*>(sUt + sw128_offset(row, 32 * half + 8 * q, 128)), u);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = u[e] - d[8 * q + e];
+            // in place: each thread reads and then overwrites only these 16 bytes of its own row
+            const uint4 pk = pack8(v);
+            *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * half + 8 * q, 128)) = pk;
+            const int b0 = 4 * q;
+            ev[b0] = pk.x; ev[b0 + 1] = pk.y; ev[b0 + 2] = pk.z; ev[b0 + 3] = pk.w;
         }
     }
-    publish_smem();
+    fence_async_smem();
+    tc_fence_before();
+    ok = !__syncthreads_or(!(ok && okS && okE));
+    tc_fence_after();
 
     // O^T = H^T Qhat^T + E^T P^T -> cols [128,192);  (P W)^T = W^T P^T -> cols [192,256)
     const bool mma2 = p.o || Zg;
@@ -417,7 +462,6 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
             sE[(32 * half + 2 * pp) * D + row] = two.x;
             sE[(32 * half + 2 * pp + 1) * D + row] = two.y;
         }
-        fence_async_smem();
     }
     if (ok && Zg) {
         // Z^T = Qhat^T - (P W)^T: row `row` (a key dimension), positions [32 half, +32); columns
@@ -432,31 +476,49 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p) {
                 const float qh = __bfloat162float(*reinterpret_cast<const bf16*>(sQK + sw128_offset(t, row, 128)));
                 v[e] = qh - d[8 * q + e];
             }
-            stage_chunk<8>(stZ, row, 4 * half + q, pack8(v));
+            *reinterpret_cast<uint4*>(stZ + sw128_offset(row, 32 * half + 8 * q, 128)) = pack8(v);
         }
     }
     if (ok && p.o) {
+        // O[t][j] for j = row, t in [32 half, +32): the [64][128] tile as two swizzled 64-column halves
         float d[32];
         tmem_ld32(trow + 128 + half * 32, d);
+        uint8_t* oh = stO + (row >> 6) * 8192;
 #pragma unroll
-        for (int c = 0; c < 32; ++c) sO[(32 * half + c) * 136 + row] = __float2bfloat16_rn(d[c]);
+        for (int c = 0; c < 32; ++c)
+            *reinterpret_cast<bf16*>(oh + sw128_offset(32 * half + c, row & 63, 64)) = __float2bfloat16_rn(d[c]);
     }
+    fence_async_smem();
     __syncthreads();
-    if (ok && Eg && tid == 0) bulk_copy_s2g(Eg, smem_u32(sE), 64 * D * 2);
-    if (ok && Zg) copy_staged<8>(Zg, stZ, tid, NTH);
-    if (ok && p.o) {
+    if (ok && tid == 0) {
+        if (Eg) bulk_copy_s2g(Eg, smem_u32(sE), 64 * D * 2);
+        if (Zg) tma_store_2d(&mp.z, 0, (int)(idx * 128), smem_u32(stZ));
+        if (p.o && L == kChunk)
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) tma_store_3d(&mp.o, 64 * hh, h, (int)t0, smem_u32(stO) + hh * 8192);
+        bulk_commit();
+    }
+    if (ok && p.o && L < kChunk) {
+        // a short chunk by rows (a 64-row box would run into the next sequence)
         bf16* Og = (bf16*)p.o + (t0 * p.H + h) * D;
         for (int e = tid; e < L * 16; e += NTH) {
             const int r = e >> 4, ch = e & 15;
             *reinterpret_cast<uint4*>(Og + (long long)r * p.H * D + 8 * ch) =
-                *reinterpret_cast<const uint4*>(sO + r * 136 + 8 * ch);
+                *reinterpret_cast<const uint4*>(stO + (ch >> 3) * 8192 + sw128_offset(r, 8 * (ch & 7), 64));
         }
     }
     if (!ok) {
-        if (tid == 0) flag_error(p);
+        if (tid == 0) {
+            flag_error(p);
+            // let the tile loads and every product end before the block's shared memory and TMEM go
+            mbar_drain(uA, 0);
+            mbar_drain(uB, 0);
+            mbar_drain(smem_u32(&barS), 0);
+            mbar_drain(smem_u32(&barE), 0);
+        }
         ms.drain(tid);
     }
-    if (ok && Eg && tid == 0) bulk_wait_all_reads();   // the E copy has read its staging before exit
+    if (ok && tid == 0) bulk_wait_all_reads();   // the stores have read their staging before exit
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -479,7 +541,20 @@ cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s) {
     const size_t sm = tc::OutTcSmem::bytes();
     cudaError_t e = cudaFuncSetAttribute(tc::k_output_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
-    if (p.slots > 0) tc::k_output_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p);
+    if (p.slots <= 0) return cudaSuccess;
+    const long long pairs = (long long)p.slots * p.H;
+    tc::OutMaps mp;
+    bool good = make_bf16_token_map(&mp.q, p.q, p.Ttot, p.H / p.vg, tc::D) &&
+                make_bf16_token_map(&mp.k, p.k, p.Ttot, p.H / p.vg, tc::D) &&
+                make_bf16_map(&mp.w, p.Wb, pairs * tc::D, 64, tc::D) &&
+                make_bf16_map(&mp.u, p.Ub, pairs * tc::D, 64, tc::D) &&
+                make_bf16_map(&mp.h, p.Hb, pairs * tc::D, tc::D, tc::D);
+    if (good && p.o) good = make_bf16_token_map(&mp.o, p.o, p.Ttot, p.H, tc::D);
+    else mp.o = mp.q;   // not used
+    if (good && p.Zb) good = make_bf16_map(&mp.z, p.Zb, pairs * tc::D, 64, tc::D);
+    else mp.z = mp.w;   // not used
+    if (!good) return cudaErrorInvalidValue;
+    tc::k_output_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p, mp);
     return cudaGetLastError();
 }
 

@@ -107,6 +107,19 @@ __device__ __forceinline__ void bulk_copy_s2g(void* g, uint32_t s, uint32_t byte
     asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
 }
 __device__ __forceinline__ void bulk_wait_all_reads() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+// Bulk tensor stores of a swizzled shared tile (2D: columns x, rows y; 3D: columns x, head y,
+// tokens z), completed as one bulk group by bulk_commit.
+__device__ __forceinline__ void tma_store_2d(const void* tmap, int x, int y, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];\n"
+                 ::"l"(tmap), "r"(x), "r"(y), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void tma_store_3d(const void* tmap, int x, int y, int z, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];\n"
+                 ::"l"(tmap), "r"(x), "r"(y), "r"(z), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
 
 }  // namespace tc
 }  // namespace comba
