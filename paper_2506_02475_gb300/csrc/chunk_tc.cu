@@ -43,12 +43,19 @@ struct PrepTcSmem {
     static constexpr size_t bytes() { return 1024 + OF + 64 * 6 * 4; }
 };
 
-// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
-__global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p) {
+// Tensor maps of the prep kernel's loads: token tiles {64 columns, 1 head, 64 tokens} of k and p
+// (key heads) and v (value heads), 128-byte swizzled.
+struct PrepMaps {
+    CUtensorMap k, p, v;
+};
+
+// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.  The
+// K (or [P; K]) and V tiles arrive by TMA while the warps load the gates and form the log-decays.
+__global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_constant__ PrepMaps mp) {
     constexpr int NTH = 256;
     using S = PrepTcSmem;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar, stall_bar;   // stall_bar: nothing arrives (COMBA_DIAG_STALL)
+    __shared__ uint64_t bar, stall_bar, ld;   // stall_bar: nothing arrives (COMBA_DIAG_STALL); ld: tiles
     __shared__ uint32_t tbase;
     const int slot = blockIdx.x, h = blockIdx.y;
     const SlotInfo si = p.slot_info[slot];
@@ -80,9 +87,13 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p) {
     // P K^T, and K (rows 64..127) is the operand of every later product that takes K.
     const bool pk = p.p != nullptr;
     const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
-    // The per-position gates go first: the first barrier waits on them, and loads issued behind
-    // the tiles' cp.async traffic would queue behind it.
     const int lane = tid & 31;
+    if (tid == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        mbar_init(smem_u32(&stall_bar), 1);
+        mbar_init(smem_u32(&ld), 1);
+        mbar_fence_init();
+    }
     const float* ag = p.alpha + t0 * Hk + hk;
     float a0 = 1.f, a1 = 1.f, bev = 0.f, alv = 1.f, bh = 1.f;
     if (warp == 0) {
@@ -94,20 +105,21 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p) {
         alv = tid < L ? ag[(long long)tid * Hk] : 1.f;
         bh = p.b ? p.b[hk] : 1.f;
     }
-    {
-        const bf16* kg = (const bf16*)p.k + (t0 * Hk + hk) * D;
-        const bf16* fg = pk ? (const bf16*)p.p + (t0 * Hk + hk) * D : kg;
-        for (int e = tid; e < 128 * 16; e += NTH) {
-            const int r = e >> 4, ch = e & 15, rr = r & 63;
-            const bool okr = rr < L;
-            const bf16* src = r < 64 ? fg : kg;
-            cp_async16(sK + sw128_offset(r, ch * 8, 128),
-                       okr ? (const void*)(src + (long long)rr * Hk * D + ch * 8) : (const void*)src, okr);
+    if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
+    tc_fence_before();
+    __syncthreads();   // barriers initialised, TMEM allocated
+    tc_fence_after();
+    if (tid == 0) {
+        const uint32_t mb = smem_u32(&ld);
+        mbar_expect_tx(mb, 32768u + 16384u);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            tma_load_3d(smem_u32(sK) + half * 16384, pk ? &mp.p : &mp.k, 64 * half, hk, (int)t0, mb);
+            tma_load_3d(smem_u32(sK) + 8192 + half * 16384, &mp.k, 64 * half, hk, (int)t0, mb);
+            tma_load_3d(smem_u32(sV) + half * 8192, &mp.v, 64 * half, h, (int)t0, mb);
         }
     }
     const uint8_t* sKk = pk ? sK + 64 * 128 : sK;   // the 64 key rows (rows 64.. of each K-half for pk)
-    load_sw(sV, 64, D, (const bf16*)p.v + (t0 * p.H + h) * D, (long long)p.H * D, L, tid, NTH);
-    cp_async_commit();
     if (warp == 0) chunk_log_cumsum_vals(a0, a1, L, sG, sGm1);
     if (tid < 64) {
         sBe[tid] = bev;
@@ -115,24 +127,30 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p) {
     }
     __syncthreads();   // sG, sGm1, sBt complete
     if (tid < 64) sWs[tid] = sBt[tid] * expf(sGm1[tid]);
-    if (tid == 0) {
-        mbar_init(smem_u32(&bar), 1);
-        mbar_init(smem_u32(&stall_bar), 1);
-        mbar_fence_init();
+    // the tiles: rows past a short chunk hold the next sequence's tokens, zeroed here
+    const bool okl = mbar_wait_polls(smem_u32(&ld), 0, p.wait_ns);
+    if (okl && L < kChunk) {
+        for (int e = tid; e < (64 - L) * 16; e += NTH) {
+            const int r = L + (e >> 4), ch = e & 15;
+            const uint4 z = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(sK + sw128_offset(r, 8 * ch, 128)) = z;
+            *reinterpret_cast<uint4*>(sK + sw128_offset(64 + r, 8 * ch, 128)) = z;
+            *reinterpret_cast<uint4*>(sV + sw128_offset(r, 8 * ch, 64)) = z;
+        }
     }
-    if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
-    cp_async_wait<0>();
-    publish_smem();
+    fence_async_smem();
+    tc_fence_before();
+    bool ok = !__syncthreads_or(!okl);
+    tc_fence_after();
     const uint32_t tmem = tbase;
     MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
     const int row = tid & 127, half = tid >> 7;   // TMEM lane / accumulator row, and which column half
     const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-    bool ok = true;
 
     // Gram K K^T over the 128-row tile (P K^T in lanes 0..63 for Comba-pk).
-    if (tid == 0) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sKk), 128, 64, D, false);
+    if (tid == 0 && ok) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sKk), 128, 64, D, false);
     if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;
-    ok = ms.finish(tid);
+    ok = ms.finish(tid) && ok;
     if (ok && !pk) {
         // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T), stored transposed; exp only
         // below the diagonal.  Lane l holds Gram row l & 63; its two threads fill columns
@@ -253,7 +271,10 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p) {
     __syncthreads();
     if (ok) copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
     if (!ok) {
-        if (tid == 0) flag_error(p);
+        if (tid == 0) {
+            flag_error(p);
+            mbar_drain(smem_u32(&ld), 0);   // the tile loads have ended before the block's memory goes
+        }
         ms.drain(tid);
     }
     tc_fence_before();
@@ -533,7 +554,14 @@ cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s) {
     const size_t sm = tc::PrepTcSmem::bytes();
     cudaError_t e = cudaFuncSetAttribute(tc::k_prep_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
-    if (p.slots > 0) tc::k_prep_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p);
+    if (p.slots <= 0) return cudaSuccess;
+    tc::PrepMaps mp;
+    bool good = make_bf16_token_map(&mp.k, p.k, p.Ttot, p.H / p.vg, tc::D) &&
+                make_bf16_token_map(&mp.v, p.v, p.Ttot, p.H, tc::D);
+    if (good && p.p) good = make_bf16_token_map(&mp.p, p.p, p.Ttot, p.H / p.vg, tc::D);
+    else mp.p = mp.k;   // not used
+    if (!good) return cudaErrorInvalidValue;
+    tc::k_prep_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p, mp);
     return cudaGetLastError();
 }
 
