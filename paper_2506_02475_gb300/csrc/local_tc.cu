@@ -57,7 +57,9 @@ struct LocalTcSmem {
     static constexpr uint32_t ODE = OP + 8192;     // dE [64][128]
     static constexpr uint32_t OF = ODE + 16384;    // fp32: 8 x 64 per-row vectors, row and column partials, reduction
     static constexpr uint32_t NF = 8 * 64 + 8 * kQ * 64 + 2 * 4 * 64 + 16;
-    static constexpr size_t bytes() { return 1024 + OF + NF * 4; }
+    static constexpr uint32_t NX = 5 * 64 + 4;     // fp32: the next unit's scalars, copied in a unit ahead,
+                                                   // and the current unit's b
+    static constexpr size_t bytes() { return 1024 + OF + (NF + NX) * 4; }
 };
 
 // M = 64 accumulator columns [taddr, +8 NT) of this warp's 16 rows as m16n8 fragments (NT = 4, 2).
@@ -175,6 +177,12 @@ __device__ __forceinline__ void bulk_commit_rows() { asm volatile("cp.async.bulk
 __device__ __forceinline__ void bulk_wait_rows_read() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_rows_done() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
 
+// 4-byte global->shared copy that bypasses registers; zero-filled when `valid` is false.
+__device__ __forceinline__ void cp_async4(float* s, const float* g, bool valid) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(smem_u32(s)), "l"(g), "r"(valid ? 4 : 0)
+                 : "memory");
+}
+
 // Named barrier 1: the two tail warps only.
 __device__ __forceinline__ void tail_sync() { asm volatile("bar.sync 1, 64;\n" ::: "memory"); }
 
@@ -203,9 +211,13 @@ struct UnitRef {
     long long idx, t0;   // (slot, head) unit index, first token
     int L, h;
 };
+// (unit indices fit 32 bits: the launcher checks slots x heads; 64-bit division would cost the
+// loop head several hundred cycles)
 __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
-    const SlotInfo si = p.slot_info[u / p.H];
-    return {u, si.start, si.len, (int)(u % p.H)};
+    const uint32_t uu = (uint32_t)u, hh = (uint32_t)p.H;
+    const uint32_t slot = uu / hh;
+    const SlotInfo si = p.slot_info[slot];
+    return {u, si.start, si.len, (int)(uu - slot * hh)};
 }
 
 // Persistent: CTA b handles units b, b + G, b + 2G, ... (G = gridDim.x, about one CTA per SM).
@@ -243,6 +255,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     // Each completes one phase per unit that has rows.
     __shared__ uint64_t ldn[4], ldu, ldp;
     __shared__ uint32_t tbase;
+    __shared__ int2 s_nslot;   // (start, length) of the unit after next, loaded during the tail
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wr = warp & 3, wc = warp >> 2, m0 = 16 * wr;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -338,19 +351,25 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     };
     uint32_t pend = 0;   // thread kTma: barriers with loads issued and not yet waited on (bit i: ldn[i],
                          // 4: ldu, 5: ldp), drained on the give-up path
-    // a unit's scalars, requested a unit ahead: per row (threads tid < 64) the log-decay G_r,
-    // G_{r-1}, beta and alpha; per head (every thread) b, d and, with Comba-pk, the feedback d
-    struct RowIn { float g, gm1, be, al, bh, dh, dfb; };
-    auto load_rows = [&](const UnitRef& x) {
+    // A unit's scalars, copied into sNx a unit ahead (asynchronous 4-byte copies, which hold no
+    // registers and wait behind no tile traffic): per row r (thread r < 64) the log-decays G_r and
+    // G_{r-1}, beta, alpha and b; per head (thread 0) d and, with Comba-pk, the feedback d.
+    float* sNx = sG + S::NF;
+    auto issue_rows = [&](const UnitRef& x) {
         const int hk = x.h / p.vg;
-        RowIn r{0.f, 0.f, 0.f, 1.f, p.b ? p.b[hk] : 1.f, p.d[hk], PK ? p.d_fb[hk] : 0.f};
         if (tid < 64) {
-            r.g = p.Gb[x.idx * 64 + tid];
-            r.gm1 = tid > 0 ? p.Gb[x.idx * 64 + tid - 1] : 0.f;
-            r.be = tid < x.L ? p.beta[(x.t0 + tid) * Hk + x.h / p.vg] : 0.f;
-            r.al = tid < x.L ? p.alpha[(x.t0 + tid) * Hk + x.h / p.vg] : 1.f;
+            const float* gb = p.Gb + x.idx * 64;
+            cp_async4(sNx + tid, gb + tid, true);
+            cp_async4(sNx + 64 + tid, gb + (tid > 0 ? tid - 1 : 0), tid > 0);
+            cp_async4(sNx + 128 + tid, p.beta + (x.t0 + (tid < x.L ? tid : 0)) * Hk + hk, tid < x.L);
+            cp_async4(sNx + 192 + tid, p.alpha + (x.t0 + (tid < x.L ? tid : 0)) * Hk + hk, tid < x.L);
+            cp_async4(sNx + 256 + tid, p.b ? p.b + hk : p.d + hk, p.b != nullptr);
         }
-        return r;
+        if (tid == 0) {
+            cp_async4(sNx + 320, p.d + hk, true);
+            cp_async4(sNx + 321, PK ? p.d_fb + hk : p.d + hk, PK);
+        }
+        cp_async_commit();
     };
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
@@ -396,16 +415,24 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     bool early = false; // thread 0: this unit's dP and R1 products were issued during the previous unit's tail
     long long u = blockIdx.x;
     UnitRef cur = u < units ? unit_ref(p, u) : UnitRef{0, 0, 0, 0};
-    RowIn rin{0.f, 0.f, 0.f, 1.f, 1.f, 0.f, 0.f};
+    bool nslot = false;   // s_nslot holds the slot of unit u + G (the previous unit's tail loaded it)
     for (int it = 0; u < units && ok; ++it) {
         const long long un = u + gridDim.x;
         UnitRef nxt{0, 0, 0, 0};
-        if (un < units) nxt = unit_ref(p, un);   // used from the first prefetch point on
+        if (un < units) {   // used from the first prefetch point on
+            if (nslot) {
+                const int2 sl = s_nslot;
+                nxt = UnitRef{un, sl.x, sl.y, (int)((uint32_t)un % (uint32_t)p.H)};
+            } else {
+                nxt = unit_ref(p, un);
+            }
+        }
         uint8_t* sQK = sm + S::OQK + (it & 1) * 32768;
         uint8_t* sQKn = sm + S::OQK + ((it + 1) & 1) * 32768;   // the next unit's Q/K tile
         if (cur.L <= 0) {
             if (tid == 0) { p.part[u * 2] = 0.f; p.part[u * 2 + 1] = 0.f; }
             pre = false;
+            nslot = false;
             u = un;
             cur = nxt;
             continue;
@@ -431,21 +458,23 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 issue_n3(cur, false);
                 pend |= 15u;
             }
-            rin = load_rows(cur);
+            issue_rows(cur);
         }
-        const float bh = rin.bh;
-        const float dh = rin.dh;
-        const float dfb = rin.dfb;
+        cp_async_wait<0>();   // this thread's copies of the unit's scalars
+        const float bh = tid < 64 ? (p.b ? sNx[256 + tid] : 1.f) : 1.f;
         if (tid < 64) {
-            sG[tid] = rin.g;
-            sGm1[tid] = rin.gm1;
-            sBe[tid] = rin.be;
-            const float fsc = feedback_scale(p.iplr, rin.al);
-            sBt[tid] = bh * rin.be * fsc;
-            sAl[tid] = rin.al;
-            const float em1 = tid > 0 ? __expf(rin.gm1) : 1.f;
+            const float g = sNx[tid], gm1 = sNx[64 + tid], be = sNx[128 + tid];
+            const float al = tid < L ? sNx[192 + tid] : 1.f;
+            sG[tid] = g;
+            sGm1[tid] = gm1;
+            sBe[tid] = be;
+            const float fsc = feedback_scale(p.iplr, al);
+            sBt[tid] = bh * be * fsc;
+            sAl[tid] = al;
+            const float em1 = tid > 0 ? __expf(gm1) : 1.f;
             sEm1[tid] = em1;
-            sWs[tid] = bh * rin.be * fsc * em1;
+            sWs[tid] = bh * be * fsc * em1;
+            if (tid == 0) sNx[322] = bh;   // the unit's b for the tail (the next unit's copies miss this slot)
         }
         // the unit's tiles have landed (all four groups)
         {
@@ -470,6 +499,8 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 break;
             }
         }
+        const float dh = sNx[320];                // thread 0's copies, published by the barrier above
+        const float dfb = PK ? sNx[321] : 0.f;
         // rows past a short chunk: zero in Q, K, dO and V (Q~ below covers rows < L only)
         if (L < kChunk) {
             zero_rows(sQK, 128, L);
@@ -668,6 +699,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             }
             if (has_next) { issue_n0(nxt, !PK); pend |= 1u; }   // M's last reader was R3
         }
+        if (ok && has_next) issue_rows(nxt);   // sNx was last read at this unit's start
         if (ok) {
             // M^T dE, unscaled and in bf16, over the dead dE tile: the R4 / R5 operand; and
             // dV = Diag(beta) M^T dE staged over the dead E tile, direct dbeta = v . (M^T dE)
@@ -849,7 +881,6 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         if (ok && has_next) {
             if (tid == kTma) { issue_n3(nxt, PK); pend |= 8u; }   // dG (over V) is dead, and P (over M)
-            rin = load_rows(nxt);
         }
         if (ok) {
             float t6[NK][4];
@@ -943,6 +974,11 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         };
         if (tid >= kTail) {
             const int r = tid - kTail;
+            // the slot of the unit after next, for the next unit's loop head (the load's latency,
+            // behind this unit's bulk traffic, would otherwise open that unit)
+            const long long unn = un + gridDim.x;
+            SlotInfo ns{0, 0, 0, 0};
+            if (r == 0 && unn < units) ns = p.slot_info[(uint32_t)unn / (uint32_t)p.H];
             if (ok) {
                 float g = 0.f;
                 if (r < L) {
@@ -994,6 +1030,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                     dbt = rsum(4, r) + sEm1[r] * rsum(7, r);
                     // dbt is the gradient of btilde_r = b beta_r f_r (f_r = 1, or 2 alpha_r for iplr)
                     const float fr = feedback_scale(p.iplr, sAl[r]);
+                    const float bh = sNx[322];
                     p.dalpha[(t0 + r) * p.H + h] = sDg[r] / sAl[r] + (p.iplr ? 2.f * bh * sBe[r] * dbt : 0.f);
                     p.dbeta[(t0 + r) * p.H + h] = rsum(2, r) + bh * fr * dbt;
                     db_c = sBe[r] * fr * dbt;
@@ -1015,14 +1052,17 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 } else {
                     flag_error(p);
                 }
+                s_nslot = make_int2(ns.start, ns.len);
             }
         }
         __syncthreads();   // the staging tile read above takes the Q/K copies of the unit after next
         pre = has_next;
+        nslot = true;
         lph ^= 1;
         u = un;
         cur = nxt;
     }
+    cp_async_wait<0>();   // no scalar copy is still writing shared memory at exit
     // no tile copy is still writing shared memory at exit (after a give-up, the next unit's tiles are
     // in the phase after this one's, U^T / W^T and P in this one's)
     if (tid == kTma && pend) {
@@ -1050,6 +1090,7 @@ cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s) {
     int dev = 0, nsm = 0;
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     const long long units = (long long)p.slots * p.H;
+    if (units >= (1ll << 31)) return cudaErrorInvalidValue;   // unit indices are 32-bit in the kernel
     const int grid = (int)(units < nsm ? units : nsm);   // one resident CTA per SM
     tc::LocalMaps mp;
     const int Hk = p.H / p.vg;
