@@ -183,6 +183,15 @@ __device__ __forceinline__ void cp_async4(float* s, const float* g, bool valid) 
                  : "memory");
 }
 
+// Hand the tiles written so far to the tensor core, with `ok` made uniform over the block.
+__device__ __forceinline__ bool publish_ok(bool ok) {
+    fence_async_smem();
+    tc_fence_before();
+    const bool bad = __syncthreads_or(!ok);
+    tc_fence_after();
+    return !bad;
+}
+
 // Named barrier 1: the two tail warps only.
 __device__ __forceinline__ void tail_sync() { asm volatile("bar.sync 1, 64;\n" ::: "memory"); }
 
@@ -224,7 +233,7 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 // While unit u computes, the tiles of unit u + G stream into buffers as soon as their last
 // reader in unit u has finished (M after R3, H^T after R4, E (after the dv copy), dH'^T, dO and
 // Q/K (into the second of two alternating tiles, which holds M^T dE until then) after R5, V after
-// R6; the per-row scalars into registers), so the loads of consecutive units overlap the
+// R6; the per-row and per-head scalars by asynchronous copies after R3), so the loads of consecutive units overlap the
 // tensor-core and epilogue work instead of every SM loading at the same moment.  U^T and W^T of
 // the unit itself load into the dH'^T tile once R1 has read it.
 //
@@ -387,6 +396,16 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     const uint32_t tmem = tbase;
     const uint32_t tq = tmem + ((uint32_t)(32 * wr) << 16);   // this warp's TMEM lanes
     MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
+    // A round's wait: every thread on the commit's mbarrier, `ok` made uniform over the warp (warp-
+    // collective TMEM and fragment instructions follow) and over the block at the next block-wide
+    // barrier, which every round reaches before its next product is issued.
+    auto mma_wait = [&]() {
+        bool w = mbar_wait_polls(ms.wbar, ms.phase, ms.limit_ns);
+        ms.phase ^= 1;
+        w = __all_sync(0xffffffffu, w);
+        tc_fence_after();
+        return w;
+    };
     uint32_t ph0 = 0;   // phase of bar0 (R0, one commit per unit)
     const int nl0 = 8 * NL * wc, nk0 = 8 * NK * wc;   // this warp's columns of 64- and 128-wide results
     const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows
@@ -560,7 +579,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         {
             const bool ok0 = mbar_wait_polls(smem_u32(&bar0), ph0, p.wait_ns);
             ph0 ^= 1;
-            ok = !__syncthreads_or(!ok0);
+            ok = __all_sync(0xffffffffu, ok0);
             tc_fence_after();
         }
         // Each epilogue below first forms what the next round reads (P, dE, M^T dE, M^T dW, dG),
@@ -589,7 +608,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             frag_store_sw<NL>(sP, 64, m0, nl0, pv);
             frag_store_sw<NL>(sdPh, 64, m0, nl0, ph);
         }
-        publish_smem();
+        ok = publish_ok(ok);
 
         // ---------------- R2: P^T dO (dE = Kbar dH' + P^T dO) into the S and dP columns (read), behind
         // R1; one commit covers both.  The commit is made even when R0's wait gave up, so that the
@@ -626,7 +645,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 }
         }
         {
-            const bool ok2 = ms.wait(tid);
+            const bool ok2 = mma_wait();
             ok = ok && ok2;
         }
         // this unit's U^T, W^T (read by R5) into the dead dH'^T tile
@@ -653,7 +672,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             }
             frag_store_sw<NK>(sdEt, 64, m0, nk0, de);
         }
-        publish_smem();
+        ok = publish_ok(ok);
 
         // ---------------- R3: M^T dE, dPhat^T Q~ (into the columns dE was read from)
         if (tid == 0) {
@@ -685,7 +704,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             put_rows(1, s0, s1);
         }
         {
-            const bool ok3 = ms.wait(tid);
+            const bool ok3 = mma_wait();
             ok = ok && ok3;
         }
         if (ok && tid == kTma) {
@@ -713,7 +732,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             for (int t = 0; t < NK; ++t) { t3[t][0] *= ba; t3[t][1] *= ba; t3[t][2] *= bb; t3[t][3] *= bb; }
             frag_stage<NK>(stV, m0, nk0, t3);
         }
-        publish_smem();
+        ok = publish_ok(ok);
 
         // ---------------- R4: (M^T dE) H^T = -M^T dW (dW = -dE H^T) into M^T dE's columns (read), and
         // K K^T, dPhat K into the columns of the two R1 products read above
@@ -727,7 +746,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         if (ok) copy_stage_rows((bf16*)p.dvv + (t0 * p.H + h) * D, (long long)p.H * D, stV, L, tid);   // dv rows
         {
-            const bool ok4 = ms.wait(tid);
+            const bool ok4 = mma_wait();
             ok = ok && ok4;
         }
         if (ok && has_next && tid == kTma) { issue_n1(nxt); pend |= 2u; }   // R4 was H^T's last reader
@@ -750,7 +769,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 if (okl && L < kChunk) zero_rows(sPf, 64, L);
             fence_async_smem();
             tc_fence_before();
-            ok = ok && !__syncthreads_or(!okl);
+            ok = !__syncthreads_or(!okl);   // okl is false wherever ok is
             tc_fence_after();
         }
 
@@ -794,7 +813,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             put_rows(6, s0, s1);
         }
         {
-            const bool ok5 = ms.wait(tid);
+            const bool ok5 = mma_wait();
             ok = ok && ok5;
         }
         // the next unit's E (the dv rows, copied before R4's wait, were the E tile's last use), dH'^T
@@ -817,7 +836,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 }
             frag_store_sw<NL>(sdG, 64, m0, nl0, g4);
         }
-        publish_smem();
+        ok = publish_ok(ok);
 
         // ---------------- R6: dK += dPhat^T Q~ (already in TMEM) + dG K + dG^T K; with Comba-pk dG K is
         // dp's (into the dPhat K columns, read) and dk takes dG^T P
@@ -876,7 +895,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 }
         }
         {
-            const bool ok6 = ms.wait(tid);
+            const bool ok6 = mma_wait();
             ok = ok && ok6;
         }
         if (ok && has_next) {
@@ -890,7 +909,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) acc_dk[t][i] += t6[t][i];
         }
-        __syncthreads();   // every row dot has read the Q~/K tile
+        ok = !__syncthreads_or(!ok);   // every row dot has read the Q~/K tile
         if (ok) {
             // a full chunk leaves by bulk tensor stores from swizzled tiles, which run behind the
             // per-position tail; a partial one by row copies (a 64-row box would pass its end)
@@ -1055,7 +1074,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
                 s_nslot = make_int2(ns.start, ns.len);
             }
         }
-        __syncthreads();   // the staging tile read above takes the Q/K copies of the unit after next
+        ok = !__syncthreads_or(!ok);   // the staging tile read above takes the Q/K copies of the unit after next
         pre = has_next;
         nslot = true;
         lph ^= 1;
