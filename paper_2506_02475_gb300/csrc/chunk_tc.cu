@@ -150,7 +150,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
     // Gram K K^T over the 128-row tile (P K^T in lanes 0..63 for Comba-pk).
     if (tid == 0 && ok) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sKk), 128, 64, D, false);
     if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;
-    ok = ms.finish(tid) && ok;
+    ok = ms.finish_warp(tid) && ok;
     if (ok && !pk) {
         // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T), stored transposed; exp only
         // below the diagonal.  Lane l holds Gram row l & 63; its two threads fill columns
@@ -176,7 +176,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
             sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
         }
     }
-    __syncthreads();
+    ok = !__syncthreads_or(!ok);   // the inverse's barriers below need a block-uniform flag
     if (ok) {
         unit_lower_inverse64_h16(sAt, sM, 65, sTi, tid);
         __syncthreads();
@@ -205,7 +205,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
         tc_gemm<true, false>(tmem + 64, smem_u32(sK), 128, smem_u32(sMw), 64, 64, 64, false);
         tc_gemm<true, false>(tmem + 128, smem_u32(sV), 64, smem_u32(sMu), 64, 64, 64, false);
     }
-    ok = ok && ms.finish(tid);
+    ok = ok && ms.finish_warp(tid);   // (ok is block-uniform here: every thread takes the same branch)
     // W^T and U^T for the workspace are staged over the dead V and Mw/Mu tiles.
     uint8_t* stW = sV;
     uint8_t* stU = sMw;
@@ -240,7 +240,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
             }
         }
     }
-    publish_smem();
+    ok = publish_ok(ok);
 
     // Atilde = -K^T (Diag(s) W) -> cols [0,128)
     if (ok && tid == 0) tc_gemm<true, false>(tmem, smem_u32(sKk), 128, smem_u32(sWt), 128, 128, 64, false);
@@ -252,7 +252,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
         for (int e = tid; e < 128 * 8; e += NTH)
             us[e] = *reinterpret_cast<const uint4*>(sUt + sw128_offset(e >> 3, 8 * (e & 7), 128));
     }
-    ok = ok && ms.finish(tid);
+    ok = ok && ms.finish_warp(tid);
     // Atilde over the dead K tile
     uint8_t* stA = sK;
     if (ok) {
@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
             }
         }
     }
-    __syncthreads();
+    ok = !__syncthreads_or(!ok);
     if (ok) copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
     if (!ok) {
         if (tid == 0) {
@@ -474,7 +474,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p, const __grid_c
         }
         if (Zg) tc_gemm<false, false>(tmem + 192, smem_u32(sWt), 128, smem_u32(sP), 64, 64, 64, false);
     }
-    if (mma2) ok = ok && ms.finish(tid);
+    if (mma2) ok = ok && ms.finish_warp(tid);   // (ok is block-uniform before it)
     // W^T, E^T and H^T are dead: E, Z^T and O are staged over them.
     if (ok && Eg) {
 #pragma unroll
@@ -510,7 +510,7 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p, const __grid_c
             *reinterpret_cast<bf16*>(oh + sw128_offset(32 * half + c, row & 63, 64)) = __float2bfloat16_rn(d[c]);
     }
     fence_async_smem();
-    __syncthreads();
+    ok = !__syncthreads_or(!ok);
     if (ok && tid == 0) {
         if (Eg) bulk_copy_s2g(Eg, smem_u32(sE), 64 * D * 2);
         if (Zg) tma_store_2d(&mp.z, 0, (int)(idx * 128), smem_u32(stZ));

@@ -183,15 +183,6 @@ __device__ __forceinline__ void cp_async4(float* s, const float* g, bool valid) 
                  : "memory");
 }
 
-// Hand the tiles written so far to the tensor core, with `ok` made uniform over the block.
-__device__ __forceinline__ bool publish_ok(bool ok) {
-    fence_async_smem();
-    tc_fence_before();
-    const bool bad = __syncthreads_or(!ok);
-    tc_fence_after();
-    return !bad;
-}
-
 // Named barrier 1: the two tail warps only.
 __device__ __forceinline__ void tail_sync() { asm volatile("bar.sync 1, 64;\n" ::: "memory"); }
 
@@ -399,13 +390,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     // A round's wait: every thread on the commit's mbarrier, `ok` made uniform over the warp (warp-
     // collective TMEM and fragment instructions follow) and over the block at the next block-wide
     // barrier, which every round reaches before its next product is issued.
-    auto mma_wait = [&]() {
-        bool w = mbar_wait_polls(ms.wbar, ms.phase, ms.limit_ns);
-        ms.phase ^= 1;
-        w = __all_sync(0xffffffffu, w);
-        tc_fence_after();
-        return w;
-    };
+    auto mma_wait = [&]() { return ms.wait_warp(); };
     uint32_t ph0 = 0;   // phase of bar0 (R0, one commit per unit)
     const int nl0 = 8 * NL * wc, nk0 = 8 * NK * wc;   // this warp's columns of 64- and 128-wide results
     const int ra = m0 + frag_row(0), rb = m0 + frag_row(2);   // this lane's two rows

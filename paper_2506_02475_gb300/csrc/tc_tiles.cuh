@@ -62,6 +62,20 @@ struct MmaSync {
         tc_fence_after();
         return !any_bad;
     }
+    // The same two without a block-wide barrier: `ok` comes out uniform over the warp only (the
+    // warp-collective TMEM reads that follow need that much), and the caller makes it uniform over
+    // the block at its next block-wide barrier, before it issues another product.
+    __device__ __forceinline__ bool finish_warp(int tid) {
+        if (tid == 0) tc_commit(bar);
+        return wait_warp();
+    }
+    __device__ __forceinline__ bool wait_warp() {
+        const bool ok = mbar_wait_polls(wbar, phase, limit_ns);
+        phase ^= 1;
+        const bool all = __all_sync(0xffffffffu, ok);
+        tc_fence_after();
+        return all;
+    }
     // After a failed finish (the kernel then issues no further product): the commit whose wait
     // gave up covers every product thread 0 has issued, so waiting (again) for that phase means
     // nothing writes TMEM once the kernel releases it.  `phase` has moved past it, and a parity
@@ -71,6 +85,15 @@ struct MmaSync {
         if (tid == 0) mbar_drain(bar, phase ^ 1);
     }
 };
+
+// Hand the tiles written so far to the tensor core, with `ok` made uniform over the block.
+__device__ __forceinline__ bool publish_ok(bool ok) {
+    fence_async_smem();
+    tc_fence_before();
+    const bool bad = __syncthreads_or(!ok);
+    tc_fence_after();
+    return !bad;
+}
 
 __device__ __forceinline__ void flag_error(const ChunkParams& p) {
     if (p.err) atomicExch(p.err, 1);
