@@ -894,7 +894,8 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) acc_dk[t][i] += t6[t][i];
         }
-        ok = !__syncthreads_or(!ok);   // every row dot has read the Q~/K tile
+        // dq, dk staged over the Q~/K tile: its last readers were R6 (complete for every warp that saw
+        // the wait end) and the row dots of R5's epilogue (before the block-wide barrier ahead of R6)
         if (ok) {
             // a full chunk leaves by bulk tensor stores from swizzled tiles, which run behind the
             // per-position tail; a partial one by row copies (a 64-row box would pass its end)
@@ -927,7 +928,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
         if (L == kChunk) fence_async_smem();
         tc_fence_before();   // every TMEM read of this unit is done: the next unit's products may follow
-        __syncthreads();
+        ok = !__syncthreads_or(!ok);
         tc_fence_after();
         if (ok) {
             if (L == kChunk) {
