@@ -303,24 +303,20 @@ struct OutMaps {
 };
 
 // 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
-// Tiles arrive by TMA in two groups: Q and K (all that Q~, S = Q~ K^T and P need), then H^T, W^T
-// and U^T, so that Q~, S and P overlap the larger load.  O and Z^T leave by bulk tensor stores
+// Persistent: two CTAs per SM, CTA b taking units b, b + G, b + 2G, ... (G = gridDim.x).  Tiles
+// arrive by TMA in two groups: Q and K (all that Q~, S = Q~ K^T and P need), requested as soon as
+// the previous unit's Qhat is dead, and H^T, W^T and U^T, requested once the previous unit's
+// bulk stores have read their staging tiles, so that a unit's Q/K load overlaps the previous
+// unit's stores and Q~, S and P overlap the larger load.  O and Z^T leave by bulk tensor stores
 // and E by a bulk copy, from staging tiles over the dead inputs.
-__global__ void __launch_bounds__(256) k_output_tc(ChunkParams p, const __grid_constant__ OutMaps mp) {
+__global__ void __launch_bounds__(256, 2) k_output_tc(ChunkParams p, long long pairs, const __grid_constant__ OutMaps mp) {
     constexpr int NTH = 256;
     using S = OutTcSmem;
     extern __shared__ uint8_t smem_raw[];
     // ldA: Q/K landed; ldB: H^T, W^T, U^T landed; barS: S; barE: H^T W^T; bar: the second products;
-    // stall_bar: nothing arrives (COMBA_DIAG_STALL)
+    // stall_bar: nothing arrives (COMBA_DIAG_STALL).  ldA .. barE complete one phase per unit.
     __shared__ uint64_t ldA, ldB, barS, barE, bar, stall_bar;
     __shared__ uint32_t tbase;
-    const int slot = blockIdx.x, h = blockIdx.y;
-    const SlotInfo si = p.slot_info[slot];
-    if (si.len <= 0) return;
-    const int L = si.len;
-    const long long t0 = si.start;
-    const long long idx = (long long)slot * p.H + h;
-    const int hk = h / p.vg;   // key head of value head h
     const int tid = threadIdx.x, warp = tid >> 5;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQK = sm + S::OQK;
@@ -344,202 +340,246 @@ __global__ void __launch_bounds__(256) k_output_tc(ChunkParams p, const __grid_c
         mbar_init(smem_u32(&stall_bar), 1);
         mbar_fence_init();
     }
-    const float dh = p.d[hk];
-    const float gv = tid < 64 ? p.Gb[idx * 64 + tid] : 0.f;
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (tid == 0) {
-        mbar_expect_tx(uA, 32768u);
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            tma_load_3d(smem_u32(sQK) + half * 16384, &mp.q, 64 * half, hk, (int)t0, uA);
-            tma_load_3d(smem_u32(sQK) + 8192 + half * 16384, &mp.k, 64 * half, hk, (int)t0, uA);
-        }
-        mbar_expect_tx(uB, 65536u);
-        tma_load_2d(smem_u32(sWt), &mp.w, 0, (int)(idx * 128), uB);
-        tma_load_2d(smem_u32(sUt), &mp.u, 0, (int)(idx * 128), uB);
-#pragma unroll
-        for (int half = 0; half < 2; ++half) tma_load_2d(smem_u32(sHt) + half * 16384, &mp.h, 64 * half, (int)(idx * 128), uB);
-    }
-    if (tid < 64) sG[tid] = gv;
     const uint32_t tmem = tbase;
     MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
     const int row = tid & 127, half = tid >> 7;   // TMEM lane, and which 32 of each 64 columns
     const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-
-    // Q and K in; rows past a short chunk hold the next sequence's tokens: zero them
-    const bool okA = mbar_wait_polls(uA, 0, p.wait_ns);
-    if (L < kChunk) {
-        for (int e = tid; okA && e < (64 - L) * 16; e += NTH) {
-            const int r = L + (e >> 4), ch = e & 15;
-            *reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128)) = make_uint4(0, 0, 0, 0);
-            *reinterpret_cast<uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128)) = make_uint4(0, 0, 0, 0);
-        }
-        __syncthreads();
-    }
-    // Q~ = Q - d K (rows < L)
-    for (int e = tid; okA && e < L * 16; e += NTH) {
-        const int r = e >> 4, ch = e & 15;
-        uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
-        const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
-        float qv[8], kv[8];
-        unpack8(*qa, qv);
-        unpack8(ka, kv);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) qv[i] -= dh * kv[i];
-        *qa = pack8(qv);
-    }
-    fence_async_smem();
-    tc_fence_before();
-    bool ok = !__syncthreads_or(!okA);
-    tc_fence_after();
-
-    // [Q~; K] K^T -> cols [0,64) (lanes 0-63: S = Q~ K^T; lanes 64-127 unused), then, once H^T, W^T
-    // and U^T are in, E^T' = H^T W^T -> cols [64,128), each on its own barrier
-    if (tid == 0) {
-        if (ok) tc_gemm<false, false>(tmem, smem_u32(sQK), 128, smem_u32(sQK) + 64 * 128, 128, 64, D, false);
-        tc_commit(smem_u32(&barS));
-    }
-    bool okB = mbar_wait_polls(uB, 0, p.wait_ns);
-    if (tid == 0) {
-        if (ok && okB) tc_gemm<false, true>(tmem + 64, smem_u32(sHt), 128, smem_u32(sWt), 128, 64, D, false);
-        tc_commit(smem_u32(&barE));
-    }
-    bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
+    const uint32_t Hh = (uint32_t)p.H;            // (unit indices fit 32 bits: the launcher checks)
     const bool Zg = p.Zb != nullptr;
-    uint32_t ev[16];   // this thread's 32 positions of row j of E^T, packed bf16 pairs
-    const bool okS = mbar_wait_polls(smem_u32(&barS), 0, p.wait_ns);
-    tc_fence_after();
-    if (ok && okS) {
-        if (row < 64) {
-            // P = Tril(S * Gamma) into a K-major [64][64] tile (B operand of E^T P^T), over K
+    const bool mma2 = p.o || Zg;
+
+    // a unit's slot, d and log-decays, requested a unit ahead
+    auto fetch = [&](long long x, SlotInfo& si, float& d, float& g) {
+        const uint32_t sl = (uint32_t)x / Hh;
+        const int hx = (int)((uint32_t)x - sl * Hh);
+        si = p.slot_info[sl];
+        d = p.d[hx / p.vg];
+        g = tid < 64 ? p.Gb[x * 64 + tid] : 0.f;
+    };
+    auto issue_qk = [&](long long t0x, int hkx) {   // thread 0
+        mbar_expect_tx(uA, 32768u);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            tma_load_3d(smem_u32(sQK) + hh * 16384, &mp.q, 64 * hh, hkx, (int)t0x, uA);
+            tma_load_3d(smem_u32(sQK) + 8192 + hh * 16384, &mp.k, 64 * hh, hkx, (int)t0x, uA);
+        }
+    };
+
+    bool ok = true;
+    uint32_t ph = 0;       // phase parity of ldA .. barE for the current unit
+    bool pendA = false;    // thread 0: the coming unit's Q/K are requested already
+    long long u = blockIdx.x;
+    SlotInfo si{0, 0, 0, 0};
+    float dh = 0.f, gv = 0.f;
+    if (u < pairs) fetch(u, si, dh, gv);
+    for (; u < pairs && ok; u += gridDim.x) {
+        const SlotInfo sc = si;
+        const float dhc = dh, gvc = gv;
+        const long long un = u + gridDim.x;
+        if (un < pairs) fetch(un, si, dh, gv);
+        if (sc.len <= 0) continue;
+        const int L = sc.len;
+        const long long t0 = sc.start;
+        const long long idx = u;
+        const int h = (int)((uint32_t)u % Hh), hk = h / p.vg;
+
+        if (tid == 0) {
+            if (!pendA) issue_qk(t0, hk);
+            pendA = false;
+            bulk_wait_all_reads();   // the previous unit's stores have read W^T, U^T, H^T's tiles
+            mbar_expect_tx(uB, 65536u);
+            tma_load_2d(smem_u32(sWt), &mp.w, 0, (int)(idx * 128), uB);
+            tma_load_2d(smem_u32(sUt), &mp.u, 0, (int)(idx * 128), uB);
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh)
+                tma_load_2d(smem_u32(sHt) + hh * 16384, &mp.h, 64 * hh, (int)(idx * 128), uB);
+        }
+        if (tid < 64) sG[tid] = gvc;
+
+        // Q and K in; rows past a short chunk hold the next sequence's tokens: zero them
+        const bool okA = mbar_wait_polls(uA, ph, p.wait_ns);
+        if (L < kChunk) {
+            for (int e = tid; okA && e < (64 - L) * 16; e += NTH) {
+                const int r = L + (e >> 4), ch = e & 15;
+                *reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128)) = make_uint4(0, 0, 0, 0);
+                *reinterpret_cast<uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128)) = make_uint4(0, 0, 0, 0);
+            }
+            __syncthreads();
+        }
+        // Q~ = Q - d K (rows < L)
+        for (int e = tid; okA && e < L * 16; e += NTH) {
+            const int r = e >> 4, ch = e & 15;
+            uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
+            const uint4 ka = *reinterpret_cast<const uint4*>(sQK + sw128_offset(64 + r, 8 * ch, 128));
+            float qv[8], kv[8];
+            unpack8(*qa, qv);
+            unpack8(ka, kv);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) qv[i] -= dhc * kv[i];
+            *qa = pack8(qv);
+        }
+        fence_async_smem();
+        tc_fence_before();
+        ok = !__syncthreads_or(!okA);
+        tc_fence_after();
+
+        // [Q~; K] K^T -> cols [0,64) (lanes 0-63: S = Q~ K^T; lanes 64-127 unused), then, once H^T,
+        // W^T and U^T are in, E^T' = H^T W^T -> cols [64,128), each on its own barrier
+        if (tid == 0) {
+            if (ok) tc_gemm<false, false>(tmem, smem_u32(sQK), 128, smem_u32(sQK) + 64 * 128, 128, 64, D, false);
+            tc_commit(smem_u32(&barS));
+        }
+        const bool okB = mbar_wait_polls(uB, ph, p.wait_ns);
+        if (tid == 0) {
+            if (ok && okB) tc_gemm<false, true>(tmem + 64, smem_u32(sHt), 128, smem_u32(sWt), 128, 64, D, false);
+            tc_commit(smem_u32(&barE));
+        }
+        bf16* Eg = p.Eb ? (bf16*)p.Eb + idx * 64 * D : nullptr;
+        uint32_t ev[16];   // this thread's 32 positions of row j of E^T, packed bf16 pairs
+        const bool okS = mbar_wait_polls(smem_u32(&barS), ph, p.wait_ns);
+        tc_fence_after();
+        if (ok && okS) {
+            if (row < 64) {
+                // P = Tril(S * Gamma) into a K-major [64][64] tile (B operand of E^T P^T), over K
+                float d[32], v[8];
+                tmem_ld32(trow + half * 32, d);
+                const float gr = sG[row];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const int i = 32 * half + 8 * q + e;
+                        v[e] = (i <= row && row < L) ? d[8 * q + e] * __expf(gr - sG[i]) : 0.f;
+                    }
+                    *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * half + 8 * q, 64)) = pack8(v);
+                }
+            } else {
+                // the warps of TMEM lanes 64-127 (no S rows): Qhat = Diag(gamma) Q~ in place
+                for (int e = (tid & 63) + 64 * half; e < 64 * 16; e += 128) {
+                    const int r = e >> 4, ch = e & 15;
+                    uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
+                    float qv[8];
+                    unpack8(*qa, qv);
+                    const float gr = __expf(sG[r]);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) qv[i] *= gr;
+                    *qa = pack8(qv);
+                }
+            }
+        }
+        const bool okE = mbar_wait_polls(smem_u32(&barE), ph, p.wait_ns) && okB;
+        tc_fence_after();
+        if (ok && okE) {
+            // E^T = U^T - H^T W^T  (half of row j of E^T per thread)
             float d[32], v[8];
-            tmem_ld32(trow + half * 32, d);
-            const float gr = sG[row];
+            tmem_ld32(trow + 64 + half * 32, d);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float uu[8];
+                unpack8(*reinterpret_cast<const uint4*>(sUt + sw128_offset(row, 32 * half + 8 * q, 128)), uu);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) v[e] = uu[e] - d[8 * q + e];
+                // in place: each thread reads and then overwrites only these 16 bytes of its own row
+                const uint4 pk = pack8(v);
+                *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * half + 8 * q, 128)) = pk;
+                const int b0 = 4 * q;
+                ev[b0] = pk.x; ev[b0 + 1] = pk.y; ev[b0 + 2] = pk.z; ev[b0 + 3] = pk.w;
+            }
+        }
+        fence_async_smem();
+        tc_fence_before();
+        ok = !__syncthreads_or(!(ok && okS && okE));
+        tc_fence_after();
+
+        // O^T = H^T Qhat^T + E^T P^T -> cols [128,192);  (P W)^T = W^T P^T -> cols [192,256)
+        if (ok && tid == 0) {
+            if (p.o) {
+                tc_gemm<false, false>(tmem + 128, smem_u32(sHt), 128, smem_u32(sQK), 128, 64, D, false);
+                tc_gemm<false, false>(tmem + 128, smem_u32(sEt), 128, smem_u32(sP), 64, 64, 64, true);
+            }
+            if (Zg) tc_gemm<false, false>(tmem + 192, smem_u32(sWt), 128, smem_u32(sP), 64, 64, 64, false);
+        }
+        if (mma2) ok = ok && ms.finish_warp(tid);   // (ok is block-uniform before it)
+        // W^T, E^T and H^T are dead: E, Z^T and O are staged over them.
+        if (ok && Eg) {
+#pragma unroll
+            for (int pp = 0; pp < 16; ++pp) {
+                const __nv_bfloat162 two = *reinterpret_cast<const __nv_bfloat162*>(&ev[pp]);
+                sE[(32 * half + 2 * pp) * D + row] = two.x;
+                sE[(32 * half + 2 * pp + 1) * D + row] = two.y;
+            }
+        }
+        if (ok && Zg) {
+            // Z^T = Qhat^T - (P W)^T: row `row` (a key dimension), positions [32 half, +32); columns
+            // past a short chunk are zero because Qhat and P rows past it are
+            float d[32], v[8];
+            tmem_ld32(trow + 192 + half * 32, d);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
-                    const int i = 32 * half + 8 * q + e;
-                    v[e] = (i <= row && row < L) ? d[8 * q + e] * __expf(gr - sG[i]) : 0.f;
+                    const int t = 32 * half + 8 * q + e;
+                    const float qh = __bfloat162float(*reinterpret_cast<const bf16*>(sQK + sw128_offset(t, row, 128)));
+                    v[e] = qh - d[8 * q + e];
                 }
-                *reinterpret_cast<uint4*>(sP + sw128_offset(row, 32 * half + 8 * q, 64)) = pack8(v);
+                *reinterpret_cast<uint4*>(stZ + sw128_offset(row, 32 * half + 8 * q, 128)) = pack8(v);
             }
-        } else {
-            // the warps of TMEM lanes 64-127 (no S rows): Qhat = Diag(gamma) Q~ in place
-            for (int e = (tid & 63) + 64 * half; e < 64 * 16; e += 128) {
+        }
+        if (ok && p.o) {
+            // O[t][j] for j = row, t in [32 half, +32): the [64][128] tile as two swizzled 64-column halves
+            float d[32];
+            tmem_ld32(trow + 128 + half * 32, d);
+            uint8_t* oh = stO + (row >> 6) * 8192;
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+                *reinterpret_cast<bf16*>(oh + sw128_offset(32 * half + c, row & 63, 64)) = __float2bfloat16_rn(d[c]);
+        }
+        fence_async_smem();
+        tc_fence_before();   // every TMEM read of the unit is done: the next unit's products may follow
+        ok = !__syncthreads_or(!ok);
+        tc_fence_after();
+        if (!ok) break;
+        if (tid == 0) {
+            if (Eg) bulk_copy_s2g(Eg, smem_u32(sE), 64 * D * 2);
+            if (Zg) tma_store_2d(&mp.z, 0, (int)(idx * 128), smem_u32(stZ));
+            if (p.o && L == kChunk)
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) tma_store_3d(&mp.o, 64 * hh, h, (int)t0, smem_u32(stO) + hh * 8192);
+            bulk_commit();
+            // the next unit's Q and K (Qhat's last readers were the Z^T staging and the second products)
+            if (un < pairs && si.len > 0) {
+                issue_qk(si.start, (int)((uint32_t)un % Hh) / p.vg);
+                pendA = true;
+            }
+        }
+        if (p.o && L < kChunk) {
+            // a short chunk by rows (a 64-row box would run into the next sequence)
+            bf16* Og = (bf16*)p.o + (t0 * p.H + h) * D;
+            for (int e = tid; e < L * 16; e += NTH) {
                 const int r = e >> 4, ch = e & 15;
-                uint4* qa = reinterpret_cast<uint4*>(sQK + sw128_offset(r, 8 * ch, 128));
-                float qv[8];
-                unpack8(*qa, qv);
-                const float gr = __expf(sG[r]);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) qv[i] *= gr;
-                *qa = pack8(qv);
+                *reinterpret_cast<uint4*>(Og + (long long)r * p.H * D + 8 * ch) =
+                    *reinterpret_cast<const uint4*>(stO + (ch >> 3) * 8192 + sw128_offset(r, 8 * (ch & 7), 64));
             }
         }
-    }
-    const bool okE = mbar_wait_polls(smem_u32(&barE), 0, p.wait_ns) && okB;
-    tc_fence_after();
-    if (ok && okE) {
-        // E^T = U^T - H^T W^T  (half of row j of E^T per thread)
-        float d[32], v[8];
-        tmem_ld32(trow + 64 + half * 32, d);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            float u[8];
-            unpack8(*reinterpret_cast<const uint4*>(sUt + sw128_offset(row, 32 * half + 8 * q, 128)), u);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) v[e] = u[e] - d[8 * q + e];
-            // in place: each thread reads and then overwrites only these 16 bytes of its own row
-            const uint4 pk = pack8(v);
-            *reinterpret_cast<uint4*>(sEt + sw128_offset(row, 32 * half + 8 * q, 128)) = pk;
-            const int b0 = 4 * q;
-            ev[b0] = pk.x; ev[b0 + 1] = pk.y; ev[b0 + 2] = pk.z; ev[b0 + 3] = pk.w;
-        }
-    }
-    fence_async_smem();
-    tc_fence_before();
-    ok = !__syncthreads_or(!(ok && okS && okE));
-    tc_fence_after();
-
-    // O^T = H^T Qhat^T + E^T P^T -> cols [128,192);  (P W)^T = W^T P^T -> cols [192,256)
-    const bool mma2 = p.o || Zg;
-    if (ok && tid == 0) {
-        if (p.o) {
-            tc_gemm<false, false>(tmem + 128, smem_u32(sHt), 128, smem_u32(sQK), 128, 64, D, false);
-            tc_gemm<false, false>(tmem + 128, smem_u32(sEt), 128, smem_u32(sP), 64, 64, 64, true);
-        }
-        if (Zg) tc_gemm<false, false>(tmem + 192, smem_u32(sWt), 128, smem_u32(sP), 64, 64, 64, false);
-    }
-    if (mma2) ok = ok && ms.finish_warp(tid);   // (ok is block-uniform before it)
-    // W^T, E^T and H^T are dead: E, Z^T and O are staged over them.
-    if (ok && Eg) {
-#pragma unroll
-        for (int pp = 0; pp < 16; ++pp) {
-            const __nv_bfloat162 two = *reinterpret_cast<const __nv_bfloat162*>(&ev[pp]);
-            sE[(32 * half + 2 * pp) * D + row] = two.x;
-            sE[(32 * half + 2 * pp + 1) * D + row] = two.y;
-        }
-    }
-    if (ok && Zg) {
-        // Z^T = Qhat^T - (P W)^T: row `row` (a key dimension), positions [32 half, +32); columns
-        // past a short chunk are zero because Qhat and P rows past it are
-        float d[32], v[8];
-        tmem_ld32(trow + 192 + half * 32, d);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const int t = 32 * half + 8 * q + e;
-                const float qh = __bfloat162float(*reinterpret_cast<const bf16*>(sQK + sw128_offset(t, row, 128)));
-                v[e] = qh - d[8 * q + e];
-            }
-            *reinterpret_cast<uint4*>(stZ + sw128_offset(row, 32 * half + 8 * q, 128)) = pack8(v);
-        }
-    }
-    if (ok && p.o) {
-        // O[t][j] for j = row, t in [32 half, +32): the [64][128] tile as two swizzled 64-column halves
-        float d[32];
-        tmem_ld32(trow + 128 + half * 32, d);
-        uint8_t* oh = stO + (row >> 6) * 8192;
-#pragma unroll
-        for (int c = 0; c < 32; ++c)
-            *reinterpret_cast<bf16*>(oh + sw128_offset(32 * half + c, row & 63, 64)) = __float2bfloat16_rn(d[c]);
-    }
-    fence_async_smem();
-    ok = !__syncthreads_or(!ok);
-    if (ok && tid == 0) {
-        if (Eg) bulk_copy_s2g(Eg, smem_u32(sE), 64 * D * 2);
-        if (Zg) tma_store_2d(&mp.z, 0, (int)(idx * 128), smem_u32(stZ));
-        if (p.o && L == kChunk)
-#pragma unroll
-            for (int hh = 0; hh < 2; ++hh) tma_store_3d(&mp.o, 64 * hh, h, (int)t0, smem_u32(stO) + hh * 8192);
-        bulk_commit();
-    }
-    if (ok && p.o && L < kChunk) {
-        // a short chunk by rows (a 64-row box would run into the next sequence)
-        bf16* Og = (bf16*)p.o + (t0 * p.H + h) * D;
-        for (int e = tid; e < L * 16; e += NTH) {
-            const int r = e >> 4, ch = e & 15;
-            *reinterpret_cast<uint4*>(Og + (long long)r * p.H * D + 8 * ch) =
-                *reinterpret_cast<const uint4*>(stO + (ch >> 3) * 8192 + sw128_offset(r, 8 * (ch & 7), 64));
-        }
+        ph ^= 1;
+        __syncthreads();   // the O rows above have read their staging before the next unit's H^T load
     }
     if (!ok) {
         if (tid == 0) {
             flag_error(p);
             // let the tile loads and every product end before the block's shared memory and TMEM go
-            mbar_drain(uA, 0);
-            mbar_drain(uB, 0);
-            mbar_drain(smem_u32(&barS), 0);
-            mbar_drain(smem_u32(&barE), 0);
+            mbar_drain(uA, ph);
+            mbar_drain(uB, ph);
+            mbar_drain(smem_u32(&barS), ph);
+            mbar_drain(smem_u32(&barE), ph);
         }
         ms.drain(tid);
     }
-    if (ok && tid == 0) bulk_wait_all_reads();   // the stores have read their staging before exit
+    if (tid == 0) bulk_wait_all_reads();   // the stores have read their staging before exit
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -571,6 +611,9 @@ cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s) {
     if (e) return e;
     if (p.slots <= 0) return cudaSuccess;
     const long long pairs = (long long)p.slots * p.H;
+    if (pairs >= (1ll << 31)) return cudaErrorInvalidValue;   // unit indices are 32-bit in the kernel
+    int dev = 0, nsm = 0;
+    if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     tc::OutMaps mp;
     bool good = make_bf16_token_map(&mp.q, p.q, p.Ttot, p.H / p.vg, tc::D) &&
                 make_bf16_token_map(&mp.k, p.k, p.Ttot, p.H / p.vg, tc::D) &&
@@ -582,7 +625,9 @@ cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s) {
     if (good && p.Zb) good = make_bf16_map(&mp.z, p.Zb, pairs * tc::D, 64, tc::D);
     else mp.z = mp.w;   // not used
     if (!good) return cudaErrorInvalidValue;
-    tc::k_output_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p, mp);
+    const long long cap = 2ll * nsm;   // two resident CTAs per SM (shared memory and TMEM)
+    const int grid = (int)(pairs < cap ? pairs : cap);
+    tc::k_output_tc<<<grid, 256, sm, s>>>(p, pairs, mp);
     return cudaGetLastError();
 }
 
