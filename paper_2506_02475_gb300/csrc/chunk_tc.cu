@@ -49,21 +49,19 @@ struct PrepMaps {
     CUtensorMap k, p, v;
 };
 
-// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.  The
-// K (or [P; K]) and V tiles arrive by TMA while the warps load the gates and form the log-decays.
-__global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_constant__ PrepMaps mp) {
+// 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
+// Persistent: two CTAs per SM, CTA b taking units b, b + G, ... (G = gridDim.x).  A unit's gates
+// are requested at the previous unit's start and its K (or [P; K]) and V tiles by TMA as soon as
+// the previous unit's Atilde product has read K (Atilde is staged in the dead W^T / U_s^T region),
+// so that loads overlap the previous unit's last epilogue and copies.
+__global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pairs, const __grid_constant__ PrepMaps mp) {
     constexpr int NTH = 256;
     using S = PrepTcSmem;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar, stall_bar, ld;   // stall_bar: nothing arrives (COMBA_DIAG_STALL); ld: tiles
+    // stall_bar: nothing arrives (COMBA_DIAG_STALL); ld: a unit's tiles (one phase per unit)
+    __shared__ uint64_t bar, stall_bar, ld;
     __shared__ uint32_t tbase;
-    const int slot = blockIdx.x, h = blockIdx.y;
-    const SlotInfo si = p.slot_info[slot];
-    if (si.len <= 0) return;
-    const int L = si.len;
-    const long long t0 = si.start;
-    const long long idx = (long long)slot * p.H + h;
-    const int tid = threadIdx.x, warp = tid >> 5;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sK = sm + S::OK;
     uint8_t* sV = sm + S::OV;
@@ -74,6 +72,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
     float* sTi = sM + 64 * 65;                         // inverse scratch, 32 x 36
     uint8_t* sWt = sm + S::OR;            // aliases A after the inverse
     uint8_t* sUt = sm + S::OR + 16384;    // aliases M after Mw/Mu are built
+    uint8_t* stA = sm + S::OR;            // Atilde staging [128][128], once W^T / U_s^T are dead
     float* sG = reinterpret_cast<float*>(sm + S::OF);
     float* sGm1 = sG + 64;
     float* sBt = sG + 128;
@@ -86,194 +85,235 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, const __grid_
     // Comba-pk feedback vectors the tile is [P; K] instead: the Gram's lanes 0..63 hold
     // P K^T, and K (rows 64..127) is the operand of every later product that takes K.
     const bool pk = p.p != nullptr;
-    const int Hk = p.H / p.vg, hk = h / p.vg;   // key head of value head h
-    const int lane = tid & 31;
+    const int Hk = p.H / p.vg;
+    const uint32_t Hh = (uint32_t)p.H;   // (unit indices fit 32 bits: the launcher checks)
     if (tid == 0) {
         mbar_init(smem_u32(&bar), 1);
         mbar_init(smem_u32(&stall_bar), 1);
         mbar_init(smem_u32(&ld), 1);
         mbar_fence_init();
     }
-    const float* ag = p.alpha + t0 * Hk + hk;
-    float a0 = 1.f, a1 = 1.f, bev = 0.f, alv = 1.f, bh = 1.f;
-    if (warp == 0) {
-        a0 = lane < L ? ag[(long long)lane * Hk] : 1.f;
-        a1 = lane + 32 < L ? ag[(long long)(lane + 32) * Hk] : 1.f;
-    }
-    if (tid < 64) {
-        bev = tid < L ? p.beta[(t0 + tid) * Hk + hk] : 0.f;
-        alv = tid < L ? ag[(long long)tid * Hk] : 1.f;
-        bh = p.b ? p.b[hk] : 1.f;
-    }
     if (warp == 0) tmem_alloc(smem_u32(&tbase), 256);
     tc_fence_before();
     __syncthreads();   // barriers initialised, TMEM allocated
-    tc_fence_after();
-    if (tid == 0) {
-        const uint32_t mb = smem_u32(&ld);
-        mbar_expect_tx(mb, 32768u + 16384u);
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            tma_load_3d(smem_u32(sK) + half * 16384, pk ? &mp.p : &mp.k, 64 * half, hk, (int)t0, mb);
-            tma_load_3d(smem_u32(sK) + 8192 + half * 16384, &mp.k, 64 * half, hk, (int)t0, mb);
-            tma_load_3d(smem_u32(sV) + half * 8192, &mp.v, 64 * half, h, (int)t0, mb);
-        }
-    }
-    const uint8_t* sKk = pk ? sK + 64 * 128 : sK;   // the 64 key rows (rows 64.. of each K-half for pk)
-    if (warp == 0) chunk_log_cumsum_vals(a0, a1, L, sG, sGm1);
-    if (tid < 64) {
-        sBe[tid] = bev;
-        sBt[tid] = bh * bev * feedback_scale(p.iplr, alv);
-    }
-    __syncthreads();   // sG, sGm1, sBt complete
-    if (tid < 64) sWs[tid] = sBt[tid] * expf(sGm1[tid]);
-    // the tiles: rows past a short chunk hold the next sequence's tokens, zeroed here
-    const bool okl = mbar_wait_polls(smem_u32(&ld), 0, p.wait_ns);
-    if (okl && L < kChunk) {
-        for (int e = tid; e < (64 - L) * 16; e += NTH) {
-            const int r = L + (e >> 4), ch = e & 15;
-            const uint4 z = make_uint4(0, 0, 0, 0);
-            *reinterpret_cast<uint4*>(sK + sw128_offset(r, 8 * ch, 128)) = z;
-            *reinterpret_cast<uint4*>(sK + sw128_offset(64 + r, 8 * ch, 128)) = z;
-            *reinterpret_cast<uint4*>(sV + sw128_offset(r, 8 * ch, 64)) = z;
-        }
-    }
-    fence_async_smem();
-    tc_fence_before();
-    bool ok = !__syncthreads_or(!okl);
     tc_fence_after();
     const uint32_t tmem = tbase;
     MmaSync ms{smem_u32(&bar), smem_u32(p.stall ? &stall_bar : &bar), 0, p.wait_ns};
     const int row = tid & 127, half = tid >> 7;   // TMEM lane / accumulator row, and which column half
     const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    const uint8_t* sKk = pk ? sK + 64 * 128 : sK;   // the 64 key rows (rows 64.. of each K-half for pk)
 
-    // Gram K K^T over the 128-row tile (P K^T in lanes 0..63 for Comba-pk).
-    if (tid == 0 && ok) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sKk), 128, 64, D, false);
-    if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;
-    ok = ms.finish_warp(tid) && ok;
-    if (ok && !pk) {
-        // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T), stored transposed; exp only
-        // below the diagonal.  Lane l holds Gram row l & 63; its two threads fill columns
-        // [32 (l >> 6) + 16 half, +16).
-        const int r = row & 63, i0 = 32 * (row >> 6) + 16 * half;
-        float d[16];
-        tmem_ld16(trow + i0, d);
-        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
-#pragma unroll
-        for (int c = 0; c < 16; ++c) {
-            const int i = i0 + c;
-            sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+    // a unit's gates into registers: warp 0 the log-decay inputs, threads < 64 beta, alpha and b
+    struct Gates { float a0, a1, bev, alv, bh; };
+    auto fetch_gates = [&](long long x, const SlotInfo& si) {
+        Gates g{1.f, 1.f, 0.f, 1.f, 1.f};
+        const int hkx = (int)((uint32_t)x % Hh) / p.vg;
+        const float* ag = p.alpha + (long long)si.start * Hk + hkx;
+        if (warp == 0) {
+            g.a0 = lane < si.len ? ag[(long long)lane * Hk] : 1.f;
+            g.a1 = lane + 32 < si.len ? ag[(long long)(lane + 32) * Hk] : 1.f;
         }
-    } else if (ok && row < 64) {
-        // Comba-pk: P K^T rows are in lanes 0..63 only; the two threads of each take one column half.
-        const int r = row, i0 = 32 * half;
-        const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
-        float d[32];
-        tmem_ld32(trow + i0, d);
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            const int i = i0 + c;
-            sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+        if (tid < 64) {
+            g.bev = tid < si.len ? p.beta[((long long)si.start + tid) * Hk + hkx] : 0.f;
+            g.alv = tid < si.len ? ag[(long long)tid * Hk] : 1.f;
+            g.bh = p.b ? p.b[hkx] : 1.f;
         }
-    }
-    ok = !__syncthreads_or(!ok);   // the inverse's barriers below need a block-uniform flag
-    if (ok) {
-        unit_lower_inverse64_h16(sAt, sM, 65, sTi, tid);
+        return g;
+    };
+    auto slot_of = [&](long long x) { return x < pairs ? p.slot_info[(uint32_t)x / Hh] : SlotInfo{0, 0, 0, 0}; };
+    auto issue_tiles = [&](long long x, const SlotInfo& si) {   // thread 0
+        const int hx = (int)((uint32_t)x % Hh), hkx = hx / p.vg;
+        const uint32_t mb = smem_u32(&ld);
+        mbar_expect_tx(mb, 32768u + 16384u);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            tma_load_3d(smem_u32(sK) + hh * 16384, pk ? &mp.p : &mp.k, 64 * hh, hkx, si.start, mb);
+            tma_load_3d(smem_u32(sK) + 8192 + hh * 16384, &mp.k, 64 * hh, hkx, si.start, mb);
+            tma_load_3d(smem_u32(sV) + hh * 8192, &mp.v, 64 * hh, hx, si.start, mb);
+        }
+    };
+
+    bool ok = true;
+    uint32_t ph = 0;      // phase parity of `ld` for the current unit
+    bool pend = false;    // thread 0: the coming unit's tiles are requested already
+    long long u = blockIdx.x;
+    const long long G = gridDim.x;
+    SlotInfo s0 = slot_of(u), s1 = slot_of(u + G);   // this unit's slot and the next one's
+    Gates g0 = s0.len > 0 ? fetch_gates(u, s0) : Gates{1.f, 1.f, 0.f, 1.f, 1.f};
+    for (; u < pairs && ok; u += G) {
+        const SlotInfo sc = s0;
+        const Gates gc = g0;
+        s0 = s1;                                        // the next unit: its gates now, its slot's
+        g0 = s0.len > 0 ? fetch_gates(u + G, s0) : Gates{1.f, 1.f, 0.f, 1.f, 1.f};
+        s1 = slot_of(u + 2 * G);                        // successor a unit later
+        if (sc.len <= 0) continue;
+        const int L = sc.len;
+        const long long idx = u;
+
+        if (tid == 0) {
+            if (!pend) issue_tiles(u, sc);
+            pend = false;
+        }
+        if (warp == 0) chunk_log_cumsum_vals(gc.a0, gc.a1, L, sG, sGm1);
+        if (tid < 64) {
+            sBe[tid] = gc.bev;
+            sBt[tid] = gc.bh * gc.bev * feedback_scale(p.iplr, gc.alv);
+        }
+        __syncthreads();   // sG, sGm1, sBt complete
+        if (tid < 64) sWs[tid] = sBt[tid] * expf(sGm1[tid]);
+        // the tiles: rows past a short chunk hold the next sequence's tokens, zeroed here
+        const bool okl = mbar_wait_polls(smem_u32(&ld), ph, p.wait_ns);
+        if (okl && L < kChunk) {
+            for (int e = tid; e < (64 - L) * 16; e += NTH) {
+                const int r = L + (e >> 4), ch = e & 15;
+                const uint4 z = make_uint4(0, 0, 0, 0);
+                *reinterpret_cast<uint4*>(sK + sw128_offset(r, 8 * ch, 128)) = z;
+                *reinterpret_cast<uint4*>(sK + sw128_offset(64 + r, 8 * ch, 128)) = z;
+                *reinterpret_cast<uint4*>(sV + sw128_offset(r, 8 * ch, 64)) = z;
+            }
+        }
+        fence_async_smem();
+        tc_fence_before();
+        ok = !__syncthreads_or(!okl);
+        tc_fence_after();
+
+        // Gram K K^T over the 128-row tile (P K^T in lanes 0..63 for Comba-pk).
+        if (tid == 0 && ok) tc_gemm<false, false>(tmem, smem_u32(sK), 128, smem_u32(sKk), 128, 64, D, false);
+        if (tid < 64) sS[tid] = tid < L ? expf(sG[L - 1] - sG[tid]) : 0.f;
+        ok = ms.finish_warp(tid) && ok;
+        if (ok && !pk) {
+            // Strictly-lower A = Diag(btilde)(gamma_{r-1}/gamma_i * K K^T), stored transposed; exp only
+            // below the diagonal.  Lane l holds Gram row l & 63; its two threads fill columns
+            // [32 (l >> 6) + 16 half, +16).
+            const int r = row & 63, i0 = 32 * (row >> 6) + 16 * half;
+            float d[16];
+            tmem_ld16(trow + i0, d);
+            const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                const int i = i0 + c;
+                sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+            }
+        } else if (ok && row < 64) {
+            // Comba-pk: P K^T rows are in lanes 0..63 only; the two threads of each take one column half.
+            const int r = row, i0 = 32 * half;
+            const float br = r < L ? sBt[r] : 0.f, gr = sGm1[r];
+            float d[32];
+            tmem_ld32(trow + i0, d);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                const int i = i0 + c;
+                sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+            }
+        }
+        ok = !__syncthreads_or(!ok);   // the inverse's barriers below need a block-uniform flag
+        if (ok) {
+            unit_lower_inverse64_h16(sAt, sM, 65, sTi, tid);
+            __syncthreads();
+            // Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta) as K-major [p][p'] tiles; M saved for the backward.
+            bf16* Mg = p.Mb ? (bf16*)p.Mb + idx * 4096 : nullptr;
+            for (int e = tid; e < 64 * 8; e += NTH) {
+                const int r = e >> 3, ch = e & 7;
+                float mw[8], mu[8], mm[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const int c = 8 * ch + q;
+                    mm[q] = sM[r * 65 + c];
+                    mw[q] = mm[q] * sWs[c];
+                    mu[q] = mm[q] * sBe[c];
+                }
+                *reinterpret_cast<uint4*>(sMw + sw128_offset(r, 8 * ch, 64)) = pack8(mw);
+                *reinterpret_cast<uint4*>(sMu + sw128_offset(r, 8 * ch, 64)) = pack8(mu);
+                if (Mg) *reinterpret_cast<uint4*>(Mg + r * 64 + 8 * ch) = pack8(mm);
+            }
+            if (tid < 64) p.Gb[idx * 64 + tid] = sG[tid];
+        }
+        publish_smem();
+
+        // W^T = K^T Mw^T (A = K as MN-major; P^T Mw^T for Comba-pk, tile rows 0..63), U^T = V^T Mu^T.
+        if (ok && tid == 0) {
+            tc_gemm<true, false>(tmem + 64, smem_u32(sK), 128, smem_u32(sMw), 64, 64, 64, false);
+            tc_gemm<true, false>(tmem + 128, smem_u32(sV), 64, smem_u32(sMu), 64, 64, 64, false);
+        }
+        ok = ok && ms.finish_warp(tid);   // (ok is block-uniform here: every thread takes the same branch)
+        // W^T and U^T for the workspace are staged over the dead V and Mw/Mu tiles.
+        uint8_t* stW = sV;
+        uint8_t* stU = sMw;
+        if (ok) {
+            float d[32], v[8], w[8];
+            {
+                const int g = half;
+                tmem_ld32(trow + 64 + g * 32, d);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        v[e] = d[8 * q + e];
+                        w[e] = v[e] * sS[32 * g + 8 * q + e];
+                    }
+                    stage_chunk<8>(stW, row, 4 * g + q, pack8(v));
+                    *reinterpret_cast<uint4*>(sWt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
+                }
+            }
+            {
+                const int g = half;
+                tmem_ld32(trow + 128 + g * 32, d);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        v[e] = d[8 * q + e];
+                        w[e] = v[e] * sS[32 * g + 8 * q + e];
+                    }
+                    stage_chunk<8>(stU, row, 4 * g + q, pack8(v));
+                    *reinterpret_cast<uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
+                }
+            }
+        }
+        ok = publish_ok(ok);
+
+        // Atilde = -K^T (Diag(s) W) -> cols [0,128)
+        if (ok && tid == 0) tc_gemm<true, false>(tmem, smem_u32(sKk), 128, smem_u32(sWt), 128, 128, 64, false);
+        if (ok) {
+            // W^T, U^T and U_s^T (un-swizzled row by row) out while the tensor core works
+            copy_staged<8>((bf16*)p.Wb + idx * D * 64, stW, tid, NTH);
+            copy_staged<8>((bf16*)p.Ub + idx * D * 64, stU, tid, NTH);
+            uint4* us = reinterpret_cast<uint4*>((bf16*)p.Usb + idx * D * 64);
+            for (int e = tid; e < 128 * 8; e += NTH)
+                us[e] = *reinterpret_cast<const uint4*>(sUt + sw128_offset(e >> 3, 8 * (e & 7), 128));
+        }
+        ok = ok && ms.finish_warp(tid);
+        // K, V and the W^T / U^T / U_s^T staging are dead now, for every thread: the next unit's
+        // tiles may load, and Atilde is staged over W^T / U_s^T's region
+        ok = !__syncthreads_or(!ok);
+        if (!ok) break;
+        if (tid == 0 && u + G < pairs && s0.len > 0) {
+            issue_tiles(u + G, s0);
+            pend = true;
+        }
+        {
+            float d[32], v[8];
+#pragma unroll
+            for (int g = 2 * half; g < 2 * half + 2; ++g) {
+                tmem_ld32(trow + g * 32, d);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[e] = -d[8 * q + e];
+                    stage_chunk<16>(stA, row, 4 * g + q, pack8(v));
+                }
+            }
+        }
+        tc_fence_before();   // the unit's last TMEM reads: the next unit's Gram may follow
         __syncthreads();
-        // Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta) as K-major [p][p'] tiles; M saved for the backward.
-        bf16* Mg = p.Mb ? (bf16*)p.Mb + idx * 4096 : nullptr;
-        for (int e = tid; e < 64 * 8; e += NTH) {
-            const int r = e >> 3, ch = e & 7;
-            float mw[8], mu[8], mm[8];
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int c = 8 * ch + q;
-                mm[q] = sM[r * 65 + c];
-                mw[q] = mm[q] * sWs[c];
-                mu[q] = mm[q] * sBe[c];
-            }
-            *reinterpret_cast<uint4*>(sMw + sw128_offset(r, 8 * ch, 64)) = pack8(mw);
-            *reinterpret_cast<uint4*>(sMu + sw128_offset(r, 8 * ch, 64)) = pack8(mu);
-            if (Mg) *reinterpret_cast<uint4*>(Mg + r * 64 + 8 * ch) = pack8(mm);
-        }
-        if (tid < 64) p.Gb[idx * 64 + tid] = sG[tid];
+        tc_fence_after();
+        copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
+        ph ^= 1;
     }
-    publish_smem();
-
-    // W^T = K^T Mw^T (A = K as MN-major; P^T Mw^T for Comba-pk, tile rows 0..63), U^T = V^T Mu^T.
-    if (ok && tid == 0) {
-        tc_gemm<true, false>(tmem + 64, smem_u32(sK), 128, smem_u32(sMw), 64, 64, 64, false);
-        tc_gemm<true, false>(tmem + 128, smem_u32(sV), 64, smem_u32(sMu), 64, 64, 64, false);
-    }
-    ok = ok && ms.finish_warp(tid);   // (ok is block-uniform here: every thread takes the same branch)
-    // W^T and U^T for the workspace are staged over the dead V and Mw/Mu tiles.
-    uint8_t* stW = sV;
-    uint8_t* stU = sMw;
-    if (ok) {
-        float d[32], v[8], w[8];
-        {
-            const int g = half;
-            tmem_ld32(trow + 64 + g * 32, d);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    v[e] = d[8 * q + e];
-                    w[e] = v[e] * sS[32 * g + 8 * q + e];
-                }
-                stage_chunk<8>(stW, row, 4 * g + q, pack8(v));
-                *reinterpret_cast<uint4*>(sWt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
-            }
-        }
-        {
-            const int g = half;
-            tmem_ld32(trow + 128 + g * 32, d);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    v[e] = d[8 * q + e];
-                    w[e] = v[e] * sS[32 * g + 8 * q + e];
-                }
-                stage_chunk<8>(stU, row, 4 * g + q, pack8(v));
-                *reinterpret_cast<uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
-            }
-        }
-    }
-    ok = publish_ok(ok);
-
-    // Atilde = -K^T (Diag(s) W) -> cols [0,128)
-    if (ok && tid == 0) tc_gemm<true, false>(tmem, smem_u32(sKk), 128, smem_u32(sWt), 128, 128, 64, false);
-    if (ok) {
-        // W^T, U^T and U_s^T (un-swizzled row by row) out while the tensor core works
-        copy_staged<8>((bf16*)p.Wb + idx * D * 64, stW, tid, NTH);
-        copy_staged<8>((bf16*)p.Ub + idx * D * 64, stU, tid, NTH);
-        uint4* us = reinterpret_cast<uint4*>((bf16*)p.Usb + idx * D * 64);
-        for (int e = tid; e < 128 * 8; e += NTH)
-            us[e] = *reinterpret_cast<const uint4*>(sUt + sw128_offset(e >> 3, 8 * (e & 7), 128));
-    }
-    ok = ok && ms.finish_warp(tid);
-    // Atilde over the dead K tile
-    uint8_t* stA = sK;
-    if (ok) {
-        float d[32], v[8];
-#pragma unroll
-        for (int g = 2 * half; g < 2 * half + 2; ++g) {
-            tmem_ld32(trow + g * 32, d);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) v[e] = -d[8 * q + e];
-                stage_chunk<16>(stA, row, 4 * g + q, pack8(v));
-            }
-        }
-    }
-    ok = !__syncthreads_or(!ok);
-    if (ok) copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
     if (!ok) {
         if (tid == 0) {
             flag_error(p);
-            mbar_drain(smem_u32(&ld), 0);   // the tile loads have ended before the block's memory goes
+            mbar_drain(smem_u32(&ld), ph);   // the tile loads have ended before the block's memory goes
         }
         ms.drain(tid);
     }
@@ -595,13 +635,19 @@ cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(tc::k_prep_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e) return e;
     if (p.slots <= 0) return cudaSuccess;
+    const long long pairs = (long long)p.slots * p.H;
+    if (pairs >= (1ll << 31)) return cudaErrorInvalidValue;   // unit indices are 32-bit in the kernel
+    int dev = 0, nsm = 0;
+    if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     tc::PrepMaps mp;
     bool good = make_bf16_token_map(&mp.k, p.k, p.Ttot, p.H / p.vg, tc::D) &&
                 make_bf16_token_map(&mp.v, p.v, p.Ttot, p.H, tc::D);
     if (good && p.p) good = make_bf16_token_map(&mp.p, p.p, p.Ttot, p.H / p.vg, tc::D);
     else mp.p = mp.k;   // not used
     if (!good) return cudaErrorInvalidValue;
-    tc::k_prep_tc<<<dim3(p.slots, p.H), 256, sm, s>>>(p, mp);
+    const long long cap = 2ll * nsm;   // two resident CTAs per SM (shared memory and TMEM)
+    const int grid = (int)(pairs < cap ? pairs : cap);
+    tc::k_prep_tc<<<grid, 256, sm, s>>>(p, pairs, mp);
     return cudaGetLastError();
 }
 
