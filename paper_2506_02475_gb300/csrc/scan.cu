@@ -440,16 +440,6 @@ __global__ void __launch_bounds__(256, 1)
                 bad = 1;
             }
             tc_commit(smem_u32(&mma_bar));
-            // the next chunk's additive term, into the other accumulator (read back a chunk ago)
-            if (!bad && it + 1 < nch) {
-                if (!wait_f(it + 1)) {
-                    bad = ybad = 1;
-                } else {
-                    if constexpr (YM == 2)
-                        if (tail_short && it + 2 == nch) zero_tail(it + 1);
-                    issue_y(it + 1);
-                }
-            }
         } else if (tid == kTma) {
 #pragma unroll
             for (int half = 0; half < DK / 64; ++half)
@@ -495,6 +485,18 @@ __global__ void __launch_bounds__(256, 1)
 #pragma unroll
             for (int i = 0; i < 4; ++i) st[t][i] = fmaf(gam, st[t][i], __uint_as_float(d[4 * t + i]));
         tc_fence_before();
+        // The next chunk's additive term, into the other accumulator (read back a chunk ago), once
+        // this chunk's products are done: issued behind them it would hold every warp at the
+        // barrier above while thread 0 waits for room in the tensor core's queue.
+        if (tid == 0 && !ybad && it + 1 < nch) {
+            if (!wait_f(it + 1)) {
+                ybad = 1;
+            } else {
+                if constexpr (YM == 2)
+                    if (tail_short && it + 2 == nch) zero_tail(it + 1);
+                issue_y(it + 1);
+            }
+        }
     }
 
     if (tid == kTma) bulk_wait_all();
