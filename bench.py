@@ -161,11 +161,11 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 94_582, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "7621d3a0e62f2bf4"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_525, ('scan.cu', 'common.cuh', 'params.cuh'), "da98cd7442c7cea5"),
-    "output": ("k_output_tc", 130_675, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "7621d3a0e62f2bf4"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_760, ('scan.cu', 'common.cuh', 'params.cuh'), "da98cd7442c7cea5"),
-    "bwd_local": ("k_bwd_local_tc", 228_477, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "b2adf0cc52ccaec7"),
+    "prep": ("k_prep_tc", 93_606, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "9b9b54558a26911a"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_579, ('scan.cu', 'common.cuh', 'params.cuh'), "879cf75841488dc5"),
+    "output": ("k_output_tc", 130_522, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "9b9b54558a26911a"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_687, ('scan.cu', 'common.cuh', 'params.cuh'), "879cf75841488dc5"),
+    "bwd_local": ("k_bwd_local_tc", 228_304, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "2c56be22676c9724"),
 }
 DECODE_TRAFFIC = (481_360_000, ('decode.cu', 'common.cuh', 'params.cuh'), "ace440567370e7de")   # whole Bd=256 H=16 launch
 
