@@ -32,8 +32,8 @@
  *     are fp32 [num_seqs, H, dk, dv].  All arithmetic accumulates in fp32.
  *   - alpha must lie in (0, 1]: the chunk form takes logarithms of alpha.
  *   - All pointers must be 16-byte aligned.
- *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
- *     stream).  Outputs are overwritten, never accumulated into.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t, as comba_stream_t; NULL =
+ *     legacy default stream).  Outputs are overwritten, never accumulated into.
  *   - Validation is host-side only; invalid arguments return an error before
  *     anything is launched.  A failed launch returns COMBA_ERR_CUDA.
  *   - No global mutable state: calls on different streams may overlap as long
@@ -56,6 +56,12 @@
 
 #include <stddef.h>
 #include <stdint.h>
+
+/* The CUDA runtime's stream handle: the same type as cudaStream_t, declared here so that this
+ * header needs no CUDA include.  A cudaStream_t passes as it is; NULL is the legacy default
+ * stream. */
+struct CUstream_st;
+typedef struct CUstream_st *comba_stream_t;
 
 #ifdef __cplusplus
 extern "C" {
@@ -160,7 +166,7 @@ comba_status_t comba_chunk_fwd_gated(const comba_shape_t *shape,
                                      const float *g_alpha, const float *g_beta,
                                      const float *a, const float *c, const float *b_raw, const float *d,
                                      const float *h0, void *o, float *hT,
-                                     void *workspace, size_t workspace_bytes, void *stream);
+                                     void *workspace, size_t workspace_bytes, comba_stream_t stream);
 
 /*
  * The gated backward: gradients of L = <o,dO> + <hT,dhT> w.r.t. the raw inputs:
@@ -177,7 +183,7 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t *shape,
                                      const float *h0, const void *dO, const float *dhT,
                                      void *dq, void *dk, void *dv, float *dg_alpha, float *dg_beta,
                                      float *da, float *dc, float *db_raw, float *dd, float *dh0,
-                                     void *workspace, size_t workspace_bytes, void *stream);
+                                     void *workspace, size_t workspace_bytes, comba_stream_t stream);
 
 /*
  * Comba-pk (appendix B.3, the "p" form of the recurrence): a per-token feedback
@@ -215,7 +221,7 @@ comba_status_t comba_chunk_fwd_pk(const comba_shape_t *shape,
                                   const float *alpha, const float *beta,
                                   const float *b, const float *d, const float *h0,
                                   void *o, float *hT,
-                                  void *workspace, size_t workspace_bytes, void *stream);
+                                  void *workspace, size_t workspace_bytes, comba_stream_t stream);
 
 /*
  * The pk backward: as comba_chunk_bwd plus p and its gradient dp [B,T,H,dk]
@@ -232,7 +238,7 @@ comba_status_t comba_chunk_bwd_pk(const comba_shape_t *shape,
                                   const void *dO, const float *dhT,
                                   void *dq, void *dk, void *dv, void *dp,
                                   float *dalpha, float *dbeta, float *db, float *dd, float *dh0,
-                                  void *workspace, size_t workspace_bytes, void *stream);
+                                  void *workspace, size_t workspace_bytes, comba_stream_t stream);
 
 /*
  * Bytes of device workspace needed by comba_chunk_fwd (backward = 0) or
@@ -260,7 +266,7 @@ comba_status_t comba_chunk_fwd(const comba_shape_t *shape,
                                const float *alpha, const float *beta,
                                const float *b, const float *d, const float *h0,
                                void *o, float *hT,
-                               void *workspace, size_t workspace_bytes, void *stream);
+                               void *workspace, size_t workspace_bytes, comba_stream_t stream);
 
 /*
  * Chunk-parallel backward: exact gradients of
@@ -286,7 +292,7 @@ comba_status_t comba_chunk_bwd(const comba_shape_t *shape,
                                const void *dO, const float *dhT,
                                void *dq, void *dk, void *dv,
                                float *dalpha, float *dbeta, float *db, float *dd, float *dh0,
-                               void *workspace, size_t workspace_bytes, void *stream);
+                               void *workspace, size_t workspace_bytes, comba_stream_t stream);
 
 /*
  * One decode token (appendix B.1, recurrent form) for Bd independent rows:
@@ -307,7 +313,7 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
                                     const void *q, const void *k, const void *v,
                                     const float *alpha, const float *beta,
                                     const float *b, const float *d,
-                                    float *state, void *o, int flags, void *stream);
+                                    float *state, void *o, int flags, comba_stream_t stream);
 
 /*
  * One Comba-pk decode token: as comba_recurrent_step with the feedback vector
@@ -319,7 +325,7 @@ comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtyp
                                        const void *q, const void *k, const void *v, const void *p,
                                        const float *alpha, const float *beta,
                                        const float *b, const float *d,
-                                       float *state, void *o, int flags, void *stream);
+                                       float *state, void *o, int flags, comba_stream_t stream);
 
 /*
  * Forward without a caller workspace, for callers that may not allocate
@@ -345,7 +351,7 @@ comba_status_t comba_chunk_fwd_noalloc(const comba_shape_t *shape,
                                        const void *q, const void *k, const void *v,
                                        const float *alpha, const float *beta,
                                        const float *b, const float *d, const float *h0,
-                                       void *o, float *hT, void *stream);
+                                       void *o, float *hT, comba_stream_t stream);
 
 /*
  * Status of the device-side waits of the calls that last used `workspace`.
@@ -361,7 +367,7 @@ comba_status_t comba_chunk_fwd_noalloc(const comba_shape_t *shape,
  * comba_chunk_fwd_noalloc on the current device.  Nothing is allocated.
  * (No counterpart in the paper: the hot-path boundary's error reporting.)
  */
-comba_status_t comba_workspace_status(const void *workspace, void *stream);
+comba_status_t comba_workspace_status(const void *workspace, comba_stream_t stream);
 
 /* Static, human-readable name of a status code. */
 const char *comba_status_string(comba_status_t status);

@@ -235,8 +235,8 @@ size_t comba_workspace_size(const comba_shape_t* shape, int backward) {
     return L.total;
 }
 
-comba_status_t comba_workspace_status(const void* workspace, void* stream) {
-    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+comba_status_t comba_workspace_status(const void* workspace, comba_stream_t stream) {
+    const cudaStream_t s = stream;
     const void* word = workspace;   // the status word is the workspace's first 4 bytes (Layout::err = 0)
     if (!word) {
         void* scratch = nullptr;
@@ -348,7 +348,7 @@ extern "C" {
 comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const void* k, const void* v,
                                const float* alpha, const float* beta, const float* b, const float* d,
                                const float* h0, void* o, float* hT, void* workspace, size_t workspace_bytes,
-                               void* stream) {
+                               comba_stream_t stream) {
     Layout L;
     const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
     comba_status_t st = plan(shape, save ? 1 : 0, &L);
@@ -360,14 +360,14 @@ comba_status_t comba_chunk_fwd(const comba_shape_t* shape, const void* q, const 
     if (shape->stage_events && shape->num_stage_events < COMBA_FWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
     return forward_run(shape, L, workspace, q, k, v, alpha, beta, b, d, h0, o, hT, save,
-                       static_cast<cudaStream_t>(stream));
+                       stream);
 }
 
 comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const void* k, const void* v,
                                const float* alpha, const float* beta, const float* b, const float* d,
                                const float* h0, const void* dO, const float* dhT, void* dq, void* dk, void* dv,
                                float* dalpha, float* dbeta, float* db, float* dd, float* dh0, void* workspace,
-                               size_t workspace_bytes, void* stream) {
+                               size_t workspace_bytes, comba_stream_t stream) {
     Layout L;
     comba_status_t st = plan(shape, 1, &L);
     if (st != COMBA_OK) return st;
@@ -380,13 +380,13 @@ comba_status_t comba_chunk_bwd(const comba_shape_t* shape, const void* q, const 
     if (shape->stage_events && shape->num_stage_events < COMBA_BWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
     return backward_run(shape, L, workspace, q, k, v, alpha, beta, b, d, h0, dO, dhT, dq, dk, dv, dalpha, dbeta, db,
-                        dd, dh0, (shape->flags & COMBA_REUSE_FACTORS) != 0, static_cast<cudaStream_t>(stream));
+                        dd, dh0, (shape->flags & COMBA_REUSE_FACTORS) != 0, stream);
 }
 
 comba_status_t comba_chunk_fwd_gated(const comba_shape_t* shape, const void* q, const void* k, const void* v,
                                      const float* g_alpha, const float* g_beta, const float* a, const float* c,
                                      const float* b_raw, const float* d, const float* h0, void* o, float* hT,
-                                     void* workspace, size_t workspace_bytes, void* stream) {
+                                     void* workspace, size_t workspace_bytes, comba_stream_t stream) {
     Layout L;
     const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
     comba_status_t st = plan(shape, save ? 1 : 0, &L);
@@ -398,7 +398,7 @@ comba_status_t comba_chunk_fwd_gated(const comba_shape_t* shape, const void* q, 
     COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
     if (shape->stage_events && shape->num_stage_events < COMBA_FWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
-    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const cudaStream_t s = stream;
     const comba::GateParams g = gate_params(shape, L, workspace, q, k, g_alpha, g_beta, a, c, b_raw);
     if (comba::launch_gate_prologue(g, shape->dtype == COMBA_BF16, shape->dk, s) != cudaSuccess) return COMBA_ERR_CUDA;
     return forward_run(shape, L, workspace, g.qh, g.kh, v, g.alpha, g.beta, g.bgate, d, h0, o, hT, save, s);
@@ -409,7 +409,7 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t* shape, const void* q, 
                                      const float* b_raw, const float* d, const float* h0, const void* dO,
                                      const float* dhT, void* dq, void* dk, void* dv, float* dg_alpha, float* dg_beta,
                                      float* da, float* dc, float* db_raw, float* dd, float* dh0, void* workspace,
-                                     size_t workspace_bytes, void* stream) {
+                                     size_t workspace_bytes, comba_stream_t stream) {
     Layout L;
     comba_status_t st = plan(shape, 1, &L);
     if (st != COMBA_OK) return st;
@@ -422,7 +422,7 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t* shape, const void* q, 
     COMBA_OPTIONAL(h0); COMBA_OPTIONAL(dhT); COMBA_OPTIONAL(db_raw); COMBA_OPTIONAL(dh0);
     if (shape->stage_events && shape->num_stage_events < COMBA_BWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
-    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const cudaStream_t s = stream;
     const bool reuse = (shape->flags & COMBA_REUSE_FACTORS) != 0;
     const bool bf = shape->dtype == COMBA_BF16;
     comba::GateParams g = gate_params(shape, L, workspace, q, k, g_alpha, g_beta, a, c, b_raw);
@@ -466,7 +466,7 @@ static comba_status_t pk_prologue(const comba_shape_t* shape, const Layout& L, v
 comba_status_t comba_chunk_fwd_pk(const comba_shape_t* shape, const void* q, const void* k, const void* v,
                                   const void* p, const float* alpha, const float* beta, const float* b,
                                   const float* d, const float* h0, void* o, float* hT, void* workspace,
-                                  size_t workspace_bytes, void* stream) {
+                                  size_t workspace_bytes, comba_stream_t stream) {
     Layout L;
     const bool save = shape && (shape->flags & COMBA_SAVE_FACTORS);
     comba_status_t st = plan(shape, save ? 1 : 0, &L);
@@ -478,7 +478,7 @@ comba_status_t comba_chunk_fwd_pk(const comba_shape_t* shape, const void* q, con
     COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(hT);
     if (shape->stage_events && shape->num_stage_events < COMBA_FWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
-    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const cudaStream_t s = stream;
     void* qt;
     float* dz;
     if ((st = pk_prologue(shape, L, workspace, q, p, d, s, &qt, &dz)) != COMBA_OK) return st;
@@ -491,7 +491,7 @@ comba_status_t comba_chunk_bwd_pk(const comba_shape_t* shape, const void* q, con
                                   const void* p, const float* alpha, const float* beta, const float* b,
                                   const float* d, const float* h0, const void* dO, const float* dhT, void* dq,
                                   void* dk, void* dv, void* dp, float* dalpha, float* dbeta, float* db, float* dd,
-                                  float* dh0, void* workspace, size_t workspace_bytes, void* stream) {
+                                  float* dh0, void* workspace, size_t workspace_bytes, comba_stream_t stream) {
     Layout L;
     comba_status_t st = plan(shape, 1, &L);
     if (st != COMBA_OK) return st;
@@ -504,7 +504,7 @@ comba_status_t comba_chunk_bwd_pk(const comba_shape_t* shape, const void* q, con
     COMBA_OPTIONAL(b); COMBA_OPTIONAL(h0); COMBA_OPTIONAL(dhT); COMBA_OPTIONAL(db); COMBA_OPTIONAL(dh0);
     if (shape->stage_events && shape->num_stage_events < COMBA_BWD_EVENTS) return COMBA_ERR_INVALID_ARG;
     if (!workspace || !aligned16(workspace) || workspace_bytes < L.total) return COMBA_ERR_WORKSPACE;
-    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const cudaStream_t s = stream;
     void* qt;
     float* dz;
     if ((st = pk_prologue(shape, L, workspace, q, p, d, s, &qt, &dz, (shape->flags & COMBA_REUSE_FACTORS) != 0)) !=
@@ -519,7 +519,7 @@ comba_status_t comba_chunk_bwd_pk(const comba_shape_t* shape, const void* q, con
 comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtype_t dtype, const void* q,
                                        const void* k, const void* v, const void* p, const float* alpha,
                                        const float* beta, const float* b, const float* d, float* state, void* o,
-                                       int flags, void* stream) {
+                                       int flags, comba_stream_t stream) {
     if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
     if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
     if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
@@ -529,7 +529,7 @@ comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtyp
     COMBA_REQUIRE(beta); COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
     COMBA_OPTIONAL(b);
     if (comba::launch_recurrent_step(Bd, H, dk, dv, dtype == COMBA_BF16, q, k, v, p, alpha, beta, b, d, state, o,
-                                     (flags & COMBA_IPLR) != 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+                                     (flags & COMBA_IPLR) != 0, stream) != cudaSuccess)
         return COMBA_ERR_CUDA;
     return COMBA_OK;
 }
@@ -537,7 +537,7 @@ comba_status_t comba_recurrent_step_pk(int Bd, int H, int dk, int dv, comba_dtyp
 comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t dtype, const void* q,
                                     const void* k, const void* v, const float* alpha, const float* beta,
                                     const float* b, const float* d, float* state, void* o, int flags,
-                                    void* stream) {
+                                    comba_stream_t stream) {
     if (Bd < 1 || H < 1) return COMBA_ERR_INVALID_ARG;
     if (flags & ~COMBA_IPLR) return COMBA_ERR_INVALID_ARG;
     if (dtype != COMBA_F32 && dtype != COMBA_BF16) return COMBA_ERR_INVALID_ARG;
@@ -547,7 +547,7 @@ comba_status_t comba_recurrent_step(int Bd, int H, int dk, int dv, comba_dtype_t
     COMBA_REQUIRE(d); COMBA_REQUIRE(state); COMBA_REQUIRE(o);
     COMBA_OPTIONAL(b);
     if (comba::launch_recurrent_step(Bd, H, dk, dv, dtype == COMBA_BF16, q, k, v, nullptr, alpha, beta, b, d, state,
-                                     o, (flags & COMBA_IPLR) != 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+                                     o, (flags & COMBA_IPLR) != 0, stream) != cudaSuccess)
         return COMBA_ERR_CUDA;
     return COMBA_OK;
 }

@@ -37,25 +37,32 @@ struct PrepTcSmem {
     static constexpr uint32_t OV = OK + 32768;           // V  [64][128]               16 KB
     static constexpr uint32_t OMW = OV + 16384;          // Mw [64][64] K-major         8 KB
     static constexpr uint32_t OMU = OMW + 8192;          // Mu [64][64]                 8 KB
-    static constexpr uint32_t OR = OMU + 8192;           // A^T (pitch 68), M (pitch 65), T fp32, then sW^T, sU^T [128][64]
+    static constexpr uint32_t OR = OMU + 8192;           // A^T (pitch 68), M (pitch 65), T fp32, then sW^T, sU_s^T [128][64],
+                                                         // then the Atilde staging [128][128]
     static constexpr uint32_t R_BYTES = (64 * 68 + 64 * 65 + 32 * 36) * 4;
     static constexpr uint32_t OF = OR + ((R_BYTES + 1023) & ~1023u);
     static constexpr size_t bytes() { return 1024 + OF + 64 * 6 * 4; }
 };
 
-// Tensor maps of the prep kernel's loads: token tiles {64 columns, 1 head, 64 tokens} of k and p
-// (key heads) and v (value heads), 128-byte swizzled.
+// Tensor maps of the prep kernel's traffic, 128-byte swizzled: token tiles {64 columns, 1 head,
+// 64 tokens} of k and p (key heads) and v (value heads) in; the workspace tiles W^T, U^T, U_s^T
+// ([pairs * 128][64], one 128-row box) and Atilde ([pairs * 128][128], two 128-row boxes of 64
+// columns) out by bulk tensor stores.
 struct PrepMaps {
     CUtensorMap k, p, v;
+    CUtensorMap w, u, us, a;
 };
 
 // 256 threads: warps w and w + 4 read the same TMEM lane quadrant and split its columns.
 // Persistent: two CTAs per SM, CTA b taking units b, b + G, ... (G = gridDim.x).  A unit's gates
 // are requested at the previous unit's start and its K (or [P; K]) and V tiles by TMA as soon as
 // the previous unit's Atilde product has read K (Atilde is staged in the dead W^T / U_s^T region),
-// so that loads overlap the previous unit's last epilogue and copies.
+// so that loads overlap the previous unit's last epilogue and copies.  W^T, U^T, U_s^T and Atilde
+// leave by bulk tensor stores (thread 32) from swizzled staging tiles; each staging tile is
+// reused only once those stores have read it.
 __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pairs, const __grid_constant__ PrepMaps mp) {
     constexpr int NTH = 256;
+    constexpr int kStore = 32;   // issues the bulk tensor stores and waits for them
     using S = PrepTcSmem;
     extern __shared__ uint8_t smem_raw[];
     // stall_bar: nothing arrives (COMBA_DIAG_STALL); ld: a unit's tiles (one phase per unit)
@@ -172,6 +179,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
                 *reinterpret_cast<uint4*>(sV + sw128_offset(r, 8 * ch, 64)) = z;
             }
         }
+        if (tid == kStore) bulk_wait_all_reads();   // the previous unit's Atilde store has read A^T's region
         fence_async_smem();
         tc_fence_before();
         ok = !__syncthreads_or(!okl);
@@ -236,7 +244,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
             tc_gemm<true, false>(tmem + 128, smem_u32(sV), 64, smem_u32(sMu), 64, 64, 64, false);
         }
         ok = ok && ms.finish_warp(tid);   // (ok is block-uniform here: every thread takes the same branch)
-        // W^T and U^T for the workspace are staged over the dead V and Mw/Mu tiles.
+        // W^T and U^T for the workspace are staged (swizzled) over the dead V and Mw/Mu tiles.
         uint8_t* stW = sV;
         uint8_t* stU = sMw;
         if (ok) {
@@ -251,7 +259,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
                         v[e] = d[8 * q + e];
                         w[e] = v[e] * sS[32 * g + 8 * q + e];
                     }
-                    stage_chunk<8>(stW, row, 4 * g + q, pack8(v));
+                    *reinterpret_cast<uint4*>(stW + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
                     *reinterpret_cast<uint4*>(sWt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
                 }
             }
@@ -265,7 +273,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
                         v[e] = d[8 * q + e];
                         w[e] = v[e] * sS[32 * g + 8 * q + e];
                     }
-                    stage_chunk<8>(stU, row, 4 * g + q, pack8(v));
+                    *reinterpret_cast<uint4*>(stU + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
                     *reinterpret_cast<uint4*>(sUt + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(w);
                 }
             }
@@ -274,13 +282,15 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
 
         // Atilde = -K^T (Diag(s) W) -> cols [0,128)
         if (ok && tid == 0) tc_gemm<true, false>(tmem, smem_u32(sKk), 128, smem_u32(sWt), 128, 128, 64, false);
-        if (ok) {
-            // W^T, U^T and U_s^T (un-swizzled row by row) out while the tensor core works
-            copy_staged<8>((bf16*)p.Wb + idx * D * 64, stW, tid, NTH);
-            copy_staged<8>((bf16*)p.Ub + idx * D * 64, stU, tid, NTH);
-            uint4* us = reinterpret_cast<uint4*>((bf16*)p.Usb + idx * D * 64);
-            for (int e = tid; e < 128 * 8; e += NTH)
-                us[e] = *reinterpret_cast<const uint4*>(sUt + sw128_offset(e >> 3, 8 * (e & 7), 128));
+        if (ok && tid == kStore) {
+            // W^T, U^T and U_s^T out while the tensor core works; their staging is reused only once
+            // the stores have read it
+            const int y = (int)((uint32_t)u * (uint32_t)D);
+            tma_store_2d(&mp.w, 0, y, smem_u32(stW));
+            tma_store_2d(&mp.u, 0, y, smem_u32(stU));
+            tma_store_2d(&mp.us, 0, y, smem_u32(sUt));
+            bulk_commit();
+            bulk_wait_all_reads();
         }
         ok = ok && ms.finish_warp(tid);
         // K, V and the W^T / U^T / U_s^T staging are dead now, for every thread: the next unit's
@@ -300,14 +310,20 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
                 for (int q = 0; q < 4; ++q) {
 #pragma unroll
                     for (int e = 0; e < 8; ++e) v[e] = -d[8 * q + e];
-                    stage_chunk<16>(stA, row, 4 * g + q, pack8(v));
+                    *reinterpret_cast<uint4*>(stA + sw128_offset(row, 32 * g + 8 * q, 128)) = pack8(v);
                 }
             }
         }
+        fence_async_smem();
         tc_fence_before();   // the unit's last TMEM reads: the next unit's Gram may follow
         __syncthreads();
         tc_fence_after();
-        copy_staged<16>((bf16*)p.Ab + idx * D * D, stA, tid, NTH);
+        if (tid == kStore) {   // Atilde out; the next unit's A^T (over the staging) waits for the read
+            const int y = (int)((uint32_t)u * (uint32_t)D);
+            tma_store_2d(&mp.a, 0, y, smem_u32(stA));
+            tma_store_2d(&mp.a, 64, y, smem_u32(stA) + 16384);
+            bulk_commit();
+        }
         ph ^= 1;
     }
     if (!ok) {
@@ -317,6 +333,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
         }
         ms.drain(tid);
     }
+    if (tid == kStore) bulk_wait_all_done();   // and every bulk store has completed
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -641,7 +658,11 @@ cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s) {
     if ((e = cudaGetDevice(&dev)) || (e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev))) return e;
     tc::PrepMaps mp;
     bool good = make_bf16_token_map(&mp.k, p.k, p.Ttot, p.H / p.vg, tc::D) &&
-                make_bf16_token_map(&mp.v, p.v, p.Ttot, p.H, tc::D);
+                make_bf16_token_map(&mp.v, p.v, p.Ttot, p.H, tc::D) && p.Wb && p.Ub && p.Usb && p.Ab &&
+                make_bf16_map(&mp.w, p.Wb, pairs * tc::D, 64, tc::D) &&
+                make_bf16_map(&mp.u, p.Ub, pairs * tc::D, 64, tc::D) &&
+                make_bf16_map(&mp.us, p.Usb, pairs * tc::D, 64, tc::D) &&
+                make_bf16_map(&mp.a, p.Ab, pairs * tc::D, tc::D, tc::D);
     if (good && p.p) good = make_bf16_token_map(&mp.p, p.p, p.Ttot, p.H / p.vg, tc::D);
     else mp.p = mp.k;   // not used
     if (!good) return cudaErrorInvalidValue;

@@ -577,11 +577,34 @@ __device__ __forceinline__ void unit_lower_inverse_diag16(const float* At, float
     }
 }
 
+// fp32 -> tf32 (round to nearest, ties away) for the tf32 tile products below.
+__device__ __forceinline__ uint32_t to_tf32(float x) {
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;\n" : "=r"(r) : "f"(x));
+    return r;
+}
+// d += a b on one m16n8k8 tile, tf32 operands and fp32 accumulators.  Fragments (g = lane / 4,
+// q = lane % 4): a = A[g][q], A[g + 8][q], A[g][q + 4], A[g + 8][q + 4]; b = B[q][g], B[q + 4][g];
+// d = D[g][2 q], D[g][2 q + 1], D[g + 8][2 q], D[g + 8][2 q + 1].
+__device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
 // (I + A)^{-1} for a strictly lower 64 x 64 A over 256 threads, in three levels: the four
-// 16 x 16 diagonal blocks (warps 0..3, one block each, a column per lane), then the 32 x 32 blocks
-// M10 = -M11 (A10 M00) of both halves, then the 64 x 64 M21 = -M22 (A21 M11).  At is A
-// transposed with pitch 68; M has pitch `pm` and is written in full (zeros above the
-// diagonal); T holds 32 x 36 floats of scratch.
+// 16 x 16 diagonal blocks by forward substitution (warps 0..3, one block each, a column per
+// lane, fp32), then the 32 x 32 blocks M10 = -M11 (A10 M00) of both halves, then the 64 x 64
+// M21 = -M22 (A21 M11).  The two off-diagonal levels are tile products on the tensor cores
+// (mma.sync m16n8k8, tf32 operands rounded to nearest, fp32 accumulation): four warps, each
+// owning an 8-column block of the level's result, form its block of the inner product, pass it
+// from the accumulator layout to the operand layout through a warp-private scratch tile and
+// finish the outer product, so each level ends at a single block-wide barrier.  The tf32
+// operand rounding (relative 2^-11) lies well below that of the bf16 copies every consumer of M
+// takes (2^-8).  At is A transposed with pitch 68; M has pitch `pm` and is written in full
+// (zeros above the diagonal); T holds 1024 floats of scratch.
 __device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float* M, int pm, float* T, int tid) {
     if (tid < 128) {
         // warp b solves diagonal block b (lanes 0..15, one column each): no divergence between blocks
@@ -602,66 +625,78 @@ __device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float*
         }
     }
     __syncthreads();
-    // level 1, both halves h (block rows 2h+1, block columns 2h): thread -> (h, r, c pair)
-    const int h1 = tid >> 7, r1 = (tid >> 3) & 15, c1 = 2 * (tid & 7);
-    const int o1 = 32 * h1;
-    {
-        // T1 = A10 M00: T1[r][c] = sum_k A[o1 + 16 + r][o1 + k] M[o1 + k][o1 + c]
-        float t0 = 0.f, t1 = 0.f;
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-            const float a = At[(o1 + k) * 68 + o1 + 16 + r1];
-            t0 = fmaf(a, M[(o1 + k) * pm + o1 + c1], t0);
-            t1 = fmaf(a, M[(o1 + k) * pm + o1 + c1 + 1], t1);
+    const int warp = tid >> 5, g = (tid >> 2) & 7, q = tid & 3;
+    if (warp < 4) {
+        // level 1: half h (rows and columns o1 .. o1 + 31), column block nt of M10 (8 columns)
+        const int o1 = 32 * (warp >> 1), nt = warp & 1, c0 = o1 + 8 * nt;
+        float* Tw = T + warp * 128;   // [16][8]: T1's column block
+        float d[4] = {0.f, 0.f, 0.f, 0.f};
+        // T1 = A10 M00; M00 is lower, so its rows above the block's first column are zero
+        for (int ks = nt; ks < 2; ++ks) {
+            const int k = o1 + 8 * ks + q;
+            const uint32_t a[4] = {to_tf32(At[k * 68 + o1 + 16 + g]), to_tf32(At[k * 68 + o1 + 24 + g]),
+                                   to_tf32(At[(k + 4) * 68 + o1 + 16 + g]), to_tf32(At[(k + 4) * 68 + o1 + 24 + g])};
+            mma_tf32(d, a, to_tf32(M[k * pm + c0 + g]), to_tf32(M[(k + 4) * pm + c0 + g]));
         }
-        *reinterpret_cast<float2*>(T + h1 * 16 * 18 + r1 * 18 + c1) = make_float2(t0, t1);
+        *reinterpret_cast<float2*>(Tw + g * 8 + 2 * q) = make_float2(d[0], d[1]);
+        *reinterpret_cast<float2*>(Tw + (g + 8) * 8 + 2 * q) = make_float2(d[2], d[3]);
+        __syncwarp();
+        // M10 = -M11 T1
+        float e[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int ks = 0; ks < 2; ++ks) {
+            const int k = o1 + 16 + 8 * ks + q;
+            const uint32_t a[4] = {to_tf32(M[(o1 + 16 + g) * pm + k]), to_tf32(M[(o1 + 24 + g) * pm + k]),
+                                   to_tf32(M[(o1 + 16 + g) * pm + k + 4]), to_tf32(M[(o1 + 24 + g) * pm + k + 4])};
+            mma_tf32(e, a, to_tf32(Tw[(8 * ks + q) * 8 + g]), to_tf32(Tw[(8 * ks + q + 4) * 8 + g]));
+        }
+        const int c = c0 + 2 * q;
+        M[(o1 + 16 + g) * pm + c] = -e[0];
+        M[(o1 + 16 + g) * pm + c + 1] = -e[1];
+        M[(o1 + 24 + g) * pm + c] = -e[2];
+        M[(o1 + 24 + g) * pm + c + 1] = -e[3];
     }
     __syncthreads();
-    {
-        // M10 = -M11 T1: M[o1 + 16 + r][o1 + c] = -sum_k M[o1 + 16 + r][o1 + 16 + k] T1[k][c]
-        float t0 = 0.f, t1 = 0.f;
+    if (warp < 4) {
+        // level 2: column block nt of M21 (rows 32..63, columns 8 nt .. + 7), both 16-row tiles
+        const int nt = warp;
+        float* Tw = T + warp * 256;   // [32][8]: T's column block
+        float d[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+        // T = A21 M11; M11 (the top-left 32 x 32 inverse) is lower: rows k < 8 nt of the block are zero
+        for (int ks = nt; ks < 4; ++ks) {
+            const int k = 8 * ks + q;
+            const uint32_t b0 = to_tf32(M[k * pm + 8 * nt + g]), b1 = to_tf32(M[(k + 4) * pm + 8 * nt + g]);
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-            const float m = M[(o1 + 16 + r1) * pm + o1 + 16 + k];
-            const float2 b = *reinterpret_cast<const float2*>(T + h1 * 16 * 18 + k * 18 + c1);
-            t0 = fmaf(m, b.x, t0);
-            t1 = fmaf(m, b.y, t1);
-        }
-        M[(o1 + 16 + r1) * pm + o1 + c1] = -t0;
-        M[(o1 + 16 + r1) * pm + o1 + c1 + 1] = -t1;
-    }
-    __syncthreads();
-    // level 2: M21 = -M22 (A21 M11) over the 32 x 32 blocks, 2 x 2 outputs per thread
-    const int r0 = 2 * (tid >> 4), c0 = 2 * (tid & 15);
-    {
-        float t[2][2] = {};
-#pragma unroll 8
-        for (int k = 0; k < 32; ++k) {
-            const float2 a2 = *reinterpret_cast<const float2*>(At + k * 68 + 32 + r0);
-            const float m0 = M[k * pm + c0], m1 = M[k * pm + c0 + 1];
-            t[0][0] = fmaf(a2.x, m0, t[0][0]); t[0][1] = fmaf(a2.x, m1, t[0][1]);
-            t[1][0] = fmaf(a2.y, m0, t[1][0]); t[1][1] = fmaf(a2.y, m1, t[1][1]);
-        }
-        *reinterpret_cast<float2*>(T + r0 * 36 + c0) = make_float2(t[0][0], t[0][1]);
-        *reinterpret_cast<float2*>(T + (r0 + 1) * 36 + c0) = make_float2(t[1][0], t[1][1]);
-    }
-    __syncthreads();
-    {
-        float t[2][2] = {};
-#pragma unroll 8
-        for (int k = 0; k < 32; ++k) {
-            const float2 b = *reinterpret_cast<const float2*>(T + k * 36 + c0);
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const float m = M[(32 + r0 + e) * pm + 32 + k];
-                t[e][0] = fmaf(m, b.x, t[e][0]);
-                t[e][1] = fmaf(m, b.y, t[e][1]);
+            for (int mt = 0; mt < 2; ++mt) {
+                const int r = 32 + 16 * mt + g;
+                const uint32_t a[4] = {to_tf32(At[k * 68 + r]), to_tf32(At[k * 68 + r + 8]),
+                                       to_tf32(At[(k + 4) * 68 + r]), to_tf32(At[(k + 4) * 68 + r + 8])};
+                mma_tf32(d[mt], a, b0, b1);
             }
         }
 #pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            M[(32 + r0 + e) * pm + c0] = -t[e][0];
-            M[(32 + r0 + e) * pm + c0 + 1] = -t[e][1];
+        for (int mt = 0; mt < 2; ++mt) {
+            *reinterpret_cast<float2*>(Tw + (16 * mt + g) * 8 + 2 * q) = make_float2(d[mt][0], d[mt][1]);
+            *reinterpret_cast<float2*>(Tw + (16 * mt + g + 8) * 8 + 2 * q) = make_float2(d[mt][2], d[mt][3]);
+        }
+        __syncwarp();
+        // M21 = -M22 T; M22 is lower: rows 16 mt .. + 15 of it reach column 16 mt + 15 at most
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+            float e[4] = {0.f, 0.f, 0.f, 0.f};
+            const int r = 32 + 16 * mt + g;
+#pragma unroll
+            for (int ks = 0; ks < 2 + 2 * mt; ++ks) {
+                const int k = 32 + 8 * ks + q;
+                const uint32_t a[4] = {to_tf32(M[r * pm + k]), to_tf32(M[(r + 8) * pm + k]),
+                                       to_tf32(M[r * pm + k + 4]), to_tf32(M[(r + 8) * pm + k + 4])};
+                mma_tf32(e, a, to_tf32(Tw[(8 * ks + q) * 8 + g]), to_tf32(Tw[(8 * ks + q + 4) * 8 + g]));
+            }
+            const int c = 8 * nt + 2 * q;
+            M[r * pm + c] = -e[0];
+            M[r * pm + c + 1] = -e[1];
+            M[(r + 8) * pm + c] = -e[2];
+            M[(r + 8) * pm + c + 1] = -e[3];
         }
     }
 }

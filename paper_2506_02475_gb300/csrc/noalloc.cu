@@ -45,7 +45,7 @@ cudaError_t static_scratch_address(void** out) {
 extern "C" comba_status_t comba_chunk_fwd_noalloc(const comba_shape_t* shape, const void* q, const void* k,
                                                   const void* v, const float* alpha, const float* beta,
                                                   const float* b, const float* d, const float* h0, void* o,
-                                                  float* hT, void* stream) {
+                                                  float* hT, comba_stream_t stream) {
     // Only the plain and iplr forms run here: saved factors would land in the shared array where no
     // caller can reach them, and the gated and pk forms have entry points of their own.
     if (shape && (shape->flags & ~COMBA_IPLR)) return COMBA_ERR_INVALID_ARG;

@@ -108,28 +108,12 @@ __device__ __forceinline__ void publish_smem() {
     tc_fence_after();
 }
 
-// Row-per-thread staging of a [128][8 NCH] bf16 tile whose 16-byte chunks are
-// rotated by row (chunk c of row r at slot (c + r) mod NCH), so the 32 lanes of a
-// warp writing one chunk of 32 consecutive rows hit distinct banks; then a
-// coalesced copy of the tile to contiguous global memory by all 128 threads.
-template <int NCH>
-__device__ __forceinline__ void stage_chunk(uint8_t* st, int row, int c, uint4 v) {
-    *reinterpret_cast<uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16) = v;
-}
-template <int NCH>
-__device__ __forceinline__ void copy_staged(bf16* g, const uint8_t* st, int tid, int nthr = 128) {
-    for (int e = tid; e < 128 * NCH; e += nthr) {
-        const int row = e / NCH, c = e % NCH;
-        reinterpret_cast<uint4*>(g)[e] = *reinterpret_cast<const uint4*>(st + row * NCH * 16 + ((c + row) % NCH) * 16);
-    }
-}
-
-
 __device__ __forceinline__ void bulk_copy_s2g(void* g, uint32_t s, uint32_t bytes) {
     asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n" ::"l"(g), "r"(s), "r"(bytes) : "memory");
     asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
 }
 __device__ __forceinline__ void bulk_wait_all_reads() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all_done() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
 // Bulk tensor stores of a swizzled shared tile (2D: columns x, rows y; 3D: columns x, head y,
 // tokens z), completed as one bulk group by bulk_commit.
 __device__ __forceinline__ void tma_store_2d(const void* tmap, int x, int y, uint32_t src) {

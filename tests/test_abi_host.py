@@ -275,3 +275,30 @@ def test_diagnostic_stall_flag_is_accepted_only_by_the_plain_chunk_calls(L):
     fn = L.comba_chunk_fwd_noalloc
     s = shape(flags=32)
     assert fn(ctypes.byref(s), *([FAKE] * 7), None, FAKE, None, None) == INVALID
+
+
+def test_header_compiles_as_c_and_takes_a_cuda_stream(tmp_path):
+    """include/comba.h is plain C (C99, no CUDA include), and in C++ next to the CUDA runtime's
+    header a cudaStream_t passes as the entry points' stream argument without a cast."""
+    import shutil
+    import subprocess
+    inc = os.path.dirname(HEADER)
+    gcc, gxx = shutil.which("gcc"), shutil.which("g++")
+    if not gcc or not gxx:
+        pytest.skip("no host compiler")
+    c_src = tmp_path / "t.c"
+    c_src.write_text('#include "comba.h"\nint main(void) { comba_stream_t s = 0; (void)s; return 0; }\n')
+    r = subprocess.run([gcc, "-std=c99", "-Wall", "-Werror", "-I" + inc, "-c", str(c_src), "-o",
+                        str(tmp_path / "t.o")], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    cuda_inc = next((d for d in ("/usr/local/cuda/include",) if os.path.exists(os.path.join(d, "cuda_runtime_api.h"))),
+                    None)
+    if cuda_inc is None:
+        pytest.skip("no CUDA runtime header")
+    cc_src = tmp_path / "t.cc"
+    cc_src.write_text('#include <cuda_runtime_api.h>\n#include "comba.h"\n'
+                      'comba_status_t f(const comba_shape_t* s, cudaStream_t st) {\n'
+                      '  return comba_chunk_fwd(s, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, st);\n}\n')
+    r = subprocess.run([gxx, "-std=c++17", "-Wall", "-Werror", "-I" + inc, "-I" + cuda_inc, "-c", str(cc_src), "-o",
+                        str(tmp_path / "t2.o")], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
