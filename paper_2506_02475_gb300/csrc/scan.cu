@@ -409,6 +409,29 @@ __global__ void __launch_bounds__(256, 1)
         const int L = (int)(len - (long long)c * kChunk < kChunk ? len - (long long)c * kChunk : kChunk);
         return __ldg(a.Gb + unit_of(it) * 64 + L - 1);
     };
+    // A give-up (a wait that ran out, or thread 0's missing F / T) reaches the whole block at the
+    // next chunk's barrier, which every warp passes before thread 0 issues another product: each
+    // warp waits for the products on its own and reads its accumulator rows without a block-wide
+    // barrier in between.  `wbad` is uniform over the warp.
+    auto give_up = [&](int it) {   // the block's failure, seen at chunk it's barrier (it <= nch)
+        if (tid == kTma) {
+            if (a.err) atomicExch(a.err, 1);
+            // chunk it - 1's loads may still be in flight when its waits ran out; later stages were
+            // not re-armed yet
+            for (int c = it > 0 ? it - 1 : 0; c < nx; ++c) mbar_drain(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
+            for (int c = it > 0 ? it - 1 : 0; c < nf; ++c) mbar_drain(smem_u32(&full_f[c % S::SF]), (c / S::SF) & 1);
+        }
+        if (tid == 0 && it > 0) {
+            // chunk it - 1's products (phase (it - 1) & 1, which may still be pending: a parity wait
+            // is only exact on the pending phase), then one more commit for an additive term issued
+            // after them
+            mbar_drain(smem_u32(&mma_bar), (it - 1) & 1);
+            tc_commit(smem_u32(&mma_bar));
+            mbar_drain(smem_u32(&mma_bar), it & 1);
+        }
+    };
+    int wbad = 0;
+    bool gave_up = false;
     float g_next = nch > 0 ? log_decay(0) : 0.f;
     for (int it = 0; it < nch; ++it) {
         const float gam = expf(g_next);
@@ -422,9 +445,16 @@ __global__ void __launch_bounds__(256, 1)
             for (int hh = 0; hh < 2; ++hh)
                 *reinterpret_cast<__nv_bfloat162*>(sA + sw128_offset(r0 + 8 * hh, cq + 8 * t, 64)) =
                     __floats2bfloat162_rn(st[t][2 * hh], st[t][2 * hh + 1]);
+        // the previous chunk's state store (issued a step ago) has read its buffer, which the next
+        // chunk's state overwrites once this barrier is passed
+        if (tid == kTma) bulk_wait_read<0>();
         fence_async_smem();
         tc_fence_before();
-        __syncthreads();
+        if (__syncthreads_or(wbad)) {
+            give_up(it);
+            gave_up = true;
+            break;
+        }
         tc_fence_after();
 
         int bad = ybad;
@@ -450,23 +480,7 @@ __global__ void __launch_bounds__(256, 1)
             if (nf < nch) issue_f(nf++);
         }
         if (!mbar_wait(smem_u32(&mma_bar), it & 1, a.wait_ns)) bad = 1;
-        if (tid == kTma) bulk_wait_read<1>();
-        if (__syncthreads_or(bad)) {
-            if (tid == kTma) {
-                if (a.err) atomicExch(a.err, 1);
-                for (int c = it; c < nx; ++c) mbar_drain(smem_u32(&full_x[c % S::SX]), (c / S::SX) & 1);
-                for (int c = it; c < nf; ++c) mbar_drain(smem_u32(&full_f[c % S::SF]), (c / S::SF) & 1);
-            }
-            if (tid == 0) {
-                // the products must finish before TMEM is released: chunk it's (phase it, which may
-                // still be pending: a parity wait is only exact on the pending phase), then one more
-                // commit for the additive term issued after it
-                mbar_drain(smem_u32(&mma_bar), it & 1);
-                tc_commit(smem_u32(&mma_bar));
-                mbar_drain(smem_u32(&mma_bar), (it + 1) & 1);
-            }
-            break;
-        }
+        wbad = __any_sync(0xffffffffu, bad);
         tc_fence_after();
 
         // S^T <- gamma S^T + (Y + S^T X^T)  on this thread's 32 values
@@ -499,6 +513,8 @@ __global__ void __launch_bounds__(256, 1)
         }
     }
 
+    // the last chunk's waits, unless the loop has given up already
+    if (__syncthreads_or(wbad) && !gave_up) give_up(nch);
     if (tid == kTma) bulk_wait_all();
     __syncthreads();
     tc_fence_after();
