@@ -37,9 +37,9 @@ struct PrepTcSmem {
     static constexpr uint32_t OV = OK + 32768;           // V  [64][128]               16 KB
     static constexpr uint32_t OMW = OV + 16384;          // Mw [64][64] K-major         8 KB
     static constexpr uint32_t OMU = OMW + 8192;          // Mu [64][64]                 8 KB
-    static constexpr uint32_t OR = OMU + 8192;           // A^T (pitch 68), M (pitch 65), T fp32, then sW^T, sU_s^T [128][64],
+    static constexpr uint32_t OR = OMU + 8192;           // A^T, M (pitches kAtPitch, kMPitch), T fp32, then sW^T, sU_s^T [128][64],
                                                          // then the Atilde staging [128][128]
-    static constexpr uint32_t R_BYTES = (64 * 68 + 64 * 65 + 32 * 36) * 4;
+    static constexpr uint32_t R_BYTES = (64 * kAtPitch + 64 * kMPitch + 1024) * 4;
     static constexpr uint32_t OF = OR + ((R_BYTES + 1023) & ~1023u);
     static constexpr size_t bytes() { return 1024 + OF + 64 * 6 * 4; }
 };
@@ -74,9 +74,9 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
     uint8_t* sV = sm + S::OV;
     uint8_t* sMw = sm + S::OMW;
     uint8_t* sMu = sm + S::OMU;
-    float* sAt = reinterpret_cast<float*>(sm + S::OR);   // A transposed, pitch 68
-    float* sM = sAt + 64 * 68;
-    float* sTi = sM + 64 * 65;                         // inverse scratch, 32 x 36
+    float* sAt = reinterpret_cast<float*>(sm + S::OR);   // A transposed
+    float* sM = sAt + 64 * kAtPitch;
+    float* sTi = sM + 64 * kMPitch;                    // inverse scratch, 1024 floats
     uint8_t* sWt = sm + S::OR;            // aliases A after the inverse
     uint8_t* sUt = sm + S::OR + 16384;    // aliases M after Mw/Mu are built
     uint8_t* stA = sm + S::OR;            // Atilde staging [128][128], once W^T / U_s^T are dead
@@ -200,7 +200,7 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
                 const int i = i0 + c;
-                sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+                sAt[i * kAtPitch + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
             }
         } else if (ok && row < 64) {
             // Comba-pk: P K^T rows are in lanes 0..63 only; the two threads of each take one column half.
@@ -211,22 +211,23 @@ __global__ void __launch_bounds__(256, 2) k_prep_tc(ChunkParams p, long long pai
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
                 const int i = i0 + c;
-                sAt[i * 68 + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
+                sAt[i * kAtPitch + r] = i < r ? br * __expf(gr - sG[i]) * d[c] : 0.f;
             }
         }
         ok = !__syncthreads_or(!ok);   // the inverse's barriers below need a block-uniform flag
         if (ok) {
-            unit_lower_inverse64_h16(sAt, sM, 65, sTi, tid);
+            unit_lower_inverse64_h16(sAt, sM, sTi, tid);
             __syncthreads();
             // Mw = M Diag(btilde gamma_{r-1}), Mu = M Diag(beta) as K-major [p][p'] tiles; M saved for the backward.
             bf16* Mg = p.Mb ? (bf16*)p.Mb + idx * 4096 : nullptr;
             for (int e = tid; e < 64 * 8; e += NTH) {
                 const int r = e >> 3, ch = e & 7;
                 float mw[8], mu[8], mm[8];
+                *reinterpret_cast<float4*>(mm) = *reinterpret_cast<const float4*>(sM + r * kMPitch + 8 * ch);
+                *reinterpret_cast<float4*>(mm + 4) = *reinterpret_cast<const float4*>(sM + r * kMPitch + 8 * ch + 4);
 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
                     const int c = 8 * ch + q;
-                    mm[q] = sM[r * 65 + c];
                     mw[q] = mm[q] * sWs[c];
                     mu[q] = mm[q] * sBe[c];
                 }

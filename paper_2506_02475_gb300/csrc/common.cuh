@@ -554,9 +554,15 @@ __device__ __forceinline__ void unit_lower_inverse64(const float* A, float* M, f
     }
 }
 
+// Row pitches (floats) of the tcgen05 prep kernel's inverse: A transposed (At) and M.  At's
+// pitch is 8 (mod 32) and M's 4 (mod 32), so the tf32 fragment loads below (lanes g = 0..7 along
+// one index, q = 0..3 along the other) fall in distinct banks: At and M as A operands, M as a B
+// operand in two lanes per bank at most.
+constexpr int kAtPitch = 72, kMPitch = 68;
+
 // Column j (of 16) of (I + A_bb)^{-1} for the 16 x 16 diagonal block starting at B0, by
 // forward substitution in registers: M[r2][j] = delta - sum_{r < r2} A[r2][r] M[r][j].
-// At is A transposed (pitch 68): its row r holds column r of A, zero at and above r.
+// At is A transposed (pitch kAtPitch): its row r holds column r of A, zero at and above r.
 template <int B0>
 __device__ __forceinline__ void unit_lower_inverse_diag16(const float* At, float* M, int pm, int j) {
     float s[16];
@@ -568,7 +574,7 @@ __device__ __forceinline__ void unit_lower_inverse_diag16(const float* At, float
         M[(B0 + r) * pm + B0 + j] = x;
 #pragma unroll
         for (int g = (r + 1) >> 2; g < 4; ++g) {
-            const float4 a = *reinterpret_cast<const float4*>(At + (B0 + r) * 68 + B0 + 4 * g);
+            const float4 a = *reinterpret_cast<const float4*>(At + (B0 + r) * kAtPitch + B0 + 4 * g);
             s[4 * g + 0] = fmaf(a.x, x, s[4 * g + 0]);
             s[4 * g + 1] = fmaf(a.y, x, s[4 * g + 1]);
             s[4 * g + 2] = fmaf(a.z, x, s[4 * g + 2]);
@@ -603,9 +609,10 @@ __device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], 
 // from the accumulator layout to the operand layout through a warp-private scratch tile and
 // finish the outer product, so each level ends at a single block-wide barrier.  The tf32
 // operand rounding (relative 2^-11) lies well below that of the bf16 copies every consumer of M
-// takes (2^-8).  At is A transposed with pitch 68; M has pitch `pm` and is written in full
-// (zeros above the diagonal); T holds 1024 floats of scratch.
-__device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float* M, int pm, float* T, int tid) {
+// takes (2^-8).  At is A transposed with pitch kAtPitch; M has pitch kMPitch and is written in
+// full (zeros above the diagonal); T holds 1024 floats of scratch.
+__device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float* M, float* T, int tid) {
+    constexpr int pm = kMPitch, pa = kAtPitch;
     if (tid < 128) {
         // warp b solves diagonal block b (lanes 0..15, one column each): no divergence between blocks
         const int j = tid & 31;
@@ -634,8 +641,8 @@ __device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float*
         // T1 = A10 M00; M00 is lower, so its rows above the block's first column are zero
         for (int ks = nt; ks < 2; ++ks) {
             const int k = o1 + 8 * ks + q;
-            const uint32_t a[4] = {to_tf32(At[k * 68 + o1 + 16 + g]), to_tf32(At[k * 68 + o1 + 24 + g]),
-                                   to_tf32(At[(k + 4) * 68 + o1 + 16 + g]), to_tf32(At[(k + 4) * 68 + o1 + 24 + g])};
+            const uint32_t a[4] = {to_tf32(At[k * pa + o1 + 16 + g]), to_tf32(At[k * pa + o1 + 24 + g]),
+                                   to_tf32(At[(k + 4) * pa + o1 + 16 + g]), to_tf32(At[(k + 4) * pa + o1 + 24 + g])};
             mma_tf32(d, a, to_tf32(M[k * pm + c0 + g]), to_tf32(M[(k + 4) * pm + c0 + g]));
         }
         *reinterpret_cast<float2*>(Tw + g * 8 + 2 * q) = make_float2(d[0], d[1]);
@@ -669,8 +676,8 @@ __device__ __forceinline__ void unit_lower_inverse64_h16(const float* At, float*
 #pragma unroll
             for (int mt = 0; mt < 2; ++mt) {
                 const int r = 32 + 16 * mt + g;
-                const uint32_t a[4] = {to_tf32(At[k * 68 + r]), to_tf32(At[k * 68 + r + 8]),
-                                       to_tf32(At[(k + 4) * 68 + r]), to_tf32(At[(k + 4) * 68 + r + 8])};
+                const uint32_t a[4] = {to_tf32(At[k * pa + r]), to_tf32(At[k * pa + r + 8]),
+                                       to_tf32(At[(k + 4) * pa + r]), to_tf32(At[(k + 4) * pa + r + 8])};
                 mma_tf32(d[mt], a, b0, b1);
             }
         }
