@@ -161,11 +161,11 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 93_606, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "9b9b54558a26911a"),
-    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_579, ('scan.cu', 'common.cuh', 'params.cuh'), "879cf75841488dc5"),
-    "output": ("k_output_tc", 130_522, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "9b9b54558a26911a"),
-    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_687, ('scan.cu', 'common.cuh', 'params.cuh'), "879cf75841488dc5"),
-    "bwd_local": ("k_bwd_local_tc", 228_304, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "2c56be22676c9724"),
+    "prep": ("k_prep_tc", 94_366, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "4f7f4249ad410e60"),
+    "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_423, ('scan.cu', 'common.cuh', 'params.cuh'), "75d844aca5b3f39b"),
+    "output": ("k_output_tc", 130_446, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "4f7f4249ad410e60"),
+    "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_703, ('scan.cu', 'common.cuh', 'params.cuh'), "75d844aca5b3f39b"),
+    "bwd_local": ("k_bwd_local_tc", 228_333, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "d31930e42fd70aca"),
 }
 DECODE_TRAFFIC = (481_360_000, ('decode.cu', 'common.cuh', 'params.cuh'), "ace440567370e7de")   # whole Bd=256 H=16 launch
 
