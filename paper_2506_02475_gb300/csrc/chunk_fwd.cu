@@ -452,7 +452,8 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     cudaError_t e;
     if ((e = cudaFuncSetAttribute(k_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
         return e;
-    if ((e = cudaFuncSetAttribute(k_output<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out)))
+    if (!(DK == 256 && sizeof(T) == 2) &&   // head dim 256 (bf16) runs the tcgen05 output kernel
+        (e = cudaFuncSetAttribute(k_output<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out)))
         return e;
     const bool tcp = use_tc_path(sizeof(T) == 2, DK, DV);
     ChunkParams q = p;
@@ -485,6 +486,8 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     if (q.o || q.Eb) {
         if (tcp) {
             if ((e = launch_output_tc(q, s))) return e;
+        } else if (DK == 256 && sizeof(T) == 2) {
+            if ((e = launch_output_wide_tc(q, s))) return e;
         } else if (q.slots > 0) {
             k_output<T, DK, DV><<<dim3(q.slots, q.H / q.vg), 128, sm_out, s>>>(q);   // one CTA per key head
         }
@@ -515,6 +518,7 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
 size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk, bool groups) {
     if (kernel == 1) return scan_smem_bytes(is_bf16, dk, dv);
     if (use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(kernel == 0 ? 0 : 1);
+    if (kernel != 0 && is_bf16 && dk == 256) return output_wide_tc_smem_bytes();
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes(pk) : OutSmem<T, DK, DV>::bytes(groups);
     if (is_bf16) {
