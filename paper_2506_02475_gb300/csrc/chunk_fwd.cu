@@ -450,7 +450,8 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     const size_t sm_prep = PrepSmem<T, DK, DV>::bytes(p.p != nullptr);
     const size_t sm_out = OutSmem<T, DK, DV>::bytes(p.vg > 1);
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(k_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
+    if (!(DK == 256 && sizeof(T) == 2) &&   // head dim 256 (bf16) runs the tcgen05 prep kernel
+        (e = cudaFuncSetAttribute(k_prep<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_prep)))
         return e;
     if (!(DK == 256 && sizeof(T) == 2) &&   // head dim 256 (bf16) runs the tcgen05 output kernel
         (e = cudaFuncSetAttribute(k_output<T, DK, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out)))
@@ -462,6 +463,8 @@ static cudaError_t run_fwd(const ChunkParams& p, bool save, cudaStream_t s, int 
     mark(q, ev0, s);
     if (tcp) {
         if ((e = launch_prep_tc(q, s))) return e;
+    } else if (DK == 256 && sizeof(T) == 2) {
+        if ((e = launch_prep_wide_tc(q, s))) return e;
     } else if (q.slots > 0) {
         k_prep<T, DK, DV><<<dim3(q.slots, q.H / q.vg), 128, sm_prep, s>>>(q);   // one CTA per key head
     }
@@ -518,7 +521,7 @@ cudaError_t launch_fwd(const ChunkParams& p, bool is_bf16, bool save, cudaStream
 size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk, bool groups) {
     if (kernel == 1) return scan_smem_bytes(is_bf16, dk, dv);
     if (use_tc_path(is_bf16, dk, dv)) return tc_smem_bytes(kernel == 0 ? 0 : 1);
-    if (kernel != 0 && is_bf16 && dk == 256) return output_wide_tc_smem_bytes();
+    if (is_bf16 && dk == 256) return kernel == 0 ? prep_wide_tc_smem_bytes() : output_wide_tc_smem_bytes();
 #define COMBA_SM(T, DK, DV) \
     if (dk == DK && dv == DV) return kernel == 0 ? PrepSmem<T, DK, DV>::bytes(pk) : OutSmem<T, DK, DV>::bytes(groups);
     if (is_bf16) {

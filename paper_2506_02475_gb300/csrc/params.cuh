@@ -177,7 +177,9 @@ size_t fwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false,
 cudaError_t launch_prep_tc(const ChunkParams& p, cudaStream_t s);
 cudaError_t launch_output_tc(const ChunkParams& p, cudaStream_t s);
 size_t tc_smem_bytes(int kernel);
-// tcgen05 output kernel of the bf16 head-dim-256 path (value heads 64 wide; out_wide.cu)
+// tcgen05 prep and output kernels of the bf16 head-dim-256 path (value heads 64 wide; wide_tc.cu)
+cudaError_t launch_prep_wide_tc(const ChunkParams& p, cudaStream_t s);
+size_t prep_wide_tc_smem_bytes();
 cudaError_t launch_output_wide_tc(const ChunkParams& p, cudaStream_t s);
 size_t output_wide_tc_smem_bytes();
 // tcgen05 local-gradient kernel of the same path (local_tc.cu)
