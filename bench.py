@@ -143,9 +143,8 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
     if tc and not pk:
         # the tcgen05 local-gradient kernel: S, K K^T per key head; per value head R1 (three
         # C x dk x dv products), (M^T dE) H^T, P^T dO, M^T dE, dPhat K, dPhat^T Q~, dA from
-        # (M^T dE) U^T + (M^T dW) W^T and dG K, dG^T K; it also reads U^T and W^T
-        m["bwd_local"]["flops"] = Pk * 2 * 2 * C * C * dk + P * 2 * (4 * C * dk * dv + 5 * C * C * dk + 4 * C * C * dv)
-        m["bwd_local"]["bytes"] += P * (C * dv + C * dk) * es
+        # (M^T dE) E^T and dG K, dG^T K
+        m["bwd_local"]["flops"] = Pk * 2 * 2 * C * C * dk + P * 2 * (4 * C * dk * dv + 4 * C * C * dk + 4 * C * C * dv)
     if pk:
         m["prep"]["bytes"] += Pk * C * dk * es
         m["bwd_local"]["bytes"] += Pk * 2 * C * dk * es
@@ -165,7 +164,7 @@ CAPTURED_TRAFFIC = {
     "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_423, ('scan.cu', 'common.cuh', 'params.cuh'), "75d844aca5b3f39b"),
     "output": ("k_output_tc", 130_446, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "4f7f4249ad410e60"),
     "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_703, ('scan.cu', 'common.cuh', 'params.cuh'), "75d844aca5b3f39b"),
-    "bwd_local": ("k_bwd_local_tc", 228_333, ('local_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "d31930e42fd70aca"),
+    "bwd_local": ("k_bwd_local_tc", 228_333, ('local_tc.cu', 'tc_frag.cuh', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "d31930e42fd70aca"),
 }
 DECODE_TRAFFIC = (481_112_064, ('decode.cu', 'common.cuh', 'params.cuh'), "a8e4d94175e2cf99")   # whole Bd=256 H=16 launch
 

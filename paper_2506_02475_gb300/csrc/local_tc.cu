@@ -12,8 +12,10 @@
 //   R2  P^T dO                       (behind R1, one wait: dE = Kbar dH' + P^T dO)
 //   R3  M^T dE, dPhat^T Q~
 //   R4  (M^T dE) H^T = -M^T dW (dW = -dE H^T), K K^T, dPhat K
-//   R5  (M^T dE) U^T + (M^T dW) W^T  (= M^T dM M^T, so dA needs neither dM nor a
-//                                     second product with M)
+//   R5  (M^T dE) E^T                 (= M^T dM M^T: dM = dE (Diag(beta) V)^T + dW Ktilde^T with
+//                                     dW = -dE H^T gives (M^T dE) U^T - (M^T dE) (W H)^T, and
+//                                     U - W H = E; so dA needs neither dM, U, W nor a second
+//                                     product with M)
 //   R6  dG K + dG^T K onto dPhat^T Q~
 //
 // Each epilogue first forms what the next round reads and lets it be issued, then does the rest
@@ -49,12 +51,12 @@ struct LocalTcSmem {
                                                    // Q -> Q~, rows 64-127 K; later dq, dk staging
     static constexpr uint32_t OV = OQK + 2 * 32768;  // V [64][128]
     static constexpr uint32_t ODO = OV + 16384;    // dO [64][128]
-    static constexpr uint32_t OE = ODO + 16384;    // E [64][128]; later dv staging
+    static constexpr uint32_t OE = ODO + 16384;    // E [64][128] (read until R5)
     static constexpr uint32_t OH = OE + 16384;     // H^T [128][128]; later dPhat, dM, Y, dG [64][64]
-    static constexpr uint32_t ODH = OH + 32768;    // dH'^T [128][128]; later dW [64][128]
+    static constexpr uint32_t ODH = OH + 32768;    // dH'^T [128][128]; after R1 dE and the dv staging [64][128]
     static constexpr uint32_t OM = ODH + 32768;    // M [64][64]
     static constexpr uint32_t OP = OM + 8192;      // P [64][64]
-    static constexpr uint32_t ODE = OP + 8192;     // dE [64][128]
+    static constexpr uint32_t ODE = OP + 8192;     // dPhat [64][64] (R0 to R3); Comba-pk: dp staging [64][128]
     static constexpr uint32_t OF = ODE + 16384;    // fp32: 8 x 64 per-row vectors, row and column partials, reduction
     static constexpr uint32_t NF = 8 * 64 + 8 * kQ * 64 + 2 * 4 * 64 + 16;
     static constexpr uint32_t NX = 5 * 64 + 4;     // fp32: the next unit's scalars, copied in a unit ahead,
@@ -128,11 +130,11 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 
 // Persistent: CTA b handles units b, b + G, b + 2G, ... (G = gridDim.x, about one CTA per SM).
 // While unit u computes, the tiles of unit u + G stream into buffers as soon as their last
-// reader in unit u has finished (M after R3, H^T after R4, E (after the dv copy), dH'^T, dO and
-// Q/K (into the second of two alternating tiles, which holds M^T dE until then) after R5, V after
-// R6; the per-row and per-head scalars by asynchronous copies after R3), so the loads of consecutive units overlap the
-// tensor-core and epilogue work instead of every SM loading at the same moment.  U^T and W^T of
-// the unit itself load into the dH'^T tile once R1 has read it.
+// reader in unit u has finished (M after R3, H^T after R4, E, dH'^T, dO and Q/K (into the second
+// of two alternating tiles, which holds M^T dE until then) after R5, V after R6; the per-row and
+// per-head scalars by asynchronous copies after R3), so the loads of consecutive units overlap the
+// tensor-core and epilogue work instead of every SM loading at the same moment.  Once R1 has read
+// the dH'^T tile it holds dE (until R3) and the dv staging.
 //
 // PK: Comba-pk feedback vectors P (p.p, shaped like K).  They replace K as the Gram's left factor
 // (P K^T, formed in R5 here), in W = M Diag(btilde gamma_{-1}) P and in the correction q - d p
@@ -146,8 +148,7 @@ __device__ __forceinline__ UnitRef unit_ref(const ChunkParams& p, long long u) {
 struct LocalMaps {
     CUtensorMap dq, dk, dp;           // stores
     CUtensorMap q, k, p, v, dO;       // token tiles (q, k, p per key head; v, dO per value head)
-    CUtensorMap e, h, dh, m, u, w;    // workspace: E [64][128], H^T, dH'^T [128][128], M [64][64],
-                                      // U^T, W^T [128][64]
+    CUtensorMap e, h, dh, m;          // workspace: E [64][128], H^T, dH'^T [128][128], M [64][64]
 };
 
 template <bool PK>
@@ -157,9 +158,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar, bar0, stall_bar;   // bar0: R0; stall_bar: nothing arrives (COMBA_DIAG_STALL)
     // TMA arrival: ldn[0..3] a unit's tiles, in the four groups the previous unit prefetches them in
-    // (M; H^T; E, dH'^T, dO, Q/K; V, and with Comba-pk M), ldu its U^T / W^T, ldp its P (Comba-pk).
-    // Each completes one phase per unit that has rows.
-    __shared__ uint64_t ldn[4], ldu, ldp;
+    // (M; H^T; E, dH'^T, dO, Q/K; V, and with Comba-pk M), ldp its P (Comba-pk).  Each completes
+    // one phase per unit that has rows.
+    __shared__ uint64_t ldn[4], ldp;
     __shared__ uint32_t tbase;
     __shared__ int2 s_nslot;   // (start, length) of the unit after next, loaded during the tail
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -174,11 +175,8 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     uint8_t* sP = sm + S::OP;
     uint8_t* sdE = sm + S::ODE;
     uint8_t* sdPh = sdE;              // dPhat [64][64], from R0's epilogue until R3
-    uint8_t* sdEt = sE;               // dE [64][128], after R1 (E's readers) until R3
-    uint8_t* stV = sE;                // dv staging, after R3
-    uint8_t* sMdW = sdO;              // M^T dW [64][128], after R2 (dO's readers) until R5
-    uint8_t* sUt = sdHt;              // U^T, W^T [128][64] each, after R1 (dH'^T's readers) until R5
-    uint8_t* sWt = sdHt + 16384;
+    uint8_t* sdEt = sdHt;             // dE [64][128], after R1 (dH'^T's readers) until R3
+    uint8_t* stV = sdHt + 16384;      // dv staging, after R3 (E itself is read once more, by R5)
     uint8_t* sdG = sV + 8192;         // dG [64][64], after R3 until R6
     uint8_t* sPf = sM;                // Comba-pk: P [64][128] over the M and P-matrix tiles, R3 to R6
     uint8_t* stP = sdE;               // Comba-pk: dp staging, at the end (dPhat is dead)
@@ -195,7 +193,6 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     float* red = colp + 2 * 4 * 64;
     const uint32_t udO = smem_u32(sdO), uE = smem_u32(sE), uH = smem_u32(sHt), udH = smem_u32(sdHt),
                    uM = smem_u32(sM), uP = smem_u32(sP), udE = smem_u32(sdEt), udPh = smem_u32(sdPh),
-                   uMdW = smem_u32(sMdW), uUt = smem_u32(sUt), uWt = smem_u32(sWt),
                    udG = smem_u32(sdG), uPf = smem_u32(sPf);
 
     const int Hk = p.H / p.vg;   // key heads: q, k, alpha, beta, b, d of value head h are key head h / vg's
@@ -256,7 +253,7 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         }
     };
     uint32_t pend = 0;   // thread kTma: barriers with loads issued and not yet waited on (bit i: ldn[i],
-                         // 4: ldu, 5: ldp), drained on the give-up path
+                         // 5: ldp), drained on the give-up path
     // A unit's scalars, copied into sNx a unit ahead (asynchronous 4-byte copies, which hold no
     // registers and wait behind no tile traffic): per row r (thread r < 64) the log-decays G_r and
     // G_{r-1}, beta, alpha and b; per head (thread 0) d and, with Comba-pk, the feedback d.
@@ -282,7 +279,6 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         mbar_init(smem_u32(&bar0), 1);
         mbar_init(smem_u32(&stall_bar), 1);
         for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&ldn[i]), 1);
-        mbar_init(smem_u32(&ldu), 1);
         mbar_init(smem_u32(&ldp), 1);
         mbar_fence_init();
     }
@@ -539,16 +535,8 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             const bool ok2 = mma_wait();
             ok = ok && ok2;
         }
-        // this unit's U^T, W^T (read by R5) into the dead dH'^T tile
-        if (ok && tid == kTma) {
-            const uint32_t mb = smem_u32(&ldu);
-            mbar_expect_tx(mb, 32768u);
-            tma_load_2d(uUt, &mp.u, 0, (int)(idx * 128), mb);
-            tma_load_2d(uWt, &mp.w, 0, (int)(idx * 128), mb);
-            pend |= 16u;
-        }
         if (ok) {
-            // dE = Kbar dH' + P^T dO (over the dead E tile: an R3 operand)
+            // dE = Kbar dH' + P^T dO (over the dead dH'^T tile: an R3 operand)
             float de[NK][4], t2[NK][4];
             uint32_t re[NK * 4], rt[NK * 4];
             tmem_issue<NK>(tq + 384 + nk0, re);
@@ -643,19 +631,19 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
         if (ok && has_next && tid == kTma) { issue_n1(nxt); pend |= 2u; }   // R4 was H^T's last reader
         float t4[NK][4];
         if (ok) {
-            // M^T dW in bf16 over the dead dO tile: the R5 operand
+            // M^T dW = -(M^T dE) H^T, for dk (the W path) and its row dots
             tmem_frag<NK>(tq + 0 + nk0, t4);
 #pragma unroll
             for (int t = 0; t < NK; ++t)
 #pragma unroll
                 for (int i = 0; i < 4; ++i) t4[t][i] = -t4[t][i];
-            frag_store_sw<NK>(sMdW, 64, m0, nk0, t4);
         }
-        // U^T, W^T have landed, and with Comba-pk P (its rows past a short chunk zeroed)
+        // every thread's dv rows are copied (the next unit's dH'^T loads over their staging after R5),
+        // and with Comba-pk P has landed (its rows past a short chunk zeroed)
         {
-            bool okl = ok && mbar_wait_polls(smem_u32(&ldu), lph, p.wait_ns);
+            bool okl = ok;
             if constexpr (PK) okl = okl && mbar_wait_polls(smem_u32(&ldp), lph, p.wait_ns);
-            if (okl && tid == kTma) pend &= ~48u;
+            if (okl && tid == kTma) pend &= ~32u;
             if constexpr (PK)
                 if (okl && L < kChunk) zero_rows(sPf, 64, L);
             fence_async_smem();
@@ -664,12 +652,12 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             tc_fence_after();
         }
 
-        // ---------------- R5: M^T dM M^T = (M^T dE) U^T + (M^T dW) W^T, with dM = dE (Diag(beta) V)^T +
-        // dW (Diag(btilde gamma_{-1}) K)^T, U = M Diag(beta) V and W = M Diag(btilde gamma_{-1}) K
+        // ---------------- R5: M^T dM M^T = (M^T dE) E^T.  With dM = dE (Diag(beta) V)^T + dW (Diag(btilde
+        // gamma_{-1}) K)^T, U = M Diag(beta) V and W = M Diag(btilde gamma_{-1}) K it is (M^T dE) U^T +
+        // (M^T dW) W^T, and dW = -dE H^T turns the second term into -(M^T dE) (W H)^T; E = U - W H.
         if (tid == 0) {
             if (ok) {
-                tc_gemm_m64<false, true>(tmem + 192, uMdE, 64, uUt, 128, 64, D, false);
-                tc_gemm_m64<false, true>(tmem + 192, uMdW, 64, uWt, 128, 64, D, true);
+                tc_gemm_m64<false, false>(tmem + 192, uMdE, 64, uE, 64, 64, D, false);
                 if constexpr (PK) tc_gemm_m64<false, false>(tmem + 128, uPf, 64, uK, 128, 64, D, false);   // P K^T
             }
             tc_commit(smem_u32(&bar));
@@ -707,9 +695,9 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
             const bool ok5 = mma_wait();
             ok = ok && ok5;
         }
-        // the next unit's E (the dv rows, copied before R4's wait, were the E tile's last use), dH'^T
-        // (U^T and W^T are dead), dO (M^T dW is dead) and Q/K (M^T dE is dead; the previous unit's
-        // dq, dk stores have read this tile: the prologue waited for them)
+        // the next unit's E (R5 was its last reader), dH'^T (dE and the dv rows staged over it are
+        // dead: the rows were copied before R4's wait), dO and Q/K (M^T dE is dead; the previous
+        // unit's dq, dk stores have read this tile: the prologue waited for them)
         if (ok && has_next && tid == kTma) { issue_n2(sQKn, nxt); pend |= 4u; }
         if (ok) {
             // dA = -(M^T dM M^T) on the strict lower triangle -> dG (the R6 operand)
@@ -975,11 +963,10 @@ __global__ void __launch_bounds__(kLocalThreads, 1)
     }
     cp_async_wait<0>();   // no scalar copy is still writing shared memory at exit
     // no tile copy is still writing shared memory at exit (after a give-up, the next unit's tiles are
-    // in the phase after this one's, U^T / W^T and P in this one's)
+    // in the phase after this one's, P in this one's)
     if (tid == kTma && pend) {
         for (int i = 0; i < 4; ++i)
             if (pend & (1u << i)) mbar_drain(smem_u32(&ldn[i]), lph);
-        if (pend & 16u) mbar_drain(smem_u32(&ldu), lph ^ 1);
         if (pend & 32u) mbar_drain(smem_u32(&ldp), lph ^ 1);
     }
     if (tid == 0) bulk_wait_rows_done();   // and no bulk store is still reading it
@@ -1014,9 +1001,7 @@ cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s) {
                 make_bf16_map(&mp.e, p.Eb, units * 64, tc::D, 64) &&
                 make_bf16_map(&mp.h, p.Hb, units * tc::D, tc::D, tc::D) &&
                 make_bf16_map(&mp.dh, p.dHb, units * tc::D, tc::D, tc::D) &&
-                make_bf16_map(&mp.m, p.Mb, units * 64, 64, 64) &&
-                make_bf16_map(&mp.u, p.Ub, units * tc::D, 64, tc::D) &&
-                make_bf16_map(&mp.w, p.Wb, units * tc::D, 64, tc::D);
+                make_bf16_map(&mp.m, p.Mb, units * 64, 64, 64);
     if (pk) {
         good = good && p.dpp && make_bf16_token_map(&mp.dp, p.dpp, p.Ttot, p.H, tc::D) &&
                make_bf16_token_map(&mp.p, p.p, p.Ttot, Hk, tc::D);
