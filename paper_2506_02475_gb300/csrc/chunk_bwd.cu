@@ -10,8 +10,9 @@
 //   (scan.cu)   : the reverse scan dH_n = gamma dH_{n+1} + Atilde^T dH_{n+1} + C_n
 //   k_bwd_local : per chunk, every local gradient given H_n, dH', E:
 //                 dE; dQ~ = dPhat K + Diag(gamma) dO H^T;  dV = Diag(beta) M^T dE;
-//                 dW = -dE H^T;  dM = dE (Diag(beta)V)^T + dW Ktilde^T;
-//                 dA = strict_lower(-M^T dM M^T);  dK from P, Kbar, W and A;
+//                 dW = -dE H^T;  dA = strict_lower(-M^T dM M^T) with M^T dM M^T = (M^T dE) E^T
+//                 (dM = dE (Diag(beta)V)^T + dW Ktilde^T, U = M Diag(beta) V, W = M Ktilde
+//                 and E = U - W H);  dK from P, Kbar, W and A;
 //                 dbeta, dbtilde, and d log alpha via a reverse cumsum of the
 //                 per-position log-decay gradient inside the chunk
 //   k_reduce_heads : deterministic sums of the per-chunk db, dd partials.
@@ -243,11 +244,11 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     float* rowp = sc.take<float>(S::NROW * 2 * 64);
     float* colp = sc.take<float>(2 * 4 * 64);
     float* red = sc.take<float>(8);
-    // P (for dE) lives where dW will go; phase-B aliases: dO, E, dE and H are dead after phase A
+    // P (for dE) lives where dW will go; phase-B aliases: dO, dE and H are dead after phase A (E is
+    // read once more, by M^T dM M^T = (M^T dE) E^T)
     T* sP = sdW;
     T* sdPh = sdO;
-    T* sdM = sE;
-    T* sY = sdE;
+    T* sMdE = sdE;   // M^T dE, from the end of phase A
     T* sdG = sH;
 
     const int hk = h / p.vg;   // key head: q, k, p, alpha, beta, b, d
@@ -426,16 +427,10 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
             for (int i = 0; i < 4; ++i) tmp[t][i] = -tmp[t][i];
         frag_store<T, NK>(sdW, PK, m0, nk0, tmp);
     }
-    float dP[4][4], dMa[4][4];
+    float dP[4][4];
     const int nl0 = 32 * wc;
     zero(dP);
     warp_gemm<true, true, 4>(dP, sdO, PV, sE, PV, m0, nl0, DV);
-    zero(dMa);
-    warp_gemm<true, true, 4>(dMa, sdE, PV, sV, PV, m0, nl0, DV);
-#pragma unroll
-    for (int t = 0; t < 4; ++t)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) dMa[t][i] *= sBe[nl0 + frag_col(t, i)];
     {
         // dV = Diag(beta) M^T dE ; direct dbeta = v . (M^T dE)
         const int nv0 = wc * (DV / 2);
@@ -451,14 +446,15 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
         float s0, s1;
         frag_rowdot(t0r, s0, s1);
         put_rows(2, s0, s1);
+        __syncthreads();   // every warp has read V (the row dots) and dE before dV and M^T dE replace them
+        frag_store<T, NV>(sMdE, PV, m0, nv0, tv);
         const float ba = sBe[ra], bb = sBe[rb];
 #pragma unroll
         for (int t = 0; t < NV; ++t) { tv[t][0] *= ba; tv[t][1] *= ba; tv[t][2] *= bb; tv[t][3] *= bb; }
-        __syncthreads();   // every warp has read V (dM, the row dots) before dV replaces it
         frag_store<T, NV>(sDV, PV, m0, nv0, tv);
     }
     if constexpr (PKV) cp_async_wait<0>();
-    __syncthreads();   // dO, E, dE, H, dH' no longer needed; dW complete (and P landed)
+    __syncthreads();   // dO, dE, H, dH' no longer needed; dW and M^T dE complete (and P landed)
 
     // ---------------- phase B: contractions over dk and the 64 x 64 algebra
     float gr[4][4], sq[4][4];
@@ -466,9 +462,6 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     warp_gemm<true, true, 4>(gr, sF, PK, sK, PK, m0, nl0, DK);   // Gram P K^T (P = K unless pk)
     zero(sq);
     warp_gemm<true, true, 4>(sq, sQ, PK, sK, PK, m0, nl0, DK);   // Q~ K^T
-    float mb[4][4];
-    zero(mb);
-    warp_gemm<true, true, 4>(mb, sdW, PK, sF, PK, m0, nl0, DK);  // dW P^T
     {
         float rs0 = 0.f, rs1 = 0.f;
         float cs[4][2];
@@ -486,8 +479,6 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
                 if (i < 2) rs0 += w; else rs1 += w;
                 cs[t][i & 1] += w;
                 sdPh[r * PL + c] = from_f<T>(dP[t][i] * gam);
-                const float dm = dMa[t][i] + mb[t][i] * sWs[c];
-                sdM[r * PL + c] = from_f<T>(dm);
             }
         }
         rs0 = quad_sum(rs0);
@@ -503,16 +494,9 @@ __global__ void __launch_bounds__(256) k_bwd_local(ChunkParams p) {
     }
     __syncthreads();
     {
-        float y[4][4];
-        zero(y);
-        warp_gemm<false, false, 4>(y, sM, PL, sdM, PL, m0, nl0, 64);   // Y = M^T dM
-        frag_store<T, 4>(sY, PL, m0, nl0, y);
-    }
-    __syncthreads();
-    {
         float da[4][4];
         zero(da);
-        warp_gemm<true, true, 4>(da, sY, PL, sM, PL, m0, nl0, 64);     // Y M^T
+        warp_gemm<true, true, 4>(da, sMdE, PV, sE, PV, m0, nl0, DV);   // M^T dM M^T = (M^T dE) E^T
         float rb0 = 0.f, rb1 = 0.f, ra0 = 0.f, ra1 = 0.f;
         float cs[4][2];
 #pragma unroll
