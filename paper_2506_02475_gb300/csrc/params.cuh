@@ -185,9 +185,9 @@ size_t output_wide_tc_smem_bytes();
 // tcgen05 local-gradient kernel of the same path (local_tc.cu)
 cudaError_t launch_bwd_local_tc(const ChunkParams& p, cudaStream_t s);
 size_t local_tc_smem_bytes();
-// The tcgen05 kernels serve bf16 dk = dv = 128 (with Comba-pk feedback vectors all but the
-// local-gradient kernel, which then is the mma.sync one); every other case runs the mma.sync
-// kernels.
+// The tcgen05 kernels of chunk_tc.cu, local_tc.cu and scan.cu serve bf16 dk = dv = 128, with or
+// without Comba-pk feedback vectors; bf16 dk = 256 runs the kernels of wide_tc.cu and
+// scan_wide.cu with the mma.sync local-gradient kernel; every other case runs the mma.sync kernels.
 inline bool use_tc_path(bool is_bf16, int dk, int dv) { return is_bf16 && dk == 128 && dv == 128; }
 size_t bwd_smem_bytes(int kernel, bool is_bf16, int dk, int dv, bool pk = false);
 // `p`: Comba-pk feedback vectors [Bd,H,dk] or null (p = k).
