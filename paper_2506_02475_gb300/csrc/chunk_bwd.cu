@@ -20,29 +20,6 @@
 
 namespace comba {
 
-template <typename T, int NT>
-__device__ __forceinline__ void frag_store_g(T* g, long long ld, int m0, int n0, const float (&acc)[NT][4], int valid) {
-#pragma unroll
-    for (int t = 0; t < NT; ++t)
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            const int r = m0 + frag_row(2 * hh);
-            if (r >= valid) continue;
-            T* dst = g + (long long)r * ld + n0 + frag_col(t, 0);
-            dst[0] = from_f<T>(acc[t][2 * hh]);
-            dst[1] = from_f<T>(acc[t][2 * hh + 1]);
-        }
-}
-
-__device__ __forceinline__ void seq_range_b(const ChunkParams& p, int n, long long& start, long long& len) {
-    long long a = p.cu ? p.cu[n] : (long long)n * p.T;
-    long long e = p.cu ? p.cu[n + 1] : (long long)(n + 1) * p.T;
-    a = a < 0 ? 0 : (a > p.Ttot ? p.Ttot : a);
-    e = e < a ? a : (e > p.Ttot ? p.Ttot : e);
-    start = a;
-    len = e - a;
-}
-
 // ------------------------------------------------- reverse-scan additive term
 
 template <typename T, int DK, int DV>

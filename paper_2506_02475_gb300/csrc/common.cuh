@@ -55,19 +55,6 @@ __device__ __forceinline__ void load_tile(T* s, int sp, const T* g, long long gs
     }
 }
 
-// Store a shared tile to a strided global matrix (rows < valid_rows only).
-template <typename T>
-__device__ __forceinline__ void store_tile(T* g, long long gstride, const T* s, int sp, int rows, int cols,
-                                           int valid_rows, int tid, int nthreads) {
-    constexpr int V = 16 / sizeof(T);
-    const int vpr = cols / V;
-    for (int idx = tid; idx < rows * vpr; idx += nthreads) {
-        const int r = idx / vpr, c = (idx % vpr) * V;
-        if (r < valid_rows)
-            *reinterpret_cast<uint4*>(g + (long long)r * gstride + c) = *reinterpret_cast<const uint4*>(s + r * sp + c);
-    }
-}
-
 // ---------------------------------------------------- tensor-core fragments
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -235,10 +222,9 @@ struct SmemCarver {
 __host__ __device__ constexpr size_t carve_bytes(size_t off, size_t bytes) { return ((off + 127) & ~size_t(127)) + bytes; }
 __host__ __device__ constexpr size_t align128(size_t off) { return (off + 127) & ~size_t(127); }
 
-// Inclusive prefix sum of log(alpha) over a chunk (warp-wide; lane handles
-// positions lane and lane + 32).  Positions >= L contribute 0, so G stays
-// finite there.  Writes G[p] and Gm1[p] = G[p-1] (Gm1[0] = 0).
-// chunk_log_cumsum_vals takes the lane's alpha values (positions lane, lane + 32) already loaded.
+// Inclusive prefix sum of log(alpha) over a chunk (warp-wide; the lane passes its
+// alpha values at positions lane and lane + 32, already loaded).  Positions >= L
+// contribute 0, so G stays finite there.  Writes G[p] and Gm1[p] = G[p-1] (Gm1[0] = 0).
 __device__ __forceinline__ void chunk_log_cumsum_vals(float a0, float a1, int L, float* G, float* Gm1) {
     const int lane = threadIdx.x & 31;
     float x0 = lane < L ? logf(a0) : 0.f;
@@ -257,12 +243,6 @@ __device__ __forceinline__ void chunk_log_cumsum_vals(float a0, float a1, int L,
     const float p1 = __shfl_up_sync(0xffffffffu, x1, 1);
     Gm1[lane] = lane == 0 ? 0.f : p0;
     Gm1[lane + 32] = lane == 0 ? tot0 : p1;
-}
-__device__ __forceinline__ void chunk_log_cumsum(const float* alpha, long long stride, int L, float* G, float* Gm1) {
-    const int lane = threadIdx.x & 31;
-    const float a0 = lane < L ? alpha[(long long)lane * stride] : 1.f;
-    const float a1 = lane + 32 < L ? alpha[(long long)(lane + 32) * stride] : 1.f;
-    chunk_log_cumsum_vals(a0, a1, L, G, Gm1);
 }
 
 // ------------------------------------------- sm_100-family async primitives
@@ -372,18 +352,6 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(taddr), "r"(ncols) : "memory");
 }
 
-// Shared-memory matrix descriptor (sm_100 format): K-major operand in the
-// 128-byte swizzle layout (8-row atoms of 128 bytes, atoms 1024 bytes apart).
-__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr >> 4) & 0x3FFF);
-    d |= (uint64_t)(16 >> 4) << 16;     // leading byte offset (unused for swizzled K-major)
-    d |= (uint64_t)(1024 >> 4) << 32;   // stride byte offset: next 8-row atom
-    d |= (uint64_t)1 << 46;             // descriptor version
-    d |= (uint64_t)2 << 61;             // 128-byte swizzle
-    return d;
-}
-
 // Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both operands K-major.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
@@ -476,11 +444,6 @@ template <bool AMN, bool BMN>
 __device__ __forceinline__ void tc_gemm_m64(uint32_t tmem, uint32_t a, int a_ext, uint32_t b, int b_ext, int N, int K,
                                             bool accumulate) {
     tc_gemm_mk<64, AMN, BMN>(tmem, a, a_ext, b, b_ext, N, K, accumulate);
-}
-
-// Byte offset of element (mn, k) of an MN-major bf16 tile (allocated K extent krows).
-__host__ __device__ constexpr uint32_t mn128_offset(int mn, int k, int krows) {
-    return (uint32_t)((mn >> 6) * krows * 128 + k * 128 + ((((mn & 63) >> 3) ^ (k & 7)) << 4) + (mn & 7) * 2);
 }
 
 // 16 consecutive fp32 accumulator columns of this thread's TMEM lane.

@@ -8,19 +8,6 @@ namespace tc {
 
 constexpr int D = 128;  // head dim of this path
 
-// cp.async a row-major bf16 matrix (rows r < valid; `cols` in {64, 128}) into a
-// 128B-swizzled tile with `alloc` rows; rows valid..alloc-1 are zero-filled.
-__device__ __forceinline__ void load_sw(uint8_t* tile, int alloc, int cols, const bf16* g, long long gstride,
-                                        int valid, int tid, int nthr = 128) {
-    const int cpr = cols / 8;
-    for (int idx = tid; idx < alloc * cpr; idx += nthr) {
-        const int r = idx / cpr, ch = idx - r * cpr;
-        const bool ok = r < valid;
-        cp_async16(tile + sw128_offset(r, ch * 8, alloc),
-                   ok ? (const void*)(g + (long long)r * gstride + ch * 8) : (const void*)g, ok);
-    }
-}
-
 __device__ __forceinline__ uint4 pack8(const float* v) {
     uint4 r;
     __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
