@@ -193,31 +193,6 @@ def make(name: str, *, B=None, T=None, H=None, dk=None, dv=None, dtype=None, see
                     dO=dO, dhT=dhT, cu_seqlens=cu)
 
 
-@dataclass
-class DecodeWorkload:
-    dtype: str
-    state: np.ndarray               # [Bd,H,dk,dv] fp32
-    q: np.ndarray                   # [S,Bd,H,dk]  one slice per decode step
-    k: np.ndarray
-    v: np.ndarray                   # [S,Bd,H,dv]
-    alpha: np.ndarray               # [S,Bd,H]
-    beta: np.ndarray
-    d: np.ndarray                   # [H]
-    b: Optional[np.ndarray] = None
-
-
-def make_decode(Bd=256, H=16, dk=128, dv=128, steps=1, dtype="bf16", seed_offset=0, with_b=False,
-                state_std=0.05) -> DecodeWorkload:
-    """Decode workload: fp32 state ~ N(0, state_std^2) plus ``steps`` tokens per (row, head)."""
-    rng = np.random.Generator(np.random.PCG64(SEED + 5000 + seed_offset))
-    state = (state_std * rng.standard_normal((Bd, H, dk, dv), dtype=np.float32)).astype(np.float32)
-    q, k, v = _tokens(rng, (steps, Bd), H, dk, dv, dtype)
-    alpha, beta = _gates(rng, (steps, Bd, H))
-    d = rng.uniform(0.0, 1.0, size=H).astype(np.float32)
-    b = rng.uniform(0.0, 1.0, size=H).astype(np.float32) if with_b else None
-    return DecodeWorkload(dtype=dtype, state=state, q=q, k=k, v=v, alpha=alpha, beta=beta, d=d, b=b)
-
-
 def decode_state(Bd=256, H=16, dk=128, dv=128, seed_offset=0, state_std=0.05) -> np.ndarray:
     """fp32 decode state [Bd,H,dk,dv] ~ N(0, state_std^2)."""
     rng = np.random.Generator(np.random.PCG64(SEED + 6000 + seed_offset))
