@@ -1,5 +1,8 @@
 """Pins of the oracle's gate and normalisation prologue (section 3.1 gates, L2-normalised q and k)."""
+import types
+
 import numpy as np
+import pytest
 
 from oracle import gated
 
@@ -37,15 +40,19 @@ def test_forward_is_invariant_to_key_and_query_scale():
 
 
 def test_gated_gradients_match_finite_differences():
+    _finite_difference_pin(gated)
+
+
+def _finite_difference_pin(mod):
     for variant in ("splr", "iplr"):
         p = _problem(3)
         rng = np.random.default_rng(4)
         dO = rng.standard_normal(p["v"].shape)
         dhT = rng.standard_normal(p["h0"].shape)
-        g = gated.bwd(**p, dO=dO, dhT=dhT, variant=variant)
+        g = mod.bwd(**p, dO=dO, dhT=dhT, variant=variant)
 
         def loss():
-            o, hT = gated.fwd(**p, variant=variant)
+            o, hT = mod.fwd(**p, variant=variant)
             return float(np.sum(o * dO) + np.sum(hT * dhT))
 
         names = {"q": "dq", "k": "dk", "v": "dv", "g_alpha": "dg_alpha", "g_beta": "dg_beta", "a": "da", "c": "dc",
@@ -62,3 +69,30 @@ def test_gated_gradients_match_finite_differences():
                 fd = (lp - lm) / 2e-6
                 an = g[gname].reshape(-1)[i]
                 assert abs(fd - an) <= 3e-6 * max(1.0, abs(an)), (variant, name, fd, an)
+
+
+# Planted mistakes in the prologue's backward, each a plausible slip of the chain rule.
+SLIPS = {
+    "l2norm_without_projection": ('dq = (g["dq"] - qh * np.sum(qh * g["dq"], axis=-1, keepdims=True)) / nq',
+                                  'dq = g["dq"] / nq'),
+    "forget_gate_without_a": ('dg_alpha = g["dalpha"] * (-a64 * alpha * sigmoid(z))',
+                              'dg_alpha = g["dalpha"] * (-alpha * sigmoid(z))'),
+    "da_with_sigmoid": ("(-alpha * softplus(z))", "(-alpha * sigmoid(z))"),
+    "input_gate_derivative_truncated": ('dg_beta = g["dbeta"] * beta * (1.0 - beta)', 'dg_beta = g["dbeta"] * beta'),
+    "dc_from_dalpha": ("dc = np.sum(dg_alpha, axis=lead)", 'dc = np.sum(g["dalpha"], axis=lead)'),
+    "feedback_gate_derivative_dropped": ('db_raw = g["db"] * b * (1.0 - b)', 'db_raw = g["db"]'),
+}
+
+
+@pytest.mark.parametrize("name", sorted(SLIPS))
+def test_planted_slip_in_the_prologue_backward_is_caught(name):
+    old, new = SLIPS[name]
+    with open(gated.__file__) as f:
+        src = f.read()
+    assert src.count(old) == 1, name
+    src = src.replace("from . import bwd as _bwd", "from oracle import bwd as _bwd")
+    src = src.replace("from . import fwd as _fwd", "from oracle import fwd as _fwd")
+    ns = {"__name__": "gated_variant"}
+    exec(compile(src.replace(old, new), "gated_variant", "exec"), ns)
+    with pytest.raises(AssertionError):
+        _finite_difference_pin(types.SimpleNamespace(fwd=ns["fwd"], bwd=ns["bwd"]))
