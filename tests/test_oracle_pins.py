@@ -52,6 +52,22 @@ def test_hand_worked_scalar_example():
     np.testing.assert_allclose(hT.ravel(), [g["expected"]["hT"]], rtol=0, atol=1e-14)
 
 
+@pytest.mark.parametrize("form", ["splr", "iplr", "pk"])
+def test_hand_worked_two_by_two_example(form):
+    """dk = dv = 2, two tokens, worked by hand: fixes the state's orientation (S = H^T), the
+    order of the transition's outer product, and the iplr and pk forms."""
+    g = json.load(open(os.path.join(GOLDEN, "matrix_two_tokens.json")))
+    x = g["inputs"]
+    q, k, v, fv = (np.array(x[n]).reshape(2, 1, 2) for n in ("q", "k", "v", "p"))
+    a = np.array(x["alpha"]).reshape(2, 1)
+    be = np.array(x["beta"]).reshape(2, 1)
+    h0 = np.array(x["S0"]).T.reshape(1, 1, 2, 2)
+    o, hT = oracle.fwd(q, k, v, a, be, np.array([x["b"]]), np.array([x["d"]]), h0=h0,
+                       variant="iplr" if form == "iplr" else "splr", p=fv if form == "pk" else None)
+    np.testing.assert_allclose(o.reshape(2, 2), g["expected"][form]["o"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(hT.reshape(2, 2), g["expected"][form]["hT"], rtol=0, atol=1e-14)
+
+
 # ------------------------------------------------------------------ reductions
 
 def test_reduces_to_gated_linear_attention_when_no_feedback():
