@@ -52,6 +52,18 @@ def test_hand_worked_scalar_example():
     np.testing.assert_allclose(hT.ravel(), [g["expected"]["hT"]], rtol=0, atol=1e-14)
 
 
+def test_hand_worked_scalar_backward():
+    """The same two tokens' gradients, worked by hand (the adjoint carried through the decay)."""
+    g = json.load(open(os.path.join(GOLDEN, "scalar_two_tokens.json")))
+    x, bw = g["inputs"], g["backward"]
+    args = [np.array(x[n]).reshape(2, 1, 1) for n in ("q", "k", "v")]
+    args += [np.array(x["alpha"]).reshape(2, 1), np.array(x["beta"]).reshape(2, 1)]
+    out = oracle.bwd(*args, np.array([x["b"]]), np.array([x["d"]]), np.array(bw["inputs"]["dO"]).reshape(2, 1, 1),
+                     h0=np.array(x["h0"]).reshape(1, 1, 1, 1), dhT=np.array(bw["inputs"]["dhT"]).reshape(1, 1, 1, 1))
+    for name, want in bw["expected"].items():
+        np.testing.assert_allclose(out[name].ravel(), np.ravel(want), rtol=0, atol=1e-13, err_msg=name)
+
+
 @pytest.mark.parametrize("form", ["splr", "iplr", "pk"])
 def test_hand_worked_two_by_two_example(form):
     """dk = dv = 2, two tokens, worked by hand: fixes the state's orientation (S = H^T), the
