@@ -160,11 +160,11 @@ def stage_model(dk, dv, slots, H, N, save=True, tc=True, pk=False, vg=1):
 # (every launch touches each unit's tiles once).  A figure is kept only while the
 # sources of its kernel hash to the captured value; otherwise traffic is null.
 CAPTURED_TRAFFIC = {
-    "prep": ("k_prep_tc", 94_366, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "d99997f061bebb13"),
+    "prep": ("k_prep_tc", 94_366, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "be4b1d27b40aa1f1"),
     "scan_fwd": ("k_scan_tc_split<128,128,0,2>", 83_423, ('scan.cu', 'common.cuh', 'params.cuh'), "2ff0c8eb7a5e3add"),
-    "output": ("k_output_tc", 130_446, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "d99997f061bebb13"),
+    "output": ("k_output_tc", 130_446, ('chunk_tc.cu', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "be4b1d27b40aa1f1"),
     "scan_bwd": ("k_scan_tc_split<128,128,1,1>", 85_703, ('scan.cu', 'common.cuh', 'params.cuh'), "2ff0c8eb7a5e3add"),
-    "bwd_local": ("k_bwd_local_tc", 193_867, ('local_tc.cu', 'tc_frag.cuh', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "4ed79ac9d74cce08"),
+    "bwd_local": ("k_bwd_local_tc", 193_867, ('local_tc.cu', 'tc_frag.cuh', 'tc_tiles.cuh', 'common.cuh', 'params.cuh'), "4eca458cdd2721f9"),
 }
 DECODE_TRAFFIC = (481_112_064, ('decode.cu', 'common.cuh', 'params.cuh'), "fba8e9172f2784c4")   # whole Bd=256 H=16 launch
 

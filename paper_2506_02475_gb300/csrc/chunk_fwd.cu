@@ -7,9 +7,10 @@
 //                 Atilde = -Kbar^T W, B = Kbar^T U (the inter-chunk state
 //                 equation with Kbar = Diag(gamma_C / gamma_r) K)
 //   (scan.cu)   : the sequential scan of those maps
-//   k_output    : per chunk, E = U - W H_n and the output equation (at head dim 256 with the
-//                 backward's workspace also Z = Diag(gamma) Q~ - P W for the reverse scan)
+//   k_output    : per chunk, E = U - W H_n and the output equation
 //                 O = Diag(gamma) Q~ H_n + Tril(Q~ K^T * Gamma) E, Q~ = Q - d K
+// These serve the shapes off the tcgen05 kernels (chunk_tc.cu for bf16 d = 128,
+// wide_tc.cu for bf16 head dim 256).
 #include "params.cuh"
 
 namespace comba {

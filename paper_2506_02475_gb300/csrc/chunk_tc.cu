@@ -1,14 +1,15 @@
 // tcgen05 (5th-generation tensor core) kernels for the bf16, dk = dv = 128 path.
 //
 // Every tile product is issued by one thread as tcgen05.mma (M = 128, fp32
-// accumulator in TMEM) on 128-byte-swizzled shared-memory tiles; the other
-// threads stage tiles with asynchronous copies and run the epilogues on the
+// accumulator in TMEM) on 128-byte-swizzled shared-memory tiles that TMA
+// loads; the other threads run the epilogues on the
 // rows they read back from TMEM (one row per thread).  Products are formed
 // transposed where that puts a 128-wide head dimension on M (W^T, U^T, E^T,
 // O^T, (P W)^T); 64 x 64 chunk products pad M to 128 with zero rows.
 //
-//   k_prep_tc      Gram K K^T -> decay/btilde mask -> UT inverse M (fp32, blocked
-//                  forward substitution) -> W^T = K^T Mw^T, U^T = V^T Mu^T ->
+//   k_prep_tc      Gram K K^T -> decay/btilde mask -> UT inverse M (fp32 forward
+//                  substitution on the 16 x 16 diagonal blocks, tf32 tile products for
+//                  the off-diagonal levels) -> W^T = K^T Mw^T, U^T = V^T Mu^T ->
 //                  Atilde = -K^T Diag(s) W  (s = gamma_C/gamma_r), and U_s^T = (Diag(s) U)^T
 //                  for the forward scan, which forms B^T = U_s^T K itself;
 //                  with Comba-pk feedback vectors P: Gram P K^T and W^T = P^T Mw^T

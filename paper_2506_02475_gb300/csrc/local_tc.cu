@@ -1,9 +1,9 @@
 // Local chunk gradients on the tcgen05 path (bf16, dk = dv = 128).
 //
 // Same algebra as k_bwd_local (chunk_bwd.cu): given a chunk's K, Q, V, dO, its
-// saved E = U - W H_n, chunk state H_n, incoming state gradient dH', inverse
-// M and WY factors U, W, form dq, dk, dv, the log-decay and beta gradients and
-// the per-chunk db, dd partials.  The tile products are tcgen05.mma groups
+// saved E = U - W H_n, chunk state H_n, incoming state gradient dH' and inverse
+// M (and Comba-pk's feedback vectors P), form dq, dk, dv (and dp), the log-decay
+// and beta gradients and the per-chunk db, dd partials.  The tile products are tcgen05.mma groups
 // with M = 64 (the chunk rows), issued by one thread into TMEM; the warps wait
 // on them six times a unit:
 //
