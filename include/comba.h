@@ -118,8 +118,9 @@ typedef struct {
  * Saved factors (training step without recomputation).
  *   comba_chunk_fwd with COMBA_SAVE_FACTORS also keeps everything the
  *   backward needs (chunk table, W, U, log-decays, the UT inverses M, the
- *   chunk-start states H_n, E = U - W H_n and, at dk = dv = 128 in bf16, the
- *   factor Z = Qhat - P W of the reverse scan's additive term) in its workspace, which must then
+ *   chunk-start states H_n, E = U - W H_n and, in bf16 at dk = dv = 128 and at
+ *   dk = 256, the factor Z = Qhat - P W of the reverse scan's additive term) in
+ *   its workspace, which must then
  *   hold comba_workspace_size(shape, 1) bytes (else COMBA_ERR_WORKSPACE).
  *   comba_chunk_bwd with COMBA_REUSE_FACTORS reads them from the workspace
  *   instead of recomputing the forward chunk factors and states.  The
@@ -195,8 +196,9 @@ comba_status_t comba_chunk_bwd_gated(const comba_shape_t *shape,
  * p = b k with b = 1 the paper's way of folding b into p).  In the chunk form the
  * Gram inside the inverse becomes P K^T and W = M Diag(btilde gamma_{r-1}) P.  The
  * shape passed to the pk calls and to comba_workspace_size must carry COMBA_PK (the
- * workspace then also holds q - d p).  The local-gradient kernel of these calls is
- * the mma.sync one for every shape.
+ * workspace then also holds q - d p).  The pk calls run the same kernels as the
+ * plain form at every head width (tcgen05 at bf16 dk = dv = 128; at head dim 256
+ * the local gradients on the mma.sync kernel, as for the plain form).
  */
 #define COMBA_PK 16
 
@@ -273,7 +275,8 @@ comba_status_t comba_chunk_fwd(const comba_shape_t *shape,
  *     L = <o, dO> + <hT, dhT>
  * through the forward above (the paper prints no backward; these are the
  * chain-rule derivatives of the chunk form).  The forward chunk factors and
- * chunk states are recomputed inside the call.
+ * chunk states are recomputed inside the call, or, with COMBA_REUSE_FACTORS,
+ * read from a workspace that a forward with COMBA_SAVE_FACTORS filled.
  *
  *   inputs as comba_chunk_fwd, plus dO [B,T,H,dv] and dhT fp32 [N,H,dk,dv] or
  *   NULL (zero);
