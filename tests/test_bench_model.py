@@ -2,7 +2,8 @@
 
 `bench.py` reports each kernel's roofline from `stage_model` (bytes and tile-product
 FLOPs per launch) and `compulsory_bytes` (the step's own inputs and outputs).  Here
-every kernel of the bf16 d = 128 tcgen05 path is listed tile by tile: the tensors one
+every kernel of the bf16 d = 128 tcgen05 path (and, for bytes, of head dim 256) is
+listed tile by tile: the tensors one
 (chunk, head) unit must read or write once and the products it must form, written out
 from the chunk equations of section 3.2 and the affine chunk maps (H_{n+1} =
 (gamma_L I + Atilde) H_n + B).  The model must agree with the lists.
@@ -115,3 +116,25 @@ def test_compulsory_bytes_per_token_head():
     assert per["bwd_local"] == th * bwd_tok
     assert per["prep"] == th * ((dk + dv) * BF + 2 * F4)
     assert per["output"] == th * ((2 * dk + dv) * BF + F4)
+
+
+def test_head_dim_256_per_key_head_bytes_match_the_tensor_lists():
+    """dk = 256 with four value heads 64 wide: key-side tiles once per (chunk, key head), the
+    value heads' own tiles four times; no chunk map, W and K (or Z) streamed by the scans."""
+    K, v = 256, 64
+    key = dict(
+        prep=tile(C, K) + tile(C, K) + 3 * C * F4 + tile(C, C),                 # K in, W out, alpha/beta/G, M out
+        scan_fwd=2 * tile(C, K) + C * F4,                                        # W, K, gamma
+        scan_bwd=3 * tile(C, K) + C * F4,                                        # W, K, Z, gamma
+        output=3 * tile(C, K) + C * F4 + tile(C, K),                             # Q, K, W, G in; Z out
+        bwd_local=2 * tile(C, K) + tile(C, C) + 3 * C * F4 + 2 * tile(C, K) + 2 * C * F4)
+    per_value = dict(
+        prep=2 * tile(C, v),                                                     # V in, U out
+        scan_fwd=tile(C, v) + tile(v, K),                                        # U in, H_n out
+        scan_bwd=tile(C, v) + tile(v, K),                                        # dO in, dH' out
+        output=tile(C, v) + tile(v, K) + 2 * tile(C, v),                         # U, H_n in; O, E out
+        bwd_local=3 * tile(C, v) + 2 * tile(v, K) + tile(C, v))                  # V, dO, E, H_n, dH' in; dv out
+    m = bench.stage_model(K, v, slots=1, H=4, N=1, vg=4)
+    for stage in key:
+        assert m[stage]["bytes"] == key[stage] + 4 * per_value[stage], stage
+    assert m["bwd_prep"]["bytes"] == 0
